@@ -1,0 +1,86 @@
+"""Alg. 1 of the paper (DeltaS: state-guided KV eviction) run end to end on the CPU oracle.
+
+Test infrastructure only.  One iteration per arriving chunk c:
+
+1. ``S_before <- S``;
+2. ``Prefill(c)``: the gated delta rule (Eq. 2) updates S over the chunk's tokens, and the
+   chunk's keys/values are appended to every full-attention cache;
+3. ``Delta S`` of Eq. 3 from S_before and S, stored (in float32, as the paper computes all scores
+   in float32) as the score of every token of c;
+4. if the cache holds more than M tokens: sink / window / spans / quota + fill (Sec. 3.3), then
+   the in-stream-order gather of every cache, keeping original positions.
+
+Scores of earlier chunks are reused at later evictions (Sec. 3.3).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+from . import compact_kv, gdn_recurrence, select_retain, state_drift
+
+
+@dataclass
+class StreamResult:
+    state: np.ndarray                 # final S [L,Hv,dv,dk] fp64
+    chunk_scores: np.ndarray          # [n_chunks] float32
+    k_cache: np.ndarray               # [Lf,Hkv,capacity,D]
+    v_cache: np.ndarray
+    tok_chunk: np.ndarray             # [capacity] int32
+    tok_pos: np.ndarray               # [capacity] int32
+    cache_len: int
+    states_after_chunk: list = field(default_factory=list)
+    evictions: list = field(default_factory=list)   # (chunk, retain_idx) per eviction event
+
+
+def run_stream(chunk_inputs, kv_inputs, state0, n_chunks: int, policy: dict, capacity: int,
+               q_scale: float | None = None, score_override=None, keep_states: bool = False):
+    """Run Alg. 1 over ``n_chunks`` chunks.
+
+    ``chunk_inputs(c)`` -> (q, k, v, g, beta) numpy arrays in the oracle layouts;
+    ``kv_inputs(c)`` -> (k_new, v_new) of shape [Lf,Hkv,C,D];
+    ``policy`` = dict(budget_M, n_sink, n_window, n_buckets);
+    ``score_override`` (optional) [n_chunks] float32: scores to rank with instead of the oracle's
+    own (so that selection can be compared given identical scores).
+    """
+    S = np.array(state0, dtype=np.float64, copy=True)
+    scores = np.zeros(n_chunks, dtype=np.float32)
+    kc = vc = None
+    tok_chunk = np.zeros(capacity, dtype=np.int32)
+    tok_pos = np.zeros(capacity, dtype=np.int32)
+    T = 0
+    pos = 0
+    res = StreamResult(S, scores, None, None, tok_chunk, tok_pos, 0)
+    for c in range(n_chunks):
+        q, k, v, g, beta = chunk_inputs(c)
+        s_before = S.copy()
+        S, _ = gdn_recurrence(None, k, v, g, beta, S, q_scale=q_scale)
+        k_new, v_new = kv_inputs(c)
+        Lf, Hkv, C, D = k_new.shape
+        if kc is None:
+            kc = np.zeros((Lf, Hkv, capacity, D), dtype=k_new.dtype)
+            vc = np.zeros_like(kc)
+        if T + C > capacity:
+            raise ValueError("cache capacity too small for the stream")
+        kc[:, :, T:T + C] = k_new
+        vc[:, :, T:T + C] = v_new
+        tok_chunk[T:T + C] = c
+        tok_pos[T:T + C] = np.arange(pos, pos + C, dtype=np.int32)
+        T += C
+        pos += C
+        scores[c] = np.float32(state_drift(s_before, S))
+        if keep_states:
+            res.states_after_chunk.append(S.copy())
+        if T > policy["budget_M"]:
+            rank_scores = scores if score_override is None else np.asarray(score_override, np.float32)
+            idx, _ = select_retain(policy["budget_M"], policy["n_sink"], policy["n_window"],
+                                   policy["n_buckets"], tok_chunk[:T], rank_scores[: c + 1])
+            kc, vc, tok_chunk, tok_pos = compact_kv(kc, vc, tok_chunk, tok_pos, idx, T)
+            res.evictions.append((c, idx))
+            T = int(idx.shape[0])
+    res.state = S
+    res.k_cache, res.v_cache = kc, vc
+    res.tok_chunk, res.tok_pos = tok_chunk, tok_pos
+    res.cache_len = T
+    return res

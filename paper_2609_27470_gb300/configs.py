@@ -1,0 +1,33 @@
+"""The five synthetic workloads, shaped like the paper's hybrid backbone (Sec. 4.1, App. A).
+
+* ``tiny``      — 1 gated-delta layer, 2 heads, d=16, fp32, 8 chunks x 64 tokens, zero start
+                  state, 1 full-attention layer (2 KV heads, D=16, fp32 KV), budget 4 chunks.
+* ``layer``     — 1 layer at the backbone's width: 16 key heads, 32 value heads, d=128, bf16
+                  activations, fp32 state, 16 chunks x 1024 tokens.
+* ``stack``     — 24 gated-delta layers x 32 value heads x 128 x 128 fp32 state (48 MiB,
+                  Sec. 3.1), 256 chunks x 1024 tokens, states carried across chunks.
+* ``kv``        — 8 full-attention layers, 2 KV heads, D=256 bf16, a 64k-token cache of
+                  64 chunks x 1024 tokens, Exp(1) chunk scores with exact ties, budget 16k.
+* ``streaming`` — ``stack`` with 512-token chunks plus ``kv`` caches, 4096 chunks, budget 32k,
+                  the paper's policy (n_s=4, n_w=1024, N=4; Sec. 4.1).
+"""
+from __future__ import annotations
+
+PAPER_POLICY = {"n_sink": 4, "n_window": 1024, "n_buckets": 4}   # Sec. 4.1
+
+TINY = dict(name="tiny", L=1, Hk=2, Hv=2, d=16, dtype="f32", chunk_len=64, n_chunks=8,
+            Lf=1, Hkv=2, D=16, kv_dtype="f32", budget_M=256, zero_state=True)
+
+LAYER = dict(name="layer", L=1, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=1024, n_chunks=16)
+
+STACK = dict(name="stack", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=1024, n_chunks=256,
+             ring=8)
+
+KV = dict(name="kv", Lf=8, Hkv=2, D=256, kv_dtype="bf16", chunk_len=1024, n_chunks=64,
+          budget_M=16384)
+
+STREAMING = dict(name="streaming", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=512,
+                 n_chunks=4096, ring=8, Lf=8, Hkv=2, D=256, kv_dtype="bf16", budget_M=32768,
+                 **PAPER_POLICY)
+
+ALL = {c["name"]: c for c in (TINY, LAYER, STACK, KV, STREAMING)}
