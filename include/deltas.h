@@ -1,0 +1,238 @@
+/*
+ * deltas.h — C ABI of the DeltaS hot path on one GB300 GPU (sm_103a).
+ *
+ * DeltaS ("Reading the Gated Linear Attention State for KV Cache Eviction in Streaming Video")
+ * scores each video chunk by the normalised change it causes in the gated-delta-rule recurrent
+ * state (state drift, Sec. 3.2) and keeps the KV entries of high-drift chunks under a token
+ * budget (Sec. 3.3, Alg. 1).  This library runs that path as CUDA kernels:
+ *
+ *   deltas_gdn_chunk_update  gated delta rule over a chunk (Eq. 1/2) + fused drift partials
+ *   deltas_state_drift       drift partials from two stored states (Eq. 3 numerator/denominator)
+ *   deltas_score_chunks      Delta S of Eq. 3 from the partials, stored as the chunk's score
+ *   deltas_select_retain     sink / window / temporal spans / quota + fill (Sec. 3.3, Alg. 1)
+ *   deltas_compact_kv        in-place, stream-order gather of the KV caches (Alg. 1, Sec. 3.3)
+ *   deltas_append_kv         append a chunk's keys/values to the caches (Alg. 1 Prefill)
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Tensor pointers are CUDA device memory owned by the caller, dense, in the layouts stated per
+ *   call, 16-byte aligned.  The library allocates nothing and keeps no state between calls.
+ * - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  Every call
+ *   only enqueues work on it and returns at once; no call synchronises, except
+ *   deltas_get_device_status.
+ * - Scratch memory is a caller-provided `workspace` of at least the size reported by the matching
+ *   deltas_*_workspace_size function, 256-byte aligned.  Its first 16 bytes are a sticky device
+ *   status word: kernels that detect an error on the device (a bounded wait that ran out, an
+ *   out-of-range index) record the first such error there and skip the unsafe part of their
+ *   work.  Zero it once with deltas_clear_device_status before first use; read it with
+ *   deltas_get_device_status.  Calls sharing a workspace must be ordered on one stream.
+ * - Return value: DELTAS_OK when the work was enqueued; DELTAS_ERR_INVALID_ARGUMENT /
+ *   DELTAS_ERR_UNSUPPORTED / DELTAS_ERR_WORKSPACE when the host-side checks reject the call
+ *   (nothing is enqueued then); DELTAS_ERR_CUDA when a launch failed.  No exception crosses the
+ *   ABI.
+ */
+#ifndef DELTAS_H
+#define DELTAS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define DELTAS_API __attribute__((visibility("default")))
+#else
+#define DELTAS_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum deltas_status_e {
+    DELTAS_OK = 0,
+    DELTAS_ERR_INVALID_ARGUMENT = 1, /* a pointer, size or value outside its stated range        */
+    DELTAS_ERR_UNSUPPORTED = 2,      /* valid, but a shape/dtype this build has no kernel for     */
+    DELTAS_ERR_WORKSPACE = 3,        /* workspace missing, misaligned or smaller than required    */
+    DELTAS_ERR_CUDA = 4,             /* a CUDA launch or runtime call failed                      */
+    DELTAS_ERR_TIMEOUT = 5,          /* device: a bounded wait ran out (work skipped)             */
+    DELTAS_ERR_DEVICE_INDEX = 6      /* device: an index array was out of range or out of order   */
+} deltas_status;
+
+typedef enum deltas_dtype_e {
+    DELTAS_F32 = 0,  /* IEEE binary32 */
+    DELTAS_BF16 = 1  /* bfloat16 */
+} deltas_dtype;
+
+/* Shape of the gated-delta (linear-attention) layers.  Value head h reads key head
+ * floor(h * num_k_heads / num_v_heads) (grouped keys). */
+typedef struct deltas_gdn_desc {
+    int32_t num_layers;   /* L >= 1 */
+    int32_t num_k_heads;  /* Hk >= 1 */
+    int32_t num_v_heads;  /* Hv >= 1, a multiple of Hk */
+    int32_t key_dim;      /* d_k in {16, 32, 64, 128} */
+    int32_t value_dim;    /* d_v, equal to d_k in this build */
+    int32_t dtype;        /* deltas_dtype of q, k, v and out; g, beta and the state are float32 */
+    float q_scale;        /* read-out scale: o_t = q_scale * S_t q_t (commonly 1/sqrt(d_k)) */
+} deltas_gdn_desc;
+
+/* Retention policy (Alg. 1 inputs; Sec. 3.3). */
+typedef struct deltas_policy {
+    int32_t budget_M;   /* M >= n_sink + n_window + 1: tokens kept per full-attention layer */
+    int32_t n_sink;     /* n_s >= 0: first slots always kept (attention sinks) */
+    int32_t n_window;   /* n_w >= 0: most recent slots always kept */
+    int32_t n_buckets;  /* N in [0, 32]: equal temporal spans; 0 means no bucketing (= 1 span) */
+} deltas_policy;
+
+/* Shape of the full-attention KV caches: K and V are separate buffers, each
+ * [num_layers][num_kv_heads][capacity][head_dim] of dtype; a (layer, head) pair is one "plane"
+ * of `capacity` rows of head_dim elements. */
+typedef struct deltas_kv_desc {
+    int32_t num_layers;    /* Lf >= 1 */
+    int32_t num_kv_heads;  /* Hkv >= 1 */
+    int32_t head_dim;      /* D >= 1; head_dim * element size must be a multiple of 16 bytes */
+    int32_t dtype;         /* deltas_dtype of the caches */
+    int32_t capacity;      /* rows allocated per plane (>= the largest cache_len used) */
+} deltas_kv_desc;
+
+/* ------------------------------------------------------------------------------------------ */
+/* Version and status text                                                                     */
+/* ------------------------------------------------------------------------------------------ */
+
+/* Static string "deltas <major>.<minor>.<patch> sm_103a". */
+DELTAS_API const char* deltas_version(void);
+
+/* Static, never NULL, description of a deltas_status value (unknown codes included). */
+DELTAS_API const char* deltas_status_string(int32_t status);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Gated delta rule over one chunk, with the state drift partials fused in.                    */
+/*                                                                                              */
+/* Paper: Sec. 3.2, Eq. 1 S_t = S_{t-1}(alpha_t (I - beta_t k_t k_t^T)) + beta_t v_t k_t^T     */
+/* (equivalently Eq. 2), run over the n_tokens tokens of one video chunk in stream order for   */
+/* every layer and value head; the state before the chunk is S_before and the state after it   */
+/* S_after of Eq. 3.  Alg. 1: "Prefill(c) updates S"; the read-out o_t = q_scale S_t q_t is     */
+/* the layer output of that prefill.                                                            */
+/*                                                                                              */
+/*   q, k   [L][n_tokens][Hk][d_k]  dtype   keys L2-normalised by the caller; q may be NULL     */
+/*                                          when out is NULL                                   */
+/*   v      [L][n_tokens][Hv][d_v]  dtype                                                      */
+/*   g      [L][n_tokens][Hv]       float   log decay, alpha_t = exp(g_t), g_t <= 0 expected    */
+/*   beta   [L][n_tokens][Hv]       float   write strength in [0, 1]                           */
+/*   state  [L][Hv][d_v][d_k]       float   in: S_before, out: S_after (updated in place)      */
+/*   out    [L][n_tokens][Hv][d_v]  dtype   o_t after each token's update; NULL to skip        */
+/*   drift_partials [L][Hv][2]      float   NULL to skip; else [l][h][0] = sum (S_after -      */
+/*                                          S_before)^2 and [l][h][1] = sum S_before^2 over    */
+/*                                          the head's d_v x d_k entries                       */
+/* n_tokens = 0 leaves the state unchanged (partials then hold 0 and ||S_before||^2).          */
+/* Errors: INVALID_ARGUMENT for NULL/misaligned pointers, negative sizes or Hv % Hk != 0;      */
+/* UNSUPPORTED for d_k != d_v or d_k outside {16,32,64,128}; WORKSPACE for a short workspace. */
+/* ------------------------------------------------------------------------------------------ */
+DELTAS_API size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens);
+
+DELTAS_API deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, int32_t n_tokens,
+                                      const void* q, const void* k, const void* v,
+                                      const float* g, const float* beta,
+                                      float* state, void* out, float* drift_partials,
+                                      void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* State drift partials from two stored states (Sec. 3.2, Eq. 3 numerator and denominator per  */
+/* layer and head; the paper keeps a copy of the previous state for this, Sec. 3.2).           */
+/*   s_before, s_after [L][Hv][d_v][d_k] float;  drift_partials [L][Hv][2] float (as above).   */
+/* Only num_layers, num_v_heads, key_dim and value_dim of desc are used.                       */
+/* ------------------------------------------------------------------------------------------ */
+DELTAS_API size_t deltas_state_drift_workspace_size(const deltas_gdn_desc* desc);
+
+DELTAS_API deltas_status deltas_state_drift(const deltas_gdn_desc* desc, const float* s_before,
+                                 const float* s_after, float* drift_partials,
+                                 void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Chunk score (Sec. 3.2, Eq. 3; Alg. 1 "Delta S <- mean_i ||S^i - S^i_before|| /             */
+/* ||S^i_before||" and "score[t] <- Delta S"):                                                  */
+/*   Delta S = (1/L) sum_l sqrt(sum_h partials[l][h][0]) / sqrt(sum_h partials[l][h][1])       */
+/* The per-layer norm runs over all heads of the layer.  A layer whose denominator is 0        */
+/* contributes 0 when its numerator is 0 and +infinity otherwise.  The reduction order is       */
+/* fixed (deterministic); sums are formed in double and the score is stored as float to        */
+/* chunk_scores[chunk_id] (device memory, [>= chunk_id + 1] floats).                           */
+/* ------------------------------------------------------------------------------------------ */
+DELTAS_API deltas_status deltas_score_chunks(int32_t num_layers, int32_t num_v_heads,
+                                  const float* drift_partials, int32_t chunk_id,
+                                  float* chunk_scores, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Retain selection (Sec. 3.3; Alg. 1 eviction branch).                                        */
+/*                                                                                              */
+/* The cache holds cache_len slots in stream order; tok_chunk[i] is the arrival chunk of slot  */
+/* i and chunk_scores[c] the stored score of chunk c (shared by all its tokens).  If cache_len  */
+/* <= M every slot is kept.  Otherwise the first n_s and the last n_w slots are kept; the rest  */
+/* (candidates) are split into N equal spans of arrival chunk,                                  */
+/*   span(i) = floor((tok_chunk[i] - c_lo) * N / (c_hi - c_lo + 1)),                            */
+/* c_lo/c_hi the smallest/largest candidate chunk; each span keeps its best                     */
+/* min(floor((M - n_s - n_w) / N), |span|) candidates and the remaining capacity goes to the    */
+/* best remaining candidates.  "Best" = higher score under the IEEE-754 total order of float,  */
+/* ties to the earlier slot.                                                                    */
+/*                                                                                              */
+/*   tok_chunk   [cache_len] int32 in [0, num_chunks)      chunk_scores [num_chunks] float     */
+/*   retain_idx  [min(cache_len, M)] int32  out: kept slots, strictly ascending                 */
+/*   n_retained  [1] int32 (device)         out: min(cache_len, M)                              */
+/*   mask        [cache_len] uint8          out: 1 = kept, 0 = evicted; NULL to skip            */
+/* A tok_chunk value outside [0, num_chunks) is reported as DEVICE_INDEX in the status word    */
+/* (outputs are then unspecified).                                                              */
+/* ------------------------------------------------------------------------------------------ */
+DELTAS_API size_t deltas_select_retain_workspace_size(int32_t cache_len);
+
+DELTAS_API deltas_status deltas_select_retain(const deltas_policy* policy, int32_t cache_len,
+                                   int32_t num_chunks, const int32_t* tok_chunk,
+                                   const float* chunk_scores, int32_t* retain_idx,
+                                   int32_t* n_retained, uint8_t* mask,
+                                   void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* In-place KV compaction (Alg. 1 "KV <- KV[I_sink u I_DeltaS u I_window]", applied to every    */
+/* full-attention layer; Sec. 3.3: survivors keep their original position indices).            */
+/*                                                                                              */
+/* For every plane of k_cache and v_cache, and for tok_chunk and tok_pos ([capacity] int32):    */
+/*   row[j] <- row[retain_idx[j]]   for j < *n_retained,  in place;                             */
+/* rows at and past *n_retained are not written.  retain_idx is read on the device and must be  */
+/* strictly ascending with j <= retain_idx[j] < cache_len (as deltas_select_retain writes it);  */
+/* otherwise nothing is moved and DEVICE_INDEX is recorded.  Positions in tok_pos are moved,    */
+/* never renumbered.  cache_len <= capacity.                                                    */
+/* ------------------------------------------------------------------------------------------ */
+DELTAS_API size_t deltas_compact_kv_workspace_size(const deltas_kv_desc* desc, int32_t cache_len);
+
+DELTAS_API deltas_status deltas_compact_kv(const deltas_kv_desc* desc, void* k_cache, void* v_cache,
+                                int32_t* tok_chunk, int32_t* tok_pos,
+                                const int32_t* retain_idx, const int32_t* n_retained,
+                                int32_t cache_len, void* workspace, size_t workspace_bytes,
+                                void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Append one chunk to the caches (Alg. 1 "Prefill(c) ... appends c to KV").                   */
+/*   k_new, v_new [Lf][Hkv][n_new][D] dtype: the chunk's keys/values of every layer;            */
+/*   rows cache_len .. cache_len + n_new - 1 of every plane receive them, tok_chunk of those    */
+/*   slots is set to chunk_id and tok_pos to first_pos, first_pos + 1, ...                      */
+/* Errors: INVALID_ARGUMENT if cache_len + n_new > capacity or a size is negative.             */
+/* ------------------------------------------------------------------------------------------ */
+DELTAS_API deltas_status deltas_append_kv(const deltas_kv_desc* desc, void* k_cache, void* v_cache,
+                               int32_t* tok_chunk, int32_t* tok_pos, int32_t cache_len,
+                               const void* k_new, const void* v_new, int32_t n_new,
+                               int32_t chunk_id, int32_t first_pos, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Device status word (first 16 bytes of a workspace).                                          */
+/* ------------------------------------------------------------------------------------------ */
+
+/* Enqueue a zeroing of the status word. */
+DELTAS_API deltas_status deltas_clear_device_status(void* workspace, void* stream);
+
+/* Synchronise `stream`, then read the status word: *status_out = first recorded deltas_status
+ * (DELTAS_OK if none), *detail_out = kernel-specific detail (e.g. the offending index); either
+ * output pointer may be NULL. */
+DELTAS_API deltas_status deltas_get_device_status(const void* workspace, void* stream,
+                                       int32_t* status_out, int32_t* detail_out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DELTAS_H */

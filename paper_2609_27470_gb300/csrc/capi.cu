@@ -1,0 +1,238 @@
+// C-ABI entry points of libdeltas (declared and documented in include/deltas.h).
+//
+// This layer validates arguments on the host (nothing is enqueued when a check fails), carves the
+// caller's workspace, and enqueues the kernels on the caller's stream.  It allocates nothing.
+#include <cstdint>
+#include <cstring>
+
+#include "internal.cuh"
+
+namespace deltas {
+
+int device_sm_count() {
+    // cached per device: the attribute query is cheap but not free
+    static int cached[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 1;
+    if (dev < 64 && cached[dev] > 0) return cached[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+    if (dev < 64) cached[dev] = n;
+    return n;
+}
+
+}  // namespace deltas
+
+using namespace deltas;
+
+namespace {
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned256(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 255u) == 0; }
+cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
+
+deltas_status check_gdn_desc(const deltas_gdn_desc* d) {
+    if (d == nullptr) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (d->num_layers < 1 || d->num_k_heads < 1 || d->num_v_heads < 1) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (d->num_v_heads % d->num_k_heads != 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (d->key_dim < 1 || d->value_dim < 1) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (d->dtype != DELTAS_F32 && d->dtype != DELTAS_BF16) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (d->key_dim != d->value_dim) return DELTAS_ERR_UNSUPPORTED;
+    if (d->key_dim != 16 && d->key_dim != 32 && d->key_dim != 64 && d->key_dim != 128) return DELTAS_ERR_UNSUPPORTED;
+    if ((long long)d->num_layers * d->num_v_heads > (1ll << 30)) return DELTAS_ERR_UNSUPPORTED;
+    return DELTAS_OK;
+}
+
+deltas_status check_workspace(const void* ws, size_t bytes, size_t need) {
+    if (ws == nullptr || !aligned256(ws) || bytes < need) return DELTAS_ERR_WORKSPACE;
+    return DELTAS_OK;
+}
+
+deltas_status check_kv_desc(const deltas_kv_desc* d) {
+    if (d == nullptr) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (d->num_layers < 1 || d->num_kv_heads < 1 || d->head_dim < 1 || d->capacity < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (d->dtype != DELTAS_F32 && d->dtype != DELTAS_BF16) return DELTAS_ERR_INVALID_ARGUMENT;
+    if ((d->head_dim * elt_bytes(d->dtype)) % 16 != 0) return DELTAS_ERR_UNSUPPORTED;
+    const long long rb = (long long)d->head_dim * elt_bytes(d->dtype);
+    if (rb > 32768) return DELTAS_ERR_UNSUPPORTED;
+    if ((long long)d->num_layers * d->num_kv_heads > (1ll << 20)) return DELTAS_ERR_UNSUPPORTED;
+    return DELTAS_OK;
+}
+
+KvPlanes make_planes(const deltas_kv_desc* d, void* k, void* v, int32_t* tc, int32_t* tp) {
+    KvPlanes p;
+    p.Lf = d->num_layers; p.Hkv = d->num_kv_heads; p.D = d->head_dim; p.dtype = d->dtype;
+    p.capacity = d->capacity; p.k_cache = k; p.v_cache = v; p.tok_chunk = tc; p.tok_pos = tp;
+    return p;
+}
+
+deltas_status from_cuda(cudaError_t e) { return e == cudaSuccess ? DELTAS_OK : DELTAS_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+const char* deltas_version(void) { return "deltas 0.1.0 sm_103a"; }
+
+const char* deltas_status_string(int32_t s) {
+    switch (s) {
+        case DELTAS_OK: return "ok";
+        case DELTAS_ERR_INVALID_ARGUMENT: return "invalid argument";
+        case DELTAS_ERR_UNSUPPORTED: return "unsupported shape or dtype";
+        case DELTAS_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+        case DELTAS_ERR_CUDA: return "CUDA launch or runtime error";
+        case DELTAS_ERR_TIMEOUT: return "device: bounded wait ran out";
+        case DELTAS_ERR_DEVICE_INDEX: return "device: index out of range or out of order";
+        default: return "unknown status";
+    }
+}
+
+size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens) {
+    (void)desc; (void)n_tokens;
+    return kStatusBytes;
+}
+
+deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, int32_t n_tokens,
+                                      const void* q, const void* k, const void* v,
+                                      const float* g, const float* beta,
+                                      float* state, void* out, float* drift_partials,
+                                      void* workspace, size_t workspace_bytes, void* stream)
+{
+    deltas_status st = check_gdn_desc(desc);
+    if (st != DELTAS_OK) return st;
+    if (n_tokens < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (state == nullptr || !aligned16(state)) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (n_tokens > 0) {
+        if (!k || !v || !g || !beta || !aligned16(k) || !aligned16(v)) return DELTAS_ERR_INVALID_ARGUMENT;
+        if (out && (!q || !aligned16(q) || !aligned16(out))) return DELTAS_ERR_INVALID_ARGUMENT;
+    }
+    if (drift_partials && !aligned16(drift_partials)) return DELTAS_ERR_INVALID_ARGUMENT;
+    st = check_workspace(workspace, workspace_bytes, deltas_gdn_chunk_update_workspace_size(desc, n_tokens));
+    if (st != DELTAS_OK) return st;
+    GdnArgs a;
+    a.L = desc->num_layers; a.Hk = desc->num_k_heads; a.Hv = desc->num_v_heads;
+    a.dk = desc->key_dim; a.dv = desc->value_dim; a.T = n_tokens; a.dtype = desc->dtype;
+    a.q_scale = desc->q_scale; a.q = q; a.k = k; a.v = v; a.g = g; a.beta = beta;
+    a.state = state; a.out = out; a.partials = drift_partials;
+    a.status = static_cast<int32_t*>(workspace);
+    if (gdn_tc_supported(a)) return from_cuda(launch_gdn_update_tc(a, as_stream(stream)));
+    return from_cuda(launch_gdn_update_simt(a, as_stream(stream)));
+}
+
+size_t deltas_state_drift_workspace_size(const deltas_gdn_desc* desc) {
+    (void)desc;
+    return kStatusBytes;
+}
+
+deltas_status deltas_state_drift(const deltas_gdn_desc* desc, const float* s_before,
+                                 const float* s_after, float* drift_partials,
+                                 void* workspace, size_t workspace_bytes, void* stream)
+{
+    if (desc == nullptr) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (desc->num_layers < 1 || desc->num_v_heads < 1 || desc->key_dim < 1 || desc->value_dim < 1)
+        return DELTAS_ERR_INVALID_ARGUMENT;
+    if (((long long)desc->key_dim * desc->value_dim) % 4 != 0) return DELTAS_ERR_UNSUPPORTED;
+    if ((long long)desc->key_dim * desc->value_dim > (1ll << 30)) return DELTAS_ERR_UNSUPPORTED;
+    if (!s_before || !s_after || !drift_partials) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!aligned16(s_before) || !aligned16(s_after)) return DELTAS_ERR_INVALID_ARGUMENT;
+    deltas_status st = check_workspace(workspace, workspace_bytes, deltas_state_drift_workspace_size(desc));
+    if (st != DELTAS_OK) return st;
+    return from_cuda(launch_state_drift(desc->num_layers, desc->num_v_heads, desc->value_dim,
+                                        desc->key_dim, s_before, s_after, drift_partials,
+                                        as_stream(stream)));
+}
+
+deltas_status deltas_score_chunks(int32_t num_layers, int32_t num_v_heads,
+                                  const float* drift_partials, int32_t chunk_id,
+                                  float* chunk_scores, void* stream)
+{
+    if (num_layers < 1 || num_v_heads < 1 || chunk_id < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!drift_partials || !chunk_scores) return DELTAS_ERR_INVALID_ARGUMENT;
+    return from_cuda(launch_score_chunks(num_layers, num_v_heads, drift_partials, chunk_id,
+                                         chunk_scores, as_stream(stream)));
+}
+
+size_t deltas_select_retain_workspace_size(int32_t cache_len) {
+    return select_workspace_bytes(cache_len);
+}
+
+deltas_status deltas_select_retain(const deltas_policy* policy, int32_t cache_len,
+                                   int32_t num_chunks, const int32_t* tok_chunk,
+                                   const float* chunk_scores, int32_t* retain_idx,
+                                   int32_t* n_retained, uint8_t* mask,
+                                   void* workspace, size_t workspace_bytes, void* stream)
+{
+    if (policy == nullptr || cache_len < 0 || num_chunks < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    const deltas_policy& p = *policy;
+    if (p.budget_M < 1 || p.n_sink < 0 || p.n_window < 0 || p.n_buckets < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if ((long long)p.budget_M < (long long)p.n_sink + p.n_window + 1) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (p.n_buckets > 32) return DELTAS_ERR_UNSUPPORTED;
+    if (!retain_idx || !n_retained) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (cache_len > 0 && (!tok_chunk || !chunk_scores)) return DELTAS_ERR_INVALID_ARGUMENT;
+    deltas_status st = check_workspace(workspace, workspace_bytes, deltas_select_retain_workspace_size(cache_len));
+    if (st != DELTAS_OK) return st;
+    return from_cuda(launch_select_retain(p, cache_len, num_chunks, tok_chunk, chunk_scores, retain_idx,
+                                          n_retained, mask, workspace, static_cast<int32_t*>(workspace),
+                                          as_stream(stream)));
+}
+
+size_t deltas_compact_kv_workspace_size(const deltas_kv_desc* desc, int32_t cache_len) {
+    if (check_kv_desc(desc) != DELTAS_OK || cache_len < 0) return 0;
+    KvPlanes kv = make_planes(desc, nullptr, nullptr, nullptr, nullptr);
+    return compact_workspace_bytes(kv, cache_len);
+}
+
+deltas_status deltas_compact_kv(const deltas_kv_desc* desc, void* k_cache, void* v_cache,
+                                int32_t* tok_chunk, int32_t* tok_pos,
+                                const int32_t* retain_idx, const int32_t* n_retained,
+                                int32_t cache_len, void* workspace, size_t workspace_bytes,
+                                void* stream)
+{
+    deltas_status st = check_kv_desc(desc);
+    if (st != DELTAS_OK) return st;
+    if (cache_len < 0 || cache_len > desc->capacity) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!k_cache || !v_cache || !tok_chunk || !tok_pos || !retain_idx || !n_retained) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!aligned16(k_cache) || !aligned16(v_cache)) return DELTAS_ERR_INVALID_ARGUMENT;
+    st = check_workspace(workspace, workspace_bytes, deltas_compact_kv_workspace_size(desc, cache_len));
+    if (st != DELTAS_OK) return st;
+    KvPlanes kv = make_planes(desc, k_cache, v_cache, tok_chunk, tok_pos);
+    return from_cuda(launch_compact_kv(kv, retain_idx, n_retained, cache_len, workspace,
+                                       static_cast<int32_t*>(workspace), as_stream(stream)));
+}
+
+deltas_status deltas_append_kv(const deltas_kv_desc* desc, void* k_cache, void* v_cache,
+                               int32_t* tok_chunk, int32_t* tok_pos, int32_t cache_len,
+                               const void* k_new, const void* v_new, int32_t n_new,
+                               int32_t chunk_id, int32_t first_pos, void* stream)
+{
+    deltas_status st = check_kv_desc(desc);
+    if (st != DELTAS_OK) return st;
+    if (cache_len < 0 || n_new < 0 || (long long)cache_len + n_new > desc->capacity) return DELTAS_ERR_INVALID_ARGUMENT;
+    if ((long long)first_pos + n_new > INT32_MAX || first_pos < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!k_cache || !v_cache || !tok_chunk || !tok_pos) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (n_new > 0 && (!k_new || !v_new || !aligned16(k_new) || !aligned16(v_new))) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!aligned16(k_cache) || !aligned16(v_cache)) return DELTAS_ERR_INVALID_ARGUMENT;
+    KvPlanes kv = make_planes(desc, k_cache, v_cache, tok_chunk, tok_pos);
+    return from_cuda(launch_append_kv(kv, cache_len, k_new, v_new, n_new, chunk_id, first_pos,
+                                      as_stream(stream)));
+}
+
+deltas_status deltas_clear_device_status(void* workspace, void* stream) {
+    if (workspace == nullptr) return DELTAS_ERR_WORKSPACE;
+    return from_cuda(cudaMemsetAsync(workspace, 0, 16, as_stream(stream)));
+}
+
+deltas_status deltas_get_device_status(const void* workspace, void* stream,
+                                       int32_t* status_out, int32_t* detail_out)
+{
+    if (workspace == nullptr) return DELTAS_ERR_WORKSPACE;
+    int32_t host[2] = {0, 0};
+    cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+    if (e == cudaSuccess) e = cudaMemcpy(host, workspace, sizeof(host), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return DELTAS_ERR_CUDA;
+    if (status_out) *status_out = host[0];
+    if (detail_out) *detail_out = host[1];
+    return DELTAS_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,307 @@
+// In-place, stream-order KV compaction (Alg. 1 "KV <- KV[I_sink u I_DeltaS u I_window]",
+// applied to every full-attention layer; Sec. 3.3: survivors keep their original positions) and
+// the per-chunk append to the caches (Alg. 1 Prefill).
+//
+// The gather row[j] <- row[retain_idx[j]] runs in place.  Because retain_idx is ascending with
+// retain_idx[j] >= j, the only hazard is a destination row that is still to be read as the
+// source of an earlier destination.  The work is cut into units (plane p, tile b of TB
+// destination rows); a unit
+//   1. stages the source rows of its tile in shared memory (16-byte loads),
+//   2. publishes "tile b of plane p has been read" (release flag),
+//   3. waits until every earlier tile whose destinations read rows of tile b has published
+//      (the first such tile, need[b], comes from a prepass over retain_idx),
+//   4. writes its tile (16-byte stores; the destination rows of a tile are contiguous).
+// Units are claimed through an atomic ticket in tile-major order, so a unit only waits for units
+// that were claimed earlier by running CTAs and that never wait before publishing: no deadlock.
+// Every wait is bounded (about one second); a wait that runs out records DELTAS_ERR_TIMEOUT,
+// raises the abort flag and skips its writes.  Traffic is the algorithmic minimum: each moved row
+// is read once and written once; rows that do not move are not touched.
+#include "internal.cuh"
+
+namespace deltas {
+namespace {
+
+constexpr int kCompactThreads = 256;
+constexpr int kStageBytes = 32768;
+
+struct CompactCtl {
+    unsigned ticket;
+    int abort;
+};
+
+struct CompactArgs {
+    char* k_cache;
+    char* v_cache;
+    char* tok_chunk;
+    char* tok_pos;
+    int n_kv_planes;       // Lf * Hkv planes in each of K and V
+    int capacity;
+    int row_bytes;         // D * element size (multiple of 16)
+    int tile_rows;         // TB
+    int n_planes;          // 2 * n_kv_planes + 2 (metadata)
+    int cache_len;
+    int max_tiles;         // ceil(cache_len / TB)
+    const int32_t* retain_idx;
+    const int32_t* n_retained;
+    CompactCtl* ctl;
+    int32_t* need;         // [max_tiles]
+    int32_t* flags;        // [n_planes][max_tiles]
+    int32_t* status;
+};
+
+__host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+__device__ __forceinline__ char* plane_base(const CompactArgs& a, int p, int& rb) {
+    if (p < a.n_kv_planes) { rb = a.row_bytes; return a.k_cache + (size_t)p * a.capacity * a.row_bytes; }
+    p -= a.n_kv_planes;
+    if (p < a.n_kv_planes) { rb = a.row_bytes; return a.v_cache + (size_t)p * a.capacity * a.row_bytes; }
+    rb = 4;
+    return p == a.n_kv_planes ? a.tok_chunk : a.tok_pos;
+}
+
+__global__ void compact_init_kernel(CompactArgs a) {
+    const int total = a.n_planes * a.max_tiles;
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x)
+        a.flags[e] = 0;
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < a.max_tiles; e += gridDim.x * blockDim.x)
+        a.need[e] = e;
+    if (blockIdx.x == 0 && threadIdx.x == 0) { a.ctl->ticket = 0; a.ctl->abort = 0; }
+}
+
+// Validates retain_idx and records, per source tile, the first earlier destination tile that
+// reads from it.
+__global__ void compact_need_kernel(CompactArgs a) {
+    const int n = *a.n_retained;
+    if (n < 0 || n > a.cache_len) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) {
+            a.ctl->abort = 1;
+            record_status(a.status, DELTAS_ERR_DEVICE_INDEX, n);
+        }
+        return;
+    }
+    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < n; j += gridDim.x * blockDim.x) {
+        const int src = a.retain_idx[j];
+        const bool ok = src >= j && src < a.cache_len && (j == 0 || src > a.retain_idx[j - 1]);
+        if (!ok) {
+            atomicExch(&a.ctl->abort, 1);
+            record_status(a.status, DELTAS_ERR_DEVICE_INDEX, j);
+            continue;
+        }
+        const int ts = src / a.tile_rows, td = j / a.tile_rows;
+        if (ts != td) atomicMin(&a.need[ts], td);
+    }
+}
+
+__device__ __forceinline__ int load_acquire(const int32_t* p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void store_release(int32_t* p, int v) {
+    asm volatile("st.release.gpu.global.b32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+
+__global__ void __launch_bounds__(kCompactThreads)
+compact_main_kernel(CompactArgs a)
+{
+    extern __shared__ uint4 stage[];
+    __shared__ int s_unit;
+    __shared__ int s_ok;
+    __shared__ int s_src[1024];
+
+    volatile int* abort_flag = &a.ctl->abort;
+    if (*abort_flag) return;
+    const int n = *a.n_retained;
+    const int n_tiles = (n + a.tile_rows - 1) / a.tile_rows;
+    const int units = n_tiles * a.n_planes;
+    const int tid = threadIdx.x;
+
+    for (;;) {
+        if (tid == 0) s_unit = (*abort_flag) ? units : (int)atomicAdd(&a.ctl->ticket, 1u);
+        __syncthreads();
+        const int u = s_unit;
+        if (u >= units) break;
+        const int b = u / a.n_planes, p = u % a.n_planes;
+        int rb;
+        char* base = plane_base(a, p, rb);
+        const int j0 = b * a.tile_rows;
+        const int rows = min(a.tile_rows, n - j0);
+        for (int r = tid; r < rows; r += kCompactThreads) s_src[r] = a.retain_idx[j0 + r];
+        __syncthreads();
+
+        // 1. stage the source rows of moved destinations
+        if (rb >= 16) {
+            const int vpr = rb >> 4;                       // 16-byte vectors per row
+            const int nv = rows * vpr;
+            for (int e = tid; e < nv; e += kCompactThreads) {
+                const int r = e / vpr, c = e - r * vpr;
+                const int src = s_src[r];
+                if (src != j0 + r)
+                    stage[e] = __ldcs(reinterpret_cast<const uint4*>(base + (size_t)src * rb) + c);
+            }
+        } else {
+            int* st = reinterpret_cast<int*>(stage);
+            for (int r = tid; r < rows; r += kCompactThreads) {
+                const int src = s_src[r];
+                if (src != j0 + r) st[r] = reinterpret_cast<const int*>(base)[src];
+            }
+        }
+        __syncthreads();
+
+        // 2. publish, 3. wait for the earlier readers of this tile
+        if (tid == 0) {
+            __threadfence();
+            store_release(a.flags + (size_t)p * a.max_tiles + b, 1);
+            int ok = 1;
+            const uint64_t t_start = global_ns();
+            for (int bb = a.need[b]; bb < b && ok; ++bb) {
+                const int32_t* f = a.flags + (size_t)p * a.max_tiles + bb;
+                while (load_acquire(f) == 0) {
+                    if (*abort_flag || global_ns() - t_start > kWaitBudgetNs) {
+                        ok = 0;
+                        break;
+                    }
+                    __nanosleep(64);
+                }
+            }
+            if (!ok) {
+                atomicExch(&a.ctl->abort, 1);
+                record_status(a.status, DELTAS_ERR_TIMEOUT, u);
+            }
+            s_ok = ok;
+        }
+        __syncthreads();
+        if (!s_ok) break;
+
+        // 4. write the tile
+        if (rb >= 16) {
+            const int vpr = rb >> 4;
+            const int nv = rows * vpr;
+            uint4* dst = reinterpret_cast<uint4*>(base + (size_t)j0 * rb);
+            for (int e = tid; e < nv; e += kCompactThreads) {
+                const int r = e / vpr;
+                if (s_src[r] != j0 + r) __stcs(dst + e, stage[e]);
+            }
+        } else {
+            const int* st = reinterpret_cast<const int*>(stage);
+            for (int r = tid; r < rows; r += kCompactThreads)
+                if (s_src[r] != j0 + r) reinterpret_cast<int*>(base)[j0 + r] = st[r];
+        }
+        __syncthreads();
+    }
+}
+
+__global__ void append_kv_kernel(char* k_cache, char* v_cache, int n_kv_planes, int capacity,
+                                 int row_bytes, int cache_len, const char* k_new, const char* v_new,
+                                 int n_new, int32_t* tok_chunk, int32_t* tok_pos, int chunk_id,
+                                 int first_pos)
+{
+    const size_t vec_per_plane = (size_t)n_new * row_bytes / 16;
+    const size_t total = 2 * (size_t)n_kv_planes * vec_per_plane;
+    const size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (size_t e = (size_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += stride) {
+        const size_t pp = e / vec_per_plane, off = e - pp * vec_per_plane;
+        const bool is_v = pp >= (size_t)n_kv_planes;
+        const size_t p = is_v ? pp - n_kv_planes : pp;
+        const uint4* src = reinterpret_cast<const uint4*>((is_v ? v_new : k_new) + p * (size_t)n_new * row_bytes);
+        uint4* dst = reinterpret_cast<uint4*>((is_v ? v_cache : k_cache) +
+                                              (p * (size_t)capacity + cache_len) * row_bytes);
+        dst[off] = __ldcs(src + off);
+    }
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < (size_t)n_new; i += stride) {
+        tok_chunk[cache_len + i] = chunk_id;
+        tok_pos[cache_len + i] = first_pos + (int)i;
+    }
+}
+
+int tile_rows_for(int row_bytes) {
+    int tb = kStageBytes / row_bytes;
+    return tb < 1 ? 1 : (tb > 1024 ? 1024 : tb);
+}
+
+struct CompactWsLayout {
+    size_t ctl, need, flags, total;
+};
+
+CompactWsLayout compact_layout(const KvPlanes& kv, int cache_len) {
+    const int rb = kv.D * elt_bytes(kv.dtype);
+    const int tb = tile_rows_for(rb);
+    const size_t max_tiles = (size_t)((cache_len + tb - 1) / tb);
+    const size_t n_planes = 2 * (size_t)kv.Lf * kv.Hkv + 2;
+    CompactWsLayout l;
+    l.ctl = kStatusBytes;
+    l.need = l.ctl + 256;
+    l.flags = l.need + align256(sizeof(int32_t) * (max_tiles > 0 ? max_tiles : 1));
+    l.total = l.flags + align256(sizeof(int32_t) * n_planes * (max_tiles > 0 ? max_tiles : 1));
+    return l;
+}
+
+}  // namespace
+
+size_t compact_workspace_bytes(const KvPlanes& kv, int cache_len) {
+    return compact_layout(kv, cache_len).total;
+}
+
+cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, const int32_t* n_retained,
+                              int cache_len, void* ws, int32_t* status, cudaStream_t s)
+{
+    if (cache_len <= 0) return cudaSuccess;
+    const CompactWsLayout l = compact_layout(kv, cache_len);
+    char* w = static_cast<char*>(ws);
+    CompactArgs a;
+    a.k_cache = static_cast<char*>(kv.k_cache);
+    a.v_cache = static_cast<char*>(kv.v_cache);
+    a.tok_chunk = reinterpret_cast<char*>(kv.tok_chunk);
+    a.tok_pos = reinterpret_cast<char*>(kv.tok_pos);
+    a.n_kv_planes = kv.Lf * kv.Hkv;
+    a.capacity = kv.capacity;
+    a.row_bytes = kv.D * elt_bytes(kv.dtype);
+    a.tile_rows = tile_rows_for(a.row_bytes);
+    a.n_planes = 2 * a.n_kv_planes + 2;
+    a.cache_len = cache_len;
+    a.max_tiles = (cache_len + a.tile_rows - 1) / a.tile_rows;
+    a.retain_idx = retain_idx;
+    a.n_retained = n_retained;
+    a.ctl = reinterpret_cast<CompactCtl*>(w + l.ctl);
+    a.need = reinterpret_cast<int32_t*>(w + l.need);
+    a.flags = reinterpret_cast<int32_t*>(w + l.flags);
+    a.status = status;
+
+    const int sms = device_sm_count();
+    const int init_blocks = min(4 * sms, (a.n_planes * a.max_tiles + 255) / 256 + 1);
+    compact_init_kernel<<<init_blocks, 256, 0, s>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    compact_need_kernel<<<min(4 * sms, (cache_len + 255) / 256), 256, 0, s>>>(a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+
+    const int smem = a.tile_rows * a.row_bytes;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, compact_main_kernel, kCompactThreads, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+    const int max_units = a.max_tiles * a.n_planes;
+    const int grid = max(1, min(max_units, per_sm * sms));
+    compact_main_kernel<<<grid, kCompactThreads, smem, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_new, const void* v_new,
+                             int n_new, int chunk_id, int first_pos, cudaStream_t s)
+{
+    if (n_new <= 0) return cudaSuccess;
+    const int rb = kv.D * elt_bytes(kv.dtype);
+    const size_t total_vec = 2 * (size_t)kv.Lf * kv.Hkv * n_new * rb / 16;
+    const int sms = device_sm_count();
+    const size_t want = (total_vec + 255) / 256;
+    const int blocks = (int)(want < (size_t)(8 * sms) ? (want > 0 ? want : 1) : (size_t)(8 * sms));
+    append_kv_kernel<<<blocks, 256, 0, s>>>(static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache),
+                                           kv.Lf * kv.Hkv, kv.capacity, rb, cache_len,
+                                           static_cast<const char*>(k_new), static_cast<const char*>(v_new),
+                                           n_new, kv.tok_chunk, kv.tok_pos, chunk_id, first_pos);
+    return cudaGetLastError();
+}
+
+}  // namespace deltas

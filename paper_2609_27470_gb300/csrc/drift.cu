@@ -1,0 +1,92 @@
+// State drift (Sec. 3.2, Eq. 3) from two stored states, and the chunk score from drift partials.
+//
+// state_drift: one CTA per (layer, value head) streams both d_v x d_k states once with 16-byte
+// loads (HBM-bound: 2 * 4 * d_v * d_k bytes per head) and writes
+//   partials[l][h] = { sum (S_after - S_before)^2, sum S_before^2 }.
+// The difference is formed element by element before squaring, never as
+// |A|^2 - 2<A,B> + |B|^2, which cancels badly when the drift is small.
+//
+// score_chunks: one warp-sized CTA reduces the [L][Hv][2] partials in a fixed order (lane-strided
+// double sums, then a fixed xor tree), applies sqrt(num_l)/sqrt(den_l) per layer with the
+// zero-norm reading (0/0 -> 0, x/0 -> +inf) and stores the layer mean as the chunk's score.
+#include "internal.cuh"
+
+namespace deltas {
+namespace {
+
+constexpr int kDriftThreads = 256;
+
+__global__ void __launch_bounds__(kDriftThreads)
+state_drift_kernel(int n_elem4, const float4* __restrict__ sb, const float4* __restrict__ sa,
+                   float* __restrict__ partials)
+{
+    const size_t base = (size_t)blockIdx.x * n_elem4;
+    float num = 0.f, den = 0.f;
+    for (int e = threadIdx.x; e < n_elem4; e += kDriftThreads) {
+        const float4 b = __ldcs(sb + base + e);   // streamed once: evict-first
+        const float4 a = __ldcs(sa + base + e);
+        const float dx = a.x - b.x, dy = a.y - b.y, dz = a.z - b.z, dw = a.w - b.w;
+        num += dx * dx + dy * dy + dz * dz + dw * dw;
+        den += b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
+    }
+    double dn = num, dd = den;
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+        dn += __shfl_xor_sync(0xffffffffu, dn, m);
+        dd += __shfl_xor_sync(0xffffffffu, dd, m);
+    }
+    __shared__ double red[2][kDriftThreads / 32];
+    if ((threadIdx.x & 31) == 0) { red[0][threadIdx.x >> 5] = dn; red[1][threadIdx.x >> 5] = dd; }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double sn = 0.0, sd = 0.0;
+        for (int w = 0; w < kDriftThreads / 32; ++w) { sn += red[0][w]; sd += red[1][w]; }
+        partials[(size_t)blockIdx.x * 2 + 0] = (float)sn;
+        partials[(size_t)blockIdx.x * 2 + 1] = (float)sd;
+    }
+}
+
+__global__ void __launch_bounds__(32)
+score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk_id,
+                    float* __restrict__ scores)
+{
+    const int lane = threadIdx.x;
+    double total = 0.0;
+    for (int l = 0; l < L; ++l) {
+        double num = 0.0, den = 0.0;
+        for (int h = lane; h < Hv; h += 32) {
+            num += (double)partials[((size_t)l * Hv + h) * 2 + 0];
+            den += (double)partials[((size_t)l * Hv + h) * 2 + 1];
+        }
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) {
+            num += __shfl_xor_sync(0xffffffffu, num, m);
+            den += __shfl_xor_sync(0xffffffffu, den, m);
+        }
+        double term;
+        if (den > 0.0) term = sqrt(num) / sqrt(den);
+        else term = (num > 0.0) ? (double)INFINITY : 0.0;
+        total += term;
+    }
+    if (lane == 0) scores[chunk_id] = (float)(total / (double)L);
+}
+
+}  // namespace
+
+cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, const float* sa,
+                               float* partials, cudaStream_t s)
+{
+    const int n4 = dv * dk / 4;
+    state_drift_kernel<<<L * Hv, kDriftThreads, 0, s>>>(n4, reinterpret_cast<const float4*>(sb),
+                                                        reinterpret_cast<const float4*>(sa), partials);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_score_chunks(int L, int Hv, const float* partials, int chunk_id, float* scores,
+                                cudaStream_t s)
+{
+    score_chunks_kernel<<<1, 32, 0, s>>>(L, Hv, partials, chunk_id, scores);
+    return cudaGetLastError();
+}
+
+}  // namespace deltas

@@ -1,0 +1,88 @@
+// Internal declarations shared by the library's kernels and its C-ABI layer.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/deltas.h"
+
+namespace deltas {
+
+// ---------------------------------------------------------------------------------------------
+// Device status word: the first 16 bytes of every workspace.
+//   word[0] = first recorded deltas_status, word[1] = detail, words 2..3 reserved.
+// ---------------------------------------------------------------------------------------------
+constexpr size_t kStatusBytes = 256;   // status word padded so the rest stays 256-byte aligned
+
+__device__ __forceinline__ void record_status(int32_t* status, int32_t code, int32_t detail) {
+    if (status == nullptr) return;
+    if (atomicCAS(status, 0, code) == 0) {
+        atomicExch(status + 1, detail);
+    }
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Bounded-wait budget for every device-side spin (inter-CTA flags, mbarriers): about one second.
+constexpr uint64_t kWaitBudgetNs = 1000000000ull;
+
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+template <typename T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) { return __float2bfloat16_rn(x); }
+
+inline int elt_bytes(int32_t dtype) { return dtype == DELTAS_BF16 ? 2 : 4; }
+
+// ---------------------------------------------------------------------------------------------
+// Launch arguments
+// ---------------------------------------------------------------------------------------------
+struct GdnArgs {
+    int L, Hk, Hv, dk, dv, T, dtype;
+    float q_scale;
+    const void* q;
+    const void* k;
+    const void* v;
+    const float* g;
+    const float* beta;
+    float* state;
+    void* out;
+    float* partials;
+    int32_t* status;
+};
+
+struct KvPlanes {
+    int Lf, Hkv, D, dtype, capacity;
+    void* k_cache;
+    void* v_cache;
+    int32_t* tok_chunk;
+    int32_t* tok_pos;
+};
+
+// Kernel launchers (return the launch error, cudaSuccess when enqueued).
+cudaError_t launch_gdn_update_simt(const GdnArgs& a, cudaStream_t s);
+bool gdn_tc_supported(const GdnArgs& a);
+cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s);
+cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, const float* sa,
+                               float* partials, cudaStream_t s);
+cudaError_t launch_score_chunks(int L, int Hv, const float* partials, int chunk_id, float* scores,
+                                cudaStream_t s);
+size_t select_workspace_bytes(int cache_len);
+cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_chunks,
+                                 const int32_t* tok_chunk, const float* scores, int32_t* retain_idx,
+                                 int32_t* n_retained, uint8_t* mask, void* ws, int32_t* status,
+                                 cudaStream_t s);
+size_t compact_workspace_bytes(const KvPlanes& kv, int cache_len);
+cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, const int32_t* n_retained,
+                              int cache_len, void* ws, int32_t* status, cudaStream_t s);
+cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_new, const void* v_new,
+                             int n_new, int chunk_id, int first_pos, cudaStream_t s);
+
+int device_sm_count();
+
+}  // namespace deltas

@@ -1,0 +1,352 @@
+// Retain selection (Sec. 3.3; Alg. 1 eviction branch) in one 1024-thread CTA.
+//
+// Every token of a chunk carries its chunk's score, so candidates form runs: maximal stretches
+// of consecutive slots with the same arrival chunk.  Inside a run the ranking key
+// (score desc, slot asc) orders tokens by slot, and two runs never interleave in slot order, so
+// the token-level rule "keep the best tokens" keeps a prefix of each run.  The kernel therefore
+// works on runs (tens of them in a streaming cache, at most one per candidate slot in general):
+//
+//   A. runs: per-thread slot segments, block scan of run starts, c_lo / c_hi reduction;
+//   B. per run: length, temporal span floor((chunk - c_lo) * N / (c_hi - c_lo + 1)), 64-bit key
+//      (total-order score bits << 32 | ~first_slot): larger key = better token;
+//   C. per span: token-weighted radix select (8 passes of 8 bits, one warp scans each span's
+//      histogram) finds the run where the span's quota min(q, |span|) runs out -> kept1[run];
+//   D. fill: the same select over all runs' remainders (key re-based at the first unkept slot)
+//      with target R - sum(kept1) -> kept[run];
+//   E. output: scan of kept over runs, every slot writes itself to retain_idx if it lies in its
+//      run's kept prefix; sink and window slots are copied through.
+// Nothing is sorted; the cost is a few passes over the slots plus 16 passes over the runs.
+#include "internal.cuh"
+
+namespace deltas {
+namespace {
+
+constexpr int kSelThreads = 1024;
+constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kMaxSpans = 32;
+
+enum SpanMode : int { kNone = 0, kAll = 1, kSome = 2 };
+
+struct SelWs {          // workspace arrays, each [cache_len]
+    int32_t* run_start;
+    int32_t* run_chunk;
+    int32_t* run_len;
+    int32_t* run_span;
+    int32_t* kept1;
+    int32_t* kept;
+    int32_t* out_off;
+    uint64_t* run_key;
+};
+
+__host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+__host__ __device__ inline SelWs carve(void* ws, int cap) {
+    char* p = static_cast<char*>(ws) + kStatusBytes;
+    SelWs w;
+    const size_t i32 = align256(sizeof(int32_t) * (size_t)(cap > 0 ? cap : 1));
+    w.run_start = reinterpret_cast<int32_t*>(p); p += i32;
+    w.run_chunk = reinterpret_cast<int32_t*>(p); p += i32;
+    w.run_len = reinterpret_cast<int32_t*>(p); p += i32;
+    w.run_span = reinterpret_cast<int32_t*>(p); p += i32;
+    w.kept1 = reinterpret_cast<int32_t*>(p); p += i32;
+    w.kept = reinterpret_cast<int32_t*>(p); p += i32;
+    w.out_off = reinterpret_cast<int32_t*>(p); p += i32;
+    w.run_key = reinterpret_cast<uint64_t*>(p);
+    return w;
+}
+
+__device__ __forceinline__ uint32_t score_order_bits(float s) {
+    const uint32_t b = __float_as_uint(s);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// Exclusive block scan of one int per thread (1024 threads); *total receives the sum.
+__device__ int block_exclusive_scan(int v, int* warp_sums, int* total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int m = 1; m < 32; m <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, m);
+        if (lane >= m) x += y;
+    }
+    if (lane == 31) warp_sums[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = warp_sums[lane];
+        int s = w;
+#pragma unroll
+        for (int m = 1; m < 32; m <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, s, m);
+            if (lane >= m) s += y;
+        }
+        warp_sums[lane] = s - w;               // exclusive prefix of the warp totals
+        if (lane == 31) *total = s;
+    }
+    __syncthreads();
+    const int r = warp_sums[warp] + x - v;
+    __syncthreads();                           // warp_sums may be reused right after
+    return r;
+}
+
+// Token-weighted top selection per group.  For every group j with mode[j] == kSome, finds the
+// key K*_j of the item at which the cumulative weight, in descending key order, first reaches
+// target[j]; on return prefix[j] = K*_j and target[j] = weight to take from that item
+// (1 <= target[j] <= its weight).  Keys are unique.  One warp scans each group's histogram.
+__device__ void weighted_select(int n_items, const uint64_t* keys, const int32_t* weights,
+                                const int32_t* groups, int G, uint64_t* prefix, int* target,
+                                const int* mode, unsigned* hist)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int j = threadIdx.x; j < G; j += kSelThreads) prefix[j] = 0;
+    for (int pass = 0; pass < 8; ++pass) {
+        const int shift = 56 - 8 * pass;
+        for (int e = threadIdx.x; e < G * 256; e += kSelThreads) hist[e] = 0;
+        __syncthreads();
+        for (int r = threadIdx.x; r < n_items; r += kSelThreads) {
+            const int j = groups ? groups[r] : 0;
+            if (mode[j] != kSome) continue;
+            const int w = weights[r];
+            if (w <= 0) continue;
+            const uint64_t key = keys[r];
+            if (pass > 0 && (key >> (shift + 8)) != (prefix[j] >> (shift + 8))) continue;
+            atomicAdd(&hist[j * 256 + (int)((key >> shift) & 255u)], (unsigned)w);
+        }
+        __syncthreads();
+        for (int j = warp; j < G; j += kSelWarps) {
+            if (mode[j] != kSome) continue;
+            // lane l holds digits 255-8l .. 248-8l (descending digit order across lanes)
+            const unsigned* hj = hist + j * 256;
+            unsigned local = 0;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) local += hj[255 - 8 * lane - e];
+            unsigned incl = local;
+#pragma unroll
+            for (int m = 1; m < 32; m <<= 1) {
+                const unsigned y = __shfl_up_sync(0xffffffffu, incl, m);
+                if (lane >= m) incl += y;
+            }
+            const unsigned t = (unsigned)target[j];
+            const unsigned hit = __ballot_sync(0xffffffffu, incl >= t);
+            const int src = __ffs(hit) - 1;                // first lane whose prefix reaches t
+            if (lane == src) {
+                unsigned cum = incl - local;
+                int digit = 255 - 8 * lane;
+                for (int e = 0; e < 8; ++e, --digit) {
+                    const unsigned c = hj[digit];
+                    if (cum + c >= t) break;
+                    cum += c;
+                }
+                prefix[j] |= (uint64_t)digit << shift;
+                target[j] = (int)(t - cum);
+            }
+        }
+        __syncthreads();
+    }
+}
+
+struct SelArgs {
+    int M, n_s, n_w, N, T, n_chunks;
+    const int32_t* tok_chunk;
+    const float* scores;
+    int32_t* retain_idx;
+    int32_t* n_retained;
+    uint8_t* mask;
+    int32_t* status;
+    SelWs ws;
+};
+
+__global__ void __launch_bounds__(kSelThreads, 1)
+select_retain_kernel(SelArgs a)
+{
+    __shared__ int warp_sums[32];
+    __shared__ int s_total;
+    __shared__ int s_bad;
+    __shared__ int s_cmin[kSelWarps], s_cmax[kSelWarps];
+    __shared__ int s_span_total[kMaxSpans];
+    __shared__ int s_mode[kMaxSpans];
+    __shared__ int s_target[kMaxSpans];
+    __shared__ uint64_t s_prefix[kMaxSpans];
+    __shared__ unsigned s_hist[kMaxSpans * 256];
+    __shared__ int s_fill_mode[1], s_fill_target[1];
+    __shared__ uint64_t s_fill_prefix[1];
+
+    const int tid = threadIdx.x;
+    const int T = a.T;
+    if (tid == 0) s_bad = -1;
+    __syncthreads();
+    for (int i = tid; i < T; i += kSelThreads) {
+        const int c = a.tok_chunk[i];
+        if (c < 0 || c >= a.n_chunks) atomicMax(&s_bad, i);
+    }
+    __syncthreads();
+    if (s_bad >= 0) {
+        if (tid == 0) { record_status(a.status, DELTAS_ERR_DEVICE_INDEX, s_bad); *a.n_retained = 0; }
+        return;
+    }
+    if (T <= a.M) {
+        for (int i = tid; i < T; i += kSelThreads) {
+            a.retain_idx[i] = i;
+            if (a.mask) a.mask[i] = 1;
+        }
+        if (tid == 0) *a.n_retained = T;
+        return;
+    }
+
+    const int N = a.N < 1 ? 1 : a.N;
+    const int lo = a.n_s, hi = T - a.n_w;
+    const int n_cand = hi - lo;
+    const int R = a.M - a.n_s - a.n_w;
+    const int quota = R / N;
+
+    // ---- A. runs over the candidate slots
+    const int items = (n_cand + kSelThreads - 1) / kSelThreads;
+    const int seg_lo = min(lo + tid * items, hi), seg_hi = min(seg_lo + items, hi);
+    int n_starts = 0, cmin = INT_MAX, cmax = INT_MIN;
+    for (int i = seg_lo; i < seg_hi; ++i) {
+        const int c = a.tok_chunk[i];
+        n_starts += (i == lo || c != a.tok_chunk[i - 1]);
+        cmin = min(cmin, c);
+        cmax = max(cmax, c);
+    }
+    const int run_base = block_exclusive_scan(n_starts, warp_sums, &s_total);
+    const int n_runs = s_total;
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+        cmin = min(cmin, __shfl_xor_sync(0xffffffffu, cmin, m));
+        cmax = max(cmax, __shfl_xor_sync(0xffffffffu, cmax, m));
+    }
+    if ((tid & 31) == 0) { s_cmin[tid >> 5] = cmin; s_cmax[tid >> 5] = cmax; }
+    {
+        int r = run_base;
+        for (int i = seg_lo; i < seg_hi; ++i) {
+            const int c = a.tok_chunk[i];
+            if (i == lo || c != a.tok_chunk[i - 1]) {
+                a.ws.run_start[r] = i;
+                a.ws.run_chunk[r] = c;
+                ++r;
+            }
+        }
+    }
+    if (tid < kMaxSpans) s_span_total[tid] = 0;
+    __syncthreads();
+    int c_lo = INT_MAX, c_hi = INT_MIN;
+    for (int w = 0; w < kSelWarps; ++w) { c_lo = min(c_lo, s_cmin[w]); c_hi = max(c_hi, s_cmax[w]); }
+    const long long span_width = (long long)c_hi - c_lo + 1;
+
+    // ---- B. per-run length, span and key
+    for (int r = tid; r < n_runs; r += kSelThreads) {
+        const int start = a.ws.run_start[r];
+        const int end = (r + 1 < n_runs) ? a.ws.run_start[r + 1] : hi;
+        const int c = a.ws.run_chunk[r];
+        const int span = (int)(((long long)(c - c_lo) * N) / span_width);
+        a.ws.run_len[r] = end - start;
+        a.ws.run_span[r] = span;
+        a.ws.run_key[r] = ((uint64_t)score_order_bits(a.scores[c]) << 32) | (uint64_t)(~(uint32_t)start);
+        atomicAdd(&s_span_total[span], end - start);
+    }
+    __syncthreads();
+    if (tid < N) {
+        const int tot = s_span_total[tid];
+        const int m = min(quota, tot);
+        s_target[tid] = m;
+        s_mode[tid] = (m == 0) ? kNone : (m == tot ? kAll : kSome);
+    }
+    __syncthreads();
+    // per-span quota actually granted (needed for the fill target)
+    int granted = 0;
+    if (tid == 0) for (int j = 0; j < N; ++j) granted += s_target[j];
+
+    // ---- C. per-span quota
+    weighted_select(n_runs, a.ws.run_key, a.ws.run_len, a.ws.run_span, N, s_prefix, s_target,
+                    s_mode, s_hist);
+    for (int r = tid; r < n_runs; r += kSelThreads) {
+        const int j = a.ws.run_span[r];
+        const int len = a.ws.run_len[r];
+        int k1 = 0;
+        if (s_mode[j] == kAll) k1 = len;
+        else if (s_mode[j] == kSome) {
+            const uint64_t key = a.ws.run_key[r];
+            k1 = key > s_prefix[j] ? len : (key == s_prefix[j] ? s_target[j] : 0);
+        }
+        a.ws.kept1[r] = k1;
+        a.ws.run_len[r] = len - k1;   // remainder weight for the fill
+        a.ws.run_key[r] = (a.ws.run_key[r] & 0xFFFFFFFF00000000ull) |
+                          (uint64_t)(~(uint32_t)(a.ws.run_start[r] + k1));
+    }
+    if (tid == 0) {
+        const int fill = R - granted;
+        s_fill_target[0] = fill;
+        s_fill_mode[0] = fill > 0 ? kSome : kNone;
+    }
+    __syncthreads();
+
+    // ---- D. fill the unused capacity from the best remaining candidates
+    weighted_select(n_runs, a.ws.run_key, a.ws.run_len, nullptr, 1, s_fill_prefix, s_fill_target,
+                    s_fill_mode, s_hist);
+    const int per = (n_runs + kSelThreads - 1) / kSelThreads;
+    const int r_lo = min(tid * per, n_runs), r_hi = min(r_lo + per, n_runs);
+    int my_kept = 0;
+    for (int r = r_lo; r < r_hi; ++r) {
+        const int rem = a.ws.run_len[r];
+        int k2 = 0;
+        if (s_fill_mode[0] == kSome && rem > 0) {
+            const uint64_t key = a.ws.run_key[r];
+            k2 = key > s_fill_prefix[0] ? rem : (key == s_fill_prefix[0] ? s_fill_target[0] : 0);
+        }
+        const int k = a.ws.kept1[r] + k2;
+        a.ws.kept[r] = k;
+        my_kept += k;
+    }
+
+    // ---- E. output offsets and slot writes
+    int off = block_exclusive_scan(my_kept, warp_sums, &s_total);
+    for (int r = r_lo; r < r_hi; ++r) {
+        a.ws.out_off[r] = off;
+        off += a.ws.kept[r];
+    }
+    __syncthreads();
+    {
+        int r = run_base - 1;
+        for (int i = seg_lo; i < seg_hi; ++i) {
+            const int c = a.tok_chunk[i];
+            if (i == lo || c != a.tok_chunk[i - 1]) ++r;
+            const int pos = i - a.ws.run_start[r];
+            const bool keep = pos < a.ws.kept[r];
+            if (keep) a.retain_idx[a.n_s + a.ws.out_off[r] + pos] = i;
+            if (a.mask) a.mask[i] = keep ? 1 : 0;
+        }
+    }
+    for (int i = tid; i < a.n_s; i += kSelThreads) {
+        a.retain_idx[i] = i;
+        if (a.mask) a.mask[i] = 1;
+    }
+    for (int i = hi + tid; i < T; i += kSelThreads) {
+        a.retain_idx[a.M - a.n_w + (i - hi)] = i;
+        if (a.mask) a.mask[i] = 1;
+    }
+    if (tid == 0) *a.n_retained = a.M;
+}
+
+}  // namespace
+
+size_t select_workspace_bytes(int cache_len) {
+    const size_t cap = (size_t)(cache_len > 0 ? cache_len : 1);
+    return kStatusBytes + 7 * align256(sizeof(int32_t) * cap) + align256(sizeof(uint64_t) * cap);
+}
+
+cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_chunks,
+                                 const int32_t* tok_chunk, const float* scores, int32_t* retain_idx,
+                                 int32_t* n_retained, uint8_t* mask, void* ws, int32_t* status,
+                                 cudaStream_t s)
+{
+    SelArgs a;
+    a.M = p.budget_M; a.n_s = p.n_sink; a.n_w = p.n_window; a.N = p.n_buckets;
+    a.T = cache_len; a.n_chunks = num_chunks;
+    a.tok_chunk = tok_chunk; a.scores = scores; a.retain_idx = retain_idx;
+    a.n_retained = n_retained; a.mask = mask; a.status = status;
+    a.ws = carve(ws, cache_len);
+    select_retain_kernel<<<1, kSelThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace deltas

@@ -1,0 +1,80 @@
+"""Alg. 1 (DeltaS: state-guided KV eviction) driven through the C ABI on one GPU.
+
+Per arriving chunk c, all on one CUDA stream and with no host synchronisation:
+
+1. ``deltas_gdn_chunk_update`` — Prefill(c) of every gated-delta layer: the state S goes from
+   S_before to S_after (Eq. 1) and the per-(layer, head) drift partials come out of the same
+   kernel (the pre-chunk state is never stored separately);
+2. ``deltas_score_chunks`` — Delta S of Eq. 3, stored as score[c] (shared by c's tokens);
+3. ``deltas_append_kv`` — c's keys/values enter every full-attention cache, with their arrival
+   chunk and stream position;
+4. if the cache holds more than M tokens: ``deltas_select_retain`` then ``deltas_compact_kv``.
+
+The host tracks the cache length without reading the device: after an eviction it is exactly M
+(the selection keeps min(T, M) tokens).
+"""
+from __future__ import annotations
+
+import torch
+
+from . import _lib as L
+
+
+class DeltaSStream:
+    def __init__(self, *, num_layers, num_k_heads, num_v_heads, head_dim, act_dtype: torch.dtype,
+                 kv_layers, kv_heads, kv_head_dim, kv_dtype: torch.dtype, budget_M, n_sink=0,
+                 n_window=0, n_buckets=1, chunk_len, max_chunks, q_scale=None, state0=None,
+                 device="cuda"):
+        self.gdn = L.gdn_desc(num_layers, num_k_heads, num_v_heads, head_dim, act_dtype, q_scale)
+        self.policy = L.policy(budget_M, n_sink, n_window, n_buckets)
+        self.capacity = budget_M + chunk_len
+        self.kv = L.kv_desc(kv_layers, kv_heads, kv_head_dim, kv_dtype, self.capacity)
+        self.chunk_len = chunk_len
+        self.max_chunks = max_chunks
+        dev = torch.device(device)
+        self.state = (state0.clone() if state0 is not None else
+                      torch.zeros(num_layers, num_v_heads, head_dim, head_dim, device=dev))
+        self.partials = torch.zeros(num_layers, num_v_heads, 2, device=dev)
+        self.chunk_scores = torch.zeros(max_chunks, device=dev)
+        self.k_cache = torch.zeros(kv_layers, kv_heads, self.capacity, kv_head_dim, dtype=kv_dtype, device=dev)
+        self.v_cache = torch.zeros_like(self.k_cache)
+        self.tok_chunk = torch.zeros(self.capacity, dtype=torch.int32, device=dev)
+        self.tok_pos = torch.zeros(self.capacity, dtype=torch.int32, device=dev)
+        self.retain_idx = torch.zeros(budget_M, dtype=torch.int32, device=dev)
+        self.n_retained = torch.zeros(1, dtype=torch.int32, device=dev)
+        ws = max(L.deltas_gdn_chunk_update_workspace_size(self.gdn, chunk_len),
+                 L.deltas_select_retain_workspace_size(self.capacity),
+                 L.deltas_compact_kv_workspace_size(self.kv, self.capacity))
+        self.workspace = L.alloc_workspace(ws, dev)
+        self.cache_len = 0
+        self.position = 0
+        self.chunk = 0
+        self.evictions = 0
+
+    def step(self, q, k, v, g, beta, k_new, v_new, out=None, stream=None):
+        """Process one chunk (Alg. 1 loop body).  Returns True if an eviction ran."""
+        c = self.chunk
+        if c >= self.max_chunks:
+            raise ValueError("stream longer than max_chunks")
+        T = int(k.shape[1])
+        L.deltas_gdn_chunk_update(self.gdn, T, q, k, v, g, beta, self.state, out, self.partials,
+                                  self.workspace, stream)
+        L.deltas_score_chunks(self.gdn.num_layers, self.gdn.num_v_heads, self.partials, c,
+                              self.chunk_scores, stream)
+        n_new = int(k_new.shape[2])
+        L.deltas_append_kv(self.kv, self.k_cache, self.v_cache, self.tok_chunk, self.tok_pos,
+                           self.cache_len, k_new, v_new, c, self.position, stream)
+        self.cache_len += n_new
+        self.position += n_new
+        self.chunk += 1
+        if self.cache_len > self.policy.budget_M:
+            L.deltas_select_retain(self.policy, self.cache_len, self.tok_chunk,
+                                   self.chunk_scores[: c + 1], self.retain_idx, self.n_retained,
+                                   None, self.workspace, stream)
+            L.deltas_compact_kv(self.kv, self.k_cache, self.v_cache, self.tok_chunk, self.tok_pos,
+                                self.retain_idx, self.n_retained, self.cache_len, self.workspace,
+                                stream)
+            self.cache_len = self.policy.budget_M
+            self.evictions += 1
+            return True
+        return False

@@ -1,0 +1,117 @@
+"""Host-side checks of the C ABI (no GPU): the library loads, exports every entry point that
+include/deltas.h declares, sizes workspaces, and rejects bad arguments before enqueueing
+anything (so these calls never touch a device)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2609_27470_gb300 import build
+    build.build()
+    from paper_2609_27470_gb300 import _lib
+    return _lib
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "deltas.h")).read()
+    return sorted(set(re.findall(r"DELTAS_API\s+[\w\s\*]+?\b(deltas_\w+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(L):
+    names = _declared()
+    assert len(names) == 14, names
+    lib = ctypes.CDLL(L.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(L.EXPORTED)
+
+
+def test_version_and_status_strings(L):
+    assert L.deltas_version().startswith("deltas ") and "sm_103a" in L.deltas_version()
+    for code in range(0, 7):
+        assert L.deltas_status_string(code) != "unknown status"
+    assert L.deltas_status_string(99) == "unknown status"
+
+
+def test_workspace_sizes(L):
+    d = L.GdnDesc(24, 16, 32, 128, 128, L.DELTAS_BF16, 0.088)
+    assert L.deltas_gdn_chunk_update_workspace_size(d, 1024) >= 16
+    assert L.deltas_state_drift_workspace_size(d) >= 16
+    a = L.deltas_select_retain_workspace_size(1000)
+    b = L.deltas_select_retain_workspace_size(100000)
+    assert 16 <= a < b
+    kv = L.KvDesc(8, 2, 256, L.DELTAS_BF16, 65536)
+    assert L.deltas_compact_kv_workspace_size(kv, 65536) > L.deltas_compact_kv_workspace_size(kv, 1024) > 0
+    bad = L.KvDesc(8, 2, 3, L.DELTAS_BF16, 100)   # 6-byte rows: not a multiple of 16 bytes
+    assert L.deltas_compact_kv_workspace_size(bad, 10) == 0
+
+
+FAKE = 0x10000   # a 256-byte aligned non-NULL address: every call below must reject before using it
+
+
+def test_gdn_update_argument_checks(L):
+    raw = L.raw()
+    ok = L.GdnDesc(1, 2, 4, 16, 16, L.DELTAS_F32, 0.25)
+    args = lambda desc, T=8, ws=FAKE, wsb=1 << 20: (ctypes.byref(desc) if desc else None, T, FAKE, FAKE, FAKE,
+                                                     FAKE, FAKE, FAKE, None, None, ws, wsb, None)
+    assert raw.deltas_gdn_chunk_update(*args(None)) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert raw.deltas_gdn_chunk_update(*args(L.GdnDesc(1, 3, 4, 16, 16, 0, 1.0))) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert raw.deltas_gdn_chunk_update(*args(L.GdnDesc(1, 2, 4, 48, 48, 0, 1.0))) == L.DELTAS_ERR_UNSUPPORTED
+    assert raw.deltas_gdn_chunk_update(*args(L.GdnDesc(1, 2, 4, 64, 32, 0, 1.0))) == L.DELTAS_ERR_UNSUPPORTED
+    assert raw.deltas_gdn_chunk_update(*args(L.GdnDesc(1, 2, 4, 16, 16, 7, 1.0))) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert raw.deltas_gdn_chunk_update(*args(ok, T=-1)) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert raw.deltas_gdn_chunk_update(*args(ok, ws=None)) == L.DELTAS_ERR_WORKSPACE
+    assert raw.deltas_gdn_chunk_update(*args(ok, ws=FAKE + 8)) == L.DELTAS_ERR_WORKSPACE
+    assert raw.deltas_gdn_chunk_update(*args(ok, wsb=4)) == L.DELTAS_ERR_WORKSPACE
+    # misaligned key pointer
+    assert raw.deltas_gdn_chunk_update(ctypes.byref(ok), 8, FAKE, FAKE + 4, FAKE, FAKE, FAKE, FAKE, None, None,
+                                       FAKE, 1 << 20, None) == L.DELTAS_ERR_INVALID_ARGUMENT
+    # output requested without q
+    assert raw.deltas_gdn_chunk_update(ctypes.byref(ok), 8, None, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None,
+                                       FAKE, 1 << 20, None) == L.DELTAS_ERR_INVALID_ARGUMENT
+
+
+def test_select_argument_checks(L):
+    raw = L.raw()
+
+    def call(pol, T=100, nch=10, ws=FAKE, wsb=1 << 24):
+        return raw.deltas_select_retain(ctypes.byref(pol) if pol else None, T, nch, FAKE, FAKE, FAKE, FAKE,
+                                        None, ws, wsb, None)
+    assert call(None) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert call(L.Policy(10, 5, 5, 1)) == L.DELTAS_ERR_INVALID_ARGUMENT     # M < n_s + n_w + 1
+    assert call(L.Policy(10, 0, 0, 33)) == L.DELTAS_ERR_UNSUPPORTED
+    assert call(L.Policy(10, 0, 0, -1)) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert call(L.Policy(10, 0, 0, 1), T=-5) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert call(L.Policy(10, 0, 0, 1), wsb=16) == L.DELTAS_ERR_WORKSPACE
+
+
+def test_compact_and_append_argument_checks(L):
+    raw = L.raw()
+    kv = L.KvDesc(2, 2, 64, L.DELTAS_BF16, 1000)
+    assert raw.deltas_compact_kv(ctypes.byref(kv), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1001, FAKE, 1 << 24,
+                                 None) == L.DELTAS_ERR_INVALID_ARGUMENT      # cache_len > capacity
+    assert raw.deltas_compact_kv(ctypes.byref(kv), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 500, FAKE, 64,
+                                 None) == L.DELTAS_ERR_WORKSPACE
+    bad = L.KvDesc(2, 2, 7, L.DELTAS_F32, 1000)
+    assert raw.deltas_compact_kv(ctypes.byref(bad), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 500, FAKE, 1 << 24,
+                                 None) == L.DELTAS_ERR_UNSUPPORTED
+    assert raw.deltas_append_kv(ctypes.byref(kv), FAKE, FAKE, FAKE, FAKE, 990, FAKE, FAKE, 20, 0, 0,
+                                None) == L.DELTAS_ERR_INVALID_ARGUMENT       # overflows capacity
+    assert raw.deltas_score_chunks(0, 4, FAKE, 0, FAKE, None) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert raw.deltas_score_chunks(2, 4, FAKE, -1, FAKE, None) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert raw.deltas_clear_device_status(None, None) == L.DELTAS_ERR_WORKSPACE
+
+
+def test_binding_refuses_cpu_tensors(L):
+    import torch
+    d = L.gdn_desc(1, 1, 1, 16, torch.float32)
+    x = torch.zeros(1, 4, 1, 16)
+    with pytest.raises(ValueError):
+        L.deltas_gdn_chunk_update(d, 4, x, x, x, torch.zeros(1, 4, 1), torch.zeros(1, 4, 1),
+                                  torch.zeros(1, 1, 16, 16), None, None, torch.zeros(256, dtype=torch.uint8))

@@ -1,0 +1,165 @@
+"""GPU parity of the gated-delta chunk update + fused drift partials (Sec. 3.2, Eq. 1-3) and of
+the standalone drift / score kernels, against the fp64 CPU oracle on the same seeded inputs.
+
+Tolerances (floating point):
+* state: relative Frobenius error <= 2e-3 per (layer, head) at every chunk boundary;
+* drift partials: relative error <= 1e-3 on sum (S_after - S_before)^2 and sum S_before^2;
+* read-out o: relative Frobenius error per (layer, head) <= 2e-3 (+ bfloat16 output rounding,
+  2^-8 relative, when the activations are bfloat16);
+* chunk score: |Delta| / |ref| <= 1e-3, and +inf must match +inf.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_27470_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+STATE_TOL = 2e-3
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2609_27470_gb300 import _lib
+    return _lib
+
+
+def _f64(t):
+    return t.detach().float().cpu().double().numpy()
+
+
+def _per_head_rel(a, b):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    axes = tuple(range(2, a.ndim))
+    num = np.sqrt(np.sum((a - b) ** 2, axis=axes))
+    den = np.sqrt(np.sum(b ** 2, axis=axes))
+    return num / np.maximum(den, 1e-30)
+
+
+def _run_gpu(L, x, state, want_out, dtype, q_scale):
+    Lg, T, Hk, d = x["k"].shape
+    Hv = x["v"].shape[2]
+    desc = L.gdn_desc(Lg, Hk, Hv, d, dtype, q_scale)
+    dev = torch.device("cuda")
+    xs = {k: v.to(dev) for k, v in x.items()}
+    st = state.to(dev).clone()
+    out = torch.empty(Lg, T, Hv, d, dtype=dtype, device=dev) if want_out else None
+    part = torch.full((Lg, Hv, 2), -1.0, device=dev)
+    ws = L.alloc_workspace(L.deltas_gdn_chunk_update_workspace_size(desc, T), dev)
+    L.deltas_gdn_chunk_update(desc, T, xs["q"] if want_out else None, xs["k"], xs["v"], xs["g"], xs["beta"],
+                              st, out, part, ws)
+    torch.cuda.synchronize()
+    assert L.deltas_get_device_status(ws) == (0, 0)
+    return st, out, part
+
+
+def _check_chunk(L, x, state0, want_out, dtype, q_scale):
+    st, out, part = _run_gpu(L, x, state0, want_out, dtype, q_scale)
+    S_ref, o_ref = oracle.gdn_recurrence(_f64(x["q"]), _f64(x["k"]), _f64(x["v"]), _f64(x["g"]), _f64(x["beta"]),
+                                         _f64(state0), q_scale=q_scale, want_out=want_out)
+    rel = _per_head_rel(_f64(st), S_ref)
+    assert rel.max() <= STATE_TOL, f"state rel err {rel.max():.3e}"
+    p_ref = oracle.drift_partials(_f64(state0), S_ref)
+    p = _f64(part)
+    np.testing.assert_allclose(p[..., 1], p_ref[..., 1], rtol=1e-5, atol=0)
+    np.testing.assert_allclose(p[..., 0], p_ref[..., 0], rtol=1e-3, atol=1e-30)
+    if want_out:
+        tol = STATE_TOL + (2.0 ** -8 if dtype == torch.bfloat16 else 0.0)
+        o = _f64(out).transpose(0, 2, 1, 3)            # [L,Hv,T,d] per (layer, head)
+        orl = _per_head_rel(o, o_ref.transpose(0, 2, 1, 3))
+        assert orl.max() <= tol, f"out rel err {orl.max():.3e}"
+    return st, rel.max()
+
+
+@pytest.mark.parametrize("d", [16, 32, 64, 128])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("T", [1, 100, 257])
+def test_gdn_update_shapes(L, d, dtype, T):
+    """Every head size, both activation dtypes, ragged token counts, grouped keys (Hk=2, Hv=4),
+    two layers, with read-out and drift partials."""
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    x = inputs.gdn_chunk(2, T, 2, 4, d, dtype, inputs.seed_for(1, d, T))
+    s0 = inputs.initial_state(2, 4, d, inputs.seed_for(2, d, T))
+    _check_chunk(L, x, s0, True, tdt, d ** -0.5)
+
+
+def test_gdn_update_tiny_stream_from_zero(L):
+    """Tiny workload: 8 chunks x 64 tokens, d = 16, fp32, zero start state; every chunk boundary
+    is compared against the oracle replaying that chunk from the GPU's own S_before, and the
+    final state against the oracle's own trajectory."""
+    Lg, Hk, Hv, d, C = 1, 2, 2, 16, 64
+    state = torch.zeros(Lg, Hv, d, d)
+    ref = np.zeros((Lg, Hv, d, d))
+    for c in range(8):
+        x = inputs.gdn_chunk(Lg, C, Hk, Hv, d, "f32", inputs.seed_for(0, 0, c))
+        st, _ = _check_chunk(L, x, state, False, torch.float32, 0.25)
+        ref, _ = oracle.gdn_recurrence(None, _f64(x["k"]), _f64(x["v"]), _f64(x["g"]), _f64(x["beta"]), ref)
+        state = st.cpu()
+    assert _per_head_rel(state.double().numpy(), ref).max() <= STATE_TOL
+
+
+def test_gdn_update_zero_tokens(L):
+    """n_tokens = 0: the state is unchanged, partials are (0, ||S_before||^2)."""
+    s0 = inputs.initial_state(1, 4, 64, 5)
+    x = inputs.gdn_chunk(1, 0, 2, 4, 64, "bf16", 6)
+    st, _, part = _run_gpu(L, x, s0, False, torch.bfloat16, 0.125)
+    assert torch.equal(st.cpu(), s0)
+    p = part.cpu().double().numpy()
+    assert np.all(p[..., 0] == 0)
+    np.testing.assert_allclose(p[..., 1], np.sum(s0.double().numpy() ** 2, axis=(2, 3)), rtol=1e-5)
+
+
+def test_gdn_update_layer_width_chunk(L):
+    """The single-layer workload's shape: 16 key heads, 32 value heads, d = 128, bf16, one chunk
+    of 1024 tokens (spans many tiles), with read-out."""
+    x = inputs.gdn_chunk(1, 1024, 16, 32, 128, "bf16", inputs.seed_for(7, 1, 0))
+    s0 = inputs.initial_state(1, 32, 128, 8)
+    _check_chunk(L, x, s0, True, torch.bfloat16, 128 ** -0.5)
+
+
+def test_gdn_update_slow_decay_four_chunks(L):
+    """Heads with long memory (alpha close to 1) keep errors from decaying away: 4 chunks of 1024
+    tokens, compared at every chunk boundary with the oracle's own trajectory."""
+    Lg, Hk, Hv, d = 1, 2, 4, 128
+    state = inputs.initial_state(Lg, Hv, d, 9)
+    ref = state.double().numpy()
+    for c in range(4):
+        x = inputs.gdn_chunk(Lg, 1024, Hk, Hv, d, "bf16", inputs.seed_for(9, c), decay_scale=0.002)
+        st, _, _ = _run_gpu(L, x, state, False, torch.bfloat16, None)
+        ref, _ = oracle.gdn_recurrence(None, _f64(x["k"]), _f64(x["v"]), _f64(x["g"]), _f64(x["beta"]), ref)
+        rel = _per_head_rel(_f64(st), ref)
+        assert rel.max() <= STATE_TOL, f"chunk {c}: {rel.max():.3e}"
+        state = st.cpu()
+
+
+def test_state_drift_kernel(L):
+    """deltas_state_drift partials == oracle (Eq. 3 numerator/denominator per layer and head)."""
+    sb = inputs.initial_state(3, 4, 128, 11)
+    sa = sb * 0.9 + 0.05 * inputs.initial_state(3, 4, 128, 12)
+    desc = L.gdn_desc(3, 4, 4, 128, torch.bfloat16)
+    part = torch.zeros(3, 4, 2, device="cuda")
+    ws = L.alloc_workspace(L.deltas_state_drift_workspace_size(desc))
+    L.deltas_state_drift(desc, sb.cuda(), sa.cuda(), part, ws)
+    p_ref = oracle.drift_partials(sb.double().numpy(), sa.double().numpy())
+    np.testing.assert_allclose(part.cpu().double().numpy(), p_ref, rtol=1e-5)
+
+
+def test_score_kernel(L):
+    """deltas_score_chunks == oracle Eq. 3 on the same float32 partials, incl. the zero-norm
+    reading (0/0 -> 0, x/0 -> inf)."""
+    rng = np.random.default_rng(13)
+    scores = torch.zeros(8, device="cuda")
+    for cid, (Lg, Hv) in enumerate([(1, 1), (3, 4), (24, 32), (5, 100)]):
+        p = rng.exponential(size=(Lg, Hv, 2)).astype(np.float32)
+        L.deltas_score_chunks(Lg, Hv, torch.from_numpy(p).cuda(), cid, scores)
+        ref = oracle.chunk_score(p.astype(np.float64))
+        assert abs(scores[cid].item() - ref) <= 1e-6 * abs(ref)
+    z = np.zeros((2, 3, 2), np.float32)
+    L.deltas_score_chunks(2, 3, torch.from_numpy(z).cuda(), 5, scores)
+    assert scores[5].item() == 0.0
+    z[1, 2, 0] = 1e-3
+    L.deltas_score_chunks(2, 3, torch.from_numpy(z).cuda(), 6, scores)
+    assert scores[6].item() == float("inf") and oracle.chunk_score(z.astype(np.float64)) == float("inf")

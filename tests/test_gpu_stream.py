@@ -1,0 +1,65 @@
+"""End-to-end Alg. 1 through the C ABI on the GPU vs the CPU oracle's Alg. 1 loop.
+
+Selection is compared given identical scores (the oracle ranks with the GPU's own float32 chunk
+scores), so a near-tie in drift cannot flip an eviction; the scores themselves are compared
+within the drift tolerance (1e-3 relative, +inf == +inf)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle.stream import run_stream
+from paper_2609_27470_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+
+def _np(t):
+    return t.view(torch.int16).numpy() if t.dtype == torch.bfloat16 else t.numpy()
+
+
+@pytest.mark.parametrize("cfg", [
+    # tiny workload, both policies: (a) pure top chunks, (b) sink + window + 2 spans
+    dict(L=1, Hk=2, Hv=2, d=16, dt="f32", C=64, n_ch=8, Lf=1, Hkv=2, D=16, M=256, n_s=0, n_w=0, N=1, zero=True),
+    dict(L=1, Hk=2, Hv=2, d=16, dt="f32", C=64, n_ch=8, Lf=1, Hkv=2, D=16, M=256, n_s=4, n_w=64, N=2, zero=True),
+    # wider heads, bf16, ragged chunk length, paper-like policy
+    dict(L=2, Hk=2, Hv=4, d=128, dt="bf16", C=120, n_ch=12, Lf=2, Hkv=2, D=256, M=600, n_s=4, n_w=128, N=4,
+         zero=False),
+])
+def test_stream_matches_oracle(cfg):
+    from paper_2609_27470_gb300.stream import DeltaSStream
+    dev = torch.device("cuda")
+    tdt = torch.float32 if cfg["dt"] == "f32" else torch.bfloat16
+    chunks = [inputs.gdn_chunk(cfg["L"], cfg["C"], cfg["Hk"], cfg["Hv"], cfg["d"], cfg["dt"], inputs.seed_for(3, c))
+              for c in range(cfg["n_ch"])]
+    kvs = [inputs.kv_chunk(cfg["Lf"], cfg["Hkv"], cfg["C"], cfg["D"], cfg["dt"], inputs.seed_for(4, c))
+           for c in range(cfg["n_ch"])]
+    s0 = (torch.zeros(cfg["L"], cfg["Hv"], cfg["d"], cfg["d"]) if cfg["zero"]
+          else inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 5))
+    s = DeltaSStream(num_layers=cfg["L"], num_k_heads=cfg["Hk"], num_v_heads=cfg["Hv"], head_dim=cfg["d"],
+                     act_dtype=tdt, kv_layers=cfg["Lf"], kv_heads=cfg["Hkv"], kv_head_dim=cfg["D"], kv_dtype=tdt,
+                     budget_M=cfg["M"], n_sink=cfg["n_s"], n_window=cfg["n_w"], n_buckets=cfg["N"],
+                     chunk_len=cfg["C"], max_chunks=cfg["n_ch"], state0=s0.to(dev), device=dev)
+    for c in range(cfg["n_ch"]):
+        x = {k: v.to(dev) for k, v in chunks[c].items()}
+        s.step(x["q"], x["k"], x["v"], x["g"], x["beta"], kvs[c][0].to(dev), kvs[c][1].to(dev))
+    torch.cuda.synchronize()
+    from paper_2609_27470_gb300 import _lib as L
+    assert L.deltas_get_device_status(s.workspace) == (0, 0)
+    gpu_scores = s.chunk_scores.cpu().numpy()
+    f = lambda t: t.float().numpy()
+    ref = run_stream(lambda c: tuple(f(chunks[c][k]) for k in ("q", "k", "v", "g", "beta")),
+                     lambda c: (_np(kvs[c][0]), _np(kvs[c][1])), s0.double().numpy(), cfg["n_ch"],
+                     dict(budget_M=cfg["M"], n_sink=cfg["n_s"], n_window=cfg["n_w"], n_buckets=cfg["N"]),
+                     capacity=s.capacity, score_override=gpu_scores)
+    fin = np.isfinite(ref.chunk_scores)
+    assert np.array_equal(np.isfinite(gpu_scores), fin)
+    np.testing.assert_allclose(gpu_scores[fin], ref.chunk_scores[fin], rtol=1e-3)
+    st = s.state.cpu().double().numpy()
+    rel = np.sqrt(((st - ref.state) ** 2).sum(axis=(2, 3)) / (ref.state ** 2).sum(axis=(2, 3)))
+    assert rel.max() <= 2e-3
+    n = s.cache_len
+    assert n == ref.cache_len and s.evictions == len(ref.evictions)
+    assert np.array_equal(_np(s.k_cache[:, :, :n].cpu()), ref.k_cache[:, :, :n])
+    assert np.array_equal(_np(s.v_cache[:, :, :n].cpu()), ref.v_cache[:, :, :n])
+    assert np.array_equal(s.tok_chunk[:n].cpu().numpy(), ref.tok_chunk[:n])
+    assert np.array_equal(s.tok_pos[:n].cpu().numpy(), ref.tok_pos[:n])
