@@ -6,9 +6,10 @@
 // The difference is formed element by element before squaring, never as
 // |A|^2 - 2<A,B> + |B|^2, which cancels badly when the drift is small.
 //
-// score_chunks: one warp-sized CTA reduces the [L][Hv][2] partials in a fixed order (lane-strided
-// double sums, then a fixed xor tree), applies sqrt(num_l)/sqrt(den_l) per layer with the
-// zero-norm reading (0/0 -> 0, x/0 -> +inf) and stores the layer mean as the chunk's score.
+// score_chunks: one CTA reduces the [L][Hv][2] partials in a fixed order (lane-strided double
+// sums, a fixed xor tree per layer, layer terms added in a fixed order), applies
+// sqrt(num_l)/sqrt(den_l) per layer with the zero-norm reading (0/0 -> 0, x/0 -> +inf) and stores
+// the layer mean as the chunk's score.
 #include "internal.cuh"
 
 namespace deltas {
@@ -46,13 +47,18 @@ state_drift_kernel(int n_elem4, const float4* __restrict__ sb, const float4* __r
     }
 }
 
-__global__ void __launch_bounds__(32)
+constexpr int kScoreThreads = 1024;
+
+// One warp per layer (layers strided over the 32 warps): lane-strided double sums over the
+// heads, a fixed xor tree, the per-layer ratio; then warp 0 adds the layer terms in layer order.
+__global__ void __launch_bounds__(kScoreThreads)
 score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk_id,
                     float* __restrict__ scores)
 {
-    const int lane = threadIdx.x;
-    double total = 0.0;
-    for (int l = 0; l < L; ++l) {
+    __shared__ double term_sum[kScoreThreads / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    double acc = 0.0;
+    for (int l = warp; l < L; l += kScoreThreads / 32) {
         double num = 0.0, den = 0.0;
         for (int h = lane; h < Hv; h += 32) {
             num += (double)partials[((size_t)l * Hv + h) * 2 + 0];
@@ -66,9 +72,15 @@ score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk
         double term;
         if (den > 0.0) term = sqrt(num) / sqrt(den);
         else term = (num > 0.0) ? (double)INFINITY : 0.0;
-        total += term;
+        acc += term;   // layers l, l + 32, ... in increasing order
     }
-    if (lane == 0) scores[chunk_id] = (float)(total / (double)L);
+    if (lane == 0) term_sum[warp] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double total = 0.0;
+        for (int w = 0; w < kScoreThreads / 32; ++w) total += term_sum[w];
+        scores[chunk_id] = (float)(total / (double)L);
+    }
 }
 
 }  // namespace
@@ -85,7 +97,7 @@ cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, c
 cudaError_t launch_score_chunks(int L, int Hv, const float* partials, int chunk_id, float* scores,
                                 cudaStream_t s)
 {
-    score_chunks_kernel<<<1, 32, 0, s>>>(L, Hv, partials, chunk_id, scores);
+    score_chunks_kernel<<<1, kScoreThreads, 0, s>>>(L, Hv, partials, chunk_id, scores);
     return cudaGetLastError();
 }
 

@@ -1,16 +1,720 @@
-// Tensor-core (tcgen05 / TMEM / TMA) gated-delta-rule chunk update for d = 128, bfloat16.
+// Gated delta rule over one chunk on the Blackwell tensor cores (tcgen05 + TMEM + TMA), d = 128,
+// bfloat16 k/v, fp32 state, with the state-drift partials fused in.
+//
+// Paper: Sec. 3.2, Eq. 1/2 (the recurrence) and Eq. 3 (drift numerator / denominator per layer
+// and head).  The chunk is processed in tiles of C = 64 tokens with the chunkwise (WY) form of
+// Eq. 1: with G the inclusive cumulative log-decay inside the tile, gamma = exp(G),
+//   A[t][i] = beta_t exp(G_t - G_i) k_t.k_i  (i < t),   T = (I + A)^-1 diag(beta),
+//   X = K S0^T,   U = T (V - diag(gamma) X),
+//   S_C = gamma_C S0 + U~^T K,   U~[t] = exp(G_C - G_t) U[t].
+// Padded tokens of a ragged last tile carry k = v = 0, g = 0, beta = 0 and change nothing.
+//
+// One CTA owns one (layer, value head) for the whole chunk.  The state lives in TMEM from the
+// first tile to the last and S_before stays in shared memory, so the state is read from and
+// written to HBM exactly once and the drift needs no second pass over it.
+//
+// Precision: every product that touches the state or T uses a two-term bfloat16 split
+// (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)); keys and values are exact in bfloat16.  With
+// X~ = -diag(gamma) X:
+//   X^T  = S0 K^T                   (S0hi + S0lo) K^T                            2 MMA groups
+//   U^T  = V^T T^T + X~^T T^T        V^T (Thi + Tlo) + X~hi (Thi + Tlo) + X~lo Thi  5 MMA groups
+//   S   += U~^T K                   (U~hi + U~lo) K                              2 MMA groups
+//   K K^T                           exact inputs                                 1 MMA group
+// All products accumulate in fp32 in TMEM; the state error stays ~1e-5 relative to fp64, where
+// one bfloat16 rounding of any of these operands costs ~1e-3.
+//
+// Operand placement: the split state-side operands (S0, X~, U~) are A operands read straight from
+// TMEM (written there by tcgen05.st), so the only operands streamed from shared memory are K, V and
+// T.  Shared-memory bandwidth is the resource the tensor pipe and the CUDA-core warps share, and
+// A tiles of 128 rows re-read for every N = 64 product would otherwise saturate it.
+//
+// Warp roles (17 warps):
+//   0-7   state chain: per tile, S0 -> (hi, lo) split, X~ split, U~ split (TMEM <-> registers)
+//   8-15  T builders: K K^T -> A -> (I + A)^-1 by 16 / 32 / 64 blocks -> T (hi, lo), a tile ahead
+//         of the chain (T depends on k, g, beta only)
+//   16    TMEM allocation, TMA loads and every tcgen05.mma (the warp stays converged; elect.sync
+//         picks the issuing lane)
+// Roles hand work to each other through mbarriers only.  Every wait is bounded; a wait that runs
+// out records DELTAS_ERR_TIMEOUT, raises a CTA-wide abort flag so the other roles stop waiting,
+// and the CTA drains its MMAs and loads before freeing TMEM.
+// TMEM (512 columns, M = 128 lanes = d_v): S [0,128), S0 hi / lo packed [128,192) / [192,256),
+// X [256,320) (fp32, then X~ hi / lo packed in place), U [320,384) (likewise U~), K K^T of even /
+// odd tiles [384,448) / [448,512).
 #include "internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace deltas {
+namespace {
+
+using namespace tc;
+
+constexpr int kC = 64;                 // tokens per tile
+constexpr int kD = 128;                // head dim (d_k = d_v)
+constexpr int kChain = 256;            // warps 0-7
+constexpr int kTB = 256;               // warps 8-15
+constexpr int kThreads = kChain + kTB + 32;
+constexpr int kCtlWarp = 16;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t TM_S = 0, TM_S0HI = 128, TM_S0LO = 192, TM_X = 256, TM_U = 320, TM_KK = 384;  // K K^T: 2 x 64
+
+constexpr int FA_S = 65;               // fp32 row stride of A (odd: one row per lane, no bank conflicts)
+constexpr int FX_S = 68;               // fp32 row stride of X^-1 (16-byte aligned rows for float4 reads)
+
+// shared-memory map (bytes from a 1024-aligned base)
+constexpr uint32_t SM_K = 0;                      // 3 x 16 KB: K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
+constexpr uint32_t SM_V = 49152;                  // 16 KB: V tile, same layout
+constexpr uint32_t SM_T = 65536;                  // 2 buffers x (hi 8 KB, lo 8 KB): T, 64 rows (t) x 64 (i)
+constexpr uint32_t SM_SB = 98304;                 // 64 KB: S_before fp32, column-major [d_k][d_v]
+constexpr uint32_t SM_FA = 163840;                // fp32 [64][FA_S]
+constexpr uint32_t SM_FX = SM_FA + 64 * FA_S * 4; // fp32 [64][FX_S]
+constexpr uint32_t SM_TMP = SM_FX + 64 * FX_S * 4;// fp32 [32][33]
+constexpr uint32_t SM_CG = SM_TMP + 32 * 33 * 4;  // chain tile constants, 3 buffers x (-gamma[64], del[64], gamma_C)
+constexpr uint32_t SM_TG = SM_CG + 3 * 132 * 4;   // T-builder constants: G2[64], beta[64], row[64], col[64], flag
+constexpr uint32_t SM_BYTES = SM_TG + 260 * 4;
+constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
+static_assert(SM_TG % 16 == 0, "beta must be 16-byte aligned");
+static_assert(kSmemAlloc <= 232448, "shared memory budget");
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct TcArgs {
+    int L, Hk, Hv, T, n_tiles;
+    float* state;
+    float* partials;
+    const float* g;
+    const float* beta;
+    int32_t* status;
+};
+
+__device__ __forceinline__ void named_sync(int id, int n) {
+    asm volatile("bar.sync %0, %1;" :: "r"(id), "r"(n) : "memory");
+}
+
+// Barrier over `n` threads that also returns the OR of `flag` over them (uniform result).
+__device__ __forceinline__ bool named_sync_or(int id, int n, bool flag) {
+    uint32_t out;
+    asm volatile("{\n\t.reg .pred p, q;\n\t"
+                 "setp.ne.u32 q, %3, 0;\n\t"
+                 "bar.red.or.pred p, %1, %2, q;\n\t"
+                 "selp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(out) : "r"(id), "r"(n), "r"((uint32_t)flag) : "memory");
+    return out != 0;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// x[0..7] -> hi = bf16(x), lo = bf16(x - hi), 8 packed values each
+__device__ __forceinline__ void split8(const float* x, uint4& hi, uint4& lo) {
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const __nv_bfloat162 hh = __floats2bfloat162_rn(x[2 * i], x[2 * i + 1]);
+        const float2 hf = __bfloat1622float2(hh);
+        h[i] = *reinterpret_cast<const uint32_t*>(&hh);
+        l[i] = pack_bf16x2(x[2 * i] - hf.x, x[2 * i + 1] - hf.y);
+    }
+    hi = make_uint4(h[0], h[1], h[2], h[3]);
+    lo = make_uint4(l[0], l[1], l[2], l[3]);
+}
+
+// (a, b) -> packed bf16 hi = (bf16(a), bf16(b)) and lo = (bf16(a - hi_a), bf16(b - hi_b)),
+// a in the low half (the TMEM A-operand packing: even k low)
+__device__ __forceinline__ void split2(float a, float b, uint32_t& hi, uint32_t& lo) {
+    const __nv_bfloat162 hh = __floats2bfloat162_rn(a, b);
+    const float2 hf = __bfloat1622float2(hh);
+    hi = *reinterpret_cast<const uint32_t*>(&hh);
+    lo = pack_bf16x2(a - hf.x, b - hf.y);
+}
+
+// 2^x with the hardware approximation (relative error about 2^-22)
+__device__ __forceinline__ float fast_exp2(float x) {
+    float y;
+    asm("ex2.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// All lanes of a converged warp wait; the result is the same on every lane (false if any lane's
+// wait ran out), so the warp stays converged for the elect.sync that follows.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
+                                          const volatile int* abort) {
+    const bool ok = mbar_wait_or_abort(bar, parity, budget_ns, abort);
+    return __all_sync(0xffffffffu, ok) != 0;
+}
+
+__device__ __forceinline__ void fail(int32_t* status, volatile int* abort, int where) {
+    record_status(status, DELTAS_ERR_TIMEOUT, where);
+    *abort = 1;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, TcArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    // TMA -> MMA: K buffers, V buffer.  MMA -> roles: kk, x, u, s.  roles -> MMA: ready flags.
+    __shared__ uint64_t mb_tk[3], mb_tv, mb_kk[2], mb_x, mb_u, mb_s, mb_sready, mb_xready, mb_uready, mb_tready, mb_fin;
+    __shared__ uint64_t mb_cready[3];                  // chain tile constants of tile t in buffer t % 3
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_abort;
+    __shared__ double s_red[2][8];
+    volatile int* abort_flag = &s_abort;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int lh = blockIdx.x;
+    const int l = lh / a.Hv, h = lh % a.Hv;
+    const int kh = (int)(((long long)h * a.Hk) / a.Hv);
+    const int n = a.n_tiles;
+
+    if (warp == kCtlWarp) {
+        tmem_alloc(&s_tmem, kTmemCols);
+        tmem_relinquish();
+        if (lane == 0) {
+            mbar_init(&mb_tk[0], 1); mbar_init(&mb_tk[1], 1); mbar_init(&mb_tk[2], 1); mbar_init(&mb_tv, 1);
+            mbar_init(&mb_kk[0], 1); mbar_init(&mb_kk[1], 1);
+            mbar_init(&mb_x, 1); mbar_init(&mb_u, 1); mbar_init(&mb_s, 1);
+            mbar_init(&mb_sready, kChain); mbar_init(&mb_xready, kChain); mbar_init(&mb_uready, kChain);
+            mbar_init(&mb_tready, kTB); mbar_init(&mb_fin, 1);
+            mbar_init(&mb_cready[0], 1); mbar_init(&mb_cready[1], 1); mbar_init(&mb_cready[2], 1);
+            fence_barrier_init();
+            prefetch_tensormap(&kmap);
+            prefetch_tensormap(&vmap);
+        }
+    }
+    if (tid == 0) s_abort = 0;
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = s_tmem;
+
+    if (warp == kCtlWarp) {
+        // =========================================================== TMA + MMA issue (whole warp,
+        // converged; elect.sync picks the issuing lane)
+        {
+            auto load_k = [&](int tile) {              // K tile `tile` -> buffer tile % 3
+                const int b = tile % 3;
+                if (elect_one()) {
+                    uint8_t* dst = sm + SM_K + b * 16384;
+                    mbar_arrive_expect_tx(&mb_tk[b], 16384);
+                    tma_load_4d(dst, &kmap, &mb_tk[b], 0, kh, tile * kC, l);
+                    tma_load_4d(dst + 8192, &kmap, &mb_tk[b], 64, kh, tile * kC, l);
+                }
+                __syncwarp();
+            };
+            auto load_v = [&](int tile) {
+                if (elect_one()) {
+                    mbar_arrive_expect_tx(&mb_tv, 16384);
+                    tma_load_4d(sm + SM_V, &vmap, &mb_tv, 0, h, tile * kC, l);
+                    tma_load_4d(sm + SM_V + 8192, &vmap, &mb_tv, 64, h, tile * kC, l);
+                }
+                __syncwarp();
+            };
+            auto mma_kk = [&](int tile) {
+                // K K^T into the K K^T buffer of the tile's parity.  M = 128: rows 64..127 of A read
+                // the next 8 KB of shared memory (valid, ignored output).
+                const uint8_t* sK = sm + SM_K + (tile % 3) * 16384;
+                const uint32_t id = idesc_bf16(128, 64, 0, 0);
+#pragma unroll
+                for (int s = 0; s < 8; ++s) {
+                    const uint64_t d = sdesc_sw128(smem_u32(sK + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
+                    mma_bf16(tm + TM_KK + 64 * (tile & 1), d, d, id, s > 0);
+                }
+                mma_commit(&mb_kk[tile & 1]);
+            };
+            int kp[3] = {-1, -1, -1};                  // tile whose K load is in flight, per buffer
+            int v_pending = 0;
+            load_k(0); kp[0] = 0;
+            if (n > 1) { load_k(1); kp[1] = 1; }
+            load_v(0);
+            bool ok = warp_wait(&mb_tk[0], 0, kWaitBudgetNs, abort_flag);
+            if (!ok) fail(a.status, abort_flag, 1);
+            if (ok) { kp[0] = -1; mma_kk(0); }
+            for (int j = 0; ok && j < n; ++j) {
+                const uint8_t* sK = sm + SM_K + (j % 3) * 16384;
+                // S0 split of tile j ready (the chain has seen MMA_S(j-1) complete)
+                if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
+                if (j + 2 < n) { load_k(j + 2); kp[(j + 2) % 3] = j + 2; }
+                tc_fence_after();
+                {   // X^T = S0 K^T   (A: S0 hi / lo from TMEM, 8 columns per K = 16 step)
+                    const uint32_t id = idesc_bf16(128, 64, 0, 0);
+#pragma unroll
+                    for (int part = 0; part < 2; ++part) {
+                        const uint32_t a0 = tm + (part == 0 ? TM_S0HI : TM_S0LO);
+#pragma unroll
+                        for (int s = 0; s < 8; ++s) {
+                            const uint64_t bd = sdesc_sw128(smem_u32(sK + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
+                            mma_bf16_ta(tm + TM_X, a0 + 8 * s, bd, id, (part | s) != 0);
+                        }
+                    }
+                    mma_commit(&mb_x);
+                }
+                if (j + 1 < n) {                       // K K^T of the next tile, for the T builders
+                    if (!warp_wait(&mb_tk[(j + 1) % 3], ((j + 1) / 3) & 1, kWaitBudgetNs, abort_flag)) {
+                        fail(a.status, abort_flag, 4); break;
+                    }
+                    kp[(j + 1) % 3] = -1;
+                    mma_kk(j + 1);
+                }
+                if (!warp_wait(&mb_tready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 3); break; }
+                if (!warp_wait(&mb_xready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 5); break; }
+                if (!warp_wait(&mb_tv, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 6); break; }
+                v_pending = -1;
+                tc_fence_after();
+                {   // U^T = V^T T^T + X~^T T^T   (X~ = -diag(gamma) X, hi / lo packed in place in X)
+                    const uint8_t* tb = sm + SM_T + (j & 1) * 16384;
+                    const uint32_t id_v = idesc_bf16(128, 64, 1, 0);      // A = V tile read MN-major
+                    const uint32_t id_x = idesc_bf16(128, 64, 0, 0);      // A = X~ from TMEM
+#pragma unroll
+                    for (int part = 0; part < 5; ++part) {
+                        const uint8_t* sb = tb + ((part == 1 || part == 3) ? 8192 : 0);
+#pragma unroll
+                        for (int s = 0; s < 4; ++s) {
+                            const uint64_t bd = sdesc_sw128(smem_u32(sb + s * 32), 16, 1024);
+                            const uint32_t acc = (part | s) != 0;
+                            if (part < 2) {
+                                mma_bf16(tm + TM_U, sdesc_sw128(smem_u32(sm + SM_V + s * 2048), 8192, 1024), bd, id_v, acc);
+                            } else {
+                                // tokens 16s..16s+15: column block s/2 of the X region, hi then lo
+                                const uint32_t a = tm + TM_X + 32 * (s >> 1) + 8 * (s & 1) + (part == 4 ? 16 : 0);
+                                mma_bf16_ta(tm + TM_U, a, bd, id_x, acc);
+                            }
+                        }
+                    }
+                    mma_commit(&mb_u);
+                }
+                if (!warp_wait(&mb_uready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 7); break; }
+                if (j + 1 < n) { load_v(j + 1); v_pending = j + 1; }
+                tc_fence_after();
+                {   // S += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major: N = d_k)
+                    const uint32_t id = idesc_bf16(128, 128, 0, 1);
+#pragma unroll
+                    for (int part = 0; part < 2; ++part) {
+#pragma unroll
+                        for (int s = 0; s < 4; ++s) {
+                            const uint32_t a = tm + TM_U + 32 * (s >> 1) + 8 * (s & 1) + (part == 1 ? 16 : 0);
+                            const uint64_t bd = sdesc_sw128(smem_u32(sK + s * 2048), 8192, 1024);
+                            mma_bf16_ta(tm + TM_S, a, bd, id, 1);
+                        }
+                    }
+                    mma_commit(&mb_s);
+                }
+            }
+            if (__any_sync(0xffffffffu, *abort_flag != 0)) {
+                // drain: every MMA this warp issued, and every load still in flight
+                mma_commit(&mb_fin);
+                mbar_wait(&mb_fin, 0, kWaitBudgetNs);
+                for (int b = 0; b < 3; ++b)
+                    if (kp[b] >= 0) mbar_wait(&mb_tk[b], (kp[b] / 3) & 1, kWaitBudgetNs);
+                if (v_pending >= 0) mbar_wait(&mb_tv, v_pending & 1, kWaitBudgetNs);
+            }
+        }
+        __syncwarp();
+    } else if (warp >= 8) {
+        // =========================================================== T builders (warps 8-15)
+        const int tw = warp - 8, tt = tid - kChain;        // tw in [0, 8), tt in [0, 256)
+        float* fA = reinterpret_cast<float*>(sm + SM_FA);
+        float* fX = reinterpret_cast<float*>(sm + SM_FX);
+        float* fT = reinterpret_cast<float*>(sm + SM_TMP);
+        float* sG2 = reinterpret_cast<float*>(sm + SM_TG);   // G * log2(e)
+        float* sBeta = sG2 + 64;
+        float* sRow = sG2 + 128;                             // beta_t 2^(G2_t - ref)
+        float* sCol = sG2 + 192;                             // 2^(ref - G2_i)
+        int* sFactored = reinterpret_cast<int*>(sG2 + 256);
+        float* cg = reinterpret_cast<float*>(sm + SM_CG);
+        float pg[2] = {0.f, 0.f}, pb[2] = {0.f, 0.f};     // g, beta of the next tile (warp 8)
+        if (tw == 0) {
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int t = 2 * lane + e;
+                const size_t gi = ((size_t)l * a.T + t) * a.Hv + h;
+                pg[e] = t < a.T ? a.g[gi] : 0.f;
+                pb[e] = t < a.T ? a.beta[gi] : 0.f;
+            }
+        }
+        for (int j = 0; j < n; ++j) {
+            if (named_sync_or(3, kTB, *abort_flag)) break;
+            if (tw == 0) {                                 // per-tile decay constants
+                float gv[2], bv[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) { gv[e] = pg[e]; bv[e] = pb[e]; }
+                if (j + 1 < n) {                           // prefetch the next tile's g, beta
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int t = (j + 1) * kC + 2 * lane + e;
+                        const size_t gi = ((size_t)l * a.T + t) * a.Hv + h;
+                        pg[e] = t < a.T ? a.g[gi] : 0.f;
+                        pb[e] = t < a.T ? a.beta[gi] : 0.f;
+                    }
+                }
+                float incl = gv[0] + gv[1];
+#pragma unroll
+                for (int m = 1; m < 32; m <<= 1) {
+                    const float y = __shfl_up_sync(0xffffffffu, incl, m);
+                    if (lane >= m) incl += y;
+                }
+                const float G0 = incl - gv[1], G1 = incl;
+                const float GC = __shfl_sync(0xffffffffu, incl, 31);
+                // the chain's constants of tile j: -gamma, exp(G_C - G), gamma_C (3 buffers: the
+                // chain is at most two tiles behind)
+                float* cgam = cg + (j % 3) * 132;
+                cgam[2 * lane] = -expf(G0); cgam[2 * lane + 1] = -expf(G1);
+                cgam[64 + 2 * lane] = expf(GC - G0); cgam[64 + 2 * lane + 1] = expf(GC - G1);
+                if (lane == 0) cgam[128] = expf(GC);
+                const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
+                float lo2 = fminf(g20, g21), hi2 = fmaxf(g20, g21);
+#pragma unroll
+                for (int m = 16; m >= 1; m >>= 1) {
+                    lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, m));
+                    hi2 = fmaxf(hi2, __shfl_xor_sync(0xffffffffu, hi2, m));
+                }
+                // exp(G_t - G_i) = row_t * col_i with the reference in the middle of the tile's
+                // range of G; both factors stay within 2^+-126 when that range spans at most 250
+                // powers of two, otherwise the exponent is taken per entry.
+                const float ref = 0.5f * (lo2 + hi2);
+                sG2[2 * lane] = g20; sG2[2 * lane + 1] = g21;
+                sBeta[2 * lane] = bv[0]; sBeta[2 * lane + 1] = bv[1];
+                sRow[2 * lane] = bv[0] * fast_exp2(g20 - ref); sRow[2 * lane + 1] = bv[1] * fast_exp2(g21 - ref);
+                sCol[2 * lane] = fast_exp2(ref - g20); sCol[2 * lane + 1] = fast_exp2(ref - g21);
+                if (lane == 0) *sFactored = (hi2 - lo2) <= 250.f;
+                fence_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&mb_cready[j % 3]);
+            }
+            named_sync(3, kTB);
+            if (!mbar_wait_or_abort(&mb_kk[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 8);
+            tc_fence_after();
+            const int q = warp & 3;
+            if (q < 2) {
+                // TMEM lanes 0..63 hold K K^T: warps 8/12 rows 0..31, 9/13 rows 32..63; column half
+                // (tw >> 2).  All shared-memory reads are made before the first store (the tile
+                // constants and A share one buffer).
+                const int t = 32 * q + lane, c0 = 32 * (tw >> 2);
+                const uint32_t lane_off = (uint32_t)(32 * q) << 16;
+                float kk[32], cf[32];
+                tmem_ld32(tm + lane_off + TM_KK + 64 * (j & 1) + c0, kk);
+                if (*sFactored) {
+                    const float rt = sRow[t];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float4 v4 = *reinterpret_cast<const float4*>(sCol + c0 + 4 * e);
+                        cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
+                    }
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? rt * cf[e] * kk[e] : 0.f;
+                } else {
+                    const float G2t = sG2[t], bt = sBeta[t];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float4 v4 = *reinterpret_cast<const float4*>(sG2 + c0 + 4 * e);
+                        cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
+                    }
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? bt * fast_exp2(G2t - cf[e]) * kk[e] : 0.f;
+                }
+#pragma unroll
+                for (int e = 0; e < 32; ++e) fA[t * FA_S + c0 + e] = kk[e];
+            }
+            tc_fence_before();
+            named_sync(3, kTB);
+            // level 0: four 16 x 16 diagonal blocks of (I + A)^-1, one column per thread
+            if (tt < 64) {
+                const int B = tt >> 4, jc = tt & 15, o = 16 * B;
+                float x[16];
+#pragma unroll
+                for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
+#pragma unroll
+                for (int rr = 1; rr < 16; ++rr) {
+                    float sacc = 0.f;
+#pragma unroll
+                    for (int c = 0; c < rr; ++c) sacc = fmaf(fA[(o + rr) * FA_S + o + c], x[c], sacc);
+                    if (rr > jc) x[rr] = -sacc;
+                }
+#pragma unroll
+                for (int rr = 0; rr < 16; ++rr) fX[(o + rr) * FX_S + o + jc] = x[rr];
+            }
+            named_sync(3, kTB);
+            // level 1: X[2p+1][2p] = -X[2p+1][2p+1] (A[2p+1][2p] X[2p][2p]), p = tw >> 2.
+            // Loop bounds follow the zero pattern of the triangular factors and are warp-uniform.
+            {
+                const int p = tw >> 2, cg = 4 * (tw & 3);
+                const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
+                const int lo16 = lane & 15, sub = 2 * (lane >> 4);
+                float acc0 = 0.f, acc1 = 0.f;             // tmp1[p][lo16][cg + sub + {0,1}]
+                for (int k = cg; k < 16; ++k) {
+                    const float av = fA[(ro + lo16) * FA_S + co + k];
+                    const float2 xv = *reinterpret_cast<const float2*>(fX + (co + k) * FX_S + co + cg + sub);
+                    acc0 = fmaf(av, xv.x, acc0);
+                    acc1 = fmaf(av, xv.y, acc1);
+                }
+                fT[p * 272 + lo16 * 17 + cg + sub] = acc0;
+                fT[p * 272 + lo16 * 17 + cg + sub + 1] = acc1;
+                named_sync(3, kTB);
+                float o0 = 0.f, o1 = 0.f;                  // rows cg + sub + {0,1}, column lo16
+                for (int k = 0; k <= cg + 3; ++k) {
+                    const float tv = fT[p * 272 + k * 17 + lo16];
+                    o0 = fmaf(fX[(ro + cg + sub) * FX_S + ro + k], tv, o0);
+                    o1 = fmaf(fX[(ro + cg + sub + 1) * FX_S + ro + k], tv, o1);
+                }
+                fX[(ro + cg + sub) * FX_S + co + lo16] = -o0;
+                fX[(ro + cg + sub + 1) * FX_S + co + lo16] = -o1;
+            }
+            named_sync(3, kTB);
+            // level 2: X[32:64][0:32] = -X[32:64][32:64] (A[32:64][0:32] X[0:32][0:32])
+            {
+                const int g4 = 4 * tw;
+                float acc[4] = {0.f, 0.f, 0.f, 0.f};       // tmp2[lane][g4..g4+3]
+                for (int k = g4; k < 32; ++k) {
+                    const float av = fA[(32 + lane) * FA_S + k];
+                    const float4 xv = *reinterpret_cast<const float4*>(fX + k * FX_S + g4);
+                    acc[0] = fmaf(av, xv.x, acc[0]); acc[1] = fmaf(av, xv.y, acc[1]);
+                    acc[2] = fmaf(av, xv.z, acc[2]); acc[3] = fmaf(av, xv.w, acc[3]);
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) fT[lane * 33 + g4 + i] = acc[i];
+                named_sync(3, kTB);
+                float o4[4] = {0.f, 0.f, 0.f, 0.f};        // rows 32+g4..32+g4+3, column lane
+                for (int k = 0; k <= g4 + 3; k += 4) {
+                    const float t0v = fT[(k + 0) * 33 + lane], t1v = fT[(k + 1) * 33 + lane];
+                    const float t2v = fT[(k + 2) * 33 + lane], t3v = fT[(k + 3) * 33 + lane];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float4 xr = *reinterpret_cast<const float4*>(fX + (32 + g4 + i) * FX_S + 32 + k);
+                        o4[i] = fmaf(xr.x, t0v, o4[i]); o4[i] = fmaf(xr.y, t1v, o4[i]);
+                        o4[i] = fmaf(xr.z, t2v, o4[i]); o4[i] = fmaf(xr.w, t3v, o4[i]);
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) fX[(32 + g4 + i) * FX_S + lane] = -o4[i];
+            }
+            named_sync(3, kTB);
+            // T = X diag(beta) (upper part zero), split into the B operand buffer of tile j
+            {
+                uint8_t* tb = sm + SM_T + (j & 1) * 16384;
+                uint4 vh[2], vl[2];
+                int tr[2], cr[2];
+#pragma unroll
+                for (int m = 0; m < 2; ++m) {
+                    const int e = tt + kTB * m;
+                    const int t = e >> 3, c8 = e & 7;
+                    const float4 x0 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8);
+                    const float4 x1 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8 + 4);
+                    const float4 b0 = *reinterpret_cast<const float4*>(sBeta + 8 * c8);
+                    const float4 b1 = *reinterpret_cast<const float4*>(sBeta + 8 * c8 + 4);
+                    const float xs[8] = {x0.x * b0.x, x0.y * b0.y, x0.z * b0.z, x0.w * b0.w,
+                                         x1.x * b1.x, x1.y * b1.y, x1.z * b1.z, x1.w * b1.w};
+                    float x[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) x[k] = (8 * c8 + k <= t) ? xs[k] : 0.f;
+                    split8(x, vh[m], vl[m]);
+                    tr[m] = t; cr[m] = c8;
+                }
+#pragma unroll
+                for (int m = 0; m < 2; ++m) {
+                    *reinterpret_cast<uint4*>(tb + sw128_offset(tr[m], cr[m])) = vh[m];
+                    *reinterpret_cast<uint4*>(tb + 8192 + sw128_offset(tr[m], cr[m])) = vl[m];
+                }
+            }
+            fence_async_smem();
+            mbar_arrive(&mb_tready);
+        }
+    } else {
+        // =========================================================== state chain (warps 0-7)
+        const int q = warp & 3, wg = warp >> 2;
+        const int r = 32 * q + lane;                       // row of S (value index)
+        const uint32_t lane_off = (uint32_t)(32 * q) << 16;
+        const uint32_t cS = TM_S + 64 * wg;                // this thread's 64 state columns
+        float* sbefore = reinterpret_cast<float*>(sm + SM_SB);   // [d_k][d_v]: column c at c * 128
+        float* cg = reinterpret_cast<float*>(sm + SM_CG);
+        float den = 0.f;
+        bool done = false;
+        for (int j = 0; j < n; ++j) {
+            float* gam = cg + (j % 3) * 132;               // -gamma (written by the T builders)
+            float* del = gam + 64;                         // exp(G_C - G)
+            if (named_sync_or(2, kChain, *abort_flag)) break;
+            if (!mbar_wait_or_abort(&mb_cready[j % 3], (j / 3) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
+            const float gC = gam[128];
+
+            // ---- S pass: S0 -> (hi, lo) packed into TMEM; gamma_C S0 -> TMEM (32 columns at a time)
+            if (j > 0) {
+                if (!mbar_wait_or_abort(&mb_s, (j - 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 9);
+                tc_fence_after();
+            }
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                float sv[32];
+                if (j == 0) {
+                    const float4* src = reinterpret_cast<const float4*>(a.state + ((size_t)lh * kD + r) * kD + 64 * wg + 32 * half);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float4 x = src[e];
+                        sv[4 * e] = x.x; sv[4 * e + 1] = x.y; sv[4 * e + 2] = x.z; sv[4 * e + 3] = x.w;
+                    }
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        den += sv[e] * sv[e];
+                        sbefore[(64 * wg + 32 * half + e) * kD + r] = sv[e];
+                    }
+                } else {
+                    tmem_ld32(tm + lane_off + cS + 32 * half, sv);
+                    tmem_ld_wait();
+                }
+                uint32_t hi[16], lo[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c) split2(sv[2 * c], sv[2 * c + 1], hi[c], lo[c]);
+                tmem_st16(tm + lane_off + TM_S0HI + 32 * wg + 16 * half, hi);
+                tmem_st16(tm + lane_off + TM_S0LO + 32 * wg + 16 * half, lo);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) sv[e] *= gC;
+                tmem_st32(tm + lane_off + cS + 32 * half, sv);
+            }
+            tmem_st_wait();
+            tc_fence_before();
+            mbar_arrive(&mb_sready);
+
+            // ---- X~^T = -X^T diag(gamma): (hi, lo) packed in place over this thread's 32 X columns
+            if (!mbar_wait_or_abort(&mb_x, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 10);
+            tc_fence_after();
+            {
+                float xv[32];
+                tmem_ld32(tm + lane_off + TM_X + 32 * wg, xv);
+                tmem_ld_wait();
+                uint32_t hi[16], lo[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c)
+                    split2(gam[32 * wg + 2 * c] * xv[2 * c], gam[32 * wg + 2 * c + 1] * xv[2 * c + 1], hi[c], lo[c]);
+                tmem_st16(tm + lane_off + TM_X + 32 * wg, hi);
+                tmem_st16(tm + lane_off + TM_X + 32 * wg + 16, lo);
+                tmem_st_wait();
+            }
+            tc_fence_before();
+            mbar_arrive(&mb_xready);
+
+            // ---- U~^T = U^T diag(exp(G_C - G)): (hi, lo) packed in place over the U columns
+            if (!mbar_wait_or_abort(&mb_u, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 11);
+            tc_fence_after();
+            {
+                float uv[32];
+                tmem_ld32(tm + lane_off + TM_U + 32 * wg, uv);
+                tmem_ld_wait();
+                uint32_t hi[16], lo[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c)
+                    split2(uv[2 * c] * del[32 * wg + 2 * c], uv[2 * c + 1] * del[32 * wg + 2 * c + 1], hi[c], lo[c]);
+                tmem_st16(tm + lane_off + TM_U + 32 * wg, hi);
+                tmem_st16(tm + lane_off + TM_U + 32 * wg + 16, lo);
+                tmem_st_wait();
+            }
+            tc_fence_before();
+            mbar_arrive(&mb_uready);
+            done = (j == n - 1);
+        }
+
+        // ---- epilogue: S_after -> HBM, drift partials against S_before
+        bool ok = done && mbar_wait_or_abort(&mb_s, (n - 1) & 1, kWaitBudgetNs, abort_flag);
+        if (done && !ok) fail(a.status, abort_flag, 12);
+        tc_fence_after();
+        float num = 0.f;
+        if (ok) {
+            float4* dst = reinterpret_cast<float4*>(a.state + ((size_t)lh * kD + r) * kD + 64 * wg);
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                float sv[32];
+                tmem_ld32(tm + lane_off + cS + 32 * half, sv);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    const float dlt = sv[e] - sbefore[(64 * wg + 32 * half + e) * kD + r];
+                    num += dlt * dlt;
+                }
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    dst[8 * half + e] = make_float4(sv[4 * e], sv[4 * e + 1], sv[4 * e + 2], sv[4 * e + 3]);
+            }
+        }
+        double dn = num, dd = den;
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) {
+            dn += __shfl_xor_sync(0xffffffffu, dn, m);
+            dd += __shfl_xor_sync(0xffffffffu, dd, m);
+        }
+        if (lane == 0) { s_red[0][warp] = dn; s_red[1][warp] = dd; }
+        const bool any_fail = named_sync_or(2, kChain, !ok);
+        if (tid == 0 && !any_fail && a.partials != nullptr) {
+            double sn = 0.0, sd = 0.0;
+            for (int w = 0; w < 8; ++w) { sn += s_red[0][w]; sd += s_red[1][w]; }
+            a.partials[(size_t)lh * 2 + 0] = (float)sn;
+            a.partials[(size_t)lh * 2 + 1] = (float)sd;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kCtlWarp) {
+        tc_fence_after();
+        tmem_dealloc(tm, kTmemCols);
+    }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        cudaDriverEntryPointQueryResult q;
+        void* p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// [L][T][H][128] bfloat16 as a 4-D map (d, H, T, L): a box of 64 features x 1 head x 64 tokens,
+// 128-byte swizzle; tokens past T read as zero.
+bool make_map(CUtensorMap* map, const void* base, int L, int T, int H) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[4] = {(cuuint64_t)kD, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)L};
+    cuuint64_t strides[3] = {(cuuint64_t)kD * 2, (cuuint64_t)H * kD * 2, (cuuint64_t)T * H * kD * 2};
+    cuuint32_t box[4] = {64, 1, (cuuint32_t)kC, 1};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
 
 bool gdn_tc_supported(const GdnArgs& a) {
-    (void)a;
-    return false;
+    return a.dk == kD && a.dv == kD && a.dtype == DELTAS_BF16 && a.out == nullptr && a.T > 0 &&
+           encode_fn() != nullptr;
 }
 
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
-    (void)a; (void)s;
-    return cudaErrorNotSupported;
+    CUtensorMap kmap, vmap;
+    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv)) return cudaErrorInvalidValue;
+    static int configured_device = -1;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (configured_device != dev) {
+        cudaError_t e = cudaFuncSetAttribute(gdn_update_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kSmemAlloc);
+        if (e != cudaSuccess) return e;
+        configured_device = dev;
+    }
+    TcArgs t;
+    t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = (a.T + kC - 1) / kC;
+    t.state = a.state; t.partials = a.partials; t.g = a.g; t.beta = a.beta; t.status = a.status;
+    gdn_update_tc_kernel<<<a.L * a.Hv, kThreads, kSmemAlloc, s>>>(kmap, vmap, t);
+    return cudaGetLastError();
 }
 
 }  // namespace deltas

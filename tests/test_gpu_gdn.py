@@ -76,14 +76,16 @@ def _check_chunk(L, x, state0, want_out, dtype, q_scale):
 
 @pytest.mark.parametrize("d", [16, 32, 64, 128])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("T", [1, 100, 257])
-def test_gdn_update_shapes(L, d, dtype, T):
-    """Every head size, both activation dtypes, ragged token counts, grouped keys (Hk=2, Hv=4),
-    two layers, with read-out and drift partials."""
+@pytest.mark.parametrize("T", [1, 63, 64, 100, 257])
+@pytest.mark.parametrize("want_out", [True, False])
+def test_gdn_update_shapes(L, d, dtype, T, want_out):
+    """Every head size, both activation dtypes, ragged token counts (one token, a tile minus one,
+    exactly one tile, several tiles with a ragged tail), grouped keys (Hk=2, Hv=4), two layers,
+    with and without the read-out (d = 128 bf16 without read-out runs on the tensor cores)."""
     tdt = torch.float32 if dtype == "f32" else torch.bfloat16
     x = inputs.gdn_chunk(2, T, 2, 4, d, dtype, inputs.seed_for(1, d, T))
     s0 = inputs.initial_state(2, 4, d, inputs.seed_for(2, d, T))
-    _check_chunk(L, x, s0, True, tdt, d ** -0.5)
+    _check_chunk(L, x, s0, want_out, tdt, d ** -0.5)
 
 
 def test_gdn_update_tiny_stream_from_zero(L):
@@ -112,12 +114,37 @@ def test_gdn_update_zero_tokens(L):
     np.testing.assert_allclose(p[..., 1], np.sum(s0.double().numpy() ** 2, axis=(2, 3)), rtol=1e-5)
 
 
-def test_gdn_update_layer_width_chunk(L):
+@pytest.mark.parametrize("want_out", [True, False])
+def test_gdn_update_layer_width_chunk(L, want_out):
     """The single-layer workload's shape: 16 key heads, 32 value heads, d = 128, bf16, one chunk
-    of 1024 tokens (spans many tiles), with read-out."""
+    of 1024 tokens (spans many tiles), with and without read-out."""
     x = inputs.gdn_chunk(1, 1024, 16, 32, 128, "bf16", inputs.seed_for(7, 1, 0))
     s0 = inputs.initial_state(1, 32, 128, 8)
-    _check_chunk(L, x, s0, True, torch.bfloat16, 128 ** -0.5)
+    _check_chunk(L, x, s0, want_out, torch.bfloat16, 128 ** -0.5)
+
+
+def test_gdn_update_stack_width_sampled(L):
+    """The full stack's width (24 layers x 32 value heads, d = 128, bf16, one 1024-token chunk)
+    in the launch configuration the benchmark times; the oracle checks a sample of 12 (layer,
+    head) pairs, each replayed from the same S_before."""
+    Lg, Hk, Hv, d, T = 24, 16, 32, 128, 1024
+    x = inputs.gdn_chunk(Lg, T, Hk, Hv, d, "bf16", inputs.seed_for(8, 2, 0))
+    s0 = inputs.initial_state(Lg, Hv, d, 10)
+    st, _, part = _run_gpu(L, x, s0, False, torch.bfloat16, None)
+    rng = np.random.default_rng(3)
+    pairs = [(0, 0), (Lg - 1, Hv - 1)] + [(int(rng.integers(Lg)), int(rng.integers(Hv))) for _ in range(10)]
+    for (l, h) in pairs:
+        kh = h * Hk // Hv
+        sub = {k: x[k][l:l + 1] for k in ("k", "v", "g", "beta")}
+        S_ref, _ = oracle.gdn_recurrence(None, _f64(sub["k"][:, :, kh:kh + 1]), _f64(sub["v"][:, :, h:h + 1]),
+                                         _f64(sub["g"][:, :, h:h + 1]), _f64(sub["beta"][:, :, h:h + 1]),
+                                         _f64(s0[l:l + 1, h:h + 1]))
+        rel = _per_head_rel(_f64(st[l:l + 1, h:h + 1]), S_ref).max()
+        assert rel <= STATE_TOL, (l, h, rel)
+        p_ref = oracle.drift_partials(_f64(s0[l:l + 1, h:h + 1]), S_ref)[0, 0]
+        np.testing.assert_allclose(_f64(part[l, h]), p_ref, rtol=1e-3)
+    # every head moved and no head was left untouched or non-finite
+    assert torch.isfinite(st).all() and (part[..., 0] > 0).all()
 
 
 def test_gdn_update_slow_decay_four_chunks(L):
