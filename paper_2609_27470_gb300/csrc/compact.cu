@@ -6,13 +6,16 @@
 // retain_idx[j] >= j, the only hazard is a destination row that is still to be read as the
 // source of an earlier destination.  The work is cut into units (plane p, tile b of TB
 // destination rows); a unit
-//   1. stages the source rows of its tile in shared memory (16-byte loads),
+//   1. stages the source rows of its tile in shared memory (16-byte cp.async loads),
 //   2. publishes "tile b of plane p has been read" (release flag),
 //   3. waits until every earlier tile whose destinations read rows of tile b has published
-//      (the first such tile, need[b], comes from a prepass over retain_idx),
+//      (the first such tile, need[b], comes from a prepass over retain_idx; one warp checks up to
+//      32 flags at once),
 //   4. writes its tile (16-byte stores; the destination rows of a tile are contiguous).
-// Units are claimed through an atomic ticket in tile-major order, so a unit only waits for units
-// that were claimed earlier by running CTAs and that never wait before publishing: no deadlock.
+// A unit publishes as soon as its own loads have landed, never after a wait, so no wait chains
+// form across tiles.  Units are claimed through an atomic ticket in tile-major order, so a unit
+// only waits for units that were claimed earlier by running CTAs whose loads complete without
+// waiting on anything: no deadlock.
 // Every wait is bounded (about one second); a wait that runs out records DELTAS_ERR_TIMEOUT,
 // raises the abort flag and skips its writes.  Traffic is the algorithmic minimum: each moved row
 // is read once and written once; rows that do not move are not touched.
@@ -22,7 +25,7 @@ namespace deltas {
 namespace {
 
 constexpr int kCompactThreads = 256;
-constexpr int kStageBytes = 32768;
+constexpr int kStageBytes = 32768;   // staged source rows of one unit
 
 struct CompactCtl {
     unsigned ticket;
@@ -92,6 +95,8 @@ __global__ void compact_need_kernel(CompactArgs a) {
     }
 }
 
+__device__ __forceinline__ bool warp_id_is_zero() { return (threadIdx.x >> 5) == 0; }
+
 __device__ __forceinline__ int load_acquire(const int32_t* p) {
     int v;
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -102,93 +107,118 @@ __device__ __forceinline__ void store_release(int32_t* p, int v) {
     asm volatile("st.release.gpu.global.b32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
 }
 
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;"
+                 :: "r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;"
+                 :: "r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+// Issues the asynchronous loads of one unit's moved source rows into a stage buffer.
+__device__ __forceinline__ void compact_issue_loads(const CompactArgs& a, int u, int n, uint8_t* stage) {
+    const int b = u / a.n_planes, p = u % a.n_planes;
+    int rb;
+    const char* base = plane_base(a, p, rb);
+    const int j0 = b * a.tile_rows;
+    const int rows = min(a.tile_rows, n - j0);
+    if (rb >= 16) {
+        const int vpr = rb >> 4;
+        const int nv = rows * vpr;
+        for (int e = threadIdx.x; e < nv; e += kCompactThreads) {
+            const int r = e / vpr, c = e - r * vpr;
+            const int src = a.retain_idx[j0 + r];
+            if (src != j0 + r) cp_async16(stage + 16 * e, base + (size_t)src * rb + 16 * c);
+        }
+    } else {
+        for (int r = threadIdx.x; r < rows; r += kCompactThreads) {
+            const int src = a.retain_idx[j0 + r];
+            if (src != j0 + r) cp_async4(stage + 4 * r, base + (size_t)src * 4);
+        }
+    }
+}
+
+// One unit at a time per CTA (several CTAs per SM keep the memory system busy): claim, load the
+// moved source rows, publish, wait for the earlier readers of this tile, store.  A CTA never holds
+// a claimed unit that it has not loaded and published while it waits on another one.
 __global__ void __launch_bounds__(kCompactThreads)
 compact_main_kernel(CompactArgs a)
 {
-    extern __shared__ uint4 stage[];
-    __shared__ int s_unit;
+    extern __shared__ uint4 stage_raw[];
+    uint8_t* stage = reinterpret_cast<uint8_t*>(stage_raw);
+    __shared__ int s_unit[2];
     __shared__ int s_ok;
-    __shared__ int s_src[1024];
 
     volatile int* abort_flag = &a.ctl->abort;
     if (*abort_flag) return;
     const int n = *a.n_retained;
     const int n_tiles = (n + a.tile_rows - 1) / a.tile_rows;
     const int units = n_tiles * a.n_planes;
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31;
 
     for (;;) {
-        if (tid == 0) s_unit = (*abort_flag) ? units : (int)atomicAdd(&a.ctl->ticket, 1u);
+        if (tid == 0) s_unit[0] = (*abort_flag) ? units : (int)atomicAdd(&a.ctl->ticket, 1u);
         __syncthreads();
-        const int u = s_unit;
-        if (u >= units) break;
-        const int b = u / a.n_planes, p = u % a.n_planes;
-        int rb;
-        char* base = plane_base(a, p, rb);
-        const int j0 = b * a.tile_rows;
-        const int rows = min(a.tile_rows, n - j0);
-        for (int r = tid; r < rows; r += kCompactThreads) s_src[r] = a.retain_idx[j0 + r];
+        const int cur = s_unit[0];
+        if (cur >= units) break;
+        compact_issue_loads(a, cur, n, stage);
+        cp_async_commit();
+        cp_async_wait_0();
         __syncthreads();
-
-        // 1. stage the source rows of moved destinations
-        if (rb >= 16) {
-            const int vpr = rb >> 4;                       // 16-byte vectors per row
-            const int nv = rows * vpr;
-            for (int e = tid; e < nv; e += kCompactThreads) {
-                const int r = e / vpr, c = e - r * vpr;
-                const int src = s_src[r];
-                if (src != j0 + r)
-                    stage[e] = __ldcs(reinterpret_cast<const uint4*>(base + (size_t)src * rb) + c);
+        const int b = cur / a.n_planes, p = cur % a.n_planes;
+        if (warp_id_is_zero()) {
+            // publish, then wait (warp-parallel) for the earlier tiles that read this tile's rows
+            if (lane == 0) {
+                __threadfence();
+                store_release(a.flags + (size_t)p * a.max_tiles + b, 1);
             }
-        } else {
-            int* st = reinterpret_cast<int*>(stage);
-            for (int r = tid; r < rows; r += kCompactThreads) {
-                const int src = s_src[r];
-                if (src != j0 + r) st[r] = reinterpret_cast<const int*>(base)[src];
-            }
-        }
-        __syncthreads();
-
-        // 2. publish, 3. wait for the earlier readers of this tile
-        if (tid == 0) {
-            __threadfence();
-            store_release(a.flags + (size_t)p * a.max_tiles + b, 1);
+            const int first = a.need[b];
             int ok = 1;
             const uint64_t t_start = global_ns();
-            for (int bb = a.need[b]; bb < b && ok; ++bb) {
-                const int32_t* f = a.flags + (size_t)p * a.max_tiles + bb;
-                while (load_acquire(f) == 0) {
-                    if (*abort_flag || global_ns() - t_start > kWaitBudgetNs) {
-                        ok = 0;
-                        break;
-                    }
-                    __nanosleep(64);
+            for (int bb = first; bb < b && ok; bb += 32) {
+                const int mine = bb + lane;
+                const int32_t* f = a.flags + (size_t)p * a.max_tiles + mine;
+                for (;;) {
+                    const bool ready = (mine >= b) || load_acquire(f) != 0;
+                    if (__all_sync(0xffffffffu, ready)) break;
+                    if (*abort_flag || global_ns() - t_start > kWaitBudgetNs) { ok = 0; break; }
+                    __nanosleep(32);
                 }
             }
-            if (!ok) {
-                atomicExch(&a.ctl->abort, 1);
-                record_status(a.status, DELTAS_ERR_TIMEOUT, u);
+            if (lane == 0) {
+                if (!ok) {
+                    atomicExch(&a.ctl->abort, 1);
+                    record_status(a.status, DELTAS_ERR_TIMEOUT, cur);
+                }
+                s_ok = ok;
             }
-            s_ok = ok;
         }
         __syncthreads();
         if (!s_ok) break;
-
-        // 4. write the tile
-        if (rb >= 16) {
-            const int vpr = rb >> 4;
-            const int nv = rows * vpr;
-            uint4* dst = reinterpret_cast<uint4*>(base + (size_t)j0 * rb);
-            for (int e = tid; e < nv; e += kCompactThreads) {
-                const int r = e / vpr;
-                if (s_src[r] != j0 + r) __stcs(dst + e, stage[e]);
+        {   // write the tile (destination rows of a tile are contiguous)
+            int rb;
+            char* base = plane_base(a, p, rb);
+            const int j0 = b * a.tile_rows;
+            const int rows = min(a.tile_rows, n - j0);
+            if (rb >= 16) {
+                const int vpr = rb >> 4;
+                const int nv = rows * vpr;
+                uint4* dst = reinterpret_cast<uint4*>(base + (size_t)j0 * rb);
+                for (int e = tid; e < nv; e += kCompactThreads) {
+                    const int r = e / vpr;
+                    if (a.retain_idx[j0 + r] != j0 + r) __stcs(dst + e, reinterpret_cast<const uint4*>(stage)[e]);
+                }
+            } else {
+                for (int r = tid; r < rows; r += kCompactThreads)
+                    if (a.retain_idx[j0 + r] != j0 + r)
+                        reinterpret_cast<int*>(base)[j0 + r] = reinterpret_cast<const int*>(stage)[r];
             }
-        } else {
-            const int* st = reinterpret_cast<const int*>(stage);
-            for (int r = tid; r < rows; r += kCompactThreads)
-                if (s_src[r] != j0 + r) reinterpret_cast<int*>(base)[j0 + r] = st[r];
         }
-        __syncthreads();
+        __syncthreads();                       // the stage is rewritten by the next unit
     }
 }
 

@@ -155,6 +155,19 @@ struct SelArgs {
     SelWs ws;
 };
 
+constexpr int kSmallRuns = 512;   // runs held in shared memory and ranked directly
+
+// Slot segments: warp w owns whole 32-slot groups [seg_lo, seg_hi) of the candidate range, so
+// every load of tok_chunk is one coalesced 128-byte line.  Returns the run-start flag of slot
+// i = base + lane (false outside the segment).
+__device__ __forceinline__ bool run_start_flag(const int32_t* tok_chunk, int lo, int seg_hi, int i, int& c) {
+    const bool valid = i < seg_hi;
+    c = valid ? tok_chunk[i] : INT_MIN;
+    int prev = __shfl_up_sync(0xffffffffu, c, 1);
+    if ((threadIdx.x & 31) == 0) prev = (valid && i > lo) ? tok_chunk[i - 1] : INT_MIN;
+    return valid && (i == lo || c != prev);
+}
+
 __global__ void __launch_bounds__(kSelThreads, 1)
 select_retain_kernel(SelArgs a)
 {
@@ -169,8 +182,11 @@ select_retain_kernel(SelArgs a)
     __shared__ unsigned s_hist[kMaxSpans * 256];
     __shared__ int s_fill_mode[1], s_fill_target[1];
     __shared__ uint64_t s_fill_prefix[1];
+    __shared__ uint64_t s_rkey[kSmallRuns];
+    __shared__ int s_rstart[kSmallRuns], s_rlen[kSmallRuns], s_rspan[kSmallRuns], s_rkept[kSmallRuns],
+        s_roff[kSmallRuns];
 
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int T = a.T;
     if (tid == 0) s_bad = -1;
     __syncthreads();
@@ -197,52 +213,72 @@ select_retain_kernel(SelArgs a)
     const int n_cand = hi - lo;
     const int R = a.M - a.n_s - a.n_w;
     const int quota = R / N;
+    const unsigned lt_mask = (1u << lane) - 1u;
 
-    // ---- A. runs over the candidate slots
-    const int items = (n_cand + kSelThreads - 1) / kSelThreads;
-    const int seg_lo = min(lo + tid * items, hi), seg_hi = min(seg_lo + items, hi);
+    // ---- A. runs over the candidate slots (warp segments of whole 32-slot groups)
+    const int per_warp = ((n_cand + kSelThreads - 1) / kSelThreads) * 32;
+    const int seg_lo = min(lo + warp * per_warp, hi), seg_hi = min(seg_lo + per_warp, hi);
     int n_starts = 0, cmin = INT_MAX, cmax = INT_MIN;
-    for (int i = seg_lo; i < seg_hi; ++i) {
-        const int c = a.tok_chunk[i];
-        n_starts += (i == lo || c != a.tok_chunk[i - 1]);
-        cmin = min(cmin, c);
-        cmax = max(cmax, c);
+    for (int base = seg_lo; base < seg_hi; base += 32) {
+        int c;
+        const bool st = run_start_flag(a.tok_chunk, lo, seg_hi, base + lane, c);
+        n_starts += __popc(__ballot_sync(0xffffffffu, st));
+        if (base + lane < seg_hi) { cmin = min(cmin, c); cmax = max(cmax, c); }
     }
-    const int run_base = block_exclusive_scan(n_starts, warp_sums, &s_total);
-    const int n_runs = s_total;
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1) {
         cmin = min(cmin, __shfl_xor_sync(0xffffffffu, cmin, m));
         cmax = max(cmax, __shfl_xor_sync(0xffffffffu, cmax, m));
     }
-    if ((tid & 31) == 0) { s_cmin[tid >> 5] = cmin; s_cmax[tid >> 5] = cmax; }
-    {
-        int r = run_base;
-        for (int i = seg_lo; i < seg_hi; ++i) {
-            const int c = a.tok_chunk[i];
-            if (i == lo || c != a.tok_chunk[i - 1]) {
-                a.ws.run_start[r] = i;
-                a.ws.run_chunk[r] = c;
-                ++r;
-            }
-        }
-    }
+    if (lane == 0) { warp_sums[warp] = n_starts; s_cmin[warp] = cmin; s_cmax[warp] = cmax; }
     if (tid < kMaxSpans) s_span_total[tid] = 0;
     __syncthreads();
+    if (warp == 0) {                                   // exclusive scan of the per-warp run counts
+        const int v = warp_sums[lane];
+        int incl = v;
+#pragma unroll
+        for (int m = 1; m < 32; m <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, m);
+            if (lane >= m) incl += y;
+        }
+        warp_sums[lane] = incl - v;
+        if (lane == 31) s_total = incl;
+    }
+    __syncthreads();
+    const int run_base = warp_sums[warp];
+    const int n_runs = s_total;
+    const bool small = n_runs <= kSmallRuns;
     int c_lo = INT_MAX, c_hi = INT_MIN;
     for (int w = 0; w < kSelWarps; ++w) { c_lo = min(c_lo, s_cmin[w]); c_hi = max(c_hi, s_cmax[w]); }
     const long long span_width = (long long)c_hi - c_lo + 1;
+    int* r_start = small ? s_rstart : a.ws.run_start;
+    int* r_len = small ? s_rlen : a.ws.run_len;
+    int* r_span = small ? s_rspan : a.ws.run_span;
+    int* r_kept = small ? s_rkept : a.ws.kept;
+    int* r_off = small ? s_roff : a.ws.out_off;
+    uint64_t* r_key = small ? s_rkey : a.ws.run_key;
+    {
+        int running = 0;
+        for (int base = seg_lo; base < seg_hi; base += 32) {
+            int c;
+            const bool st = run_start_flag(a.tok_chunk, lo, seg_hi, base + lane, c);
+            const unsigned bal = __ballot_sync(0xffffffffu, st);
+            if (st) r_start[run_base + running + __popc(bal & lt_mask)] = base + lane;
+            running += __popc(bal);
+        }
+    }
+    __syncthreads();
 
-    // ---- B. per-run length, span and key
+    // ---- B. per-run length, span and key (larger key = better: score desc, first slot asc)
     for (int r = tid; r < n_runs; r += kSelThreads) {
-        const int start = a.ws.run_start[r];
-        const int end = (r + 1 < n_runs) ? a.ws.run_start[r + 1] : hi;
-        const int c = a.ws.run_chunk[r];
+        const int st = r_start[r];
+        const int end = (r + 1 < n_runs) ? r_start[r + 1] : hi;
+        const int c = a.tok_chunk[st];
         const int span = (int)(((long long)(c - c_lo) * N) / span_width);
-        a.ws.run_len[r] = end - start;
-        a.ws.run_span[r] = span;
-        a.ws.run_key[r] = ((uint64_t)score_order_bits(a.scores[c]) << 32) | (uint64_t)(~(uint32_t)start);
-        atomicAdd(&s_span_total[span], end - start);
+        r_len[r] = end - st;
+        r_span[r] = span;
+        r_key[r] = ((uint64_t)score_order_bits(a.scores[c]) << 32) | (uint64_t)(~(uint32_t)st);
+        atomicAdd(&s_span_total[span], end - st);
     }
     __syncthreads();
     if (tid < N) {
@@ -252,68 +288,110 @@ select_retain_kernel(SelArgs a)
         s_mode[tid] = (m == 0) ? kNone : (m == tot ? kAll : kSome);
     }
     __syncthreads();
-    // per-span quota actually granted (needed for the fill target)
     int granted = 0;
-    if (tid == 0) for (int j = 0; j < N; ++j) granted += s_target[j];
+    for (int jj = 0; jj < N; ++jj) granted += s_target[jj];
+    const int fill = R - granted;
 
-    // ---- C. per-span quota
-    weighted_select(n_runs, a.ws.run_key, a.ws.run_len, a.ws.run_span, N, s_prefix, s_target,
-                    s_mode, s_hist);
-    for (int r = tid; r < n_runs; r += kSelThreads) {
-        const int j = a.ws.run_span[r];
-        const int len = a.ws.run_len[r];
-        int k1 = 0;
-        if (s_mode[j] == kAll) k1 = len;
-        else if (s_mode[j] == kSome) {
-            const uint64_t key = a.ws.run_key[r];
-            k1 = key > s_prefix[j] ? len : (key == s_prefix[j] ? s_target[j] : 0);
+    if (small) {
+        // ---- C/D (at most 512 runs, one per thread): a run keeps the part of its span quota
+        // (then of the fill) that the runs ranked above it leave over.
+        int k1 = 0, rem = 0, len = 0, st = 0;
+        uint64_t key = 0;
+        if (tid < n_runs) {
+            len = s_rlen[tid]; st = s_rstart[tid]; key = s_rkey[tid];
+            const int j = s_rspan[tid];
+            int above = 0;
+            for (int r = 0; r < n_runs; ++r)
+                if (s_rspan[r] == j && s_rkey[r] > key) above += s_rlen[r];
+            k1 = min(len, max(0, s_target[j] - above));
+            rem = len - k1;
         }
-        a.ws.kept1[r] = k1;
-        a.ws.run_len[r] = len - k1;   // remainder weight for the fill
-        a.ws.run_key[r] = (a.ws.run_key[r] & 0xFFFFFFFF00000000ull) |
-                          (uint64_t)(~(uint32_t)(a.ws.run_start[r] + k1));
-    }
-    if (tid == 0) {
-        const int fill = R - granted;
-        s_fill_target[0] = fill;
-        s_fill_mode[0] = fill > 0 ? kSome : kNone;
-    }
-    __syncthreads();
-
-    // ---- D. fill the unused capacity from the best remaining candidates
-    weighted_select(n_runs, a.ws.run_key, a.ws.run_len, nullptr, 1, s_fill_prefix, s_fill_target,
-                    s_fill_mode, s_hist);
-    const int per = (n_runs + kSelThreads - 1) / kSelThreads;
-    const int r_lo = min(tid * per, n_runs), r_hi = min(r_lo + per, n_runs);
-    int my_kept = 0;
-    for (int r = r_lo; r < r_hi; ++r) {
-        const int rem = a.ws.run_len[r];
-        int k2 = 0;
-        if (s_fill_mode[0] == kSome && rem > 0) {
-            const uint64_t key = a.ws.run_key[r];
-            k2 = key > s_fill_prefix[0] ? rem : (key == s_fill_prefix[0] ? s_fill_target[0] : 0);
+        __syncthreads();
+        if (tid < n_runs) {
+            s_rlen[tid] = rem;
+            s_rkey[tid] = (key & 0xFFFFFFFF00000000ull) | (uint64_t)(~(uint32_t)(st + k1));
         }
-        const int k = a.ws.kept1[r] + k2;
-        a.ws.kept[r] = k;
-        my_kept += k;
+        __syncthreads();
+        int kept = 0;
+        if (tid < n_runs) {
+            int k2 = 0;
+            if (fill > 0 && rem > 0) {
+                const uint64_t key2 = s_rkey[tid];
+                int above = 0;
+                for (int r = 0; r < n_runs; ++r)
+                    if (s_rkey[r] > key2) above += s_rlen[r];
+                k2 = min(rem, max(0, fill - above));
+            }
+            kept = k1 + k2;
+            s_rkept[tid] = kept;
+        }
+        const int off = block_exclusive_scan(kept, warp_sums, &s_total);
+        if (tid < n_runs) s_roff[tid] = off;
+        __syncthreads();
+    } else {
+        // ---- C. per-span quota by token-weighted radix selection
+        weighted_select(n_runs, a.ws.run_key, a.ws.run_len, a.ws.run_span, N, s_prefix, s_target,
+                        s_mode, s_hist);
+        for (int r = tid; r < n_runs; r += kSelThreads) {
+            const int j = a.ws.run_span[r];
+            const int len = a.ws.run_len[r];
+            int k1 = 0;
+            if (s_mode[j] == kAll) k1 = len;
+            else if (s_mode[j] == kSome) {
+                const uint64_t key = a.ws.run_key[r];
+                k1 = key > s_prefix[j] ? len : (key == s_prefix[j] ? s_target[j] : 0);
+            }
+            a.ws.kept1[r] = k1;
+            a.ws.run_len[r] = len - k1;
+            a.ws.run_key[r] = (a.ws.run_key[r] & 0xFFFFFFFF00000000ull) |
+                              (uint64_t)(~(uint32_t)(a.ws.run_start[r] + k1));
+        }
+        if (tid == 0) {
+            s_fill_target[0] = fill;
+            s_fill_mode[0] = fill > 0 ? kSome : kNone;
+        }
+        __syncthreads();
+        // ---- D. fill the unused capacity from the best remaining candidates
+        weighted_select(n_runs, a.ws.run_key, a.ws.run_len, nullptr, 1, s_fill_prefix, s_fill_target,
+                        s_fill_mode, s_hist);
+        const int per = (n_runs + kSelThreads - 1) / kSelThreads;
+        const int r_lo = min(tid * per, n_runs), r_hi = min(r_lo + per, n_runs);
+        int my_kept = 0;
+        for (int r = r_lo; r < r_hi; ++r) {
+            const int remr = a.ws.run_len[r];
+            int k2 = 0;
+            if (s_fill_mode[0] == kSome && remr > 0) {
+                const uint64_t key = a.ws.run_key[r];
+                k2 = key > s_fill_prefix[0] ? remr : (key == s_fill_prefix[0] ? s_fill_target[0] : 0);
+            }
+            const int k = a.ws.kept1[r] + k2;
+            a.ws.kept[r] = k;
+            my_kept += k;
+        }
+        int off = block_exclusive_scan(my_kept, warp_sums, &s_total);
+        for (int r = r_lo; r < r_hi; ++r) {
+            a.ws.out_off[r] = off;
+            off += a.ws.kept[r];
+        }
+        __syncthreads();
     }
 
-    // ---- E. output offsets and slot writes
-    int off = block_exclusive_scan(my_kept, warp_sums, &s_total);
-    for (int r = r_lo; r < r_hi; ++r) {
-        a.ws.out_off[r] = off;
-        off += a.ws.kept[r];
-    }
-    __syncthreads();
+    // ---- E. every slot writes itself if it lies in its run's kept prefix
     {
-        int r = run_base - 1;
-        for (int i = seg_lo; i < seg_hi; ++i) {
-            const int c = a.tok_chunk[i];
-            if (i == lo || c != a.tok_chunk[i - 1]) ++r;
-            const int pos = i - a.ws.run_start[r];
-            const bool keep = pos < a.ws.kept[r];
-            if (keep) a.retain_idx[a.n_s + a.ws.out_off[r] + pos] = i;
-            if (a.mask) a.mask[i] = keep ? 1 : 0;
+        int running = 0;
+        for (int base = seg_lo; base < seg_hi; base += 32) {
+            int c;
+            const int i = base + lane;
+            const bool st = run_start_flag(a.tok_chunk, lo, seg_hi, i, c);
+            const unsigned bal = __ballot_sync(0xffffffffu, st);
+            if (i < seg_hi) {
+                const int r = run_base + running + __popc(bal & (lt_mask | (1u << lane))) - 1;
+                const int pos = i - r_start[r];
+                const bool keep = pos < r_kept[r];
+                if (keep) a.retain_idx[a.n_s + r_off[r] + pos] = i;
+                if (a.mask) a.mask[i] = keep ? 1 : 0;
+            }
+            running += __popc(bal);
         }
     }
     for (int i = tid; i < a.n_s; i += kSelThreads) {
