@@ -188,6 +188,31 @@ DELTAS_API deltas_status deltas_select_retain(const deltas_policy* policy, int32
                                    void* workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------------------------ */
+/* Retain selection without a caller workspace (the paper has no counterpart: this is a         */
+/* library convenience).  For callers that may not allocate device memory: a serving runtime    */
+/* that owns all of HBM through its own pool, or code running where cudaMalloc is not allowed.  */
+/* It calls no cudaMalloc, cudaFree or other allocating routine.                                */
+/*                                                                                              */
+/* Arguments, outputs and results are those of deltas_select_retain without the workspace.  The */
+/* scratch is a fixed device array inside the library sized for                                 */
+/* DELTAS_SELECT_STATIC_MAX_CACHE_LEN slots (about 2.25 MiB); a larger cache_len returns        */
+/* DELTAS_ERR_UNSUPPORTED with nothing enqueued.                                                */
+/*   - The first call on a device looks up the array's address (with that device current, the  */
+/*     stream must belong to it) and caches it; make that first call before any stream capture. */
+/*   - All calls on a device share the array.  Calls whose kernels may run at the same time on   */
+/*     the GPU (streams with no ordering between them) race and give undefined results.         */
+/*   - Each call clears the status word at the head of the array on its stream before the       */
+/*     launch.  A tok_chunk value outside [0, num_chunks) is reported on the device by          */
+/*     *n_retained == 0 while cache_len > 0 (a valid call always keeps at least one slot).      */
+/* ------------------------------------------------------------------------------------------ */
+#define DELTAS_SELECT_STATIC_MAX_CACHE_LEN 65536
+
+DELTAS_API deltas_status deltas_select_retain_static(const deltas_policy* policy, int32_t cache_len,
+                                   int32_t num_chunks, const int32_t* tok_chunk,
+                                   const float* chunk_scores, int32_t* retain_idx,
+                                   int32_t* n_retained, uint8_t* mask, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
 /* In-place KV compaction (Alg. 1 "KV <- KV[I_sink u I_DeltaS u I_window]", applied to every    */
 /* full-attention layer; Sec. 3.3: survivors keep their original position indices).            */
 /*                                                                                              */

@@ -35,7 +35,7 @@ EXPORTED = (
     "deltas_gdn_chunk_update_workspace_size", "deltas_gdn_chunk_update",
     "deltas_state_drift_workspace_size", "deltas_state_drift",
     "deltas_score_chunks",
-    "deltas_select_retain_workspace_size", "deltas_select_retain",
+    "deltas_select_retain_workspace_size", "deltas_select_retain", "deltas_select_retain_static",
     "deltas_compact_kv_workspace_size", "deltas_compact_kv",
     "deltas_append_kv",
     "deltas_clear_device_status", "deltas_get_device_status",
@@ -85,6 +85,7 @@ _sig("deltas_state_drift", ctypes.c_int, _P, _P, _P, _P, _P, _SZ, _P)
 _sig("deltas_score_chunks", ctypes.c_int, _I32, _I32, _P, _I32, _P, _P)
 _sig("deltas_select_retain_workspace_size", _SZ, _I32)
 _sig("deltas_select_retain", ctypes.c_int, _P, _I32, _I32, _P, _P, _P, _P, _P, _P, _SZ, _P)
+_sig("deltas_select_retain_static", ctypes.c_int, _P, _I32, _I32, _P, _P, _P, _P, _P, _P)
 _sig("deltas_compact_kv_workspace_size", _SZ, _P, _I32)
 _sig("deltas_compact_kv", ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, _I32, _P, _SZ, _P)
 _sig("deltas_append_kv", ctypes.c_int, _P, _P, _P, _P, _P, _I32, _P, _P, _I32, _I32, _I32, _P)
@@ -220,6 +221,25 @@ def deltas_select_retain(pol: Policy, cache_len: int, tok_chunk, chunk_scores, r
                                    _ptr(workspace, torch.uint8, None, "workspace"), workspace.numel(),
                                    _stream(stream))
     _check(st, "deltas_select_retain")
+
+
+SELECT_STATIC_MAX_CACHE_LEN = 65536   # DELTAS_SELECT_STATIC_MAX_CACHE_LEN
+
+
+def deltas_select_retain_static(pol: Policy, cache_len: int, tok_chunk, chunk_scores, retain_idx, n_retained,
+                                mask, stream=None):
+    """deltas_select_retain with the library's own fixed scratch: no workspace and no allocation."""
+    T = int(cache_len)
+    if tok_chunk.numel() < T or retain_idx.numel() < min(T, pol.budget_M) or (mask is not None and mask.numel() < T):
+        raise ValueError("select_retain_static: an output or input is shorter than cache_len / budget")
+    st = _lib.deltas_select_retain_static(ctypes.byref(pol), T, int(chunk_scores.numel()),
+                                          _ptr(tok_chunk, torch.int32, None, "tok_chunk"),
+                                          _ptr(chunk_scores, torch.float32, None, "chunk_scores"),
+                                          _ptr(retain_idx, torch.int32, None, "retain_idx"),
+                                          _ptr(n_retained, torch.int32, None, "n_retained"),
+                                          _ptr(mask, torch.uint8, None, "mask"),
+                                          _stream(stream))
+    _check(st, "deltas_select_retain_static")
 
 
 def deltas_compact_kv_workspace_size(desc: KvDesc, cache_len: int) -> int:

@@ -428,3 +428,74 @@ cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_
 }
 
 }  // namespace deltas
+
+// -------------------------------------------------------------------------------------------------
+// deltas_select_retain_static: the same selection with its scratch in this module's own device
+// memory, for callers that may not allocate device memory at all (a runtime that owns every byte of
+// HBM through its own pool or arena, or code running where cudaMalloc and friends are not allowed).
+//
+// The scratch is one file-scope array sized for DELTAS_SELECT_STATIC_MAX_CACHE_LEN slots.  Its
+// address is looked up with cudaGetSymbolAddress the first time the entry point runs on a device
+// (with that device current) and cached per device.  Every call on a device shares the array and
+// finds it as the previous call left it: the status word at its head is the only part that has to
+// start at zero, and it is cleared on the caller's stream before each launch; every other word the
+// kernel reads was written earlier in the same launch.  Calls whose kernels can overlap on the GPU
+// (different streams without ordering between them) race on the array.
+// -------------------------------------------------------------------------------------------------
+#include <mutex>
+
+namespace {
+
+constexpr size_t kStaticMaxSlots = DELTAS_SELECT_STATIC_MAX_CACHE_LEN;
+// the layout carve() gives for kStaticMaxSlots slots: status word, 7 int32 arrays, 1 uint64 array
+constexpr size_t kStaticScratchBytes =
+    deltas::kStatusBytes + 7 * sizeof(int32_t) * kStaticMaxSlots + sizeof(uint64_t) * kStaticMaxSlots;
+static_assert(kStaticScratchBytes % 256 == 0, "every scratch array must stay 256-byte aligned");
+
+static __device__ __align__(256) unsigned char g_select_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+deltas_status static_scratch_for_current_device(void** out) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) return DELTAS_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices) return DELTAS_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_scratch_mutex);
+    if (g_scratch_ptr[dev] == nullptr) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_select_scratch) != cudaSuccess || p == nullptr) return DELTAS_ERR_CUDA;
+        g_scratch_ptr[dev] = p;
+    }
+    *out = g_scratch_ptr[dev];
+    return DELTAS_OK;
+}
+
+}  // namespace
+
+extern "C" deltas_status deltas_select_retain_static(const deltas_policy* policy, int32_t cache_len,
+                                                     int32_t num_chunks, const int32_t* tok_chunk,
+                                                     const float* chunk_scores, int32_t* retain_idx,
+                                                     int32_t* n_retained, uint8_t* mask, void* stream)
+{
+    // the checks of deltas_select_retain, made here so that nothing is enqueued when one fails
+    if (policy == nullptr || cache_len < 0 || num_chunks < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    const deltas_policy& p = *policy;
+    if (p.budget_M < 1 || p.n_sink < 0 || p.n_window < 0 || p.n_buckets < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if ((long long)p.budget_M < (long long)p.n_sink + p.n_window + 1) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (p.n_buckets > 32) return DELTAS_ERR_UNSUPPORTED;
+    if (!retain_idx || !n_retained) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (cache_len > 0 && (!tok_chunk || !chunk_scores)) return DELTAS_ERR_INVALID_ARGUMENT;
+    if ((size_t)cache_len > kStaticMaxSlots) return DELTAS_ERR_UNSUPPORTED;     // beyond the scratch
+
+    void* scratch = nullptr;
+    const deltas_status st = static_scratch_for_current_device(&scratch);
+    if (st != DELTAS_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaMemsetAsync(scratch, 0, deltas::kStatusBytes, s) != cudaSuccess) return DELTAS_ERR_CUDA;
+    const cudaError_t e = deltas::launch_select_retain(p, cache_len, num_chunks, tok_chunk, chunk_scores,
+                                                       retain_idx, n_retained, mask, scratch,
+                                                       static_cast<int32_t*>(scratch), s);
+    return e == cudaSuccess ? DELTAS_OK : DELTAS_ERR_CUDA;
+}
