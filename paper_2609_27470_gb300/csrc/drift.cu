@@ -69,10 +69,15 @@ score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk
             num += __shfl_xor_sync(0xffffffffu, num, m);
             den += __shfl_xor_sync(0xffffffffu, den, m);
         }
-        double term;
-        if (den > 0.0) term = sqrt(num) / sqrt(den);
-        else term = (num > 0.0) ? (double)INFINITY : 0.0;
-        acc += term;   // layers l, l + 32, ... in increasing order
+        // The square roots and the quotient are taken in float (correctly rounded, a few ulp of
+        // float in all): double square roots and divisions run on the slow FP64 pipe.
+        if (lane == 0) {
+            const float nf = (float)num, df = (float)den;
+            double term;
+            if (den > 0.0) term = (double)(sqrtf(nf) / sqrtf(df));
+            else term = (num > 0.0) ? (double)INFINITY : 0.0;
+            acc += term;   // layers l, l + 32, ... in increasing order
+        }
     }
     if (lane == 0) term_sum[warp] = acc;
     __syncthreads();
