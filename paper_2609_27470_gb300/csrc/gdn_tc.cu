@@ -9,9 +9,11 @@
 //   S_C = gamma_C S0 + U~^T K,   U~[t] = exp(G_C - G_t) U[t].
 // Padded tokens of a ragged last tile carry k = v = 0, g = 0, beta = 0 and change nothing.
 //
-// One CTA owns one (layer, value head) for the whole chunk.  The state lives in TMEM from the
-// first tile to the last and S_before stays in shared memory, so the state is read from and
-// written to HBM exactly once and the drift needs no second pass over it.
+// One persistent CTA per SM takes (layer, value head) pairs in turn, each for the whole chunk;
+// the tiles of its heads form one pipeline, so a head's loads and T builds start while the
+// previous head drains.  A head's state lives in TMEM from its first tile to its last and
+// S_before stays in shared memory, so the state is read from and written to HBM exactly once and
+// the drift needs no second pass over it.
 //
 // Precision: every product that touches the state or T uses a two-term bfloat16 split
 // (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)); keys and values are exact in bfloat16.  With
@@ -40,6 +42,8 @@
 // TMEM (512 columns, M = 128 lanes = d_v): S [0,128), S0 hi / lo packed [128,192) / [192,256),
 // X [256,320) (fp32, then X~ hi / lo packed in place), U [320,384) (likewise U~), K K^T of even /
 // odd tiles [384,448) / [448,512).
+#include <algorithm>
+
 #include "internal.cuh"
 #include "tc_ptx.cuh"
 
@@ -64,7 +68,7 @@ constexpr int FX_S = 68;               // fp32 row stride of X^-1 (16-byte align
 constexpr uint32_t SM_K = 0;                      // 3 x 16 KB: K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
 constexpr uint32_t SM_V = 49152;                  // 16 KB: V tile, same layout
 constexpr uint32_t SM_T = 65536;                  // 2 buffers x (hi 8 KB, lo 8 KB): T, 64 rows (t) x 64 (i)
-constexpr uint32_t SM_SB = 98304;                 // 64 KB: S_before fp32, column-major [d_k][d_v]
+constexpr uint32_t SM_SB = 98304;                 // 64 KB: S_before fp32, 4 column blocks x 128 rows x 128 B, SW128
 constexpr uint32_t SM_FA = 163840;                // fp32 [64][FA_S]
 constexpr uint32_t SM_FX = SM_FA + 64 * FA_S * 4; // fp32 [64][FX_S]
 constexpr uint32_t SM_TMP = SM_FX + 64 * FX_S * 4;// fp32 [32][33]
@@ -77,6 +81,14 @@ static_assert(kSmemAlloc <= 232448, "shared memory budget");
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// S_before: the head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each 128 rows x
+// 128 bytes with the 128-byte swizzle (16-byte chunk ^ (row & 7)) that TMA writes and reads; eight
+// threads reading chunk c of eight consecutive rows (one row per thread) hit distinct banks.
+// Float offset of 16-byte chunk `chunk` (0..31) of row `row`:
+__device__ __forceinline__ int sb_idx(int row, int chunk) {
+    return (chunk >> 3) * 4096 + row * 32 + (((chunk & 7) ^ (row & 7)) << 2);
+}
+
 struct TcArgs {
     int L, Hk, Hv, T, n_tiles;
     float* state;
@@ -84,6 +96,20 @@ struct TcArgs {
     const float* g;
     const float* beta;
     int32_t* status;
+};
+
+// Where a global tile lies: tile jt of head lh = (layer l, value head h), key head kh.  Each role
+// walks the tiles in order; a step costs integer divisions only when it crosses into the next head.
+struct TileCursor {
+    int jt, lh, l, h, kh;
+    __device__ __forceinline__ void set_head(int head, const TcArgs& a) {
+        lh = head; l = head / a.Hv; h = head - l * a.Hv;
+        kh = (int)(((long long)h * a.Hk) / a.Hv);
+    }
+    __device__ __forceinline__ void init(const TcArgs& a) { jt = 0; set_head((int)blockIdx.x, a); }
+    __device__ __forceinline__ void next(int n, const TcArgs& a) {
+        if (++jt == n) { jt = 0; set_head(lh + (int)gridDim.x, a); }
+    }
 };
 
 __device__ __forceinline__ void named_sync(int id, int n) {
@@ -150,23 +176,27 @@ __device__ __forceinline__ void fail(int32_t* status, volatile int* abort, int w
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, TcArgs a)
+gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                     const __grid_constant__ CUtensorMap smap, TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
     // TMA -> MMA: K buffers, V buffer.  MMA -> roles: kk, x, u, s.  roles -> MMA: ready flags.
     __shared__ uint64_t mb_tk[3], mb_tv, mb_kk[2], mb_x, mb_u, mb_s, mb_sready, mb_xready, mb_uready, mb_tready, mb_fin;
     __shared__ uint64_t mb_cready[3];                  // chain tile constants of tile t in buffer t % 3
+    __shared__ uint64_t mb_st;                         // a head's state landed in S_before
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ double s_red[2][8];
     volatile int* abort_flag = &s_abort;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int lh = blockIdx.x;
-    const int l = lh / a.Hv, h = lh % a.Hv;
-    const int kh = (int)(((long long)h * a.Hk) / a.Hv);
     const int n = a.n_tiles;
+    // Persistent CTA: it owns heads blockIdx.x, blockIdx.x + gridDim.x, ...  Their tiles form one
+    // sequence J = head slot * n + tile, over which every role keeps its barrier phases, so the
+    // next head's loads and T builds overlap the current head's last tiles.
+    const int n_heads = a.L * a.Hv;
+    const int NJ = ((n_heads - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x) * n;
 
     if (warp == kCtlWarp) {
         tmem_alloc(&s_tmem, kTmemCols);
@@ -178,9 +208,11 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             mbar_init(&mb_sready, kChain); mbar_init(&mb_xready, kChain); mbar_init(&mb_uready, kChain);
             mbar_init(&mb_tready, kTB); mbar_init(&mb_fin, 1);
             mbar_init(&mb_cready[0], 1); mbar_init(&mb_cready[1], 1); mbar_init(&mb_cready[2], 1);
+            mbar_init(&mb_st, 1);
             fence_barrier_init();
             prefetch_tensormap(&kmap);
             prefetch_tensormap(&vmap);
+            prefetch_tensormap(&smap);
         }
     }
     if (tid == 0) s_abort = 0;
@@ -193,23 +225,27 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         // =========================================================== TMA + MMA issue (whole warp,
         // converged; elect.sync picks the issuing lane)
         {
-            auto load_k = [&](int tile) {              // K tile `tile` -> buffer tile % 3
-                const int b = tile % 3;
+            TileCursor kc, vc;                         // next K / V tile to load (loaded in order)
+            kc.init(a); vc.init(a);
+            auto load_k = [&](int J) {                 // K tile of global tile J -> buffer J % 3
+                const int b = J % 3;
                 if (elect_one()) {
                     uint8_t* dst = sm + SM_K + b * 16384;
                     mbar_arrive_expect_tx(&mb_tk[b], 16384);
-                    tma_load_4d(dst, &kmap, &mb_tk[b], 0, kh, tile * kC, l);
-                    tma_load_4d(dst + 8192, &kmap, &mb_tk[b], 64, kh, tile * kC, l);
+                    tma_load_4d(dst, &kmap, &mb_tk[b], 0, kc.kh, kc.jt * kC, kc.l);
+                    tma_load_4d(dst + 8192, &kmap, &mb_tk[b], 64, kc.kh, kc.jt * kC, kc.l);
                 }
                 __syncwarp();
+                kc.next(n, a);
             };
-            auto load_v = [&](int tile) {
+            auto load_v = [&]() {
                 if (elect_one()) {
                     mbar_arrive_expect_tx(&mb_tv, 16384);
-                    tma_load_4d(sm + SM_V, &vmap, &mb_tv, 0, h, tile * kC, l);
-                    tma_load_4d(sm + SM_V + 8192, &vmap, &mb_tv, 64, h, tile * kC, l);
+                    tma_load_4d(sm + SM_V, &vmap, &mb_tv, 0, vc.h, vc.jt * kC, vc.l);
+                    tma_load_4d(sm + SM_V + 8192, &vmap, &mb_tv, 64, vc.h, vc.jt * kC, vc.l);
                 }
                 __syncwarp();
+                vc.next(n, a);
             };
             auto mma_kk = [&](int tile) {
                 // K K^T into the K K^T buffer of the tile's parity.  M = 128: rows 64..127 of A read
@@ -226,16 +262,15 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             int kp[3] = {-1, -1, -1};                  // tile whose K load is in flight, per buffer
             int v_pending = 0;
             load_k(0); kp[0] = 0;
-            if (n > 1) { load_k(1); kp[1] = 1; }
-            load_v(0);
+            if (NJ > 1) { load_k(1); kp[1] = 1; }
+            load_v();
             bool ok = warp_wait(&mb_tk[0], 0, kWaitBudgetNs, abort_flag);
             if (!ok) fail(a.status, abort_flag, 1);
             if (ok) { kp[0] = -1; mma_kk(0); }
-            for (int j = 0; ok && j < n; ++j) {
+            for (int j = 0; ok && j < NJ; ++j) {          // j: global tile index
                 const uint8_t* sK = sm + SM_K + (j % 3) * 16384;
                 // S0 split of tile j ready (the chain has seen MMA_S(j-1) complete)
                 if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
-                if (j + 2 < n) { load_k(j + 2); kp[(j + 2) % 3] = j + 2; }
                 tc_fence_after();
                 {   // X^T = S0 K^T   (A: S0 hi / lo from TMEM, 8 columns per K = 16 step)
                     const uint32_t id = idesc_bf16(128, 64, 0, 0);
@@ -250,7 +285,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     }
                     mma_commit(&mb_x);
                 }
-                if (j + 1 < n) {                       // K K^T of the next tile, for the T builders
+                if (j + 1 < NJ) {                      // K K^T of the next tile, for the T builders
                     if (!warp_wait(&mb_tk[(j + 1) % 3], ((j + 1) / 3) & 1, kWaitBudgetNs, abort_flag)) {
                         fail(a.status, abort_flag, 4); break;
                     }
@@ -284,8 +319,11 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     }
                     mma_commit(&mb_u);
                 }
+                // TMA loads are issued behind MMA groups, never between a wait and the MMAs it
+                // releases (a TMA write burst into shared memory slows the issue of a group).
+                // K(j+2) reuses the buffer of K(j-1), whose last reader MMA_S(j-1) has completed.
+                if (j + 2 < NJ) { load_k(j + 2); kp[(j + 2) % 3] = j + 2; }
                 if (!warp_wait(&mb_uready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 7); break; }
-                if (j + 1 < n) { load_v(j + 1); v_pending = j + 1; }
                 tc_fence_after();
                 {   // S += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major: N = d_k)
                     const uint32_t id = idesc_bf16(128, 128, 0, 1);
@@ -300,6 +338,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     }
                     mma_commit(&mb_s);
                 }
+                // V(j+1) into the single V buffer: MMA_U(j), its reader, completed before uready
+                if (j + 1 < NJ) { load_v(); v_pending = j + 1; }
             }
             if (__any_sync(0xffffffffu, *abort_flag != 0)) {
                 // drain: every MMA this warp issued, and every load still in flight
@@ -324,30 +364,26 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         int* sFactored = reinterpret_cast<int*>(sG2 + 256);
         float* cg = reinterpret_cast<float*>(sm + SM_CG);
         float pg[2] = {0.f, 0.f}, pb[2] = {0.f, 0.f};     // g, beta of the next tile (warp 8)
-        if (tw == 0) {
+        TileCursor gc;                                     // next tile whose g, beta to load
+        gc.init(a);
+        auto load_gb = [&]() {                             // g, beta of the next tile (warp 8)
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-                const int t = 2 * lane + e;
-                const size_t gi = ((size_t)l * a.T + t) * a.Hv + h;
+                const int t = gc.jt * kC + 2 * lane + e;
+                const size_t gi = ((size_t)gc.l * a.T + t) * a.Hv + gc.h;
                 pg[e] = t < a.T ? a.g[gi] : 0.f;
                 pb[e] = t < a.T ? a.beta[gi] : 0.f;
             }
-        }
-        for (int j = 0; j < n; ++j) {
+            gc.next(n, a);
+        };
+        if (tw == 0) load_gb();
+        for (int j = 0; j < NJ; ++j) {                     // j: global tile index
             if (named_sync_or(3, kTB, *abort_flag)) break;
             if (tw == 0) {                                 // per-tile decay constants
                 float gv[2], bv[2];
 #pragma unroll
                 for (int e = 0; e < 2; ++e) { gv[e] = pg[e]; bv[e] = pb[e]; }
-                if (j + 1 < n) {                           // prefetch the next tile's g, beta
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int t = (j + 1) * kC + 2 * lane + e;
-                        const size_t gi = ((size_t)l * a.T + t) * a.Hv + h;
-                        pg[e] = t < a.T ? a.g[gi] : 0.f;
-                        pb[e] = t < a.T ? a.beta[gi] : 0.f;
-                    }
-                }
+                if (j + 1 < NJ) load_gb();                 // prefetch the next tile's g, beta
                 float incl = gv[0] + gv[1];
 #pragma unroll
                 for (int m = 1; m < 32; m <<= 1) {
@@ -527,37 +563,58 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         const int r = 32 * q + lane;                       // row of S (value index)
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
         const uint32_t cS = TM_S + 64 * wg;                // this thread's 64 state columns
-        float* sbefore = reinterpret_cast<float*>(sm + SM_SB);   // [d_k][d_v]: column c at c * 128
+        float* sbefore = reinterpret_cast<float*>(sm + SM_SB);   // swizzled rows, see sb_idx
         float* cg = reinterpret_cast<float*>(sm + SM_CG);
+        // a head's state (128 rows of the state viewed as [L * Hv * d_v][d_k]) into S_before by TMA,
+        // issued by thread 0 of the chain, completing on mb_st
+        int st_issued = 0, st_seen = 0;                    // state loads issued / waited for (uniform)
+        auto load_state = [&](int lh) {
+            ++st_issued;
+            if (tid == 0) {
+                mbar_arrive_expect_tx(&mb_st, kD * kD * 4);
+#pragma unroll
+                for (int b = 0; b < 4; ++b) tma_load_2d(sbefore + 4096 * b, &smap, &mb_st, 32 * b, lh * kD);
+            }
+        };
+        if (NJ > 0) load_state((int)blockIdx.x);
+        TileCursor cc;                                     // the chain's tile
+        cc.init(a);
         float den = 0.f;
-        bool done = false;
-        for (int j = 0; j < n; ++j) {
+        for (int j = 0; j < NJ; ++j) {                     // j: global tile index
+            const int lh = cc.lh, jt = cc.jt;              // head and tile within the head
             float* gam = cg + (j % 3) * 132;               // -gamma (written by the T builders)
             float* del = gam + 64;                         // exp(G_C - G)
             if (named_sync_or(2, kChain, *abort_flag)) break;
             if (!mbar_wait_or_abort(&mb_cready[j % 3], (j / 3) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
             const float gC = gam[128];
 
-            // ---- S pass: S0 -> (hi, lo) packed into TMEM; gamma_C S0 -> TMEM (32 columns at a time)
-            if (j > 0) {
+            // ---- S pass: S0 -> (hi, lo) packed into TMEM; gamma_C S0 -> TMEM (32 columns at a time).
+            // A head's first tile reads S0 from HBM (the previous head's epilogue has already read
+            // its state out of TMEM); later tiles read it from TMEM once MMA_S has landed.
+            if (jt > 0) {
                 if (!mbar_wait_or_abort(&mb_s, (j - 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 9);
                 tc_fence_after();
+            } else {
+                // the head's state in S_before (loaded by TMA, issued at the previous head's end)
+                if (!mbar_wait_or_abort(&mb_st, (j / n) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 14);
+                ++st_seen;
+                if (j + n < NJ) {                          // the next head's state towards L2
+                    const char* nxt = reinterpret_cast<const char*>(a.state + (size_t)(lh + (int)gridDim.x) * kD * kD);
+                    asm volatile("prefetch.L2 [%0];" :: "l"(nxt + 256 * tid) : "memory");
+                    asm volatile("prefetch.L2 [%0];" :: "l"(nxt + 256 * tid + 128) : "memory");
+                }
             }
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
                 float sv[32];
-                if (j == 0) {
-                    const float4* src = reinterpret_cast<const float4*>(a.state + ((size_t)lh * kD + r) * kD + 64 * wg + 32 * half);
+                if (jt == 0) {
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
-                        const float4 x = src[e];
+                        const float4 x = *reinterpret_cast<const float4*>(sbefore + sb_idx(r, 16 * wg + 8 * half + e));
                         sv[4 * e] = x.x; sv[4 * e + 1] = x.y; sv[4 * e + 2] = x.z; sv[4 * e + 3] = x.w;
                     }
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        den += sv[e] * sv[e];
-                        sbefore[(64 * wg + 32 * half + e) * kD + r] = sv[e];
-                    }
+                    for (int e = 0; e < 32; ++e) den += sv[e] * sv[e];
                 } else {
                     tmem_ld32(tm + lane_off + cS + 32 * half, sv);
                     tmem_ld_wait();
@@ -610,44 +667,67 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             }
             tc_fence_before();
             mbar_arrive(&mb_uready);
-            done = (j == n - 1);
-        }
 
-        // ---- epilogue: S_after -> HBM, drift partials against S_before
-        bool ok = done && mbar_wait_or_abort(&mb_s, (n - 1) & 1, kWaitBudgetNs, abort_flag);
-        if (done && !ok) fail(a.status, abort_flag, 12);
-        tc_fence_after();
-        float num = 0.f;
-        if (ok) {
-            float4* dst = reinterpret_cast<float4*>(a.state + ((size_t)lh * kD + r) * kD + 64 * wg);
+            if (jt == n - 1) {
+                // ---- epilogue of the head: S_after -> HBM, drift partials against S_before
+                const bool ok = mbar_wait_or_abort(&mb_s, j & 1, kWaitBudgetNs, abort_flag);
+                if (!ok) fail(a.status, abort_flag, 12);
+                tc_fence_after();
+                float num = 0.f;
+                if (ok) {
+                    // S_after replaces S_before in shared memory (each thread its own row) ...
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                float sv[32];
-                tmem_ld32(tm + lane_off + cS + 32 * half, sv);
-                tmem_ld_wait();
+                    for (int half = 0; half < 2; ++half) {
+                        float sv[32];
+                        tmem_ld32(tm + lane_off + cS + 32 * half, sv);
+                        tmem_ld_wait();
 #pragma unroll
-                for (int e = 0; e < 32; ++e) {
-                    const float dlt = sv[e] - sbefore[(64 * wg + 32 * half + e) * kD + r];
-                    num += dlt * dlt;
+                        for (int e = 0; e < 8; ++e) {
+                            float4* p = reinterpret_cast<float4*>(sbefore + sb_idx(r, 16 * wg + 8 * half + e));
+                            const float4 b = *p;
+                            const float d0 = sv[4 * e] - b.x, d1 = sv[4 * e + 1] - b.y;
+                            const float d2 = sv[4 * e + 2] - b.z, d3 = sv[4 * e + 3] - b.w;
+                            num += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+                            *p = make_float4(sv[4 * e], sv[4 * e + 1], sv[4 * e + 2], sv[4 * e + 3]);
+                        }
+                    }
                 }
+                tc_fence_before();
+                fence_async_smem();
+                // ... and goes to HBM by TMA; once TMA has read it out, the next head's state
+                // comes in
+                if (named_sync_or(2, kChain, !ok)) break;
+                if (tid == 0) {
 #pragma unroll
-                for (int e = 0; e < 8; ++e)
-                    dst[8 * half + e] = make_float4(sv[4 * e], sv[4 * e + 1], sv[4 * e + 2], sv[4 * e + 3]);
+                    for (int b = 0; b < 4; ++b) tma_store_2d(&smap, sbefore + 4096 * b, 32 * b, lh * kD);
+                    bulk_commit();
+                    bulk_wait_read0();
+                }
+                if (j + 1 < NJ) load_state(lh + (int)gridDim.x);
+                // partial sums: float within a warp (the FP64 pipe is slow), double across warps
+                float fn = num, fd = den;
+#pragma unroll
+                for (int m = 16; m >= 1; m >>= 1) {
+                    fn += __shfl_xor_sync(0xffffffffu, fn, m);
+                    fd += __shfl_xor_sync(0xffffffffu, fd, m);
+                }
+                if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
+                const bool any_fail = named_sync_or(2, kChain, !ok);
+                if (tid == 0 && !any_fail && a.partials != nullptr) {
+                    double sn = 0.0, sd = 0.0;
+                    for (int w = 0; w < 8; ++w) { sn += s_red[0][w]; sd += s_red[1][w]; }
+                    a.partials[(size_t)lh * 2 + 0] = (float)sn;
+                    a.partials[(size_t)lh * 2 + 1] = (float)sd;
+                }
+                if (any_fail) break;
+                den = 0.f;
             }
+            cc.next(n, a);
         }
-        double dn = num, dd = den;
-#pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) {
-            dn += __shfl_xor_sync(0xffffffffu, dn, m);
-            dd += __shfl_xor_sync(0xffffffffu, dd, m);
-        }
-        if (lane == 0) { s_red[0][warp] = dn; s_red[1][warp] = dd; }
-        const bool any_fail = named_sync_or(2, kChain, !ok);
-        if (tid == 0 && !any_fail && a.partials != nullptr) {
-            double sn = 0.0, sd = 0.0;
-            for (int w = 0; w < 8; ++w) { sn += s_red[0][w]; sd += s_red[1][w]; }
-            a.partials[(size_t)lh * 2 + 0] = (float)sn;
-            a.partials[(size_t)lh * 2 + 1] = (float)sd;
+        if (tid == 0) {
+            bulk_wait0();                                  // the last state store is complete
+            // abort path: a state load issued but not waited for lands before the CTA ends
+            if (st_issued > st_seen) mbar_wait(&mb_st, (st_issued - 1) & 1, kWaitBudgetNs);
         }
     }
 
@@ -691,16 +771,32 @@ bool make_map(CUtensorMap* map, const void* base, int L, int T, int H) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The state [L * Hv * 128][128] fp32 as a 2-D map: a box of 32 columns x 128 rows (one column block
+// of one head), 128-byte swizzle.
+bool make_state_map(CUtensorMap* map, void* base, int heads) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)heads * kD};
+    cuuint64_t strides[1] = {(cuuint64_t)kD * 4};
+    cuuint32_t box[2] = {32, (cuuint32_t)kD};
+    cuuint32_t es[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 bool gdn_tc_supported(const GdnArgs& a) {
     return a.dk == kD && a.dv == kD && a.dtype == DELTAS_BF16 && a.out == nullptr && a.T > 0 &&
-           encode_fn() != nullptr;
+           (long long)a.L * a.Hv * kD < (1ll << 31) && encode_fn() != nullptr;   // TMA row coordinate
 }
 
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
-    CUtensorMap kmap, vmap;
-    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv)) return cudaErrorInvalidValue;
+    CUtensorMap kmap, vmap, smap;
+    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
+        !make_state_map(&smap, a.state, a.L * a.Hv))
+        return cudaErrorInvalidValue;
     static int configured_device = -1;
     int dev = 0;
     cudaGetDevice(&dev);
@@ -713,7 +809,10 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     TcArgs t;
     t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = (a.T + kC - 1) / kC;
     t.state = a.state; t.partials = a.partials; t.g = a.g; t.beta = a.beta; t.status = a.status;
-    gdn_update_tc_kernel<<<a.L * a.Hv, kThreads, kSmemAlloc, s>>>(kmap, vmap, t);
+    // one persistent CTA per SM (the kernel needs the whole SM: 512 TMEM columns, ~206 KB of
+    // shared memory); each takes every grid-th head
+    const int grid = std::min(a.L * a.Hv, device_sm_count());
+    gdn_update_tc_kernel<<<grid, kThreads, kSmemAlloc, s>>>(kmap, vmap, smap, t);
     return cudaGetLastError();
 }
 

@@ -123,6 +123,16 @@ def test_gdn_update_layer_width_chunk(L, want_out):
     _check_chunk(L, x, s0, want_out, torch.bfloat16, 128 ** -0.5)
 
 
+@pytest.mark.parametrize("T", [1, 130])
+def test_gdn_update_more_heads_than_sms(L, T):
+    """160 (layer, head) pairs (5 layers x 32 value heads, d = 128, bf16): more heads than SMs, so
+    the tensor-core kernel's persistent CTAs each run several heads back to back; every head is
+    compared with the oracle (one tile, and three tiles with a ragged tail)."""
+    x = inputs.gdn_chunk(5, T, 16, 32, 128, "bf16", inputs.seed_for(12, T))
+    s0 = inputs.initial_state(5, 32, 128, inputs.seed_for(13, T))
+    _check_chunk(L, x, s0, False, torch.bfloat16, 128 ** -0.5)
+
+
 def test_gdn_update_stack_width_sampled(L):
     """The full stack's width (24 layers x 32 value heads, d = 128, bf16, one 1024-token chunk)
     in the launch configuration the benchmark times; the oracle checks a sample of 12 (layer,
