@@ -19,6 +19,8 @@
 // Every wait is bounded (about one second); a wait that runs out records DELTAS_ERR_TIMEOUT,
 // raises the abort flag and skips its writes.  Traffic is the algorithmic minimum: each moved row
 // is read once and written once; rows that do not move are not touched.
+#include <climits>
+
 #include "internal.cuh"
 
 namespace deltas {
@@ -30,6 +32,7 @@ constexpr int kStageBytes = 32768;   // staged source rows of one unit
 struct CompactCtl {
     unsigned ticket;
     int abort;
+    int first;             // first destination row that moves (INT_MAX: none)
 };
 
 struct CompactArgs {
@@ -66,13 +69,14 @@ __global__ void compact_init_kernel(CompactArgs a) {
     const int total = a.n_planes * a.max_tiles;
     for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x)
         a.flags[e] = 0;
-    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < a.max_tiles; e += gridDim.x * blockDim.x)
-        a.need[e] = e;
-    if (blockIdx.x == 0 && threadIdx.x == 0) { a.ctl->ticket = 0; a.ctl->abort = 0; }
+    if (blockIdx.x == 0 && threadIdx.x == 0) { a.ctl->ticket = 0; a.ctl->abort = 0; a.ctl->first = INT_MAX; }
 }
 
-// Validates retain_idx and records, per source tile, the first earlier destination tile that
-// reads from it.
+// Validates retain_idx and records, per source tile, the first destination tile that reads from
+// it (itself if none does), and the first destination row that moves.  retain_idx is ascending,
+// so the rows reading one source tile are consecutive: the first of them writes need[] for its
+// source tile and for the unread tiles before it, each tile exactly once.  Rows with
+// retain_idx[j] == j form a prefix (a moved row pushes every later source further on).
 __global__ void compact_need_kernel(CompactArgs a) {
     const int n = *a.n_retained;
     if (n < 0 || n > a.cache_len) {
@@ -84,14 +88,22 @@ __global__ void compact_need_kernel(CompactArgs a) {
     }
     for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < n; j += gridDim.x * blockDim.x) {
         const int src = a.retain_idx[j];
-        const bool ok = src >= j && src < a.cache_len && (j == 0 || src > a.retain_idx[j - 1]);
+        const int prev = j > 0 ? a.retain_idx[j - 1] : -1;
+        const bool ok = src >= j && src < a.cache_len && src > prev;
         if (!ok) {
             atomicExch(&a.ctl->abort, 1);
             record_status(a.status, DELTAS_ERR_DEVICE_INDEX, j);
             continue;
         }
         const int ts = src / a.tile_rows, td = j / a.tile_rows;
-        if (ts != td) atomicMin(&a.need[ts], td);
+        const int tp = prev < 0 ? -1 : prev / a.tile_rows;
+        if (ts != tp) {
+            for (int t = tp + 1; t < ts; ++t) a.need[t] = t;        // unread tiles
+            a.need[ts] = td;
+        }
+        if (j == n - 1)
+            for (int t = ts + 1; t < a.max_tiles; ++t) a.need[t] = t;
+        if (src != j && prev == j - 1) a.ctl->first = j;           // unique: the first moved row
     }
 }
 
@@ -120,8 +132,7 @@ __device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_
 __device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 // Issues the asynchronous loads of one unit's moved source rows into a stage buffer.
-__device__ __forceinline__ void compact_issue_loads(const CompactArgs& a, int u, int n, uint8_t* stage) {
-    const int b = u / a.n_planes, p = u % a.n_planes;
+__device__ __forceinline__ void compact_issue_loads(const CompactArgs& a, int b, int p, int n, uint8_t* stage) {
     int rb;
     const char* base = plane_base(a, p, rb);
     const int j0 = b * a.tile_rows;
@@ -156,8 +167,11 @@ compact_main_kernel(CompactArgs a)
     volatile int* abort_flag = &a.ctl->abort;
     if (*abort_flag) return;
     const int n = *a.n_retained;
+    const int first = a.ctl->first;
+    if (first >= n) return;                                        // nothing moves
+    const int t0 = first / a.tile_rows;                            // tiles before t0 stay put
     const int n_tiles = (n + a.tile_rows - 1) / a.tile_rows;
-    const int units = n_tiles * a.n_planes;
+    const int units = (n_tiles - t0) * a.n_planes;
     const int tid = threadIdx.x, lane = tid & 31;
 
     for (;;) {
@@ -165,21 +179,21 @@ compact_main_kernel(CompactArgs a)
         __syncthreads();
         const int cur = s_unit[0];
         if (cur >= units) break;
-        compact_issue_loads(a, cur, n, stage);
+        const int b = t0 + cur / a.n_planes, p = cur % a.n_planes;
+        compact_issue_loads(a, b, p, n, stage);
         cp_async_commit();
         cp_async_wait_0();
         __syncthreads();
-        const int b = cur / a.n_planes, p = cur % a.n_planes;
         if (warp_id_is_zero()) {
             // publish, then wait (warp-parallel) for the earlier tiles that read this tile's rows
             if (lane == 0) {
                 __threadfence();
                 store_release(a.flags + (size_t)p * a.max_tiles + b, 1);
             }
-            const int first = a.need[b];
+            const int first_reader = a.need[b];
             int ok = 1;
             const uint64_t t_start = global_ns();
-            for (int bb = first; bb < b && ok; bb += 32) {
+            for (int bb = first_reader; bb < b && ok; bb += 32) {
                 const int mine = bb + lane;
                 const int32_t* f = a.flags + (size_t)p * a.max_tiles + mine;
                 for (;;) {
@@ -192,7 +206,7 @@ compact_main_kernel(CompactArgs a)
             if (lane == 0) {
                 if (!ok) {
                     atomicExch(&a.ctl->abort, 1);
-                    record_status(a.status, DELTAS_ERR_TIMEOUT, cur);
+                    record_status(a.status, DELTAS_ERR_TIMEOUT, b * a.n_planes + p);
                 }
                 s_ok = ok;
             }
