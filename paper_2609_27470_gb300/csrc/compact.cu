@@ -5,13 +5,14 @@
 // The gather row[j] <- row[retain_idx[j]] runs in place.  Because retain_idx is ascending with
 // retain_idx[j] >= j, the only hazard is a destination row that is still to be read as the
 // source of an earlier destination.  The work is cut into units (plane p, tile b of TB
-// destination rows); a unit
-//   1. stages the source rows of its tile in shared memory (16-byte cp.async loads),
+// destination rows, starting at the tile of the first row that moves); a unit
+//   1. stages the source rows of its tile in shared memory (TMA bulk copies, one per run of
+//      consecutive sources),
 //   2. publishes "tile b of plane p has been read" (release flag),
 //   3. waits until every earlier tile whose destinations read rows of tile b has published
-//      (the first such tile, need[b], comes from a prepass over retain_idx; one warp checks up to
+//      (the first such tile, need[b], comes from a prepass over retain_idx; the warp checks up to
 //      32 flags at once),
-//   4. writes its tile (16-byte stores; the destination rows of a tile are contiguous).
+//   4. writes its tile with one bulk store (the destination rows of a tile are contiguous).
 // A unit publishes as soon as its own loads have landed, never after a wait, so no wait chains
 // form across tiles.  Units are claimed through an atomic ticket in tile-major order, so a unit
 // only waits for units that were claimed earlier by running CTAs whose loads complete without
@@ -22,11 +23,13 @@
 #include <climits>
 
 #include "internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace deltas {
 namespace {
 
-constexpr int kCompactThreads = 256;
+using namespace tc;
+
 constexpr int kStageBytes = 32768;   // staged source rows of one unit
 
 struct CompactCtl {
@@ -107,7 +110,6 @@ __global__ void compact_need_kernel(CompactArgs a) {
     }
 }
 
-__device__ __forceinline__ bool warp_id_is_zero() { return (threadIdx.x >> 5) == 0; }
 
 __device__ __forceinline__ int load_acquire(const int32_t* p) {
     int v;
@@ -119,50 +121,30 @@ __device__ __forceinline__ void store_release(int32_t* p, int v) {
     asm volatile("st.release.gpu.global.b32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
 }
 
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;"
-                 :: "r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;"
-                 :: "r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
-// Issues the asynchronous loads of one unit's moved source rows into a stage buffer.
-__device__ __forceinline__ void compact_issue_loads(const CompactArgs& a, int b, int p, int n, uint8_t* stage) {
-    int rb;
-    const char* base = plane_base(a, p, rb);
-    const int j0 = b * a.tile_rows;
-    const int rows = min(a.tile_rows, n - j0);
-    if (rb >= 16) {
-        const int vpr = rb >> 4;
-        const int nv = rows * vpr;
-        for (int e = threadIdx.x; e < nv; e += kCompactThreads) {
-            const int r = e / vpr, c = e - r * vpr;
-            const int src = a.retain_idx[j0 + r];
-            if (src != j0 + r) cp_async16(stage + 16 * e, base + (size_t)src * rb + 16 * c);
-        }
-    } else {
-        for (int r = threadIdx.x; r < rows; r += kCompactThreads) {
-            const int src = a.retain_idx[j0 + r];
-            if (src != j0 + r) cp_async4(stage + 4 * r, base + (size_t)src * 4);
-        }
-    }
+// Bulk (TMA) copies between global and shared memory: 16-byte aligned addresses, sizes in
+// multiples of 16 bytes.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 :: "r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
 }
+__device__ __forceinline__ void bulk_store(void* dst, const void* src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
+                 :: "l"(dst), "r"(smem_u32(src)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async;" ::: "memory"); }
 
-// One unit at a time per CTA (several CTAs per SM keep the memory system busy): claim, load the
-// moved source rows, publish, wait for the earlier readers of this tile, store.  A CTA never holds
-// a claimed unit that it has not loaded and published while it waits on another one.
-__global__ void __launch_bounds__(kCompactThreads)
+// One warp per CTA (several CTAs per SM): claim a unit, load its moved source rows, publish, wait
+// for the earlier readers of this tile, store.  For key / value planes the rows move by TMA bulk
+// copies (one per run of consecutive sources, split at 32-row boundaries) into a shared-memory
+// stage and back out in one bulk store; the 4-byte metadata rows go through registers.  A CTA
+// never holds a claimed unit that it has not loaded and published while it waits on another one.
+__global__ void __launch_bounds__(32)
 compact_main_kernel(CompactArgs a)
 {
     extern __shared__ uint4 stage_raw[];
     uint8_t* stage = reinterpret_cast<uint8_t*>(stage_raw);
-    __shared__ int s_unit[2];
-    __shared__ int s_ok;
+    __shared__ uint64_t bar;
 
     volatile int* abort_flag = &a.ctl->abort;
     if (*abort_flag) return;
@@ -172,68 +154,106 @@ compact_main_kernel(CompactArgs a)
     const int t0 = first / a.tile_rows;                            // tiles before t0 stay put
     const int n_tiles = (n + a.tile_rows - 1) / a.tile_rows;
     const int units = (n_tiles - t0) * a.n_planes;
-    const int tid = threadIdx.x, lane = tid & 31;
+    const int lane = threadIdx.x;
+    if (lane == 0) { mbar_init(&bar, 1); fence_barrier_init(); }
+    __syncwarp();
 
+    uint32_t phase = 0;
+    bool store_pending = false;                                    // lane 0's bulk store in flight
+    bool load_pending = false;
     for (;;) {
-        if (tid == 0) s_unit[0] = (*abort_flag) ? units : (int)atomicAdd(&a.ctl->ticket, 1u);
-        __syncthreads();
-        const int cur = s_unit[0];
-        if (cur >= units) break;
-        const int b = t0 + cur / a.n_planes, p = cur % a.n_planes;
-        compact_issue_loads(a, b, p, n, stage);
-        cp_async_commit();
-        cp_async_wait_0();
-        __syncthreads();
-        if (warp_id_is_zero()) {
-            // publish, then wait (warp-parallel) for the earlier tiles that read this tile's rows
+        int u = 0;
+        if (lane == 0) u = (*abort_flag) ? units : (int)atomicAdd(&a.ctl->ticket, 1u);
+        u = __shfl_sync(0xffffffffu, u, 0);
+        if (u >= units) break;
+        const int b = t0 + u / a.n_planes, p = u % a.n_planes;
+        int rb;
+        char* base = plane_base(a, p, rb);
+        const int j0 = b * a.tile_rows;
+        const int j_end = min(j0 + a.tile_rows, n);
+        const int js = max(j0, first);                             // rows before `first` stay
+        const int nrows = j_end - js;
+        const bool kv = rb >= 16;
+
+        // ---- load the sources
+        bool ok = true;
+        if (kv) {
             if (lane == 0) {
-                __threadfence();
-                store_release(a.flags + (size_t)p * a.max_tiles + b, 1);
+                if (store_pending) bulk_wait_read0();              // the stage is free again
+                mbar_arrive_expect_tx(&bar, (uint32_t)nrows * rb);
             }
-            const int first_reader = a.need[b];
-            int ok = 1;
-            const uint64_t t_start = global_ns();
-            for (int bb = first_reader; bb < b && ok; bb += 32) {
-                const int mine = bb + lane;
-                const int32_t* f = a.flags + (size_t)p * a.max_tiles + mine;
-                for (;;) {
-                    const bool ready = (mine >= b) || load_acquire(f) != 0;
-                    if (__all_sync(0xffffffffu, ready)) break;
-                    if (*abort_flag || global_ns() - t_start > kWaitBudgetNs) { ok = 0; break; }
-                    __nanosleep(32);
+            __syncwarp();
+            for (int c0 = js; c0 < j_end; c0 += 32) {
+                const int r = c0 + lane;
+                const bool in = r < j_end;
+                const int src = in ? a.retain_idx[r] : 0;
+                int prev = __shfl_up_sync(0xffffffffu, src, 1);
+                const bool start = in && (lane == 0 || src != prev + 1);
+                const unsigned starts = __ballot_sync(0xffffffffu, start);
+                if (start) {
+                    const unsigned above = starts & ~((2u << lane) - 1u);   // later starts in this chunk
+                    const int stop = above ? c0 + __ffs(above) - 1 : min(c0 + 32, j_end);
+                    bulk_load(stage + (size_t)(r - j0) * rb, base + (size_t)src * rb, (uint32_t)(stop - r) * rb, &bar);
                 }
             }
-            if (lane == 0) {
-                if (!ok) {
-                    atomicExch(&a.ctl->abort, 1);
-                    record_status(a.status, DELTAS_ERR_TIMEOUT, b * a.n_planes + p);
-                }
-                s_ok = ok;
+            load_pending = true;
+            ok = mbar_wait_or_abort(&bar, phase, kWaitBudgetNs, abort_flag);
+            ok = __all_sync(0xffffffffu, ok) != 0;
+            if (ok) { phase ^= 1; load_pending = false; }
+        } else {                                                   // 4-byte rows via the stage
+            if (lane == 0 && store_pending) bulk_wait_read0();
+            __syncwarp();
+            int* st = reinterpret_cast<int*>(stage);
+            for (int r = js + lane; r < j_end; r += 32) st[r - j0] = reinterpret_cast<const int*>(base)[a.retain_idx[r]];
+            __syncwarp();
+        }
+        if (!ok) {
+            if (lane == 0) { atomicExch(&a.ctl->abort, 1); record_status(a.status, DELTAS_ERR_TIMEOUT, u); }
+            break;
+        }
+
+        // ---- publish, then wait (warp-parallel) for the earlier tiles that read this tile's rows
+        if (lane == 0) {
+            fence_proxy_async();
+            __threadfence();
+            store_release(a.flags + (size_t)p * a.max_tiles + b, 1);
+        }
+        const int first_reader = a.need[b];
+        const uint64_t t_start = global_ns();
+        for (int bb = first_reader; bb < b && ok; bb += 32) {
+            const int mine = bb + lane;
+            const int32_t* f = a.flags + (size_t)p * a.max_tiles + mine;
+            for (;;) {
+                const bool ready = (mine >= b) || load_acquire(f) != 0;
+                if (__all_sync(0xffffffffu, ready)) break;
+                if (*abort_flag || global_ns() - t_start > kWaitBudgetNs) { ok = false; break; }
+                __nanosleep(32);
             }
         }
-        __syncthreads();
-        if (!s_ok) break;
-        {   // write the tile (destination rows of a tile are contiguous)
-            int rb;
-            char* base = plane_base(a, p, rb);
-            const int j0 = b * a.tile_rows;
-            const int rows = min(a.tile_rows, n - j0);
-            if (rb >= 16) {
-                const int vpr = rb >> 4;
-                const int nv = rows * vpr;
-                uint4* dst = reinterpret_cast<uint4*>(base + (size_t)j0 * rb);
-                for (int e = tid; e < nv; e += kCompactThreads) {
-                    const int r = e / vpr;
-                    if (a.retain_idx[j0 + r] != j0 + r) __stcs(dst + e, reinterpret_cast<const uint4*>(stage)[e]);
-                }
-            } else {
-                for (int r = tid; r < rows; r += kCompactThreads)
-                    if (a.retain_idx[j0 + r] != j0 + r)
-                        reinterpret_cast<int*>(base)[j0 + r] = reinterpret_cast<const int*>(stage)[r];
-            }
+        if (!ok) {
+            if (lane == 0) { atomicExch(&a.ctl->abort, 1); record_status(a.status, DELTAS_ERR_TIMEOUT, u); }
+            break;
         }
-        __syncthreads();                       // the stage is rewritten by the next unit
+
+        // ---- store the tile (destination rows of a tile are contiguous)
+        if (kv) {
+            if (lane == 0) {
+                fence_proxy_async();
+                bulk_store(base + (size_t)js * rb, stage + (size_t)(js - j0) * rb, (uint32_t)nrows * rb);
+                bulk_commit();
+                store_pending = true;
+            }
+        } else {
+            const int* st = reinterpret_cast<const int*>(stage);
+            for (int r = js + lane; r < j_end; r += 32) reinterpret_cast<int*>(base)[r] = st[r - j0];
+            __syncwarp();                                          // the stage is rewritten next
+        }
     }
+    if (lane == 0) {
+        bulk_wait0();                                              // stores complete before exit
+        if (load_pending) mbar_wait(&bar, phase, kWaitBudgetNs);   // abort path: loads land first
+    }
+    __syncwarp();
 }
 
 __global__ void append_kv_kernel(char* k_cache, char* v_cache, int n_kv_planes, int capacity,
@@ -323,12 +343,12 @@ cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, con
 
     const int smem = a.tile_rows * a.row_bytes;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, compact_main_kernel, kCompactThreads, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, compact_main_kernel, 32, smem);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
     const int max_units = a.max_tiles * a.n_planes;
     const int grid = max(1, min(max_units, per_sm * sms));
-    compact_main_kernel<<<grid, kCompactThreads, smem, s>>>(a);
+    compact_main_kernel<<<grid, 32, smem, s>>>(a);
     return cudaGetLastError();
 }
 
