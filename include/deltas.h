@@ -152,9 +152,9 @@ DELTAS_API deltas_status deltas_state_drift(const deltas_gdn_desc* desc, const f
 /*   Delta S = (1/L) sum_l sqrt(sum_h partials[l][h][0]) / sqrt(sum_h partials[l][h][1])       */
 /* The per-layer norm runs over all heads of the layer.  A layer whose denominator is 0        */
 /* contributes 0 when its numerator is 0 and +infinity otherwise.  The reduction order is       */
-/* fixed (deterministic); sums are formed in double, each layer's square roots and quotient in  */
-/* float (correctly rounded), and the score is stored as float to chunk_scores[chunk_id]        */
-/* (device memory, [>= chunk_id + 1] floats).                                                   */
+/* fixed (deterministic): per-layer sums over the heads in float (pairwise tree), each layer's   */
+/* square roots and quotient in float (correctly rounded), the mean over layers in double; the  */
+/* score is stored as float to chunk_scores[chunk_id] (device memory, [>= chunk_id + 1]).       */
 /* ------------------------------------------------------------------------------------------ */
 DELTAS_API deltas_status deltas_score_chunks(int32_t num_layers, int32_t num_v_heads,
                                   const float* drift_partials, int32_t chunk_id,

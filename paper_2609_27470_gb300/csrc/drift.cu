@@ -49,8 +49,10 @@ state_drift_kernel(int n_elem4, const float4* __restrict__ sb, const float4* __r
 
 constexpr int kScoreThreads = 1024;
 
-// One warp per layer (layers strided over the 32 warps): lane-strided double sums over the
-// heads, a fixed xor tree, the per-layer ratio; then warp 0 adds the layer terms in layer order.
+// One warp per layer (layers strided over the 32 warps): lane-strided float sums over the heads and
+// a fixed xor tree (pairwise: a few ulp of float), the layer's ratio in float on lane 0, then
+// warp 0 adds the layer terms in layer order in double.  (The FP64 pipe is slow on this part, so
+// double arithmetic is kept to one addition per layer.)
 __global__ void __launch_bounds__(kScoreThreads)
 score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk_id,
                     float* __restrict__ scores)
@@ -59,23 +61,20 @@ score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     double acc = 0.0;
     for (int l = warp; l < L; l += kScoreThreads / 32) {
-        double num = 0.0, den = 0.0;
+        float num = 0.f, den = 0.f;
         for (int h = lane; h < Hv; h += 32) {
-            num += (double)partials[((size_t)l * Hv + h) * 2 + 0];
-            den += (double)partials[((size_t)l * Hv + h) * 2 + 1];
+            num += partials[((size_t)l * Hv + h) * 2 + 0];
+            den += partials[((size_t)l * Hv + h) * 2 + 1];
         }
 #pragma unroll
         for (int m = 16; m >= 1; m >>= 1) {
             num += __shfl_xor_sync(0xffffffffu, num, m);
             den += __shfl_xor_sync(0xffffffffu, den, m);
         }
-        // The square roots and the quotient are taken in float (correctly rounded, a few ulp of
-        // float in all): double square roots and divisions run on the slow FP64 pipe.
         if (lane == 0) {
-            const float nf = (float)num, df = (float)den;
             double term;
-            if (den > 0.0) term = (double)(sqrtf(nf) / sqrtf(df));
-            else term = (num > 0.0) ? (double)INFINITY : 0.0;
+            if (den > 0.f) term = (double)(sqrtf(num) / sqrtf(den));
+            else term = (num > 0.f) ? (double)INFINITY : 0.0;
             acc += term;   // layers l, l + 32, ... in increasing order
         }
     }

@@ -61,7 +61,8 @@ constexpr int kCtlWarp = 16;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t TM_S = 0, TM_S0HI = 128, TM_S0LO = 192, TM_X = 256, TM_U = 320, TM_KK = 384;  // K K^T: 2 x 64
 
-constexpr int FA_S = 65;               // fp32 row stride of A (odd: one row per lane, no bank conflicts)
+constexpr int FA_S = 68;               // fp32 row stride of A: 16-byte rows; a 16-byte access by 8 threads
+                                       // of 8 consecutive rows hits 8 distinct bank groups
 constexpr int FX_S = 68;               // fp32 row stride of X^-1 (16-byte aligned rows for float4 reads)
 
 // shared-memory map (bytes from a 1024-aligned base)
@@ -73,8 +74,10 @@ constexpr uint32_t SM_FA = 163840;                // fp32 [64][FA_S]
 constexpr uint32_t SM_FX = SM_FA + 64 * FA_S * 4; // fp32 [64][FX_S]
 constexpr uint32_t SM_TMP = SM_FX + 64 * FX_S * 4;// fp32 [32][33]
 constexpr uint32_t SM_CG = SM_TMP + 32 * 33 * 4;  // chain tile constants, 3 buffers x (-gamma[64], del[64], gamma_C)
-constexpr uint32_t SM_TG = SM_CG + 3 * 132 * 4;   // T-builder constants: G2[64], beta[64], row[64], col[64], flag
-constexpr uint32_t SM_BYTES = SM_TG + 260 * 4;
+constexpr uint32_t SM_TG = SM_CG + 3 * 132 * 4;   // T-builder constants, 2 buffers (tile parity) x
+                                                  // (G2[64], beta[64], row[64], col[64], flag)
+constexpr uint32_t kTgFloats = 260;
+constexpr uint32_t SM_BYTES = SM_TG + 2 * kTgFloats * 4;
 constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
 static_assert(SM_TG % 16 == 0, "beta must be 16-byte aligned");
 static_assert(kSmemAlloc <= 232448, "shared memory budget");
@@ -357,16 +360,11 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         float* fA = reinterpret_cast<float*>(sm + SM_FA);
         float* fX = reinterpret_cast<float*>(sm + SM_FX);
         float* fT = reinterpret_cast<float*>(sm + SM_TMP);
-        float* sG2 = reinterpret_cast<float*>(sm + SM_TG);   // G * log2(e)
-        float* sBeta = sG2 + 64;
-        float* sRow = sG2 + 128;                             // beta_t 2^(G2_t - ref)
-        float* sCol = sG2 + 192;                             // 2^(ref - G2_i)
-        int* sFactored = reinterpret_cast<int*>(sG2 + 256);
         float* cg = reinterpret_cast<float*>(sm + SM_CG);
-        float pg[2] = {0.f, 0.f}, pb[2] = {0.f, 0.f};     // g, beta of the next tile (warp 8)
+        float pg[2] = {0.f, 0.f}, pb[2] = {0.f, 0.f};     // g, beta of the next tile (warp 15)
         TileCursor gc;                                     // next tile whose g, beta to load
         gc.init(a);
-        auto load_gb = [&]() {                             // g, beta of the next tile (warp 8)
+        auto load_gb = [&]() {                             // g, beta of the next tile (warp 15)
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 const int t = gc.jt * kC + 2 * lane + e;
@@ -376,49 +374,64 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             }
             gc.next(n, a);
         };
-        if (tw == 0) load_gb();
+        // Decay constants of tile jj from the loaded g, beta (warp 15, one tile ahead of the
+        // T build that uses them): the chain's -gamma, exp(G_C - G), gamma_C, and the T builders'
+        // G2, beta, row and column factors (buffer jj & 1).
+        auto tile_constants = [&](int jj) {
+            float* tg = reinterpret_cast<float*>(sm + SM_TG) + (jj & 1) * kTgFloats;
+            float gv[2], bv[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) { gv[e] = pg[e]; bv[e] = pb[e]; }
+            float incl = gv[0] + gv[1];
+#pragma unroll
+            for (int m = 1; m < 32; m <<= 1) {
+                const float y = __shfl_up_sync(0xffffffffu, incl, m);
+                if (lane >= m) incl += y;
+            }
+            const float G0 = incl - gv[1], G1 = incl;
+            const float GC = __shfl_sync(0xffffffffu, incl, 31);
+            // the chain's constants of tile jj (3 buffers: the chain is at most two tiles behind
+            // the T builders' current tile)
+            float* cgam = cg + (jj % 3) * 132;
+            cgam[2 * lane] = -expf(G0); cgam[2 * lane + 1] = -expf(G1);
+            cgam[64 + 2 * lane] = expf(GC - G0); cgam[64 + 2 * lane + 1] = expf(GC - G1);
+            if (lane == 0) cgam[128] = expf(GC);
+            const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
+            float lo2 = fminf(g20, g21), hi2 = fmaxf(g20, g21);
+#pragma unroll
+            for (int m = 16; m >= 1; m >>= 1) {
+                lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, m));
+                hi2 = fmaxf(hi2, __shfl_xor_sync(0xffffffffu, hi2, m));
+            }
+            // exp(G_t - G_i) = row_t * col_i with the reference in the middle of the tile's range
+            // of G; both factors stay within 2^+-126 when that range spans at most 250 powers of
+            // two, otherwise the exponent is taken per entry.
+            const float ref = 0.5f * (lo2 + hi2);
+            tg[2 * lane] = g20; tg[2 * lane + 1] = g21;
+            tg[64 + 2 * lane] = bv[0]; tg[64 + 2 * lane + 1] = bv[1];
+            tg[128 + 2 * lane] = bv[0] * fast_exp2(g20 - ref); tg[128 + 2 * lane + 1] = bv[1] * fast_exp2(g21 - ref);
+            tg[192 + 2 * lane] = fast_exp2(ref - g20); tg[192 + 2 * lane + 1] = fast_exp2(ref - g21);
+            if (lane == 0) reinterpret_cast<int*>(tg)[256] = (hi2 - lo2) <= 250.f;
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&mb_cready[jj % 3]);
+        };
+        // The strictly upper 16 x 16 blocks of X are never written; zeros there let every level
+        // run fixed-length (unrolled) loops over the triangular factors.
+        for (int e = tt; e < 64 * FX_S; e += kTB) fX[e] = 0.f;
+        if (tw == 7 && NJ > 0) {
+            load_gb();
+            tile_constants(0);
+            if (NJ > 1) load_gb();
+        }
         for (int j = 0; j < NJ; ++j) {                     // j: global tile index
             if (named_sync_or(3, kTB, *abort_flag)) break;
-            if (tw == 0) {                                 // per-tile decay constants
-                float gv[2], bv[2];
-#pragma unroll
-                for (int e = 0; e < 2; ++e) { gv[e] = pg[e]; bv[e] = pb[e]; }
-                if (j + 1 < NJ) load_gb();                 // prefetch the next tile's g, beta
-                float incl = gv[0] + gv[1];
-#pragma unroll
-                for (int m = 1; m < 32; m <<= 1) {
-                    const float y = __shfl_up_sync(0xffffffffu, incl, m);
-                    if (lane >= m) incl += y;
-                }
-                const float G0 = incl - gv[1], G1 = incl;
-                const float GC = __shfl_sync(0xffffffffu, incl, 31);
-                // the chain's constants of tile j: -gamma, exp(G_C - G), gamma_C (3 buffers: the
-                // chain is at most two tiles behind)
-                float* cgam = cg + (j % 3) * 132;
-                cgam[2 * lane] = -expf(G0); cgam[2 * lane + 1] = -expf(G1);
-                cgam[64 + 2 * lane] = expf(GC - G0); cgam[64 + 2 * lane + 1] = expf(GC - G1);
-                if (lane == 0) cgam[128] = expf(GC);
-                const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
-                float lo2 = fminf(g20, g21), hi2 = fmaxf(g20, g21);
-#pragma unroll
-                for (int m = 16; m >= 1; m >>= 1) {
-                    lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, m));
-                    hi2 = fmaxf(hi2, __shfl_xor_sync(0xffffffffu, hi2, m));
-                }
-                // exp(G_t - G_i) = row_t * col_i with the reference in the middle of the tile's
-                // range of G; both factors stay within 2^+-126 when that range spans at most 250
-                // powers of two, otherwise the exponent is taken per entry.
-                const float ref = 0.5f * (lo2 + hi2);
-                sG2[2 * lane] = g20; sG2[2 * lane + 1] = g21;
-                sBeta[2 * lane] = bv[0]; sBeta[2 * lane + 1] = bv[1];
-                sRow[2 * lane] = bv[0] * fast_exp2(g20 - ref); sRow[2 * lane + 1] = bv[1] * fast_exp2(g21 - ref);
-                sCol[2 * lane] = fast_exp2(ref - g20); sCol[2 * lane + 1] = fast_exp2(ref - g21);
-                if (lane == 0) *sFactored = (hi2 - lo2) <= 250.f;
-                fence_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&mb_cready[j % 3]);
-            }
-            named_sync(3, kTB);
+            const float* tg = reinterpret_cast<const float*>(sm + SM_TG) + (j & 1) * kTgFloats;
+            const float* sG2 = tg;                         // G * log2(e)
+            const float* sBeta = tg + 64;
+            const float* sRow = tg + 128;                  // beta_t 2^(G2_t - ref)
+            const float* sCol = tg + 192;                  // 2^(ref - G2_i)
+            const int factored = reinterpret_cast<const int*>(tg)[256];
             if (!mbar_wait_or_abort(&mb_kk[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 8);
             tc_fence_after();
             const int q = warp & 3;
@@ -430,7 +443,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 const uint32_t lane_off = (uint32_t)(32 * q) << 16;
                 float kk[32], cf[32];
                 tmem_ld32(tm + lane_off + TM_KK + 64 * (j & 1) + c0, kk);
-                if (*sFactored) {
+                if (factored) {
                     const float rt = sRow[t];
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
@@ -452,7 +465,12 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? bt * fast_exp2(G2t - cf[e]) * kk[e] : 0.f;
                 }
 #pragma unroll
-                for (int e = 0; e < 32; ++e) fA[t * FA_S + c0 + e] = kk[e];
+                for (int e = 0; e < 8; ++e)
+                    *reinterpret_cast<float4*>(fA + t * FA_S + c0 + 4 * e) =
+                        make_float4(kk[4 * e], kk[4 * e + 1], kk[4 * e + 2], kk[4 * e + 3]);
+            } else if (tw == 7 && j + 1 < NJ) {
+                tile_constants(j + 1);                     // the next tile's, off this tile's path
+                if (j + 2 < NJ) load_gb();
             }
             tc_fence_before();
             named_sync(3, kTB);
@@ -464,33 +482,45 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
 #pragma unroll
                 for (int rr = 1; rr < 16; ++rr) {
-                    float sacc = 0.f;
+                    float s0 = 0.f, s1 = 0.f;              // two chains: half the dependent FMAs
 #pragma unroll
-                    for (int c = 0; c < rr; ++c) sacc = fmaf(fA[(o + rr) * FA_S + o + c], x[c], sacc);
-                    if (rr > jc) x[rr] = -sacc;
+                    for (int c = 0; c < rr; c += 4) {
+                        const float4 av = *reinterpret_cast<const float4*>(fA + (o + rr) * FA_S + o + c);
+                        s0 = fmaf(av.x, x[c], s0);
+                        if (c + 1 < rr) s1 = fmaf(av.y, x[c + 1], s1);
+                        if (c + 2 < rr) s0 = fmaf(av.z, x[c + 2], s0);
+                        if (c + 3 < rr) s1 = fmaf(av.w, x[c + 3], s1);
+                    }
+                    if (rr > jc) x[rr] = -(s0 + s1);
                 }
 #pragma unroll
                 for (int rr = 0; rr < 16; ++rr) fX[(o + rr) * FX_S + o + jc] = x[rr];
             }
             named_sync(3, kTB);
             // level 1: X[2p+1][2p] = -X[2p+1][2p+1] (A[2p+1][2p] X[2p][2p]), p = tw >> 2.
-            // Loop bounds follow the zero pattern of the triangular factors and are warp-uniform.
+            // Fixed-length loops: the zeros of the triangular factors are stored.
             {
                 const int p = tw >> 2, cg = 4 * (tw & 3);
                 const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
                 const int lo16 = lane & 15, sub = 2 * (lane >> 4);
                 float acc0 = 0.f, acc1 = 0.f;             // tmp1[p][lo16][cg + sub + {0,1}]
-                for (int k = cg; k < 16; ++k) {
-                    const float av = fA[(ro + lo16) * FA_S + co + k];
-                    const float2 xv = *reinterpret_cast<const float2*>(fX + (co + k) * FX_S + co + cg + sub);
-                    acc0 = fmaf(av, xv.x, acc0);
-                    acc1 = fmaf(av, xv.y, acc1);
+#pragma unroll
+                for (int k4 = 0; k4 < 16; k4 += 4) {
+                    const float4 a4 = *reinterpret_cast<const float4*>(fA + (ro + lo16) * FA_S + co + k4);
+                    const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+                    for (int kk4 = 0; kk4 < 4; ++kk4) {
+                        const float2 xv = *reinterpret_cast<const float2*>(fX + (co + k4 + kk4) * FX_S + co + cg + sub);
+                        acc0 = fmaf(av[kk4], xv.x, acc0);
+                        acc1 = fmaf(av[kk4], xv.y, acc1);
+                    }
                 }
                 fT[p * 272 + lo16 * 17 + cg + sub] = acc0;
                 fT[p * 272 + lo16 * 17 + cg + sub + 1] = acc1;
                 named_sync(3, kTB);
                 float o0 = 0.f, o1 = 0.f;                  // rows cg + sub + {0,1}, column lo16
-                for (int k = 0; k <= cg + 3; ++k) {
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
                     const float tv = fT[p * 272 + k * 17 + lo16];
                     o0 = fmaf(fX[(ro + cg + sub) * FX_S + ro + k], tv, o0);
                     o1 = fmaf(fX[(ro + cg + sub + 1) * FX_S + ro + k], tv, o1);
@@ -503,17 +533,23 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             {
                 const int g4 = 4 * tw;
                 float acc[4] = {0.f, 0.f, 0.f, 0.f};       // tmp2[lane][g4..g4+3]
-                for (int k = g4; k < 32; ++k) {
-                    const float av = fA[(32 + lane) * FA_S + k];
-                    const float4 xv = *reinterpret_cast<const float4*>(fX + k * FX_S + g4);
-                    acc[0] = fmaf(av, xv.x, acc[0]); acc[1] = fmaf(av, xv.y, acc[1]);
-                    acc[2] = fmaf(av, xv.z, acc[2]); acc[3] = fmaf(av, xv.w, acc[3]);
+#pragma unroll
+                for (int k4 = 0; k4 < 32; k4 += 4) {
+                    const float4 a4 = *reinterpret_cast<const float4*>(fA + (32 + lane) * FA_S + k4);
+                    const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+                    for (int kk4 = 0; kk4 < 4; ++kk4) {
+                        const float4 xv = *reinterpret_cast<const float4*>(fX + (k4 + kk4) * FX_S + g4);
+                        acc[0] = fmaf(av[kk4], xv.x, acc[0]); acc[1] = fmaf(av[kk4], xv.y, acc[1]);
+                        acc[2] = fmaf(av[kk4], xv.z, acc[2]); acc[3] = fmaf(av[kk4], xv.w, acc[3]);
+                    }
                 }
 #pragma unroll
                 for (int i = 0; i < 4; ++i) fT[lane * 33 + g4 + i] = acc[i];
                 named_sync(3, kTB);
                 float o4[4] = {0.f, 0.f, 0.f, 0.f};        // rows 32+g4..32+g4+3, column lane
-                for (int k = 0; k <= g4 + 3; k += 4) {
+#pragma unroll
+                for (int k = 0; k < 32; k += 4) {
                     const float t0v = fT[(k + 0) * 33 + lane], t1v = fT[(k + 1) * 33 + lane];
                     const float t2v = fT[(k + 2) * 33 + lane], t3v = fT[(k + 3) * 33 + lane];
 #pragma unroll
@@ -641,8 +677,11 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tmem_ld_wait();
                 uint32_t hi[16], lo[16];
 #pragma unroll
-                for (int c = 0; c < 16; ++c)
-                    split2(gam[32 * wg + 2 * c] * xv[2 * c], gam[32 * wg + 2 * c + 1] * xv[2 * c + 1], hi[c], lo[c]);
+                for (int c4 = 0; c4 < 8; ++c4) {
+                    const float4 g4 = *reinterpret_cast<const float4*>(gam + 32 * wg + 4 * c4);
+                    split2(g4.x * xv[4 * c4], g4.y * xv[4 * c4 + 1], hi[2 * c4], lo[2 * c4]);
+                    split2(g4.z * xv[4 * c4 + 2], g4.w * xv[4 * c4 + 3], hi[2 * c4 + 1], lo[2 * c4 + 1]);
+                }
                 tmem_st16(tm + lane_off + TM_X + 32 * wg, hi);
                 tmem_st16(tm + lane_off + TM_X + 32 * wg + 16, lo);
                 tmem_st_wait();
@@ -659,8 +698,11 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tmem_ld_wait();
                 uint32_t hi[16], lo[16];
 #pragma unroll
-                for (int c = 0; c < 16; ++c)
-                    split2(uv[2 * c] * del[32 * wg + 2 * c], uv[2 * c + 1] * del[32 * wg + 2 * c + 1], hi[c], lo[c]);
+                for (int c4 = 0; c4 < 8; ++c4) {
+                    const float4 d4 = *reinterpret_cast<const float4*>(del + 32 * wg + 4 * c4);
+                    split2(uv[4 * c4] * d4.x, uv[4 * c4 + 1] * d4.y, hi[2 * c4], lo[2 * c4]);
+                    split2(uv[4 * c4 + 2] * d4.z, uv[4 * c4 + 3] * d4.w, hi[2 * c4 + 1], lo[2 * c4 + 1]);
+                }
                 tmem_st16(tm + lane_off + TM_U + 32 * wg, hi);
                 tmem_st16(tm + lane_off + TM_U + 32 * wg + 16, lo);
                 tmem_st_wait();

@@ -158,14 +158,29 @@ struct SelArgs {
 constexpr int kSmallRuns = 512;   // runs held in shared memory and ranked directly
 
 // Slot segments: warp w owns whole 32-slot groups [seg_lo, seg_hi) of the candidate range, so
-// every load of tok_chunk is one coalesced 128-byte line.  Returns the run-start flag of slot
-// i = base + lane (false outside the segment).
-__device__ __forceinline__ bool run_start_flag(const int32_t* tok_chunk, int lo, int seg_hi, int i, int& c) {
-    const bool valid = i < seg_hi;
-    c = valid ? tok_chunk[i] : INT_MIN;
-    int prev = __shfl_up_sync(0xffffffffu, c, 1);
-    if ((threadIdx.x & 31) == 0) prev = (valid && i > lo) ? tok_chunk[i - 1] : INT_MIN;
-    return valid && (i == lo || c != prev);
+// every load of tok_chunk is one coalesced 128-byte line.  A warp loads kBatch groups at once
+// (the loads are independent, so their latencies overlap), then walks them.
+constexpr int kBatch = 8;
+struct SlotBatch {
+    int c[kBatch];     // tok_chunk of slot base0 + 32 k + lane (INT_MIN outside the segment)
+    int p[kBatch];     // lane 0: tok_chunk of the slot before its group (INT_MIN at lo)
+};
+
+__device__ __forceinline__ void load_batch(const int32_t* tok_chunk, int lo, int seg_hi, int base0, SlotBatch& b) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int k = 0; k < kBatch; ++k) {
+        const int i = base0 + 32 * k + lane;
+        b.c[k] = i < seg_hi ? tok_chunk[i] : INT_MIN;
+        b.p[k] = (lane == 0 && i < seg_hi && i > lo) ? tok_chunk[i - 1] : INT_MIN;
+    }
+}
+
+// Run-start flag of slot i = base0 + 32 k + lane (false outside the segment).
+__device__ __forceinline__ bool batch_start(const SlotBatch& b, int k, int lo, int seg_hi, int i) {
+    int prev = __shfl_up_sync(0xffffffffu, b.c[k], 1);
+    if ((threadIdx.x & 31) == 0) prev = b.p[k];
+    return i < seg_hi && (i == lo || b.c[k] != prev);
 }
 
 __global__ void __launch_bounds__(kSelThreads, 1)
@@ -190,9 +205,13 @@ select_retain_kernel(SelArgs a)
     const int T = a.T;
     if (tid == 0) s_bad = -1;
     __syncthreads();
-    for (int i = tid; i < T; i += kSelThreads) {
-        const int c = a.tok_chunk[i];
-        if (c < 0 || c >= a.n_chunks) atomicMax(&s_bad, i);
+    for (int i0 = tid; i0 < T; i0 += kSelThreads * kBatch) {
+        int cv[kBatch];
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) cv[k] = i0 + k * kSelThreads < T ? a.tok_chunk[i0 + k * kSelThreads] : 0;
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k)
+            if (cv[k] < 0 || cv[k] >= a.n_chunks) atomicMax(&s_bad, i0 + k * kSelThreads);
     }
     __syncthreads();
     if (s_bad >= 0) {
@@ -219,11 +238,16 @@ select_retain_kernel(SelArgs a)
     const int per_warp = ((n_cand + kSelThreads - 1) / kSelThreads) * 32;
     const int seg_lo = min(lo + warp * per_warp, hi), seg_hi = min(seg_lo + per_warp, hi);
     int n_starts = 0, cmin = INT_MAX, cmax = INT_MIN;
-    for (int base = seg_lo; base < seg_hi; base += 32) {
-        int c;
-        const bool st = run_start_flag(a.tok_chunk, lo, seg_hi, base + lane, c);
-        n_starts += __popc(__ballot_sync(0xffffffffu, st));
-        if (base + lane < seg_hi) { cmin = min(cmin, c); cmax = max(cmax, c); }
+    for (int base0 = seg_lo; base0 < seg_hi; base0 += 32 * kBatch) {
+        SlotBatch sb;
+        load_batch(a.tok_chunk, lo, seg_hi, base0, sb);
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) {
+            const int i = base0 + 32 * k + lane;
+            const bool st = batch_start(sb, k, lo, seg_hi, i);
+            n_starts += __popc(__ballot_sync(0xffffffffu, st));
+            if (i < seg_hi) { cmin = min(cmin, sb.c[k]); cmax = max(cmax, sb.c[k]); }
+        }
     }
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1) {
@@ -259,12 +283,17 @@ select_retain_kernel(SelArgs a)
     uint64_t* r_key = small ? s_rkey : a.ws.run_key;
     {
         int running = 0;
-        for (int base = seg_lo; base < seg_hi; base += 32) {
-            int c;
-            const bool st = run_start_flag(a.tok_chunk, lo, seg_hi, base + lane, c);
-            const unsigned bal = __ballot_sync(0xffffffffu, st);
-            if (st) r_start[run_base + running + __popc(bal & lt_mask)] = base + lane;
-            running += __popc(bal);
+        for (int base0 = seg_lo; base0 < seg_hi; base0 += 32 * kBatch) {
+            SlotBatch sb;
+            load_batch(a.tok_chunk, lo, seg_hi, base0, sb);
+#pragma unroll
+            for (int k = 0; k < kBatch; ++k) {
+                const int i = base0 + 32 * k + lane;
+                const bool st = batch_start(sb, k, lo, seg_hi, i);
+                const unsigned bal = __ballot_sync(0xffffffffu, st);
+                if (st) r_start[run_base + running + __popc(bal & lt_mask)] = i;
+                running += __popc(bal);
+            }
         }
     }
     __syncthreads();
@@ -379,19 +408,23 @@ select_retain_kernel(SelArgs a)
     // ---- E. every slot writes itself if it lies in its run's kept prefix
     {
         int running = 0;
-        for (int base = seg_lo; base < seg_hi; base += 32) {
-            int c;
-            const int i = base + lane;
-            const bool st = run_start_flag(a.tok_chunk, lo, seg_hi, i, c);
-            const unsigned bal = __ballot_sync(0xffffffffu, st);
-            if (i < seg_hi) {
-                const int r = run_base + running + __popc(bal & (lt_mask | (1u << lane))) - 1;
-                const int pos = i - r_start[r];
-                const bool keep = pos < r_kept[r];
-                if (keep) a.retain_idx[a.n_s + r_off[r] + pos] = i;
-                if (a.mask) a.mask[i] = keep ? 1 : 0;
+        for (int base0 = seg_lo; base0 < seg_hi; base0 += 32 * kBatch) {
+            SlotBatch sb;
+            load_batch(a.tok_chunk, lo, seg_hi, base0, sb);
+#pragma unroll
+            for (int k = 0; k < kBatch; ++k) {
+                const int i = base0 + 32 * k + lane;
+                const bool st = batch_start(sb, k, lo, seg_hi, i);
+                const unsigned bal = __ballot_sync(0xffffffffu, st);
+                if (i < seg_hi) {
+                    const int r = run_base + running + __popc(bal & (lt_mask | (1u << lane))) - 1;
+                    const int pos = i - r_start[r];
+                    const bool keep = pos < r_kept[r];
+                    if (keep) a.retain_idx[a.n_s + r_off[r] + pos] = i;
+                    if (a.mask) a.mask[i] = keep ? 1 : 0;
+                }
+                running += __popc(bal);
             }
-            running += __popc(bal);
         }
     }
     for (int i = tid; i < a.n_s; i += kSelThreads) {
