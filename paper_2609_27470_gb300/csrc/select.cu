@@ -13,9 +13,11 @@
 //      histogram) finds the run where the span's quota min(q, |span|) runs out -> kept1[run];
 //   D. fill: the same select over all runs' remainders (key re-based at the first unkept slot)
 //      with target R - sum(kept1) -> kept[run];
-//   E. output: scan of kept over runs, every slot writes itself to retain_idx if it lies in its
-//      run's kept prefix; sink and window slots are copied through.
+//   E. output (a second, grid-wide kernel): every slot writes itself to retain_idx if it lies in
+//      its run's kept prefix; sink and window slots are copied through.
 // Nothing is sorted; the cost is a few passes over the slots plus 16 passes over the runs.
+#include <algorithm>
+
 #include "internal.cuh"
 
 namespace deltas {
@@ -26,6 +28,13 @@ constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kMaxSpans = 32;
 
 enum SpanMode : int { kNone = 0, kAll = 1, kSome = 2 };
+
+// Select -> emit handoff, in the workspace's status area after the 16-byte status word.
+struct SelCtl {
+    int emit;           // 1: the eviction path ran and the emit kernel writes the outputs
+    int n_runs;
+};
+constexpr size_t kSelCtlOffset = 64;
 
 struct SelWs {          // workspace arrays, each [cache_len]
     int32_t* run_start;
@@ -152,6 +161,7 @@ struct SelArgs {
     int32_t* n_retained;
     uint8_t* mask;
     int32_t* status;
+    SelCtl* ctl;
     SelWs ws;
 };
 
@@ -203,22 +213,22 @@ select_retain_kernel(SelArgs a)
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int T = a.T;
-    if (tid == 0) s_bad = -1;
+    if (tid == 0) { s_bad = -1; a.ctl->emit = 0; }
     __syncthreads();
-    for (int i0 = tid; i0 < T; i0 += kSelThreads * kBatch) {
-        int cv[kBatch];
+    if (T <= a.M) {                                    // keep everything (after validation)
+        for (int i0 = tid; i0 < T; i0 += kSelThreads * kBatch) {
+            int cv[kBatch];
 #pragma unroll
-        for (int k = 0; k < kBatch; ++k) cv[k] = i0 + k * kSelThreads < T ? a.tok_chunk[i0 + k * kSelThreads] : 0;
+            for (int k = 0; k < kBatch; ++k) cv[k] = i0 + k * kSelThreads < T ? a.tok_chunk[i0 + k * kSelThreads] : 0;
 #pragma unroll
-        for (int k = 0; k < kBatch; ++k)
-            if (cv[k] < 0 || cv[k] >= a.n_chunks) atomicMax(&s_bad, i0 + k * kSelThreads);
-    }
-    __syncthreads();
-    if (s_bad >= 0) {
-        if (tid == 0) { record_status(a.status, DELTAS_ERR_DEVICE_INDEX, s_bad); *a.n_retained = 0; }
-        return;
-    }
-    if (T <= a.M) {
+            for (int k = 0; k < kBatch; ++k)
+                if (cv[k] < 0 || cv[k] >= a.n_chunks) atomicMax(&s_bad, i0 + k * kSelThreads);
+        }
+        __syncthreads();
+        if (s_bad >= 0) {
+            if (tid == 0) { record_status(a.status, DELTAS_ERR_DEVICE_INDEX, s_bad); *a.n_retained = 0; }
+            return;
+        }
         for (int i = tid; i < T; i += kSelThreads) {
             a.retain_idx[i] = i;
             if (a.mask) a.mask[i] = 1;
@@ -246,8 +256,19 @@ select_retain_kernel(SelArgs a)
             const int i = base0 + 32 * k + lane;
             const bool st = batch_start(sb, k, lo, seg_hi, i);
             n_starts += __popc(__ballot_sync(0xffffffffu, st));
-            if (i < seg_hi) { cmin = min(cmin, sb.c[k]); cmax = max(cmax, sb.c[k]); }
+            if (i < seg_hi) {
+                cmin = min(cmin, sb.c[k]); cmax = max(cmax, sb.c[k]);
+                if (sb.c[k] < 0 || sb.c[k] >= a.n_chunks) atomicMax(&s_bad, i);   // validation
+            }
         }
+    }
+    for (int i = tid; i < lo; i += kSelThreads) {       // sink and window slots
+        const int c = a.tok_chunk[i];
+        if (c < 0 || c >= a.n_chunks) atomicMax(&s_bad, i);
+    }
+    for (int i = hi + tid; i < T; i += kSelThreads) {
+        const int c = a.tok_chunk[i];
+        if (c < 0 || c >= a.n_chunks) atomicMax(&s_bad, i);
     }
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1) {
@@ -257,6 +278,10 @@ select_retain_kernel(SelArgs a)
     if (lane == 0) { warp_sums[warp] = n_starts; s_cmin[warp] = cmin; s_cmax[warp] = cmax; }
     if (tid < kMaxSpans) s_span_total[tid] = 0;
     __syncthreads();
+    if (s_bad >= 0) {
+        if (tid == 0) { record_status(a.status, DELTAS_ERR_DEVICE_INDEX, s_bad); *a.n_retained = 0; }
+        return;
+    }
     if (warp == 0) {                                   // exclusive scan of the per-warp run counts
         const int v = warp_sums[lane];
         int incl = v;
@@ -278,8 +303,6 @@ select_retain_kernel(SelArgs a)
     int* r_start = small ? s_rstart : a.ws.run_start;
     int* r_len = small ? s_rlen : a.ws.run_len;
     int* r_span = small ? s_rspan : a.ws.run_span;
-    int* r_kept = small ? s_rkept : a.ws.kept;
-    int* r_off = small ? s_roff : a.ws.out_off;
     uint64_t* r_key = small ? s_rkey : a.ws.run_key;
     {
         int running = 0;
@@ -405,37 +428,47 @@ select_retain_kernel(SelArgs a)
         __syncthreads();
     }
 
-    // ---- E. every slot writes itself if it lies in its run's kept prefix
-    {
-        int running = 0;
-        for (int base0 = seg_lo; base0 < seg_hi; base0 += 32 * kBatch) {
-            SlotBatch sb;
-            load_batch(a.tok_chunk, lo, seg_hi, base0, sb);
-#pragma unroll
-            for (int k = 0; k < kBatch; ++k) {
-                const int i = base0 + 32 * k + lane;
-                const bool st = batch_start(sb, k, lo, seg_hi, i);
-                const unsigned bal = __ballot_sync(0xffffffffu, st);
-                if (i < seg_hi) {
-                    const int r = run_base + running + __popc(bal & (lt_mask | (1u << lane))) - 1;
-                    const int pos = i - r_start[r];
-                    const bool keep = pos < r_kept[r];
-                    if (keep) a.retain_idx[a.n_s + r_off[r] + pos] = i;
-                    if (a.mask) a.mask[i] = keep ? 1 : 0;
-                }
-                running += __popc(bal);
-            }
+    // ---- hand the runs to the emit kernel (E): the shared-memory arrays of the small path go to
+    // the workspace, where the radix path keeps them already
+    if (small) {
+        for (int r = tid; r < n_runs; r += kSelThreads) {
+            a.ws.run_start[r] = s_rstart[r];
+            a.ws.kept[r] = s_rkept[r];
+            a.ws.out_off[r] = s_roff[r];
         }
     }
-    for (int i = tid; i < a.n_s; i += kSelThreads) {
-        a.retain_idx[i] = i;
-        if (a.mask) a.mask[i] = 1;
-    }
-    for (int i = hi + tid; i < T; i += kSelThreads) {
-        a.retain_idx[a.M - a.n_w + (i - hi)] = i;
-        if (a.mask) a.mask[i] = 1;
-    }
+    if (tid == 0) { a.ctl->n_runs = n_runs; a.ctl->emit = 1; }
     if (tid == 0) *a.n_retained = a.M;
+}
+
+// ---- E. every slot writes itself: a candidate slot goes to retain_idx if it lies in its run's
+// kept prefix (its run found by binary search over the run starts); sink and window slots are
+// copied through.  Grid-wide, one slot per thread.
+__global__ void __launch_bounds__(256)
+select_emit_kernel(SelArgs a)
+{
+    if (!a.ctl->emit) return;
+    const int n_runs = a.ctl->n_runs;
+    const int T = a.T, lo = a.n_s, hi = T - a.n_w;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
+        if (i < lo) {
+            a.retain_idx[i] = i;
+            if (a.mask) a.mask[i] = 1;
+        } else if (i >= hi) {
+            a.retain_idx[a.M - a.n_w + (i - hi)] = i;
+            if (a.mask) a.mask[i] = 1;
+        } else {
+            int l = 0, h = n_runs - 1;                     // last run with start <= i
+            while (l < h) {
+                const int m = (l + h + 1) >> 1;
+                if (a.ws.run_start[m] <= i) l = m; else h = m - 1;
+            }
+            const int pos = i - a.ws.run_start[l];
+            const bool keep = pos < a.ws.kept[l];
+            if (keep) a.retain_idx[a.n_s + a.ws.out_off[l] + pos] = i;
+            if (a.mask) a.mask[i] = keep ? 1 : 0;
+        }
+    }
 }
 
 }  // namespace
@@ -455,8 +488,14 @@ cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_
     a.T = cache_len; a.n_chunks = num_chunks;
     a.tok_chunk = tok_chunk; a.scores = scores; a.retain_idx = retain_idx;
     a.n_retained = n_retained; a.mask = mask; a.status = status;
+    a.ctl = reinterpret_cast<SelCtl*>(static_cast<char*>(ws) + kSelCtlOffset);
     a.ws = carve(ws, cache_len);
     select_retain_kernel<<<1, kSelThreads, 0, s>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int sms = device_sm_count();
+    const int blocks = std::max(1, std::min((cache_len + 255) / 256, 2 * sms));
+    select_emit_kernel<<<blocks, 256, 0, s>>>(a);
     return cudaGetLastError();
 }
 
