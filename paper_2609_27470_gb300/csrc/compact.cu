@@ -256,26 +256,45 @@ compact_main_kernel(CompactArgs a)
     __syncwarp();
 }
 
-__global__ void append_kv_kernel(char* k_cache, char* v_cache, int n_kv_planes, int capacity,
-                                 int row_bytes, int cache_len, const char* k_new, const char* v_new,
-                                 int n_new, int32_t* tok_chunk, int32_t* tok_pos, int chunk_id,
-                                 int first_pos)
+// Append: block b copies kAppendVecs 16-byte vectors of one plane (plane b / blocks_per_plane),
+// each thread kAppendUnroll of them with the loads issued before the stores; the last blocks also
+// write the chunk id and positions of the new rows.
+constexpr int kAppendThreads = 256;
+constexpr int kAppendUnroll = 4;
+constexpr int kAppendVecs = kAppendThreads * kAppendUnroll;
+
+__global__ void __launch_bounds__(kAppendThreads)
+append_kv_kernel(char* k_cache, char* v_cache, int n_kv_planes, int capacity, int row_bytes, int cache_len,
+                 const char* k_new, const char* v_new, int n_new, int32_t* tok_chunk, int32_t* tok_pos,
+                 int chunk_id, int first_pos, int blocks_per_plane)
 {
-    const size_t vec_per_plane = (size_t)n_new * row_bytes / 16;
-    const size_t total = 2 * (size_t)n_kv_planes * vec_per_plane;
-    const size_t stride = (size_t)gridDim.x * blockDim.x;
-    for (size_t e = (size_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += stride) {
-        const size_t pp = e / vec_per_plane, off = e - pp * vec_per_plane;
-        const bool is_v = pp >= (size_t)n_kv_planes;
-        const size_t p = is_v ? pp - n_kv_planes : pp;
-        const uint4* src = reinterpret_cast<const uint4*>((is_v ? v_new : k_new) + p * (size_t)n_new * row_bytes);
-        uint4* dst = reinterpret_cast<uint4*>((is_v ? v_cache : k_cache) +
-                                              (p * (size_t)capacity + cache_len) * row_bytes);
-        dst[off] = __ldcs(src + off);
+    const int b = blockIdx.x;
+    const int n_copy_blocks = 2 * n_kv_planes * blocks_per_plane;
+    if (b >= n_copy_blocks) {                                  // metadata of the new rows
+        for (int i = (b - n_copy_blocks) * kAppendThreads + threadIdx.x; i < n_new;
+             i += (gridDim.x - n_copy_blocks) * kAppendThreads) {
+            tok_chunk[cache_len + i] = chunk_id;
+            tok_pos[cache_len + i] = first_pos + i;
+        }
+        return;
     }
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < (size_t)n_new; i += stride) {
-        tok_chunk[cache_len + i] = chunk_id;
-        tok_pos[cache_len + i] = first_pos + (int)i;
+    const int pp = b / blocks_per_plane, chunk = b - pp * blocks_per_plane;
+    const bool is_v = pp >= n_kv_planes;
+    const size_t p = is_v ? pp - n_kv_planes : pp;
+    const int vec_per_plane = (int)((size_t)n_new * row_bytes / 16);
+    const uint4* src = reinterpret_cast<const uint4*>((is_v ? v_new : k_new) + p * (size_t)n_new * row_bytes);
+    uint4* dst = reinterpret_cast<uint4*>((is_v ? v_cache : k_cache) + (p * (size_t)capacity + cache_len) * row_bytes);
+    const int e0 = chunk * kAppendVecs + threadIdx.x;
+    uint4 v[kAppendUnroll];
+#pragma unroll
+    for (int u = 0; u < kAppendUnroll; ++u) {
+        const int e = e0 + u * kAppendThreads;
+        if (e < vec_per_plane) v[u] = __ldcs(src + e);
+    }
+#pragma unroll
+    for (int u = 0; u < kAppendUnroll; ++u) {
+        const int e = e0 + u * kAppendThreads;
+        if (e < vec_per_plane) dst[e] = v[u];
     }
 }
 
@@ -357,14 +376,16 @@ cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_ne
 {
     if (n_new <= 0) return cudaSuccess;
     const int rb = kv.D * elt_bytes(kv.dtype);
-    const size_t total_vec = 2 * (size_t)kv.Lf * kv.Hkv * n_new * rb / 16;
-    const int sms = device_sm_count();
-    const size_t want = (total_vec + 255) / 256;
-    const int blocks = (int)(want < (size_t)(8 * sms) ? (want > 0 ? want : 1) : (size_t)(8 * sms));
-    append_kv_kernel<<<blocks, 256, 0, s>>>(static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache),
-                                           kv.Lf * kv.Hkv, kv.capacity, rb, cache_len,
-                                           static_cast<const char*>(k_new), static_cast<const char*>(v_new),
-                                           n_new, kv.tok_chunk, kv.tok_pos, chunk_id, first_pos);
+    const size_t vec_per_plane = (size_t)n_new * rb / 16;
+    if (vec_per_plane > (size_t)INT_MAX / 2) return cudaErrorInvalidValue;
+    const int blocks_per_plane = (int)((vec_per_plane + kAppendVecs - 1) / kAppendVecs);
+    const long long copy_blocks = 2ll * kv.Lf * kv.Hkv * blocks_per_plane;
+    const int meta_blocks = (n_new + kAppendThreads - 1) / kAppendThreads;
+    if (copy_blocks + meta_blocks > INT_MAX) return cudaErrorInvalidValue;
+    append_kv_kernel<<<(int)(copy_blocks + meta_blocks), kAppendThreads, 0, s>>>(
+        static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache), kv.Lf * kv.Hkv, kv.capacity, rb, cache_len,
+        static_cast<const char*>(k_new), static_cast<const char*>(v_new), n_new, kv.tok_chunk, kv.tok_pos, chunk_id,
+        first_pos, blocks_per_plane);
     return cudaGetLastError();
 }
 
