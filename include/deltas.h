@@ -178,8 +178,11 @@ DELTAS_API deltas_status deltas_score_chunks(int32_t num_layers, int32_t num_v_h
 /*   n_retained  [1] int32 (device)         out: min(cache_len, M)                              */
 /*   mask        [cache_len] uint8          out: 1 = kept, 0 = evicted; NULL to skip            */
 /* A tok_chunk value outside [0, num_chunks) is reported as DEVICE_INDEX in the status word    */
-/* (outputs are then unspecified).                                                              */
+/* (outputs are then unspecified).  cache_len above DELTAS_SELECT_MAX_CACHE_LEN (2^20) returns   */
+/* UNSUPPORTED.                                                                                 */
 /* ------------------------------------------------------------------------------------------ */
+#define DELTAS_SELECT_MAX_CACHE_LEN 1048576
+
 DELTAS_API size_t deltas_select_retain_workspace_size(int32_t cache_len);
 
 DELTAS_API deltas_status deltas_select_retain(const deltas_policy* policy, int32_t cache_len,

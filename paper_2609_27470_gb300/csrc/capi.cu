@@ -167,6 +167,7 @@ deltas_status deltas_select_retain(const deltas_policy* policy, int32_t cache_le
     if (p.budget_M < 1 || p.n_sink < 0 || p.n_window < 0 || p.n_buckets < 0) return DELTAS_ERR_INVALID_ARGUMENT;
     if ((long long)p.budget_M < (long long)p.n_sink + p.n_window + 1) return DELTAS_ERR_INVALID_ARGUMENT;
     if (p.n_buckets > 32) return DELTAS_ERR_UNSUPPORTED;
+    if (cache_len > DELTAS_SELECT_MAX_CACHE_LEN) return DELTAS_ERR_UNSUPPORTED;
     if (!retain_idx || !n_retained) return DELTAS_ERR_INVALID_ARGUMENT;
     if (cache_len > 0 && (!tok_chunk || !chunk_scores)) return DELTAS_ERR_INVALID_ARGUMENT;
     deltas_status st = check_workspace(workspace, workspace_bytes, deltas_select_retain_workspace_size(cache_len));

@@ -1,4 +1,5 @@
-// Retain selection (Sec. 3.3; Alg. 1 eviction branch) in one 1024-thread CTA.
+// Retain selection (Sec. 3.3; Alg. 1 eviction branch): a grid-wide run scan, a one-CTA decision,
+// a grid-wide emit.
 //
 // Every token of a chunk carries its chunk's score, so candidates form runs: maximal stretches
 // of consecutive slots with the same arrival chunk.  Inside a run the ranking key
@@ -6,13 +7,16 @@
 // the token-level rule "keep the best tokens" keeps a prefix of each run.  The kernel therefore
 // works on runs (tens of them in a streaming cache, at most one per candidate slot in general):
 //
-//   A. runs: per-thread slot segments, block scan of run starts, c_lo / c_hi reduction;
+//   A. runs (a grid-wide kernel): each block validates 1024 slots' chunk ids and writes its run
+//      starts, their count and the min / max candidate chunk; the decision kernel (one 1024-thread
+//      CTA) scans the counts and gathers the starts in slot order;
 //   B. per run: length, temporal span floor((chunk - c_lo) * N / (c_hi - c_lo + 1)), 64-bit key
 //      (total-order score bits << 32 | ~first_slot): larger key = better token;
-//   C. per span: token-weighted radix select (8 passes of 8 bits, one warp scans each span's
-//      histogram) finds the run where the span's quota min(q, |span|) runs out -> kept1[run];
-//   D. fill: the same select over all runs' remainders (key re-based at the first unkept slot)
-//      with target R - sum(kept1) -> kept[run];
+//   C. per span: the run where the span's quota min(q, |span|) runs out -> kept1[run];
+//   D. fill: the same over all runs' remainders (key re-based at the first unkept slot) with
+//      target R - sum(kept1) -> kept[run].  Up to 512 runs (a streaming cache holds about one run
+//      per cached chunk) are ranked directly in shared memory; more go through a token-weighted
+//      radix select (8 passes of 8 bits, one warp scans each span's histogram) on workspace arrays;
 //   E. output (a second, grid-wide kernel): every slot writes itself to retain_idx if it lies in
 //      its run's kept prefix; sink and window slots are copied through.
 // Nothing is sorted; the cost is a few passes over the slots plus 16 passes over the runs.
@@ -167,30 +171,76 @@ struct SelArgs {
 
 constexpr int kSmallRuns = 512;   // runs held in shared memory and ranked directly
 
-// Slot segments: warp w owns whole 32-slot groups [seg_lo, seg_hi) of the candidate range, so
-// every load of tok_chunk is one coalesced 128-byte line.  A warp loads kBatch groups at once
-// (the loads are independent, so their latencies overlap), then walks them.
-constexpr int kBatch = 8;
-struct SlotBatch {
-    int c[kBatch];     // tok_chunk of slot base0 + 32 k + lane (INT_MIN outside the segment)
-    int p[kBatch];     // lane 0: tok_chunk of the slot before its group (INT_MIN at lo)
-};
 
-__device__ __forceinline__ void load_batch(const int32_t* tok_chunk, int lo, int seg_hi, int base0, SlotBatch& b) {
-    const int lane = threadIdx.x & 31;
+// ---- A. runs, grid-wide: block k scans slots [1024 k, 1024 k + 1024) (4 per thread, coalesced):
+// validates their chunk ids, flags the run starts among the candidates [lo, hi), and writes its
+// starts in slot order to run_chunk[1024 k ...] with its count, the min / max candidate chunk and
+// the highest bad slot (or -1) in slot k of run_len / kept / out_off / kept1 (the decision kernel
+// reads these before it reuses the arrays).
+constexpr int kScanThreads = 256;
+constexpr int kScanPer = 4;
+constexpr int kScanSlots = kScanThreads * kScanPer;
+
+__global__ void __launch_bounds__(kScanThreads)
+select_runs_kernel(SelArgs a)
+{
+    __shared__ int s_wsum[kScanThreads / 32];
+    __shared__ int s_min[kScanThreads / 32], s_max[kScanThreads / 32], s_bad[kScanThreads / 32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int T = a.T, lo = a.n_s, hi = T - a.n_w;
+    const int b0 = blockIdx.x * kScanSlots;
+    int c[kScanPer], p[kScanPer];
 #pragma unroll
-    for (int k = 0; k < kBatch; ++k) {
-        const int i = base0 + 32 * k + lane;
-        b.c[k] = i < seg_hi ? tok_chunk[i] : INT_MIN;
-        b.p[k] = (lane == 0 && i < seg_hi && i > lo) ? tok_chunk[i - 1] : INT_MIN;
+    for (int u = 0; u < kScanPer; ++u) {                  // slot b0 + u * 256 + tid
+        const int i = b0 + u * kScanThreads + tid;
+        c[u] = i < T ? a.tok_chunk[i] : 0;
+        p[u] = (i < T && i > lo) ? a.tok_chunk[i - 1] : INT_MIN;
     }
-}
-
-// Run-start flag of slot i = base0 + 32 k + lane (false outside the segment).
-__device__ __forceinline__ bool batch_start(const SlotBatch& b, int k, int lo, int seg_hi, int i) {
-    int prev = __shfl_up_sync(0xffffffffu, b.c[k], 1);
-    if ((threadIdx.x & 31) == 0) prev = b.p[k];
-    return i < seg_hi && (i == lo || b.c[k] != prev);
+    int cmin = INT_MAX, cmax = INT_MIN, bad = -1, flags = 0;
+#pragma unroll
+    for (int u = 0; u < kScanPer; ++u) {
+        const int i = b0 + u * kScanThreads + tid;
+        if (i >= T) continue;
+        if (c[u] < 0 || c[u] >= a.n_chunks) bad = i;
+        if (i >= lo && i < hi) {
+            cmin = min(cmin, c[u]); cmax = max(cmax, c[u]);
+            if (i == lo || c[u] != p[u]) flags |= 1 << u;
+        }
+    }
+    // starts in slot order: group u of 256 slots before group u + 1; inside a group by thread
+    int rank_base = 0;
+    for (int u = 0; u < kScanPer; ++u) {
+        const bool f = (flags >> u) & 1;
+        const unsigned bal = __ballot_sync(0xffffffffu, f);
+        if (lane == 0) s_wsum[warp] = __popc(bal);
+        __syncthreads();
+        int before = 0, total = 0;
+        for (int w = 0; w < kScanThreads / 32; ++w) {
+            const int v = s_wsum[w];
+            before += w < warp ? v : 0;
+            total += v;
+        }
+        if (f) a.ws.run_chunk[b0 + rank_base + before + __popc(bal & ((1u << lane) - 1u))] = b0 + u * kScanThreads + tid;
+        rank_base += total;
+        __syncthreads();
+    }
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+        cmin = min(cmin, __shfl_xor_sync(0xffffffffu, cmin, m));
+        cmax = max(cmax, __shfl_xor_sync(0xffffffffu, cmax, m));
+        bad = max(bad, __shfl_xor_sync(0xffffffffu, bad, m));
+    }
+    if (lane == 0) { s_min[warp] = cmin; s_max[warp] = cmax; s_bad[warp] = bad; }
+    __syncthreads();
+    if (tid == 0) {
+        for (int w = 1; w < kScanThreads / 32; ++w) {
+            cmin = min(cmin, s_min[w]); cmax = max(cmax, s_max[w]); bad = max(bad, s_bad[w]);
+        }
+        a.ws.run_len[blockIdx.x] = rank_base;
+        a.ws.kept[blockIdx.x] = cmin;
+        a.ws.out_off[blockIdx.x] = cmax;
+        a.ws.kept1[blockIdx.x] = bad;
+    }
 }
 
 __global__ void __launch_bounds__(kSelThreads, 1)
@@ -213,22 +263,21 @@ select_retain_kernel(SelArgs a)
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int T = a.T;
+    const int n_blocks = (T + kScanSlots - 1) / kScanSlots;
+    // per-block results of the run scan (read before the arrays are reused below)
+    int b_cnt = 0, b_min = INT_MAX, b_max = INT_MIN, b_bad = -1;
+    for (int k = tid; k < n_blocks; k += kSelThreads) {   // n_blocks <= 1024 for T <= 1M slots
+        b_cnt = a.ws.run_len[k]; b_min = a.ws.kept[k]; b_max = a.ws.out_off[k]; b_bad = a.ws.kept1[k];
+    }
     if (tid == 0) { s_bad = -1; a.ctl->emit = 0; }
     __syncthreads();
-    if (T <= a.M) {                                    // keep everything (after validation)
-        for (int i0 = tid; i0 < T; i0 += kSelThreads * kBatch) {
-            int cv[kBatch];
-#pragma unroll
-            for (int k = 0; k < kBatch; ++k) cv[k] = i0 + k * kSelThreads < T ? a.tok_chunk[i0 + k * kSelThreads] : 0;
-#pragma unroll
-            for (int k = 0; k < kBatch; ++k)
-                if (cv[k] < 0 || cv[k] >= a.n_chunks) atomicMax(&s_bad, i0 + k * kSelThreads);
-        }
-        __syncthreads();
-        if (s_bad >= 0) {
-            if (tid == 0) { record_status(a.status, DELTAS_ERR_DEVICE_INDEX, s_bad); *a.n_retained = 0; }
-            return;
-        }
+    if (b_bad >= 0) atomicMax(&s_bad, b_bad);
+    __syncthreads();
+    if (s_bad >= 0) {
+        if (tid == 0) { record_status(a.status, DELTAS_ERR_DEVICE_INDEX, s_bad); *a.n_retained = 0; }
+        return;
+    }
+    if (T <= a.M) {                                    // keep everything
         for (int i = tid; i < T; i += kSelThreads) {
             a.retain_idx[i] = i;
             if (a.mask) a.mask[i] = 1;
@@ -238,64 +287,22 @@ select_retain_kernel(SelArgs a)
     }
 
     const int N = a.N < 1 ? 1 : a.N;
-    const int lo = a.n_s, hi = T - a.n_w;
-    const int n_cand = hi - lo;
+    const int hi = T - a.n_w;
     const int R = a.M - a.n_s - a.n_w;
     const int quota = R / N;
-    const unsigned lt_mask = (1u << lane) - 1u;
 
-    // ---- A. runs over the candidate slots (warp segments of whole 32-slot groups)
-    const int per_warp = ((n_cand + kSelThreads - 1) / kSelThreads) * 32;
-    const int seg_lo = min(lo + warp * per_warp, hi), seg_hi = min(seg_lo + per_warp, hi);
-    int n_starts = 0, cmin = INT_MAX, cmax = INT_MIN;
-    for (int base0 = seg_lo; base0 < seg_hi; base0 += 32 * kBatch) {
-        SlotBatch sb;
-        load_batch(a.tok_chunk, lo, seg_hi, base0, sb);
-#pragma unroll
-        for (int k = 0; k < kBatch; ++k) {
-            const int i = base0 + 32 * k + lane;
-            const bool st = batch_start(sb, k, lo, seg_hi, i);
-            n_starts += __popc(__ballot_sync(0xffffffffu, st));
-            if (i < seg_hi) {
-                cmin = min(cmin, sb.c[k]); cmax = max(cmax, sb.c[k]);
-                if (sb.c[k] < 0 || sb.c[k] >= a.n_chunks) atomicMax(&s_bad, i);   // validation
-            }
-        }
-    }
-    for (int i = tid; i < lo; i += kSelThreads) {       // sink and window slots
-        const int c = a.tok_chunk[i];
-        if (c < 0 || c >= a.n_chunks) atomicMax(&s_bad, i);
-    }
-    for (int i = hi + tid; i < T; i += kSelThreads) {
-        const int c = a.tok_chunk[i];
-        if (c < 0 || c >= a.n_chunks) atomicMax(&s_bad, i);
-    }
+    // ---- A (gather). block run counts -> offsets; starts copied to r_start in slot order
+    const int b_off = block_exclusive_scan(b_cnt, warp_sums, &s_total);
+    const int n_runs = s_total;
+    int cmin = b_min, cmax = b_max;
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1) {
         cmin = min(cmin, __shfl_xor_sync(0xffffffffu, cmin, m));
         cmax = max(cmax, __shfl_xor_sync(0xffffffffu, cmax, m));
     }
-    if (lane == 0) { warp_sums[warp] = n_starts; s_cmin[warp] = cmin; s_cmax[warp] = cmax; }
+    if (lane == 0) { s_cmin[warp] = cmin; s_cmax[warp] = cmax; }
     if (tid < kMaxSpans) s_span_total[tid] = 0;
     __syncthreads();
-    if (s_bad >= 0) {
-        if (tid == 0) { record_status(a.status, DELTAS_ERR_DEVICE_INDEX, s_bad); *a.n_retained = 0; }
-        return;
-    }
-    if (warp == 0) {                                   // exclusive scan of the per-warp run counts
-        const int v = warp_sums[lane];
-        int incl = v;
-#pragma unroll
-        for (int m = 1; m < 32; m <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, m);
-            if (lane >= m) incl += y;
-        }
-        warp_sums[lane] = incl - v;
-        if (lane == 31) s_total = incl;
-    }
-    __syncthreads();
-    const int run_base = warp_sums[warp];
-    const int n_runs = s_total;
     const bool small = n_runs <= kSmallRuns;
     int c_lo = INT_MAX, c_hi = INT_MIN;
     for (int w = 0; w < kSelWarps; ++w) { c_lo = min(c_lo, s_cmin[w]); c_hi = max(c_hi, s_cmax[w]); }
@@ -305,22 +312,18 @@ select_retain_kernel(SelArgs a)
     int* r_span = small ? s_rspan : a.ws.run_span;
     uint64_t* r_key = small ? s_rkey : a.ws.run_key;
     {
-        int running = 0;
-        for (int base0 = seg_lo; base0 < seg_hi; base0 += 32 * kBatch) {
-            SlotBatch sb;
-            load_batch(a.tok_chunk, lo, seg_hi, base0, sb);
-#pragma unroll
-            for (int k = 0; k < kBatch; ++k) {
-                const int i = base0 + 32 * k + lane;
-                const bool st = batch_start(sb, k, lo, seg_hi, i);
-                const unsigned bal = __ballot_sync(0xffffffffu, st);
-                if (st) r_start[run_base + running + __popc(bal & lt_mask)] = i;
-                running += __popc(bal);
-            }
+        // block counts / offsets through shared memory (the radix path's histogram space, not yet
+        // in use); warp w copies the starts of blocks w, w + 32, ...
+        int* s_bcnt = reinterpret_cast<int*>(s_hist);
+        int* s_boff = s_bcnt + kSelThreads;
+        if (tid < n_blocks) { s_bcnt[tid] = b_cnt; s_boff[tid] = b_off; }
+        __syncthreads();
+        for (int k = warp; k < n_blocks; k += kSelWarps) {
+            const int cnt = s_bcnt[k], off = s_boff[k];
+            for (int i = lane; i < cnt; i += 32) r_start[off + i] = a.ws.run_chunk[k * kScanSlots + i];
         }
     }
     __syncthreads();
-
     // ---- B. per-run length, span and key (larger key = better: score desc, first slot asc)
     for (int r = tid; r < n_runs; r += kSelThreads) {
         const int st = r_start[r];
@@ -490,6 +493,11 @@ cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_
     a.n_retained = n_retained; a.mask = mask; a.status = status;
     a.ctl = reinterpret_cast<SelCtl*>(static_cast<char*>(ws) + kSelCtlOffset);
     a.ws = carve(ws, cache_len);
+    if (cache_len > 0) {
+        select_runs_kernel<<<(cache_len + kScanSlots - 1) / kScanSlots, kScanThreads, 0, s>>>(a);
+        cudaError_t e0 = cudaGetLastError();
+        if (e0 != cudaSuccess) return e0;
+    }
     select_retain_kernel<<<1, kSelThreads, 0, s>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
