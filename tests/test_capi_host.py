@@ -89,6 +89,7 @@ def test_select_argument_checks(L):
     assert call(L.Policy(10, 0, 0, -1)) == L.DELTAS_ERR_INVALID_ARGUMENT
     assert call(L.Policy(10, 0, 0, 1), T=-5) == L.DELTAS_ERR_INVALID_ARGUMENT
     assert call(L.Policy(10, 0, 0, 1), wsb=16) == L.DELTAS_ERR_WORKSPACE
+    assert call(L.Policy(10, 0, 0, 1), T=(1 << 20) + 1) == L.DELTAS_ERR_UNSUPPORTED   # beyond the run scan
 
 
 def test_compact_and_append_argument_checks(L):
