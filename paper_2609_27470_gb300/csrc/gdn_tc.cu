@@ -15,23 +15,35 @@
 // S_before stays in shared memory, so the state is read from and written to HBM exactly once and
 // the drift needs no second pass over it.
 //
-// Precision: every product that touches the state or T uses a two-term bfloat16 split
-// (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)); keys and values are exact in bfloat16.  With
-// X~ = -diag(gamma) X:
-//   X^T  = S0 K^T                   (S0hi + S0lo) K^T                            2 MMA groups
+// Precision.  Keys and values are exact in bfloat16.  The state never leaves fp32 inside the
+// tile loop: TMEM holds S~ with S = sig S~, and X = K S0^T reads S~ straight from TMEM as the A
+// operand of a kind::tf32 product (B = K converted to fp32 in shared memory); the hardware keeps
+// 10 mantissa bits of S~ (a relative error below 2^-10 per element), an error that reaches the
+// state only through the delta correction and decays with it (a CPU simulation of the truncation
+// gives a state error vs fp64 of ~2e-4 at the slowest decay the inputs use, 5e-6 at a typical
+// one).  The other products take a
+// two-term bfloat16 split (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)) of their state-side
+// operand.  With X~ = -diag(gamma) X:
+//   X^T  = S0 K^T                   S~ (tf32, from TMEM) K32^T                    1 MMA group
 //   U^T  = V^T T^T + X~^T T^T        V^T (Thi + Tlo) + X~hi (Thi + Tlo) + X~lo Thi  5 MMA groups
 //   S   += U~^T K                   (U~hi + U~lo) K                              2 MMA groups
 //   K K^T                           exact inputs                                 1 MMA group
-// All products accumulate in fp32 in TMEM; the state error stays ~1e-5 relative to fp64, where
-// one bfloat16 rounding of any of these operands costs ~1e-3.
+// All products accumulate in fp32 in TMEM.
 //
-// Operand placement: the split state-side operands (S0, X~, U~) are A operands read straight from
-// TMEM (written there by tcgen05.st), so the only operands streamed from shared memory are K, V and
-// T.  Shared-memory bandwidth is the resource the tensor pipe and the CUDA-core warps share, and
-// A tiles of 128 rows re-read for every N = 64 product would otherwise saturate it.
+// Deferred decay: the tile decay gamma_C is folded into the scalar sig instead of a pass that
+// multiplies S by gamma_C; X~ is scaled by sig and U~ by 1 / (gamma_C sig) so that MMA_S adds
+// onto S~ directly.  When sig gamma_C would fall below 2^-30 the tile writes gamma_C sig S~ back
+// into TMEM and sig restarts at 1, so 1 / sig stays far from the fp32 range limit.  The head's
+// last tile multiplies by sig when it reads the state out.
+//
+// Operand placement: the state-side operands (S~, X~, U~) are A operands read straight from TMEM
+// (written there by tcgen05.st), so the only operands streamed from shared memory are K, V and T.
+// Shared-memory bandwidth is the resource the tensor pipe and the CUDA-core warps share, and A
+// tiles of 128 rows re-read for every N = 64 product would otherwise saturate it.
 //
 // Warp roles (17 warps):
-//   0-7   state chain: per tile, S0 -> (hi, lo) split, X~ split, U~ split (TMEM <-> registers)
+//   0-7   state chain: per tile, X~ split, U~ split (TMEM <-> registers), next tile's K -> fp32,
+//         and at a head's first / last tile the state load / store and the drift partials
 //   8-15  T builders: K K^T -> A -> (I + A)^-1 by 16 / 32 / 64 blocks -> T (hi, lo), a tile ahead
 //         of the chain (T depends on k, g, beta only)
 //   16    TMEM allocation, TMA loads and every tcgen05.mma (the warp stays converged; elect.sync
@@ -39,9 +51,9 @@
 // Roles hand work to each other through mbarriers only.  Every wait is bounded; a wait that runs
 // out records DELTAS_ERR_TIMEOUT, raises a CTA-wide abort flag so the other roles stop waiting,
 // and the CTA drains its MMAs and loads before freeing TMEM.
-// TMEM (512 columns, M = 128 lanes = d_v): S [0,128), S0 hi / lo packed [128,192) / [192,256),
-// X [256,320) (fp32, then X~ hi / lo packed in place), U [320,384) (likewise U~), K K^T of even /
-// odd tiles [384,448) / [448,512).
+// TMEM (512 columns, M = 128 lanes = d_v): S~ [0,128) (fp32), X [256,320) (fp32, then X~ hi / lo
+// packed in place), U [320,384) (likewise U~), K K^T of even / odd tiles [384,448) / [448,512);
+// [128,256) is unused.
 #include <algorithm>
 
 #include "internal.cuh"
@@ -59,7 +71,7 @@ constexpr int kTB = 256;               // warps 8-15
 constexpr int kThreads = kChain + kTB + 32;
 constexpr int kCtlWarp = 16;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t TM_S = 0, TM_S0HI = 128, TM_S0LO = 192, TM_X = 256, TM_U = 320, TM_KK = 384;  // K K^T: 2 x 64
+constexpr uint32_t TM_S = 0, TM_X = 256, TM_U = 320, TM_KK = 384;  // K K^T: 2 x 64; [128,256) unused
 
 constexpr int FA_S = 68;               // fp32 row stride of A: 16-byte rows; a 16-byte access by 8 threads
                                        // of 8 consecutive rows hits 8 distinct bank groups
@@ -68,9 +80,11 @@ constexpr int FX_S = 68;               // fp32 row stride of X^-1 (16-byte align
 // shared-memory map (bytes from a 1024-aligned base)
 constexpr uint32_t SM_K = 0;                      // 3 x 16 KB: K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
 constexpr uint32_t SM_V = 49152;                  // 16 KB: V tile, same layout
-constexpr uint32_t SM_T = 65536;                  // 2 buffers x (hi 8 KB, lo 8 KB): T, 64 rows (t) x 64 (i)
-constexpr uint32_t SM_SB = 98304;                 // 64 KB: S_before fp32, 4 column blocks x 128 rows x 128 B, SW128
-constexpr uint32_t SM_FA = 163840;                // fp32 [64][FA_S]
+constexpr uint32_t SM_T = 65536;                  // hi 8 KB, lo 8 KB: T, 64 rows (t) x 64 (i)
+constexpr uint32_t SM_K32 = 81920;                // 32 KB: K tile in fp32 (the tf32 B operand of X), 4 column
+                                                  // blocks (32 dims) x 64 rows x 128 B, SW128
+constexpr uint32_t SM_SB = 114688;                // 64 KB: S_before fp32, 4 column blocks x 128 rows x 128 B, SW128
+constexpr uint32_t SM_FA = 180224;                // fp32 [64][FA_S]
 constexpr uint32_t SM_FX = SM_FA + 64 * FA_S * 4; // fp32 [64][FX_S]
 constexpr uint32_t SM_TMP = SM_FX + 64 * FX_S * 4;// fp32 [32][33]
 constexpr uint32_t SM_CG = SM_TMP + 32 * 33 * 4;  // chain tile constants, 3 buffers x (-gamma[64], del[64], gamma_C)
@@ -83,6 +97,7 @@ static_assert(SM_TG % 16 == 0, "beta must be 16-byte aligned");
 static_assert(kSmemAlloc <= 232448, "shared memory budget");
 
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kSigMin = 9.313225746154785e-10f;   // 2^-30: smallest deferred decay of the state
 
 // S_before: the head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each 128 rows x
 // 128 bytes with the 128-byte swizzle (16-byte chunk ^ (row & 7)) that TMA writes and reads; eight
@@ -272,19 +287,18 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             if (ok) { kp[0] = -1; mma_kk(0); }
             for (int j = 0; ok && j < NJ; ++j) {          // j: global tile index
                 const uint8_t* sK = sm + SM_K + (j % 3) * 16384;
-                // S0 split of tile j ready (the chain has seen MMA_S(j-1) complete)
+                // tile j ready for X: the fp32 copy of K(j) is written and, at a head's first tile, the
+                // state is in TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe order)
                 if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
                 tc_fence_after();
-                {   // X^T = S0 K^T   (A: S0 hi / lo from TMEM, 8 columns per K = 16 step)
-                    const uint32_t id = idesc_bf16(128, 64, 0, 0);
+                {   // X~^T = S~ K^T: A = the fp32 state straight from TMEM read as tf32 (8 columns per
+                    // K = 8 step), B = K in fp32
+                    const uint32_t id = idesc_tf32(128, 64);
+                    const uint8_t* k32 = sm + SM_K32;
 #pragma unroll
-                    for (int part = 0; part < 2; ++part) {
-                        const uint32_t a0 = tm + (part == 0 ? TM_S0HI : TM_S0LO);
-#pragma unroll
-                        for (int s = 0; s < 8; ++s) {
-                            const uint64_t bd = sdesc_sw128(smem_u32(sK + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
-                            mma_bf16_ta(tm + TM_X, a0 + 8 * s, bd, id, (part | s) != 0);
-                        }
+                    for (int s = 0; s < 16; ++s) {
+                        const uint64_t bd = sdesc_sw128(smem_u32(k32 + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
+                        mma_tf32_ta(tm + TM_X, tm + TM_S + 8 * s, bd, id, s != 0);
                     }
                     mma_commit(&mb_x);
                 }
@@ -301,7 +315,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 v_pending = -1;
                 tc_fence_after();
                 {   // U^T = V^T T^T + X~^T T^T   (X~ = -diag(gamma) X, hi / lo packed in place in X)
-                    const uint8_t* tb = sm + SM_T + (j & 1) * 16384;
+                    const uint8_t* tb = sm + SM_T;
                     const uint32_t id_v = idesc_bf16(128, 64, 1, 0);      // A = V tile read MN-major
                     const uint32_t id_x = idesc_bf16(128, 64, 0, 0);      // A = X~ from TMEM
 #pragma unroll
@@ -562,10 +576,14 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
 #pragma unroll
                 for (int i = 0; i < 4; ++i) fX[(32 + g4 + i) * FX_S + lane] = -o4[i];
             }
+            // the single T buffer is free once MMA_U(j-1) has read it (it completes long before this
+            // point in steady state; MMA_U(j) cannot complete before T(j) is written, so the
+            // barrier is never two phases ahead)
+            if (j > 0 && !mbar_wait_or_abort(&mb_u, (j - 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 15);
             named_sync(3, kTB);
-            // T = X diag(beta) (upper part zero), split into the B operand buffer of tile j
+            // T = X diag(beta) (upper part zero), split into the B operand buffer
             {
-                uint8_t* tb = sm + SM_T + (j & 1) * 16384;
+                uint8_t* tb = sm + SM_T;
                 uint4 vh[2], vl[2];
                 int tr[2], cr[2];
 #pragma unroll
@@ -615,7 +633,39 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         if (NJ > 0) load_state((int)blockIdx.x);
         TileCursor cc;                                     // the chain's tile
         cc.init(a);
+        // K(jj) bf16 (TMA tile, buffer jj % 3) -> fp32 copy for the tf32 X product.  Called between
+        // MMA_X(jj-1), the last reader of the copy, and the ready signal of tile jj.
+        auto k_to_fp32 = [&](int jj) -> bool {
+            const bool ok = mbar_wait_or_abort(&mb_tk[jj % 3], (jj / 3) & 1, kWaitBudgetNs, abort_flag);
+            const uint8_t* kb = sm + SM_K + (jj % 3) * 16384;
+            uint8_t* k32 = sm + SM_K32;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {                  // 64 rows x 16 chunks of 8 bf16
+                const int e = tid + kChain * u;
+                const int t = e >> 4, cc16 = e & 15, cb = cc16 >> 3, c = cc16 & 7;
+                const uint4 w = *reinterpret_cast<const uint4*>(kb + cb * 8192 + sw128_offset(t, c));
+                const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
+                float f[8];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    f[2 * i] = __uint_as_float(wv[i] << 16);
+                    f[2 * i + 1] = __uint_as_float(wv[i] & 0xFFFF0000u);
+                }
+                // dims 64 cb + 8 c .. + 7: fp32 block 2 cb + c / 4, chunks 2 (c % 4) and 2 (c % 4) + 1
+                uint8_t* rowp = k32 + (2 * cb + (c >> 2)) * 8192;
+                const int q0 = 2 * (c & 3);
+                *reinterpret_cast<float4*>(rowp + sw128_offset(t, q0)) = make_float4(f[0], f[1], f[2], f[3]);
+                *reinterpret_cast<float4*>(rowp + sw128_offset(t, q0 + 1)) = make_float4(f[4], f[5], f[6], f[7]);
+            }
+            fence_async_smem();                            // generic writes -> the tensor core's reads
+            return ok;
+        };
         float den = 0.f;
+        // Deferred decay: TMEM holds S~ with the head's state S = sig * S~.  A tile folds its decay
+        // gamma_C into sig (X is rescaled by sig in the X~ pass, U~ by 1 / (gamma_C sig) in the U~
+        // pass, so MMA_S accumulates onto S~ with no pass over the state); when sig gamma_C would
+        // drop below kSigMin the tile instead writes gamma_C S back into TMEM and sig restarts at 1.
+        float sig = 1.f;
         for (int j = 0; j < NJ; ++j) {                     // j: global tile index
             const int lh = cc.lh, jt = cc.jt;              // head and tile within the head
             float* gam = cg + (j % 3) * 132;               // -gamma (written by the T builders)
@@ -624,14 +674,9 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             if (!mbar_wait_or_abort(&mb_cready[j % 3], (j / 3) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
             const float gC = gam[128];
 
-            // ---- S pass: S0 -> (hi, lo) packed into TMEM; gamma_C S0 -> TMEM (32 columns at a time).
-            // A head's first tile reads S0 from HBM (the previous head's epilogue has already read
-            // its state out of TMEM); later tiles read it from TMEM once MMA_S has landed.
-            if (jt > 0) {
-                if (!mbar_wait_or_abort(&mb_s, (j - 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 9);
-                tc_fence_after();
-            } else {
-                // the head's state in S_before (loaded by TMA, issued at the previous head's end)
+            if (jt == 0) {
+                // ---- a head's first tile: its state (TMA-loaded into S_before at the previous
+                // head's end) into TMEM as S~ with sig = 1, and sum S_before^2
                 if (!mbar_wait_or_abort(&mb_st, (j / n) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 14);
                 ++st_seen;
                 if (j + n < NJ) {                          // the next head's state towards L2
@@ -639,11 +684,9 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     asm volatile("prefetch.L2 [%0];" :: "l"(nxt + 256 * tid) : "memory");
                     asm volatile("prefetch.L2 [%0];" :: "l"(nxt + 256 * tid + 128) : "memory");
                 }
-            }
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                float sv[32];
-                if (jt == 0) {
+                for (int half = 0; half < 2; ++half) {
+                    float sv[32];
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
                         const float4 x = *reinterpret_cast<const float4*>(sbefore + sb_idx(r, 16 * wg + 8 * half + e));
@@ -651,22 +694,17 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     }
 #pragma unroll
                     for (int e = 0; e < 32; ++e) den += sv[e] * sv[e];
-                } else {
-                    tmem_ld32(tm + lane_off + cS + 32 * half, sv);
-                    tmem_ld_wait();
+                    tmem_st32(tm + lane_off + cS + 32 * half, sv);
                 }
-                uint32_t hi[16], lo[16];
-#pragma unroll
-                for (int c = 0; c < 16; ++c) split2(sv[2 * c], sv[2 * c + 1], hi[c], lo[c]);
-                tmem_st16(tm + lane_off + TM_S0HI + 32 * wg + 16 * half, hi);
-                tmem_st16(tm + lane_off + TM_S0LO + 32 * wg + 16 * half, lo);
-#pragma unroll
-                for (int e = 0; e < 32; ++e) sv[e] *= gC;
-                tmem_st32(tm + lane_off + cS + 32 * half, sv);
+                sig = 1.f;
+                if (j == 0 && !k_to_fp32(0)) fail(a.status, abort_flag, 16);
+                tmem_st_wait();
+                tc_fence_before();
+                mbar_arrive(&mb_sready);
             }
-            tmem_st_wait();
-            tc_fence_before();
-            mbar_arrive(&mb_sready);
+            const bool rescale = sig * gC < kSigMin;       // uniform over the CTA
+            const float x_scale = sig;                     // X = sig * (K S~^T)
+            const float u_scale = rescale ? 1.f : 1.f / (gC * sig);
 
             // ---- X~^T = -X^T diag(gamma): (hi, lo) packed in place over this thread's 32 X columns
             if (!mbar_wait_or_abort(&mb_x, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 10);
@@ -678,7 +716,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 uint32_t hi[16], lo[16];
 #pragma unroll
                 for (int c4 = 0; c4 < 8; ++c4) {
-                    const float4 g4 = *reinterpret_cast<const float4*>(gam + 32 * wg + 4 * c4);
+                    float4 g4 = *reinterpret_cast<const float4*>(gam + 32 * wg + 4 * c4);
+                    g4.x *= x_scale; g4.y *= x_scale; g4.z *= x_scale; g4.w *= x_scale;
                     split2(g4.x * xv[4 * c4], g4.y * xv[4 * c4 + 1], hi[2 * c4], lo[2 * c4]);
                     split2(g4.z * xv[4 * c4 + 2], g4.w * xv[4 * c4 + 3], hi[2 * c4 + 1], lo[2 * c4 + 1]);
                 }
@@ -689,7 +728,24 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             tc_fence_before();
             mbar_arrive(&mb_xready);
 
-            // ---- U~^T = U^T diag(exp(G_C - G)): (hi, lo) packed in place over the U columns
+            // ---- while MMA_U runs: rescale S~ if the decay would underflow the deferred scale
+            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and the fp32 copy of K(j+1)
+            if (rescale) {
+                const float f = gC * sig;
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    float sv[32];
+                    tmem_ld32(tm + lane_off + cS + 32 * half, sv);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) sv[e] *= f;
+                    tmem_st32(tm + lane_off + cS + 32 * half, sv);
+                }
+                tmem_st_wait();
+            }
+            if (j + 1 < NJ && !k_to_fp32(j + 1)) fail(a.status, abort_flag, 16);
+
+            // ---- U~^T = U^T diag(exp(G_C - G)) / (gamma_C sig): (hi, lo) packed in place over U
             if (!mbar_wait_or_abort(&mb_u, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 11);
             tc_fence_after();
             {
@@ -699,7 +755,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 uint32_t hi[16], lo[16];
 #pragma unroll
                 for (int c4 = 0; c4 < 8; ++c4) {
-                    const float4 d4 = *reinterpret_cast<const float4*>(del + 32 * wg + 4 * c4);
+                    float4 d4 = *reinterpret_cast<const float4*>(del + 32 * wg + 4 * c4);
+                    d4.x *= u_scale; d4.y *= u_scale; d4.z *= u_scale; d4.w *= u_scale;
                     split2(uv[4 * c4] * d4.x, uv[4 * c4 + 1] * d4.y, hi[2 * c4], lo[2 * c4]);
                     split2(uv[4 * c4 + 2] * d4.z, uv[4 * c4 + 3] * d4.w, hi[2 * c4 + 1], lo[2 * c4 + 1]);
                 }
@@ -709,6 +766,9 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             }
             tc_fence_before();
             mbar_arrive(&mb_uready);
+            sig = rescale ? 1.f : gC * sig;
+            // the next tile of this head may start X as soon as MMA_S(j) is queued
+            if (jt < n - 1) mbar_arrive(&mb_sready);
 
             if (jt == n - 1) {
                 // ---- epilogue of the head: S_after -> HBM, drift partials against S_before
@@ -717,12 +777,14 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tc_fence_after();
                 float num = 0.f;
                 if (ok) {
-                    // S_after replaces S_before in shared memory (each thread its own row) ...
+                    // S_after = sig S~ replaces S_before in shared memory (each thread its own row) ...
 #pragma unroll
                     for (int half = 0; half < 2; ++half) {
                         float sv[32];
                         tmem_ld32(tm + lane_off + cS + 32 * half, sv);
                         tmem_ld_wait();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) sv[e] *= sig;
 #pragma unroll
                         for (int e = 0; e < 8; ++e) {
                             float4* p = reinterpret_cast<float4*>(sbefore + sb_idx(r, 16 * wg + 8 * half + e));
