@@ -88,8 +88,9 @@ const char* deltas_status_string(int32_t s) {
 }
 
 size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens) {
-    (void)desc; (void)n_tokens;
-    return kStatusBytes;
+    if (desc == nullptr || n_tokens <= 0) return kStatusBytes;
+    return kStatusBytes + gdn_tc_scratch_bytes(desc->num_layers, desc->num_v_heads, desc->key_dim,
+                                               desc->value_dim, desc->dtype, n_tokens);
 }
 
 deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, int32_t n_tokens,
@@ -115,6 +116,8 @@ deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, int32_t n_tok
     a.q_scale = desc->q_scale; a.q = q; a.k = k; a.v = v; a.g = g; a.beta = beta;
     a.state = state; a.out = out; a.partials = drift_partials;
     a.status = static_cast<int32_t*>(workspace);
+    a.scratch = static_cast<uint8_t*>(workspace) + kStatusBytes;
+    a.scratch_bytes = workspace_bytes - kStatusBytes;
     if (gdn_tc_supported(a)) return from_cuda(launch_gdn_update_tc(a, as_stream(stream)));
     return from_cuda(launch_gdn_update_simt(a, as_stream(stream)));
 }

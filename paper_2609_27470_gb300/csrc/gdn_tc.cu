@@ -5,55 +5,66 @@
 // and head).  The chunk is processed in tiles of C = 64 tokens with the chunkwise (WY) form of
 // Eq. 1: with G the inclusive cumulative log-decay inside the tile, gamma = exp(G),
 //   A[t][i] = beta_t exp(G_t - G_i) k_t.k_i  (i < t),   T = (I + A)^-1 diag(beta),
-//   X = K S0^T,   U = T (V - diag(gamma) X),
+//   X = K S0^T,   W = V - diag(gamma) X,   U = T W,
 //   S_C = gamma_C S0 + U~^T K,   U~[t] = exp(G_C - G_t) U[t].
 // Padded tokens of a ragged last tile carry k = v = 0, g = 0, beta = 0 and change nothing.
 //
-// One persistent CTA per SM takes (layer, value head) pairs in turn, each for the whole chunk;
-// the tiles of its heads form one pipeline, so a head's loads and T builds start while the
-// previous head drains.  A head's state lives in TMEM from its first tile to its last and
-// S_before stays in shared memory, so the state is read from and written to HBM exactly once and
-// the drift needs no second pass over it.
+// Two kernels.  T and the tile's decay constants depend on k, g and beta only, so the factor
+// kernel builds them for every (layer, value head, tile) at once, several CTAs per SM, and writes
+// one record per tile into the workspace: T~ = diag(exp(G_C - G)) T as the bfloat16 (hi, lo) pair
+// in the swizzled layout the tensor core reads, -gamma and gamma_C.  The update kernel then runs
+// the part that is sequential in the tiles, the state chain, with nothing else on the SM.
+//
+// Update kernel: one persistent CTA per SM takes (layer, value head) pairs in turn; the tiles of
+// its heads form one pipeline.  A head's state lives in TMEM from its first tile to its last
+// (S_before beside it, for the drift), so the state is read from and written to HBM exactly once;
+// the next head's state is loaded into shared memory while the current head runs, and the head
+// boundary swaps the two in one pass that also forms the drift partials.  Per tile:
+//   X region  <- V^T                       (MMA: V tile times an identity matrix, exact)
+//   X region  += S~ K'^T = W^T / ...        (tf32 MMA, K' = K scaled per token by -gamma_t sig)
+//   W pass:   W (x u_scale) -> (hi, lo) in place            (chain)
+//   U region  <- W^T T~^T = U~^T / ...      (MMA)
+//   U~ pass:  -> (hi, lo) in place                          (chain)
+//   S~        += U~^T K                     (MMA)
+// so the chain's passes are a load, a split and a store per element, and the per-token decays
+// ride on K' (formed while the chain converts K to fp32 anyway) and on T~.
 //
 // Precision.  Keys and values are exact in bfloat16.  The state never leaves fp32 inside the
-// tile loop: TMEM holds S~ with S = sig S~, and X = K S0^T reads S~ straight from TMEM as the A
-// operand of a kind::tf32 product (B = K converted to fp32 in shared memory); the hardware keeps
-// 10 mantissa bits of S~ (a relative error below 2^-10 per element), an error that reaches the
-// state only through the delta correction and decays with it (a CPU simulation of the truncation
-// gives a state error vs fp64 of ~2e-4 at the slowest decay the inputs use, 5e-6 at a typical
-// one).  The other products take a
-// two-term bfloat16 split (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)) of their state-side
-// operand.  With X~ = -diag(gamma) X:
-//   X^T  = S0 K^T                   S~ (tf32, from TMEM) K32^T                    1 MMA group
-//   U^T  = V^T T^T + X~^T T^T        V^T (Thi + Tlo) + X~hi (Thi + Tlo) + X~lo Thi  5 MMA groups
+// tile loop: TMEM holds S~ with S = sig S~, and X reads S~ straight from TMEM as the A operand of
+// a kind::tf32 product; the hardware keeps 10 mantissa bits of S~ (a relative error below 2^-10
+// per element) and K' is rounded to tf32 (2^-11), errors that reach the state only through the
+// delta correction and decay with it (a CPU simulation of the truncation gives a state error vs
+// fp64 of ~2e-4 at the slowest decay the inputs use, 5e-6 at a typical one).  The other products
+// take a two-term bfloat16 split (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)) of each fp32
+// operand:
+//   V^T I                           exact                                        1 MMA group
+//   X^T  = S0 K'^T                  S~ (tf32, from TMEM) K'^T (tf32)              1 MMA group
+//   U~^T = W^T T~^T                  Whi T~hi + Whi T~lo + Wlo T~hi                3 MMA groups
 //   S   += U~^T K                   (U~hi + U~lo) K                              2 MMA groups
-//   K K^T                           exact inputs                                 1 MMA group
+//   K K^T (factor kernel)           exact inputs                                 1 MMA group
 // All products accumulate in fp32 in TMEM.
 //
 // Deferred decay: the tile decay gamma_C is folded into the scalar sig instead of a pass that
-// multiplies S by gamma_C; X~ is scaled by sig and U~ by 1 / (gamma_C sig) so that MMA_S adds
-// onto S~ directly.  When sig gamma_C would fall below 2^-30 the tile writes gamma_C sig S~ back
-// into TMEM and sig restarts at 1, so 1 / sig stays far from the fp32 range limit.  The head's
-// last tile multiplies by sig when it reads the state out.
+// multiplies S by gamma_C; K' carries sig and W is scaled by u_scale = 1 / (gamma_C sig) so that
+// MMA_S adds onto S~ directly.  When sig gamma_C would fall below 2^-30 the tile writes
+// gamma_C sig S~ back into TMEM and sig restarts at 1 (u_scale = 1), so 1 / sig stays far from the
+// fp32 range limit.  The head's last tile multiplies by sig when it reads the state out.
 //
-// Operand placement: the state-side operands (S~, X~, U~) are A operands read straight from TMEM
-// (written there by tcgen05.st), so the only operands streamed from shared memory are K, V and T.
-// Shared-memory bandwidth is the resource the tensor pipe and the CUDA-core warps share, and A
-// tiles of 128 rows re-read for every N = 64 product would otherwise saturate it.
-//
-// Warp roles (17 warps):
-//   0-7   state chain: per tile, X~ split, U~ split (TMEM <-> registers), next tile's K -> fp32,
-//         and at a head's first / last tile the state load / store and the drift partials
-//   8-15  T builders: K K^T -> A -> (I + A)^-1 by 16 / 32 / 64 blocks -> T (hi, lo), a tile ahead
-//         of the chain (T depends on k, g, beta only)
-//   16    TMEM allocation, TMA loads and every tcgen05.mma (the warp stays converged; elect.sync
-//         picks the issuing lane)
-// Roles hand work to each other through mbarriers only.  Every wait is bounded; a wait that runs
-// out records DELTAS_ERR_TIMEOUT, raises a CTA-wide abort flag so the other roles stop waiting,
-// and the CTA drains its MMAs and loads before freeing TMEM.
-// TMEM (512 columns, M = 128 lanes = d_v): S~ [0,128) (fp32), X [256,320) (fp32, then X~ hi / lo
-// packed in place), U [320,384) (likewise U~), K K^T of even / odd tiles [384,448) / [448,512);
-// [128,256) is unused.
+// Update-kernel warp roles (19 warps):
+//   0-15  state chain: warp w serves TMEM lanes 32 (w % 4) .. + 31 (state rows) and column group
+//         w / 4; per tile the W and U~ passes (16 token columns each) and the next tile's K'
+//         (two 16-byte chunks each), at head boundaries the state swap and the drift partials
+//   16    TMEM allocation and every tcgen05.mma (one elected lane issues; the warp stays
+//         converged); it also releases the input buffers by tcgen05.commit
+//   17    tile loads: K, V (TMA) and the WY records (bulk copy), as buffers are released
+//   18    state moves: each head's state into the staging buffer, S_after out of it
+// A TMA or bulk copy occupies the issuing thread for a time that grows with its size, so no copy
+// is issued from a role on the chain's critical path.  Roles hand work to each other through
+// mbarriers only.  Every wait is bounded; a wait that runs out records DELTAS_ERR_TIMEOUT, raises
+// a CTA-wide abort flag so the other roles stop waiting, and the CTA drains its MMAs and copies
+// before freeing TMEM.
+// TMEM (512 columns, M = 128 lanes = d_v): S~ [0,128), S_before [128,256), X [256,320) (V^T + X,
+// then W hi / lo packed in place), U [320,384) (likewise U~); [384,512) unused.
 #include <algorithm>
 
 #include "internal.cuh"
@@ -66,73 +77,18 @@ using namespace tc;
 
 constexpr int kC = 64;                 // tokens per tile
 constexpr int kD = 128;                // head dim (d_k = d_v)
-constexpr int kChain = 256;            // warps 0-7
-constexpr int kTB = 256;               // warps 8-15
-constexpr int kThreads = kChain + kTB + 32;
-constexpr int kCtlWarp = 16;
-constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t TM_S = 0, TM_X = 256, TM_U = 320, TM_KK = 384;  // K K^T: 2 x 64; [128,256) unused
-
-constexpr int FA_S = 68;               // fp32 row stride of A: 16-byte rows; a 16-byte access by 8 threads
-                                       // of 8 consecutive rows hits 8 distinct bank groups
-constexpr int FX_S = 68;               // fp32 row stride of X^-1 (16-byte aligned rows for float4 reads)
-
-// shared-memory map (bytes from a 1024-aligned base)
-constexpr uint32_t SM_K = 0;                      // 3 x 16 KB: K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
-constexpr uint32_t SM_V = 49152;                  // 16 KB: V tile, same layout
-constexpr uint32_t SM_T = 65536;                  // hi 8 KB, lo 8 KB: T, 64 rows (t) x 64 (i)
-constexpr uint32_t SM_K32 = 81920;                // 32 KB: K tile in fp32 (the tf32 B operand of X), 4 column
-                                                  // blocks (32 dims) x 64 rows x 128 B, SW128
-constexpr uint32_t SM_SB = 114688;                // 64 KB: S_before fp32, 4 column blocks x 128 rows x 128 B, SW128
-constexpr uint32_t SM_FA = 180224;                // fp32 [64][FA_S]
-constexpr uint32_t SM_FX = SM_FA + 64 * FA_S * 4; // fp32 [64][FX_S]
-constexpr uint32_t SM_TMP = SM_FX + 64 * FX_S * 4;// fp32 [32][33]
-constexpr uint32_t SM_CG = SM_TMP + 32 * 33 * 4;  // chain tile constants, 3 buffers x (-gamma[64], del[64], gamma_C)
-constexpr uint32_t SM_TG = SM_CG + 3 * 132 * 4;   // T-builder constants, 2 buffers (tile parity) x
-                                                  // (G2[64], beta[64], row[64], col[64], flag)
-constexpr uint32_t kTgFloats = 260;
-constexpr uint32_t SM_BYTES = SM_TG + 2 * kTgFloats * 4;
-constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
-static_assert(SM_TG % 16 == 0, "beta must be 16-byte aligned");
-static_assert(kSmemAlloc <= 232448, "shared memory budget");
-
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kSigMin = 9.313225746154785e-10f;   // 2^-30: smallest deferred decay of the state
 
-// S_before: the head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each 128 rows x
-// 128 bytes with the 128-byte swizzle (16-byte chunk ^ (row & 7)) that TMA writes and reads; eight
-// threads reading chunk c of eight consecutive rows (one row per thread) hit distinct banks.
-// Float offset of 16-byte chunk `chunk` (0..31) of row `row`:
-__device__ __forceinline__ int sb_idx(int row, int chunk) {
-    return (chunk >> 3) * 4096 + row * 32 + (((chunk & 7) ^ (row & 7)) << 2);
-}
-
-struct TcArgs {
-    int L, Hk, Hv, T, n_tiles;
-    float* state;
-    float* partials;
-    const float* g;
-    const float* beta;
-    int32_t* status;
-};
-
-// Where a global tile lies: tile jt of head lh = (layer l, value head h), key head kh.  Each role
-// walks the tiles in order; a step costs integer divisions only when it crosses into the next head.
-struct TileCursor {
-    int jt, lh, l, h, kh;
-    __device__ __forceinline__ void set_head(int head, const TcArgs& a) {
-        lh = head; l = head / a.Hv; h = head - l * a.Hv;
-        kh = (int)(((long long)h * a.Hk) / a.Hv);
-    }
-    __device__ __forceinline__ void init(const TcArgs& a) { jt = 0; set_head((int)blockIdx.x, a); }
-    __device__ __forceinline__ void next(int n, const TcArgs& a) {
-        if (++jt == n) { jt = 0; set_head(lh + (int)gridDim.x, a); }
-    }
-};
-
-__device__ __forceinline__ void named_sync(int id, int n) {
-    asm volatile("bar.sync %0, %1;" :: "r"(id), "r"(n) : "memory");
-}
+// ---- WY record of one (layer, value head, tile), written by the factor kernel, read by the update
+// kernel with one bulk copy:
+//   [0, 8192)       T~ hi: bfloat16 [64 t][64 i], 128-byte rows, 128-byte swizzle (K-major B operand)
+//   [8192, 16384)   T~ lo, same layout
+//   [16384, 16656)  float: -gamma[64], gamma_C, 3 unused
+constexpr uint32_t kRecT = 16384;
+constexpr uint32_t kRecConsts = 68;
+constexpr uint32_t kRecBytes = kRecT + kRecConsts * 4;
+static_assert(kRecBytes % 16 == 0, "records are bulk-copied: 16-byte multiples");
 
 // Barrier over `n` threads that also returns the OR of `flag` over them (uniform result).
 __device__ __forceinline__ bool named_sync_or(int id, int n, bool flag) {
@@ -173,6 +129,51 @@ __device__ __forceinline__ void split2(float a, float b, uint32_t& hi, uint32_t&
     lo = pack_bf16x2(a - hf.x, b - hf.y);
 }
 
+// fp32 -> the nearest tf32 value (ties away from zero), in an fp32 container
+__device__ __forceinline__ float round_tf32(float x) {
+    uint32_t y;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(y) : "f"(x));
+    return __uint_as_float(y);
+}
+
+// x -> (hi, lo) tf32 pair with x = hi + lo to about 2^-22 relative
+__device__ __forceinline__ void split_tf32(float x, uint32_t& hi, uint32_t& lo) {
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(lo) : "f"(x - __uint_as_float(hi)));
+}
+
+// D (16 x 8) += A (16 x 8, row) B (8 x 8, col) on the warp's tensor-core path, tf32 in, fp32
+// accumulate.  Fragments: g = lane / 4, t = lane % 4; a = A[g][t], A[g+8][t], A[g][t+4],
+// A[g+8][t+4]; b = B[t][g], B[t+4][g]; d = D[g][2t], D[g][2t+1], D[g+8][2t], D[g+8][2t+1].
+__device__ __forceinline__ void mma_m16n8k8_tf32(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                 "{%0,%1,%2,%3};"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+// D (16 x 8) += A B over K = 8 k-steps of 8, fp32-accurate: each operand split into a tf32 pair
+// and the three products hi*hi + hi*lo + lo*hi accumulated (small terms first).  A(r, k) and
+// B(k, c) read shared memory (r < 16, k < 8 ksteps, c < 8).
+template <int KSTEPS, typename FA, typename FB>
+__device__ __forceinline__ void mma_3xtf32(float (&d)[4], FA A, FB B, int lane) {
+    const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+    for (int ks = 0; ks < KSTEPS; ++ks) {
+        const int k0 = 8 * ks;
+        uint32_t ah[4], al[4], bh[2], bl[2];
+        split_tf32(A(g, k0 + t), ah[0], al[0]);
+        split_tf32(A(g + 8, k0 + t), ah[1], al[1]);
+        split_tf32(A(g, k0 + t + 4), ah[2], al[2]);
+        split_tf32(A(g + 8, k0 + t + 4), ah[3], al[3]);
+        split_tf32(B(k0 + t, g), bh[0], bl[0]);
+        split_tf32(B(k0 + t + 4, g), bh[1], bl[1]);
+        mma_m16n8k8_tf32(d, al, bh);
+        mma_m16n8k8_tf32(d, ah, bl);
+        mma_m16n8k8_tf32(d, ah, bh);
+    }
+}
+
 // 2^x with the hardware approximation (relative error about 2^-22)
 __device__ __forceinline__ float fast_exp2(float x) {
     float y;
@@ -193,403 +194,291 @@ __device__ __forceinline__ void fail(int32_t* status, volatile int* abort, int w
     *abort = 1;
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
-gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                     const __grid_constant__ CUtensorMap smap, TcArgs a)
+// shared-memory descriptor advanced by `bytes` (the start address field counts 16-byte units)
+__device__ __forceinline__ uint64_t dadd(uint64_t desc, uint32_t bytes) { return desc + (uint64_t)(bytes >> 4); }
+
+// =============================================================================================
+// Factor kernel: T~ = diag(exp(G_C - G)) (I + A)^-1 diag(beta) and the decay constants of every tile
+// =============================================================================================
+constexpr int kWyThreads = 256;
+constexpr int kWyCtasPerSm = 3;
+constexpr uint32_t kWyTmemCols = 64;
+constexpr int FA_S = 68;               // fp32 row stride of A: 16-byte rows; a 16-byte access by 8 threads
+                                       // of 8 consecutive rows hits 8 distinct bank groups
+constexpr int FX_S = 68;               // fp32 row stride of X = (I + A)^-1 (16-byte aligned rows)
+// shared-memory map (bytes from a 1024-aligned base)
+constexpr uint32_t WY_K = 0;                          // K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
+constexpr uint32_t WY_FA = 16384;                     // fp32 [64][FA_S]; the M = 128 product of K K^T reads its
+                                                      // first 8 KB as rows 64..127 of A (output ignored)
+constexpr uint32_t WY_FX = WY_FA + 64 * FA_S * 4;     // fp32 [64][FX_S]
+constexpr uint32_t WY_TMP = WY_FX + 64 * FX_S * 4;    // fp32 [32][33]
+constexpr uint32_t WY_TG = WY_TMP + 32 * 33 * 4;      // 2 buffers (item parity) x (G2[64], beta[64], row[64],
+                                                      // col[64], del[64], flag)
+constexpr uint32_t kTgFloats = 324;
+constexpr uint32_t WY_BYTES = WY_TG + 2 * kTgFloats * 4;
+constexpr uint32_t kWySmemAlloc = WY_BYTES + 1024;
+static_assert(WY_TG % 16 == 0 && (kTgFloats * 4) % 16 == 0, "tile factors must be 16-byte aligned");
+static_assert(kWyCtasPerSm * (kWySmemAlloc + 1024) <= 233472, "factor kernel: CTAs per SM");
+
+struct WyArgs {
+    int L, Hk, Hv, T, n_tiles;
+    const float* g;
+    const float* beta;
+    uint8_t* rec;              // [L * Hv][n_tiles] records of kRecBytes
+    int32_t* status;
+};
+
+__global__ void __launch_bounds__(kWyThreads, kWyCtasPerSm)
+gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
-    // TMA -> MMA: K buffers, V buffer.  MMA -> roles: kk, x, u, s.  roles -> MMA: ready flags.
-    __shared__ uint64_t mb_tk[3], mb_tv, mb_kk[2], mb_x, mb_u, mb_s, mb_sready, mb_xready, mb_uready, mb_tready, mb_fin;
-    __shared__ uint64_t mb_cready[3];                  // chain tile constants of tile t in buffer t % 3
-    __shared__ uint64_t mb_st;                         // a head's state landed in S_before
+    __shared__ uint64_t mb_k, mb_kk;
     __shared__ uint32_t s_tmem;
-    __shared__ int s_abort;
-    __shared__ double s_red[2][8];
-    volatile int* abort_flag = &s_abort;
-
+    __shared__ int s_fail;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int n = a.n_tiles;
-    // Persistent CTA: it owns heads blockIdx.x, blockIdx.x + gridDim.x, ...  Their tiles form one
-    // sequence J = head slot * n + tile, over which every role keeps its barrier phases, so the
-    // next head's loads and T builds overlap the current head's last tiles.
-    const int n_heads = a.L * a.Hv;
-    const int NJ = ((n_heads - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x) * n;
+    const int items = a.L * a.Hv * n;                 // item = (layer * Hv + head) * n + tile
+    float* fA = reinterpret_cast<float*>(sm + WY_FA);
+    float* fX = reinterpret_cast<float*>(sm + WY_FX);
+    float* fT = reinterpret_cast<float*>(sm + WY_TMP);
 
-    if (warp == kCtlWarp) {
-        tmem_alloc(&s_tmem, kTmemCols);
-        tmem_relinquish();
-        if (lane == 0) {
-            mbar_init(&mb_tk[0], 1); mbar_init(&mb_tk[1], 1); mbar_init(&mb_tk[2], 1); mbar_init(&mb_tv, 1);
-            mbar_init(&mb_kk[0], 1); mbar_init(&mb_kk[1], 1);
-            mbar_init(&mb_x, 1); mbar_init(&mb_u, 1); mbar_init(&mb_s, 1);
-            mbar_init(&mb_sready, kChain); mbar_init(&mb_xready, kChain); mbar_init(&mb_uready, kChain);
-            mbar_init(&mb_tready, kTB); mbar_init(&mb_fin, 1);
-            mbar_init(&mb_cready[0], 1); mbar_init(&mb_cready[1], 1); mbar_init(&mb_cready[2], 1);
-            mbar_init(&mb_st, 1);
-            fence_barrier_init();
-            prefetch_tensormap(&kmap);
-            prefetch_tensormap(&vmap);
-            prefetch_tensormap(&smap);
-        }
+    if (warp == 0) { tmem_alloc(&s_tmem, kWyTmemCols); tmem_relinquish(); }
+    if (tid == 0) {
+        mbar_init(&mb_k, 1); mbar_init(&mb_kk, 1);
+        fence_barrier_init();
+        prefetch_tensormap(&kmap);
+        s_fail = 0;
     }
-    if (tid == 0) s_abort = 0;
+    // The strictly upper 16 x 16 blocks of X are never written; zeros there let every level run
+    // fixed-length (unrolled) loops over the triangular factors.
+    for (int e = tid; e < 64 * FX_S; e += kWyThreads) fX[e] = 0.f;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tm = s_tmem;
 
-    if (warp == kCtlWarp) {
-        // =========================================================== TMA + MMA issue (whole warp,
-        // converged; elect.sync picks the issuing lane)
-        {
-            TileCursor kc, vc;                         // next K / V tile to load (loaded in order)
-            kc.init(a); vc.init(a);
-            auto load_k = [&](int J) {                 // K tile of global tile J -> buffer J % 3
-                const int b = J % 3;
-                if (elect_one()) {
-                    uint8_t* dst = sm + SM_K + b * 16384;
-                    mbar_arrive_expect_tx(&mb_tk[b], 16384);
-                    tma_load_4d(dst, &kmap, &mb_tk[b], 0, kc.kh, kc.jt * kC, kc.l);
-                    tma_load_4d(dst + 8192, &kmap, &mb_tk[b], 64, kc.kh, kc.jt * kC, kc.l);
-                }
-                __syncwarp();
-                kc.next(n, a);
-            };
-            auto load_v = [&]() {
-                if (elect_one()) {
-                    mbar_arrive_expect_tx(&mb_tv, 16384);
-                    tma_load_4d(sm + SM_V, &vmap, &mb_tv, 0, vc.h, vc.jt * kC, vc.l);
-                    tma_load_4d(sm + SM_V + 8192, &vmap, &mb_tv, 64, vc.h, vc.jt * kC, vc.l);
-                }
-                __syncwarp();
-                vc.next(n, a);
-            };
-            auto mma_kk = [&](int tile) {
-                // K K^T into the K K^T buffer of the tile's parity.  M = 128: rows 64..127 of A read
-                // the next 8 KB of shared memory (valid, ignored output).
-                const uint8_t* sK = sm + SM_K + (tile % 3) * 16384;
+    auto item_pos = [&](int it, int& l, int& h, int& jt) {
+        const int lh = it / n;
+        jt = it - lh * n; l = lh / a.Hv; h = lh - l * a.Hv;
+    };
+    auto load_k = [&](int it) {                        // thread 0: the item's K tile
+        int l, h, jt;
+        item_pos(it, l, h, jt);
+        const int kh = (int)(((long long)h * a.Hk) / a.Hv);
+        mbar_arrive_expect_tx(&mb_k, 16384);
+        tma_load_4d(sm + WY_K, &kmap, &mb_k, 0, kh, jt * kC, l);
+        tma_load_4d(sm + WY_K + 8192, &kmap, &mb_k, 64, kh, jt * kC, l);
+    };
+    // g and beta of an item's 64 tokens, two per lane of warp 7, loaded one item ahead of use
+    float pg[2] = {0.f, 0.f}, pb[2] = {0.f, 0.f};
+    auto load_gb = [&](int it) {
+        int l, h, jt;
+        item_pos(it, l, h, jt);
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int t = jt * kC + 2 * lane + e;
+            const size_t gi = ((size_t)l * a.T + t) * a.Hv + h;
+            pg[e] = t < a.T ? a.g[gi] : 0.f;
+            pb[e] = t < a.T ? a.beta[gi] : 0.f;
+        }
+    };
+    // Decay constants of an item from the loaded g, beta (warp 7): the update kernel's -gamma and
+    // gamma_C into the record, and this kernel's G2, beta, row and column factors and
+    // exp(G_C - G) into buffer `buf`.
+    auto tile_constants = [&](int it, int buf) {
+        float incl = pg[0] + pg[1];
+#pragma unroll
+        for (int m = 1; m < 32; m <<= 1) {
+            const float y = __shfl_up_sync(0xffffffffu, incl, m);
+            if (lane >= m) incl += y;
+        }
+        const float G0 = incl - pg[1], G1 = incl;
+        const float GC = __shfl_sync(0xffffffffu, incl, 31);
+        float* rc = reinterpret_cast<float*>(a.rec + (size_t)it * kRecBytes + kRecT);
+        *reinterpret_cast<float2*>(rc + 2 * lane) = make_float2(-expf(G0), -expf(G1));
+        if (lane == 0) *reinterpret_cast<float4*>(rc + 64) = make_float4(expf(GC), 0.f, 0.f, 0.f);
+        const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
+        float lo2 = fminf(g20, g21), hi2 = fmaxf(g20, g21);
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) {
+            lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, m));
+            hi2 = fmaxf(hi2, __shfl_xor_sync(0xffffffffu, hi2, m));
+        }
+        // exp(G_t - G_i) = row_t * col_i with the reference in the middle of the tile's range of
+        // G; both factors stay within 2^+-126 when that range spans at most 250 powers of two,
+        // otherwise the exponent is taken per entry.
+        const float ref = 0.5f * (lo2 + hi2);
+        float* tg = reinterpret_cast<float*>(sm + WY_TG) + buf * kTgFloats;
+        tg[2 * lane] = g20; tg[2 * lane + 1] = g21;
+        tg[64 + 2 * lane] = pb[0]; tg[64 + 2 * lane + 1] = pb[1];
+        tg[128 + 2 * lane] = pb[0] * fast_exp2(g20 - ref); tg[128 + 2 * lane + 1] = pb[1] * fast_exp2(g21 - ref);
+        tg[192 + 2 * lane] = fast_exp2(ref - g20); tg[192 + 2 * lane + 1] = fast_exp2(ref - g21);
+        tg[256 + 2 * lane] = expf(GC - G0); tg[256 + 2 * lane + 1] = expf(GC - G1);
+        if (lane == 0) reinterpret_cast<int*>(tg)[320] = (hi2 - lo2) <= 250.f;
+    };
+
+    const int first = (int)blockIdx.x;
+    if (first < items) {
+        if (tid == 0) load_k(first);
+        if (warp == 7) {
+            load_gb(first);
+            tile_constants(first, 0);
+            if (first + (int)gridDim.x < items) load_gb(first + (int)gridDim.x);
+        }
+    }
+    __syncthreads();
+    int c = 0;                                         // items done by this CTA (barrier phases)
+    for (int it = first; it < items; it += (int)gridDim.x, ++c) {
+        const float* tg = reinterpret_cast<const float*>(sm + WY_TG) + (c & 1) * kTgFloats;
+        const float* sG2 = tg;                         // G * log2(e)
+        const float* sBeta = tg + 64;
+        const float* sRow = tg + 128;                  // beta_t 2^(G2_t - ref)
+        const float* sCol = tg + 192;                  // 2^(ref - G2_i)
+        const float* sDel = tg + 256;                  // exp(G_C - G_t)
+        const int factored = reinterpret_cast<const int*>(tg)[320];
+        // K K^T (M = 128: rows 64..127 of A read the 8 KB past the tile; their output is ignored)
+        if (warp == 0) {
+            const bool ok = __all_sync(0xffffffffu, mbar_wait(&mb_k, c & 1, kWaitBudgetNs)) != 0;
+            if (!ok) {
+                if (lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 21); s_fail = 1; }
+            } else {
+                tc_fence_after();
                 const uint32_t id = idesc_bf16(128, 64, 0, 0);
 #pragma unroll
                 for (int s = 0; s < 8; ++s) {
-                    const uint64_t d = sdesc_sw128(smem_u32(sK + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
-                    mma_bf16(tm + TM_KK + 64 * (tile & 1), d, d, id, s > 0);
+                    const uint64_t d = sdesc_sw128(smem_u32(sm + WY_K + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
+                    mma_bf16(tm, d, d, id, s > 0);
                 }
-                mma_commit(&mb_kk[tile & 1]);
-            };
-            int kp[3] = {-1, -1, -1};                  // tile whose K load is in flight, per buffer
-            int v_pending = 0;
-            load_k(0); kp[0] = 0;
-            if (NJ > 1) { load_k(1); kp[1] = 1; }
-            load_v();
-            bool ok = warp_wait(&mb_tk[0], 0, kWaitBudgetNs, abort_flag);
-            if (!ok) fail(a.status, abort_flag, 1);
-            if (ok) { kp[0] = -1; mma_kk(0); }
-            for (int j = 0; ok && j < NJ; ++j) {          // j: global tile index
-                const uint8_t* sK = sm + SM_K + (j % 3) * 16384;
-                // tile j ready for X: the fp32 copy of K(j) is written and, at a head's first tile, the
-                // state is in TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe order)
-                if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
-                tc_fence_after();
-                {   // X~^T = S~ K^T: A = the fp32 state straight from TMEM read as tf32 (8 columns per
-                    // K = 8 step), B = K in fp32
-                    const uint32_t id = idesc_tf32(128, 64);
-                    const uint8_t* k32 = sm + SM_K32;
-#pragma unroll
-                    for (int s = 0; s < 16; ++s) {
-                        const uint64_t bd = sdesc_sw128(smem_u32(k32 + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
-                        mma_tf32_ta(tm + TM_X, tm + TM_S + 8 * s, bd, id, s != 0);
-                    }
-                    mma_commit(&mb_x);
-                }
-                if (j + 1 < NJ) {                      // K K^T of the next tile, for the T builders
-                    if (!warp_wait(&mb_tk[(j + 1) % 3], ((j + 1) / 3) & 1, kWaitBudgetNs, abort_flag)) {
-                        fail(a.status, abort_flag, 4); break;
-                    }
-                    kp[(j + 1) % 3] = -1;
-                    mma_kk(j + 1);
-                }
-                if (!warp_wait(&mb_tready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 3); break; }
-                if (!warp_wait(&mb_xready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 5); break; }
-                if (!warp_wait(&mb_tv, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 6); break; }
-                v_pending = -1;
-                tc_fence_after();
-                {   // U^T = V^T T^T + X~^T T^T   (X~ = -diag(gamma) X, hi / lo packed in place in X)
-                    const uint8_t* tb = sm + SM_T;
-                    const uint32_t id_v = idesc_bf16(128, 64, 1, 0);      // A = V tile read MN-major
-                    const uint32_t id_x = idesc_bf16(128, 64, 0, 0);      // A = X~ from TMEM
-#pragma unroll
-                    for (int part = 0; part < 5; ++part) {
-                        const uint8_t* sb = tb + ((part == 1 || part == 3) ? 8192 : 0);
-#pragma unroll
-                        for (int s = 0; s < 4; ++s) {
-                            const uint64_t bd = sdesc_sw128(smem_u32(sb + s * 32), 16, 1024);
-                            const uint32_t acc = (part | s) != 0;
-                            if (part < 2) {
-                                mma_bf16(tm + TM_U, sdesc_sw128(smem_u32(sm + SM_V + s * 2048), 8192, 1024), bd, id_v, acc);
-                            } else {
-                                // tokens 16s..16s+15: column block s/2 of the X region, hi then lo
-                                const uint32_t a = tm + TM_X + 32 * (s >> 1) + 8 * (s & 1) + (part == 4 ? 16 : 0);
-                                mma_bf16_ta(tm + TM_U, a, bd, id_x, acc);
-                            }
-                        }
-                    }
-                    mma_commit(&mb_u);
-                }
-                // TMA loads are issued behind MMA groups, never between a wait and the MMAs it
-                // releases (a TMA write burst into shared memory slows the issue of a group).
-                // K(j+2) reuses the buffer of K(j-1), whose last reader MMA_S(j-1) has completed.
-                if (j + 2 < NJ) { load_k(j + 2); kp[(j + 2) % 3] = j + 2; }
-                if (!warp_wait(&mb_uready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 7); break; }
-                tc_fence_after();
-                {   // S += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major: N = d_k)
-                    const uint32_t id = idesc_bf16(128, 128, 0, 1);
-#pragma unroll
-                    for (int part = 0; part < 2; ++part) {
-#pragma unroll
-                        for (int s = 0; s < 4; ++s) {
-                            const uint32_t a = tm + TM_U + 32 * (s >> 1) + 8 * (s & 1) + (part == 1 ? 16 : 0);
-                            const uint64_t bd = sdesc_sw128(smem_u32(sK + s * 2048), 8192, 1024);
-                            mma_bf16_ta(tm + TM_S, a, bd, id, 1);
-                        }
-                    }
-                    mma_commit(&mb_s);
-                }
-                // V(j+1) into the single V buffer: MMA_U(j), its reader, completed before uready
-                if (j + 1 < NJ) { load_v(); v_pending = j + 1; }
-            }
-            if (__any_sync(0xffffffffu, *abort_flag != 0)) {
-                // drain: every MMA this warp issued, and every load still in flight
-                mma_commit(&mb_fin);
-                mbar_wait(&mb_fin, 0, kWaitBudgetNs);
-                for (int b = 0; b < 3; ++b)
-                    if (kp[b] >= 0) mbar_wait(&mb_tk[b], (kp[b] / 3) & 1, kWaitBudgetNs);
-                if (v_pending >= 0) mbar_wait(&mb_tv, v_pending & 1, kWaitBudgetNs);
+                mma_commit(&mb_kk);
             }
         }
-        __syncwarp();
-    } else if (warp >= 8) {
-        // =========================================================== T builders (warps 8-15)
-        const int tw = warp - 8, tt = tid - kChain;        // tw in [0, 8), tt in [0, 256)
-        float* fA = reinterpret_cast<float*>(sm + SM_FA);
-        float* fX = reinterpret_cast<float*>(sm + SM_FX);
-        float* fT = reinterpret_cast<float*>(sm + SM_TMP);
-        float* cg = reinterpret_cast<float*>(sm + SM_CG);
-        float pg[2] = {0.f, 0.f}, pb[2] = {0.f, 0.f};     // g, beta of the next tile (warp 15)
-        TileCursor gc;                                     // next tile whose g, beta to load
-        gc.init(a);
-        auto load_gb = [&]() {                             // g, beta of the next tile (warp 15)
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int t = gc.jt * kC + 2 * lane + e;
-                const size_t gi = ((size_t)gc.l * a.T + t) * a.Hv + gc.h;
-                pg[e] = t < a.T ? a.g[gi] : 0.f;
-                pb[e] = t < a.T ? a.beta[gi] : 0.f;
-            }
-            gc.next(n, a);
-        };
-        // Decay constants of tile jj from the loaded g, beta (warp 15, one tile ahead of the
-        // T build that uses them): the chain's -gamma, exp(G_C - G), gamma_C, and the T builders'
-        // G2, beta, row and column factors (buffer jj & 1).
-        auto tile_constants = [&](int jj) {
-            float* tg = reinterpret_cast<float*>(sm + SM_TG) + (jj & 1) * kTgFloats;
-            float gv[2], bv[2];
-#pragma unroll
-            for (int e = 0; e < 2; ++e) { gv[e] = pg[e]; bv[e] = pb[e]; }
-            float incl = gv[0] + gv[1];
-#pragma unroll
-            for (int m = 1; m < 32; m <<= 1) {
-                const float y = __shfl_up_sync(0xffffffffu, incl, m);
-                if (lane >= m) incl += y;
-            }
-            const float G0 = incl - gv[1], G1 = incl;
-            const float GC = __shfl_sync(0xffffffffu, incl, 31);
-            // the chain's constants of tile jj (3 buffers: the chain is at most two tiles behind
-            // the T builders' current tile)
-            float* cgam = cg + (jj % 3) * 132;
-            cgam[2 * lane] = -expf(G0); cgam[2 * lane + 1] = -expf(G1);
-            cgam[64 + 2 * lane] = expf(GC - G0); cgam[64 + 2 * lane + 1] = expf(GC - G1);
-            if (lane == 0) cgam[128] = expf(GC);
-            const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
-            float lo2 = fminf(g20, g21), hi2 = fmaxf(g20, g21);
-#pragma unroll
-            for (int m = 16; m >= 1; m >>= 1) {
-                lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, m));
-                hi2 = fmaxf(hi2, __shfl_xor_sync(0xffffffffu, hi2, m));
-            }
-            // exp(G_t - G_i) = row_t * col_i with the reference in the middle of the tile's range
-            // of G; both factors stay within 2^+-126 when that range spans at most 250 powers of
-            // two, otherwise the exponent is taken per entry.
-            const float ref = 0.5f * (lo2 + hi2);
-            tg[2 * lane] = g20; tg[2 * lane + 1] = g21;
-            tg[64 + 2 * lane] = bv[0]; tg[64 + 2 * lane + 1] = bv[1];
-            tg[128 + 2 * lane] = bv[0] * fast_exp2(g20 - ref); tg[128 + 2 * lane + 1] = bv[1] * fast_exp2(g21 - ref);
-            tg[192 + 2 * lane] = fast_exp2(ref - g20); tg[192 + 2 * lane + 1] = fast_exp2(ref - g21);
-            if (lane == 0) reinterpret_cast<int*>(tg)[256] = (hi2 - lo2) <= 250.f;
-            fence_async_smem();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&mb_cready[jj % 3]);
-        };
-        // The strictly upper 16 x 16 blocks of X are never written; zeros there let every level
-        // run fixed-length (unrolled) loops over the triangular factors.
-        for (int e = tt; e < 64 * FX_S; e += kTB) fX[e] = 0.f;
-        if (tw == 7 && NJ > 0) {
-            load_gb();
-            tile_constants(0);
-            if (NJ > 1) load_gb();
-        }
-        for (int j = 0; j < NJ; ++j) {                     // j: global tile index
-            if (named_sync_or(3, kTB, *abort_flag)) break;
-            const float* tg = reinterpret_cast<const float*>(sm + SM_TG) + (j & 1) * kTgFloats;
-            const float* sG2 = tg;                         // G * log2(e)
-            const float* sBeta = tg + 64;
-            const float* sRow = tg + 128;                  // beta_t 2^(G2_t - ref)
-            const float* sCol = tg + 192;                  // 2^(ref - G2_i)
-            const int factored = reinterpret_cast<const int*>(tg)[256];
-            if (!mbar_wait_or_abort(&mb_kk[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 8);
+        const int q = warp & 3;
+        if (q < 2) {
+            // TMEM lanes 0..63 hold K K^T: warps 0/4 rows 0..31, 1/5 rows 32..63; column half
+            // (warp >> 2).
+            const bool ok = mbar_wait_or_abort(&mb_kk, c & 1, kWaitBudgetNs, &s_fail);
+            if (!ok && lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 22); s_fail = 1; }
             tc_fence_after();
-            const int q = warp & 3;
-            if (q < 2) {
-                // TMEM lanes 0..63 hold K K^T: warps 8/12 rows 0..31, 9/13 rows 32..63; column half
-                // (tw >> 2).  All shared-memory reads are made before the first store (the tile
-                // constants and A share one buffer).
-                const int t = 32 * q + lane, c0 = 32 * (tw >> 2);
-                const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-                float kk[32], cf[32];
-                tmem_ld32(tm + lane_off + TM_KK + 64 * (j & 1) + c0, kk);
-                if (factored) {
-                    const float rt = sRow[t];
+            const int t = 32 * q + lane, c0 = 32 * (warp >> 2);
+            const uint32_t lane_off = (uint32_t)(32 * q) << 16;
+            float kk[32], cf[32];
+            tmem_ld32(tm + lane_off + c0, kk);
+            if (factored) {
+                const float rt = sRow[t];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float4 v4 = *reinterpret_cast<const float4*>(sCol + c0 + 4 * e);
-                        cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
-                    }
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? rt * cf[e] * kk[e] : 0.f;
-                } else {
-                    const float G2t = sG2[t], bt = sBeta[t];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float4 v4 = *reinterpret_cast<const float4*>(sG2 + c0 + 4 * e);
-                        cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
-                    }
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? bt * fast_exp2(G2t - cf[e]) * kk[e] : 0.f;
+                for (int e = 0; e < 8; ++e) {
+                    const float4 v4 = *reinterpret_cast<const float4*>(sCol + c0 + 4 * e);
+                    cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
                 }
+                tmem_ld_wait();
 #pragma unroll
-                for (int e = 0; e < 8; ++e)
-                    *reinterpret_cast<float4*>(fA + t * FA_S + c0 + 4 * e) =
-                        make_float4(kk[4 * e], kk[4 * e + 1], kk[4 * e + 2], kk[4 * e + 3]);
-            } else if (tw == 7 && j + 1 < NJ) {
-                tile_constants(j + 1);                     // the next tile's, off this tile's path
-                if (j + 2 < NJ) load_gb();
+                for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? rt * cf[e] * kk[e] : 0.f;
+            } else {
+                const float G2t = sG2[t], bt = sBeta[t];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float4 v4 = *reinterpret_cast<const float4*>(sG2 + c0 + 4 * e);
+                    cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
+                }
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? bt * fast_exp2(G2t - cf[e]) * kk[e] : 0.f;
             }
-            tc_fence_before();
-            named_sync(3, kTB);
-            // level 0: four 16 x 16 diagonal blocks of (I + A)^-1, one column per thread
-            if (tt < 64) {
-                const int B = tt >> 4, jc = tt & 15, o = 16 * B;
-                float x[16];
 #pragma unroll
-                for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
+            for (int e = 0; e < 8; ++e)
+                *reinterpret_cast<float4*>(fA + t * FA_S + c0 + 4 * e) =
+                    make_float4(kk[4 * e], kk[4 * e + 1], kk[4 * e + 2], kk[4 * e + 3]);
+        }
+        tc_fence_before();
+        __syncthreads();
+        if (s_fail) break;
+        // K K^T is in fA: the K tile and the TMEM columns are free for the next item
+        const int nxt = it + (int)gridDim.x;
+        if (tid == 0 && nxt < items) load_k(nxt);
+        // level 0: four 16 x 16 diagonal blocks of (I + A)^-1, one column per thread (warps 0-1);
+        // meanwhile warp 7 prepares the next item's constants and loads the one after
+        if (tid < 64) {
+            const int B = tid >> 4, jc = tid & 15, o = 16 * B;
+            float x[16];
 #pragma unroll
-                for (int rr = 1; rr < 16; ++rr) {
-                    float s0 = 0.f, s1 = 0.f;              // two chains: half the dependent FMAs
+            for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
 #pragma unroll
-                    for (int c = 0; c < rr; c += 4) {
-                        const float4 av = *reinterpret_cast<const float4*>(fA + (o + rr) * FA_S + o + c);
-                        s0 = fmaf(av.x, x[c], s0);
-                        if (c + 1 < rr) s1 = fmaf(av.y, x[c + 1], s1);
-                        if (c + 2 < rr) s0 = fmaf(av.z, x[c + 2], s0);
-                        if (c + 3 < rr) s1 = fmaf(av.w, x[c + 3], s1);
-                    }
-                    if (rr > jc) x[rr] = -(s0 + s1);
+            for (int rr = 1; rr < 16; ++rr) {
+                float s0 = 0.f, s1 = 0.f;              // two chains: half the dependent FMAs
+#pragma unroll
+                for (int cc = 0; cc < rr; cc += 4) {
+                    const float4 av = *reinterpret_cast<const float4*>(fA + (o + rr) * FA_S + o + cc);
+                    s0 = fmaf(av.x, x[cc], s0);
+                    if (cc + 1 < rr) s1 = fmaf(av.y, x[cc + 1], s1);
+                    if (cc + 2 < rr) s0 = fmaf(av.z, x[cc + 2], s0);
+                    if (cc + 3 < rr) s1 = fmaf(av.w, x[cc + 3], s1);
                 }
-#pragma unroll
-                for (int rr = 0; rr < 16; ++rr) fX[(o + rr) * FX_S + o + jc] = x[rr];
+                if (rr > jc) x[rr] = -(s0 + s1);
             }
-            named_sync(3, kTB);
-            // level 1: X[2p+1][2p] = -X[2p+1][2p+1] (A[2p+1][2p] X[2p][2p]), p = tw >> 2.
-            // Fixed-length loops: the zeros of the triangular factors are stored.
-            {
-                const int p = tw >> 2, cg = 4 * (tw & 3);
-                const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
-                const int lo16 = lane & 15, sub = 2 * (lane >> 4);
-                float acc0 = 0.f, acc1 = 0.f;             // tmp1[p][lo16][cg + sub + {0,1}]
 #pragma unroll
-                for (int k4 = 0; k4 < 16; k4 += 4) {
-                    const float4 a4 = *reinterpret_cast<const float4*>(fA + (ro + lo16) * FA_S + co + k4);
-                    const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+            for (int rr = 0; rr < 16; ++rr) fX[(o + rr) * FX_S + o + jc] = x[rr];
+        } else if (warp == 7 && nxt < items) {
+            tile_constants(nxt, (c + 1) & 1);
+            if (nxt + (int)gridDim.x < items) load_gb(nxt + (int)gridDim.x);
+        }
+        __syncthreads();
+        // level 1: X[2p+1][2p] = -X[2p+1][2p+1] (A[2p+1][2p] X[2p][2p]) for the 16 x 16 blocks,
+        // p = 0, 1; warps 0-3 take (p, 8-column half) = (warp / 2, warp % 2)
+        const int g = lane >> 2, tq = lane & 3;
+        if (warp < 4) {
+            const int p = warp >> 1, nc = 8 * (warp & 1);
+            const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            mma_3xtf32<2>(d, [&](int r, int k) { return fA[(ro + r) * FA_S + co + k]; },
+                             [&](int k, int cc) { return fX[(co + k) * FX_S + co + nc + cc]; }, lane);
+            float* P = fT + p * 272;                   // [16][17]
+            P[g * 17 + nc + 2 * tq] = d[0]; P[g * 17 + nc + 2 * tq + 1] = d[1];
+            P[(g + 8) * 17 + nc + 2 * tq] = d[2]; P[(g + 8) * 17 + nc + 2 * tq + 1] = d[3];
+        }
+        __syncthreads();
+        if (warp < 4) {
+            const int p = warp >> 1, nc = 8 * (warp & 1);
+            const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
+            const float* P = fT + p * 272;
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            mma_3xtf32<2>(d, [&](int r, int k) { return fX[(ro + r) * FX_S + ro + k]; },
+                             [&](int k, int cc) { return P[k * 17 + nc + cc]; }, lane);
+            fX[(ro + g) * FX_S + co + nc + 2 * tq] = -d[0]; fX[(ro + g) * FX_S + co + nc + 2 * tq + 1] = -d[1];
+            fX[(ro + g + 8) * FX_S + co + nc + 2 * tq] = -d[2]; fX[(ro + g + 8) * FX_S + co + nc + 2 * tq + 1] = -d[3];
+        }
+        __syncthreads();
+        // level 2: X[32:64][0:32] = -X[32:64][32:64] (A[32:64][0:32] X[0:32][0:32]); warp w takes
+        // the 16 x 8 output tile (w / 4, w % 4)
+        {
+            const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            mma_3xtf32<4>(d, [&](int r, int k) { return fA[(32 + mr + r) * FA_S + k]; },
+                             [&](int k, int cc) { return fX[k * FX_S + nc + cc]; }, lane);
+            fT[(mr + g) * 33 + nc + 2 * tq] = d[0]; fT[(mr + g) * 33 + nc + 2 * tq + 1] = d[1];
+            fT[(mr + g + 8) * 33 + nc + 2 * tq] = d[2]; fT[(mr + g + 8) * 33 + nc + 2 * tq + 1] = d[3];
+        }
+        __syncthreads();
+        {
+            const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            mma_3xtf32<4>(d, [&](int r, int k) { return fX[(32 + mr + r) * FX_S + 32 + k]; },
+                             [&](int k, int cc) { return fT[k * 33 + nc + cc]; }, lane);
+            fX[(32 + mr + g) * FX_S + nc + 2 * tq] = -d[0]; fX[(32 + mr + g) * FX_S + nc + 2 * tq + 1] = -d[1];
+            fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq] = -d[2]; fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq + 1] = -d[3];
+        }
+        __syncthreads();
+        // T~ = diag(exp(G_C - G)) X diag(beta) (upper part zero), split into the record's (hi, lo)
+        // images
+        {
+            uint8_t* rec = a.rec + (size_t)it * kRecBytes;
 #pragma unroll
-                    for (int kk4 = 0; kk4 < 4; ++kk4) {
-                        const float2 xv = *reinterpret_cast<const float2*>(fX + (co + k4 + kk4) * FX_S + co + cg + sub);
-                        acc0 = fmaf(av[kk4], xv.x, acc0);
-                        acc1 = fmaf(av[kk4], xv.y, acc1);
-                    }
-                }
-                fT[p * 272 + lo16 * 17 + cg + sub] = acc0;
-                fT[p * 272 + lo16 * 17 + cg + sub + 1] = acc1;
-                named_sync(3, kTB);
-                float o0 = 0.f, o1 = 0.f;                  // rows cg + sub + {0,1}, column lo16
-#pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    const float tv = fT[p * 272 + k * 17 + lo16];
-                    o0 = fmaf(fX[(ro + cg + sub) * FX_S + ro + k], tv, o0);
-                    o1 = fmaf(fX[(ro + cg + sub + 1) * FX_S + ro + k], tv, o1);
-                }
-                fX[(ro + cg + sub) * FX_S + co + lo16] = -o0;
-                fX[(ro + cg + sub + 1) * FX_S + co + lo16] = -o1;
-            }
-            named_sync(3, kTB);
-            // level 2: X[32:64][0:32] = -X[32:64][32:64] (A[32:64][0:32] X[0:32][0:32])
-            {
-                const int g4 = 4 * tw;
-                float acc[4] = {0.f, 0.f, 0.f, 0.f};       // tmp2[lane][g4..g4+3]
-#pragma unroll
-                for (int k4 = 0; k4 < 32; k4 += 4) {
-                    const float4 a4 = *reinterpret_cast<const float4*>(fA + (32 + lane) * FA_S + k4);
-                    const float av[4] = {a4.x, a4.y, a4.z, a4.w};
-#pragma unroll
-                    for (int kk4 = 0; kk4 < 4; ++kk4) {
-                        const float4 xv = *reinterpret_cast<const float4*>(fX + (k4 + kk4) * FX_S + g4);
-                        acc[0] = fmaf(av[kk4], xv.x, acc[0]); acc[1] = fmaf(av[kk4], xv.y, acc[1]);
-                        acc[2] = fmaf(av[kk4], xv.z, acc[2]); acc[3] = fmaf(av[kk4], xv.w, acc[3]);
-                    }
-                }
-#pragma unroll
-                for (int i = 0; i < 4; ++i) fT[lane * 33 + g4 + i] = acc[i];
-                named_sync(3, kTB);
-                float o4[4] = {0.f, 0.f, 0.f, 0.f};        // rows 32+g4..32+g4+3, column lane
-#pragma unroll
-                for (int k = 0; k < 32; k += 4) {
-                    const float t0v = fT[(k + 0) * 33 + lane], t1v = fT[(k + 1) * 33 + lane];
-                    const float t2v = fT[(k + 2) * 33 + lane], t3v = fT[(k + 3) * 33 + lane];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const float4 xr = *reinterpret_cast<const float4*>(fX + (32 + g4 + i) * FX_S + 32 + k);
-                        o4[i] = fmaf(xr.x, t0v, o4[i]); o4[i] = fmaf(xr.y, t1v, o4[i]);
-                        o4[i] = fmaf(xr.z, t2v, o4[i]); o4[i] = fmaf(xr.w, t3v, o4[i]);
-                    }
-                }
-#pragma unroll
-                for (int i = 0; i < 4; ++i) fX[(32 + g4 + i) * FX_S + lane] = -o4[i];
-            }
-            // the single T buffer is free once MMA_U(j-1) has read it (it completes long before this
-            // point in steady state; MMA_U(j) cannot complete before T(j) is written, so the
-            // barrier is never two phases ahead)
-            if (j > 0 && !mbar_wait_or_abort(&mb_u, (j - 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 15);
-            named_sync(3, kTB);
-            // T = X diag(beta) (upper part zero), split into the B operand buffer
-            {
-                uint8_t* tb = sm + SM_T;
-                uint4 vh[2], vl[2];
-                int tr[2], cr[2];
-#pragma unroll
-                for (int m = 0; m < 2; ++m) {
-                    const int e = tt + kTB * m;
-                    const int t = e >> 3, c8 = e & 7;
+            for (int m = 0; m < 2; ++m) {
+                const int e = tid + kWyThreads * m;
+                const int t = e >> 3, c8 = e & 7;
+                uint4 vh = make_uint4(0u, 0u, 0u, 0u), vl = vh;
+                if (8 * c8 <= t) {                     // chunks right of the diagonal stay zero
+                    const float dt = sDel[t];
                     const float4 x0 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8);
                     const float4 x1 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8 + 4);
                     const float4 b0 = *reinterpret_cast<const float4*>(sBeta + 8 * c8);
@@ -598,58 +487,334 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                                          x1.x * b1.x, x1.y * b1.y, x1.z * b1.z, x1.w * b1.w};
                     float x[8];
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) x[k] = (8 * c8 + k <= t) ? xs[k] : 0.f;
-                    split8(x, vh[m], vl[m]);
-                    tr[m] = t; cr[m] = c8;
+                    for (int k = 0; k < 8; ++k) x[k] = (8 * c8 + k <= t) ? dt * xs[k] : 0.f;
+                    split8(x, vh, vl);
                 }
+                *reinterpret_cast<uint4*>(rec + sw128_offset(t, c8)) = vh;
+                *reinterpret_cast<uint4*>(rec + 8192 + sw128_offset(t, c8)) = vl;
+            }
+        }
+        // the next item's level 0 rewrites fX's diagonal blocks: everyone has read this one's
+        __syncthreads();
+    }
+    if (tid == 0 && s_fail) {
+        // after a failure at item c: its K load and K K^T product land before TMEM is freed
+        mbar_wait(&mb_k, c & 1, kWaitBudgetNs);
+        mbar_wait(&mb_kk, c & 1, kWaitBudgetNs);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tm, kWyTmemCols);
+    }
+}
+
+// =============================================================================================
+// Update kernel: the state chain
+// =============================================================================================
+constexpr int kChainWarps = 16;
+constexpr int kChain = 32 * kChainWarps;         // chain threads
+constexpr int kMmaWarp = kChainWarps;            // 16
+constexpr int kLoadWarp = kChainWarps + 1;       // 17
+constexpr int kStateWarp = kChainWarps + 2;      // 18
+constexpr int kThreads = kChain + 96;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t TM_S = 0, TM_SB = 128, TM_X = 256, TM_U = 320;
+
+// shared-memory map (bytes from a 1024-aligned base)
+constexpr uint32_t SM_K = 0;                     // 3 x 16 KB: K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
+constexpr uint32_t SM_K32 = 49152;               // 32 KB: K' in tf32 (the B operand of X), 4 column blocks
+                                                 // (32 dims) x 64 rows x 128 B, SW128
+constexpr uint32_t SM_V = 81920;                 // 2 x 16 KB: V tile (tile parity), layout of K
+constexpr uint32_t SM_R = 114688;                // 2 x kRecSlot: WY records (tile parity)
+constexpr uint32_t kRecSlot = 17408;             // 1024-aligned slots
+constexpr uint32_t SM_I = SM_R + 2 * kRecSlot;   // 8 KB: 64 x 64 bfloat16 identity, K-major SW128
+constexpr uint32_t SM_SB = SM_I + 8192;          // 64 KB: state staging, 4 column blocks x 128 rows x 128 B, SW128
+constexpr uint32_t SM_BYTES = SM_SB + 65536;
+constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
+static_assert(SM_I % 1024 == 0 && SM_SB % 1024 == 0 && kRecSlot >= kRecBytes, "shared-memory map");
+static_assert(kSmemAlloc <= 232448, "shared memory budget");
+
+// The staging buffer holds a head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each
+// 128 rows x 128 bytes with the 128-byte swizzle (16-byte chunk ^ (row & 7)) that TMA writes and
+// reads; eight threads reading chunk c of eight consecutive rows (one row per thread) hit distinct
+// banks.  Float offset of 16-byte chunk `chunk` (0..31) of row `row`:
+__device__ __forceinline__ int sb_idx(int row, int chunk) {
+    return (chunk >> 3) * 4096 + row * 32 + (((chunk & 7) ^ (row & 7)) << 2);
+}
+
+struct TcArgs {
+    int L, Hk, Hv, T, n_tiles;
+    float* state;
+    float* partials;
+    const uint8_t* rec;
+    int32_t* status;
+};
+
+// Where a global tile lies: tile jt of head lh = (layer l, value head h), key head kh.  Each role
+// walks the tiles in order; a step costs integer divisions only when it crosses into the next head.
+struct TileCursor {
+    int jt, lh, l, h, kh;
+    __device__ __forceinline__ void set_head(int head, const TcArgs& a) {
+        lh = head; l = head / a.Hv; h = head - l * a.Hv;
+        kh = (int)(((long long)h * a.Hk) / a.Hv);
+    }
+    __device__ __forceinline__ void init(const TcArgs& a) { jt = 0; set_head((int)blockIdx.x, a); }
+    __device__ __forceinline__ void next(int n, const TcArgs& a) {
+        if (++jt == n) { jt = 0; set_head(lh + (int)gridDim.x, a); }
+    }
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                     const __grid_constant__ CUtensorMap smap, TcArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    // copies -> roles: K (3), V (2), WY records (2) full; MMA -> loader: their empties; state
+    // staging full (mb_st) and released by the chain (mb_sfree); MMA -> chain: x, u, s; chain ->
+    // MMA: ready flags.
+    __shared__ uint64_t mb_tk[3], mb_ke[3], mb_tv[2], mb_ve[2], mb_tr[2], mb_re[2];
+    __shared__ uint64_t mb_st, mb_sfree, mb_x, mb_u, mb_s, mb_sready, mb_xready, mb_uready, mb_fin;
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_abort;
+    __shared__ float s_red[2][kChainWarps];
+    volatile int* abort_flag = &s_abort;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int n = a.n_tiles;
+    // Persistent CTA: it owns heads blockIdx.x, blockIdx.x + gridDim.x, ...  Their tiles form one
+    // sequence J = head slot * n + tile, over which every role keeps its barrier phases.
+    const int n_heads = a.L * a.Hv;
+    const int n_slots = (n_heads - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+    const int NJ = n_slots * n;
+
+    if (warp == kMmaWarp) {
+        tmem_alloc(&s_tmem, kTmemCols);
+        tmem_relinquish();
+        if (lane == 0) {
+            for (int b = 0; b < 3; ++b) { mbar_init(&mb_tk[b], 1); mbar_init(&mb_ke[b], 1); }
+            for (int b = 0; b < 2; ++b) {
+                mbar_init(&mb_tv[b], 1); mbar_init(&mb_ve[b], 1);
+                mbar_init(&mb_tr[b], 1); mbar_init(&mb_re[b], 1);
+            }
+            mbar_init(&mb_st, 1); mbar_init(&mb_sfree, kChain);
+            mbar_init(&mb_x, 1); mbar_init(&mb_u, 1); mbar_init(&mb_s, 1);
+            mbar_init(&mb_sready, kChain); mbar_init(&mb_xready, kChain); mbar_init(&mb_uready, kChain);
+            mbar_init(&mb_fin, 1);
+            fence_barrier_init();
+        }
+    }
+    if (warp == kLoadWarp && lane == 0) { prefetch_tensormap(&kmap); prefetch_tensormap(&vmap); }
+    if (warp == kStateWarp && lane == 0) prefetch_tensormap(&smap);
+    if (tid < kChain) {
+        // the 64 x 64 identity (B operand of V^T I): row t holds 1.0 at column t
+        const int t = tid >> 3, c8 = tid & 7;
+        uint32_t w[4] = {0u, 0u, 0u, 0u};
+        if ((t >> 3) == c8) w[(t & 7) >> 1] = (t & 1) ? 0x3F800000u : 0x00003F80u;
+        *reinterpret_cast<uint4*>(sm + SM_I + sw128_offset(t, c8)) = make_uint4(w[0], w[1], w[2], w[3]);
+        fence_async_smem();
+    }
+    if (tid == 0) s_abort = 0;
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = s_tmem;
+
+    if (warp == kMmaWarp) {
+        // =========================================================== MMA issue (converged warp;
+        // one elected lane issues each group and commits it)
+        const uint64_t dK = sdesc_sw128(smem_u32(sm + SM_K), 8192, 1024);    // MN-major B of MMA_S
+        const uint64_t dK32 = sdesc_sw128(smem_u32(sm + SM_K32), 16, 1024);
+        const uint64_t dV = sdesc_sw128(smem_u32(sm + SM_V), 8192, 1024);    // MN-major A of V^T I
+        const uint64_t dR = sdesc_sw128(smem_u32(sm + SM_R), 16, 1024);
+        const uint64_t dI = sdesc_sw128(smem_u32(sm + SM_I), 16, 1024);
+        // X region <- V(J)^T: A = the V tile read MN-major (k-step s = tokens 16 s ..), B = I.  V(J)'s
+        // buffer is released when the product completes.
+        auto issue_vi = [&](int J) -> bool {
+            if (!warp_wait(&mb_tv[J & 1], (J >> 1) & 1, kWaitBudgetNs, abort_flag)) return false;
+            tc_fence_after();
+            if (elect_one()) {
+                const uint32_t id = idesc_bf16(128, 64, 1, 0);
 #pragma unroll
-                for (int m = 0; m < 2; ++m) {
-                    *reinterpret_cast<uint4*>(tb + sw128_offset(tr[m], cr[m])) = vh[m];
-                    *reinterpret_cast<uint4*>(tb + 8192 + sw128_offset(tr[m], cr[m])) = vl[m];
+                for (int s = 0; s < 4; ++s)
+                    mma_bf16_1t(tm + TM_X, dadd(dV, (J & 1) * 16384 + s * 2048), dadd(dI, s * 32), id, s != 0);
+            }
+            __syncwarp();
+            mma_commit(&mb_ve[J & 1]);
+            return true;
+        };
+        bool ok = NJ == 0 || issue_vi(0);
+        if (!ok) fail(a.status, abort_flag, 1);
+        for (int j = 0; ok && j < NJ; ++j) {           // j: global tile index
+            // tile j ready for X: K'(j) is written and, at a head's first tile, the state is in
+            // TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe order)
+            if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
+            tc_fence_after();
+            if (elect_one()) {   // X region += S~ K'^T: A = the fp32 state from TMEM read as tf32 (8
+                                 // columns per K = 8 step), B = K'
+                const uint32_t id = idesc_tf32(128, 64);
+#pragma unroll
+                for (int s = 0; s < 16; ++s)
+                    mma_tf32_ta_1t(tm + TM_X, tm + TM_S + 8 * s, dadd(dK32, (s >> 2) * 8192 + (s & 3) * 32), id, 1);
+            }
+            __syncwarp();
+            mma_commit(&mb_x);
+            if (!warp_wait(&mb_xready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 5); break; }
+            if (!warp_wait(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 3); break; }
+            tc_fence_after();
+            if (elect_one()) {   // U region <- W^T T~^T with W (hi, lo) packed in place in X (k-step s:
+                                 // hi at column 16 s, lo at 16 s + 8): W hi T~ hi + W hi T~ lo + W lo T~ hi
+                const uint32_t id = idesc_bf16(128, 64, 0, 0);
+                const uint32_t rb = (j & 1) * kRecSlot;
+#pragma unroll
+                for (int part = 0; part < 3; ++part) {
+#pragma unroll
+                    for (int s = 0; s < 4; ++s)
+                        mma_bf16_ta_1t(tm + TM_U, tm + TM_X + 16 * s + (part == 2 ? 8 : 0),
+                                       dadd(dR, rb + (part == 1 ? 8192 : 0) + s * 32), id, (part | s) != 0);
                 }
             }
-            fence_async_smem();
-            mbar_arrive(&mb_tready);
+            __syncwarp();
+            mma_commit(&mb_u);
+            mma_commit(&mb_re[j & 1]);                 // record slot free once MMA_U(j) has read T~
+            // the next tile's V^T into the X region (MMA_U(j), its last reader, is ahead in the pipe)
+            if (j + 1 < NJ && !issue_vi(j + 1)) { fail(a.status, abort_flag, 4); break; }
+            if (!warp_wait(&mb_uready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 7); break; }
+            tc_fence_after();
+            if (elect_one()) {   // S~ += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major)
+                const uint32_t id = idesc_bf16(128, 128, 0, 1);
+                const uint32_t kb = (j % 3) * 16384;
+#pragma unroll
+                for (int part = 0; part < 2; ++part) {
+#pragma unroll
+                    for (int s = 0; s < 4; ++s)
+                        mma_bf16_ta_1t(tm + TM_S, tm + TM_U + 16 * s + (part == 1 ? 8 : 0),
+                                       dadd(dK, kb + s * 2048), id, 1);
+                }
+            }
+            __syncwarp();
+            mma_commit(&mb_s);
+            mma_commit(&mb_ke[j % 3]);                 // K(j)'s buffer free once MMA_S(j) has read it
         }
-    } else {
-        // =========================================================== state chain (warps 0-7)
-        const int q = warp & 3, wg = warp >> 2;
-        const int r = 32 * q + lane;                       // row of S (value index)
-        const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-        const uint32_t cS = TM_S + 64 * wg;                // this thread's 64 state columns
-        float* sbefore = reinterpret_cast<float*>(sm + SM_SB);   // swizzled rows, see sb_idx
-        float* cg = reinterpret_cast<float*>(sm + SM_CG);
-        // a head's state (128 rows of the state viewed as [L * Hv * d_v][d_k]) into S_before by TMA,
-        // issued by thread 0 of the chain, completing on mb_st
-        int st_issued = 0, st_seen = 0;                    // state loads issued / waited for (uniform)
-        auto load_state = [&](int lh) {
-            ++st_issued;
-            if (tid == 0) {
+        if (__any_sync(0xffffffffu, *abort_flag != 0)) {
+            mma_commit(&mb_fin);                       // every MMA this warp issued has completed
+            mbar_wait(&mb_fin, 0, kWaitBudgetNs);
+        }
+        __syncwarp();
+    } else if (warp == kLoadWarp) {
+        // =========================================================== K, V, records in tile order,
+        // each into its buffer once the MMA that last read the buffer has completed
+        TileCursor cc;
+        cc.init(a);
+        int kp[3] = {-1, -1, -1}, vp[2] = {-1, -1}, rp[2] = {-1, -1};   // last tile loaded per buffer
+        for (int J = 0; J < NJ; ++J) {
+            const int bk = J % 3, b2 = J & 1;
+            if (J >= 3 && !warp_wait(&mb_ke[bk], ((J / 3) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 30); break; }
+            if (elect_one()) {
+                uint8_t* dst = sm + SM_K + bk * 16384;
+                mbar_arrive_expect_tx(&mb_tk[bk], 16384);
+                tma_load_4d(dst, &kmap, &mb_tk[bk], 0, cc.kh, cc.jt * kC, cc.l);
+                tma_load_4d(dst + 8192, &kmap, &mb_tk[bk], 64, cc.kh, cc.jt * kC, cc.l);
+            }
+            __syncwarp();
+            kp[bk] = J;
+            if (J >= 2 && !warp_wait(&mb_ve[b2], ((J >> 1) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 31); break; }
+            if (elect_one()) {
+                uint8_t* dst = sm + SM_V + b2 * 16384;
+                mbar_arrive_expect_tx(&mb_tv[b2], 16384);
+                tma_load_4d(dst, &vmap, &mb_tv[b2], 0, cc.h, cc.jt * kC, cc.l);
+                tma_load_4d(dst + 8192, &vmap, &mb_tv[b2], 64, cc.h, cc.jt * kC, cc.l);
+            }
+            __syncwarp();
+            vp[b2] = J;
+            if (J >= 2 && !warp_wait(&mb_re[b2], ((J >> 1) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 32); break; }
+            if (elect_one()) {
+                mbar_arrive_expect_tx(&mb_tr[b2], kRecBytes);
+                bulk_load_tx(sm + SM_R + b2 * kRecSlot, a.rec + ((size_t)cc.lh * n + cc.jt) * kRecBytes,
+                             kRecBytes, &mb_tr[b2]);
+            }
+            __syncwarp();
+            rp[b2] = J;
+            cc.next(n, a);
+        }
+        if (__any_sync(0xffffffffu, *abort_flag != 0) && lane == 0) {
+            // every copy this warp issued lands before the CTA ends
+            for (int b = 0; b < 3; ++b)
+                if (kp[b] >= 0) mbar_wait(&mb_tk[b], (kp[b] / 3) & 1, kWaitBudgetNs);
+            for (int b = 0; b < 2; ++b) {
+                if (vp[b] >= 0) mbar_wait(&mb_tv[b], (vp[b] >> 1) & 1, kWaitBudgetNs);
+                if (rp[b] >= 0) mbar_wait(&mb_tr[b], (rp[b] >> 1) & 1, kWaitBudgetNs);
+            }
+        }
+        __syncwarp();
+    } else if (warp == kStateWarp) {
+        // =========================================================== state moves (lane 0).  Phases
+        // of mb_st: 0 = the first head's state staged; k + 1 = what the boundary after slot k
+        // needs: the state of slot k + 1, or (after the last slot's) a free buffer.  Phases of
+        // mb_sfree: 0 = the first state is in TMEM; k + 1 = S_after of slot k is staged.
+        if (lane == 0 && n_slots > 0) {
+            float* sbuf = reinterpret_cast<float*>(sm + SM_SB);
+            int loads = 0, seen = 0;                   // copies into the staging buffer issued / landed
+            auto load_state = [&](int slot) {
+                const int lh = (int)blockIdx.x + slot * (int)gridDim.x;
                 mbar_arrive_expect_tx(&mb_st, kD * kD * 4);
 #pragma unroll
-                for (int b = 0; b < 4; ++b) tma_load_2d(sbefore + 4096 * b, &smap, &mb_st, 32 * b, lh * kD);
+                for (int b = 0; b < 4; ++b) tma_load_2d(sbuf + 4096 * b, &smap, &mb_st, 32 * b, lh * kD);
+                ++loads;
+            };
+            load_state(0);
+            bool ok = mbar_wait_or_abort(&mb_sfree, 0, kWaitBudgetNs, abort_flag);
+            if (!ok) fail(a.status, abort_flag, 40);
+            seen = loads;                              // the chain has consumed it
+            if (ok) {
+                if (n_slots > 1) load_state(1); else mbar_arrive(&mb_st);
             }
-        };
-        if (NJ > 0) load_state((int)blockIdx.x);
-        TileCursor cc;                                     // the chain's tile
+            for (int k = 0; ok && k < n_slots; ++k) {
+                if (!mbar_wait_or_abort(&mb_sfree, (k + 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 41); break; }
+                seen = loads;
+                const int lh = (int)blockIdx.x + k * (int)gridDim.x;
+#pragma unroll
+                for (int b = 0; b < 4; ++b) tma_store_2d(&smap, sbuf + 4096 * b, 32 * b, lh * kD);
+                bulk_commit();
+                if (k + 2 <= n_slots) {
+                    bulk_wait_read0();                 // S_after(k) has left the buffer
+                    if (k + 2 < n_slots) load_state(k + 2); else mbar_arrive(&mb_st);
+                }
+            }
+            bulk_wait0();                              // every state store is complete
+            if (loads > seen) mbar_wait(&mb_st, (loads - 1) & 1, kWaitBudgetNs);   // abort: a load in flight
+        }
+        __syncwarp();
+    } else {
+        // =========================================================== state chain (warps 0-15)
+        const int q = warp & 3, cgp = warp >> 2;         // TMEM lane quadrant, column group
+        const int r = 32 * q + lane;                     // row of S (value index)
+        const uint32_t lane_off = (uint32_t)(32 * q) << 16;
+        float* sbuf = reinterpret_cast<float*>(sm + SM_SB);   // swizzled rows, see sb_idx
+        int st_seen = 0;                                 // mb_st phases waited for (uniform)
+        TileCursor cc;                                   // the chain's tile
         cc.init(a);
-        // K(jj) bf16 (TMA tile, buffer jj % 3) -> fp32 copy for the tf32 X product.  Called between
-        // MMA_X(jj-1), the last reader of the copy, and the ready signal of tile jj.
-        auto k_to_fp32 = [&](int jj) -> bool {
+        // K'(jj) = K(jj) (TMA tile, buffer jj % 3) scaled per token t by gm[t] * xs = -gamma_t sig,
+        // rounded to tf32, into the B operand buffer of X.  Called between MMA_X(jj-1), the last
+        // reader of the buffer, and the ready signal of tile jj.
+        auto make_kprime = [&](int jj, float xs, const float* gm) -> bool {
             const bool ok = mbar_wait_or_abort(&mb_tk[jj % 3], (jj / 3) & 1, kWaitBudgetNs, abort_flag);
             const uint8_t* kb = sm + SM_K + (jj % 3) * 16384;
             uint8_t* k32 = sm + SM_K32;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {                  // 64 rows x 16 chunks of 8 bf16
+            for (int u = 0; u < 2; ++u) {                  // 64 rows x 16 chunks of 8 bf16
                 const int e = tid + kChain * u;
-                const int t = e >> 4, cc16 = e & 15, cb = cc16 >> 3, c = cc16 & 7;
+                const int t = e >> 4, c16 = e & 15, cb = c16 >> 3, c = c16 & 7;
+                const float sc = gm[t] * xs;
                 const uint4 w = *reinterpret_cast<const uint4*>(kb + cb * 8192 + sw128_offset(t, c));
                 const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
                 float f[8];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    f[2 * i] = __uint_as_float(wv[i] << 16);
-                    f[2 * i + 1] = __uint_as_float(wv[i] & 0xFFFF0000u);
+                    f[2 * i] = round_tf32(__uint_as_float(wv[i] << 16) * sc);
+                    f[2 * i + 1] = round_tf32(__uint_as_float(wv[i] & 0xFFFF0000u) * sc);
                 }
                 // dims 64 cb + 8 c .. + 7: fp32 block 2 cb + c / 4, chunks 2 (c % 4) and 2 (c % 4) + 1
                 uint8_t* rowp = k32 + (2 * cb + (c >> 2)) * 8192;
@@ -660,155 +825,157 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             fence_async_smem();                            // generic writes -> the tensor core's reads
             return ok;
         };
+        auto rec_consts = [&](int jj) {                    // -gamma[64], gamma_C of tile jj's record
+            return reinterpret_cast<const float*>(sm + SM_R + (jj & 1) * kRecSlot + kRecT);
+        };
         float den = 0.f;
         // Deferred decay: TMEM holds S~ with the head's state S = sig * S~.  A tile folds its decay
-        // gamma_C into sig (X is rescaled by sig in the X~ pass, U~ by 1 / (gamma_C sig) in the U~
-        // pass, so MMA_S accumulates onto S~ with no pass over the state); when sig gamma_C would
-        // drop below kSigMin the tile instead writes gamma_C S back into TMEM and sig restarts at 1.
+        // gamma_C into sig (K' carries sig, W is scaled by u_scale = 1 / (gamma_C sig), so MMA_S
+        // accumulates onto S~ with no pass over the state); when sig gamma_C would drop below
+        // kSigMin the tile instead writes gamma_C S back into TMEM and sig restarts at 1.
         float sig = 1.f;
         for (int j = 0; j < NJ; ++j) {                     // j: global tile index
             const int lh = cc.lh, jt = cc.jt;              // head and tile within the head
-            float* gam = cg + (j % 3) * 132;               // -gamma (written by the T builders)
-            float* del = gam + 64;                         // exp(G_C - G)
+            const bool last = jt == n - 1;
             if (named_sync_or(2, kChain, *abort_flag)) break;
-            if (!mbar_wait_or_abort(&mb_cready[j % 3], (j / 3) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
-            const float gC = gam[128];
+            if (!mbar_wait_or_abort(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
+            const float gC = rec_consts(j)[64];
 
-            if (jt == 0) {
-                // ---- a head's first tile: its state (TMA-loaded into S_before at the previous
-                // head's end) into TMEM as S~ with sig = 1, and sum S_before^2
-                if (!mbar_wait_or_abort(&mb_st, (j / n) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 14);
-                ++st_seen;
-                if (j + n < NJ) {                          // the next head's state towards L2
-                    const char* nxt = reinterpret_cast<const char*>(a.state + (size_t)(lh + (int)gridDim.x) * kD * kD);
-                    asm volatile("prefetch.L2 [%0];" :: "l"(nxt + 256 * tid) : "memory");
-                    asm volatile("prefetch.L2 [%0];" :: "l"(nxt + 256 * tid + 128) : "memory");
+            if (j == 0) {
+                // ---- the CTA's first head: its state from the staging buffer into TMEM, as S~
+                // (sig = 1) and as S_before, and sum S_before^2
+                if (!mbar_wait_or_abort(&mb_st, 0, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 14);
+                st_seen = 1;
+                float sv[32];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, 8 * cgp + e));
+                    sv[4 * e] = x.x; sv[4 * e + 1] = x.y; sv[4 * e + 2] = x.z; sv[4 * e + 3] = x.w;
                 }
 #pragma unroll
-                for (int half = 0; half < 2; ++half) {
-                    float sv[32];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float4 x = *reinterpret_cast<const float4*>(sbefore + sb_idx(r, 16 * wg + 8 * half + e));
-                        sv[4 * e] = x.x; sv[4 * e + 1] = x.y; sv[4 * e + 2] = x.z; sv[4 * e + 3] = x.w;
-                    }
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) den += sv[e] * sv[e];
-                    tmem_st32(tm + lane_off + cS + 32 * half, sv);
-                }
-                sig = 1.f;
-                if (j == 0 && !k_to_fp32(0)) fail(a.status, abort_flag, 16);
+                for (int e = 0; e < 32; ++e) den = fmaf(sv[e], sv[e], den);
+                mbar_arrive(&mb_sfree);                    // the staging buffer has been read
+                tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
+                tmem_st32(tm + lane_off + TM_SB + 32 * cgp, sv);
+                if (!make_kprime(0, 1.f, rec_consts(0))) fail(a.status, abort_flag, 16);
                 tmem_st_wait();
                 tc_fence_before();
                 mbar_arrive(&mb_sready);
             }
             const bool rescale = sig * gC < kSigMin;       // uniform over the CTA
-            const float x_scale = sig;                     // X = sig * (K S~^T)
             const float u_scale = rescale ? 1.f : 1.f / (gC * sig);
 
-            // ---- X~^T = -X^T diag(gamma): (hi, lo) packed in place over this thread's 32 X columns
+            // ---- W pass: the X region holds W^T = V^T - X^T diag(gamma); scaled by u_scale, (hi,
+            // lo) in place over this thread's 16 columns (tokens 16 cgp ..)
             if (!mbar_wait_or_abort(&mb_x, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 10);
             tc_fence_after();
             {
-                float xv[32];
-                tmem_ld32(tm + lane_off + TM_X + 32 * wg, xv);
+                float wv[16];
+                tmem_ld16(tm + lane_off + TM_X + 16 * cgp, wv);
                 tmem_ld_wait();
-                uint32_t hi[16], lo[16];
+                uint32_t hi[8], lo[8];
 #pragma unroll
-                for (int c4 = 0; c4 < 8; ++c4) {
-                    float4 g4 = *reinterpret_cast<const float4*>(gam + 32 * wg + 4 * c4);
-                    g4.x *= x_scale; g4.y *= x_scale; g4.z *= x_scale; g4.w *= x_scale;
-                    split2(g4.x * xv[4 * c4], g4.y * xv[4 * c4 + 1], hi[2 * c4], lo[2 * c4]);
-                    split2(g4.z * xv[4 * c4 + 2], g4.w * xv[4 * c4 + 3], hi[2 * c4 + 1], lo[2 * c4 + 1]);
-                }
-                tmem_st16(tm + lane_off + TM_X + 32 * wg, hi);
-                tmem_st16(tm + lane_off + TM_X + 32 * wg + 16, lo);
+                for (int i = 0; i < 8; ++i) split2(wv[2 * i] * u_scale, wv[2 * i + 1] * u_scale, hi[i], lo[i]);
+                tmem_st8(tm + lane_off + TM_X + 16 * cgp, hi);
+                tmem_st8(tm + lane_off + TM_X + 16 * cgp + 8, lo);
                 tmem_st_wait();
             }
             tc_fence_before();
             mbar_arrive(&mb_xready);
 
             // ---- while MMA_U runs: rescale S~ if the decay would underflow the deferred scale
-            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and the fp32 copy of K(j+1)
+            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K'(j+1)
             if (rescale) {
                 const float f = gC * sig;
+                float sv[32];
+                tmem_ld32(tm + lane_off + TM_S + 32 * cgp, sv);
+                tmem_ld_wait();
 #pragma unroll
-                for (int half = 0; half < 2; ++half) {
-                    float sv[32];
-                    tmem_ld32(tm + lane_off + cS + 32 * half, sv);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) sv[e] *= f;
-                    tmem_st32(tm + lane_off + cS + 32 * half, sv);
-                }
+                for (int e = 0; e < 32; ++e) sv[e] *= f;
+                tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
                 tmem_st_wait();
             }
-            if (j + 1 < NJ && !k_to_fp32(j + 1)) fail(a.status, abort_flag, 16);
+            sig = rescale ? 1.f : gC * sig;                // the deferred decay after tile j
+            if (j + 1 < NJ) {
+                // K'(j+1): its tile's -gamma and the sig it starts with (1 at a head's first tile)
+                if (!mbar_wait_or_abort(&mb_tr[(j + 1) & 1], ((j + 1) >> 1) & 1, kWaitBudgetNs, abort_flag))
+                    fail(a.status, abort_flag, 15);
+                if (!make_kprime(j + 1, last ? 1.f : sig, rec_consts(j + 1))) fail(a.status, abort_flag, 16);
+            }
 
-            // ---- U~^T = U^T diag(exp(G_C - G)) / (gamma_C sig): (hi, lo) packed in place over U
+            // ---- U~ pass: (hi, lo) in place over this thread's 16 U columns
             if (!mbar_wait_or_abort(&mb_u, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 11);
             tc_fence_after();
             {
-                float uv[32];
-                tmem_ld32(tm + lane_off + TM_U + 32 * wg, uv);
+                float uv[16];
+                tmem_ld16(tm + lane_off + TM_U + 16 * cgp, uv);
                 tmem_ld_wait();
-                uint32_t hi[16], lo[16];
+                uint32_t hi[8], lo[8];
 #pragma unroll
-                for (int c4 = 0; c4 < 8; ++c4) {
-                    float4 d4 = *reinterpret_cast<const float4*>(del + 32 * wg + 4 * c4);
-                    d4.x *= u_scale; d4.y *= u_scale; d4.z *= u_scale; d4.w *= u_scale;
-                    split2(uv[4 * c4] * d4.x, uv[4 * c4 + 1] * d4.y, hi[2 * c4], lo[2 * c4]);
-                    split2(uv[4 * c4 + 2] * d4.z, uv[4 * c4 + 3] * d4.w, hi[2 * c4 + 1], lo[2 * c4 + 1]);
-                }
-                tmem_st16(tm + lane_off + TM_U + 32 * wg, hi);
-                tmem_st16(tm + lane_off + TM_U + 32 * wg + 16, lo);
+                for (int i = 0; i < 8; ++i) split2(uv[2 * i], uv[2 * i + 1], hi[i], lo[i]);
+                tmem_st8(tm + lane_off + TM_U + 16 * cgp, hi);
+                tmem_st8(tm + lane_off + TM_U + 16 * cgp + 8, lo);
                 tmem_st_wait();
             }
             tc_fence_before();
             mbar_arrive(&mb_uready);
-            sig = rescale ? 1.f : gC * sig;
-            // the next tile of this head may start X as soon as MMA_S(j) is queued
-            if (jt < n - 1) mbar_arrive(&mb_sready);
-
-            if (jt == n - 1) {
-                // ---- epilogue of the head: S_after -> HBM, drift partials against S_before
-                const bool ok = mbar_wait_or_abort(&mb_s, j & 1, kWaitBudgetNs, abort_flag);
+            if (!last) {
+                // the next tile of this head may start X as soon as MMA_S(j) is queued
+                mbar_arrive(&mb_sready);
+            } else {
+                // ---- head boundary: S_after = sig S~ out through the staging buffer, the next
+                // head's state (staged meanwhile) into TMEM, drift partials against S_before
+                const bool has_next = j + 1 < NJ;          // uniform
+                bool ok = mbar_wait_or_abort(&mb_s, j & 1, kWaitBudgetNs, abort_flag);
                 if (!ok) fail(a.status, abort_flag, 12);
+                if (!mbar_wait_or_abort(&mb_st, st_seen & 1, kWaitBudgetNs, abort_flag)) {
+                    fail(a.status, abort_flag, 14);
+                    ok = false;
+                }
+                ++st_seen;
                 tc_fence_after();
-                float num = 0.f;
+                float num = 0.f, den_next = 0.f;
                 if (ok) {
-                    // S_after = sig S~ replaces S_before in shared memory (each thread its own row) ...
 #pragma unroll
                     for (int half = 0; half < 2; ++half) {
-                        float sv[32];
-                        tmem_ld32(tm + lane_off + cS + 32 * half, sv);
+                        const uint32_t col = 32 * cgp + 16 * half;
+                        const int ch = 8 * cgp + 4 * half;     // this half's 16-byte chunks of row r
+                        float sa[16], sb[16];
+                        tmem_ld16(tm + lane_off + TM_S + col, sa);
+                        tmem_ld16(tm + lane_off + TM_SB + col, sb);
                         tmem_ld_wait();
 #pragma unroll
-                        for (int e = 0; e < 32; ++e) sv[e] *= sig;
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            float4* p = reinterpret_cast<float4*>(sbefore + sb_idx(r, 16 * wg + 8 * half + e));
-                            const float4 b = *p;
-                            const float d0 = sv[4 * e] - b.x, d1 = sv[4 * e + 1] - b.y;
-                            const float d2 = sv[4 * e + 2] - b.z, d3 = sv[4 * e + 3] - b.w;
-                            num += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
-                            *p = make_float4(sv[4 * e], sv[4 * e + 1], sv[4 * e + 2], sv[4 * e + 3]);
+                        for (int e = 0; e < 16; ++e) {
+                            sa[e] *= sig;
+                            const float d = sa[e] - sb[e];
+                            num = fmaf(d, d, num);
                         }
+                        if (has_next) {
+                            uint32_t sn[16];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
+                                den_next = fmaf(x.x, x.x, den_next); den_next = fmaf(x.y, x.y, den_next);
+                                den_next = fmaf(x.z, x.z, den_next); den_next = fmaf(x.w, x.w, den_next);
+                                sn[4 * e] = __float_as_uint(x.x); sn[4 * e + 1] = __float_as_uint(x.y);
+                                sn[4 * e + 2] = __float_as_uint(x.z); sn[4 * e + 3] = __float_as_uint(x.w);
+                            }
+                            tmem_st16(tm + lane_off + TM_S + col, sn);
+                            tmem_st16(tm + lane_off + TM_SB + col, sn);
+                        }
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            *reinterpret_cast<float4*>(sbuf + sb_idx(r, ch + e)) =
+                                make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
                     }
+                    tmem_st_wait();
                 }
                 tc_fence_before();
-                fence_async_smem();
-                // ... and goes to HBM by TMA; once TMA has read it out, the next head's state
-                // comes in
-                if (named_sync_or(2, kChain, !ok)) break;
-                if (tid == 0) {
-#pragma unroll
-                    for (int b = 0; b < 4; ++b) tma_store_2d(&smap, sbefore + 4096 * b, 32 * b, lh * kD);
-                    bulk_commit();
-                    bulk_wait_read0();
-                }
-                if (j + 1 < NJ) load_state(lh + (int)gridDim.x);
-                // partial sums: float within a warp (the FP64 pipe is slow), double across warps
+                fence_async_smem();                        // S_after -> the state warp's TMA store
+                mbar_arrive(&mb_sfree);
+                if (has_next) mbar_arrive(&mb_sready);     // the next head's state is in TMEM
+                // partial sums: pairwise in fp32, over the warp's lanes and then over the 16 warps
+                // (the FP64 pipe is far too slow for this path)
                 float fn = num, fd = den;
 #pragma unroll
                 for (int m = 16; m >= 1; m >>= 1) {
@@ -816,28 +983,30 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     fd += __shfl_xor_sync(0xffffffffu, fd, m);
                 }
                 if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
-                const bool any_fail = named_sync_or(2, kChain, !ok);
-                if (tid == 0 && !any_fail && a.partials != nullptr) {
-                    double sn = 0.0, sd = 0.0;
-                    for (int w = 0; w < 8; ++w) { sn += s_red[0][w]; sd += s_red[1][w]; }
-                    a.partials[(size_t)lh * 2 + 0] = (float)sn;
-                    a.partials[(size_t)lh * 2 + 1] = (float)sd;
+                if (named_sync_or(2, kChain, !ok)) break;
+                if (warp == 0 && a.partials != nullptr) {
+                    float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
+                    float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
+#pragma unroll
+                    for (int m = kChainWarps / 2; m >= 1; m >>= 1) {
+                        pn += __shfl_xor_sync(0xffffffffu, pn, m);
+                        pd += __shfl_xor_sync(0xffffffffu, pd, m);
+                    }
+                    if (lane == 0) {
+                        a.partials[(size_t)lh * 2 + 0] = pn;
+                        a.partials[(size_t)lh * 2 + 1] = pd;
+                    }
                 }
-                if (any_fail) break;
-                den = 0.f;
+                den = den_next;
+                sig = 1.f;
             }
             cc.next(n, a);
-        }
-        if (tid == 0) {
-            bulk_wait0();                                  // the last state store is complete
-            // abort path: a state load issued but not waited for lands before the CTA ends
-            if (st_issued > st_seen) mbar_wait(&mb_st, (st_issued - 1) & 1, kWaitBudgetNs);
         }
     }
 
     tc_fence_before();
     __syncthreads();
-    if (warp == kCtlWarp) {
+    if (warp == kMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tm, kTmemCols);
     }
@@ -891,9 +1060,18 @@ bool make_state_map(CUtensorMap* map, void* base, int heads) {
 
 }  // namespace
 
+size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T) {
+    if (dk != kD || dv != kD || dtype != DELTAS_BF16 || L <= 0 || Hv <= 0 || T <= 0) return 0;
+    return (size_t)L * Hv * ((T + kC - 1) / kC) * kRecBytes;
+}
+
 bool gdn_tc_supported(const GdnArgs& a) {
     return a.dk == kD && a.dv == kD && a.dtype == DELTAS_BF16 && a.out == nullptr && a.T > 0 &&
-           (long long)a.L * a.Hv * kD < (1ll << 31) && encode_fn() != nullptr;   // TMA row coordinate
+           (long long)a.L * a.Hv * kD < (1ll << 31) &&                          // TMA row coordinate
+           (long long)a.L * a.Hv * ((a.T + kC - 1) / kC) < (1ll << 31) &&       // factor-kernel items
+           a.scratch != nullptr &&
+           a.scratch_bytes >= gdn_tc_scratch_bytes(a.L, a.Hv, a.dk, a.dv, a.dtype, a.T) &&
+           encode_fn() != nullptr;
 }
 
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
@@ -907,15 +1085,28 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     if (configured_device != dev) {
         cudaError_t e = cudaFuncSetAttribute(gdn_update_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)kSmemAlloc);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(gdn_wy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kWySmemAlloc);
         if (e != cudaSuccess) return e;
         configured_device = dev;
     }
+    const int n_tiles = (a.T + kC - 1) / kC;
+    const int sms = device_sm_count();
+    // factor kernel: one record per (layer, value head, tile), kWyCtasPerSm persistent CTAs per SM
+    WyArgs w;
+    w.L = a.L; w.Hk = a.Hk; w.Hv = a.Hv; w.T = a.T; w.n_tiles = n_tiles;
+    w.g = a.g; w.beta = a.beta; w.rec = a.scratch; w.status = a.status;
+    const long long items = (long long)a.L * a.Hv * n_tiles;
+    const int wgrid = (int)std::min<long long>(items, (long long)sms * kWyCtasPerSm);
+    gdn_wy_kernel<<<wgrid, kWyThreads, kWySmemAlloc, s>>>(kmap, w);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // update kernel: one persistent CTA per SM (the kernel needs the whole SM: 512 TMEM columns,
+    // ~211 KB of shared memory); each takes every grid-th head
     TcArgs t;
-    t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = (a.T + kC - 1) / kC;
-    t.state = a.state; t.partials = a.partials; t.g = a.g; t.beta = a.beta; t.status = a.status;
-    // one persistent CTA per SM (the kernel needs the whole SM: 512 TMEM columns, ~206 KB of
-    // shared memory); each takes every grid-th head
-    const int grid = std::min(a.L * a.Hv, device_sm_count());
+    t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = n_tiles;
+    t.state = a.state; t.partials = a.partials; t.rec = a.scratch; t.status = a.status;
+    const int grid = std::min(a.L * a.Hv, sms);
     gdn_update_tc_kernel<<<grid, kThreads, kSmemAlloc, s>>>(kmap, vmap, smap, t);
     return cudaGetLastError();
 }

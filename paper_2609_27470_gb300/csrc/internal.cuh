@@ -54,6 +54,8 @@ struct GdnArgs {
     void* out;
     float* partials;
     int32_t* status;
+    uint8_t* scratch;        // workspace past the status word (the tensor-core path's WY factors)
+    size_t scratch_bytes;
 };
 
 struct KvPlanes {
@@ -67,6 +69,7 @@ struct KvPlanes {
 // Kernel launchers (return the launch error, cudaSuccess when enqueued).
 cudaError_t launch_gdn_update_simt(const GdnArgs& a, cudaStream_t s);
 bool gdn_tc_supported(const GdnArgs& a);
+size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T);
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s);
 cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, const float* sa,
                                float* partials, cudaStream_t s);
