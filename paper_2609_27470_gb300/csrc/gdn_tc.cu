@@ -174,6 +174,48 @@ __device__ __forceinline__ void mma_3xtf32(float (&d)[4], FA A, FB B, int lane) 
     }
 }
 
+// D (16 x 8) += A (16 x 16, row) B (16 x 8, col) on the warp's tensor-core path, bf16 in, fp32
+// accumulate.  Fragments (g = lane / 4, t = lane % 4), each register a bf16 pair, lower k in the
+// low half: a = A[g][2t..], A[g+8][2t..], A[g][2t+8..], A[g+8][2t+8..]; b = B[2t..][g],
+// B[2t+8..][g]; d as for the tf32 form.
+__device__ __forceinline__ void mma_m16n8k16_bf16(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                 "{%0,%1,%2,%3};"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+// A 32 x 32 operand stored split: row r is 32 words at rows + r * stride, words 0..15 the bf16
+// pairs (2p, 2p+1) of hi = bf16(x), words 16..31 those of lo = bf16(x - hi).  D (16 x 8) +=
+// A[r0 .. r0+15][0..32) B[0..32)[n0 .. n0+7] over the three products lo*hi + hi*lo + hi*hi, A
+// row-major and B stored n-major (row n of B's storage holds column n of B).
+__device__ __forceinline__ void mma_32_split_bf16(float (&d)[4], const uint32_t* A, int as, int r0,
+                                                  const uint32_t* B, int bs, int n0, int lane) {
+    const int g = lane >> 2, t = lane & 3;
+    const uint32_t* a0 = A + (r0 + g) * as;
+    const uint32_t* a1 = A + (r0 + g + 8) * as;
+    const uint32_t* b0 = B + (n0 + g) * bs;
+#pragma unroll
+    for (int ks = 0; ks < 2; ++ks) {
+        const int p0 = 8 * ks + t, p1 = p0 + 4;
+        const uint32_t ah[4] = {a0[p0], a1[p0], a0[p1], a1[p1]};
+        const uint32_t al[4] = {a0[16 + p0], a1[16 + p0], a0[16 + p1], a1[16 + p1]};
+        const uint32_t bh[2] = {b0[p0], b0[p1]};
+        const uint32_t bl[2] = {b0[16 + p0], b0[16 + p1]};
+        mma_m16n8k16_bf16(d, al, bh);
+        mma_m16n8k16_bf16(d, ah, bl);
+        mma_m16n8k16_bf16(d, ah, bh);
+    }
+}
+
+// One element of a split row (see mma_32_split_bf16): hi / lo halfwords of column k of row `row`.
+__device__ __forceinline__ void put_split(uint32_t* row, int k, float x) {
+    const __nv_bfloat16 h = __float2bfloat16_rn(x);
+    const __nv_bfloat16 l = __float2bfloat16_rn(x - __bfloat162float(h));
+    reinterpret_cast<__nv_bfloat16*>(row)[k] = h;
+    reinterpret_cast<__nv_bfloat16*>(row + 16)[k] = l;
+}
+
 // 2^x with the hardware approximation (relative error about 2^-22)
 __device__ __forceinline__ float fast_exp2(float x) {
     float y;
@@ -194,6 +236,13 @@ __device__ __forceinline__ void fail(int32_t* status, volatile int* abort, int w
     *abort = 1;
 }
 
+// One arrival per warp on a chain -> MMA barrier: every lane's TMEM stores / shared-memory
+// writes were completed and fenced before the __syncwarp; lane 0 then arrives (release).
+__device__ __forceinline__ void warp_arrive(uint64_t* bar, int lane) {
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar);
+}
+
 // shared-memory descriptor advanced by `bytes` (the start address field counts 16-byte units)
 __device__ __forceinline__ uint64_t dadd(uint64_t desc, uint32_t bytes) { return desc + (uint64_t)(bytes >> 4); }
 
@@ -201,18 +250,25 @@ __device__ __forceinline__ uint64_t dadd(uint64_t desc, uint32_t bytes) { return
 // Factor kernel: T~ = diag(exp(G_C - G)) (I + A)^-1 diag(beta) and the decay constants of every tile
 // =============================================================================================
 constexpr int kWyThreads = 256;
-constexpr int kWyCtasPerSm = 3;
+constexpr int kWyCtasPerSm = 4;
 constexpr uint32_t kWyTmemCols = 64;
 constexpr int FA_S = 68;               // fp32 row stride of A: 16-byte rows; a 16-byte access by 8 threads
                                        // of 8 consecutive rows hits 8 distinct bank groups
 constexpr int FX_S = 68;               // fp32 row stride of X = (I + A)^-1 (16-byte aligned rows)
 // shared-memory map (bytes from a 1024-aligned base)
-constexpr uint32_t WY_K = 0;                          // K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
-constexpr uint32_t WY_FA = 16384;                     // fp32 [64][FA_S]; the M = 128 product of K K^T reads its
-                                                      // first 8 KB as rows 64..127 of A (output ignored)
-constexpr uint32_t WY_FX = WY_FA + 64 * FA_S * 4;     // fp32 [64][FX_S]
-constexpr uint32_t WY_TMP = WY_FX + 64 * FX_S * 4;    // fp32 [32][33]
-constexpr uint32_t WY_TG = WY_TMP + 32 * 33 * 4;      // 2 buffers (item parity) x (G2[64], beta[64], row[64],
+constexpr uint32_t WY_FA = 0;                         // fp32 [64][FA_S].  Its two 32 x 32 quarters that are
+                                                      // never read as fp32 hold split operands of level 2:
+                                                      // rows 32..63 x cols 0..31 = A21 (row-major), rows
+                                                      // 0..31 x cols 32..63 = X11 stored n-major
+constexpr uint32_t WY_K = WY_FA;                      // the next item's K tile (2 column blocks (d 0-63,
+                                                      // 64-127) x 64 rows x 128 B) lands over A once level 2
+                                                      // has read it; the M = 128 product of K K^T reads the
+                                                      // 8 KB past the tile as rows 64..127 (output ignored)
+constexpr uint32_t WY_FX = WY_FA + 64 * FA_S * 4;     // fp32 [64][FX_S]; rows 0..31 x cols 32..63 (the zero
+                                                      // upper quarter) hold X22 split, row-major
+constexpr uint32_t WY_TMP = WY_FX + 64 * FX_S * 4;    // level 1 products (fp32), then level 2's P split,
+                                                      // n-major, rows of 36 words
+constexpr uint32_t WY_TG = WY_TMP + 32 * 36 * 4;      // 2 buffers (item parity) x (G2[64], beta[64], row[64],
                                                       // col[64], del[64], flag)
 constexpr uint32_t kTgFloats = 324;
 constexpr uint32_t WY_BYTES = WY_TG + 2 * kTgFloats * 4;
@@ -242,6 +298,12 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
     float* fA = reinterpret_cast<float*>(sm + WY_FA);
     float* fX = reinterpret_cast<float*>(sm + WY_FX);
     float* fT = reinterpret_cast<float*>(sm + WY_TMP);
+    // split level-2 operands (see the shared-memory map), row strides in 32-bit words
+    uint32_t* sA21 = reinterpret_cast<uint32_t*>(fA + 32 * FA_S);        // A[32 + r][k]
+    uint32_t* sX11 = reinterpret_cast<uint32_t*>(fA + 32);               // row n: X[k][n], k < 32
+    uint32_t* sX22 = reinterpret_cast<uint32_t*>(fX + 32);               // row r: X[32 + r][32 + k]
+    uint32_t* sP = reinterpret_cast<uint32_t*>(fT);                      // row n: P[k][n]
+    constexpr int kPS = 36;
 
     if (warp == 0) { tmem_alloc(&s_tmem, kWyTmemCols); tmem_relinquish(); }
     if (tid == 0) {
@@ -252,7 +314,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
     }
     // The strictly upper 16 x 16 blocks of X are never written; zeros there let every level run
     // fixed-length (unrolled) loops over the triangular factors.
-    for (int e = tid; e < 64 * FX_S; e += kWyThreads) fX[e] = 0.f;
+    for (int e = tid; e < 64 * FX_S; e += kWyThreads) { fX[e] = 0.f; fA[e] = 0.f; }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -262,9 +324,11 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         const int lh = it / n;
         jt = it - lh * n; l = lh / a.Hv; h = lh - l * a.Hv;
     };
+    int nk = 0, nkk = 0;                               // K loads (thread 0) / K K^T products (warp 0) issued
     auto load_k = [&](int it) {                        // thread 0: the item's K tile
         int l, h, jt;
         item_pos(it, l, h, jt);
+        ++nk;
         const int kh = (int)(((long long)h * a.Hk) / a.Hv);
         mbar_arrive_expect_tx(&mb_k, 16384);
         tma_load_4d(sm + WY_K, &kmap, &mb_k, 0, kh, jt * kC, l);
@@ -318,6 +382,25 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         if (lane == 0) reinterpret_cast<int*>(tg)[320] = (hi2 - lo2) <= 250.f;
     };
 
+    // K K^T of the item-th item of this CTA into TMEM (warp 0; M = 128: rows 64..127 of A read the
+    // 8 KB past the tile, their output is ignored)
+    auto issue_kk = [&](int item) {
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&mb_k, item & 1, kWaitBudgetNs)) != 0;
+        if (!ok) {
+            if (lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 21); s_fail = 1; }
+            return;
+        }
+        tc_fence_after();
+        const uint32_t id = idesc_bf16(128, 64, 0, 0);
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {
+            const uint64_t d = sdesc_sw128(smem_u32(sm + WY_K + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
+            mma_bf16(tm, d, d, id, s > 0);
+        }
+        mma_commit(&mb_kk);
+        ++nkk;
+    };
+
     const int first = (int)blockIdx.x;
     if (first < items) {
         if (tid == 0) load_k(first);
@@ -337,65 +420,57 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         const float* sCol = tg + 192;                  // 2^(ref - G2_i)
         const float* sDel = tg + 256;                  // exp(G_C - G_t)
         const int factored = reinterpret_cast<const int*>(tg)[320];
-        // K K^T (M = 128: rows 64..127 of A read the 8 KB past the tile; their output is ignored)
-        if (warp == 0) {
-            const bool ok = __all_sync(0xffffffffu, mbar_wait(&mb_k, c & 1, kWaitBudgetNs)) != 0;
-            if (!ok) {
-                if (lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 21); s_fail = 1; }
-            } else {
-                tc_fence_after();
-                const uint32_t id = idesc_bf16(128, 64, 0, 0);
-#pragma unroll
-                for (int s = 0; s < 8; ++s) {
-                    const uint64_t d = sdesc_sw128(smem_u32(sm + WY_K + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
-                    mma_bf16(tm, d, d, id, s > 0);
-                }
-                mma_commit(&mb_kk);
-            }
-        }
+        if (warp == 0) issue_kk(c);
         const int q = warp & 3;
-        if (q < 2) {
+        if (q < 2 && warp != 4) {
             // TMEM lanes 0..63 hold K K^T: warps 0/4 rows 0..31, 1/5 rows 32..63; column half
-            // (warp >> 2).
+            // (warp >> 2).  Warp 4's quarter (rows 0..31, cols 32..63) lies above the diagonal and
+            // is never needed; warp 1's (rows 32..63, cols 0..31) is A21, stored split.
             const bool ok = mbar_wait_or_abort(&mb_kk, c & 1, kWaitBudgetNs, &s_fail);
             if (!ok && lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 22); s_fail = 1; }
             tc_fence_after();
             const int t = 32 * q + lane, c0 = 32 * (warp >> 2);
             const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-            float kk[32], cf[32];
-            tmem_ld32(tm + lane_off + c0, kk);
-            if (factored) {
-                const float rt = sRow[t];
+            const float rt = factored ? sRow[t] : sBeta[t];
+            const float G2t = sG2[t];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float4 v4 = *reinterpret_cast<const float4*>(sCol + c0 + 4 * e);
+            for (int half = 0; half < 2; ++half) {     // 16 columns at a time
+                const int cb = c0 + 16 * half;
+                float kk[16], cf[16];
+                tmem_ld16(tm + lane_off + cb, kk);
+                const float* src = factored ? sCol : sG2;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float4 v4 = *reinterpret_cast<const float4*>(src + cb + 4 * e);
                     cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
                 }
                 tmem_ld_wait();
 #pragma unroll
-                for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? rt * cf[e] * kk[e] : 0.f;
-            } else {
-                const float G2t = sG2[t], bt = sBeta[t];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float4 v4 = *reinterpret_cast<const float4*>(sG2 + c0 + 4 * e);
-                    cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
+                for (int e = 0; e < 16; ++e) {
+                    const float f = factored ? cf[e] : fast_exp2(G2t - cf[e]);
+                    kk[e] = (cb + e < t) ? rt * f * kk[e] : 0.f;
                 }
-                tmem_ld_wait();
+                if (warp == 1) {                       // A21, split
+                    uint32_t* row = sA21 + (t - 32) * FA_S + 8 * half;
+                    uint32_t h[8], l[8];
 #pragma unroll
-                for (int e = 0; e < 32; ++e) kk[e] = (c0 + e < t) ? bt * fast_exp2(G2t - cf[e]) * kk[e] : 0.f;
+                    for (int i = 0; i < 8; ++i) split2(kk[2 * i], kk[2 * i + 1], h[i], l[i]);
+                    *reinterpret_cast<uint4*>(row) = make_uint4(h[0], h[1], h[2], h[3]);
+                    *reinterpret_cast<uint4*>(row + 4) = make_uint4(h[4], h[5], h[6], h[7]);
+                    *reinterpret_cast<uint4*>(row + 16) = make_uint4(l[0], l[1], l[2], l[3]);
+                    *reinterpret_cast<uint4*>(row + 20) = make_uint4(l[4], l[5], l[6], l[7]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        *reinterpret_cast<float4*>(fA + t * FA_S + cb + 4 * e) =
+                            make_float4(kk[4 * e], kk[4 * e + 1], kk[4 * e + 2], kk[4 * e + 3]);
+                }
             }
-#pragma unroll
-            for (int e = 0; e < 8; ++e)
-                *reinterpret_cast<float4*>(fA + t * FA_S + c0 + 4 * e) =
-                    make_float4(kk[4 * e], kk[4 * e + 1], kk[4 * e + 2], kk[4 * e + 3]);
         }
         tc_fence_before();
         __syncthreads();
         if (s_fail) break;
-        // K K^T is in fA: the K tile and the TMEM columns are free for the next item
         const int nxt = it + (int)gridDim.x;
-        if (tid == 0 && nxt < items) load_k(nxt);
         // level 0: four 16 x 16 diagonal blocks of (I + A)^-1, one column per thread (warps 0-1);
         // meanwhile warp 7 prepares the next item's constants and loads the one after
         if (tid < 64) {
@@ -418,6 +493,25 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
             }
 #pragma unroll
             for (int rr = 0; rr < 16; ++rr) fX[(o + rr) * FX_S + o + jc] = x[rr];
+            if (B < 2) {                               // X11, n-major: row o + jc holds column o + jc
+                uint32_t* row = sX11 + (o + jc) * FA_S;
+                if (B == 1) {                          // X[0..16][16..32] = 0 (the K tile overwrote it)
+                    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+                    *reinterpret_cast<uint4*>(row) = z; *reinterpret_cast<uint4*>(row + 4) = z;
+                    *reinterpret_cast<uint4*>(row + 16) = z; *reinterpret_cast<uint4*>(row + 20) = z;
+                }
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    uint32_t h[4], l[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) split2(x[8 * e + 2 * i], x[8 * e + 2 * i + 1], h[i], l[i]);
+                    *reinterpret_cast<uint4*>(row + o / 2 + 4 * e) = make_uint4(h[0], h[1], h[2], h[3]);
+                    *reinterpret_cast<uint4*>(row + 16 + o / 2 + 4 * e) = make_uint4(l[0], l[1], l[2], l[3]);
+                }
+            } else {                                   // X22, row-major
+#pragma unroll
+                for (int rr = 0; rr < 16; ++rr) put_split(sX22 + (o - 32 + rr) * FX_S, o - 32 + jc, x[rr]);
+            }
         } else if (warp == 7 && nxt < items) {
             tile_constants(nxt, (c + 1) & 1);
             if (nxt + (int)gridDim.x < items) load_gb(nxt + (int)gridDim.x);
@@ -446,24 +540,38 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
                              [&](int k, int cc) { return P[k * 17 + nc + cc]; }, lane);
             fX[(ro + g) * FX_S + co + nc + 2 * tq] = -d[0]; fX[(ro + g) * FX_S + co + nc + 2 * tq + 1] = -d[1];
             fX[(ro + g + 8) * FX_S + co + nc + 2 * tq] = -d[2]; fX[(ro + g + 8) * FX_S + co + nc + 2 * tq + 1] = -d[3];
+            if (p == 0) {                              // X[16..32][0..16] into X11, n-major
+                put_split(sX11 + (nc + 2 * tq) * FA_S, 16 + g, -d[0]);
+                put_split(sX11 + (nc + 2 * tq + 1) * FA_S, 16 + g, -d[1]);
+                put_split(sX11 + (nc + 2 * tq) * FA_S, 24 + g, -d[2]);
+                put_split(sX11 + (nc + 2 * tq + 1) * FA_S, 24 + g, -d[3]);
+            } else {                                   // X[48..64][32..48] into X22, row-major
+                put_split(sX22 + (16 + g) * FX_S, nc + 2 * tq, -d[0]);
+                put_split(sX22 + (16 + g) * FX_S, nc + 2 * tq + 1, -d[1]);
+                put_split(sX22 + (24 + g) * FX_S, nc + 2 * tq, -d[2]);
+                put_split(sX22 + (24 + g) * FX_S, nc + 2 * tq + 1, -d[3]);
+            }
         }
         __syncthreads();
-        // level 2: X[32:64][0:32] = -X[32:64][32:64] (A[32:64][0:32] X[0:32][0:32]); warp w takes
-        // the 16 x 8 output tile (w / 4, w % 4)
+        // level 2: X[32:64][0:32] = -X[32:64][32:64] (A[32:64][0:32] X[0:32][0:32]) from the split
+        // operands; warp w takes the 16 x 8 output tile (w / 4, w % 4).  P = A21 X11 goes to fT
+        // split and n-major.
         {
             const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
             float d[4] = {0.f, 0.f, 0.f, 0.f};
-            mma_3xtf32<4>(d, [&](int r, int k) { return fA[(32 + mr + r) * FA_S + k]; },
-                             [&](int k, int cc) { return fX[k * FX_S + nc + cc]; }, lane);
-            fT[(mr + g) * 33 + nc + 2 * tq] = d[0]; fT[(mr + g) * 33 + nc + 2 * tq + 1] = d[1];
-            fT[(mr + g + 8) * 33 + nc + 2 * tq] = d[2]; fT[(mr + g + 8) * 33 + nc + 2 * tq + 1] = d[3];
+            mma_32_split_bf16(d, sA21, FA_S, mr, sX11, FA_S, nc, lane);
+            put_split(sP + (nc + 2 * tq) * kPS, mr + g, d[0]);
+            put_split(sP + (nc + 2 * tq + 1) * kPS, mr + g, d[1]);
+            put_split(sP + (nc + 2 * tq) * kPS, mr + g + 8, d[2]);
+            put_split(sP + (nc + 2 * tq + 1) * kPS, mr + g + 8, d[3]);
         }
         __syncthreads();
+        // A (fp32 and split) has been read for the last time: the next item's K tile lands there
+        if (tid == 0 && nxt < items) load_k(nxt);
         {
             const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
             float d[4] = {0.f, 0.f, 0.f, 0.f};
-            mma_3xtf32<4>(d, [&](int r, int k) { return fX[(32 + mr + r) * FX_S + 32 + k]; },
-                             [&](int k, int cc) { return fT[k * 33 + nc + cc]; }, lane);
+            mma_32_split_bf16(d, sX22, FX_S, mr, sP, kPS, nc, lane);
             fX[(32 + mr + g) * FX_S + nc + 2 * tq] = -d[0]; fX[(32 + mr + g) * FX_S + nc + 2 * tq + 1] = -d[1];
             fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq] = -d[2]; fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq + 1] = -d[3];
         }
@@ -498,9 +606,9 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         __syncthreads();
     }
     if (tid == 0 && s_fail) {
-        // after a failure at item c: its K load and K K^T product land before TMEM is freed
-        mbar_wait(&mb_k, c & 1, kWaitBudgetNs);
-        mbar_wait(&mb_kk, c & 1, kWaitBudgetNs);
+        // after a failure: the last K load and K K^T product issued land before TMEM is freed
+        if (nk > 0) mbar_wait(&mb_k, (nk - 1) & 1, kWaitBudgetNs);
+        if (nkk > 0) mbar_wait(&mb_kk, (nkk - 1) & 1, kWaitBudgetNs);
     }
     tc_fence_before();
     __syncthreads();
@@ -599,9 +707,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 mbar_init(&mb_tv[b], 1); mbar_init(&mb_ve[b], 1);
                 mbar_init(&mb_tr[b], 1); mbar_init(&mb_re[b], 1);
             }
-            mbar_init(&mb_st, 1); mbar_init(&mb_sfree, kChain);
+            mbar_init(&mb_st, 1); mbar_init(&mb_sfree, kChainWarps);
             mbar_init(&mb_x, 1); mbar_init(&mb_u, 1); mbar_init(&mb_s, 1);
-            mbar_init(&mb_sready, kChain); mbar_init(&mb_xready, kChain); mbar_init(&mb_uready, kChain);
+            mbar_init(&mb_sready, kChainWarps); mbar_init(&mb_xready, kChainWarps);
+            mbar_init(&mb_uready, kChainWarps);
             mbar_init(&mb_fin, 1);
             fence_barrier_init();
         }
@@ -630,17 +739,21 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         const uint64_t dV = sdesc_sw128(smem_u32(sm + SM_V), 8192, 1024);    // MN-major A of V^T I
         const uint64_t dR = sdesc_sw128(smem_u32(sm + SM_R), 16, 1024);
         const uint64_t dI = sdesc_sw128(smem_u32(sm + SM_I), 16, 1024);
+        // Each group's operands are formed before the wait that releases it, so that only the
+        // MMA instructions themselves follow the wait (this warp shares its scheduler with four
+        // chain warps).
         // X region <- V(J)^T: A = the V tile read MN-major (k-step s = tokens 16 s ..), B = I.  V(J)'s
         // buffer is released when the product completes.
         auto issue_vi = [&](int J) -> bool {
+            uint64_t av[4], bv[4];
+#pragma unroll
+            for (int s = 0; s < 4; ++s) {
+                av[s] = dadd(dV, (J & 1) * 16384 + s * 2048); bv[s] = dadd(dI, s * 32);
+                pin(av[s]); pin(bv[s]);
+            }
             if (!warp_wait(&mb_tv[J & 1], (J >> 1) & 1, kWaitBudgetNs, abort_flag)) return false;
             tc_fence_after();
-            if (elect_one()) {
-                const uint32_t id = idesc_bf16(128, 64, 1, 0);
-#pragma unroll
-                for (int s = 0; s < 4; ++s)
-                    mma_bf16_1t(tm + TM_X, dadd(dV, (J & 1) * 16384 + s * 2048), dadd(dI, s * 32), id, s != 0);
-            }
+            if (elect_one()) mma4_bf16_ss_1t(tm + TM_X, av, bv, idesc_bf16(128, 64, 1, 0), 0);
             __syncwarp();
             mma_commit(&mb_ve[J & 1]);
             return true;
@@ -648,55 +761,78 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         bool ok = NJ == 0 || issue_vi(0);
         if (!ok) fail(a.status, abort_flag, 1);
         for (int j = 0; ok && j < NJ; ++j) {           // j: global tile index
-            // tile j ready for X: K'(j) is written and, at a head's first tile, the state is in
-            // TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe order)
-            if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
-            tc_fence_after();
-            if (elect_one()) {   // X region += S~ K'^T: A = the fp32 state from TMEM read as tf32 (8
-                                 // columns per K = 8 step), B = K'
-                const uint32_t id = idesc_tf32(128, 64);
+            {   // X region += S~ K'^T: A = the fp32 state from TMEM read as tf32 (8 columns per K = 8
+                // step), B = K'.  Tile j ready for X: K'(j) is written and, at a head's first tile,
+                // the state is in TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe order).
+                uint32_t ax[4][4];
+                uint64_t bx[4][4];
 #pragma unroll
-                for (int s = 0; s < 16; ++s)
-                    mma_tf32_ta_1t(tm + TM_X, tm + TM_S + 8 * s, dadd(dK32, (s >> 2) * 8192 + (s & 3) * 32), id, 1);
+                for (int s = 0; s < 16; ++s) {
+                    ax[s >> 2][s & 3] = tm + TM_S + 8 * s;
+                    bx[s >> 2][s & 3] = dadd(dK32, (s >> 2) * 8192 + (s & 3) * 32);
+                    pin(ax[s >> 2][s & 3]); pin(bx[s >> 2][s & 3]);
+                }
+                if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
+                tc_fence_after();
+                if (elect_one()) {
+#pragma unroll
+                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + TM_X, ax[g4], bx[g4], idesc_tf32(128, 64), 1);
+                }
+                __syncwarp();
+                mma_commit(&mb_x);
             }
-            __syncwarp();
-            mma_commit(&mb_x);
-            if (!warp_wait(&mb_xready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 5); break; }
-            if (!warp_wait(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 3); break; }
-            tc_fence_after();
-            if (elect_one()) {   // U region <- W^T T~^T with W (hi, lo) packed in place in X (k-step s:
-                                 // hi at column 16 s, lo at 16 s + 8): W hi T~ hi + W hi T~ lo + W lo T~ hi
-                const uint32_t id = idesc_bf16(128, 64, 0, 0);
+            {   // U region <- W^T T~^T with W (hi, lo) packed in place in X (k-step s: hi at column
+                // 16 s, lo at 16 s + 8): W hi T~ hi + W hi T~ lo + W lo T~ hi
+                uint32_t au[3][4];
+                uint64_t bu[3][4];
                 const uint32_t rb = (j & 1) * kRecSlot;
 #pragma unroll
                 for (int part = 0; part < 3; ++part) {
 #pragma unroll
-                    for (int s = 0; s < 4; ++s)
-                        mma_bf16_ta_1t(tm + TM_U, tm + TM_X + 16 * s + (part == 2 ? 8 : 0),
-                                       dadd(dR, rb + (part == 1 ? 8192 : 0) + s * 32), id, (part | s) != 0);
+                    for (int s = 0; s < 4; ++s) {
+                        au[part][s] = tm + TM_X + 16 * s + (part == 2 ? 8 : 0);
+                        bu[part][s] = dadd(dR, rb + (part == 1 ? 8192 : 0) + s * 32);
+                        pin(au[part][s]); pin(bu[part][s]);
+                    }
                 }
+                if (!warp_wait(&mb_xready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 5); break; }
+                if (!warp_wait(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 3); break; }
+                tc_fence_after();
+                if (elect_one()) {
+#pragma unroll
+                    for (int part = 0; part < 3; ++part)
+                        mma4_bf16_ta_1t(tm + TM_U, au[part], bu[part], idesc_bf16(128, 64, 0, 0), part != 0);
+                }
+                __syncwarp();
+                mma_commit(&mb_u);
+                mma_commit(&mb_re[j & 1]);             // record slot free once MMA_U(j) has read T~
             }
-            __syncwarp();
-            mma_commit(&mb_u);
-            mma_commit(&mb_re[j & 1]);                 // record slot free once MMA_U(j) has read T~
             // the next tile's V^T into the X region (MMA_U(j), its last reader, is ahead in the pipe)
             if (j + 1 < NJ && !issue_vi(j + 1)) { fail(a.status, abort_flag, 4); break; }
-            if (!warp_wait(&mb_uready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 7); break; }
-            tc_fence_after();
-            if (elect_one()) {   // S~ += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major)
-                const uint32_t id = idesc_bf16(128, 128, 0, 1);
+            {   // S~ += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major)
+                uint32_t as_[2][4];
+                uint64_t bs[2][4];
                 const uint32_t kb = (j % 3) * 16384;
 #pragma unroll
                 for (int part = 0; part < 2; ++part) {
 #pragma unroll
-                    for (int s = 0; s < 4; ++s)
-                        mma_bf16_ta_1t(tm + TM_S, tm + TM_U + 16 * s + (part == 1 ? 8 : 0),
-                                       dadd(dK, kb + s * 2048), id, 1);
+                    for (int s = 0; s < 4; ++s) {
+                        as_[part][s] = tm + TM_U + 16 * s + (part == 1 ? 8 : 0);
+                        bs[part][s] = dadd(dK, kb + s * 2048);
+                        pin(as_[part][s]); pin(bs[part][s]);
+                    }
                 }
+                if (!warp_wait(&mb_uready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 7); break; }
+                tc_fence_after();
+                if (elect_one()) {
+#pragma unroll
+                    for (int part = 0; part < 2; ++part)
+                        mma4_bf16_ta_1t(tm + TM_S, as_[part], bs[part], idesc_bf16(128, 128, 0, 1), 1);
+                }
+                __syncwarp();
+                mma_commit(&mb_s);
+                mma_commit(&mb_ke[j % 3]);             // K(j)'s buffer free once MMA_S(j) has read it
             }
-            __syncwarp();
-            mma_commit(&mb_s);
-            mma_commit(&mb_ke[j % 3]);                 // K(j)'s buffer free once MMA_S(j) has read it
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0)) {
             mma_commit(&mb_fin);                       // every MMA this warp issued has completed
@@ -854,13 +990,13 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
 #pragma unroll
                 for (int e = 0; e < 32; ++e) den = fmaf(sv[e], sv[e], den);
-                mbar_arrive(&mb_sfree);                    // the staging buffer has been read
+                warp_arrive(&mb_sfree, lane);                    // the staging buffer has been read
                 tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
                 tmem_st32(tm + lane_off + TM_SB + 32 * cgp, sv);
                 if (!make_kprime(0, 1.f, rec_consts(0))) fail(a.status, abort_flag, 16);
                 tmem_st_wait();
                 tc_fence_before();
-                mbar_arrive(&mb_sready);
+                warp_arrive(&mb_sready, lane);
             }
             const bool rescale = sig * gC < kSigMin;       // uniform over the CTA
             const float u_scale = rescale ? 1.f : 1.f / (gC * sig);
@@ -881,7 +1017,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tmem_st_wait();
             }
             tc_fence_before();
-            mbar_arrive(&mb_xready);
+            warp_arrive(&mb_xready, lane);
 
             // ---- while MMA_U runs: rescale S~ if the decay would underflow the deferred scale
             // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K'(j+1)
@@ -918,10 +1054,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tmem_st_wait();
             }
             tc_fence_before();
-            mbar_arrive(&mb_uready);
+            warp_arrive(&mb_uready, lane);
             if (!last) {
                 // the next tile of this head may start X as soon as MMA_S(j) is queued
-                mbar_arrive(&mb_sready);
+                warp_arrive(&mb_sready, lane);
             } else {
                 // ---- head boundary: S_after = sig S~ out through the staging buffer, the next
                 // head's state (staged meanwhile) into TMEM, drift partials against S_before
@@ -972,8 +1108,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
                 tc_fence_before();
                 fence_async_smem();                        // S_after -> the state warp's TMA store
-                mbar_arrive(&mb_sfree);
-                if (has_next) mbar_arrive(&mb_sready);     // the next head's state is in TMEM
+                warp_arrive(&mb_sfree, lane);
+                if (has_next) warp_arrive(&mb_sready, lane);     // the next head's state is in TMEM
                 // partial sums: pairwise in fp32, over the warp's lanes and then over the 16 warps
                 // (the FP64 pipe is far too slow for this path)
                 float fn = num, fd = den;

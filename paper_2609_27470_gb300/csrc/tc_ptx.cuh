@@ -311,6 +311,51 @@ __device__ __forceinline__ void mma_tf32_ta_1t(uint32_t d_tmem, uint32_t a_tmem,
                  :: "r"(d_tmem), "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate) : "memory");
 }
 
+// Four MMAs into one accumulator from one thread: the first accumulates iff acc0 != 0, the other
+// three always.  A from TMEM (tf32 or f16 kinds) or from shared memory (f16, descriptors).
+__device__ __forceinline__ void mma4_tf32_ta_1t(uint32_t d, const uint32_t (&a)[4], const uint64_t (&b)[4],
+                                                uint32_t idesc, uint32_t acc0) {
+    asm volatile("{\n\t.reg .pred p, q;\n\t"
+                 "setp.ne.b32 p, %10, 0;\n\t"
+                 "setp.eq.b32 q, %10, %10;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %5, %9, p;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%2], %6, %9, q;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%3], %7, %9, q;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%4], %8, %9, q;\n\t}"
+                 :: "r"(d), "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "l"(b[0]), "l"(b[1]), "l"(b[2]), "l"(b[3]),
+                    "r"(idesc), "r"(acc0) : "memory");
+}
+__device__ __forceinline__ void mma4_bf16_ta_1t(uint32_t d, const uint32_t (&a)[4], const uint64_t (&b)[4],
+                                                uint32_t idesc, uint32_t acc0) {
+    asm volatile("{\n\t.reg .pred p, q;\n\t"
+                 "setp.ne.b32 p, %10, 0;\n\t"
+                 "setp.eq.b32 q, %10, %10;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %5, %9, p;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%2], %6, %9, q;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%3], %7, %9, q;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%4], %8, %9, q;\n\t}"
+                 :: "r"(d), "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "l"(b[0]), "l"(b[1]), "l"(b[2]), "l"(b[3]),
+                    "r"(idesc), "r"(acc0) : "memory");
+}
+__device__ __forceinline__ void mma4_bf16_ss_1t(uint32_t d, const uint64_t (&a)[4], const uint64_t (&b)[4],
+                                                uint32_t idesc, uint32_t acc0) {
+    asm volatile("{\n\t.reg .pred p, q;\n\t"
+                 "setp.ne.b32 p, %10, 0;\n\t"
+                 "setp.eq.b32 q, %10, %10;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %5, %9, p;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %2, %6, %9, q;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %3, %7, %9, q;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %4, %8, %9, q;\n\t}"
+                 :: "r"(d), "l"(a[0]), "l"(a[1]), "l"(a[2]), "l"(a[3]), "l"(b[0]), "l"(b[1]), "l"(b[2]), "l"(b[3]),
+                    "r"(idesc), "r"(acc0) : "memory");
+}
+
+// Pins register values before the next volatile statement (e.g. operands prepared ahead of a wait).
+template <typename T>
+__device__ __forceinline__ void pin(const T& v) {
+    asm volatile("" :: "l"((uint64_t)v));
+}
+
 // Arrive (once) on an mbarrier when every tcgen05 operation issued so far by the issuing lane is
 // done.  Called by all 32 lanes of the warp that issued the MMAs; one elected lane commits.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
