@@ -136,44 +136,6 @@ __device__ __forceinline__ float round_tf32(float x) {
     return __uint_as_float(y);
 }
 
-// x -> (hi, lo) tf32 pair with x = hi + lo to about 2^-22 relative
-__device__ __forceinline__ void split_tf32(float x, uint32_t& hi, uint32_t& lo) {
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(lo) : "f"(x - __uint_as_float(hi)));
-}
-
-// D (16 x 8) += A (16 x 8, row) B (8 x 8, col) on the warp's tensor-core path, tf32 in, fp32
-// accumulate.  Fragments: g = lane / 4, t = lane % 4; a = A[g][t], A[g+8][t], A[g][t+4],
-// A[g+8][t+4]; b = B[t][g], B[t+4][g]; d = D[g][2t], D[g][2t+1], D[g+8][2t], D[g+8][2t+1].
-__device__ __forceinline__ void mma_m16n8k8_tf32(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
-    asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-                 "{%0,%1,%2,%3};"
-                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
-}
-
-// D (16 x 8) += A B over K = 8 k-steps of 8, fp32-accurate: each operand split into a tf32 pair
-// and the three products hi*hi + hi*lo + lo*hi accumulated (small terms first).  A(r, k) and
-// B(k, c) read shared memory (r < 16, k < 8 ksteps, c < 8).
-template <int KSTEPS, typename FA, typename FB>
-__device__ __forceinline__ void mma_3xtf32(float (&d)[4], FA A, FB B, int lane) {
-    const int g = lane >> 2, t = lane & 3;
-#pragma unroll
-    for (int ks = 0; ks < KSTEPS; ++ks) {
-        const int k0 = 8 * ks;
-        uint32_t ah[4], al[4], bh[2], bl[2];
-        split_tf32(A(g, k0 + t), ah[0], al[0]);
-        split_tf32(A(g + 8, k0 + t), ah[1], al[1]);
-        split_tf32(A(g, k0 + t + 4), ah[2], al[2]);
-        split_tf32(A(g + 8, k0 + t + 4), ah[3], al[3]);
-        split_tf32(B(k0 + t, g), bh[0], bl[0]);
-        split_tf32(B(k0 + t + 4, g), bh[1], bl[1]);
-        mma_m16n8k8_tf32(d, al, bh);
-        mma_m16n8k8_tf32(d, ah, bl);
-        mma_m16n8k8_tf32(d, ah, bh);
-    }
-}
-
 // D (16 x 8) += A (16 x 16, row) B (16 x 8, col) on the warp's tensor-core path, bf16 in, fp32
 // accumulate.  Fragments (g = lane / 4, t = lane % 4), each register a bf16 pair, lower k in the
 // low half: a = A[g][2t..], A[g+8][2t..], A[g][2t+8..], A[g+8][2t+8..]; b = B[2t..][g],
@@ -185,35 +147,48 @@ __device__ __forceinline__ void mma_m16n8k16_bf16(float (&d)[4], const uint32_t 
                  : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
-// A 32 x 32 operand stored split: row r is 32 words at rows + r * stride, words 0..15 the bf16
-// pairs (2p, 2p+1) of hi = bf16(x), words 16..31 those of lo = bf16(x - hi).  D (16 x 8) +=
-// A[r0 .. r0+15][0..32) B[0..32)[n0 .. n0+7] over the three products lo*hi + hi*lo + hi*hi, A
-// row-major and B stored n-major (row n of B's storage holds column n of B).
-__device__ __forceinline__ void mma_32_split_bf16(float (&d)[4], const uint32_t* A, int as, int r0,
-                                                  const uint32_t* B, int bs, int n0, int lane) {
+// Operands stored split: row r of A is at A + r * as (32-bit words), its word p the bf16 pair of
+// hi = bf16(x) for columns (2p, 2p+1) and word a_lo + p the pair of lo = bf16(x - hi); likewise B,
+// stored n-major (row n of B's storage holds column n of B).  D (16 x 8) += A[r0 .. r0+15][0..16K)
+// B[0..16K)[n0 .. n0+7] over the three products lo*hi + hi*lo + hi*hi.
+template <int KSTEPS>
+__device__ __forceinline__ void mma_split_bf16(float (&d)[4], const uint32_t* A, int as, int a_lo, int r0,
+                                               const uint32_t* B, int bs, int b_lo, int n0, int lane) {
     const int g = lane >> 2, t = lane & 3;
     const uint32_t* a0 = A + (r0 + g) * as;
     const uint32_t* a1 = A + (r0 + g + 8) * as;
     const uint32_t* b0 = B + (n0 + g) * bs;
 #pragma unroll
-    for (int ks = 0; ks < 2; ++ks) {
+    for (int ks = 0; ks < KSTEPS; ++ks) {
         const int p0 = 8 * ks + t, p1 = p0 + 4;
         const uint32_t ah[4] = {a0[p0], a1[p0], a0[p1], a1[p1]};
-        const uint32_t al[4] = {a0[16 + p0], a1[16 + p0], a0[16 + p1], a1[16 + p1]};
+        const uint32_t al[4] = {a0[a_lo + p0], a1[a_lo + p0], a0[a_lo + p1], a1[a_lo + p1]};
         const uint32_t bh[2] = {b0[p0], b0[p1]};
-        const uint32_t bl[2] = {b0[16 + p0], b0[16 + p1]};
+        const uint32_t bl[2] = {b0[b_lo + p0], b0[b_lo + p1]};
         mma_m16n8k16_bf16(d, al, bh);
         mma_m16n8k16_bf16(d, ah, bl);
         mma_m16n8k16_bf16(d, ah, bh);
     }
 }
 
-// One element of a split row (see mma_32_split_bf16): hi / lo halfwords of column k of row `row`.
-__device__ __forceinline__ void put_split(uint32_t* row, int k, float x) {
+// One element of a split row (see mma_split_bf16): hi / lo halfwords of column k; lo words start
+// lo_words after the row's first word.
+__device__ __forceinline__ void put_split(uint32_t* row, int k, float x, int lo_words = 16) {
     const __nv_bfloat16 h = __float2bfloat16_rn(x);
     const __nv_bfloat16 l = __float2bfloat16_rn(x - __bfloat162float(h));
     reinterpret_cast<__nv_bfloat16*>(row)[k] = h;
-    reinterpret_cast<__nv_bfloat16*>(row + 16)[k] = l;
+    reinterpret_cast<__nv_bfloat16*>(row + lo_words)[k] = l;
+}
+
+// 16 consecutive values -> split row of a 16-column operand (words 0..7 hi, 8..15 lo)
+__device__ __forceinline__ void put_split16(uint32_t* row, const float* x) {
+    uint32_t h[8], l[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) split2(x[2 * i], x[2 * i + 1], h[i], l[i]);
+    *reinterpret_cast<uint4*>(row) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4*>(row + 4) = make_uint4(h[4], h[5], h[6], h[7]);
+    *reinterpret_cast<uint4*>(row + 8) = make_uint4(l[0], l[1], l[2], l[3]);
+    *reinterpret_cast<uint4*>(row + 12) = make_uint4(l[4], l[5], l[6], l[7]);
 }
 
 // 2^x with the hardware approximation (relative error about 2^-22)
@@ -268,7 +243,10 @@ constexpr uint32_t WY_FX = WY_FA + 64 * FA_S * 4;     // fp32 [64][FX_S]; rows 0
                                                       // upper quarter) hold X22 split, row-major
 constexpr uint32_t WY_TMP = WY_FX + 64 * FX_S * 4;    // level 1 products (fp32), then level 2's P split,
                                                       // n-major, rows of 36 words
-constexpr uint32_t WY_TG = WY_TMP + 32 * 36 * 4;      // 2 buffers (item parity) x (G2[64], beta[64], row[64],
+constexpr uint32_t WY_L1 = WY_TMP + 32 * 36 * 4;      // level-1 split operands, 6 x 16 rows of 20 words: A10,
+                                                      // A32, X11' (row-major), X22' (n-major), P1 for p = 0, 1
+constexpr int kL1S = 20;                              // row stride (words): fragment loads hit distinct banks
+constexpr uint32_t WY_TG = WY_L1 + 6 * 16 * kL1S * 4; // 2 buffers (item parity) x (G2[64], beta[64], row[64],
                                                       // col[64], del[64], flag)
 constexpr uint32_t kTgFloats = 324;
 constexpr uint32_t WY_BYTES = WY_TG + 2 * kTgFloats * 4;
@@ -304,6 +282,13 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
     uint32_t* sX22 = reinterpret_cast<uint32_t*>(fX + 32);               // row r: X[32 + r][32 + k]
     uint32_t* sP = reinterpret_cast<uint32_t*>(fT);                      // row n: P[k][n]
     constexpr int kPS = 36;
+    // split level-1 operands: 16 x 16 blocks, rows of kL1S words (hi words 0..7, lo words 8..15)
+    uint32_t* sL1 = reinterpret_cast<uint32_t*>(sm + WY_L1);
+    uint32_t* sA10 = sL1;                                                 // A[16 + r][k]
+    uint32_t* sA32 = sL1 + 16 * kL1S;                                     // A[48 + r][32 + k]
+    uint32_t* sX11r = sL1 + 32 * kL1S;                                    // X[16 + r][16 + k]
+    uint32_t* sX22n = sL1 + 48 * kL1S;                                    // row n: X[32 + k][32 + n]
+    uint32_t* sP1 = sL1 + 64 * kL1S;                                      // p: row n of P1_p, 16 rows each
 
     if (warp == 0) { tmem_alloc(&s_tmem, kWyTmemCols); tmem_relinquish(); }
     if (tid == 0) {
@@ -450,6 +435,8 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
                     const float f = factored ? cf[e] : fast_exp2(G2t - cf[e]);
                     kk[e] = (cb + e < t) ? rt * f * kk[e] : 0.f;
                 }
+                if (half == 0 && lane >= 16 && (warp == 0 || warp == 5))   // A10 / A32, split
+                    put_split16((warp == 0 ? sA10 : sA32) + (lane - 16) * kL1S, kk);
                 if (warp == 1) {                       // A21, split
                     uint32_t* row = sA21 + (t - 32) * FA_S + 8 * half;
                     uint32_t h[8], l[8];
@@ -493,6 +480,12 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
             }
 #pragma unroll
             for (int rr = 0; rr < 16; ++rr) fX[(o + rr) * FX_S + o + jc] = x[rr];
+            if (B == 1) {                              // X11' row-major
+#pragma unroll
+                for (int rr = 0; rr < 16; ++rr) put_split(sX11r + rr * kL1S, jc, x[rr], 8);
+            } else if (B == 2) {                       // X22' n-major
+                put_split16(sX22n + jc * kL1S, x);
+            }
             if (B < 2) {                               // X11, n-major: row o + jc holds column o + jc
                 uint32_t* row = sX11 + (o + jc) * FA_S;
                 if (B == 1) {                          // X[0..16][16..32] = 0 (the K tile overwrote it)
@@ -522,22 +515,23 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         const int g = lane >> 2, tq = lane & 3;
         if (warp < 4) {
             const int p = warp >> 1, nc = 8 * (warp & 1);
-            const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
             float d[4] = {0.f, 0.f, 0.f, 0.f};
-            mma_3xtf32<2>(d, [&](int r, int k) { return fA[(ro + r) * FA_S + co + k]; },
-                             [&](int k, int cc) { return fX[(co + k) * FX_S + co + nc + cc]; }, lane);
-            float* P = fT + p * 272;                   // [16][17]
-            P[g * 17 + nc + 2 * tq] = d[0]; P[g * 17 + nc + 2 * tq + 1] = d[1];
-            P[(g + 8) * 17 + nc + 2 * tq] = d[2]; P[(g + 8) * 17 + nc + 2 * tq + 1] = d[3];
+            if (p == 0) mma_split_bf16<1>(d, sA10, kL1S, 8, 0, sX11, FA_S, 16, nc, lane);    // A10 X00
+            else        mma_split_bf16<1>(d, sA32, kL1S, 8, 0, sX22n, kL1S, 8, nc, lane);   // A32 X22'
+            uint32_t* P = sP1 + p * 16 * kL1S;         // n-major
+            put_split(P + (nc + 2 * tq) * kL1S, g, d[0], 8);
+            put_split(P + (nc + 2 * tq + 1) * kL1S, g, d[1], 8);
+            put_split(P + (nc + 2 * tq) * kL1S, g + 8, d[2], 8);
+            put_split(P + (nc + 2 * tq + 1) * kL1S, g + 8, d[3], 8);
         }
         __syncthreads();
         if (warp < 4) {
             const int p = warp >> 1, nc = 8 * (warp & 1);
             const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
-            const float* P = fT + p * 272;
+            const uint32_t* P = sP1 + p * 16 * kL1S;
             float d[4] = {0.f, 0.f, 0.f, 0.f};
-            mma_3xtf32<2>(d, [&](int r, int k) { return fX[(ro + r) * FX_S + ro + k]; },
-                             [&](int k, int cc) { return P[k * 17 + nc + cc]; }, lane);
+            if (p == 0) mma_split_bf16<1>(d, sX11r, kL1S, 8, 0, P, kL1S, 8, nc, lane);        // X11' P1
+            else        mma_split_bf16<1>(d, sX22 + 16 * FX_S + 8, FX_S, 16, 0, P, kL1S, 8, nc, lane);  // X33' P1'
             fX[(ro + g) * FX_S + co + nc + 2 * tq] = -d[0]; fX[(ro + g) * FX_S + co + nc + 2 * tq + 1] = -d[1];
             fX[(ro + g + 8) * FX_S + co + nc + 2 * tq] = -d[2]; fX[(ro + g + 8) * FX_S + co + nc + 2 * tq + 1] = -d[3];
             if (p == 0) {                              // X[16..32][0..16] into X11, n-major
@@ -559,7 +553,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         {
             const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
             float d[4] = {0.f, 0.f, 0.f, 0.f};
-            mma_32_split_bf16(d, sA21, FA_S, mr, sX11, FA_S, nc, lane);
+            mma_split_bf16<2>(d, sA21, FA_S, 16, mr, sX11, FA_S, 16, nc, lane);
             put_split(sP + (nc + 2 * tq) * kPS, mr + g, d[0]);
             put_split(sP + (nc + 2 * tq + 1) * kPS, mr + g, d[1]);
             put_split(sP + (nc + 2 * tq) * kPS, mr + g + 8, d[2]);
@@ -571,7 +565,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         {
             const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
             float d[4] = {0.f, 0.f, 0.f, 0.f};
-            mma_32_split_bf16(d, sX22, FX_S, mr, sP, kPS, nc, lane);
+            mma_split_bf16<2>(d, sX22, FX_S, 16, mr, sP, kPS, 16, nc, lane);
             fX[(32 + mr + g) * FX_S + nc + 2 * tq] = -d[0]; fX[(32 + mr + g) * FX_S + nc + 2 * tq + 1] = -d[1];
             fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq] = -d[2]; fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq + 1] = -d[3];
         }
