@@ -125,6 +125,9 @@ DELTAS_API const char* deltas_status_string(int32_t status);
 /* n_tokens = 0 leaves the state unchanged (partials then hold 0 and ||S_before||^2).          */
 /* Errors: INVALID_ARGUMENT for NULL/misaligned pointers, negative sizes or Hv % Hk != 0;      */
 /* UNSUPPORTED for d_k != d_v or d_k outside {16,32,64,128}; WORKSPACE for a short workspace. */
+/* Workspace: the status word plus, for d = 128 bf16 without read-out, the per-tile factors of  */
+/* the chunkwise form (16,656 bytes per layer, value head and 64-token tile), written and read   */
+/* within the call.                                                                             */
 /* ------------------------------------------------------------------------------------------ */
 DELTAS_API size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens);
 
