@@ -305,9 +305,12 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
     tc_fence_after();
     const uint32_t tm = s_tmem;
 
+    // Items are taken in reverse record order: the records written last, still in L2 when this
+    // kernel ends, are the ones of the lowest heads, which the update kernel reads first.
+    auto rec_of = [&](int it) { return items - 1 - it; };
     auto item_pos = [&](int it, int& l, int& h, int& jt) {
-        const int lh = it / n;
-        jt = it - lh * n; l = lh / a.Hv; h = lh - l * a.Hv;
+        const int r = rec_of(it), lh = r / n;
+        jt = r - lh * n; l = lh / a.Hv; h = lh - l * a.Hv;
     };
     int nk = 0, nkk = 0;                               // K loads (thread 0) / K K^T products (warp 0) issued
     auto load_k = [&](int it) {                        // thread 0: the item's K tile
@@ -344,7 +347,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         }
         const float G0 = incl - pg[1], G1 = incl;
         const float GC = __shfl_sync(0xffffffffu, incl, 31);
-        float* rc = reinterpret_cast<float*>(a.rec + (size_t)it * kRecBytes + kRecT);
+        float* rc = reinterpret_cast<float*>(a.rec + (size_t)rec_of(it) * kRecBytes + kRecT);
         *reinterpret_cast<float2*>(rc + 2 * lane) = make_float2(-expf(G0), -expf(G1));
         if (lane == 0) *reinterpret_cast<float4*>(rc + 64) = make_float4(expf(GC), 0.f, 0.f, 0.f);
         const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
@@ -573,7 +576,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         // T~ = diag(exp(G_C - G)) X diag(beta) (upper part zero), split into the record's (hi, lo)
         // images
         {
-            uint8_t* rec = a.rec + (size_t)it * kRecBytes;
+            uint8_t* rec = a.rec + (size_t)rec_of(it) * kRecBytes;
 #pragma unroll
             for (int m = 0; m < 2; ++m) {
                 const int e = tid + kWyThreads * m;
