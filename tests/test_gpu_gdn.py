@@ -172,6 +172,24 @@ def test_gdn_update_slow_decay_four_chunks(L):
         state = st.cpu()
 
 
+@pytest.mark.parametrize("decay_scale", [0.0, 4.0])
+def test_gdn_update_decay_extremes(L, decay_scale):
+    """No decay (g = 0: alpha = 1, the deferred decay never moves) and very strong decay (a tile's
+    cumulative log-decay spans more than 250 powers of two, so the factors take the per-entry
+    exponential, and gamma_C underflows, so every tile rescales the state): state and partials
+    against the oracle over four tiles and a ragged tail."""
+    Lg, Hk, Hv, d = 1, 2, 4, 128
+    x = inputs.gdn_chunk(Lg, 300, Hk, Hv, d, "bf16", inputs.seed_for(13, int(decay_scale)), decay_scale=decay_scale)
+    g = x["g"].double()
+    if decay_scale > 0:                                 # the regimes this case is meant to reach
+        span = (g[:, 64:128].sum(dim=1) / np.log(2)).abs()
+        assert (span > 250).any()
+    else:
+        assert (g == 0).all()
+    state0 = inputs.initial_state(Lg, Hv, d, 14)
+    _check_chunk(L, x, state0, False, torch.bfloat16, None)
+
+
 def test_state_drift_kernel(L):
     """deltas_state_drift partials == oracle (Eq. 3 numerator/denominator per layer and head)."""
     sb = inputs.initial_state(3, 4, 128, 11)
