@@ -161,10 +161,12 @@ class _EvCtx:
 # ----------------------------------------------------------------------------------- workloads
 
 class GdnRing:
-    """R distinct per-chunk input sets on the device (generated from seeds, outside timing)."""
+    """R distinct per-chunk input sets on the device (generated from seeds, outside timing); set r
+    has chunk_lens[r] tokens (one length for all when chunk_lens is an int)."""
 
-    def __init__(self, cfg, chunk_len, dev, seed):
-        self.sets = [inputs.gdn_chunk(cfg["L"], chunk_len, cfg["Hk"], cfg["Hv"], cfg["d"], cfg["dtype"],
+    def __init__(self, cfg, chunk_lens, dev, seed):
+        lens = [chunk_lens] * RING if isinstance(chunk_lens, int) else list(chunk_lens)
+        self.sets = [inputs.gdn_chunk(cfg["L"], lens[r], cfg["Hk"], cfg["Hv"], cfg["d"], cfg["dtype"],
                                       inputs.seed_for(seed, r), device=dev) for r in range(RING)]
 
     def __getitem__(self, i):
@@ -190,20 +192,24 @@ def algorithmic_gdn_flops(L, T, Hv, d, with_out):
 
 
 class StreamingWorkload:
-    name = "streaming"
+    """One chunk per step through the whole path (update + drift, score, append, select, compact)
+    on a cache kept at the budget: streaming (512-token chunks) and paper (118-132-token chunks,
+    the length cycling through the ring)."""
 
     def __init__(self, dev, L, cfg=None):
         cfg = dict(cfg or configs.STREAMING)
         self.cfg = cfg
+        self.name = cfg["name"]
         self.L = L
         self.dev = dev
-        C = cfg["chunk_len"]
+        C = cfg["chunk_len"]                                   # the longest chunk
         self.C = C
-        self.ring = GdnRing(cfg, C, dev, seed=40)
-        self.kv_ring = [inputs.kv_chunk(cfg["Lf"], cfg["Hkv"], C, cfg["D"], cfg["kv_dtype"], inputs.seed_for(41, r),
-                                        device=dev) for r in range(RING)]
+        self.lens = list(cfg.get("chunk_lens", (C,) * RING))
+        assert len(self.lens) == RING and max(self.lens) <= C
+        self.ring = GdnRing(cfg, self.lens, dev, seed=40)
+        self.kv_ring = [inputs.kv_chunk(cfg["Lf"], cfg["Hkv"], self.lens[r], cfg["D"], cfg["kv_dtype"],
+                                        inputs.seed_for(41, r), device=dev) for r in range(RING)]
         from paper_2609_27470_gb300.stream import DeltaSStream
-        n_fill = cfg["budget_M"] // C
         self.s = DeltaSStream(num_layers=cfg["L"], num_k_heads=cfg["Hk"], num_v_heads=cfg["Hv"], head_dim=cfg["d"],
                               act_dtype=torch.bfloat16, kv_layers=cfg["Lf"], kv_heads=cfg["Hkv"],
                               kv_head_dim=cfg["D"], kv_dtype=torch.bfloat16, budget_M=cfg["budget_M"],
@@ -211,16 +217,23 @@ class StreamingWorkload:
                               chunk_len=C, max_chunks=cfg["n_chunks"],
                               state0=inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 42, device=dev),
                               device=dev)
-        # fill the cache to the budget (setup, not timed): appended chunks with Exp(1) scores
+        # fill the cache to exactly the budget (setup, not timed): appended chunks with Exp(1)
+        # scores, the last one cut to fit, so that every timed step evicts
+        M = cfg["budget_M"]
+        fills = []
+        while sum(fills) < M:
+            fills.append(min(self.lens[len(fills) % RING], M - sum(fills)))
+        n_fill = len(fills)
         gen = torch.Generator(device=dev)
         gen.manual_seed(43)
         self.s.chunk_scores[:n_fill] = torch.empty(n_fill, device=dev).exponential_(1.0, generator=gen)
-        for c in range(n_fill):
+        for c, n in enumerate(fills):
             kn, vn = self.kv_ring[c % RING]
+            kn, vn = kn[:, :, :n].contiguous(), vn[:, :, :n].contiguous()
             L.deltas_append_kv(self.s.kv, self.s.k_cache, self.s.v_cache, self.s.tok_chunk, self.s.tok_pos,
                                self.s.cache_len, kn, vn, c, self.s.position)
-            self.s.cache_len += C
-            self.s.position += C
+            self.s.cache_len += n
+            self.s.position += n
         self.s.chunk = n_fill
         self.step_i = 0
         self.moved = None
@@ -228,17 +241,18 @@ class StreamingWorkload:
     def step(self, timer):
         x = self.ring[self.step_i]
         kn, vn = self.kv_ring[self.step_i % RING]
+        T = self.lens[self.step_i % RING]
         s, L, c = self.s, self.L, self.s.chunk
         with timer.mark("gdn_update"):
-            L.deltas_gdn_chunk_update(s.gdn, self.C, None, x["k"], x["v"], x["g"], x["beta"], s.state, None,
+            L.deltas_gdn_chunk_update(s.gdn, T, None, x["k"], x["v"], x["g"], x["beta"], s.state, None,
                                       s.partials, s.workspace)
         with timer.mark("score"):
             L.deltas_score_chunks(s.gdn.num_layers, s.gdn.num_v_heads, s.partials, c, s.chunk_scores)
         with timer.mark("append"):
             L.deltas_append_kv(s.kv, s.k_cache, s.v_cache, s.tok_chunk, s.tok_pos, s.cache_len, kn, vn, c,
                                s.position)
-        s.cache_len += self.C
-        s.position += self.C
+        s.cache_len += T
+        s.position += T
         s.chunk += 1
         with timer.mark("select"):
             L.deltas_select_retain(s.policy, s.cache_len, s.tok_chunk, s.chunk_scores[: c + 1], s.retain_idx,
@@ -257,16 +271,18 @@ class StreamingWorkload:
         self.moved = cnt if self.moved is None else self.moved + cnt
 
     def launches_per_step(self):
-        return 1 + 1 + 1 + 1 + 3
+        return 2 + 1 + 1 + 3 + 3                                # update (2), score, append, select (3), compact (3)
 
     def tokens_per_step(self):
-        return self.C
+        # the mean chunk length (exact when the timed steps are a multiple of the ring)
+        return sum(self.lens) / len(self.lens)
 
     def kernel_roofline(self, name, avg_ms, peaks, steps):
         cfg = self.cfg
         if name == "gdn_update":
-            by = algorithmic_gdn_bytes(cfg["L"], self.C, cfg["Hk"], cfg["Hv"], cfg["d"], 2, False)
-            fl = algorithmic_gdn_flops(cfg["L"], self.C, cfg["Hv"], cfg["d"], False)
+            T = self.tokens_per_step()
+            by = algorithmic_gdn_bytes(cfg["L"], T, cfg["Hk"], cfg["Hv"], cfg["d"], 2, False)
+            fl = algorithmic_gdn_flops(cfg["L"], T, cfg["Hv"], cfg["d"], False)
             return {"bound": "hbm", "achieved": by / (avg_ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"],
                     "unit": "GB/s", "bytes_per_launch": by,
                     "tensor_frac": fl / (avg_ms * 1e-3) / 1e12 / peaks["bf16_tflops_sustained"]}
@@ -314,7 +330,7 @@ class GdnOnlyWorkload:
         self.step_i += 1
 
     def launches_per_step(self):
-        return 2
+        return 2 + 1                                            # factor + chain kernels, score
 
     def tokens_per_step(self):
         return self.C
@@ -378,7 +394,7 @@ class KvWorkload:
             self.L.deltas_compact_kv(self.kv, self.k, self.v, self.tc, self.tp, self.idx, self.n, self.cap, self.ws)
 
     def launches_per_step(self):
-        return 4
+        return 3 + 3                                            # selection: runs, retain, emit; compaction: init, need, main
 
     def tokens_per_step(self):
         return self.cap
@@ -414,6 +430,8 @@ KERNEL_SOURCES = {"gdn_update": "paper_2609_27470_gb300/csrc/gdn_tc.cu",
 def make_workload(name, dev, L):
     if name == "streaming":
         return StreamingWorkload(dev, L)
+    if name == "paper":
+        return StreamingWorkload(dev, L, configs.PAPER)
     if name == "stack":
         return GdnOnlyWorkload(dev, L, configs.STACK)
     if name == "layer":
@@ -451,7 +469,8 @@ def e2e_sequential(wl, host, steps, stream, timer_off, reset):
     for _ in range(steps):
         reset()
         e0.record(stream)
-        for h, d in zip(host, wl.h2d_tensors(getattr(wl, "step_i", 0))):
+        i = getattr(wl, "step_i", 0)
+        for h, d in zip(host[i % len(host)], wl.h2d_tensors(i)):
             d.copy_(h, non_blocking=True)
         wl.step(timer_off)
         host_out.copy_(wl.result_scalar(), non_blocking=True)
@@ -479,7 +498,7 @@ def e2e_pipelined(wl, host, steps, stream, dev, timer_off):
         with torch.cuda.stream(cs):
             if i >= 2:
                 cs.wait_event(done[i - 2])                 # at most two steps in flight
-            for h, d in zip(host, wl.h2d_tensors(slot0 + i)):
+            for h, d in zip(host[(slot0 + i) % len(host)], wl.h2d_tensors(slot0 + i)):
                 d.copy_(h, non_blocking=True)
             copied[i].record(cs)
         stream.wait_event(copied[i])
@@ -502,12 +521,11 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
     extrapolates to a whole step.  Returns (tokens_per_s, sample description, seconds spent)."""
     import oracle
     t_start = time.perf_counter()
-    cfg = {"streaming": configs.STREAMING, "stack": configs.STACK, "layer": configs.LAYER,
-           "kv": configs.KV}[workload]
+    cfg = _cfg(workload)
     parts = []
     total = 0.0
-    if workload in ("streaming", "stack", "layer"):
-        C = cfg["chunk_len"]
+    if workload in ("streaming", "paper", "stack", "layer"):
+        C = int(round(_tokens(workload)))
         heads_total = cfg["L"] * cfg["Hv"]
         n_heads = 2
         x = inputs.gdn_chunk(1, C, 1, 1, cfg["d"], "bf16", 77)
@@ -526,9 +544,9 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         t_head = (time.perf_counter() - t0) / reps
         total += t_head * heads_total
         parts.append(f"gdn: {reps} (layer,head) x {C} tokens, x{heads_total / reps:.0f} extrapolated")
-    if workload in ("streaming", "kv"):
+    if workload in ("streaming", "paper", "kv"):
         M = cfg["budget_M"]
-        if workload == "streaming":
+        if workload != "kv":
             T = M + cfg["chunk_len"]
             rng = np.random.default_rng(5)
             lens = rng.integers(1, cfg["chunk_len"] + 1, size=4 * T // cfg["chunk_len"])
@@ -550,8 +568,7 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         t_cmp = (time.perf_counter() - t0) * planes_total / 2
         total += t_sel + t_cmp
         parts.append(f"select on {T} slots; compact 2 of {planes_total} planes x{planes_total // 2}")
-    tokens = cfg["chunk_len"] if workload != "kv" else cfg["n_chunks"] * cfg["chunk_len"]
-    return tokens / total, "; ".join(parts), time.perf_counter() - t_start
+    return _tokens(workload) / total, "; ".join(parts), time.perf_counter() - t_start
 
 
 # ----------------------------------------------------------------------------------- main
@@ -583,8 +600,8 @@ def config_line(workload):
     c = _cfg(workload)
     line = {"workload": workload, "l2": "flushed between timed steps (256 MiB write)",
             "inputs": "ring of 8 distinct per-chunk input sets, generated on device"}
-    for key in ("L", "Hk", "Hv", "d", "chunk_len", "Lf", "Hkv", "D", "budget_M", "n_sink", "n_window",
-                "n_buckets"):
+    for key in ("L", "Hk", "Hv", "d", "chunk_len", "chunk_lens", "Lf", "Hkv", "D", "budget_M", "n_sink",
+                "n_window", "n_buckets"):
         if key in c:
             line[key] = c[key]
     if workload == "kv":
@@ -593,13 +610,17 @@ def config_line(workload):
 
 
 def _cfg(workload):
-    return {"streaming": configs.STREAMING, "stack": configs.STACK, "layer": configs.LAYER,
-            "kv": configs.KV}[workload]
+    return {"streaming": configs.STREAMING, "paper": configs.PAPER, "stack": configs.STACK,
+            "layer": configs.LAYER, "kv": configs.KV}[workload]
 
 
 def _tokens(workload):
-    cfg = {"streaming": configs.STREAMING, "stack": configs.STACK, "layer": configs.LAYER, "kv": configs.KV}[workload]
-    return cfg["chunk_len"] if workload != "kv" else cfg["n_chunks"] * cfg["chunk_len"]
+    """Tokens per step: the chunk length (the mean of the cycle for paper), the cache for kv."""
+    cfg = _cfg(workload)
+    if workload == "kv":
+        return cfg["n_chunks"] * cfg["chunk_len"]
+    lens = cfg.get("chunk_lens")
+    return sum(lens) / len(lens) if lens else cfg["chunk_len"]
 
 
 def main():
@@ -608,7 +629,7 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="streaming", choices=["streaming", "stack", "layer", "kv"])
+    ap.add_argument("--workload", default="streaming", choices=["streaming", "paper", "stack", "layer", "kv"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -672,8 +693,11 @@ def main():
     ms_per_step = t_max / args.steps
 
     # end to end through the public API: pinned host inputs copied in, score read back, every step
-    host = [x.detach().cpu().pin_memory() for x in wl.h2d_tensors(0)]
-    h2d = sum(x.numel() * x.element_size() for x in host)
+    # pinned host copies of the step inputs: one set, or one per ring slot when the chunk length
+    # cycles (the paper workload)
+    n_host = RING if len(set(getattr(wl, "lens", [0]))) > 1 else 1
+    host = [[x.detach().cpu().pin_memory() for x in wl.h2d_tensors(r)] for r in range(n_host)]
+    h2d = sum(x.numel() * x.element_size() for hs in host for x in hs) / len(host)   # mean bytes per step
     timer_off = Timer(stream)
     barrier()
     if hasattr(wl, "reset"):

@@ -10,6 +10,9 @@
                   64 chunks x 1024 tokens, Exp(1) chunk scores with exact ties, budget 16k.
 * ``streaming`` — ``stack`` with 512-token chunks plus ``kv`` caches, 4096 chunks, budget 32k,
                   the paper's policy (n_s=4, n_w=1024, N=4; Sec. 4.1).
+* ``paper``     — the paper's own stream shape (Sec. 4.1, App. A): chunks of two frames, 118-132
+                  tokens each (a cycle of eight lengths), 8 full-attention layers x 4 KV heads x
+                  D = 256, budget 8192, the paper's policy; gated-delta stack as ``stack``.
 """
 from __future__ import annotations
 
@@ -30,4 +33,11 @@ STREAMING = dict(name="streaming", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chun
                  n_chunks=4096, ring=8, Lf=8, Hkv=2, D=256, kv_dtype="bf16", budget_M=32768,
                  **PAPER_POLICY)
 
-ALL = {c["name"]: c for c in (TINY, LAYER, STACK, KV, STREAMING)}
+# chunk lengths cycle through these (118-132 tokens: two frames plus timestamps, Sec. 4.1)
+PAPER_CHUNK_LENS = (118, 132, 124, 121, 129, 119, 127, 125)
+
+PAPER = dict(name="paper", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=max(PAPER_CHUNK_LENS),
+             chunk_lens=PAPER_CHUNK_LENS, n_chunks=4096, ring=8, Lf=8, Hkv=4, D=256, kv_dtype="bf16",
+             budget_M=8192, **PAPER_POLICY)
+
+ALL = {c["name"]: c for c in (TINY, LAYER, STACK, KV, STREAMING, PAPER)}

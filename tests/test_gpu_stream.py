@@ -24,14 +24,20 @@ def _np(t):
     # wider heads, bf16, ragged chunk length, paper-like policy
     dict(L=2, Hk=2, Hv=4, d=128, dt="bf16", C=120, n_ch=12, Lf=2, Hkv=2, D=256, M=600, n_s=4, n_w=128, N=4,
          zero=False),
+    # the paper's stream shape: chunk lengths varying over 118-132 tokens, 4 KV heads, sink, window
+    # and spans (Sec. 4.1), budget a few chunks so that most chunks evict
+    dict(L=2, Hk=2, Hv=4, d=128, dt="bf16", Cs=[118, 132, 124, 121, 129, 119, 127, 125, 130, 118, 126, 131, 122, 128],
+         Lf=2, Hkv=4, D=256, M=500, n_s=4, n_w=128, N=4, zero=False),
 ])
 def test_stream_matches_oracle(cfg):
     from paper_2609_27470_gb300.stream import DeltaSStream
     dev = torch.device("cuda")
     tdt = torch.float32 if cfg["dt"] == "f32" else torch.bfloat16
-    chunks = [inputs.gdn_chunk(cfg["L"], cfg["C"], cfg["Hk"], cfg["Hv"], cfg["d"], cfg["dt"], inputs.seed_for(3, c))
+    lens = cfg["Cs"] if "Cs" in cfg else [cfg["C"]] * cfg["n_ch"]
+    cfg = dict(cfg, n_ch=len(lens), C=max(lens))
+    chunks = [inputs.gdn_chunk(cfg["L"], lens[c], cfg["Hk"], cfg["Hv"], cfg["d"], cfg["dt"], inputs.seed_for(3, c))
               for c in range(cfg["n_ch"])]
-    kvs = [inputs.kv_chunk(cfg["Lf"], cfg["Hkv"], cfg["C"], cfg["D"], cfg["dt"], inputs.seed_for(4, c))
+    kvs = [inputs.kv_chunk(cfg["Lf"], cfg["Hkv"], lens[c], cfg["D"], cfg["dt"], inputs.seed_for(4, c))
            for c in range(cfg["n_ch"])]
     s0 = (torch.zeros(cfg["L"], cfg["Hv"], cfg["d"], cfg["d"]) if cfg["zero"]
           else inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 5))
