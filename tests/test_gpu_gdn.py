@@ -172,6 +172,16 @@ def test_gdn_update_slow_decay_four_chunks(L):
         state = st.cpu()
 
 
+@pytest.mark.parametrize("Hk,Hv", [(2, 6), (4, 4)])
+def test_gdn_update_other_head_groupings(L, Hk, Hv):
+    """Key heads serving three value heads and one value head each (the other cases share a key
+    head between two): the key-head index of every value head, several tiles and a ragged tail,
+    two layers."""
+    x = inputs.gdn_chunk(2, 257, Hk, Hv, 128, "bf16", inputs.seed_for(15, Hk, Hv))
+    state0 = inputs.initial_state(2, Hv, 128, 16)
+    _check_chunk(L, x, state0, False, torch.bfloat16, None)
+
+
 @pytest.mark.parametrize("decay_scale", [0.0, 4.0])
 def test_gdn_update_decay_extremes(L, decay_scale):
     """No decay (g = 0: alpha = 1, the deferred decay never moves) and very strong decay (a tile's
