@@ -424,7 +424,74 @@ KERNEL_SOURCES = {"gdn_update": "paper_2609_27470_gb300/csrc/gdn_tc.cu",
                   "compact": "paper_2609_27470_gb300/csrc/compact.cu",
                   "select": "paper_2609_27470_gb300/csrc/select.cu",
                   "score": "paper_2609_27470_gb300/csrc/drift.cu",
-                  "append": "paper_2609_27470_gb300/csrc/compact.cu"}
+                  "append": "paper_2609_27470_gb300/csrc/compact.cu",
+                  "snapshot": "paper_2609_27470_gb300/csrc/snapshot.cu",
+                  "restore": "paper_2609_27470_gb300/csrc/snapshot.cu"}
+
+
+class SnapshotWorkload:
+    """Question-time snapshot and restore (Sec. 3.3) of a paper-shaped stream at its budget: the
+    24 x 32 x 128 x 128 fp32 recurrent state (48 MiB), the 8,192-token caches of 8 layers x 4 KV
+    heads (256 MiB), the slots' chunk ids and positions and 4,096 chunk scores.  A step saves the
+    whole state and puts it back (deltas_copy_stream_state twice: one launch each)."""
+    name = "snapshot"
+
+    def __init__(self, dev, L, cfg=None):
+        cfg = dict(cfg or configs.PAPER)
+        self.cfg = cfg
+        self.L = L
+        from paper_2609_27470_gb300.stream import DeltaSStream, StreamSnapshot
+        self.s = DeltaSStream(num_layers=cfg["L"], num_k_heads=cfg["Hk"], num_v_heads=cfg["Hv"], head_dim=cfg["d"],
+                              act_dtype=torch.bfloat16, kv_layers=cfg["Lf"], kv_heads=cfg["Hkv"],
+                              kv_head_dim=cfg["D"], kv_dtype=torch.bfloat16, budget_M=cfg["budget_M"],
+                              n_sink=cfg["n_sink"], n_window=cfg["n_window"], n_buckets=cfg["n_buckets"],
+                              chunk_len=cfg["chunk_len"], max_chunks=cfg["n_chunks"],
+                              state0=inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 90, device=dev),
+                              device=dev)
+        s = self.s
+        k, v = inputs.kv_cache(cfg["Lf"], cfg["Hkv"], s.capacity, cfg["D"], "bf16", seed=91, device=dev)
+        s.k_cache.copy_(k)
+        s.v_cache.copy_(v)
+        del k, v
+        M = cfg["budget_M"]
+        s.tok_chunk[:M] = torch.arange(M, device=dev, dtype=torch.int32) // cfg["chunk_len"]
+        s.tok_pos[:M] = torch.arange(M, device=dev, dtype=torch.int32) * 3
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(92)
+        s.chunk_scores.exponential_(1.0, generator=gen)
+        s.cache_len, s.position, s.chunk = M, 3 * M, cfg["n_chunks"]
+        self.snap = StreamSnapshot(s, full=True)
+
+    def step(self, timer):
+        with timer.mark("snapshot"):
+            self.s.snapshot(into=self.snap)
+        with timer.mark("restore"):
+            self.s.restore(self.snap)
+
+    def bytes_per_copy(self):
+        c, s = self.cfg, self.s
+        return (s.state.numel() * 4 + s.chunk * 4 + 2 * c["Lf"] * c["Hkv"] * s.cache_len * c["D"] * 2
+                + 2 * s.cache_len * 4)
+
+    def launches_per_step(self):
+        return 2
+
+    def tokens_per_step(self):
+        return self.s.cache_len
+
+    def kernel_roofline(self, name, avg_ms, peaks, steps):
+        by = 2.0 * self.bytes_per_copy()                       # every byte read once and written once
+        return {"bound": "hbm", "achieved": by / (avg_ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "bytes_per_launch": by}
+
+    def post_step(self):
+        pass
+
+    def h2d_tensors(self, i=0):
+        return [self.s.chunk_scores]
+
+    def result_scalar(self):
+        return self.s.chunk_scores[:1]
 
 
 def make_workload(name, dev, L):
@@ -438,6 +505,8 @@ def make_workload(name, dev, L):
         return GdnOnlyWorkload(dev, L, configs.LAYER)
     if name == "kv":
         return KvWorkload(dev, L)
+    if name == "snapshot":
+        return SnapshotWorkload(dev, L)
     raise ValueError(name)
 
 
@@ -544,6 +613,22 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         t_head = (time.perf_counter() - t0) / reps
         total += t_head * heads_total
         parts.append(f"gdn: {reps} (layer,head) x {C} tokens, x{heads_total / reps:.0f} extrapolated")
+    if workload == "snapshot":
+        # the oracle's question handling copies the whole stream state (numpy .copy()); timed on
+        # a 64 MiB slice and scaled to the bytes of one save and one restore
+        M = cfg["budget_M"]
+        per_copy = (cfg["L"] * cfg["Hv"] * cfg["d"] ** 2 * 8 + cfg["n_chunks"] * 4
+                    + 2 * cfg["Lf"] * cfg["Hkv"] * M * cfg["D"] * 2 + 2 * M * 4)
+        a = np.random.default_rng(7).standard_normal(8 << 20)
+        t0 = time.perf_counter()
+        reps = 0
+        while reps < 2 or time.perf_counter() - t0 < budget_s * 0.25:
+            a.copy()
+            reps += 1
+        t_byte = (time.perf_counter() - t0) / (reps * a.nbytes)
+        total += 2 * per_copy * t_byte
+        parts.append(f"numpy copy of 64 MiB x{reps}, scaled to 2 x {per_copy / 2**20:.0f} MiB "
+                     "(fp64 state, as the oracle keeps it)")
     if workload in ("streaming", "paper", "kv"):
         M = cfg["budget_M"]
         if workload != "kv":
@@ -606,12 +691,16 @@ def config_line(workload):
             line[key] = c[key]
     if workload == "kv":
         line["cache_len"] = c["n_chunks"] * c["chunk_len"]
+    if workload == "snapshot":
+        line["cache_len"] = c["budget_M"]
+        line["copied"] = "state, chunk scores, live cache rows, chunk ids, positions: snapshot + restore per step"
+        line["inputs"] = "one stream state generated on device"
     return line
 
 
 def _cfg(workload):
     return {"streaming": configs.STREAMING, "paper": configs.PAPER, "stack": configs.STACK,
-            "layer": configs.LAYER, "kv": configs.KV}[workload]
+            "layer": configs.LAYER, "kv": configs.KV, "snapshot": configs.PAPER}[workload]
 
 
 def _tokens(workload):
@@ -619,6 +708,8 @@ def _tokens(workload):
     cfg = _cfg(workload)
     if workload == "kv":
         return cfg["n_chunks"] * cfg["chunk_len"]
+    if workload == "snapshot":
+        return cfg["budget_M"]
     lens = cfg.get("chunk_lens")
     return sum(lens) / len(lens) if lens else cfg["chunk_len"]
 
@@ -629,7 +720,8 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="streaming", choices=["streaming", "paper", "stack", "layer", "kv"])
+    ap.add_argument("--workload", default="streaming",
+                    choices=["streaming", "paper", "stack", "layer", "kv", "snapshot"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)

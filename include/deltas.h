@@ -251,6 +251,41 @@ DELTAS_API deltas_status deltas_append_kv(const deltas_kv_desc* desc, void* k_ca
                                int32_t chunk_id, int32_t first_pos, void* stream);
 
 /* ------------------------------------------------------------------------------------------ */
+/* Question-time snapshot and restore (Sec. 3.3, "Question answering": before a question the  */
+/* stream state, both memories, is saved; after the answer it is restored together with the    */
+/* retention scores and chunk indices, so that question turns leave the stream unchanged).      */
+/*                                                                                              */
+/* A stream state is the set of buffers below.  src and dst are two such sets laid out by the  */
+/* same descriptors (snapshot: live -> saved copy; restore: saved copy -> live):                */
+/*   state          [L][Hv][d_v][d_k] fp32 (gdn desc)             copied whole;                  */
+/*   chunk_scores   fp32                                          entries 0 .. n_chunks - 1;     */
+/*   k_cache, v_cache [Lf][Hkv][capacity][D] (kv desc dtype)      rows 0 .. cache_len - 1 of     */
+/*                                                                every plane;                   */
+/*   tok_chunk, tok_pos [capacity] int32                          entries 0 .. cache_len - 1.    */
+/* kv == NULL copies state and scores only; the four cache pointers of both sets must then be  */
+/* NULL.  That is enough when the question appends to the caches but evicts nothing: the rows  */
+/* it appends lie past cache_len, which the caller restores on the host along with the stream  */
+/* position and the chunk counter (the library keeps none of them).  Everything moves in one    */
+/* kernel launch on `stream`, 16 bytes per load and store; the sets must not overlap.           */
+/* Errors (nothing enqueued): INVALID_ARGUMENT for a NULL required pointer, a pointer that is   */
+/* not 16-byte aligned, n_chunks < 0, cache_len outside [0, capacity], or overlapping source   */
+/* and destination ranges; the descriptor checks of the other calls.                           */
+/* ------------------------------------------------------------------------------------------ */
+typedef struct {
+    float* state;
+    float* chunk_scores;
+    void* k_cache;
+    void* v_cache;
+    int32_t* tok_chunk;
+    int32_t* tok_pos;
+} deltas_stream_buffers;
+
+DELTAS_API deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, const deltas_kv_desc* kv,
+                                       int32_t cache_len, int32_t n_chunks,
+                                       const deltas_stream_buffers* src,
+                                       const deltas_stream_buffers* dst, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
 /* Device status word (first 16 bytes of a workspace).                                          */
 /* ------------------------------------------------------------------------------------------ */
 

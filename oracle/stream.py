@@ -11,6 +11,11 @@ Test infrastructure only.  One iteration per arriving chunk c:
    the in-stream-order gather of every cache, keeping original positions.
 
 Scores of earlier chunks are reused at later evictions (Sec. 3.3).
+
+A question (Sec. 3.3, "Question answering") arriving before chunk c saves the whole stream state
+(recurrent state, caches with chunk ids and positions, scores, counters), runs the question's
+tokens through the same loop body, and then puts the saved state back: question turns change
+nothing that later chunks see.
 """
 from __future__ import annotations
 
@@ -32,17 +37,21 @@ class StreamResult:
     cache_len: int
     states_after_chunk: list = field(default_factory=list)
     evictions: list = field(default_factory=list)   # (chunk, retain_idx) per eviction event
+    question_states: list = field(default_factory=list)   # S right after each question, before the restore
 
 
 def run_stream(chunk_inputs, kv_inputs, state0, n_chunks: int, policy: dict, capacity: int,
-               q_scale: float | None = None, score_override=None, keep_states: bool = False):
+               q_scale: float | None = None, score_override=None, keep_states: bool = False,
+               questions: dict | None = None):
     """Run Alg. 1 over ``n_chunks`` chunks.
 
     ``chunk_inputs(c)`` -> (q, k, v, g, beta) numpy arrays in the oracle layouts;
     ``kv_inputs(c)`` -> (k_new, v_new) of shape [Lf,Hkv,C,D];
     ``policy`` = dict(budget_M, n_sink, n_window, n_buckets);
     ``score_override`` (optional) [n_chunks] float32: scores to rank with instead of the oracle's
-    own (so that selection can be compared given identical scores).
+    own (so that selection can be compared given identical scores);
+    ``questions`` (optional) {c: () -> ((q, k, v, g, beta), (k_new, v_new))}: a question arriving
+    before chunk c, run as a loop body and then undone.
     """
     S = np.array(state0, dtype=np.float64, copy=True)
     scores = np.zeros(n_chunks, dtype=np.float32)
@@ -52,11 +61,13 @@ def run_stream(chunk_inputs, kv_inputs, state0, n_chunks: int, policy: dict, cap
     T = 0
     pos = 0
     res = StreamResult(S, scores, None, None, tok_chunk, tok_pos, 0)
-    for c in range(n_chunks):
-        q, k, v, g, beta = chunk_inputs(c)
+
+    def body(c, gdn_in, kv_in, rank_scores_of):
+        nonlocal S, kc, vc, tok_chunk, tok_pos, T, pos
+        q, k, v, g, beta = gdn_in
         s_before = S.copy()
         S, _ = gdn_recurrence(None, k, v, g, beta, S, q_scale=q_scale)
-        k_new, v_new = kv_inputs(c)
+        k_new, v_new = kv_in
         Lf, Hkv, C, D = k_new.shape
         if kc is None:
             kc = np.zeros((Lf, Hkv, capacity, D), dtype=k_new.dtype)
@@ -70,16 +81,30 @@ def run_stream(chunk_inputs, kv_inputs, state0, n_chunks: int, policy: dict, cap
         T += C
         pos += C
         scores[c] = np.float32(state_drift(s_before, S))
+        if T > policy["budget_M"]:
+            idx, _ = select_retain(policy["budget_M"], policy["n_sink"], policy["n_window"],
+                                   policy["n_buckets"], tok_chunk[:T], rank_scores_of()[: c + 1])
+            kc, vc, tok_chunk, tok_pos = compact_kv(kc, vc, tok_chunk, tok_pos, idx, T)
+            T = int(idx.shape[0])
+            return idx
+        return None
+
+    for c in range(n_chunks):
+        if questions and c in questions:
+            saved = (S.copy(), scores.copy(), None if kc is None else kc.copy(), None if vc is None else vc.copy(),
+                     tok_chunk.copy(), tok_pos.copy(), T, pos)
+            gdn_q, kv_q = questions[c]()
+            body(c, gdn_q, kv_q, lambda: scores)
+            res.question_states.append(S.copy())
+            S, scores, kc, vc, tok_chunk, tok_pos, T, pos = saved
+        idx = body(c, chunk_inputs(c), kv_inputs(c),
+                   lambda: scores if score_override is None else np.asarray(score_override, np.float32))
         if keep_states:
             res.states_after_chunk.append(S.copy())
-        if T > policy["budget_M"]:
-            rank_scores = scores if score_override is None else np.asarray(score_override, np.float32)
-            idx, _ = select_retain(policy["budget_M"], policy["n_sink"], policy["n_window"],
-                                   policy["n_buckets"], tok_chunk[:T], rank_scores[: c + 1])
-            kc, vc, tok_chunk, tok_pos = compact_kv(kc, vc, tok_chunk, tok_pos, idx, T)
+        if idx is not None:
             res.evictions.append((c, idx))
-            T = int(idx.shape[0])
     res.state = S
+    res.chunk_scores = scores
     res.k_cache, res.v_cache = kc, vc
     res.tok_chunk, res.tok_pos = tok_chunk, tok_pos
     res.cache_len = T

@@ -37,7 +37,7 @@ EXPORTED = (
     "deltas_score_chunks",
     "deltas_select_retain_workspace_size", "deltas_select_retain", "deltas_select_retain_static",
     "deltas_compact_kv_workspace_size", "deltas_compact_kv",
-    "deltas_append_kv",
+    "deltas_append_kv", "deltas_copy_stream_state",
     "deltas_clear_device_status", "deltas_get_device_status",
 )
 
@@ -89,6 +89,7 @@ _sig("deltas_select_retain_static", ctypes.c_int, _P, _I32, _I32, _P, _P, _P, _P
 _sig("deltas_compact_kv_workspace_size", _SZ, _P, _I32)
 _sig("deltas_compact_kv", ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, _I32, _P, _SZ, _P)
 _sig("deltas_append_kv", ctypes.c_int, _P, _P, _P, _P, _P, _I32, _P, _P, _I32, _I32, _I32, _P)
+_sig("deltas_copy_stream_state", ctypes.c_int, _P, _P, _I32, _I32, _P, _P, _P)
 _sig("deltas_clear_device_status", ctypes.c_int, _P, _P)
 _sig("deltas_get_device_status", ctypes.c_int, _P, _P, _P, _P)
 
@@ -272,6 +273,42 @@ def deltas_append_kv(desc: KvDesc, k_cache, v_cache, tok_chunk, tok_pos, cache_l
                                _ptr(k_new, dt, nshp, "k_new"), _ptr(v_new, dt, nshp, "v_new"), n_new,
                                int(chunk_id), int(first_pos), _stream(stream))
     _check(st, "deltas_append_kv")
+
+
+STREAM_BUFFERS = ("state", "chunk_scores", "k_cache", "v_cache", "tok_chunk", "tok_pos")
+
+
+class StreamBuffers(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in STREAM_BUFFERS]
+
+
+def deltas_copy_stream_state(gdn: GdnDesc, kv: KvDesc | None, cache_len: int, n_chunks: int, src: dict, dst: dict,
+                             stream=None):
+    """Copy a stream state between two buffer sets (dicts keyed by STREAM_BUFFERS; the cache
+    entries None when kv is None)."""
+    sshape = (gdn.num_layers, gdn.num_v_heads, gdn.value_dim, gdn.key_dim)
+    shapes = {"state": (torch.float32, sshape), "chunk_scores": (torch.float32, None),
+              "tok_chunk": (torch.int32, (kv.capacity,) if kv else None),
+              "tok_pos": (torch.int32, (kv.capacity,) if kv else None)}
+    if kv is not None:
+        cshape = (kv.num_layers, kv.num_kv_heads, kv.capacity, kv.head_dim)
+        shapes["k_cache"] = shapes["v_cache"] = (_TORCH_DT[kv.dtype], cshape)
+
+    def pack(d, side):
+        vals = []
+        for n in STREAM_BUFFERS:
+            t = d.get(n)
+            if t is not None and n == "chunk_scores" and t.numel() < n_chunks:
+                raise ValueError(f"{side} chunk_scores holds fewer than {n_chunks} entries")
+            dt, shp = shapes.get(n, (None, None))
+            vals.append(_ptr(t, dt, shp, f"{side} {n}"))
+        return StreamBuffers(*vals)
+
+    s, d = pack(src, "src"), pack(dst, "dst")
+    st = _lib.deltas_copy_stream_state(ctypes.byref(gdn), ctypes.byref(kv) if kv is not None else None,
+                                       int(cache_len), int(n_chunks), ctypes.byref(s), ctypes.byref(d),
+                                       _stream(stream))
+    _check(st, "deltas_copy_stream_state")
 
 
 def deltas_clear_device_status(workspace, stream=None):

@@ -221,6 +221,69 @@ deltas_status deltas_append_kv(const deltas_kv_desc* desc, void* k_cache, void* 
                                       as_stream(stream)));
 }
 
+deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, const deltas_kv_desc* kv,
+                                       int32_t cache_len, int32_t n_chunks,
+                                       const deltas_stream_buffers* src,
+                                       const deltas_stream_buffers* dst, void* stream)
+{
+    deltas_status st = check_gdn_desc(gdn);
+    if (st != DELTAS_OK) return st;
+    if (src == nullptr || dst == nullptr || n_chunks < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!src->state || !dst->state) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (n_chunks > 0 && (!src->chunk_scores || !dst->chunk_scores)) return DELTAS_ERR_INVALID_ARGUMENT;
+    const void* cache_ptrs[8] = {src->k_cache, src->v_cache, src->tok_chunk, src->tok_pos,
+                                 dst->k_cache, dst->v_cache, dst->tok_chunk, dst->tok_pos};
+    if (kv == nullptr) {
+        for (const void* p : cache_ptrs)
+            if (p != nullptr) return DELTAS_ERR_INVALID_ARGUMENT;
+    } else {
+        st = check_kv_desc(kv);
+        if (st != DELTAS_OK) return st;
+        if (cache_len < 0 || cache_len > kv->capacity) return DELTAS_ERR_INVALID_ARGUMENT;
+        for (const void* p : cache_ptrs)
+            if (p == nullptr || !aligned16(p)) return DELTAS_ERR_INVALID_ARGUMENT;
+    }
+    if (!aligned16(src->state) || !aligned16(dst->state)) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (n_chunks > 0 && (!aligned16(src->chunk_scores) || !aligned16(dst->chunk_scores)))
+        return DELTAS_ERR_INVALID_ARGUMENT;
+
+    CopyBatch b;
+    b.n = 0;
+    auto add = [&](const void* from, void* to, uint64_t row_bytes, uint64_t stride, int64_t rows) {
+        if (row_bytes == 0 || rows == 0) return;
+        CopySeg& g = b.seg[b.n++];
+        g.src = static_cast<const uint8_t*>(from); g.dst = static_cast<uint8_t*>(to);
+        g.row_bytes = row_bytes; g.stride = stride; g.rows = rows;
+    };
+    add(src->state, dst->state,
+        (uint64_t)gdn->num_layers * gdn->num_v_heads * gdn->value_dim * gdn->key_dim * 4, 0, 1);
+    add(src->chunk_scores, dst->chunk_scores, (uint64_t)n_chunks * 4, 0, 1);
+    if (kv != nullptr) {
+        const uint64_t rb = (uint64_t)kv->head_dim * elt_bytes(kv->dtype);
+        const int64_t planes = (int64_t)kv->num_layers * kv->num_kv_heads;
+        add(src->k_cache, dst->k_cache, rb * cache_len, rb * kv->capacity, planes);
+        add(src->v_cache, dst->v_cache, rb * cache_len, rb * kv->capacity, planes);
+        add(src->tok_chunk, dst->tok_chunk, (uint64_t)cache_len * 4, 0, 1);
+        add(src->tok_pos, dst->tok_pos, (uint64_t)cache_len * 4, 0, 1);
+    }
+    // no destination range may overlap a source range or another destination range
+    auto extent_end = [](const CopySeg& g) { return (uint64_t)(g.rows - 1) * g.stride + g.row_bytes; };
+    auto overlap = [](uintptr_t a0, uint64_t an, uintptr_t b0, uint64_t bn) {
+        return a0 < b0 + bn && b0 < a0 + an;
+    };
+    for (int i = 0; i < b.n; ++i) {
+        const uintptr_t d0 = reinterpret_cast<uintptr_t>(b.seg[i].dst);
+        const uint64_t dn = extent_end(b.seg[i]);
+        for (int j = 0; j < b.n; ++j) {
+            if (overlap(d0, dn, reinterpret_cast<uintptr_t>(b.seg[j].src), extent_end(b.seg[j])))
+                return DELTAS_ERR_INVALID_ARGUMENT;
+            if (j != i && overlap(d0, dn, reinterpret_cast<uintptr_t>(b.seg[j].dst), extent_end(b.seg[j])))
+                return DELTAS_ERR_INVALID_ARGUMENT;
+        }
+    }
+    return from_cuda(launch_copy_batch(b, as_stream(stream)));
+}
+
 deltas_status deltas_clear_device_status(void* workspace, void* stream) {
     if (workspace == nullptr) return DELTAS_ERR_WORKSPACE;
     return from_cuda(cudaMemsetAsync(workspace, 0, 16, as_stream(stream)));

@@ -66,6 +66,21 @@ struct KvPlanes {
     int32_t* tok_pos;
 };
 
+// A batch of row copies for one kernel: segment s moves `rows` rows of row_bytes bytes (16-byte
+// aligned rows, row_bytes a multiple of 4), row r at src + r * stride to dst + r * stride.
+struct CopySeg {
+    const uint8_t* src;
+    uint8_t* dst;
+    uint64_t row_bytes;
+    uint64_t stride;
+    int64_t rows;
+};
+constexpr int kMaxCopySegs = 8;
+struct CopyBatch {
+    CopySeg seg[kMaxCopySegs];
+    int n;
+};
+
 // Kernel launchers (return the launch error, cudaSuccess when enqueued).
 cudaError_t launch_gdn_update_simt(const GdnArgs& a, cudaStream_t s);
 bool gdn_tc_supported(const GdnArgs& a);
@@ -83,6 +98,7 @@ cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_
 size_t compact_workspace_bytes(const KvPlanes& kv, int cache_len);
 cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, const int32_t* n_retained,
                               int cache_len, void* ws, int32_t* status, cudaStream_t s);
+cudaError_t launch_copy_batch(const CopyBatch& b, cudaStream_t s);
 cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_new, const void* v_new,
                              int n_new, int chunk_id, int first_pos, cudaStream_t s);
 

@@ -12,12 +12,32 @@ Per arriving chunk c, all on one CUDA stream and with no host synchronisation:
 
 The host tracks the cache length without reading the device: after an eviction it is exactly M
 (the selection keeps min(T, M) tokens).
+
+Questions (Sec. 3.3): ``snapshot()`` saves the stream state before a question and ``restore()``
+puts it back after the answer (``deltas_copy_stream_state``: the recurrent state, the chunk
+scores, and unless ``full=False`` the live cache rows with their chunk ids and positions; the host
+counters travel with it), so whatever the question ran on the stream in between, appends,
+updates or evictions, leaves no trace in the subsequent stream.
 """
 from __future__ import annotations
 
 import torch
 
 from . import _lib as L
+
+
+class StreamSnapshot:
+    """A saved stream state: device copies of the buffers ``deltas_copy_stream_state`` moves and
+    the host counters.  ``full=False`` keeps the recurrent state and the scores only (enough when
+    the question appends to the caches but evicts nothing)."""
+
+    def __init__(self, s: "DeltaSStream", full: bool = True):
+        self.full = full
+        self.buffers = {"state": torch.empty_like(s.state), "chunk_scores": torch.empty_like(s.chunk_scores)}
+        if full:
+            for n in ("k_cache", "v_cache", "tok_chunk", "tok_pos"):
+                self.buffers[n] = torch.empty_like(getattr(s, n))
+        self.cache_len = self.position = self.chunk = self.evictions = 0
 
 
 class DeltaSStream:
@@ -78,3 +98,29 @@ class DeltaSStream:
             self.evictions += 1
             return True
         return False
+
+    def _buffers(self, full: bool) -> dict:
+        b = {"state": self.state, "chunk_scores": self.chunk_scores}
+        if full:
+            b.update(k_cache=self.k_cache, v_cache=self.v_cache, tok_chunk=self.tok_chunk, tok_pos=self.tok_pos)
+        return b
+
+    def snapshot(self, full: bool = True, into: StreamSnapshot | None = None, stream=None) -> StreamSnapshot:
+        """Save the stream state before a question (Sec. 3.3); ``into`` reuses a snapshot's buffers."""
+        snap = into if into is not None else StreamSnapshot(self, full)
+        if snap.full != full:
+            raise ValueError("the snapshot's buffers were made for the other kind of snapshot")
+        L.deltas_copy_stream_state(self.gdn, self.kv if full else None, self.cache_len, self.chunk,
+                                   self._buffers(full), snap.buffers, stream)
+        snap.cache_len, snap.position, snap.chunk, snap.evictions = (self.cache_len, self.position, self.chunk,
+                                                                     self.evictions)
+        return snap
+
+    def restore(self, snap: StreamSnapshot, stream=None):
+        """Put the stream back to ``snap`` after the answer: nothing the question ran remains."""
+        if not snap.full and self.evictions != snap.evictions:
+            raise ValueError("the question evicted from the cache: only a full snapshot can restore it")
+        L.deltas_copy_stream_state(self.gdn, self.kv if snap.full else None, snap.cache_len, snap.chunk,
+                                   snap.buffers, self._buffers(snap.full), stream)
+        self.cache_len, self.position, self.chunk, self.evictions = (snap.cache_len, snap.position, snap.chunk,
+                                                                     snap.evictions)

@@ -25,7 +25,7 @@ def _declared():
 
 def test_every_declared_symbol_is_exported(L):
     names = _declared()
-    assert len(names) == 15, names
+    assert len(names) == 16, names
     lib = ctypes.CDLL(L.LIB_PATH)
     for n in names:
         assert hasattr(lib, n), n
@@ -116,3 +116,39 @@ def test_binding_refuses_cpu_tensors(L):
     with pytest.raises(ValueError):
         L.deltas_gdn_chunk_update(d, 4, x, x, x, torch.zeros(1, 4, 1), torch.zeros(1, 4, 1),
                                   torch.zeros(1, 1, 16, 16), None, None, torch.zeros(256, dtype=torch.uint8))
+
+
+def test_copy_stream_state_argument_checks(L):
+    """Snapshot / restore (deltas_copy_stream_state): every bad argument is refused on the host
+    before anything is enqueued (the addresses below are never dereferenced)."""
+    raw = L.raw()
+    gdn = L.GdnDesc(2, 2, 4, 16, 16, L.DELTAS_F32, 0.25)
+    kv = L.KvDesc(2, 2, 64, L.DELTAS_BF16, 1000)
+    MB = 1 << 20
+    full = lambda base: L.StreamBuffers(base, base + MB, base + 2 * MB, base + 3 * MB, base + 4 * MB, base + 5 * MB)
+    light = lambda base: L.StreamBuffers(base, base + MB, None, None, None, None)
+
+    def call(src, dst, kvd=kv, cache_len=500, n_chunks=7, desc=gdn):
+        return raw.deltas_copy_stream_state(ctypes.byref(desc) if desc else None,
+                                            ctypes.byref(kvd) if kvd else None, cache_len, n_chunks,
+                                            ctypes.byref(src) if src else None, ctypes.byref(dst) if dst else None,
+                                            None)
+    A, B = 1 << 28, 1 << 30
+    bad = L.DELTAS_ERR_INVALID_ARGUMENT
+    assert call(full(A), full(B), desc=None) == bad
+    assert call(None, full(B)) == bad
+    assert call(full(A), None) == bad
+    assert call(full(A), full(B), n_chunks=-1) == bad
+    assert call(full(A), full(B), cache_len=1001) == bad                 # past the capacity
+    assert call(full(A), full(B), cache_len=-1) == bad
+    assert call(full(A), full(B), kvd=None) == bad                       # cache pointers without a kv desc
+    assert call(light(A), light(B), kvd=kv) == bad                       # a kv desc without cache pointers
+    mis = full(A)
+    mis.v_cache = A + 3 * MB + 8                                          # not 16-byte aligned
+    assert call(mis, full(B)) == bad
+    assert call(full(A), full(A)) == bad                                 # a set copied onto itself
+    ov = full(B)
+    ov.state = A + 2 * MB + 4096                                          # inside the source k_cache
+    assert call(full(A), ov) == bad
+    assert call(full(A), full(B), kvd=L.KvDesc(2, 2, 7, L.DELTAS_F32, 1000)) == L.DELTAS_ERR_UNSUPPORTED
+    assert call(full(A), full(B), desc=L.GdnDesc(2, 2, 4, 24, 24, L.DELTAS_F32, 0.25)) == L.DELTAS_ERR_UNSUPPORTED

@@ -409,3 +409,34 @@ def test_stream_loop_invariants_tiny():
     pos = res.tok_pos[: res.cache_len]
     assert np.all(np.diff(pos) > 0) and pos[:4].tolist() == [0, 1, 2, 3]
     assert pos[-64:].tolist() == list(range(n_ch * C - 64, n_ch * C))
+
+
+def test_question_turn_leaves_stream_unchanged():
+    """Sec. 3.3: a question saved-and-restored around changes nothing later chunks see.  The
+    question (one chunk of other tokens) does run: it moves the state and, with the cache at its
+    budget, forces an eviction; after the restore the stream equals a run without it, exactly."""
+    rng = np.random.default_rng(43)
+    L, Hk, Hv, d, C, n_ch = 1, 2, 2, 16, 64, 8
+    chunks = [_rand_inputs(rng, L, C, Hk, Hv, d) for _ in range(n_ch)]
+    kvs = [(rng.standard_normal((1, 2, C, 16)).astype(np.float32),
+            rng.standard_normal((1, 2, C, 16)).astype(np.float32)) for _ in range(n_ch)]
+    qin = _rand_inputs(rng, L, C, Hk, Hv, d)
+    qkv = (rng.standard_normal((1, 2, C, 16)).astype(np.float32),
+           rng.standard_normal((1, 2, C, 16)).astype(np.float32))
+    policy = dict(budget_M=256, n_sink=4, n_window=64, n_buckets=2)
+    s0 = np.zeros((L, Hv, d, d))
+    plain = run_stream(lambda c: chunks[c], lambda c: kvs[c], s0, n_ch, policy, capacity=256 + C,
+                       keep_states=True)
+    asked = run_stream(lambda c: chunks[c], lambda c: kvs[c], s0, n_ch, policy, capacity=256 + C,
+                       questions={5: lambda: (qin, qkv)})
+    assert len(asked.question_states) == 1
+    assert not np.allclose(asked.question_states[0], plain.states_after_chunk[4])
+    assert len(asked.evictions) == len(plain.evictions)
+    np.testing.assert_array_equal(asked.state, plain.state)
+    np.testing.assert_array_equal(asked.chunk_scores, plain.chunk_scores)
+    assert asked.cache_len == plain.cache_len
+    for name in ("k_cache", "v_cache", "tok_chunk", "tok_pos"):
+        np.testing.assert_array_equal(getattr(asked, name), getattr(plain, name))
+    for (c1, i1), (c2, i2) in zip(asked.evictions, plain.evictions):
+        assert c1 == c2
+        np.testing.assert_array_equal(i1, i2)
