@@ -216,7 +216,7 @@ class StreamingWorkload:
                               n_sink=cfg["n_sink"], n_window=cfg["n_window"], n_buckets=cfg["n_buckets"],
                               chunk_len=C, max_chunks=cfg["n_chunks"],
                               state0=inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 42, device=dev),
-                              device=dev)
+                              device=dev, signal=cfg.get("signal", "drift"))
         # fill the cache to exactly the budget (setup, not timed): appended chunks with Exp(1)
         # scores, the last one cut to fit, so that every timed step evicts
         M = cfg["budget_M"]
@@ -245,9 +245,12 @@ class StreamingWorkload:
         s, L, c = self.s, self.L, self.s.chunk
         with timer.mark("gdn_update"):
             L.deltas_gdn_chunk_update(s.gdn, T, None, x["k"], x["v"], x["g"], x["beta"], s.state, None,
-                                      s.partials, s.workspace)
+                                      s.partials, s.workspace, write_norms=s.write_norms)
         with timer.mark("score"):
-            L.deltas_score_chunks(s.gdn.num_layers, s.gdn.num_v_heads, s.partials, c, s.chunk_scores)
+            if s.signal == "write_norm":
+                L.deltas_score_write_norms(s.gdn.num_layers, s.gdn.num_v_heads, s.write_norms, T, c, s.chunk_scores)
+            else:
+                L.deltas_score_chunks(s.gdn.num_layers, s.gdn.num_v_heads, s.partials, c, s.chunk_scores)
         with timer.mark("append"):
             L.deltas_append_kv(s.kv, s.k_cache, s.v_cache, s.tok_chunk, s.tok_pos, s.cache_len, kn, vn, c,
                                s.position)
@@ -499,6 +502,8 @@ def make_workload(name, dev, L):
         return StreamingWorkload(dev, L)
     if name == "paper":
         return StreamingWorkload(dev, L, configs.PAPER)
+    if name == "paper_write_norm":
+        return StreamingWorkload(dev, L, configs.PAPER_WRITE_NORM)
     if name == "stack":
         return GdnOnlyWorkload(dev, L, configs.STACK)
     if name == "layer":
@@ -593,7 +598,7 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
     cfg = _cfg(workload)
     parts = []
     total = 0.0
-    if workload in ("streaming", "paper", "stack", "layer"):
+    if workload in ("streaming", "paper", "paper_write_norm", "stack", "layer"):
         C = int(round(_tokens(workload)))
         heads_total = cfg["L"] * cfg["Hv"]
         n_heads = 2
@@ -603,8 +608,11 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         t0 = time.perf_counter()
         reps = 0
         while True:
-            S, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
-            oracle.drift_partials(s0, S)
+            if workload == "paper_write_norm":
+                S, _, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0, want_write_norms=True)
+            else:
+                S, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
+                oracle.drift_partials(s0, S)
             reps += 1
             if reps >= n_heads and time.perf_counter() - t0 > budget_s * 0.5:
                 break
@@ -629,7 +637,7 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         total += 2 * per_copy * t_byte
         parts.append(f"numpy copy of 64 MiB x{reps}, scaled to 2 x {per_copy / 2**20:.0f} MiB "
                      "(fp64 state, as the oracle keeps it)")
-    if workload in ("streaming", "paper", "kv"):
+    if workload in ("streaming", "paper", "paper_write_norm", "kv"):
         M = cfg["budget_M"]
         if workload != "kv":
             T = M + cfg["chunk_len"]
@@ -686,7 +694,7 @@ def config_line(workload):
     line = {"workload": workload, "l2": "flushed between timed steps (256 MiB write)",
             "inputs": "ring of 8 distinct per-chunk input sets, generated on device"}
     for key in ("L", "Hk", "Hv", "d", "chunk_len", "chunk_lens", "Lf", "Hkv", "D", "budget_M", "n_sink",
-                "n_window", "n_buckets"):
+                "n_window", "n_buckets", "signal"):
         if key in c:
             line[key] = c[key]
     if workload == "kv":
@@ -700,7 +708,8 @@ def config_line(workload):
 
 def _cfg(workload):
     return {"streaming": configs.STREAMING, "paper": configs.PAPER, "stack": configs.STACK,
-            "layer": configs.LAYER, "kv": configs.KV, "snapshot": configs.PAPER}[workload]
+            "layer": configs.LAYER, "kv": configs.KV, "snapshot": configs.PAPER,
+            "paper_write_norm": configs.PAPER_WRITE_NORM}[workload]
 
 
 def _tokens(workload):
@@ -721,7 +730,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="streaming",
-                    choices=["streaming", "paper", "stack", "layer", "kv", "snapshot"])
+                    choices=["streaming", "paper", "paper_write_norm", "stack", "layer", "kv", "snapshot"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)

@@ -138,6 +138,31 @@ DELTAS_API deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, in
                                       void* workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------------------------ */
+/* The same update, also returning the comparison signal of Sec. 4.3 (the write size of HOLA's */
+/* score, as the appendix describes it): the rank-one write of token t is u_t k_t^T with        */
+/* u_t = beta_t (v_t - alpha_t S_{t-1} k_t), of Frobenius norm ||u_t||_2 for a unit key.        */
+/*   write_norms [L][Hv] float  (required here) receives per (layer, value head) the sum over  */
+/*                              the n_tokens tokens of beta_t ||v_t - alpha_t S_{t-1} k_t||_2    */
+/* (0 for n_tokens = 0).  Every other argument, result and error as deltas_gdn_chunk_update;    */
+/* INVALID_ARGUMENT also for a NULL or misaligned write_norms.  On the tensor-core path a tile  */
+/* whose decay over its 64 tokens exp(G_C) is below 2^-60 (G_C < -41.6) adds nothing.          */
+/* ------------------------------------------------------------------------------------------ */
+DELTAS_API deltas_status deltas_gdn_chunk_update_write_norms(const deltas_gdn_desc* desc, int32_t n_tokens,
+                                      const void* q, const void* k, const void* v,
+                                      const float* g, const float* beta,
+                                      float* state, void* out, float* drift_partials,
+                                      float* write_norms, void* workspace,
+                                      size_t workspace_bytes, void* stream);
+
+/* The comparison signal's chunk score: write sizes averaged over heads, layers and the chunk's */
+/* n_tokens tokens, chunk_scores[chunk_id] = sum(write_norms) / (L * Hv * n_tokens), 0 when     */
+/* n_tokens = 0 (float32; the sum is taken in double on the device).                           */
+/* Errors: INVALID_ARGUMENT for NULL pointers or negative sizes / chunk_id.                     */
+DELTAS_API deltas_status deltas_score_write_norms(int32_t num_layers, int32_t num_v_heads,
+                                      const float* write_norms, int32_t n_tokens,
+                                      int32_t chunk_id, float* chunk_scores, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
 /* State drift partials from two stored states (Sec. 3.2, Eq. 3 numerator and denominator per  */
 /* layer and head; the paper keeps a copy of the previous state for this, Sec. 3.2).           */
 /*   s_before, s_after [L][Hv][d_v][d_k] float;  drift_partials [L][Hv][2] float (as above).   */

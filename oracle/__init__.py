@@ -53,7 +53,7 @@ def _load():
     with _lock:
         if _lib is None:
             lib = ctypes.CDLL(build())
-            lib.oracle_gdn_recurrence.argtypes = [_I] * 6 + [_P] * 7 + [ctypes.c_double]
+            lib.oracle_gdn_recurrence.argtypes = [_I] * 6 + [_P] * 7 + [ctypes.c_double, _P]
             lib.oracle_gdn_recurrence.restype = _I
             lib.oracle_gdn_recurrence_product_form.argtypes = [_I] * 6 + [_P] * 5
             lib.oracle_gdn_recurrence_product_form.restype = _I
@@ -61,6 +61,8 @@ def _load():
             lib.oracle_drift_partials.restype = _I
             lib.oracle_chunk_score.argtypes = [_I, _I, _P]
             lib.oracle_chunk_score.restype = ctypes.c_double
+            lib.oracle_write_norm_score.argtypes = [_I, _I, _I, _P]
+            lib.oracle_write_norm_score.restype = ctypes.c_double
             lib.oracle_select_retain.argtypes = [_I] * 6 + [_P] * 5
             lib.oracle_select_retain.restype = _I
             lib.oracle_compact_rows.argtypes = [_I] * 4 + [_P] * 3 + [_I]
@@ -82,9 +84,12 @@ def _check(rc: int, what: str):
         raise ValueError(f"oracle {what} rejected its arguments (code {rc})")
 
 
-def gdn_recurrence(q, k, v, g, beta, state, q_scale: float | None = None, want_out: bool = False):
+def gdn_recurrence(q, k, v, g, beta, state, q_scale: float | None = None, want_out: bool = False,
+                   want_write_norms: bool = False):
     """Eq. 2 token loop.  Shapes: q,k [L,T,Hk,dk]; v [L,T,Hv,dv]; g,beta [L,T,Hv];
-    state [L,Hv,dv,dk] (copied, not modified).  Returns ``(S_after, out_or_None)`` in fp64."""
+    state [L,Hv,dv,dk] (copied, not modified).  Returns ``(S_after, out_or_None)`` in fp64, and
+    with ``want_write_norms`` a third item: [L,Hv] sums over the tokens of
+    beta_t ||v_t - alpha_t S_{t-1} k_t||_2."""
     k = _f32(k)
     v = _f32(v)
     g = _f32(g)
@@ -98,10 +103,18 @@ def gdn_recurrence(q, k, v, g, beta, state, q_scale: float | None = None, want_o
     out = np.zeros((L, T, Hv, dv), dtype=np.float64) if want_out else None
     if q_scale is None:
         q_scale = 1.0 / np.sqrt(dk)
+    wn = np.zeros((L, Hv), dtype=np.float64) if want_write_norms else None
     rc = _load().oracle_gdn_recurrence(L, Hk, Hv, dk, dv, T, _ptr(qa), _ptr(k), _ptr(v), _ptr(g),
-                                       _ptr(beta), _ptr(S), _ptr(out), float(q_scale))
+                                       _ptr(beta), _ptr(S), _ptr(out), float(q_scale), _ptr(wn))
     _check(rc, "gdn_recurrence")
-    return S, out
+    return (S, out, wn) if want_write_norms else (S, out)
+
+
+def write_norm_score(write_norms, n_tokens: int) -> float:
+    """The comparison signal's chunk score: write sizes averaged over heads, layers and tokens."""
+    wn = np.ascontiguousarray(write_norms, dtype=np.float64)
+    L, Hv = wn.shape
+    return float(_load().oracle_write_norm_score(L, Hv, int(n_tokens), _ptr(wn)))
 
 
 def gdn_recurrence_product_form(k, v, g, beta, state):

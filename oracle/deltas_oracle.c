@@ -33,16 +33,20 @@
 /*     S_t = alpha_t S_{t-1} + beta_t (v_t - alpha_t S_{t-1} k_t) k_t^T                         */
 /* processed token by token in stream order.  If out != NULL, o_t = q_scale * S_t q_t is        */
 /* written after the update of token t (the read-out of the prefill, Alg. 1 "Prefill").        */
+/* If wnorm != NULL ([L][Hv]), it receives per (layer, head) the sum over the chunk's tokens of */
+/* the write size beta_t ||v_t - alpha_t S_{t-1} k_t||_2 (the comparison signal of Sec. 4.3 and */
+/* the appendix's description of it: the residual times the write strength, per head).         */
 /* ------------------------------------------------------------------------------------------ */
 int oracle_gdn_recurrence(int L, int Hk, int Hv, int dk, int dv, int T,
                           const float* q, const float* k, const float* v,
                           const float* g, const float* beta,
-                          double* S, double* out, double q_scale)
+                          double* S, double* out, double q_scale, double* wnorm)
 {
     if (L < 1 || Hk < 1 || Hv < 1 || dk < 1 || dv < 1 || T < 0 || Hv % Hk != 0) return ORACLE_BAD_ARG;
     if (!k || !v || !g || !beta || !S || (out && !q)) return ORACLE_BAD_ARG;
     double* r = (double*)malloc(sizeof(double) * (size_t)dv);
     if (!r) return ORACLE_NO_MEMORY;
+    if (wnorm) memset(wnorm, 0, sizeof(double) * (size_t)L * Hv);
     for (int l = 0; l < L; ++l) {
         for (int h = 0; h < Hv; ++h) {
             const int kh = (int)(((long long)h * Hk) / Hv);
@@ -62,11 +66,14 @@ int oracle_gdn_recurrence(int L, int Hk, int Hv, int dk, int dv, int T,
                     r[i] = acc;
                 }
                 /* S_t = alpha S_{t-1} + u k^T  with  u = beta (v - alpha r) */
+                double uu = 0.0;
                 for (int i = 0; i < dv; ++i) {
                     const double u = b * ((double)vt[i] - alpha * r[i]);
+                    uu += u * u;
                     for (int j = 0; j < dk; ++j)
                         Sh[(size_t)i * dk + j] = alpha * Sh[(size_t)i * dk + j] + u * (double)kt[j];
                 }
+                if (wnorm) wnorm[(size_t)l * Hv + h] += sqrt(uu);
                 if (out) {
                     const float* qt = q + kofs;
                     double* ot = out + vofs;
@@ -179,6 +186,19 @@ double oracle_chunk_score(int L, int Hv, const double* partials)
         total += term;
     }
     return total / (double)L;
+}
+
+/* ------------------------------------------------------------------------------------------ */
+/* The comparison signal's chunk score (Sec. 4.3; appendix): the write size averaged over the  */
+/* heads, the gated-delta layers and the chunk's T tokens, i.e. the sum of all per-(layer,      */
+/* head, token) write sizes over L * Hv * T.  T = 0 gives 0.                                    */
+/* ------------------------------------------------------------------------------------------ */
+double oracle_write_norm_score(int L, int Hv, int T, const double* wnorm)
+{
+    if (T <= 0) return 0.0;
+    double total = 0.0;
+    for (size_t i = 0; i < (size_t)L * Hv; ++i) total += wnorm[i];
+    return total / ((double)L * Hv * T);
 }
 
 /* ------------------------------------------------------------------------------------------ */

@@ -6,7 +6,9 @@ Test infrastructure only.  One iteration per arriving chunk c:
 2. ``Prefill(c)``: the gated delta rule (Eq. 2) updates S over the chunk's tokens, and the
    chunk's keys/values are appended to every full-attention cache;
 3. ``Delta S`` of Eq. 3 from S_before and S, stored (in float32, as the paper computes all scores
-   in float32) as the score of every token of c;
+   in float32) as the score of every token of c (or, with ``signal="write_norm"``, the comparison
+   signal of Sec. 4.3: the tokens' write sizes beta_t ||v_t - alpha_t S_{t-1} k_t|| averaged over
+   heads, layers and the chunk's tokens);
 4. if the cache holds more than M tokens: sink / window / spans / quota + fill (Sec. 3.3), then
    the in-stream-order gather of every cache, keeping original positions.
 
@@ -23,7 +25,7 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
-from . import compact_kv, gdn_recurrence, select_retain, state_drift
+from . import compact_kv, gdn_recurrence, select_retain, state_drift, write_norm_score
 
 
 @dataclass
@@ -42,7 +44,7 @@ class StreamResult:
 
 def run_stream(chunk_inputs, kv_inputs, state0, n_chunks: int, policy: dict, capacity: int,
                q_scale: float | None = None, score_override=None, keep_states: bool = False,
-               questions: dict | None = None):
+               questions: dict | None = None, signal: str = "drift"):
     """Run Alg. 1 over ``n_chunks`` chunks.
 
     ``chunk_inputs(c)`` -> (q, k, v, g, beta) numpy arrays in the oracle layouts;
@@ -66,7 +68,10 @@ def run_stream(chunk_inputs, kv_inputs, state0, n_chunks: int, policy: dict, cap
         nonlocal S, kc, vc, tok_chunk, tok_pos, T, pos
         q, k, v, g, beta = gdn_in
         s_before = S.copy()
-        S, _ = gdn_recurrence(None, k, v, g, beta, S, q_scale=q_scale)
+        if signal == "write_norm":
+            S, _, wn = gdn_recurrence(None, k, v, g, beta, S, q_scale=q_scale, want_write_norms=True)
+        else:
+            S, _ = gdn_recurrence(None, k, v, g, beta, S, q_scale=q_scale)
         k_new, v_new = kv_in
         Lf, Hkv, C, D = k_new.shape
         if kc is None:
@@ -80,7 +85,10 @@ def run_stream(chunk_inputs, kv_inputs, state0, n_chunks: int, policy: dict, cap
         tok_pos[T:T + C] = np.arange(pos, pos + C, dtype=np.int32)
         T += C
         pos += C
-        scores[c] = np.float32(state_drift(s_before, S))
+        if signal == "write_norm":
+            scores[c] = np.float32(write_norm_score(wn, k.shape[1]))
+        else:
+            scores[c] = np.float32(state_drift(s_before, S))
         if T > policy["budget_M"]:
             idx, _ = select_retain(policy["budget_M"], policy["n_sink"], policy["n_window"],
                                    policy["n_buckets"], tok_chunk[:T], rank_scores_of()[: c + 1])

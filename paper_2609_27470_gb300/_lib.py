@@ -34,7 +34,7 @@ EXPORTED = (
     "deltas_version", "deltas_status_string",
     "deltas_gdn_chunk_update_workspace_size", "deltas_gdn_chunk_update",
     "deltas_state_drift_workspace_size", "deltas_state_drift",
-    "deltas_score_chunks",
+    "deltas_score_chunks", "deltas_gdn_chunk_update_write_norms", "deltas_score_write_norms",
     "deltas_select_retain_workspace_size", "deltas_select_retain", "deltas_select_retain_static",
     "deltas_compact_kv_workspace_size", "deltas_compact_kv",
     "deltas_append_kv", "deltas_copy_stream_state",
@@ -83,6 +83,8 @@ _sig("deltas_gdn_chunk_update", ctypes.c_int, _P, _I32, _P, _P, _P, _P, _P, _P, 
 _sig("deltas_state_drift_workspace_size", _SZ, _P)
 _sig("deltas_state_drift", ctypes.c_int, _P, _P, _P, _P, _P, _SZ, _P)
 _sig("deltas_score_chunks", ctypes.c_int, _I32, _I32, _P, _I32, _P, _P)
+_sig("deltas_gdn_chunk_update_write_norms", ctypes.c_int, _P, _I32, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P)
+_sig("deltas_score_write_norms", ctypes.c_int, _I32, _I32, _P, _I32, _I32, _P, _P)
 _sig("deltas_select_retain_workspace_size", _SZ, _I32)
 _sig("deltas_select_retain", ctypes.c_int, _P, _I32, _I32, _P, _P, _P, _P, _P, _P, _SZ, _P)
 _sig("deltas_select_retain_static", ctypes.c_int, _P, _I32, _I32, _P, _P, _P, _P, _P, _P)
@@ -163,20 +165,38 @@ def deltas_gdn_chunk_update_workspace_size(desc: GdnDesc, n_tokens: int) -> int:
 
 
 def deltas_gdn_chunk_update(desc: GdnDesc, n_tokens: int, q, k, v, g, beta, state, out, drift_partials,
-                            workspace, stream=None):
+                            workspace, stream=None, write_norms=None):
+    """The chunk update; with ``write_norms`` ([L, Hv] float32) the call is
+    deltas_gdn_chunk_update_write_norms and also sums the tokens' write sizes."""
     L, Hk, Hv, dk, dv = desc.num_layers, desc.num_k_heads, desc.num_v_heads, desc.key_dim, desc.value_dim
     adt = _TORCH_DT[desc.dtype]
     T = int(n_tokens)
-    st = _lib.deltas_gdn_chunk_update(
-        ctypes.byref(desc), T,
-        _ptr(q, adt, (L, T, Hk, dk), "q"), _ptr(k, adt, (L, T, Hk, dk), "k"),
-        _ptr(v, adt, (L, T, Hv, dv), "v"), _ptr(g, torch.float32, (L, T, Hv), "g"),
-        _ptr(beta, torch.float32, (L, T, Hv), "beta"),
-        _ptr(state, torch.float32, (L, Hv, dv, dk), "state"),
-        _ptr(out, adt, (L, T, Hv, dv), "out"),
-        _ptr(drift_partials, torch.float32, (L, Hv, 2), "drift_partials"),
-        _ptr(workspace, torch.uint8, None, "workspace"), workspace.numel(), _stream(stream))
-    _check(st, "deltas_gdn_chunk_update")
+    args = [_ptr(q, adt, (L, T, Hk, dk), "q"), _ptr(k, adt, (L, T, Hk, dk), "k"),
+            _ptr(v, adt, (L, T, Hv, dv), "v"), _ptr(g, torch.float32, (L, T, Hv), "g"),
+            _ptr(beta, torch.float32, (L, T, Hv), "beta"),
+            _ptr(state, torch.float32, (L, Hv, dv, dk), "state"),
+            _ptr(out, adt, (L, T, Hv, dv), "out"),
+            _ptr(drift_partials, torch.float32, (L, Hv, 2), "drift_partials")]
+    tail = [_ptr(workspace, torch.uint8, None, "workspace"), workspace.numel(), _stream(stream)]
+    if write_norms is None:
+        st = _lib.deltas_gdn_chunk_update(ctypes.byref(desc), T, *args, *tail)
+        _check(st, "deltas_gdn_chunk_update")
+    else:
+        st = _lib.deltas_gdn_chunk_update_write_norms(ctypes.byref(desc), T, *args,
+                                                      _ptr(write_norms, torch.float32, (L, Hv), "write_norms"),
+                                                      *tail)
+        _check(st, "deltas_gdn_chunk_update_write_norms")
+
+
+def deltas_score_write_norms(num_layers: int, num_v_heads: int, write_norms, n_tokens: int, chunk_id: int,
+                             chunk_scores, stream=None):
+    if chunk_scores.numel() <= chunk_id:
+        raise ValueError("chunk_scores too short for chunk_id")
+    st = _lib.deltas_score_write_norms(int(num_layers), int(num_v_heads),
+                                       _ptr(write_norms, torch.float32, (num_layers, num_v_heads), "write_norms"),
+                                       int(n_tokens), int(chunk_id),
+                                       _ptr(chunk_scores, torch.float32, None, "chunk_scores"), _stream(stream))
+    _check(st, "deltas_score_write_norms")
 
 
 def deltas_state_drift_workspace_size(desc: GdnDesc) -> int:

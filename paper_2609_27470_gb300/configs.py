@@ -40,4 +40,7 @@ PAPER = dict(name="paper", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=ma
              chunk_lens=PAPER_CHUNK_LENS, n_chunks=4096, ring=8, Lf=8, Hkv=4, D=256, kv_dtype="bf16",
              budget_M=8192, **PAPER_POLICY)
 
-ALL = {c["name"]: c for c in (TINY, LAYER, STACK, KV, STREAMING, PAPER)}
+# the paper stream scored by the comparison signal of Sec. 4.3 (write sizes) instead of drift
+PAPER_WRITE_NORM = dict(PAPER, name="paper_write_norm", signal="write_norm")
+
+ALL = {c["name"]: c for c in (TINY, LAYER, STACK, KV, STREAMING, PAPER, PAPER_WRITE_NORM)}

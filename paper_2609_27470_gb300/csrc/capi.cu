@@ -93,11 +93,12 @@ size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32
                                                desc->value_dim, desc->dtype, n_tokens);
 }
 
-deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, int32_t n_tokens,
-                                      const void* q, const void* k, const void* v,
-                                      const float* g, const float* beta,
-                                      float* state, void* out, float* drift_partials,
-                                      void* workspace, size_t workspace_bytes, void* stream)
+namespace {
+
+deltas_status gdn_update(const deltas_gdn_desc* desc, int32_t n_tokens, const void* q, const void* k,
+                         const void* v, const float* g, const float* beta, float* state, void* out,
+                         float* drift_partials, float* write_norms, void* workspace, size_t workspace_bytes,
+                         void* stream)
 {
     deltas_status st = check_gdn_desc(desc);
     if (st != DELTAS_OK) return st;
@@ -108,18 +109,43 @@ deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, int32_t n_tok
         if (out && (!q || !aligned16(q) || !aligned16(out))) return DELTAS_ERR_INVALID_ARGUMENT;
     }
     if (drift_partials && !aligned16(drift_partials)) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (write_norms && !aligned16(write_norms)) return DELTAS_ERR_INVALID_ARGUMENT;
     st = check_workspace(workspace, workspace_bytes, deltas_gdn_chunk_update_workspace_size(desc, n_tokens));
     if (st != DELTAS_OK) return st;
     GdnArgs a;
     a.L = desc->num_layers; a.Hk = desc->num_k_heads; a.Hv = desc->num_v_heads;
     a.dk = desc->key_dim; a.dv = desc->value_dim; a.T = n_tokens; a.dtype = desc->dtype;
     a.q_scale = desc->q_scale; a.q = q; a.k = k; a.v = v; a.g = g; a.beta = beta;
-    a.state = state; a.out = out; a.partials = drift_partials;
+    a.state = state; a.out = out; a.partials = drift_partials; a.wnorm = write_norms;
     a.status = static_cast<int32_t*>(workspace);
     a.scratch = static_cast<uint8_t*>(workspace) + kStatusBytes;
     a.scratch_bytes = workspace_bytes - kStatusBytes;
     if (gdn_tc_supported(a)) return from_cuda(launch_gdn_update_tc(a, as_stream(stream)));
     return from_cuda(launch_gdn_update_simt(a, as_stream(stream)));
+}
+
+}  // namespace
+
+deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, int32_t n_tokens,
+                                      const void* q, const void* k, const void* v,
+                                      const float* g, const float* beta,
+                                      float* state, void* out, float* drift_partials,
+                                      void* workspace, size_t workspace_bytes, void* stream)
+{
+    return gdn_update(desc, n_tokens, q, k, v, g, beta, state, out, drift_partials, nullptr, workspace,
+                      workspace_bytes, stream);
+}
+
+deltas_status deltas_gdn_chunk_update_write_norms(const deltas_gdn_desc* desc, int32_t n_tokens,
+                                                  const void* q, const void* k, const void* v,
+                                                  const float* g, const float* beta,
+                                                  float* state, void* out, float* drift_partials,
+                                                  float* write_norms, void* workspace,
+                                                  size_t workspace_bytes, void* stream)
+{
+    if (write_norms == nullptr) return DELTAS_ERR_INVALID_ARGUMENT;
+    return gdn_update(desc, n_tokens, q, k, v, g, beta, state, out, drift_partials, write_norms, workspace,
+                      workspace_bytes, stream);
 }
 
 size_t deltas_state_drift_workspace_size(const deltas_gdn_desc* desc) {
@@ -143,6 +169,16 @@ deltas_status deltas_state_drift(const deltas_gdn_desc* desc, const float* s_bef
     return from_cuda(launch_state_drift(desc->num_layers, desc->num_v_heads, desc->value_dim,
                                         desc->key_dim, s_before, s_after, drift_partials,
                                         as_stream(stream)));
+}
+
+deltas_status deltas_score_write_norms(int32_t num_layers, int32_t num_v_heads, const float* write_norms,
+                                       int32_t n_tokens, int32_t chunk_id, float* chunk_scores, void* stream)
+{
+    if (num_layers < 1 || num_v_heads < 1 || n_tokens < 0 || chunk_id < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if ((long long)num_layers * num_v_heads > (1ll << 30)) return DELTAS_ERR_UNSUPPORTED;
+    if (!write_norms || !chunk_scores) return DELTAS_ERR_INVALID_ARGUMENT;
+    return from_cuda(launch_score_write_norms(num_layers, num_v_heads, write_norms, n_tokens, chunk_id,
+                                              chunk_scores, as_stream(stream)));
 }
 
 deltas_status deltas_score_chunks(int32_t num_layers, int32_t num_v_heads,

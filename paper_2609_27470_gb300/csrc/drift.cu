@@ -87,7 +87,29 @@ score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk
     }
 }
 
+// The comparison signal's chunk score (Sec. 4.3): write sizes averaged over the heads, the layers
+// and the chunk's tokens, i.e. their total over L * Hv * n_tokens; the total is summed in double
+// in a fixed order (one warp, lane-strided, then a fixed xor tree).
+__global__ void __launch_bounds__(32)
+score_write_norms_kernel(int n, const float* __restrict__ wnorm, double inv_count, int chunk_id,
+                         float* __restrict__ scores)
+{
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < n; i += 32) acc += (double)wnorm[i];
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, m);
+    if (threadIdx.x == 0) scores[chunk_id] = (float)(acc * inv_count);
+}
+
 }  // namespace
+
+cudaError_t launch_score_write_norms(int L, int Hv, const float* wnorm, int n_tokens, int chunk_id, float* scores,
+                                     cudaStream_t s)
+{
+    const double inv = n_tokens > 0 ? 1.0 / ((double)L * Hv * n_tokens) : 0.0;
+    score_write_norms_kernel<<<1, 32, 0, s>>>(L * Hv, wnorm, inv, chunk_id, scores);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, const float* sa,
                                float* partials, cudaStream_t s)

@@ -10,7 +10,9 @@
 // so that the TPR threads of a row read the staged key with distinct shared-memory banks).  Per
 // token: r = S k (TPR-lane shuffle reduction), u = beta (v - alpha r), S = alpha S + u k^T.  The
 // state before the chunk stays in registers too, so the drift partials need no second read of
-// the state from memory.
+// the state from memory.  Optionally the same pass sums the write sizes ||u_t|| (u = beta (v -
+// alpha r), the comparison signal of Sec. 4.3) over the chunk: each warp adds its rows' u^2 for
+// the token into shared memory, and after each staged pass one thread takes the square roots.
 #include "internal.cuh"
 
 namespace deltas {
@@ -35,6 +37,7 @@ gdn_update_simt_kernel(GdnArgs a)
     __shared__ __align__(16) float sv[TB][D];
     __shared__ __align__(16) float so[TB][D];
     __shared__ float salpha[TB], sbeta[TB];
+    __shared__ float su2[TB];                        // per-token sum of u^2 over the rows
     __shared__ double red[2][NT / 32 + 1];
 
     const int lh = blockIdx.x;
@@ -43,6 +46,10 @@ gdn_update_simt_kernel(GdnArgs a)
     const int tid = threadIdx.x;
     const int row = tid / TPR, sub = tid % TPR;
     const bool want_out = a.out != nullptr;
+    const bool want_w = a.wnorm != nullptr;
+    constexpr unsigned kLanes = NT >= 32 ? 0xffffffffu : ((1u << NT) - 1u);
+    float wsum = 0.f;                                // thread 0: sum over tokens of ||u_t||
+    for (int e = tid; e < TB; e += NT) su2[e] = 0.f;
 
     float* Srow = a.state + ((size_t)lh * D + row) * D;
     float4 S[NG], S0[NG];
@@ -88,6 +95,12 @@ gdn_update_simt_kernel(GdnArgs a)
             for (int m = 1; m < TPR; m <<= 1) r += __shfl_xor_sync(0xffffffffu, r, m);
             const float alpha = salpha[tt];
             const float u = sbeta[tt] * (sv[tt][row] - alpha * r);
+            if (want_w) {
+                float u2 = sub == 0 ? u * u : 0.f;          // the TPR threads of a row share u
+#pragma unroll
+                for (int m = (NT >= 32 ? 16 : NT / 2); m >= 1; m >>= 1) u2 += __shfl_xor_sync(kLanes, u2, m);
+                if ((tid & 31) == 0) atomicAdd(&su2[tt], u2);
+            }
 #pragma unroll
             for (int j = 0; j < NG; ++j) {
                 const float4 kk = kv4[j * TPR + sub];
@@ -120,7 +133,17 @@ gdn_update_simt_kernel(GdnArgs a)
                 oout[(tok * a.Hv + h) * D + c] = from_f32<Tin>(so[tt][c]);
             }
         }
+        if (want_w) {
+            __syncthreads();
+            if (tid == 0) {
+                for (int tt = 0; tt < nt; ++tt) {
+                    wsum += sqrtf(su2[tt]);
+                    su2[tt] = 0.f;
+                }
+            }
+        }
     }
+    if (want_w && tid == 0) a.wnorm[lh] = wsum;
 
     float num = 0.f, den = 0.f;
 #pragma unroll
@@ -133,7 +156,6 @@ gdn_update_simt_kernel(GdnArgs a)
     if (a.partials == nullptr) return;
     double dn = num, dd = den;
     // fixed-order xor tree over the lanes that exist (NT < 32 only for d = 16)
-    constexpr unsigned kLanes = NT >= 32 ? 0xffffffffu : ((1u << NT) - 1u);
 #pragma unroll
     for (int m = (NT >= 32 ? 16 : NT / 2); m >= 1; m >>= 1) {
         dn += __shfl_xor_sync(kLanes, dn, m);

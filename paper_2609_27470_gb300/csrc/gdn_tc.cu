@@ -653,6 +653,7 @@ struct TcArgs {
     int L, Hk, Hv, T, n_tiles;
     float* state;
     float* partials;
+    float* wnorm;
     const uint8_t* rec;
     int32_t* status;
 };
@@ -685,6 +686,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ float s_red[2][kChainWarps];
+    __shared__ float s_u2[2][kC];                 // per-token squared write sizes (tile parity)
     volatile int* abort_flag = &s_abort;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -723,6 +725,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         fence_async_smem();
     }
     if (tid == 0) s_abort = 0;
+    if (tid < 2 * kC) s_u2[tid >> 6][tid & (kC - 1)] = 0.f;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -967,12 +970,41 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         // accumulates onto S~ with no pass over the state); when sig gamma_C would drop below
         // kSigMin the tile instead writes gamma_C S back into TMEM and sig restarts at 1.
         float sig = 1.f;
+        // Write sizes (optional): column t of the U region is u_t scaled by u_scale gamma_C /
+        // gamma_t, u_t = beta_t (v_t - alpha_t S_{t-1} k_t) the token's write.  The Ũ pass sums
+        // each column's squares over this warp's 32 rows and adds them, rescaled to u_t, into
+        // s_u2 (four warps per column); after the next barrier warp 0 takes the square roots and
+        // sums them over the tile's tokens into the head's total.
+        const bool want_w = a.wnorm != nullptr;
+        float wacc = 0.f;                                  // warp 0: the head's running sum
+        int prev_lh = -1;
+        bool prev_last = false;
+        auto fold_writes = [&](int jj) {                   // warp 0: tile jj's sizes into wacc
+            float* b = s_u2[jj & 1];
+            float sacc = sqrtf(b[lane]) + sqrtf(b[lane + 32]);
+            b[lane] = 0.f;
+            b[lane + 32] = 0.f;
+#pragma unroll
+            for (int m = 16; m >= 1; m >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, m);
+            wacc += sacc;
+        };
         for (int j = 0; j < NJ; ++j) {                     // j: global tile index
             const int lh = cc.lh, jt = cc.jt;              // head and tile within the head
             const bool last = jt == n - 1;
             if (named_sync_or(2, kChain, *abort_flag)) break;
             if (!mbar_wait_or_abort(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
             const float gC = rec_consts(j)[64];
+            float w_gamma = 0.f;                           // gamma_t of this lane's column in the Ũ pass
+            if (want_w) {
+                w_gamma = -rec_consts(j)[16 * cgp + (lane >> 1)];
+                if (j > 0 && warp == 0) {
+                    fold_writes(j - 1);
+                    if (prev_last) {
+                        if (lane == 0) a.wnorm[prev_lh] = wacc;
+                        wacc = 0.f;
+                    }
+                }
+            }
 
             if (j == 0) {
                 // ---- the CTA's first head: its state from the staging buffer into TMEM, as S~
@@ -1043,6 +1075,30 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 float uv[16];
                 tmem_ld16(tm + lane_off + TM_U + 16 * cgp, uv);
                 tmem_ld_wait();
+                if (want_w) {
+                    // squares summed over the warp's 32 rows, column by column: halving exchanges
+                    // leave lanes 2c and 2c + 1 with column c (token 16 cgp + c) of the 16
+                    float x[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) x[i] = uv[i] * uv[i];
+#pragma unroll
+                    for (int w = 8, bit = 16; w >= 1; w >>= 1, bit >>= 1) {
+                        const bool up = (lane & bit) != 0;
+#pragma unroll
+                        for (int i = 0; i < w; ++i) {
+                            const float send = up ? x[i] : x[i + w];
+                            x[i] = (up ? x[i + w] : x[i]) + __shfl_xor_sync(0xffffffffu, send, bit);
+                        }
+                    }
+                    x[0] += __shfl_xor_sync(0xffffffffu, x[0], 1);
+                    // U column -> u_t.  u_scale gamma_C is 1 / sig >= 1 unless the tile restarts
+                    // the deferred decay; then it is gamma_C, and below 2^-60 the columns of the
+                    // early tokens, scaled by gamma_C / gamma_t, are no longer representable: such
+                    // a tile contributes nothing
+                    const float sc = u_scale * gC;
+                    const float wf = sc >= 0x1p-60f ? w_gamma / sc : 0.f;
+                    if ((lane & 1) == 0) atomicAdd(&s_u2[j & 1][16 * cgp + (lane >> 1)], x[0] * wf * wf);
+                }
                 uint32_t hi[8], lo[8];
 #pragma unroll
                 for (int i = 0; i < 8; ++i) split2(uv[2 * i], uv[2 * i + 1], hi[i], lo[i]);
@@ -1133,7 +1189,14 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 den = den_next;
                 sig = 1.f;
             }
+            prev_lh = lh;
+            prev_last = last;
             cc.next(n, a);
+        }
+        // the CTA's last tile (always a head's last) once every warp's Ũ pass has added to it
+        if (want_w && NJ > 0 && !named_sync_or(2, kChain, *abort_flag) && warp == 0) {
+            fold_writes(NJ - 1);
+            if (lane == 0) a.wnorm[prev_lh] = wacc;
         }
     }
 
@@ -1238,7 +1301,7 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     // ~211 KB of shared memory); each takes every grid-th head
     TcArgs t;
     t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = n_tiles;
-    t.state = a.state; t.partials = a.partials; t.rec = a.scratch; t.status = a.status;
+    t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.rec = a.scratch; t.status = a.status;
     const int grid = std::min(a.L * a.Hv, sms);
     gdn_update_tc_kernel<<<grid, kThreads, kSmemAlloc, s>>>(kmap, vmap, smap, t);
     return cudaGetLastError();

@@ -53,6 +53,7 @@ struct GdnArgs {
     float* state;
     void* out;
     float* partials;
+    float* wnorm;            // [L][Hv] sums over the chunk of beta_t ||v_t - alpha_t S_{t-1} k_t||, or null
     int32_t* status;
     uint8_t* scratch;        // workspace past the status word (the tensor-core path's WY factors)
     size_t scratch_bytes;
@@ -88,6 +89,8 @@ size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T);
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s);
 cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, const float* sa,
                                float* partials, cudaStream_t s);
+cudaError_t launch_score_write_norms(int L, int Hv, const float* wnorm, int n_tokens, int chunk_id, float* scores,
+                                     cudaStream_t s);
 cudaError_t launch_score_chunks(int L, int Hv, const float* partials, int chunk_id, float* scores,
                                 cudaStream_t s);
 size_t select_workspace_bytes(int cache_len);

@@ -5,7 +5,10 @@ Per arriving chunk c, all on one CUDA stream and with no host synchronisation:
 1. ``deltas_gdn_chunk_update`` — Prefill(c) of every gated-delta layer: the state S goes from
    S_before to S_after (Eq. 1) and the per-(layer, head) drift partials come out of the same
    kernel (the pre-chunk state is never stored separately);
-2. ``deltas_score_chunks`` — Delta S of Eq. 3, stored as score[c] (shared by c's tokens);
+2. ``deltas_score_chunks`` — Delta S of Eq. 3, stored as score[c] (shared by c's tokens); with
+   ``signal="write_norm"`` the chunk is scored instead by the comparison signal of Sec. 4.3, the
+   tokens' write sizes beta_t ||v_t - alpha_t S_{t-1} k_t|| averaged over heads, layers and
+   tokens (``deltas_gdn_chunk_update_write_norms`` + ``deltas_score_write_norms``);
 3. ``deltas_append_kv`` — c's keys/values enter every full-attention cache, with their arrival
    chunk and stream position;
 4. if the cache holds more than M tokens: ``deltas_select_retain`` then ``deltas_compact_kv``.
@@ -44,7 +47,10 @@ class DeltaSStream:
     def __init__(self, *, num_layers, num_k_heads, num_v_heads, head_dim, act_dtype: torch.dtype,
                  kv_layers, kv_heads, kv_head_dim, kv_dtype: torch.dtype, budget_M, n_sink=0,
                  n_window=0, n_buckets=1, chunk_len, max_chunks, q_scale=None, state0=None,
-                 device="cuda"):
+                 device="cuda", signal: str = "drift"):
+        if signal not in ("drift", "write_norm"):
+            raise ValueError(f"unknown signal {signal!r}")
+        self.signal = signal
         self.gdn = L.gdn_desc(num_layers, num_k_heads, num_v_heads, head_dim, act_dtype, q_scale)
         self.policy = L.policy(budget_M, n_sink, n_window, n_buckets)
         self.capacity = budget_M + chunk_len
@@ -55,6 +61,7 @@ class DeltaSStream:
         self.state = (state0.clone() if state0 is not None else
                       torch.zeros(num_layers, num_v_heads, head_dim, head_dim, device=dev))
         self.partials = torch.zeros(num_layers, num_v_heads, 2, device=dev)
+        self.write_norms = torch.zeros(num_layers, num_v_heads, device=dev) if signal == "write_norm" else None
         self.chunk_scores = torch.zeros(max_chunks, device=dev)
         self.k_cache = torch.zeros(kv_layers, kv_heads, self.capacity, kv_head_dim, dtype=kv_dtype, device=dev)
         self.v_cache = torch.zeros_like(self.k_cache)
@@ -78,9 +85,13 @@ class DeltaSStream:
             raise ValueError("stream longer than max_chunks")
         T = int(k.shape[1])
         L.deltas_gdn_chunk_update(self.gdn, T, q, k, v, g, beta, self.state, out, self.partials,
-                                  self.workspace, stream)
-        L.deltas_score_chunks(self.gdn.num_layers, self.gdn.num_v_heads, self.partials, c,
-                              self.chunk_scores, stream)
+                                  self.workspace, stream, write_norms=self.write_norms)
+        if self.signal == "write_norm":
+            L.deltas_score_write_norms(self.gdn.num_layers, self.gdn.num_v_heads, self.write_norms, T, c,
+                                       self.chunk_scores, stream)
+        else:
+            L.deltas_score_chunks(self.gdn.num_layers, self.gdn.num_v_heads, self.partials, c,
+                                  self.chunk_scores, stream)
         n_new = int(k_new.shape[2])
         L.deltas_append_kv(self.kv, self.k_cache, self.v_cache, self.tok_chunk, self.tok_pos,
                            self.cache_len, k_new, v_new, c, self.position, stream)

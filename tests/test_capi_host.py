@@ -25,7 +25,7 @@ def _declared():
 
 def test_every_declared_symbol_is_exported(L):
     names = _declared()
-    assert len(names) == 16, names
+    assert len(names) == 18, names
     lib = ctypes.CDLL(L.LIB_PATH)
     for n in names:
         assert hasattr(lib, n), n
@@ -152,3 +152,18 @@ def test_copy_stream_state_argument_checks(L):
     assert call(full(A), ov) == bad
     assert call(full(A), full(B), kvd=L.KvDesc(2, 2, 7, L.DELTAS_F32, 1000)) == L.DELTAS_ERR_UNSUPPORTED
     assert call(full(A), full(B), desc=L.GdnDesc(2, 2, 4, 24, 24, L.DELTAS_F32, 0.25)) == L.DELTAS_ERR_UNSUPPORTED
+
+
+def test_write_norm_argument_checks(L):
+    """The comparison-signal entry points refuse bad arguments on the host."""
+    raw = L.raw()
+    ok = L.GdnDesc(1, 2, 4, 16, 16, L.DELTAS_F32, 0.25)
+    bad = L.DELTAS_ERR_INVALID_ARGUMENT
+    call = lambda wn: raw.deltas_gdn_chunk_update_write_norms(ctypes.byref(ok), 8, None, FAKE, FAKE, FAKE, FAKE,
+                                                              FAKE, None, None, wn, FAKE, 1 << 20, None)
+    assert call(None) == bad                                            # the output is required here
+    assert call(FAKE + 4) == bad                                        # misaligned
+    assert raw.deltas_score_write_norms(0, 4, FAKE, 10, 0, FAKE, None) == bad
+    assert raw.deltas_score_write_norms(2, 4, FAKE, -1, 0, FAKE, None) == bad
+    assert raw.deltas_score_write_norms(2, 4, FAKE, 10, -1, FAKE, None) == bad
+    assert raw.deltas_score_write_norms(2, 4, None, 10, 0, FAKE, None) == bad

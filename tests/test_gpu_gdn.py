@@ -228,3 +228,70 @@ def test_score_kernel(L):
     z[1, 2, 0] = 1e-3
     L.deltas_score_chunks(2, 3, torch.from_numpy(z).cuda(), 6, scores)
     assert scores[6].item() == float("inf") and oracle.chunk_score(z.astype(np.float64)) == float("inf")
+
+
+# ---------------------------------------------------------------- write sizes (Sec. 4.3 comparison signal)
+
+@pytest.mark.parametrize("d,dtype,T,Hk,Hv,decay", [
+    (128, "bf16", 257, 2, 4, 1.0),      # tensor cores: several tiles, ragged tail, grouped keys
+    (128, "bf16", 64, 1, 3, 1.0),       # one full tile, three value heads per key head
+    (128, "bf16", 300, 2, 4, 4.0),      # strong decay: the deferred decay restarts every tile
+    (64, "f32", 100, 2, 4, 1.0),        # CUDA-core kernel
+    (16, "bf16", 33, 1, 2, 1.0),
+    (128, "f32", 1, 2, 2, 1.0),
+])
+def test_write_norms_match_oracle(L, d, dtype, T, Hk, Hv, decay):
+    """Per (layer, head) sums over the chunk of beta_t ||v_t - alpha_t S_{t-1} k_t|| against the
+    oracle's token loop (relative 1e-3, the drift tolerance); asking for them changes neither the
+    state nor the drift partials, bit for bit."""
+    x = inputs.gdn_chunk(2, T, Hk, Hv, d, dtype, inputs.seed_for(70, d, T))
+    if decay != 1.0:
+        x["g"] = x["g"] * decay
+    s0 = inputs.initial_state(2, Hv, d, inputs.seed_for(71, d, T))
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    dev = torch.device("cuda")
+    desc = L.gdn_desc(2, Hk, Hv, d, tdt, None)
+    xs = {k: v.to(dev) for k, v in x.items()}
+    ws = L.alloc_workspace(L.deltas_gdn_chunk_update_workspace_size(desc, T), dev)
+    runs = []
+    for want in (False, True):
+        st = s0.to(dev).clone()
+        part = torch.full((2, Hv, 2), -1.0, device=dev)
+        wn = torch.full((2, Hv), -1.0, device=dev) if want else None
+        L.deltas_gdn_chunk_update(desc, T, None, xs["k"], xs["v"], xs["g"], xs["beta"], st, None, part, ws,
+                                  write_norms=wn)
+        torch.cuda.synchronize()
+        assert L.deltas_get_device_status(ws) == (0, 0)
+        runs.append((st, part, wn))
+    assert torch.equal(runs[0][0].view(torch.int32), runs[1][0].view(torch.int32))
+    assert torch.equal(runs[0][1].view(torch.int32), runs[1][1].view(torch.int32))
+    _, _, wn_ref = oracle.gdn_recurrence(None, _f64(x["k"]), _f64(x["v"]), _f64(x["g"]), _f64(x["beta"]), _f64(s0),
+                                         want_write_norms=True)
+    assert np.all(wn_ref > 0)
+    np.testing.assert_allclose(_f64(runs[1][2]), wn_ref, rtol=1e-3, atol=0)
+
+
+def test_write_norms_zero_tokens(L):
+    dev = torch.device("cuda")
+    desc = L.gdn_desc(1, 2, 2, 128, torch.bfloat16, None)
+    st = torch.ones(1, 2, 128, 128, device=dev)
+    wn = torch.full((1, 2), -1.0, device=dev)
+    ws = L.alloc_workspace(L.deltas_gdn_chunk_update_workspace_size(desc, 0), dev)
+    L.deltas_gdn_chunk_update(desc, 0, None, None, None, None, None, st, None, None, ws, write_norms=wn)
+    torch.cuda.synchronize()
+    assert torch.all(wn == 0)
+
+
+def test_write_norm_score(L):
+    """Chunk score of the comparison signal: the mean over heads, layers and tokens, as the oracle
+    computes it from the same float32 sums."""
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(72)
+    wn = rng.exponential(size=(24, 32)).astype(np.float32)
+    scores = torch.full((10,), -1.0, device=dev)
+    L.deltas_score_write_norms(24, 32, torch.from_numpy(wn).to(dev), 125, 7, scores)
+    L.deltas_score_write_norms(24, 32, torch.from_numpy(wn).to(dev), 0, 8, scores)
+    torch.cuda.synchronize()
+    sc = scores.cpu().numpy()
+    assert sc[7] == pytest.approx(oracle.write_norm_score(wn.astype(np.float64), 125), rel=1e-6)
+    assert sc[8] == 0.0 and sc[6] == -1.0

@@ -28,6 +28,11 @@ def _np(t):
     # and spans (Sec. 4.1), budget a few chunks so that most chunks evict
     dict(L=2, Hk=2, Hv=4, d=128, dt="bf16", Cs=[118, 132, 124, 121, 129, 119, 127, 125, 130, 118, 126, 131, 122, 128],
          Lf=2, Hkv=4, D=256, M=500, n_s=4, n_w=128, N=4, zero=False),
+    # the same stream scored by the comparison signal of Sec. 4.3 (write sizes) instead of drift
+    dict(L=2, Hk=2, Hv=4, d=128, dt="bf16", Cs=[118, 132, 124, 121, 129, 119, 127, 125, 130, 118, 126, 131, 122, 128],
+         Lf=2, Hkv=4, D=256, M=500, n_s=4, n_w=128, N=4, zero=False, signal="write_norm"),
+    dict(L=1, Hk=2, Hv=2, d=16, dt="f32", C=64, n_ch=8, Lf=1, Hkv=2, D=16, M=256, n_s=4, n_w=64, N=2, zero=True,
+         signal="write_norm"),
 ])
 def test_stream_matches_oracle(cfg):
     from paper_2609_27470_gb300.stream import DeltaSStream
@@ -44,7 +49,8 @@ def test_stream_matches_oracle(cfg):
     s = DeltaSStream(num_layers=cfg["L"], num_k_heads=cfg["Hk"], num_v_heads=cfg["Hv"], head_dim=cfg["d"],
                      act_dtype=tdt, kv_layers=cfg["Lf"], kv_heads=cfg["Hkv"], kv_head_dim=cfg["D"], kv_dtype=tdt,
                      budget_M=cfg["M"], n_sink=cfg["n_s"], n_window=cfg["n_w"], n_buckets=cfg["N"],
-                     chunk_len=cfg["C"], max_chunks=cfg["n_ch"], state0=s0.to(dev), device=dev)
+                     chunk_len=cfg["C"], max_chunks=cfg["n_ch"], state0=s0.to(dev), device=dev,
+                     signal=cfg.get("signal", "drift"))
     for c in range(cfg["n_ch"]):
         x = {k: v.to(dev) for k, v in chunks[c].items()}
         s.step(x["q"], x["k"], x["v"], x["g"], x["beta"], kvs[c][0].to(dev), kvs[c][1].to(dev))
@@ -56,7 +62,7 @@ def test_stream_matches_oracle(cfg):
     ref = run_stream(lambda c: tuple(f(chunks[c][k]) for k in ("q", "k", "v", "g", "beta")),
                      lambda c: (_np(kvs[c][0]), _np(kvs[c][1])), s0.double().numpy(), cfg["n_ch"],
                      dict(budget_M=cfg["M"], n_sink=cfg["n_s"], n_window=cfg["n_w"], n_buckets=cfg["N"]),
-                     capacity=s.capacity, score_override=gpu_scores)
+                     capacity=s.capacity, score_override=gpu_scores, signal=cfg.get("signal", "drift"))
     fin = np.isfinite(ref.chunk_scores)
     assert np.array_equal(np.isfinite(gpu_scores), fin)
     np.testing.assert_allclose(gpu_scores[fin], ref.chunk_scores[fin], rtol=1e-3)

@@ -138,6 +138,63 @@ def test_orthonormal_keys_rebuild_value_matrix():
     np.testing.assert_allclose(S[0, 0], v[0, :, 0].T.astype(np.float64), rtol=0, atol=1e-15)
 
 
+def test_write_norm_first_token_and_repeated_key():
+    """The write size beta_t ||v_t - alpha_t S_{t-1} k_t|| (Sec. 4.3 comparison signal), by hand:
+    from S_0 = 0 the first token writes beta_1 v_1; with alpha = beta = 1 a second token on the
+    same unit key writes v_2 - v_1 (the state already returns v_1 for that key)."""
+    d = 4
+    k = np.zeros((1, 2, 1, d), np.float32)
+    k[0, :, 0, 1] = 1.0                                              # e_2 twice
+    v = np.array([[[[1, 2, 3, 4]], [[2, 0, 3, 8]]]], np.float32)
+    g = np.zeros((1, 2, 1), np.float32)
+    beta = np.array([[[0.5], [1.0]]], np.float32)
+    S0 = np.zeros((1, 1, d, d))
+    _, _, wn = oracle.gdn_recurrence(None, k[:, :1], v[:, :1], g[:, :1], beta[:, :1], S0, want_write_norms=True)
+    assert wn[0, 0] == pytest.approx(0.5 * np.sqrt(30.0), rel=1e-15)
+    beta[:] = 1.0
+    _, _, wn = oracle.gdn_recurrence(None, k, v, g, beta, S0, want_write_norms=True)
+    assert wn[0, 0] == pytest.approx(np.sqrt(30.0) + np.sqrt(1 + 4 + 0 + 16), rel=1e-15)
+
+
+def test_write_norm_equals_state_step_change():
+    """For a unit key the write u_t k_t^T has Frobenius norm ||u_t||: the sum of write sizes equals
+    the sum over tokens of ||S_t - alpha_t S_{t-1}||_F, with the states taken one token at a time
+    from the product form of Eq. 1 (a second formulation), for several heads and grouped keys."""
+    rng = np.random.default_rng(15)
+    L, T, Hk, Hv, d = 2, 9, 1, 2, 6
+    q, k, v, g, beta = _rand_inputs(rng, L, T, Hk, Hv, d)
+    k = (k.astype(np.float64) / np.linalg.norm(k.astype(np.float64), axis=-1, keepdims=True)).astype(np.float32)
+    S0 = rng.standard_normal((L, Hv, d, d))
+    _, _, wn = oracle.gdn_recurrence(None, k, v, g, beta, S0, want_write_norms=True)
+    S = S0.copy()
+    ref = np.zeros((L, Hv))
+    for t in range(T):
+        sl = slice(t, t + 1)
+        S1 = oracle.gdn_recurrence_product_form(k[:, sl], v[:, sl], g[:, sl], beta[:, sl], S)
+        alpha = np.exp(g[:, t].astype(np.float64))                  # [L, Hv]
+        kk = k[:, t, 0].astype(np.float64)
+        n2 = np.sum(kk * kk, axis=-1)                                 # |k|^2 = 1 up to float32 rounding
+        ref += np.linalg.norm(S1 - alpha[:, :, None, None] * S, axis=(2, 3)) / np.sqrt(n2)[:, None]
+        S = S1
+    np.testing.assert_allclose(wn, ref, rtol=1e-10)
+
+
+def test_write_norm_score_is_the_mean_over_heads_layers_tokens():
+    """The chunk score averages the write sizes over heads, layers and the chunk's tokens."""
+    wn = np.array([[1.0, 2.0, 3.0], [4.0, 5.0, 6.5]])
+    assert oracle.write_norm_score(wn, 7) == pytest.approx(21.5 / (2 * 3 * 7), rel=1e-15)
+    assert oracle.write_norm_score(wn, 0) == 0.0
+
+
+def test_write_norm_zero_without_write():
+    """beta = 0: nothing is written, every write size is 0 whatever the state and values."""
+    rng = np.random.default_rng(16)
+    q, k, v, g, beta = _rand_inputs(rng, 1, 12, 1, 2, 8)
+    beta[:] = 0
+    _, _, wn = oracle.gdn_recurrence(None, k, v, g, beta, rng.standard_normal((1, 2, 8, 8)), want_write_norms=True)
+    assert np.all(wn == 0.0)
+
+
 def test_contraction_bound():
     """||I - beta k k^T||_2 <= 1 for beta in [0,1], ||k|| = 1, so
     ||S_t||_F <= alpha_t ||S_{t-1}||_F + beta_t ||v_t|| (Eq. 1)."""
