@@ -69,6 +69,7 @@ __device__ __forceinline__ char* plane_base(const CompactArgs& a, int p, int& rb
 }
 
 __global__ void compact_init_kernel(CompactArgs a) {
+    grid_dep_launch();                                 // the prepass may be scheduled now
     const int total = a.n_planes * a.max_tiles;
     for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x)
         a.flags[e] = 0;
@@ -81,6 +82,8 @@ __global__ void compact_init_kernel(CompactArgs a) {
 // source tile and for the unread tiles before it, each tile exactly once.  Rows with
 // retain_idx[j] == j form a prefix (a moved row pushes every later source further on).
 __global__ void compact_need_kernel(CompactArgs a) {
+    grid_dep_wait();                                   // the reset (and all earlier work) is done
+    grid_dep_launch();
     const int n = *a.n_retained;
     if (n < 0 || n > a.cache_len) {
         if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -146,6 +149,7 @@ compact_main_kernel(CompactArgs a)
     uint8_t* stage = reinterpret_cast<uint8_t*>(stage_raw);
     __shared__ uint64_t bar;
 
+    grid_dep_wait();                                   // the prepass is done
     volatile int* abort_flag = &a.ctl->abort;
     if (*abort_flag) return;
     const int n = *a.n_retained;
@@ -356,8 +360,10 @@ cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, con
     compact_init_kernel<<<init_blocks, 256, 0, s>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    compact_need_kernel<<<min(4 * sms, (cache_len + 255) / 256), 256, 0, s>>>(a);
-    e = cudaGetLastError();
+    // the prepass and the moves start while their predecessor finishes (each waits for it before
+    // reading or writing anything); the flag reset above is not overlapped: it writes the
+    // workspace that the preceding call may still be using
+    e = launch_dependent(compact_need_kernel, dim3(min(4 * sms, (cache_len + 255) / 256)), dim3(256), 0, s, a);
     if (e != cudaSuccess) return e;
 
     const int smem = a.tile_rows * a.row_bytes;
@@ -367,8 +373,7 @@ cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, con
     if (per_sm < 1) per_sm = 1;
     const int max_units = a.max_tiles * a.n_planes;
     const int grid = max(1, min(max_units, per_sm * sms));
-    compact_main_kernel<<<grid, 32, smem, s>>>(a);
-    return cudaGetLastError();
+    return launch_dependent(compact_main_kernel, dim3(grid), dim3(32), (size_t)smem, s, a);
 }
 
 cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_new, const void* v_new,

@@ -270,6 +270,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
     __shared__ uint64_t mb_k, mb_kk;
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
+    grid_dep_launch();                                // the update kernel may take SMs as they free up
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int n = a.n_tiles;
     const int items = a.L * a.Hv * n;                 // item = (layer * Hv + head) * n + tile
@@ -845,6 +846,9 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         TileCursor cc;
         cc.init(a);
         int kp[3] = {-1, -1, -1}, vp[2] = {-1, -1}, rp[2] = {-1, -1};   // last tile loaded per buffer
+        // the kernel may start while the factor kernel finishes (its set-up and the first state
+        // load overlap that tail); the records it wrote are read only after it has completed
+        grid_dep_wait();
         for (int J = 0; J < NJ; ++J) {
             const int bk = J % 3, b2 = J & 1;
             if (J >= 3 && !warp_wait(&mb_ke[bk], ((J / 3) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 30); break; }
@@ -1303,8 +1307,8 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = n_tiles;
     t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.rec = a.scratch; t.status = a.status;
     const int grid = std::min(a.L * a.Hv, sms);
-    gdn_update_tc_kernel<<<grid, kThreads, kSmemAlloc, s>>>(kmap, vmap, smap, t);
-    return cudaGetLastError();
+    return launch_dependent(gdn_update_tc_kernel, dim3(grid), dim3(kThreads), (size_t)kSmemAlloc, s, kmap, vmap,
+                            smap, t);
 }
 
 }  // namespace deltas

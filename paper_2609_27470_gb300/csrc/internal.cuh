@@ -39,6 +39,31 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
 
 inline int elt_bytes(int32_t dtype) { return dtype == DELTAS_BF16 ? 2 : 4; }
 
+// Programmatic dependent launch.  A kernel launched with launch_dependent() may be scheduled while
+// the previous kernel of the stream is still running (it then overlaps that kernel's tail and its
+// own launch latency); before it touches anything earlier work wrote it calls grid_dep_wait(),
+// which returns once the previous kernel has completed and its writes are visible (hardware
+// managed: no flag, no spin).  A kernel calls grid_dep_launch() to let its dependent be scheduled
+// before it ends; the dependent's wait still covers all of it.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                             Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // ---------------------------------------------------------------------------------------------
 // Launch arguments
 // ---------------------------------------------------------------------------------------------

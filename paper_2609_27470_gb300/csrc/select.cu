@@ -186,6 +186,7 @@ select_runs_kernel(SelArgs a)
 {
     __shared__ int s_wsum[kScanThreads / 32];
     __shared__ int s_min[kScanThreads / 32], s_max[kScanThreads / 32], s_bad[kScanThreads / 32];
+    grid_dep_launch();                                 // the decision kernel may be scheduled now
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int T = a.T, lo = a.n_s, hi = T - a.n_w;
     const int b0 = blockIdx.x * kScanSlots;
@@ -261,6 +262,8 @@ select_retain_kernel(SelArgs a)
     __shared__ int s_rstart[kSmallRuns], s_rlen[kSmallRuns], s_rspan[kSmallRuns], s_rkept[kSmallRuns],
         s_roff[kSmallRuns];
 
+    grid_dep_wait();                                   // the run scan (and all earlier work) is done
+    grid_dep_launch();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int T = a.T;
     const int n_blocks = (T + kScanSlots - 1) / kScanSlots;
@@ -450,6 +453,7 @@ select_retain_kernel(SelArgs a)
 __global__ void __launch_bounds__(256)
 select_emit_kernel(SelArgs a)
 {
+    grid_dep_wait();                                   // the decision is complete
     if (!a.ctl->emit) return;
     const int n_runs = a.ctl->n_runs;
     const int T = a.T, lo = a.n_s, hi = T - a.n_w;
@@ -498,13 +502,13 @@ cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_
         cudaError_t e0 = cudaGetLastError();
         if (e0 != cudaSuccess) return e0;
     }
-    select_retain_kernel<<<1, kSelThreads, 0, s>>>(a);
-    cudaError_t e = cudaGetLastError();
+    // the decision and the emission start while their predecessor finishes (each waits for it
+    // before reading anything)
+    cudaError_t e = launch_dependent(select_retain_kernel, dim3(1), dim3(kSelThreads), 0, s, a);
     if (e != cudaSuccess) return e;
     const int sms = device_sm_count();
     const int blocks = std::max(1, std::min((cache_len + 255) / 256, 2 * sms));
-    select_emit_kernel<<<blocks, 256, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_dependent(select_emit_kernel, dim3(blocks), dim3(256), 0, s, a);
 }
 
 }  // namespace deltas
