@@ -110,6 +110,22 @@ def test_select_streaming_shape(L):
     _assert_same_selection(L, 32768, 4, 1024, 4, tc, sc)
 
 
+@pytest.mark.parametrize("T,n_ch,run_max", [(100000, 700, 400), (150000, 20000, 6)])
+def test_select_large_caches(L, T, n_ch, run_max):
+    """Caches past the one-CTA size (64k slots) take the grid-wide run scan, the decision kernel
+    and the grid-wide emission: a few hundred long runs (ranked in shared memory) and tens of
+    thousands of short ones (the radix path); the paper's policy and exact score ties."""
+    rng = np.random.default_rng(T + n_ch)
+    lens = rng.integers(1, run_max + 1, size=4 * T // (run_max + 1) + 8)
+    ids = np.sort(rng.integers(0, n_ch, size=lens.size)).astype(np.int32)
+    tc = np.repeat(ids, lens)[:T].astype(np.int32)
+    assert tc.size == T
+    sc = rng.exponential(size=n_ch).astype(np.float32)
+    sc[rng.integers(0, n_ch, size=6)] = sc[3]
+    _assert_same_selection(L, T // 3, 4, 1024, 4, tc, sc)
+    _assert_same_selection(L, T - 1, 0, 0, 1, tc, sc)
+
+
 def test_select_edge_cases(L):
     rng = np.random.default_rng(105)
     tc = np.repeat(np.arange(10, dtype=np.int32), 10)
