@@ -20,40 +20,40 @@
 // (S_before beside it, for the drift), so the state is read from and written to HBM exactly once;
 // the next head's state is loaded into shared memory while the current head runs, and the head
 // boundary swaps the two in one pass that also forms the drift partials.  Per tile:
-//   X region  <- V^T                       (MMA: V tile times an identity matrix, exact)
-//   X region  += S~ K'^T = W^T / ...        (tf32 MMA, K' = K scaled per token by -gamma_t sig)
-//   W pass:   W (x u_scale) -> (hi, lo) in place            (chain)
+//   V region  <- V^T                       (MMA: V tile times an identity matrix, exact)
+//   X region  <- S~ K^T                     (tf32 MMA, K exact in fp32)
+//   W pass:   W^T = V^T - sig X diag(gamma), x u_scale -> (hi, lo) in place over X   (chain)
 //   U region  <- W^T T~^T = U~^T / ...      (MMA)
 //   U~ pass:  -> (hi, lo) in place                          (chain)
 //   S~        += U~^T K                     (MMA)
-// so the chain's passes are a load, a split and a store per element, and the per-token decays
-// ride on K' (formed while the chain converts K to fp32 anyway) and on T~.
+// so the chain's passes are a few loads, an FMA, a split and a store per element, and the
+// per-token decays ride on the W pass and on T~.
 //
 // Precision.  Keys and values are exact in bfloat16.  The state never leaves fp32 inside the
 // tile loop: TMEM holds S~ with S = sig S~, and X reads S~ straight from TMEM as the A operand of
 // a kind::tf32 product; the hardware keeps 10 mantissa bits of S~ (a relative error below 2^-10
-// per element) and K' is rounded to tf32 (2^-11), errors that reach the state only through the
+// per element) while K is exact, an error that reaches the state only through the
 // delta correction and decay with it (a CPU simulation of the truncation gives a state error vs
 // fp64 of ~2e-4 at the slowest decay the inputs use, 5e-6 at a typical one).  The other products
 // take a two-term bfloat16 split (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)) of each fp32
 // operand:
 //   V^T I                           exact                                        1 MMA group
-//   X^T  = S0 K'^T                  S~ (tf32, from TMEM) K'^T (tf32)              1 MMA group
+//   X^T  = S~ K^T                   S~ (tf32, from TMEM) K (exact in tf32)       1 MMA group
 //   U~^T = W^T T~^T                  Whi T~hi + Whi T~lo + Wlo T~hi                3 MMA groups
 //   S   += U~^T K                   (U~hi + U~lo) K                              2 MMA groups
 //   K K^T (factor kernel)           exact inputs                                 1 MMA group
 // All products accumulate in fp32 in TMEM.
 //
 // Deferred decay: the tile decay gamma_C is folded into the scalar sig instead of a pass that
-// multiplies S by gamma_C; K' carries sig and W is scaled by u_scale = 1 / (gamma_C sig) so that
+// multiplies S by gamma_C; the W pass applies sig and scales W by u_scale = 1 / (gamma_C sig) so that
 // MMA_S adds onto S~ directly.  When sig gamma_C would fall below 2^-30 the tile writes
 // gamma_C sig S~ back into TMEM and sig restarts at 1 (u_scale = 1), so 1 / sig stays far from the
 // fp32 range limit.  The head's last tile multiplies by sig when it reads the state out.
 //
 // Update-kernel warp roles (19 warps):
 //   0-15  state chain: warp w serves TMEM lanes 32 (w % 4) .. + 31 (state rows) and column group
-//         w / 4; per tile the W and U~ passes (16 token columns each) and the next tile's K'
-//         (two 16-byte chunks each), at head boundaries the state swap and the drift partials
+//         w / 4; per tile the W and U~ passes (16 token columns each) and the next tile's K in
+//         fp32 (two 16-byte chunks each), at head boundaries the state swap and the drift partials
 //   16    TMEM allocation and every tcgen05.mma (one elected lane issues; the warp stays
 //         converged); it also releases the input buffers by tcgen05.commit
 //   17    tile loads: K, V (TMA) and the WY records (bulk copy), as buffers are released
@@ -63,8 +63,8 @@
 // mbarriers only.  Every wait is bounded; a wait that runs out records DELTAS_ERR_TIMEOUT, raises
 // a CTA-wide abort flag so the other roles stop waiting, and the CTA drains its MMAs and copies
 // before freeing TMEM.
-// TMEM (512 columns, M = 128 lanes = d_v): S~ [0,128), S_before [128,256), X [256,320) (V^T + X,
-// then W hi / lo packed in place), U [320,384) (likewise U~); [384,512) unused.
+// TMEM (512 columns, M = 128 lanes = d_v): S~ [0,128), S_before [128,256), X [256,320) (X, then
+// W hi / lo packed in place), U [320,384) (likewise U~), V^T [384,448); [448,512) unused.
 #include <algorithm>
 
 #include "internal.cuh"
@@ -626,11 +626,11 @@ constexpr int kLoadWarp = kChainWarps + 1;       // 17
 constexpr int kStateWarp = kChainWarps + 2;      // 18
 constexpr int kThreads = kChain + 96;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t TM_S = 0, TM_SB = 128, TM_X = 256, TM_U = 320;
+constexpr uint32_t TM_S = 0, TM_SB = 128, TM_X = 256, TM_U = 320, TM_V = 384;
 
 // shared-memory map (bytes from a 1024-aligned base)
 constexpr uint32_t SM_K = 0;                     // 3 x 16 KB: K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
-constexpr uint32_t SM_K32 = 49152;               // 32 KB: K' in tf32 (the B operand of X), 4 column blocks
+constexpr uint32_t SM_K32 = 49152;               // 32 KB: K in fp32 (the B operand of X), 4 column blocks
                                                  // (32 dims) x 64 rows x 128 B, SW128
 constexpr uint32_t SM_V = 81920;                 // 2 x 16 KB: V tile (tile parity), layout of K
 constexpr uint32_t SM_R = 114688;                // 2 x kRecSlot: WY records (tile parity)
@@ -743,7 +743,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         // Each group's operands are formed before the wait that releases it, so that only the
         // MMA instructions themselves follow the wait (this warp shares its scheduler with four
         // chain warps).
-        // X region <- V(J)^T: A = the V tile read MN-major (k-step s = tokens 16 s ..), B = I.  V(J)'s
+        // V region <- V(J)^T: A = the V tile read MN-major (k-step s = tokens 16 s ..), B = I.  V(J)'s
         // buffer is released when the product completes.
         auto issue_vi = [&](int J) -> bool {
             uint64_t av[4], bv[4];
@@ -754,7 +754,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             }
             if (!warp_wait(&mb_tv[J & 1], (J >> 1) & 1, kWaitBudgetNs, abort_flag)) return false;
             tc_fence_after();
-            if (elect_one()) mma4_bf16_ss_1t(tm + TM_X, av, bv, idesc_bf16(128, 64, 1, 0), 0);
+            if (elect_one()) mma4_bf16_ss_1t(tm + TM_V, av, bv, idesc_bf16(128, 64, 1, 0), 0);
             __syncwarp();
             mma_commit(&mb_ve[J & 1]);
             return true;
@@ -762,9 +762,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         bool ok = NJ == 0 || issue_vi(0);
         if (!ok) fail(a.status, abort_flag, 1);
         for (int j = 0; ok && j < NJ; ++j) {           // j: global tile index
-            {   // X region += S~ K'^T: A = the fp32 state from TMEM read as tf32 (8 columns per K = 8
-                // step), B = K'.  Tile j ready for X: K'(j) is written and, at a head's first tile,
-                // the state is in TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe order).
+            {   // X region <- S~ K^T: A = the fp32 state from TMEM read as tf32 (8 columns per K = 8
+                // step), B = K in fp32.  Tile j ready for X: K(j) is converted and, at a head's first
+                // tile, the state is in TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe
+                // order).
                 uint32_t ax[4][4];
                 uint64_t bx[4][4];
 #pragma unroll
@@ -777,7 +778,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tc_fence_after();
                 if (elect_one()) {
 #pragma unroll
-                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + TM_X, ax[g4], bx[g4], idesc_tf32(128, 64), 1);
+                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + TM_X, ax[g4], bx[g4], idesc_tf32(128, 64), g4 != 0);
                 }
                 __syncwarp();
                 mma_commit(&mb_x);
@@ -808,7 +809,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 mma_commit(&mb_u);
                 mma_commit(&mb_re[j & 1]);             // record slot free once MMA_U(j) has read T~
             }
-            // the next tile's V^T into the X region (MMA_U(j), its last reader, is ahead in the pipe)
+            // the next tile's V^T into the V region (its last reader, the W pass of tile j, has
+            // finished: MMA_U(j) waited for xready)
             if (j + 1 < NJ && !issue_vi(j + 1)) { fail(a.status, abort_flag, 4); break; }
             {   // S~ += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major)
                 uint32_t as_[2][4];
@@ -936,10 +938,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         int st_seen = 0;                                 // mb_st phases waited for (uniform)
         TileCursor cc;                                   // the chain's tile
         cc.init(a);
-        // K'(jj) = K(jj) (TMA tile, buffer jj % 3) scaled per token t by gm[t] * xs = -gamma_t sig,
-        // rounded to tf32, into the B operand buffer of X.  Called between MMA_X(jj-1), the last
-        // reader of the buffer, and the ready signal of tile jj.
-        auto make_kprime = [&](int jj, float xs, const float* gm) -> bool {
+        // K(jj) (TMA tile, buffer jj % 3) in fp32 (exact, and exact in tf32) into the B operand
+        // buffer of X.  Called between MMA_X(jj-1), the last reader of the buffer, and the ready
+        // signal of tile jj.
+        auto make_k32 = [&](int jj) -> bool {
             const bool ok = mbar_wait_or_abort(&mb_tk[jj % 3], (jj / 3) & 1, kWaitBudgetNs, abort_flag);
             const uint8_t* kb = sm + SM_K + (jj % 3) * 16384;
             uint8_t* k32 = sm + SM_K32;
@@ -947,20 +949,19 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             for (int u = 0; u < 2; ++u) {                  // 64 rows x 16 chunks of 8 bf16
                 const int e = tid + kChain * u;
                 const int t = e >> 4, c16 = e & 15, cb = c16 >> 3, c = c16 & 7;
-                const float sc = gm[t] * xs;
                 const uint4 w = *reinterpret_cast<const uint4*>(kb + cb * 8192 + sw128_offset(t, c));
                 const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
-                float f[8];
+                uint32_t f[8];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    f[2 * i] = round_tf32(__uint_as_float(wv[i] << 16) * sc);
-                    f[2 * i + 1] = round_tf32(__uint_as_float(wv[i] & 0xFFFF0000u) * sc);
+                    f[2 * i] = wv[i] << 16;
+                    f[2 * i + 1] = wv[i] & 0xFFFF0000u;
                 }
                 // dims 64 cb + 8 c .. + 7: fp32 block 2 cb + c / 4, chunks 2 (c % 4) and 2 (c % 4) + 1
                 uint8_t* rowp = k32 + (2 * cb + (c >> 2)) * 8192;
                 const int q0 = 2 * (c & 3);
-                *reinterpret_cast<float4*>(rowp + sw128_offset(t, q0)) = make_float4(f[0], f[1], f[2], f[3]);
-                *reinterpret_cast<float4*>(rowp + sw128_offset(t, q0 + 1)) = make_float4(f[4], f[5], f[6], f[7]);
+                *reinterpret_cast<uint4*>(rowp + sw128_offset(t, q0)) = make_uint4(f[0], f[1], f[2], f[3]);
+                *reinterpret_cast<uint4*>(rowp + sw128_offset(t, q0 + 1)) = make_uint4(f[4], f[5], f[6], f[7]);
             }
             fence_async_smem();                            // generic writes -> the tensor core's reads
             return ok;
@@ -970,7 +971,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         };
         float den = 0.f;
         // Deferred decay: TMEM holds S~ with the head's state S = sig * S~.  A tile folds its decay
-        // gamma_C into sig (K' carries sig, W is scaled by u_scale = 1 / (gamma_C sig), so MMA_S
+        // gamma_C into sig (the W pass applies sig and u_scale = 1 / (gamma_C sig), so MMA_S
         // accumulates onto S~ with no pass over the state); when sig gamma_C would drop below
         // kSigMin the tile instead writes gamma_C S back into TMEM and sig restarts at 1.
         float sig = 1.f;
@@ -1026,7 +1027,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 warp_arrive(&mb_sfree, lane);                    // the staging buffer has been read
                 tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
                 tmem_st32(tm + lane_off + TM_SB + 32 * cgp, sv);
-                if (!make_kprime(0, 1.f, rec_consts(0))) fail(a.status, abort_flag, 16);
+                if (!make_k32(0)) fail(a.status, abort_flag, 16);
                 tmem_st_wait();
                 tc_fence_before();
                 warp_arrive(&mb_sready, lane);
@@ -1034,17 +1035,26 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             const bool rescale = sig * gC < kSigMin;       // uniform over the CTA
             const float u_scale = rescale ? 1.f : 1.f / (gC * sig);
 
-            // ---- W pass: the X region holds W^T = V^T - X^T diag(gamma); scaled by u_scale, (hi,
-            // lo) in place over this thread's 16 columns (tokens 16 cgp ..)
+            // ---- W pass: W^T = V^T - sig X~^T diag(gamma) from the V and X regions (X~ = S~ K^T),
+            // scaled by u_scale, (hi, lo) in place over this thread's 16 X columns (tokens 16 cgp ..)
             if (!mbar_wait_or_abort(&mb_x, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 10);
             tc_fence_after();
             {
-                float wv[16];
-                tmem_ld16(tm + lane_off + TM_X + 16 * cgp, wv);
+                float xv[16], vv[16], cf[16];
+                tmem_ld16(tm + lane_off + TM_X + 16 * cgp, xv);
+                tmem_ld16(tm + lane_off + TM_V + 16 * cgp, vv);
+                const float* gm = rec_consts(j) + 16 * cgp;         // -gamma of the thread's tokens
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float4 g4 = *reinterpret_cast<const float4*>(gm + 4 * e);
+                    cf[4 * e] = g4.x * sig; cf[4 * e + 1] = g4.y * sig; cf[4 * e + 2] = g4.z * sig; cf[4 * e + 3] = g4.w * sig;
+                }
                 tmem_ld_wait();
                 uint32_t hi[8], lo[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) split2(wv[2 * i] * u_scale, wv[2 * i + 1] * u_scale, hi[i], lo[i]);
+                for (int i = 0; i < 8; ++i)
+                    split2(fmaf(cf[2 * i], xv[2 * i], vv[2 * i]) * u_scale,
+                           fmaf(cf[2 * i + 1], xv[2 * i + 1], vv[2 * i + 1]) * u_scale, hi[i], lo[i]);
                 tmem_st8(tm + lane_off + TM_X + 16 * cgp, hi);
                 tmem_st8(tm + lane_off + TM_X + 16 * cgp + 8, lo);
                 tmem_st_wait();
@@ -1053,7 +1063,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             warp_arrive(&mb_xready, lane);
 
             // ---- while MMA_U runs: rescale S~ if the decay would underflow the deferred scale
-            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K'(j+1)
+            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K(j+1) in fp32
             if (rescale) {
                 const float f = gC * sig;
                 float sv[32];
@@ -1065,12 +1075,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tmem_st_wait();
             }
             sig = rescale ? 1.f : gC * sig;                // the deferred decay after tile j
-            if (j + 1 < NJ) {
-                // K'(j+1): its tile's -gamma and the sig it starts with (1 at a head's first tile)
-                if (!mbar_wait_or_abort(&mb_tr[(j + 1) & 1], ((j + 1) >> 1) & 1, kWaitBudgetNs, abort_flag))
-                    fail(a.status, abort_flag, 15);
-                if (!make_kprime(j + 1, last ? 1.f : sig, rec_consts(j + 1))) fail(a.status, abort_flag, 16);
-            }
+            if (j + 1 < NJ && !make_k32(j + 1)) fail(a.status, abort_flag, 16);
 
             // ---- U~ pass: (hi, lo) in place over this thread's 16 U columns
             if (!mbar_wait_or_abort(&mb_u, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 11);
