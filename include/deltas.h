@@ -50,7 +50,7 @@ extern "C" {
 typedef enum deltas_status_e {
     DELTAS_OK = 0,
     DELTAS_ERR_INVALID_ARGUMENT = 1, /* a pointer, size or value outside its stated range        */
-    DELTAS_ERR_UNSUPPORTED = 2,      /* valid, but a shape/dtype this build has no kernel for     */
+    DELTAS_ERR_UNSUPPORTED = 2,      /* valid, but a shape/dtype the library has no kernel for    */
     DELTAS_ERR_WORKSPACE = 3,        /* workspace missing, misaligned or smaller than required    */
     DELTAS_ERR_CUDA = 4,             /* a CUDA launch or runtime call failed                      */
     DELTAS_ERR_TIMEOUT = 5,          /* device: a bounded wait ran out (work skipped)             */
@@ -69,7 +69,7 @@ typedef struct deltas_gdn_desc {
     int32_t num_k_heads;  /* Hk >= 1 */
     int32_t num_v_heads;  /* Hv >= 1, a multiple of Hk */
     int32_t key_dim;      /* d_k in {16, 32, 64, 128} */
-    int32_t value_dim;    /* d_v, equal to d_k in this build */
+    int32_t value_dim;    /* d_v, equal to d_k (the only supported case) */
     int32_t dtype;        /* deltas_dtype of q, k, v and out; g, beta and the state are float32 */
     float q_scale;        /* read-out scale: o_t = q_scale * S_t q_t (commonly 1/sqrt(d_k)) */
 } deltas_gdn_desc;
