@@ -11,6 +11,9 @@ only marshals numpy arrays.  Each wrapper names the paper passage its C function
 * :func:`gdn_recurrence_product_form` — the same rule in product form (Eq. 1), a self-check.
 * :func:`drift_partials`, :func:`chunk_score` — state drift (Eq. 3; Alg. 1).
 * :func:`select_retain` — sink / window / temporal spans / quota + fill (Sec. 3.3; Alg. 1).
+* :func:`row_norm_scores`, :func:`select_retain_tokens`, :func:`compact_kv_heads` — the
+  cache-internal token signals of the controlled comparison (Sec. 4.3: key norm, value norm; per KV
+  head, per token) ranked under the same policy, and the per-head gather that follows.
 * :func:`compact_rows`, :func:`compact_kv` — KV gather in stream order (Alg. 1; Sec. 3.3).
 * :func:`stream` (in :mod:`oracle.stream`) — the Alg. 1 loop over a whole stream.
 
@@ -67,6 +70,10 @@ def _load():
             lib.oracle_select_retain.restype = _I
             lib.oracle_compact_rows.argtypes = [_I] * 4 + [_P] * 3 + [_I]
             lib.oracle_compact_rows.restype = _I
+            lib.oracle_row_norm_scores.argtypes = [_I, _I, _P, _I, _P]
+            lib.oracle_row_norm_scores.restype = _I
+            lib.oracle_select_retain_tokens.argtypes = [_I] * 5 + [_P] * 5
+            lib.oracle_select_retain_tokens.restype = _I
             _lib = lib
     return _lib
 
@@ -194,3 +201,59 @@ def compact_kv(k_cache, v_cache, tok_chunk, tok_pos, retain_idx, cache_len: int)
     tc = compact_rows(np.asarray(tok_chunk, dtype=np.int32).reshape(1, cap, 1), retain_idx, cache_len)
     tp = compact_rows(np.asarray(tok_pos, dtype=np.int32).reshape(1, cap, 1), retain_idx, cache_len)
     return k2, v2, tc.reshape(cap), tp.reshape(cap)
+
+
+TOKEN_SIGNALS = ("key_norm", "value_norm")
+
+
+def row_norm_scores(rows, signal: str) -> np.ndarray:
+    """Token scores of the cache-internal signals (Sec. 4.3, appendix table of signals):
+    ``key_norm`` -> -||k||_2 of each key row, ``value_norm`` -> ||v||_2 of each value row.
+    ``rows`` is [..., D] (bf16 values widened exactly by the caller); the fp64 result is rounded
+    to float32, the precision the paper computes every score in."""
+    if signal not in TOKEN_SIGNALS:
+        raise ValueError(f"unknown token signal {signal!r}")
+    r = np.asarray(rows)
+    shape = r.shape[:-1]
+    D = r.shape[-1]
+    a = _f32(r.reshape(-1, D))
+    out = np.zeros(max(a.shape[0], 1), dtype=np.float64)
+    rc = _load().oracle_row_norm_scores(int(a.shape[0]), int(D), _ptr(a), 1 if signal == "key_norm" else 0,
+                                        _ptr(out))
+    _check(rc, "row_norm_scores")
+    return out[: a.shape[0]].astype(np.float32).reshape(shape)
+
+
+def select_retain_tokens(budget_M: int, n_sink: int, n_window: int, n_buckets: int, tok_chunk, tok_scores):
+    """Sec. 3.3 retention with one float32 score per slot (the token signals of Sec. 4.3).
+    Returns ``(retain_idx int32[n], mask uint8[T])``."""
+    tc = np.ascontiguousarray(np.asarray(tok_chunk, dtype=np.int32))
+    sc = _f32(tok_scores)
+    T = tc.shape[0]
+    if sc.shape[0] != T:
+        raise ValueError("one score per slot expected")
+    idx = np.zeros(max(T, 1), dtype=np.int32)
+    mask = np.zeros(max(T, 1), dtype=np.uint8)
+    n = ctypes.c_int32(0)
+    rc = _load().oracle_select_retain_tokens(int(budget_M), int(n_sink), int(n_window), int(n_buckets), T,
+                                             _ptr(tc), _ptr(sc), _ptr(idx),
+                                             ctypes.cast(ctypes.pointer(n), ctypes.c_void_p), _ptr(mask))
+    _check(rc, "select_retain_tokens")
+    return idx[: n.value].copy(), mask[:T].copy()
+
+
+def compact_kv_heads(k_cache, v_cache, tok_chunk, tok_pos, tok_score, retain_lists, cache_len: int):
+    """Per-head gather (each KV head keeps its own tokens): plane p = (layer, KV head) of K, V and
+    of the per-head metadata tok_chunk / tok_pos / tok_score [Lf, Hkv, cap] is gathered by its own
+    list ``retain_lists[p]`` (all lists have the same length)."""
+    kc, vc = np.asarray(k_cache), np.asarray(v_cache)
+    Lf, Hkv, cap = kc.shape[:3]
+    P = Lf * Hkv
+    if len(retain_lists) != P:
+        raise ValueError("one retain list per (layer, KV head) plane expected")
+    outs = []
+    for arr in (kc, vc, tok_chunk, tok_pos, tok_score):
+        a = np.asarray(arr).reshape(P, cap, -1)
+        o = np.stack([compact_rows(a[p:p + 1], retain_lists[p], cache_len)[0] for p in range(P)])
+        outs.append(o.reshape(np.asarray(arr).shape))
+    return tuple(outs)

@@ -308,6 +308,104 @@ int oracle_select_retain(int M, int n_sink, int n_window, int n_buckets,
 }
 
 /* ------------------------------------------------------------------------------------------ */
+/* Cache-internal token signals of the controlled comparison (Sec. 4.3 and the appendix table   */
+/* of retention signals): the key-norm signal scores a cached token by -||k||_2 and the         */
+/* value-norm signal by ||v||_2, per KV head and per token.  Row r of rows[n_rows][D] gets       */
+/*     out[r] = sign * sqrt(sum_i rows[r][i]^2),   sign = -1 (negate != 0) or +1.               */
+/* ------------------------------------------------------------------------------------------ */
+int oracle_row_norm_scores(int n_rows, int D, const float* rows, int negate, double* out)
+{
+    if (n_rows < 0 || D < 1 || (n_rows > 0 && (!rows || !out))) return ORACLE_BAD_ARG;
+    for (int r = 0; r < n_rows; ++r) {
+        double s = 0.0;
+        for (int i = 0; i < D; ++i) {
+            const double x = rows[(size_t)r * D + i];
+            s += x * x;
+        }
+        out[r] = negate ? -sqrt(s) : sqrt(s);
+    }
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------------------------ */
+/* Retain selection with one score per token (the token-granular signals of Sec. 4.3, ranked  */
+/* under the shared policy of Sec. 3.3: the same sink, window, temporal spans, quota and fill  */
+/* as oracle_select_retain above).  The only difference: slot i is ranked by tok_scores[i]     */
+/* instead of the score of its chunk.  Spans still split the candidates' arrival chunks.        */
+/* Ranking key: higher score first (float32 total order), ties to the lower slot.              */
+/* ------------------------------------------------------------------------------------------ */
+int oracle_select_retain_tokens(int M, int n_sink, int n_window, int n_buckets, int T,
+                                const int32_t* tok_chunk, const float* tok_scores,
+                                int32_t* retain_idx, int32_t* n_retained, uint8_t* mask)
+{
+    if (M < 1 || n_sink < 0 || n_window < 0 || n_buckets < 0 || T < 0) return ORACLE_BAD_ARG;
+    if ((long long)M < (long long)n_sink + n_window + 1) return ORACLE_BAD_ARG;
+    if (!retain_idx || !n_retained || (T > 0 && (!tok_chunk || !tok_scores))) return ORACLE_BAD_ARG;
+    for (int i = 0; i < T; ++i)
+        if (tok_chunk[i] < 0) return ORACLE_BAD_ARG;
+    const int N = n_buckets < 1 ? 1 : n_buckets;
+
+    uint8_t* keep = (uint8_t*)calloc((size_t)(T > 0 ? T : 1), 1);
+    if (!keep) return ORACLE_NO_MEMORY;
+
+    if (T <= M) {
+        for (int i = 0; i < T; ++i) keep[i] = 1;
+    } else {
+        const int cand_lo = n_sink, cand_hi = T - n_window;
+        for (int i = 0; i < n_sink; ++i) keep[i] = 1;
+        for (int i = cand_hi; i < T; ++i) keep[i] = 1;
+        const int R = M - n_sink - n_window;
+        int c_lo = tok_chunk[cand_lo], c_hi = tok_chunk[cand_lo];
+        for (int i = cand_lo; i < cand_hi; ++i) {
+            if (tok_chunk[i] < c_lo) c_lo = tok_chunk[i];
+            if (tok_chunk[i] > c_hi) c_hi = tok_chunk[i];
+        }
+        const long long span = (long long)c_hi - c_lo + 1;
+        const int quota = R / N;
+        const int n_cand = cand_hi - cand_lo;
+        ranked_slot* list = (ranked_slot*)malloc(sizeof(ranked_slot) * (size_t)n_cand);
+        if (!list) { free(keep); return ORACLE_NO_MEMORY; }
+        int kept = 0;
+        /* phase 1: per-span quota, best tokens first */
+        for (int j = 0; j < N; ++j) {
+            int m = 0;
+            for (int i = cand_lo; i < cand_hi; ++i) {
+                const long long b = ((long long)(tok_chunk[i] - c_lo) * N) / span;
+                if (b == j) {
+                    list[m].score_key = total_order_key(tok_scores[i]);
+                    list[m].slot = i;
+                    ++m;
+                }
+            }
+            qsort(list, (size_t)m, sizeof(ranked_slot), ranked_cmp);
+            const int take = m < quota ? m : quota;
+            for (int r = 0; r < take; ++r) keep[list[r].slot] = 1;
+            kept += take;
+        }
+        /* phase 2: the unused capacity goes to the best remaining tokens of any span */
+        int m = 0;
+        for (int i = cand_lo; i < cand_hi; ++i)
+            if (!keep[i]) {
+                list[m].score_key = total_order_key(tok_scores[i]);
+                list[m].slot = i;
+                ++m;
+            }
+        qsort(list, (size_t)m, sizeof(ranked_slot), ranked_cmp);
+        const int fill = R - kept;
+        for (int r = 0; r < fill && r < m; ++r) keep[list[r].slot] = 1;
+        free(list);
+    }
+    int n = 0;
+    for (int i = 0; i < T; ++i) {
+        if (keep[i]) retain_idx[n++] = i;
+        if (mask) mask[i] = keep[i];
+    }
+    *n_retained = n;
+    free(keep);
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------------------------ */
 /* KV compaction (Alg. 1, "KV <- KV[I_sink u I_DeltaS u I_window]"; Sec. 3.3: survivors keep    */
 /* their original position indices).  Out-of-place gather of fixed-size rows, applied to every */
 /* plane independently (each full-attention layer, K and V, each KV head):                      */

@@ -14,6 +14,10 @@ Test infrastructure only.  One iteration per arriving chunk c:
 
 Scores of earlier chunks are reused at later evictions (Sec. 3.3).
 
+:func:`run_stream_heads` runs the same loop with a cache-internal token signal of Sec. 4.3 (key
+norm or value norm) in place of the chunk score: every KV head ranks its own tokens, so every
+(layer, KV head) plane keeps its own M tokens, with its own chunk ids, positions and scores.
+
 A question (Sec. 3.3, "Question answering") arriving before chunk c saves the whole stream state
 (recurrent state, caches with chunk ids and positions, scores, counters), runs the question's
 tokens through the same loop body, and then puts the saved state back: question turns change
@@ -25,7 +29,8 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
-from . import compact_kv, gdn_recurrence, select_retain, state_drift, write_norm_score
+from . import (compact_kv, compact_kv_heads, gdn_recurrence, row_norm_scores, select_retain,
+               select_retain_tokens, state_drift, write_norm_score)
 
 
 @dataclass
@@ -115,5 +120,67 @@ def run_stream(chunk_inputs, kv_inputs, state0, n_chunks: int, policy: dict, cap
     res.chunk_scores = scores
     res.k_cache, res.v_cache = kc, vc
     res.tok_chunk, res.tok_pos = tok_chunk, tok_pos
+    res.cache_len = T
+    return res
+
+
+@dataclass
+class HeadStreamResult:
+    k_cache: np.ndarray               # [Lf,Hkv,capacity,D]
+    v_cache: np.ndarray
+    tok_chunk: np.ndarray             # [Lf,Hkv,capacity] int32
+    tok_pos: np.ndarray               # [Lf,Hkv,capacity] int32
+    tok_score: np.ndarray             # [Lf,Hkv,capacity] float32
+    cache_len: int
+    evictions: list = field(default_factory=list)   # (chunk, [retain list per plane])
+
+
+def run_stream_heads(kv_inputs, n_chunks: int, policy: dict, capacity: int, signal: str,
+                     score_override=None):
+    """Alg. 1's append / select / gather loop with a token signal of Sec. 4.3 ranked per KV head.
+
+    ``kv_inputs(c)`` -> (k_new, v_new) [Lf,Hkv,C,D]; ``signal`` is ``key_norm`` (-||k||) or
+    ``value_norm`` (||v||); each appended token gets its score once, from its own row (the score
+    depends on nothing else, so it equals a score recomputed from the cache at eviction time).
+    ``score_override(c)`` (optional) -> [Lf,Hkv,C] float32 scores to rank chunk c's tokens with
+    instead of the oracle's own (selection compared given identical scores).  The recurrent state
+    is not involved: run :func:`run_stream` or the recurrence for it."""
+    kc = vc = None
+    T = pos = 0
+    res = HeadStreamResult(None, None, None, None, None, 0)
+    for c in range(n_chunks):
+        k_new, v_new = kv_inputs(c)
+        Lf, Hkv, C, D = k_new.shape
+        if kc is None:
+            kc = np.zeros((Lf, Hkv, capacity, D), dtype=k_new.dtype)
+            vc = np.zeros_like(kc)
+            tok_chunk = np.zeros((Lf, Hkv, capacity), np.int32)
+            tok_pos = np.zeros((Lf, Hkv, capacity), np.int32)
+            tok_score = np.zeros((Lf, Hkv, capacity), np.float32)
+        if T + C > capacity:
+            raise ValueError("cache capacity too small for the stream")
+        kc[:, :, T:T + C] = k_new
+        vc[:, :, T:T + C] = v_new
+        tok_chunk[:, :, T:T + C] = c
+        tok_pos[:, :, T:T + C] = np.arange(pos, pos + C, dtype=np.int32)
+        if score_override is not None:
+            tok_score[:, :, T:T + C] = np.asarray(score_override(c), np.float32)
+        else:
+            rows = k_new if signal == "key_norm" else v_new
+            if rows.dtype == np.int16:                       # bf16 bit patterns -> float32, exactly
+                rows = (rows.astype(np.int32) << 16).view(np.float32)
+            tok_score[:, :, T:T + C] = row_norm_scores(rows, signal)
+        T += C
+        pos += C
+        if T > policy["budget_M"]:
+            lists = [select_retain_tokens(policy["budget_M"], policy["n_sink"], policy["n_window"],
+                                          policy["n_buckets"], tok_chunk[l, h, :T], tok_score[l, h, :T])[0]
+                     for l in range(Lf) for h in range(Hkv)]
+            kc, vc, tok_chunk, tok_pos, tok_score = compact_kv_heads(kc, vc, tok_chunk, tok_pos, tok_score,
+                                                                     lists, T)
+            T = int(lists[0].shape[0])
+            res.evictions.append((c, lists))
+    res.k_cache, res.v_cache = kc, vc
+    res.tok_chunk, res.tok_pos, res.tok_score = tok_chunk, tok_pos, tok_score
     res.cache_len = T
     return res

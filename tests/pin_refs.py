@@ -12,6 +12,9 @@
   M - n_s - n_w that give every span at least min(quota, |span|) members, the one with the largest
   sum of 2^rank (rank in the score order).  Quota-then-fill is the greedy algorithm on this
   (matroid) constraint family, so with strictly ordered keys the two coincide.
+
+Both selection references take ``per_slot=True`` for the token signals of Sec. 4.3: ``scores``
+then holds one score per slot instead of one per chunk.
 """
 from __future__ import annotations
 
@@ -64,8 +67,13 @@ def _spans(tok_chunk, lo, hi, N):
     return ((a - c_lo) * N) // (c_hi - c_lo + 1)
 
 
-def select_by_global_sort(M, n_s, n_w, N, tok_chunk, scores):
+def _slot_score(tok_chunk, scores, per_slot):
+    return (lambda i: scores[i]) if per_slot else (lambda i: scores[tok_chunk[i]])
+
+
+def select_by_global_sort(M, n_s, n_w, N, tok_chunk, scores, per_slot=False):
     tok_chunk = np.asarray(tok_chunk)
+    score_of = _slot_score(tok_chunk, scores, per_slot)
     T = len(tok_chunk)
     if T <= M:
         return list(range(T))
@@ -74,7 +82,7 @@ def select_by_global_sort(M, n_s, n_w, N, tok_chunk, scores):
     R = M - n_s - n_w
     quota = R // N
     spans = _spans(tok_chunk, lo, hi, N)
-    order = sorted(range(lo, hi), key=lambda i: (-_score_key(scores[tok_chunk[i]]), i))
+    order = sorted(range(lo, hi), key=lambda i: (-_score_key(score_of(i)), i))
     keep = set(range(n_s)) | set(range(hi, T))
     used = [0] * N
     for i in order:
@@ -92,8 +100,9 @@ def select_by_global_sort(M, n_s, n_w, N, tok_chunk, scores):
     return sorted(keep)
 
 
-def select_by_max_weight(M, n_s, n_w, N, tok_chunk, scores):
+def select_by_max_weight(M, n_s, n_w, N, tok_chunk, scores, per_slot=False):
     tok_chunk = np.asarray(tok_chunk)
+    score_of = _slot_score(tok_chunk, scores, per_slot)
     T = len(tok_chunk)
     if T <= M:
         return list(range(T))
@@ -103,7 +112,7 @@ def select_by_max_weight(M, n_s, n_w, N, tok_chunk, scores):
     quota = R // N
     spans = _spans(tok_chunk, lo, hi, N)
     cand = list(range(lo, hi))
-    order = sorted(cand, key=lambda i: (_score_key(scores[tok_chunk[i]]), -i))  # worst first
+    order = sorted(cand, key=lambda i: (_score_key(score_of(i)), -i))  # worst first
     weight = {i: 1 << r for r, i in enumerate(order)}
     need = [min(quota, int(np.sum(spans == j))) for j in range(N)]
     best, best_w = None, -1

@@ -11,7 +11,7 @@ import numpy as np
 import pytest
 
 import oracle
-from oracle.stream import run_stream
+from oracle.stream import run_stream, run_stream_heads
 from pin_refs import gdn_chunked_wy, select_by_global_sort, select_by_max_weight
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
@@ -497,3 +497,170 @@ def test_question_turn_leaves_stream_unchanged():
     for (c1, i1), (c2, i2) in zip(asked.evictions, plain.evictions):
         assert c1 == c2
         np.testing.assert_array_equal(i1, i2)
+
+
+
+# ---------------------------------------------------------------- token signals (Sec. 4.3)
+
+def test_row_norm_scores_are_signed_l2_norms():
+    """Key norm scores -||k||_2, value norm ||v||_2 (the appendix's table of signals): equal to
+    numpy.linalg.norm on random rows (bf16-rounded values included), sqrt(D) for a row of ones,
+    |x| for a one-hot row, and |lambda| times the score for a scaled row."""
+    rng = np.random.default_rng(71)
+    rows = rng.standard_normal((3, 5, 256)).astype(np.float32)
+    bf = ((rows.view(np.uint32) + 0x8000) & 0xFFFF0000).view(np.float32)      # bf16 values
+    for r in (rows, bf):
+        ref = np.linalg.norm(r.astype(np.float64), axis=-1)
+        np.testing.assert_allclose(oracle.row_norm_scores(r, "value_norm"), ref, rtol=1e-7)
+        np.testing.assert_allclose(oracle.row_norm_scores(r, "key_norm"), -ref, rtol=1e-7)
+    assert oracle.row_norm_scores(np.ones((1, 256), np.float32), "value_norm")[0] == 16.0
+    hot = np.zeros((1, 16), np.float32)
+    hot[0, 5] = -3.5
+    assert oracle.row_norm_scores(hot, "key_norm")[0] == -3.5
+    assert oracle.row_norm_scores(hot, "value_norm")[0] == 3.5
+    np.testing.assert_allclose(oracle.row_norm_scores(4.0 * rows, "value_norm"),
+                               4.0 * oracle.row_norm_scores(rows, "value_norm"), rtol=1e-7)
+    with pytest.raises(ValueError):
+        oracle.row_norm_scores(rows, "attention")
+
+
+def _random_token_case(rng, T_max, ties=True):
+    M, n_s, n_w, N, tc, _ = _random_case(rng, T_max, ties=False)
+    sc = rng.standard_normal(len(tc)).astype(np.float32)
+    if ties and len(tc) > 3:
+        sc[rng.integers(0, len(tc), size=3)] = sc[0]
+    return M, n_s, n_w, N, tc, sc
+
+
+def test_select_tokens_equals_chunk_selection_on_shared_scores():
+    """With every token carrying its chunk's score, the token-level selection is the Sec. 3.3
+    chunk selection (pinned above)."""
+    rng = np.random.default_rng(72)
+    for _ in range(300):
+        n_ch = int(rng.integers(2, 40))
+        tc = np.repeat(np.arange(n_ch, dtype=np.int32), rng.integers(1, 25, size=n_ch))
+        sc = rng.exponential(size=n_ch).astype(np.float32)
+        sc[rng.integers(0, n_ch, size=4)] = sc[0]
+        T = len(tc)
+        n_s, n_w = int(rng.integers(0, 5)), int(rng.integers(0, 30))
+        M = int(rng.integers(n_s + n_w + 1, max(T, n_s + n_w + 1) + 5))
+        N = int(rng.integers(0, 7))
+        a = oracle.select_retain(M, n_s, n_w, N, tc, sc)
+        b = oracle.select_retain_tokens(M, n_s, n_w, N, tc, sc[tc])
+        np.testing.assert_array_equal(a[0], b[0])
+        np.testing.assert_array_equal(a[1], b[1])
+
+
+def test_select_tokens_matches_exhaustive_max_weight():
+    """Per-token scores: quota-then-fill == the max-weight subset under the span lower bounds
+    (exhaustive over all subsets, T <= 12)."""
+    rng = np.random.default_rng(73)
+    n = 0
+    while n < 300:
+        M, n_s, n_w, N, tc, sc = _random_token_case(rng, 12)
+        if len(tc) <= M:
+            continue
+        idx, _ = oracle.select_retain_tokens(M, n_s, n_w, N, tc, sc)
+        assert idx.tolist() == select_by_max_weight(M, n_s, n_w, N, tc, sc, per_slot=True)
+        n += 1
+
+
+def test_select_tokens_matches_global_sort_implementation():
+    rng = np.random.default_rng(74)
+    for _ in range(200):
+        n_ch = int(rng.integers(2, 60))
+        tc = np.repeat(np.arange(n_ch, dtype=np.int32), rng.integers(1, 40, size=n_ch))
+        T = len(tc)
+        sc = np.round(rng.standard_normal(T), 2).astype(np.float32)             # many exact ties
+        sc[rng.integers(0, T, size=3)] = -0.0
+        n_s, n_w = int(rng.integers(0, 5)), int(rng.integers(0, 50))
+        M = int(rng.integers(n_s + n_w + 1, max(T, n_s + n_w + 1) + 5))
+        N = int(rng.integers(0, 9))
+        idx, _ = oracle.select_retain_tokens(M, n_s, n_w, N, tc, sc)
+        assert idx.tolist() == select_by_global_sort(M, n_s, n_w, N, tc, sc, per_slot=True)
+
+
+def test_select_tokens_single_span_is_stable_top_m():
+    """N = 1, no sink or window: the M best tokens by score, earlier slot first on ties
+    (numpy's stable argsort as the reference)."""
+    rng = np.random.default_rng(75)
+    for _ in range(50):
+        T = int(rng.integers(2, 300))
+        tc = np.sort(rng.integers(0, 20, size=T)).astype(np.int32)
+        sc = np.round(rng.standard_normal(T), 1).astype(np.float32)
+        M = int(rng.integers(1, T + 3))
+        idx, _ = oracle.select_retain_tokens(M, 0, 0, 1, tc, sc)
+        order = np.argsort(-sc.astype(np.float64), kind="stable")
+        assert idx.tolist() == sorted(order[:M].tolist())
+
+
+def test_select_tokens_invariants():
+    """Budget, sink and window, stream order, per-span minimum, and inside every span the kept
+    candidates are the best ones of that span (quota and fill both take from the top)."""
+    rng = np.random.default_rng(76)
+    for _ in range(200):
+        n_ch = int(rng.integers(2, 40))
+        tc = np.repeat(np.arange(n_ch, dtype=np.int32), rng.integers(1, 30, size=n_ch))
+        T = len(tc)
+        sc = rng.standard_normal(T).astype(np.float32)
+        n_s, n_w = int(rng.integers(0, 6)), int(rng.integers(0, 40))
+        M = int(rng.integers(n_s + n_w + 1, max(T, n_s + n_w + 1) + 5))
+        N = int(rng.integers(1, 7))
+        idx, mask = oracle.select_retain_tokens(M, n_s, n_w, N, tc, sc)
+        assert len(idx) == min(T, M) and np.all(np.diff(idx) > 0)
+        if T <= M:
+            continue
+        assert np.all(mask[:n_s] == 1) and np.all(mask[T - n_w:] == 1)
+        lo, hi = n_s, T - n_w
+        a = tc[lo:hi].astype(np.int64)
+        span = ((a - a.min()) * N) // (a.max() - a.min() + 1)
+        q = (M - n_s - n_w) // N
+        for j in range(N):
+            members = np.nonzero(span == j)[0] + lo
+            kept = members[mask[members] == 1]
+            dropped = members[mask[members] == 0]
+            assert len(kept) >= min(q, len(members))
+            if len(kept) and len(dropped):
+                assert sc[kept].min() >= sc[dropped].max()
+
+
+def test_compact_heads_gathers_each_plane_by_its_own_list():
+    """Per-head gather: plane p of K, V and of the per-head metadata equals numpy.take by list p;
+    rows past the kept length are untouched."""
+    rng = np.random.default_rng(77)
+    Lf, Hkv, cap, D, T, n = 2, 3, 40, 8, 33, 20
+    kc = rng.standard_normal((Lf, Hkv, cap, D)).astype(np.float32)
+    vc = rng.standard_normal((Lf, Hkv, cap, D)).astype(np.float32)
+    tc = rng.integers(0, 9, size=(Lf, Hkv, cap)).astype(np.int32)
+    tp = rng.integers(0, 999, size=(Lf, Hkv, cap)).astype(np.int32)
+    ts = rng.standard_normal((Lf, Hkv, cap)).astype(np.float32)
+    lists = [np.sort(rng.choice(T, size=n, replace=False)).astype(np.int32) for _ in range(Lf * Hkv)]
+    out = oracle.compact_kv_heads(kc, vc, tc, tp, ts, lists, T)
+    for arr, o in zip((kc, vc, tc, tp, ts), out):
+        for p in range(Lf * Hkv):
+            l, h = divmod(p, Hkv)
+            np.testing.assert_array_equal(o[l, h, :n], np.take(arr[l, h], lists[p], axis=0))
+            np.testing.assert_array_equal(o[l, h, n:], arr[l, h, n:])
+
+
+@pytest.mark.parametrize("signal", ["key_norm", "value_norm"])
+def test_stream_heads_invariants_tiny(signal):
+    """The per-head loop: every plane keeps M tokens with sinks and window, in stream order; the
+    stored score of every kept token equals its signal recomputed from the cache row it now sits
+    in (the score is a function of the row alone); planes disagree on what they keep."""
+    rng = np.random.default_rng(78)
+    Lf, Hkv, C, D, n_ch = 1, 2, 64, 16, 8
+    kvs = [(rng.standard_normal((Lf, Hkv, C, D)).astype(np.float32),
+            rng.standard_normal((Lf, Hkv, C, D)).astype(np.float32)) for _ in range(n_ch)]
+    policy = dict(budget_M=256, n_sink=4, n_window=64, n_buckets=2)
+    res = run_stream_heads(lambda c: kvs[c], n_ch, policy, capacity=256 + C, signal=signal)
+    n = res.cache_len
+    assert n == 256 and len(res.evictions) == n_ch - 4
+    rows = res.k_cache if signal == "key_norm" else res.v_cache
+    np.testing.assert_array_equal(res.tok_score[:, :, :n], oracle.row_norm_scores(rows[:, :, :n], signal))
+    for h in range(Hkv):
+        pos = res.tok_pos[0, h, :n]
+        assert np.all(np.diff(pos) > 0) and pos[:4].tolist() == [0, 1, 2, 3]
+        assert pos[-64:].tolist() == list(range(n_ch * C - 64, n_ch * C))
+        np.testing.assert_array_equal(res.tok_chunk[0, h, :n], pos // C)
+    assert not np.array_equal(res.tok_pos[0, 0, :n], res.tok_pos[0, 1, :n])
