@@ -12,6 +12,8 @@
  *   deltas_select_retain     sink / window / temporal spans / quota + fill (Sec. 3.3, Alg. 1)
  *   deltas_compact_kv        in-place, stream-order gather of the KV caches (Alg. 1, Sec. 3.3)
  *   deltas_append_kv         append a chunk's keys/values to the caches (Alg. 1 Prefill)
+ *   deltas_*_heads           the same append / select / compact with a cache-internal token
+ *                            signal (key norm, value norm; Sec. 4.3) ranked per KV head
  *
  * Conventions shared by every call
  * --------------------------------
@@ -309,6 +311,68 @@ DELTAS_API deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, co
                                        int32_t cache_len, int32_t n_chunks,
                                        const deltas_stream_buffers* src,
                                        const deltas_stream_buffers* dst, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Per-head token signals (Sec. 4.3, the controlled comparison of retention signals, and the   */
+/* appendix table of signals).  Instead of one score per chunk, every cached token of every     */
+/* (layer, KV head) plane carries its own score, read from the cache rows themselves:           */
+/*   DELTAS_SIGNAL_KEY_NORM    score = -||k||_2 of the token's key row   (key-norm signal)      */
+/*   DELTAS_SIGNAL_VALUE_NORM  score = +||v||_2 of the token's value row (value-norm signal)    */
+/* Each plane is ranked on its own under the policy of deltas_select_retain, so every plane     */
+/* keeps its own min(cache_len, M) tokens; the per-slot metadata is therefore per plane:        */
+/*   tok_chunk, tok_pos [Lf][Hkv][capacity] int32    tok_score [Lf][Hkv][capacity] float       */
+/* (plane p = layer * Hkv + head).  All planes hold the same number of tokens, cache_len.       */
+/* ------------------------------------------------------------------------------------------ */
+typedef enum deltas_signal_e {
+    DELTAS_SIGNAL_KEY_NORM = 1,
+    DELTAS_SIGNAL_VALUE_NORM = 2
+} deltas_signal;
+
+/* Append one chunk and score its tokens: as deltas_append_kv, and in every plane p the new     */
+/* slots get tok_chunk[p][.] = chunk_id, tok_pos[p][.] = first_pos, first_pos + 1, ... and      */
+/* tok_score[p][.] = the signal of the row just stored (squares summed in float32 from the      */
+/* stored values, then a correctly rounded square root).  A token's score depends on its row    */
+/* alone, so it is computed once, here, and moved with the row by deltas_compact_kv_heads; it   */
+/* equals the score recomputed from the cache at eviction time.                                 */
+/* Errors: those of deltas_append_kv; INVALID_ARGUMENT for an unknown signal or a NULL          */
+/* tok_score.                                                                                   */
+DELTAS_API deltas_status deltas_append_kv_heads(const deltas_kv_desc* desc, int32_t signal,
+                                     void* k_cache, void* v_cache, int32_t* tok_chunk,
+                                     int32_t* tok_pos, float* tok_score, int32_t cache_len,
+                                     const void* k_new, const void* v_new, int32_t n_new,
+                                     int32_t chunk_id, int32_t first_pos, void* stream);
+
+/* Per-plane retain selection: for each of the num_planes planes, the rule of                   */
+/* deltas_select_retain with the slot's own score tok_score[p][i] in place of its chunk's      */
+/* (spans still split the candidates' arrival chunks tok_chunk[p][.], computed per plane).      */
+/*   tok_chunk, tok_score  [num_planes][plane_stride], slots 0 .. cache_len - 1 read             */
+/*   retain_idx  [num_planes][M] int32  out: row p = the kept slots of plane p, ascending        */
+/*   n_retained  [1] int32 (device)     out: min(cache_len, M), the same for every plane        */
+/*   mask        [num_planes][plane_stride] uint8  out: 1 = kept; NULL to skip                   */
+/* One CTA ranks one plane (a radix select on the score's total-order bits, then on the slot    */
+/* for ties); the plane's keys sit in shared memory when they fit, else in the workspace.       */
+/* A negative tok_chunk value is reported as DEVICE_INDEX.  cache_len above                     */
+/* DELTAS_SELECT_MAX_CACHE_LEN or plane_stride < cache_len: UNSUPPORTED / INVALID_ARGUMENT.     */
+DELTAS_API size_t deltas_select_retain_heads_workspace_size(int32_t num_planes, int32_t cache_len);
+
+DELTAS_API deltas_status deltas_select_retain_heads(const deltas_policy* policy, int32_t num_planes,
+                                         int32_t cache_len, int32_t plane_stride,
+                                         const int32_t* tok_chunk, const float* tok_score,
+                                         int32_t* retain_idx, int32_t* n_retained, uint8_t* mask,
+                                         void* workspace, size_t workspace_bytes, void* stream);
+
+/* Per-plane in-place compaction: as deltas_compact_kv, except that plane p of k_cache and      */
+/* v_cache and row p of tok_chunk, tok_pos and tok_score ([Lf][Hkv][capacity]) are gathered by */
+/* their own list, row p of retain_idx ([Lf * Hkv][list_stride], list_stride >= *n_retained).   */
+/* Every list must be strictly ascending with j <= retain_idx[p][j] < cache_len; otherwise      */
+/* nothing is moved and DEVICE_INDEX is recorded.                                               */
+DELTAS_API size_t deltas_compact_kv_heads_workspace_size(const deltas_kv_desc* desc, int32_t cache_len);
+
+DELTAS_API deltas_status deltas_compact_kv_heads(const deltas_kv_desc* desc, void* k_cache, void* v_cache,
+                                      int32_t* tok_chunk, int32_t* tok_pos, float* tok_score,
+                                      const int32_t* retain_idx, int32_t list_stride,
+                                      const int32_t* n_retained, int32_t cache_len,
+                                      void* workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------------------------ */
 /* Device status word (first 16 bytes of a workspace).                                          */

@@ -38,6 +38,8 @@ EXPORTED = (
     "deltas_select_retain_workspace_size", "deltas_select_retain", "deltas_select_retain_static",
     "deltas_compact_kv_workspace_size", "deltas_compact_kv",
     "deltas_append_kv", "deltas_copy_stream_state",
+    "deltas_append_kv_heads", "deltas_select_retain_heads_workspace_size", "deltas_select_retain_heads",
+    "deltas_compact_kv_heads_workspace_size", "deltas_compact_kv_heads",
     "deltas_clear_device_status", "deltas_get_device_status",
 )
 
@@ -92,6 +94,11 @@ _sig("deltas_compact_kv_workspace_size", _SZ, _P, _I32)
 _sig("deltas_compact_kv", ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, _I32, _P, _SZ, _P)
 _sig("deltas_append_kv", ctypes.c_int, _P, _P, _P, _P, _P, _I32, _P, _P, _I32, _I32, _I32, _P)
 _sig("deltas_copy_stream_state", ctypes.c_int, _P, _P, _I32, _I32, _P, _P, _P)
+_sig("deltas_append_kv_heads", ctypes.c_int, _P, _I32, _P, _P, _P, _P, _P, _I32, _P, _P, _I32, _I32, _I32, _P)
+_sig("deltas_select_retain_heads_workspace_size", _SZ, _I32, _I32)
+_sig("deltas_select_retain_heads", ctypes.c_int, _P, _I32, _I32, _I32, _P, _P, _P, _P, _P, _P, _SZ, _P)
+_sig("deltas_compact_kv_heads_workspace_size", _SZ, _P, _I32)
+_sig("deltas_compact_kv_heads", ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, _I32, _P, _I32, _P, _SZ, _P)
 _sig("deltas_clear_device_status", ctypes.c_int, _P, _P)
 _sig("deltas_get_device_status", ctypes.c_int, _P, _P, _P, _P)
 
@@ -293,6 +300,80 @@ def deltas_append_kv(desc: KvDesc, k_cache, v_cache, tok_chunk, tok_pos, cache_l
                                _ptr(k_new, dt, nshp, "k_new"), _ptr(v_new, dt, nshp, "v_new"), n_new,
                                int(chunk_id), int(first_pos), _stream(stream))
     _check(st, "deltas_append_kv")
+
+
+# Per-head token signals (Sec. 4.3): the key norm scores -||k||, the value norm ||v||
+DELTAS_SIGNAL_KEY_NORM = 1
+DELTAS_SIGNAL_VALUE_NORM = 2
+SIGNALS = {"key_norm": DELTAS_SIGNAL_KEY_NORM, "value_norm": DELTAS_SIGNAL_VALUE_NORM}
+
+
+def deltas_append_kv_heads(desc: KvDesc, signal: str, k_cache, v_cache, tok_chunk, tok_pos, tok_score,
+                           cache_len: int, k_new, v_new, chunk_id: int, first_pos: int, stream=None):
+    """Append a chunk and score its tokens per (layer, KV head); metadata is [Lf, Hkv, capacity]."""
+    dt = _TORCH_DT[desc.dtype]
+    shp = (desc.num_layers, desc.num_kv_heads, desc.capacity, desc.head_dim)
+    mshp = shp[:3]
+    n_new = int(k_new.shape[2])
+    nshp = (desc.num_layers, desc.num_kv_heads, n_new, desc.head_dim)
+    st = _lib.deltas_append_kv_heads(ctypes.byref(desc), SIGNALS[signal], _ptr(k_cache, dt, shp, "k_cache"),
+                                     _ptr(v_cache, dt, shp, "v_cache"), _ptr(tok_chunk, torch.int32, mshp, "tok_chunk"),
+                                     _ptr(tok_pos, torch.int32, mshp, "tok_pos"),
+                                     _ptr(tok_score, torch.float32, mshp, "tok_score"), int(cache_len),
+                                     _ptr(k_new, dt, nshp, "k_new"), _ptr(v_new, dt, nshp, "v_new"), n_new,
+                                     int(chunk_id), int(first_pos), _stream(stream))
+    _check(st, "deltas_append_kv_heads")
+
+
+def deltas_select_retain_heads_workspace_size(num_planes: int, cache_len: int) -> int:
+    return int(_lib.deltas_select_retain_heads_workspace_size(int(num_planes), int(cache_len)))
+
+
+def deltas_select_retain_heads(pol: Policy, cache_len: int, tok_chunk, tok_score, retain_idx, n_retained, mask,
+                               workspace, stream=None):
+    """Per-plane selection: tok_chunk / tok_score [..., plane_stride] (planes flattened), retain_idx
+    [planes, M], mask [planes, plane_stride] or None."""
+    T = int(cache_len)
+    stride = int(tok_chunk.shape[-1])
+    planes = tok_chunk.numel() // max(stride, 1)
+    if tok_score.shape != tok_chunk.shape or stride < T:
+        raise ValueError("select_retain_heads: tok_score must match tok_chunk, with at least cache_len slots")
+    if retain_idx.numel() < planes * pol.budget_M or (mask is not None and tuple(mask.shape) != tuple(tok_chunk.shape)):
+        raise ValueError("select_retain_heads: retain_idx needs [planes, M], mask the shape of tok_chunk")
+    st = _lib.deltas_select_retain_heads(ctypes.byref(pol), planes, T, stride,
+                                         _ptr(tok_chunk, torch.int32, None, "tok_chunk"),
+                                         _ptr(tok_score, torch.float32, None, "tok_score"),
+                                         _ptr(retain_idx, torch.int32, None, "retain_idx"),
+                                         _ptr(n_retained, torch.int32, None, "n_retained"),
+                                         _ptr(mask, torch.uint8, None, "mask"),
+                                         _ptr(workspace, torch.uint8, None, "workspace"), workspace.numel(),
+                                         _stream(stream))
+    _check(st, "deltas_select_retain_heads")
+
+
+def deltas_compact_kv_heads_workspace_size(desc: KvDesc, cache_len: int) -> int:
+    return int(_lib.deltas_compact_kv_heads_workspace_size(ctypes.byref(desc), int(cache_len)))
+
+
+def deltas_compact_kv_heads(desc: KvDesc, k_cache, v_cache, tok_chunk, tok_pos, tok_score, retain_idx, n_retained,
+                            cache_len: int, workspace, stream=None):
+    """Gather every (layer, KV head) plane by its own row of retain_idx [Lf * Hkv, list_stride]."""
+    dt = _TORCH_DT[desc.dtype]
+    shp = (desc.num_layers, desc.num_kv_heads, desc.capacity, desc.head_dim)
+    mshp = shp[:3]
+    planes = desc.num_layers * desc.num_kv_heads
+    if retain_idx.dim() != 2 or retain_idx.shape[0] != planes:
+        raise ValueError("compact_kv_heads: retain_idx must be [Lf * Hkv, list_stride]")
+    st = _lib.deltas_compact_kv_heads(ctypes.byref(desc), _ptr(k_cache, dt, shp, "k_cache"),
+                                      _ptr(v_cache, dt, shp, "v_cache"),
+                                      _ptr(tok_chunk, torch.int32, mshp, "tok_chunk"),
+                                      _ptr(tok_pos, torch.int32, mshp, "tok_pos"),
+                                      _ptr(tok_score, torch.float32, mshp, "tok_score"),
+                                      _ptr(retain_idx, torch.int32, None, "retain_idx"), int(retain_idx.shape[1]),
+                                      _ptr(n_retained, torch.int32, None, "n_retained"), int(cache_len),
+                                      _ptr(workspace, torch.uint8, None, "workspace"), workspace.numel(),
+                                      _stream(stream))
+    _check(st, "deltas_compact_kv_heads")
 
 
 STREAM_BUFFERS = ("state", "chunk_scores", "k_cache", "v_cache", "tok_chunk", "tok_pos")

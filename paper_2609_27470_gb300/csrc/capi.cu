@@ -257,6 +257,79 @@ deltas_status deltas_append_kv(const deltas_kv_desc* desc, void* k_cache, void* 
                                       as_stream(stream)));
 }
 
+deltas_status deltas_append_kv_heads(const deltas_kv_desc* desc, int32_t signal, void* k_cache, void* v_cache,
+                                     int32_t* tok_chunk, int32_t* tok_pos, float* tok_score, int32_t cache_len,
+                                     const void* k_new, const void* v_new, int32_t n_new, int32_t chunk_id,
+                                     int32_t first_pos, void* stream)
+{
+    deltas_status st = check_kv_desc(desc);
+    if (st != DELTAS_OK) return st;
+    if (signal != DELTAS_SIGNAL_KEY_NORM && signal != DELTAS_SIGNAL_VALUE_NORM) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (cache_len < 0 || n_new < 0 || (long long)cache_len + n_new > desc->capacity) return DELTAS_ERR_INVALID_ARGUMENT;
+    if ((long long)first_pos + n_new > INT32_MAX || first_pos < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!k_cache || !v_cache || !tok_chunk || !tok_pos || !tok_score) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (n_new > 0 && (!k_new || !v_new || !aligned16(k_new) || !aligned16(v_new))) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!aligned16(k_cache) || !aligned16(v_cache)) return DELTAS_ERR_INVALID_ARGUMENT;
+    KvPlanes kv = make_planes(desc, k_cache, v_cache, tok_chunk, tok_pos);
+    kv.tok_score = tok_score;
+    return from_cuda(launch_append_kv_heads(kv, signal, cache_len, k_new, v_new, n_new, chunk_id, first_pos,
+                                            as_stream(stream)));
+}
+
+size_t deltas_select_retain_heads_workspace_size(int32_t num_planes, int32_t cache_len) {
+    if (num_planes < 0 || cache_len < 0) return 0;
+    return select_heads_workspace_bytes(num_planes, cache_len);
+}
+
+deltas_status deltas_select_retain_heads(const deltas_policy* policy, int32_t num_planes, int32_t cache_len,
+                                         int32_t plane_stride, const int32_t* tok_chunk, const float* tok_score,
+                                         int32_t* retain_idx, int32_t* n_retained, uint8_t* mask,
+                                         void* workspace, size_t workspace_bytes, void* stream)
+{
+    if (policy == nullptr || num_planes < 1 || cache_len < 0 || plane_stride < cache_len)
+        return DELTAS_ERR_INVALID_ARGUMENT;
+    const deltas_policy& p = *policy;
+    if (p.budget_M < 1 || p.n_sink < 0 || p.n_window < 0 || p.n_buckets < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if ((long long)p.budget_M < (long long)p.n_sink + p.n_window + 1) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (p.n_buckets > 32) return DELTAS_ERR_UNSUPPORTED;
+    if (cache_len > DELTAS_SELECT_MAX_CACHE_LEN || num_planes > 65535) return DELTAS_ERR_UNSUPPORTED;
+    if (!retain_idx || !n_retained) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (cache_len > 0 && (!tok_chunk || !tok_score)) return DELTAS_ERR_INVALID_ARGUMENT;
+    deltas_status st = check_workspace(workspace, workspace_bytes,
+                                       deltas_select_retain_heads_workspace_size(num_planes, cache_len));
+    if (st != DELTAS_OK) return st;
+    return from_cuda(launch_select_heads(p, num_planes, cache_len, plane_stride, tok_chunk, tok_score, retain_idx,
+                                         n_retained, mask, workspace, static_cast<int32_t*>(workspace),
+                                         as_stream(stream)));
+}
+
+size_t deltas_compact_kv_heads_workspace_size(const deltas_kv_desc* desc, int32_t cache_len) {
+    if (check_kv_desc(desc) != DELTAS_OK || cache_len < 0) return 0;
+    KvPlanes kv = make_planes(desc, nullptr, nullptr, nullptr, nullptr);
+    return compact_heads_workspace_bytes(kv, cache_len);
+}
+
+deltas_status deltas_compact_kv_heads(const deltas_kv_desc* desc, void* k_cache, void* v_cache,
+                                      int32_t* tok_chunk, int32_t* tok_pos, float* tok_score,
+                                      const int32_t* retain_idx, int32_t list_stride,
+                                      const int32_t* n_retained, int32_t cache_len,
+                                      void* workspace, size_t workspace_bytes, void* stream)
+{
+    deltas_status st = check_kv_desc(desc);
+    if (st != DELTAS_OK) return st;
+    if (cache_len < 0 || cache_len > desc->capacity || list_stride < 0) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!k_cache || !v_cache || !tok_chunk || !tok_pos || !tok_score || !retain_idx || !n_retained)
+        return DELTAS_ERR_INVALID_ARGUMENT;
+    if (!aligned16(k_cache) || !aligned16(v_cache)) return DELTAS_ERR_INVALID_ARGUMENT;
+    if (desc->num_layers * desc->num_kv_heads > 1 && list_stride < 1) return DELTAS_ERR_INVALID_ARGUMENT;
+    st = check_workspace(workspace, workspace_bytes, deltas_compact_kv_heads_workspace_size(desc, cache_len));
+    if (st != DELTAS_OK) return st;
+    KvPlanes kv = make_planes(desc, k_cache, v_cache, tok_chunk, tok_pos);
+    kv.tok_score = tok_score;
+    return from_cuda(launch_compact_kv_heads(kv, retain_idx, list_stride, n_retained, cache_len, workspace,
+                                             static_cast<int32_t*>(workspace), as_stream(stream)));
+}
+
 deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, const deltas_kv_desc* kv,
                                        int32_t cache_len, int32_t n_chunks,
                                        const deltas_stream_buffers* src,

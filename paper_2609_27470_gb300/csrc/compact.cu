@@ -1,6 +1,8 @@
 // In-place, stream-order KV compaction (Alg. 1 "KV <- KV[I_sink u I_DeltaS u I_window]",
 // applied to every full-attention layer; Sec. 3.3: survivors keep their original positions) and
-// the per-chunk append to the caches (Alg. 1 Prefill).
+// the per-chunk append to the caches (Alg. 1 Prefill).  With a token signal ranked per KV head
+// (Sec. 4.3) every (layer, head) plane has its own retain list and its own metadata rows; the
+// same kernels then gather each plane by its list (one `need` table and first row per list).
 //
 // The gather row[j] <- row[retain_idx[j]] runs in place.  Because retain_idx is ascending with
 // retain_idx[j] >= j, the only hazard is a destination row that is still to be read as the
@@ -20,6 +22,7 @@
 // Every wait is bounded (about one second); a wait that runs out records DELTAS_ERR_TIMEOUT,
 // raises the abort flag and skips its writes.  Traffic is the algorithmic minimum: each moved row
 // is read once and written once; rows that do not move are not touched.
+#include <algorithm>
 #include <climits>
 
 #include "internal.cuh"
@@ -35,52 +38,70 @@ constexpr int kStageBytes = 32768;   // staged source rows of one unit
 struct CompactCtl {
     unsigned ticket;
     int abort;
-    int first;             // first destination row that moves (INT_MAX: none)
+    int first_min;         // first destination row that moves, over all lists (INT_MAX: none)
 };
 
 struct CompactArgs {
     char* k_cache;
     char* v_cache;
-    char* tok_chunk;
-    char* tok_pos;
+    char* meta[3];         // 4-byte metadata arrays: tok_chunk, tok_pos, tok_score (per-head only)
     int n_kv_planes;       // Lf * Hkv planes in each of K and V
+    int n_lists;           // 1: one list moves every plane; n_kv_planes: one list per (layer, head)
+    int list_stride;       // elements between two lists of retain_idx
+    int n_meta;            // metadata arrays: 2 (shared list) or 3 (per head)
     int capacity;
     int row_bytes;         // D * element size (multiple of 16)
     int tile_rows;         // TB
-    int n_planes;          // 2 * n_kv_planes + 2 (metadata)
+    int n_planes;          // 2 * n_kv_planes + metadata rows (2, or 3 * n_kv_planes per head)
     int cache_len;
     int max_tiles;         // ceil(cache_len / TB)
     const int32_t* retain_idx;
     const int32_t* n_retained;
     CompactCtl* ctl;
-    int32_t* need;         // [max_tiles]
+    int32_t* first;        // [n_lists] first destination row that moves (INT_MAX: none)
+    int32_t* need;         // [n_lists][max_tiles]
     int32_t* flags;        // [n_planes][max_tiles]
     int32_t* status;
 };
 
 __host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-__device__ __forceinline__ char* plane_base(const CompactArgs& a, int p, int& rb) {
-    if (p < a.n_kv_planes) { rb = a.row_bytes; return a.k_cache + (size_t)p * a.capacity * a.row_bytes; }
+// Plane p of the unit order: K planes, V planes, then the metadata rows.  Returns its base, its
+// row size and the retain list that moves it.
+__device__ __forceinline__ char* plane_base(const CompactArgs& a, int p, int& rb, int& list) {
+    const bool shared_list = a.n_lists == 1;
+    if (p < a.n_kv_planes) {
+        rb = a.row_bytes; list = shared_list ? 0 : p;
+        return a.k_cache + (size_t)p * a.capacity * a.row_bytes;
+    }
     p -= a.n_kv_planes;
-    if (p < a.n_kv_planes) { rb = a.row_bytes; return a.v_cache + (size_t)p * a.capacity * a.row_bytes; }
+    if (p < a.n_kv_planes) {
+        rb = a.row_bytes; list = shared_list ? 0 : p;
+        return a.v_cache + (size_t)p * a.capacity * a.row_bytes;
+    }
+    p -= a.n_kv_planes;
     rb = 4;
-    return p == a.n_kv_planes ? a.tok_chunk : a.tok_pos;
+    const int per = shared_list ? 1 : a.n_kv_planes;             // rows of one metadata array
+    const int m = p / per;
+    list = p - m * per;
+    return a.meta[m] + (size_t)list * a.capacity * 4;
 }
 
 __global__ void compact_init_kernel(CompactArgs a) {
     grid_dep_launch();                                 // the prepass may be scheduled now
     const int total = a.n_planes * a.max_tiles;
-    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x)
-        a.flags[e] = 0;
-    if (blockIdx.x == 0 && threadIdx.x == 0) { a.ctl->ticket = 0; a.ctl->abort = 0; a.ctl->first = INT_MAX; }
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total + a.n_lists; e += gridDim.x * blockDim.x) {
+        if (e < total) a.flags[e] = 0;
+        else a.first[e - total] = INT_MAX;
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) { a.ctl->ticket = 0; a.ctl->abort = 0; a.ctl->first_min = INT_MAX; }
 }
 
-// Validates retain_idx and records, per source tile, the first destination tile that reads from
-// it (itself if none does), and the first destination row that moves.  retain_idx is ascending,
-// so the rows reading one source tile are consecutive: the first of them writes need[] for its
-// source tile and for the unread tiles before it, each tile exactly once.  Rows with
-// retain_idx[j] == j form a prefix (a moved row pushes every later source further on).
+// Validates every retain list and records, per list and source tile, the first destination tile
+// that reads from it (itself if none does), and the list's first destination row that moves.  A
+// list is ascending, so the rows reading one source tile are consecutive: the first of them
+// writes need[] for its source tile and for the unread tiles before it, each tile exactly once.
+// Rows with retain_idx[j] == j form a prefix (a moved row pushes every later source further on).
 __global__ void compact_need_kernel(CompactArgs a) {
     grid_dep_wait();                                   // the reset (and all earlier work) is done
     grid_dep_launch();
@@ -92,9 +113,14 @@ __global__ void compact_need_kernel(CompactArgs a) {
         }
         return;
     }
-    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < n; j += gridDim.x * blockDim.x) {
-        const int src = a.retain_idx[j];
-        const int prev = j > 0 ? a.retain_idx[j - 1] : -1;
+    const long long total = (long long)n * a.n_lists;
+    for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+         e += (long long)gridDim.x * blockDim.x) {
+        const int l = (int)(e / n), j = (int)(e - (long long)l * n);
+        const int32_t* ri = a.retain_idx + (size_t)l * a.list_stride;
+        int32_t* need = a.need + (size_t)l * a.max_tiles;
+        const int src = ri[j];
+        const int prev = j > 0 ? ri[j - 1] : -1;
         const bool ok = src >= j && src < a.cache_len && src > prev;
         if (!ok) {
             atomicExch(&a.ctl->abort, 1);
@@ -104,12 +130,15 @@ __global__ void compact_need_kernel(CompactArgs a) {
         const int ts = src / a.tile_rows, td = j / a.tile_rows;
         const int tp = prev < 0 ? -1 : prev / a.tile_rows;
         if (ts != tp) {
-            for (int t = tp + 1; t < ts; ++t) a.need[t] = t;        // unread tiles
-            a.need[ts] = td;
+            for (int t = tp + 1; t < ts; ++t) need[t] = t;          // unread tiles
+            need[ts] = td;
         }
         if (j == n - 1)
-            for (int t = ts + 1; t < a.max_tiles; ++t) a.need[t] = t;
-        if (src != j && prev == j - 1) a.ctl->first = j;           // unique: the first moved row
+            for (int t = ts + 1; t < a.max_tiles; ++t) need[t] = t;
+        if (src != j && prev == j - 1) {                           // unique: the list's first moved row
+            a.first[l] = j;
+            atomicMin(&a.ctl->first_min, j);
+        }
     }
 }
 
@@ -153,9 +182,9 @@ compact_main_kernel(CompactArgs a)
     volatile int* abort_flag = &a.ctl->abort;
     if (*abort_flag) return;
     const int n = *a.n_retained;
-    const int first = a.ctl->first;
-    if (first >= n) return;                                        // nothing moves
-    const int t0 = first / a.tile_rows;                            // tiles before t0 stay put
+    const int first_min = a.ctl->first_min;
+    if (first_min >= n) return;                                    // nothing moves
+    const int t0 = first_min / a.tile_rows;                        // tiles before t0 stay put
     const int n_tiles = (n + a.tile_rows - 1) / a.tile_rows;
     const int units = (n_tiles - t0) * a.n_planes;
     const int lane = threadIdx.x;
@@ -171,11 +200,13 @@ compact_main_kernel(CompactArgs a)
         u = __shfl_sync(0xffffffffu, u, 0);
         if (u >= units) break;
         const int b = t0 + u / a.n_planes, p = u % a.n_planes;
-        int rb;
-        char* base = plane_base(a, p, rb);
+        int rb, list;
+        char* base = plane_base(a, p, rb, list);
+        const int32_t* retain_idx = a.retain_idx + (size_t)list * a.list_stride;
         const int j0 = b * a.tile_rows;
         const int j_end = min(j0 + a.tile_rows, n);
-        const int js = max(j0, first);                             // rows before `first` stay
+        const int js = max(j0, a.first[list]);                     // rows before the list's first stay
+        if (js >= j_end) continue;                                 // (no unit ever waits for such a tile)
         const int nrows = j_end - js;
         const bool kv = rb >= 16;
 
@@ -190,7 +221,7 @@ compact_main_kernel(CompactArgs a)
             for (int c0 = js; c0 < j_end; c0 += 32) {
                 const int r = c0 + lane;
                 const bool in = r < j_end;
-                const int src = in ? a.retain_idx[r] : 0;
+                const int src = in ? retain_idx[r] : 0;
                 int prev = __shfl_up_sync(0xffffffffu, src, 1);
                 const bool start = in && (lane == 0 || src != prev + 1);
                 const unsigned starts = __ballot_sync(0xffffffffu, start);
@@ -208,7 +239,7 @@ compact_main_kernel(CompactArgs a)
             if (lane == 0 && store_pending) bulk_wait_read0();
             __syncwarp();
             int* st = reinterpret_cast<int*>(stage);
-            for (int r = js + lane; r < j_end; r += 32) st[r - j0] = reinterpret_cast<const int*>(base)[a.retain_idx[r]];
+            for (int r = js + lane; r < j_end; r += 32) st[r - j0] = reinterpret_cast<const int*>(base)[retain_idx[r]];
             __syncwarp();
         }
         if (!ok) {
@@ -222,7 +253,7 @@ compact_main_kernel(CompactArgs a)
             __threadfence();
             store_release(a.flags + (size_t)p * a.max_tiles + b, 1);
         }
-        const int first_reader = a.need[b];
+        const int first_reader = a.need[(size_t)list * a.max_tiles + b];
         const uint64_t t_start = global_ns();
         for (int bb = first_reader; bb < b && ok; bb += 32) {
             const int mine = bb + lane;
@@ -302,68 +333,132 @@ append_kv_kernel(char* k_cache, char* v_cache, int n_kv_planes, int capacity, in
     }
 }
 
+// Append with a token signal (Sec. 4.3: key norm -||k||, value norm ||v||, per KV head): one
+// warp per (plane, new row) copies the key and the value row into the caches (lane l moves the
+// 16-byte vectors l, l + 32, ...), sums the squares of the signal's row in float32 (each lane its
+// own elements, then a butterfly over the lanes), and writes the row's score -- a correctly
+// rounded square root, negated for keys -- with the plane's chunk id and position.
+constexpr int kAppendHeadsWarps = 8;
+
+__device__ __forceinline__ float sum_squares16(const uint4& v, bool bf16) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        if (bf16) {
+            const float lo = __uint_as_float(w[i] << 16), hi = __uint_as_float(w[i] & 0xffff0000u);
+            s = fmaf(lo, lo, s);
+            s = fmaf(hi, hi, s);
+        } else {
+            const float x = __uint_as_float(w[i]);
+            s = fmaf(x, x, s);
+        }
+    }
+    return s;
+}
+
+__global__ void __launch_bounds__(kAppendHeadsWarps * 32)
+append_kv_heads_kernel(char* k_cache, char* v_cache, int n_kv_planes, int capacity, int row_bytes, int bf16,
+                       int cache_len, const char* k_new, const char* v_new, int n_new, int32_t* tok_chunk,
+                       int32_t* tok_pos, float* tok_score, int key_signal, int chunk_id, int first_pos)
+{
+    const long long row = (long long)blockIdx.x * kAppendHeadsWarps + (threadIdx.x >> 5);
+    if (row >= (long long)n_kv_planes * n_new) return;
+    const int lane = threadIdx.x & 31;
+    const int p = (int)(row / n_new), i = (int)(row - (long long)p * n_new);
+    const size_t src = ((size_t)p * n_new + i) * row_bytes;
+    const size_t slot = (size_t)p * capacity + cache_len + i;
+    const uint4* ks = reinterpret_cast<const uint4*>(k_new + src);
+    const uint4* vs = reinterpret_cast<const uint4*>(v_new + src);
+    uint4* kd = reinterpret_cast<uint4*>(k_cache + slot * row_bytes);
+    uint4* vd = reinterpret_cast<uint4*>(v_cache + slot * row_bytes);
+    const int nv = row_bytes / 16;
+    float s = 0.f;
+    for (int e = lane; e < nv; e += 32) {
+        const uint4 kr = __ldcs(ks + e), vr = __ldcs(vs + e);
+        kd[e] = kr;
+        vd[e] = vr;
+        s += sum_squares16(key_signal ? kr : vr, bf16 != 0);
+    }
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) s += __shfl_xor_sync(0xffffffffu, s, m);
+    if (lane == 0) {
+        const float r = __fsqrt_rn(s);
+        tok_score[slot] = key_signal ? -r : r;
+        tok_chunk[slot] = chunk_id;
+        tok_pos[slot] = first_pos + i;
+    }
+}
+
 int tile_rows_for(int row_bytes) {
     int tb = kStageBytes / row_bytes;
     return tb < 1 ? 1 : (tb > 1024 ? 1024 : tb);
 }
 
 struct CompactWsLayout {
-    size_t ctl, need, flags, total;
+    size_t ctl, first, need, flags, total;
 };
 
-CompactWsLayout compact_layout(const KvPlanes& kv, int cache_len) {
+// per_head: one list per (layer, head) and three metadata arrays per plane.
+CompactWsLayout compact_layout(const KvPlanes& kv, int cache_len, bool per_head) {
     const int rb = kv.D * elt_bytes(kv.dtype);
     const int tb = tile_rows_for(rb);
     const size_t max_tiles = (size_t)((cache_len + tb - 1) / tb);
-    const size_t n_planes = 2 * (size_t)kv.Lf * kv.Hkv + 2;
+    const size_t mt = max_tiles > 0 ? max_tiles : 1;
+    const size_t n_kv = (size_t)kv.Lf * kv.Hkv;
+    const size_t n_lists = per_head ? n_kv : 1;
+    const size_t n_planes = 2 * n_kv + (per_head ? 3 * n_kv : 2);
     CompactWsLayout l;
     l.ctl = kStatusBytes;
-    l.need = l.ctl + 256;
-    l.flags = l.need + align256(sizeof(int32_t) * (max_tiles > 0 ? max_tiles : 1));
-    l.total = l.flags + align256(sizeof(int32_t) * n_planes * (max_tiles > 0 ? max_tiles : 1));
+    l.first = l.ctl + 256;
+    l.need = l.first + align256(sizeof(int32_t) * n_lists);
+    l.flags = l.need + align256(sizeof(int32_t) * n_lists * mt);
+    l.total = l.flags + align256(sizeof(int32_t) * n_planes * mt);
     return l;
 }
 
-}  // namespace
-
-size_t compact_workspace_bytes(const KvPlanes& kv, int cache_len) {
-    return compact_layout(kv, cache_len).total;
-}
-
-cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, const int32_t* n_retained,
-                              int cache_len, void* ws, int32_t* status, cudaStream_t s)
+cudaError_t launch_compact(const KvPlanes& kv, bool per_head, const int32_t* retain_idx, int list_stride,
+                           const int32_t* n_retained, int cache_len, void* ws, int32_t* status, cudaStream_t s)
 {
     if (cache_len <= 0) return cudaSuccess;
-    const CompactWsLayout l = compact_layout(kv, cache_len);
+    const CompactWsLayout l = compact_layout(kv, cache_len, per_head);
     char* w = static_cast<char*>(ws);
     CompactArgs a;
     a.k_cache = static_cast<char*>(kv.k_cache);
     a.v_cache = static_cast<char*>(kv.v_cache);
-    a.tok_chunk = reinterpret_cast<char*>(kv.tok_chunk);
-    a.tok_pos = reinterpret_cast<char*>(kv.tok_pos);
+    a.meta[0] = reinterpret_cast<char*>(kv.tok_chunk);
+    a.meta[1] = reinterpret_cast<char*>(kv.tok_pos);
+    a.meta[2] = reinterpret_cast<char*>(kv.tok_score);
     a.n_kv_planes = kv.Lf * kv.Hkv;
+    a.n_lists = per_head ? a.n_kv_planes : 1;
+    a.list_stride = per_head ? list_stride : 0;
+    a.n_meta = per_head ? 3 : 2;
     a.capacity = kv.capacity;
     a.row_bytes = kv.D * elt_bytes(kv.dtype);
     a.tile_rows = tile_rows_for(a.row_bytes);
-    a.n_planes = 2 * a.n_kv_planes + 2;
+    a.n_planes = 2 * a.n_kv_planes + a.n_meta * (per_head ? a.n_kv_planes : 1);
     a.cache_len = cache_len;
     a.max_tiles = (cache_len + a.tile_rows - 1) / a.tile_rows;
     a.retain_idx = retain_idx;
     a.n_retained = n_retained;
     a.ctl = reinterpret_cast<CompactCtl*>(w + l.ctl);
+    a.first = reinterpret_cast<int32_t*>(w + l.first);
     a.need = reinterpret_cast<int32_t*>(w + l.need);
     a.flags = reinterpret_cast<int32_t*>(w + l.flags);
     a.status = status;
 
     const int sms = device_sm_count();
-    const int init_blocks = min(4 * sms, (a.n_planes * a.max_tiles + 255) / 256 + 1);
+    const long long init_items = (long long)a.n_planes * a.max_tiles + a.n_lists;
+    const int init_blocks = (int)std::min<long long>(4ll * sms, (init_items + 255) / 256 + 1);
     compact_init_kernel<<<init_blocks, 256, 0, s>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     // the prepass and the moves start while their predecessor finishes (each waits for it before
     // reading or writing anything); the flag reset above is not overlapped: it writes the
     // workspace that the preceding call may still be using
-    e = launch_dependent(compact_need_kernel, dim3(min(4 * sms, (cache_len + 255) / 256)), dim3(256), 0, s, a);
+    const long long need_items = (long long)cache_len * a.n_lists;
+    const int need_blocks = (int)std::min<long long>(4ll * sms, (need_items + 255) / 256);
+    e = launch_dependent(compact_need_kernel, dim3(need_blocks), dim3(256), 0, s, a);
     if (e != cudaSuccess) return e;
 
     const int smem = a.tile_rows * a.row_bytes;
@@ -371,9 +466,32 @@ cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, con
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, compact_main_kernel, 32, smem);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
-    const int max_units = a.max_tiles * a.n_planes;
-    const int grid = max(1, min(max_units, per_sm * sms));
+    const long long max_units = (long long)a.max_tiles * a.n_planes;
+    const int grid = (int)std::max<long long>(1, std::min<long long>(max_units, (long long)per_sm * sms));
     return launch_dependent(compact_main_kernel, dim3(grid), dim3(32), (size_t)smem, s, a);
+}
+
+}  // namespace
+
+size_t compact_workspace_bytes(const KvPlanes& kv, int cache_len) {
+    return compact_layout(kv, cache_len, false).total;
+}
+
+size_t compact_heads_workspace_bytes(const KvPlanes& kv, int cache_len) {
+    return compact_layout(kv, cache_len, true).total;
+}
+
+cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, const int32_t* n_retained,
+                              int cache_len, void* ws, int32_t* status, cudaStream_t s)
+{
+    return launch_compact(kv, false, retain_idx, 0, n_retained, cache_len, ws, status, s);
+}
+
+cudaError_t launch_compact_kv_heads(const KvPlanes& kv, const int32_t* retain_idx, int list_stride,
+                                    const int32_t* n_retained, int cache_len, void* ws, int32_t* status,
+                                    cudaStream_t s)
+{
+    return launch_compact(kv, true, retain_idx, list_stride, n_retained, cache_len, ws, status, s);
 }
 
 cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_new, const void* v_new,
@@ -391,6 +509,21 @@ cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_ne
         static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache), kv.Lf * kv.Hkv, kv.capacity, rb, cache_len,
         static_cast<const char*>(k_new), static_cast<const char*>(v_new), n_new, kv.tok_chunk, kv.tok_pos, chunk_id,
         first_pos, blocks_per_plane);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append_kv_heads(const KvPlanes& kv, int signal, int cache_len, const void* k_new,
+                                   const void* v_new, int n_new, int chunk_id, int first_pos, cudaStream_t s)
+{
+    if (n_new <= 0) return cudaSuccess;
+    const int rb = kv.D * elt_bytes(kv.dtype);
+    const long long rows = (long long)kv.Lf * kv.Hkv * n_new;
+    const long long blocks = (rows + kAppendHeadsWarps - 1) / kAppendHeadsWarps;
+    if (blocks > INT_MAX) return cudaErrorInvalidValue;
+    append_kv_heads_kernel<<<(int)blocks, kAppendHeadsWarps * 32, 0, s>>>(
+        static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache), kv.Lf * kv.Hkv, kv.capacity, rb,
+        kv.dtype == DELTAS_BF16 ? 1 : 0, cache_len, static_cast<const char*>(k_new), static_cast<const char*>(v_new),
+        n_new, kv.tok_chunk, kv.tok_pos, kv.tok_score, signal == DELTAS_SIGNAL_KEY_NORM ? 1 : 0, chunk_id, first_pos);
     return cudaGetLastError();
 }
 

@@ -88,8 +88,9 @@ struct KvPlanes {
     int Lf, Hkv, D, dtype, capacity;
     void* k_cache;
     void* v_cache;
-    int32_t* tok_chunk;
+    int32_t* tok_chunk;      // [capacity], or [Lf][Hkv][capacity] with a per-head signal
     int32_t* tok_pos;
+    float* tok_score = nullptr;   // [Lf][Hkv][capacity]: per-head token scores (Sec. 4.3 signals)
 };
 
 // A batch of row copies for one kernel: segment s moves `rows` rows of row_bytes bytes (16-byte
@@ -127,6 +128,17 @@ size_t compact_workspace_bytes(const KvPlanes& kv, int cache_len);
 cudaError_t launch_compact_kv(const KvPlanes& kv, const int32_t* retain_idx, const int32_t* n_retained,
                               int cache_len, void* ws, int32_t* status, cudaStream_t s);
 cudaError_t launch_copy_batch(const CopyBatch& b, cudaStream_t s);
+// Per-head token signals (key norm, value norm; Sec. 4.3).
+cudaError_t launch_append_kv_heads(const KvPlanes& kv, int signal, int cache_len, const void* k_new,
+                                   const void* v_new, int n_new, int chunk_id, int first_pos, cudaStream_t s);
+size_t select_heads_workspace_bytes(int n_planes, int cache_len);
+cudaError_t launch_select_heads(const deltas_policy& p, int n_planes, int cache_len, int plane_stride,
+                                const int32_t* tok_chunk, const float* tok_score, int32_t* retain_idx,
+                                int32_t* n_retained, uint8_t* mask, void* ws, int32_t* status, cudaStream_t s);
+size_t compact_heads_workspace_bytes(const KvPlanes& kv, int cache_len);
+cudaError_t launch_compact_kv_heads(const KvPlanes& kv, const int32_t* retain_idx, int list_stride,
+                                    const int32_t* n_retained, int cache_len, void* ws, int32_t* status,
+                                    cudaStream_t s);
 cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_new, const void* v_new,
                              int n_new, int chunk_id, int first_pos, cudaStream_t s);
 

@@ -16,6 +16,13 @@ Per arriving chunk c, all on one CUDA stream and with no host synchronisation:
 The host tracks the cache length without reading the device: after an eviction it is exactly M
 (the selection keeps min(T, M) tokens).
 
+With ``signal="key_norm"`` or ``"value_norm"`` the stream ranks tokens by a cache-internal signal
+of Sec. 4.3 instead (-||k|| or ||v||, per KV head and per token): step 2 is dropped (the update
+runs without drift partials), step 3 is ``deltas_append_kv_heads`` (which also scores the new
+tokens) and step 4 is ``deltas_select_retain_heads`` + ``deltas_compact_kv_heads``: every
+(layer, KV head) plane keeps its own M tokens, so ``tok_chunk``, ``tok_pos`` and ``tok_score``
+are [Lf, Hkv, capacity] and ``retain_idx`` is [Lf * Hkv, M].
+
 Questions (Sec. 3.3): ``snapshot()`` saves the stream state before a question and ``restore()``
 puts it back after the answer (``deltas_copy_stream_state``: the recurrent state, the chunk
 scores, and unless ``full=False`` the live cache rows with their chunk ids and positions; the host
@@ -48,9 +55,10 @@ class DeltaSStream:
                  kv_layers, kv_heads, kv_head_dim, kv_dtype: torch.dtype, budget_M, n_sink=0,
                  n_window=0, n_buckets=1, chunk_len, max_chunks, q_scale=None, state0=None,
                  device="cuda", signal: str = "drift"):
-        if signal not in ("drift", "write_norm"):
+        if signal not in ("drift", "write_norm") + tuple(L.SIGNALS):
             raise ValueError(f"unknown signal {signal!r}")
         self.signal = signal
+        self.per_head = signal in L.SIGNALS
         self.gdn = L.gdn_desc(num_layers, num_k_heads, num_v_heads, head_dim, act_dtype, q_scale)
         self.policy = L.policy(budget_M, n_sink, n_window, n_buckets)
         self.capacity = budget_M + chunk_len
@@ -60,18 +68,26 @@ class DeltaSStream:
         dev = torch.device(device)
         self.state = (state0.clone() if state0 is not None else
                       torch.zeros(num_layers, num_v_heads, head_dim, head_dim, device=dev))
-        self.partials = torch.zeros(num_layers, num_v_heads, 2, device=dev)
+        self.partials = None if self.per_head else torch.zeros(num_layers, num_v_heads, 2, device=dev)
         self.write_norms = torch.zeros(num_layers, num_v_heads, device=dev) if signal == "write_norm" else None
         self.chunk_scores = torch.zeros(max_chunks, device=dev)
         self.k_cache = torch.zeros(kv_layers, kv_heads, self.capacity, kv_head_dim, dtype=kv_dtype, device=dev)
         self.v_cache = torch.zeros_like(self.k_cache)
-        self.tok_chunk = torch.zeros(self.capacity, dtype=torch.int32, device=dev)
-        self.tok_pos = torch.zeros(self.capacity, dtype=torch.int32, device=dev)
-        self.retain_idx = torch.zeros(budget_M, dtype=torch.int32, device=dev)
+        meta = (kv_layers, kv_heads, self.capacity) if self.per_head else (self.capacity,)
+        self.tok_chunk = torch.zeros(meta, dtype=torch.int32, device=dev)
+        self.tok_pos = torch.zeros(meta, dtype=torch.int32, device=dev)
+        self.tok_score = torch.zeros(meta, device=dev) if self.per_head else None
+        lists = (kv_layers * kv_heads, budget_M) if self.per_head else (budget_M,)
+        self.retain_idx = torch.zeros(lists, dtype=torch.int32, device=dev)
         self.n_retained = torch.zeros(1, dtype=torch.int32, device=dev)
-        ws = max(L.deltas_gdn_chunk_update_workspace_size(self.gdn, chunk_len),
-                 L.deltas_select_retain_workspace_size(self.capacity),
-                 L.deltas_compact_kv_workspace_size(self.kv, self.capacity))
+        if self.per_head:
+            ws = max(L.deltas_gdn_chunk_update_workspace_size(self.gdn, chunk_len),
+                     L.deltas_select_retain_heads_workspace_size(kv_layers * kv_heads, self.capacity),
+                     L.deltas_compact_kv_heads_workspace_size(self.kv, self.capacity))
+        else:
+            ws = max(L.deltas_gdn_chunk_update_workspace_size(self.gdn, chunk_len),
+                     L.deltas_select_retain_workspace_size(self.capacity),
+                     L.deltas_compact_kv_workspace_size(self.kv, self.capacity))
         self.workspace = L.alloc_workspace(ws, dev)
         self.cache_len = 0
         self.position = 0
@@ -86,6 +102,8 @@ class DeltaSStream:
         T = int(k.shape[1])
         L.deltas_gdn_chunk_update(self.gdn, T, q, k, v, g, beta, self.state, out, self.partials,
                                   self.workspace, stream, write_norms=self.write_norms)
+        if self.per_head:
+            return self._step_heads(k_new, v_new, stream)
         if self.signal == "write_norm":
             L.deltas_score_write_norms(self.gdn.num_layers, self.gdn.num_v_heads, self.write_norms, T, c,
                                        self.chunk_scores, stream)
@@ -110,6 +128,27 @@ class DeltaSStream:
             return True
         return False
 
+    def _step_heads(self, k_new, v_new, stream):
+        c = self.chunk
+        n_new = int(k_new.shape[2])
+        L.deltas_append_kv_heads(self.kv, self.signal, self.k_cache, self.v_cache, self.tok_chunk, self.tok_pos,
+                                 self.tok_score, self.cache_len, k_new, v_new, c, self.position, stream)
+        self.cache_len += n_new
+        self.position += n_new
+        self.chunk += 1
+        if self.cache_len > self.policy.budget_M:
+            P = self.kv.num_layers * self.kv.num_kv_heads
+            L.deltas_select_retain_heads(self.policy, self.cache_len, self.tok_chunk.view(P, -1),
+                                         self.tok_score.view(P, -1), self.retain_idx, self.n_retained, None,
+                                         self.workspace, stream)
+            L.deltas_compact_kv_heads(self.kv, self.k_cache, self.v_cache, self.tok_chunk, self.tok_pos,
+                                      self.tok_score, self.retain_idx, self.n_retained, self.cache_len,
+                                      self.workspace, stream)
+            self.cache_len = self.policy.budget_M
+            self.evictions += 1
+            return True
+        return False
+
     def _buffers(self, full: bool) -> dict:
         b = {"state": self.state, "chunk_scores": self.chunk_scores}
         if full:
@@ -118,6 +157,8 @@ class DeltaSStream:
 
     def snapshot(self, full: bool = True, into: StreamSnapshot | None = None, stream=None) -> StreamSnapshot:
         """Save the stream state before a question (Sec. 3.3); ``into`` reuses a snapshot's buffers."""
+        if self.per_head:
+            raise ValueError("snapshot of a stream ranked by a per-head token signal is not supported")
         snap = into if into is not None else StreamSnapshot(self, full)
         if snap.full != full:
             raise ValueError("the snapshot's buffers were made for the other kind of snapshot")

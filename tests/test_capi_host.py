@@ -25,7 +25,7 @@ def _declared():
 
 def test_every_declared_symbol_is_exported(L):
     names = _declared()
-    assert len(names) == 18, names
+    assert len(names) == 23, names
     lib = ctypes.CDLL(L.LIB_PATH)
     for n in names:
         assert hasattr(lib, n), n
@@ -167,3 +167,43 @@ def test_write_norm_argument_checks(L):
     assert raw.deltas_score_write_norms(2, 4, FAKE, -1, 0, FAKE, None) == bad
     assert raw.deltas_score_write_norms(2, 4, FAKE, 10, -1, FAKE, None) == bad
     assert raw.deltas_score_write_norms(2, 4, None, 10, 0, FAKE, None) == bad
+
+
+def test_token_signal_argument_checks(L):
+    """The per-head calls of the Sec. 4.3 token signals reject bad arguments on the host."""
+    raw = L.raw()
+    kv = L.KvDesc(2, 2, 64, L.DELTAS_BF16, 1000)
+    K = L.DELTAS_SIGNAL_KEY_NORM
+
+    def append(signal=K, score=FAKE, cache_len=10, n_new=20):
+        return raw.deltas_append_kv_heads(ctypes.byref(kv), signal, FAKE, FAKE, FAKE, FAKE, score, cache_len,
+                                          FAKE, FAKE, n_new, 0, 0, None)
+    assert append(signal=0) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert append(signal=3) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert append(score=None) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert append(cache_len=990) == L.DELTAS_ERR_INVALID_ARGUMENT           # past capacity
+    assert append(n_new=-1) == L.DELTAS_ERR_INVALID_ARGUMENT
+
+    def select(pol, planes=4, T=100, stride=100, ws=FAKE, wsb=1 << 24):
+        return raw.deltas_select_retain_heads(ctypes.byref(pol) if pol else None, planes, T, stride, FAKE, FAKE,
+                                              FAKE, FAKE, None, ws, wsb, None)
+    ok = L.Policy(10, 0, 0, 1)
+    assert select(None) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert select(L.Policy(10, 5, 5, 1)) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert select(L.Policy(10, 0, 0, 33)) == L.DELTAS_ERR_UNSUPPORTED
+    assert select(ok, planes=0) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert select(ok, stride=99) == L.DELTAS_ERR_INVALID_ARGUMENT          # plane_stride < cache_len
+    assert select(ok, T=(1 << 20) + 1, stride=(1 << 20) + 1) == L.DELTAS_ERR_UNSUPPORTED
+    assert select(ok, wsb=16) == L.DELTAS_ERR_WORKSPACE
+    small = L.deltas_select_retain_heads_workspace_size(4, 100)
+    assert 16 < small < L.deltas_select_retain_heads_workspace_size(4, 10000)
+
+    def compact(cache_len=500, stride=600, score=FAKE, wsb=1 << 24):
+        return raw.deltas_compact_kv_heads(ctypes.byref(kv), FAKE, FAKE, FAKE, FAKE, score, FAKE, stride, FAKE,
+                                           cache_len, FAKE, wsb, None)
+    assert compact(cache_len=1001) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert compact(score=None) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert compact(stride=0) == L.DELTAS_ERR_INVALID_ARGUMENT
+    assert compact(wsb=64) == L.DELTAS_ERR_WORKSPACE
+    big = L.KvDesc(8, 2, 256, L.DELTAS_BF16, 65536)
+    assert L.deltas_compact_kv_heads_workspace_size(big, 65536) > L.deltas_compact_kv_workspace_size(big, 65536) > 0

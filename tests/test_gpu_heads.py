@@ -1,0 +1,260 @@
+"""Per-head token signals (Sec. 4.3: key norm -||k||, value norm ||v||, ranked per KV head under the
+Sec. 3.3 policy) through the C ABI on the GPU, against the CPU oracle.
+
+Scores are float32 sums of squares on the GPU and fp64 in the oracle, so they are compared within a
+relative 2e-6 (a float32 sum of 256 exact squares, a warp tree and a rounded square root stay well
+inside it).  Selection and compaction are index and byte work: they must match the oracle exactly,
+given identical scores (the oracle ranks with the GPU's float32 scores)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle.stream import run_stream_heads
+from paper_2609_27470_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+SCORE_RTOL = 2e-6
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2609_27470_gb300 import build
+    build.build()
+    from paper_2609_27470_gb300 import _lib
+    return _lib
+
+
+def _bits(t):
+    return t.view(torch.int16) if t.dtype == torch.bfloat16 else t.view(torch.int32)
+
+
+def _np(t):
+    return t.view(torch.int16).numpy() if t.dtype == torch.bfloat16 else t.numpy()
+
+
+@pytest.mark.parametrize("signal", ["key_norm", "value_norm"])
+@pytest.mark.parametrize("D,dt,cache_len,n_new", [
+    (256, "bf16", 1000, 512),
+    (256, "bf16", 0, 131),        # first chunk, ragged length
+    (16, "f32", 37, 64),
+    (128, "bf16", 5, 1),
+])
+def test_append_heads_copies_rows_and_scores_them(L, signal, D, dt, cache_len, n_new):
+    dev = torch.device("cuda")
+    tdt = torch.float32 if dt == "f32" else torch.bfloat16
+    Lf, Hkv, cap = 2, 3, cache_len + n_new + 7
+    kv = L.kv_desc(Lf, Hkv, D, tdt, cap)
+    gen = torch.Generator().manual_seed(D + cache_len + n_new)
+    kc = torch.randn(Lf, Hkv, cap, D, generator=gen).to(tdt)
+    vc = torch.randn(Lf, Hkv, cap, D, generator=gen).to(tdt)
+    meta = [torch.randint(0, 99, (Lf, Hkv, cap), generator=gen, dtype=torch.int32) for _ in range(2)]
+    ts = torch.randn(Lf, Hkv, cap, generator=gen)
+    kn = torch.randn(Lf, Hkv, n_new, D, generator=gen).to(tdt)
+    vn = 3.0 * torch.randn(Lf, Hkv, n_new, D, generator=gen).to(tdt)
+    kn[0, 1, 0] = 0                                      # a zero row scores (-)0
+    d = [t.to(dev) for t in (kc, vc, meta[0], meta[1], ts)]
+    L.deltas_append_kv_heads(kv, signal, d[0], d[1], d[2], d[3], d[4], cache_len, kn.to(dev), vn.to(dev), 41, 9000)
+    torch.cuda.synchronize()
+    kc2, vc2, tc2, tp2, ts2 = (t.cpu() for t in d)
+    sl = slice(cache_len, cache_len + n_new)
+    assert torch.equal(_bits(kc2[:, :, sl]), _bits(kn)) and torch.equal(_bits(vc2[:, :, sl]), _bits(vn))
+    for new, old in ((kc2, kc), (vc2, vc), (tc2, meta[0]), (tp2, meta[1]), (ts2, ts)):
+        assert torch.equal(_bits(new[:, :, :cache_len]), _bits(old[:, :, :cache_len]))
+        assert torch.equal(_bits(new[:, :, cache_len + n_new:]), _bits(old[:, :, cache_len + n_new:]))
+    assert torch.all(tc2[:, :, sl] == 41)
+    assert torch.equal(tp2[:, :, sl], (9000 + torch.arange(n_new, dtype=torch.int32)).expand(Lf, Hkv, n_new))
+    rows = (kn if signal == "key_norm" else vn).float().numpy()
+    ref = oracle.row_norm_scores(rows, signal)
+    np.testing.assert_allclose(ts2[:, :, sl].numpy(), ref, rtol=SCORE_RTOL, atol=0)
+    if signal == "key_norm":
+        assert ts2[0, 1, cache_len].item() == 0.0
+
+
+def _plane_inputs(rng, planes, T, n_chunks, stride):
+    """Per-plane chunk ids (ascending, with the gaps repeated evictions leave) and scores with
+    exact ties, signed zeros and infinities."""
+    tc = np.zeros((planes, stride), np.int32)
+    ts = np.zeros((planes, stride), np.float32)
+    for p in range(planes):
+        tc[p, :T] = np.sort(rng.integers(0, n_chunks, size=T))
+        s = np.round(rng.standard_normal(T), 2).astype(np.float32)       # ties
+        if T > 20:
+            idx = rng.choice(T, size=8, replace=False)
+            s[idx[:2]] = -0.0
+            s[idx[2:4]] = 0.0
+            s[idx[4]] = np.inf
+            s[idx[5]] = -np.inf
+        ts[p, :T] = s
+    return tc, ts
+
+
+SELECT_CASES = [
+    # planes, T, M, n_s, n_w, N
+    (4, 1000, 600, 4, 128, 4),
+    (3, 777, 700, 0, 0, 1),
+    (2, 3000, 2500, 2, 10, 32),
+    (2, 300, 40, 4, 30, 8),            # quota 0: everything comes from the fill
+    (3, 500, 600, 4, 128, 4),          # no eviction: the identity
+    (5, 2049, 1024, 4, 1000, 0),       # N = 0 read as one span
+    (16, 33280, 32768, 4, 1024, 4),    # streaming shape: keys in shared memory
+    (16, 65536, 16384, 4, 1024, 4),    # 64k slots: keys in the workspace
+]
+
+
+@pytest.mark.parametrize("planes,T,M,n_s,n_w,N", SELECT_CASES)
+@pytest.mark.parametrize("with_mask", [True, False])
+def test_select_heads_matches_oracle(L, planes, T, M, n_s, n_w, N, with_mask):
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(T + M + N)
+    stride = T + 13
+    tc, ts = _plane_inputs(rng, planes, T, max(4, T // 50), stride)
+    pol = L.policy(M, n_s, n_w, N)
+    ws = L.alloc_workspace(L.deltas_select_retain_heads_workspace_size(planes, T), dev)
+    ri = torch.full((planes, M), -1, dtype=torch.int32, device=dev)
+    nr = torch.zeros(1, dtype=torch.int32, device=dev)
+    mk = torch.full((planes, stride), 7, dtype=torch.uint8, device=dev) if with_mask else None
+    L.deltas_select_retain_heads(pol, T, torch.from_numpy(tc).to(dev), torch.from_numpy(ts).to(dev), ri, nr, mk, ws)
+    torch.cuda.synchronize()
+    assert L.deltas_get_device_status(ws) == (0, 0)
+    n = min(T, M)
+    assert nr.item() == n
+    ri = ri.cpu().numpy()
+    for p in range(planes):
+        idx, mask = oracle.select_retain_tokens(M, n_s, n_w, N, tc[p, :T], ts[p, :T])
+        assert np.array_equal(ri[p, :n], idx), p
+        assert np.all(ri[p, n:] == -1)
+        if with_mask:
+            m = mk[p].cpu().numpy()
+            assert np.array_equal(m[:T], mask) and np.all(m[T:] == 7)
+
+
+def test_select_heads_reports_negative_chunk_ids(L):
+    dev = torch.device("cuda")
+    tc = torch.zeros(2, 100, dtype=torch.int32)
+    tc[1, 50] = -3
+    ts = torch.randn(2, 100)
+    ws = L.alloc_workspace(L.deltas_select_retain_heads_workspace_size(2, 100), dev)
+    L.deltas_clear_device_status(ws)
+    ri = torch.zeros(2, 60, dtype=torch.int32, device=dev)
+    nr = torch.zeros(1, dtype=torch.int32, device=dev)
+    L.deltas_select_retain_heads(L.policy(60, 0, 0, 1), 100, tc.to(dev), ts.to(dev), ri, nr, None, ws)
+    assert L.deltas_get_device_status(ws)[0] == L.DELTAS_ERR_DEVICE_INDEX
+
+
+@pytest.mark.parametrize("D,dt,T,M", [
+    (256, "bf16", 33280, 32768),
+    (256, "bf16", 5000, 1111),
+    (16, "f32", 777, 500),
+    (64, "bf16", 130, 129),
+])
+def test_compact_heads_matches_oracle(L, D, dt, T, M):
+    dev = torch.device("cuda")
+    tdt = torch.float32 if dt == "f32" else torch.bfloat16
+    Lf, Hkv, cap = 2, 3, T + 9
+    P = Lf * Hkv
+    rng = np.random.default_rng(T + D)
+    lists = []
+    for p in range(P):
+        if p == 0:
+            lists.append(np.arange(M, dtype=np.int32))                         # nothing moves
+        elif p == 1:
+            lists.append(np.r_[np.arange(M - 1), T - 1].astype(np.int32))      # only the last row moves
+        else:
+            lists.append(np.sort(rng.choice(T, size=M, replace=False)).astype(np.int32))
+    kv = L.kv_desc(Lf, Hkv, D, tdt, cap)
+    gen = torch.Generator().manual_seed(T)
+    kc = torch.randn(Lf, Hkv, cap, D, generator=gen).to(tdt)
+    vc = torch.randn(Lf, Hkv, cap, D, generator=gen).to(tdt)
+    tc = torch.randint(0, 1 << 20, (Lf, Hkv, cap), generator=gen, dtype=torch.int32)
+    tp = torch.randint(0, 1 << 20, (Lf, Hkv, cap), generator=gen, dtype=torch.int32)
+    ts = torch.randn(Lf, Hkv, cap, generator=gen)
+    ref = oracle.compact_kv_heads(_np(kc), _np(vc), tc.numpy(), tp.numpy(), ts.numpy(), lists, T)
+    d = [t.to(dev) for t in (kc, vc, tc, tp, ts)]
+    ri = torch.from_numpy(np.stack(lists)).to(dev)
+    nr = torch.tensor([M], dtype=torch.int32, device=dev)
+    ws = L.alloc_workspace(L.deltas_compact_kv_heads_workspace_size(kv, T), dev)
+    L.deltas_compact_kv_heads(kv, d[0], d[1], d[2], d[3], d[4], ri, nr, T, ws)
+    torch.cuda.synchronize()
+    assert L.deltas_get_device_status(ws) == (0, 0)
+    for got, want in zip(d, ref):
+        g = got.cpu()
+        g = _np(g) if g.dtype == torch.bfloat16 else g.numpy()
+        assert np.array_equal(g.view(np.int32) if g.dtype == np.float32 else g,
+                              want.view(np.int32) if want.dtype == np.float32 else want)
+
+
+def test_compact_heads_rejects_a_bad_list(L):
+    dev = torch.device("cuda")
+    kv = L.kv_desc(1, 2, 64, torch.bfloat16, 100)
+    kc = torch.randn(1, 2, 100, 64, device=dev).to(torch.bfloat16)
+    before = kc.clone()
+    tc = torch.zeros(1, 2, 100, dtype=torch.int32, device=dev)
+    ri = torch.tensor([[0, 5, 9], [0, 7, 3]], dtype=torch.int32, device=dev)   # plane 1 not ascending
+    nr = torch.tensor([3], dtype=torch.int32, device=dev)
+    ws = L.alloc_workspace(L.deltas_compact_kv_heads_workspace_size(kv, 50), dev)
+    L.deltas_clear_device_status(ws)
+    L.deltas_compact_kv_heads(kv, kc, kc.clone(), tc, tc.clone(), torch.zeros(1, 2, 100, device=dev), ri, nr, 50, ws)
+    assert L.deltas_get_device_status(ws)[0] == L.DELTAS_ERR_DEVICE_INDEX
+    assert torch.equal(_bits(kc), _bits(before))
+
+
+STREAM_CFG = dict(L=2, Hk=2, Hv=4, d=128, Lf=2, Hkv=2, D=256, M=600, n_s=4, n_w=128, N=4,
+                  lens=[118, 132, 124, 121, 129, 119, 127, 125, 130, 118, 126, 131])
+
+
+@pytest.mark.parametrize("signal", ["key_norm", "value_norm"])
+def test_stream_heads_matches_oracle(L, signal):
+    """The stream driver with a per-head signal vs the oracle's per-head loop, given the GPU's own
+    token scores; the scores themselves against the oracle's; the recurrent state still moves."""
+    from paper_2609_27470_gb300.stream import DeltaSStream
+    cfg = STREAM_CFG
+    dev = torch.device("cuda")
+    lens = cfg["lens"]
+    chunks = [inputs.gdn_chunk(cfg["L"], lens[c], cfg["Hk"], cfg["Hv"], cfg["d"], "bf16", inputs.seed_for(81, c))
+              for c in range(len(lens))]
+    kvs = [inputs.kv_chunk(cfg["Lf"], cfg["Hkv"], lens[c], cfg["D"], "bf16", inputs.seed_for(82, c))
+           for c in range(len(lens))]
+    s0 = inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 83)
+    s = DeltaSStream(num_layers=cfg["L"], num_k_heads=cfg["Hk"], num_v_heads=cfg["Hv"], head_dim=cfg["d"],
+                     act_dtype=torch.bfloat16, kv_layers=cfg["Lf"], kv_heads=cfg["Hkv"], kv_head_dim=cfg["D"],
+                     kv_dtype=torch.bfloat16, budget_M=cfg["M"], n_sink=cfg["n_s"], n_window=cfg["n_w"],
+                     n_buckets=cfg["N"], chunk_len=max(lens), max_chunks=len(lens), state0=s0.to(dev), device=dev,
+                     signal=signal)
+    state_before = s.state.clone()
+    for c in range(len(lens)):
+        x = {k: v.to(dev) for k, v in chunks[c].items()}
+        s.step(x["q"], x["k"], x["v"], x["g"], x["beta"], kvs[c][0].to(dev), kvs[c][1].to(dev))
+    torch.cuda.synchronize()
+    assert L.deltas_get_device_status(s.workspace) == (0, 0)
+    assert not torch.equal(s.state, state_before)
+    assert s.evictions > 0
+
+    # the GPU's score of every chunk's tokens: the same append into a scratch cache
+    kvd = L.kv_desc(cfg["Lf"], cfg["Hkv"], cfg["D"], torch.bfloat16, max(lens))
+    shp = (cfg["Lf"], cfg["Hkv"], max(lens))
+    scratch = [torch.zeros(*shp, cfg["D"], dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    meta = [torch.zeros(shp, dtype=torch.int32, device=dev) for _ in range(2)]
+    gpu_scores = []
+    for c in range(len(lens)):
+        sc = torch.zeros(shp, device=dev)
+        L.deltas_append_kv_heads(kvd, signal, scratch[0], scratch[1], meta[0], meta[1], sc, 0,
+                                 kvs[c][0].to(dev), kvs[c][1].to(dev), c, 0)
+        gpu_scores.append(sc[:, :, : lens[c]].cpu().numpy())
+    policy = dict(budget_M=cfg["M"], n_sink=cfg["n_s"], n_window=cfg["n_w"], n_buckets=cfg["N"])
+    ref = run_stream_heads(lambda c: (_np(kvs[c][0]), _np(kvs[c][1])), len(lens), policy, s.capacity, signal,
+                           score_override=lambda c: gpu_scores[c])
+    own = run_stream_heads(lambda c: (_np(kvs[c][0]), _np(kvs[c][1])), 1, dict(policy, budget_M=10 ** 6),
+                           max(lens), signal)
+    np.testing.assert_allclose(gpu_scores[0], own.tok_score[:, :, : lens[0]], rtol=SCORE_RTOL, atol=0)
+    n = s.cache_len
+    assert n == ref.cache_len and s.evictions == len(ref.evictions)
+    assert np.array_equal(_np(s.k_cache.cpu())[:, :, :n], ref.k_cache[:, :, :n])
+    assert np.array_equal(_np(s.v_cache.cpu())[:, :, :n], ref.v_cache[:, :, :n])
+    for name in ("tok_chunk", "tok_pos"):
+        assert np.array_equal(getattr(s, name).cpu().numpy()[:, :, :n], getattr(ref, name)[:, :, :n]), name
+    assert np.array_equal(s.tok_score.cpu().numpy()[:, :, :n].view(np.int32), ref.tok_score[:, :, :n].view(np.int32))
+    # heads really differ in what they keep
+    tp = s.tok_pos.cpu().numpy()
+    assert not np.array_equal(tp[0, 0, :n], tp[0, 1, :n])
