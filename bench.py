@@ -194,7 +194,9 @@ def algorithmic_gdn_flops(L, T, Hv, d, with_out):
 class StreamingWorkload:
     """One chunk per step through the whole path (update + drift, score, append, select, compact)
     on a cache kept at the budget: streaming (512-token chunks) and paper (118-132-token chunks,
-    the length cycling through the ring)."""
+    the length cycling through the ring).  With a per-head token signal (paper_key_norm,
+    paper_value_norm: Sec. 4.3) the step is update (no drift), append with scores, per-plane
+    select and per-plane compact."""
 
     def __init__(self, dev, L, cfg=None):
         cfg = dict(cfg or configs.STREAMING)
@@ -230,8 +232,13 @@ class StreamingWorkload:
         for c, n in enumerate(fills):
             kn, vn = self.kv_ring[c % RING]
             kn, vn = kn[:, :, :n].contiguous(), vn[:, :, :n].contiguous()
-            L.deltas_append_kv(self.s.kv, self.s.k_cache, self.s.v_cache, self.s.tok_chunk, self.s.tok_pos,
-                               self.s.cache_len, kn, vn, c, self.s.position)
+            if self.s.per_head:
+                L.deltas_append_kv_heads(self.s.kv, self.s.signal, self.s.k_cache, self.s.v_cache, self.s.tok_chunk,
+                                         self.s.tok_pos, self.s.tok_score, self.s.cache_len, kn, vn, c,
+                                         self.s.position)
+            else:
+                L.deltas_append_kv(self.s.kv, self.s.k_cache, self.s.v_cache, self.s.tok_chunk, self.s.tok_pos,
+                                   self.s.cache_len, kn, vn, c, self.s.position)
             self.s.cache_len += n
             self.s.position += n
         self.s.chunk = n_fill
@@ -243,6 +250,9 @@ class StreamingWorkload:
         kn, vn = self.kv_ring[self.step_i % RING]
         T = self.lens[self.step_i % RING]
         s, L, c = self.s, self.L, self.s.chunk
+        if s.per_head:
+            self._step_heads(timer, x, kn, vn, T)
+            return
         with timer.mark("gdn_update"):
             L.deltas_gdn_chunk_update(s.gdn, T, None, x["k"], x["v"], x["g"], x["beta"], s.state, None,
                                       s.partials, s.workspace, write_norms=s.write_norms)
@@ -266,14 +276,37 @@ class StreamingWorkload:
         s.cache_len = s.policy.budget_M
         self.step_i += 1
 
+    def _step_heads(self, timer, x, kn, vn, T):
+        s, L, c = self.s, self.L, self.s.chunk
+        P = s.kv.num_layers * s.kv.num_kv_heads
+        with timer.mark("gdn_update"):
+            L.deltas_gdn_chunk_update(s.gdn, T, None, x["k"], x["v"], x["g"], x["beta"], s.state, None, None,
+                                      s.workspace)
+        with timer.mark("append"):
+            L.deltas_append_kv_heads(s.kv, s.signal, s.k_cache, s.v_cache, s.tok_chunk, s.tok_pos, s.tok_score,
+                                     s.cache_len, kn, vn, c, s.position)
+        s.cache_len += T
+        s.position += T
+        s.chunk += 1
+        with timer.mark("select"):
+            L.deltas_select_retain_heads(s.policy, s.cache_len, s.tok_chunk.view(P, -1), s.tok_score.view(P, -1),
+                                         s.retain_idx, s.n_retained, None, s.workspace)
+        with timer.mark("compact"):
+            L.deltas_compact_kv_heads(s.kv, s.k_cache, s.v_cache, s.tok_chunk, s.tok_pos, s.tok_score,
+                                      s.retain_idx, s.n_retained, s.cache_len, s.workspace)
+        s.cache_len = s.policy.budget_M
+        self.step_i += 1
+
     def post_step(self):
-        # rows the last compaction moved (slots j whose source differs from j); runs between the
-        # timed steps, on the device, without a host sync
+        # rows the last compaction moved (slots j whose source differs from j; per plane with a
+        # per-head signal); runs between the timed steps, on the device, without a host sync
         idx = self.s.retain_idx
-        cnt = (idx != torch.arange(idx.numel(), device=idx.device, dtype=torch.int32)).sum()
+        cnt = (idx != torch.arange(idx.shape[-1], device=idx.device, dtype=torch.int32)).sum()
         self.moved = cnt if self.moved is None else self.moved + cnt
 
     def launches_per_step(self):
+        if self.s.per_head:
+            return 2 + 1 + 1 + 3                                # update (2), append, select, compact (3)
         return 2 + 1 + 1 + 3 + 3                                # update (2), score, append, select (3), compact (3)
 
     def tokens_per_step(self):
@@ -291,7 +324,10 @@ class StreamingWorkload:
                     "tensor_frac": fl / (avg_ms * 1e-3) / 1e12 / peaks["bf16_tflops_sustained"]}
         if name == "compact":
             moved = float(self.moved.item()) / steps if self.moved is not None else 0.0
-            row = cfg["D"] * 2 * cfg["Lf"] * cfg["Hkv"] * 2 + 8
+            if self.s.per_head:      # moved (plane, row) pairs: a K row, a V row, 3 metadata words
+                row = cfg["D"] * 2 * 2 + 12
+            else:                    # moved slots: every plane's K and V row, 2 metadata words
+                row = cfg["D"] * 2 * cfg["Lf"] * cfg["Hkv"] * 2 + 8
             by = 2 * moved * row
             return {"bound": "hbm", "achieved": by / (avg_ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"],
                     "unit": "GB/s", "bytes_per_launch": by, "moved_rows_per_launch": moved}
@@ -303,6 +339,8 @@ class StreamingWorkload:
         return [x["k"], x["v"], x["g"], x["beta"], kn, vn]
 
     def result_scalar(self):
+        if self.s.per_head:                     # the score of the newest token of plane 0
+            return self.s.tok_score.view(-1)[self.s.cache_len - 1: self.s.cache_len]
         return self.s.chunk_scores[self.s.chunk - 1: self.s.chunk]
 
 
@@ -502,8 +540,8 @@ def make_workload(name, dev, L):
         return StreamingWorkload(dev, L)
     if name == "paper":
         return StreamingWorkload(dev, L, configs.PAPER)
-    if name == "paper_write_norm":
-        return StreamingWorkload(dev, L, configs.PAPER_WRITE_NORM)
+    if name in ("paper_write_norm", "paper_key_norm", "paper_value_norm"):
+        return StreamingWorkload(dev, L, _cfg(name))
     if name == "stack":
         return GdnOnlyWorkload(dev, L, configs.STACK)
     if name == "layer":
@@ -598,7 +636,9 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
     cfg = _cfg(workload)
     parts = []
     total = 0.0
-    if workload in ("streaming", "paper", "paper_write_norm", "stack", "layer"):
+    head_signal = cfg.get("signal") in ("key_norm", "value_norm")
+    if workload in ("streaming", "paper", "paper_write_norm", "paper_key_norm", "paper_value_norm", "stack",
+                    "layer"):
         C = int(round(_tokens(workload)))
         heads_total = cfg["L"] * cfg["Hv"]
         n_heads = 2
@@ -610,6 +650,8 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         while True:
             if workload == "paper_write_norm":
                 S, _, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0, want_write_norms=True)
+            elif head_signal:                              # the state moves; no drift is formed
+                S, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
             else:
                 S, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
                 oracle.drift_partials(s0, S)
@@ -661,6 +703,31 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         t_cmp = (time.perf_counter() - t0) * planes_total / 2
         total += t_sel + t_cmp
         parts.append(f"select on {T} slots; compact 2 of {planes_total} planes x{planes_total // 2}")
+    if head_signal:
+        # score the chunk's rows, then per (layer, KV head) plane: select among M + C slots with
+        # per-token scores and gather the plane's K and V rows; one plane timed, x planes
+        M, C, D = cfg["budget_M"], cfg["chunk_len"], cfg["D"]
+        T = M + C
+        P = cfg["Lf"] * cfg["Hkv"]
+        rng = np.random.default_rng(8)
+        lens = rng.integers(1, C + 1, size=4 * T // C)
+        tc = np.concatenate([np.full(n, c, np.int32) for c, n in enumerate(lens)])[-T:]
+        ts = rng.standard_normal(T).astype(np.float32)
+        rows = rng.standard_normal((P, C, D)).astype(np.float32)
+        t0 = time.perf_counter()
+        oracle.row_norm_scores(rows, cfg["signal"])
+        t_score = time.perf_counter() - t0
+        t0 = time.perf_counter()
+        idx, _ = oracle.select_retain_tokens(M, cfg["n_sink"], cfg["n_window"], cfg["n_buckets"], tc, ts)
+        t_sel = time.perf_counter() - t0
+        plane = rng.integers(-2**15, 2**15, size=(2, T, D), dtype=np.int16)
+        meta = np.zeros((3, T, 1), np.int32)
+        t0 = time.perf_counter()
+        oracle.compact_rows(plane, idx, T)
+        oracle.compact_rows(meta, idx, T)
+        t_cmp = time.perf_counter() - t0
+        total += t_score + P * (t_sel + t_cmp)
+        parts.append(f"score {P}x{C} rows; select on {T} slots and compact K, V, metadata of 1 of {P} planes x{P}")
     return _tokens(workload) / total, "; ".join(parts), time.perf_counter() - t_start
 
 
@@ -709,7 +776,8 @@ def config_line(workload):
 def _cfg(workload):
     return {"streaming": configs.STREAMING, "paper": configs.PAPER, "stack": configs.STACK,
             "layer": configs.LAYER, "kv": configs.KV, "snapshot": configs.PAPER,
-            "paper_write_norm": configs.PAPER_WRITE_NORM}[workload]
+            "paper_write_norm": configs.PAPER_WRITE_NORM, "paper_key_norm": configs.PAPER_KEY_NORM,
+            "paper_value_norm": configs.PAPER_VALUE_NORM}[workload]
 
 
 def _tokens(workload):
@@ -730,7 +798,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="streaming",
-                    choices=["streaming", "paper", "paper_write_norm", "stack", "layer", "kv", "snapshot"])
+                    choices=["streaming", "paper", "paper_write_norm", "paper_key_norm", "paper_value_norm",
+                             "stack", "layer", "kv", "snapshot"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)

@@ -1,4 +1,4 @@
-"""The five synthetic workloads, shaped like the paper's hybrid backbone (Sec. 4.1, App. A).
+"""The synthetic workloads, shaped like the paper's hybrid backbone (Sec. 4.1, App. A).
 
 * ``tiny``      — 1 gated-delta layer, 2 heads, d=16, fp32, 8 chunks x 64 tokens, zero start
                   state, 1 full-attention layer (2 KV heads, D=16, fp32 KV), budget 4 chunks.
@@ -10,6 +10,8 @@
                   64 chunks x 1024 tokens, Exp(1) chunk scores with exact ties, budget 16k.
 * ``streaming`` — ``stack`` with 512-token chunks plus ``kv`` caches, 4096 chunks, budget 32k,
                   the paper's policy (n_s=4, n_w=1024, N=4; Sec. 4.1).
+* ``paper_key_norm``, ``paper_value_norm`` — ``paper`` ranked per KV head by the key norm or the
+                  value norm (Sec. 4.3), each plane keeping its own M tokens.
 * ``paper``     — the paper's own stream shape (Sec. 4.1, App. A): chunks of two frames, 118-132
                   tokens each (a cycle of eight lengths), 8 full-attention layers x 4 KV heads x
                   D = 256, budget 8192, the paper's policy; gated-delta stack as ``stack``.
@@ -43,4 +45,10 @@ PAPER = dict(name="paper", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=ma
 # the paper stream scored by the comparison signal of Sec. 4.3 (write sizes) instead of drift
 PAPER_WRITE_NORM = dict(PAPER, name="paper_write_norm", signal="write_norm")
 
-ALL = {c["name"]: c for c in (TINY, LAYER, STACK, KV, STREAMING, PAPER, PAPER_WRITE_NORM)}
+# the paper stream ranked by a cache-internal token signal of Sec. 4.3, per KV head and token:
+# the key norm (-||k||) or the value norm (||v||)
+PAPER_KEY_NORM = dict(PAPER, name="paper_key_norm", signal="key_norm")
+PAPER_VALUE_NORM = dict(PAPER, name="paper_value_norm", signal="value_norm")
+
+ALL = {c["name"]: c for c in (TINY, LAYER, STACK, KV, STREAMING, PAPER, PAPER_WRITE_NORM, PAPER_KEY_NORM,
+                              PAPER_VALUE_NORM)}

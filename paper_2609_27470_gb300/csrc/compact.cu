@@ -52,7 +52,7 @@ struct CompactArgs {
     int capacity;
     int row_bytes;         // D * element size (multiple of 16)
     int tile_rows;         // TB
-    int n_planes;          // 2 * n_kv_planes + metadata rows (2, or 3 * n_kv_planes per head)
+    int n_planes;          // 2 * n_kv_planes (K and V); metadata moves with the K planes
     int cache_len;
     int max_tiles;         // ceil(cache_len / TB)
     const int32_t* retain_idx;
@@ -66,25 +66,21 @@ struct CompactArgs {
 
 __host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Plane p of the unit order: K planes, V planes, then the metadata rows.  Returns its base, its
-// row size and the retain list that moves it.
-__device__ __forceinline__ char* plane_base(const CompactArgs& a, int p, int& rb, int& list) {
+// Plane p of the unit order: K planes, then V planes.  Returns its base and the retain list that
+// moves it.  The metadata rows (4 bytes per slot) ride with the K plane that owns them: with one
+// shared list K plane 0 moves tok_chunk and tok_pos, with one list per (layer, head) K plane p
+// moves row p of tok_chunk, tok_pos and tok_score.
+__device__ __forceinline__ char* plane_base(const CompactArgs& a, int p, int& list, bool& owns_meta) {
     const bool shared_list = a.n_lists == 1;
     if (p < a.n_kv_planes) {
-        rb = a.row_bytes; list = shared_list ? 0 : p;
+        list = shared_list ? 0 : p;
+        owns_meta = shared_list ? p == 0 : true;
         return a.k_cache + (size_t)p * a.capacity * a.row_bytes;
     }
     p -= a.n_kv_planes;
-    if (p < a.n_kv_planes) {
-        rb = a.row_bytes; list = shared_list ? 0 : p;
-        return a.v_cache + (size_t)p * a.capacity * a.row_bytes;
-    }
-    p -= a.n_kv_planes;
-    rb = 4;
-    const int per = shared_list ? 1 : a.n_kv_planes;             // rows of one metadata array
-    const int m = p / per;
-    list = p - m * per;
-    return a.meta[m] + (size_t)list * a.capacity * 4;
+    list = shared_list ? 0 : p;
+    owns_meta = false;
+    return a.v_cache + (size_t)p * a.capacity * a.row_bytes;
 }
 
 __global__ void compact_init_kernel(CompactArgs a) {
@@ -167,15 +163,18 @@ __device__ __forceinline__ void bulk_store(void* dst, const void* src, uint32_t 
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async;" ::: "memory"); }
 
 // One warp per CTA (several CTAs per SM): claim a unit, load its moved source rows, publish, wait
-// for the earlier readers of this tile, store.  For key / value planes the rows move by TMA bulk
-// copies (one per run of consecutive sources, split at 32-row boundaries) into a shared-memory
-// stage and back out in one bulk store; the 4-byte metadata rows go through registers.  A CTA
-// never holds a claimed unit that it has not loaded and published while it waits on another one.
+// for the earlier readers of this tile, store.  The rows move by TMA bulk copies (one per run of
+// consecutive sources, split at 32-row boundaries) into a shared-memory stage and back out in one
+// bulk store; a K unit that owns metadata also gathers those words (plain loads into a second
+// stage) before it publishes and writes them after its wait, so they follow the same hazard rule
+// as its rows.  A CTA never holds a claimed unit that it has not loaded and published while it
+// waits on another one.
 __global__ void __launch_bounds__(32)
 compact_main_kernel(CompactArgs a)
 {
     extern __shared__ uint4 stage_raw[];
     uint8_t* stage = reinterpret_cast<uint8_t*>(stage_raw);
+    int32_t* mstage = reinterpret_cast<int32_t*>(stage + (size_t)a.tile_rows * a.row_bytes);   // [n_meta][TB]
     __shared__ uint64_t bar;
 
     grid_dep_wait();                                   // the prepass is done
@@ -188,6 +187,7 @@ compact_main_kernel(CompactArgs a)
     const int n_tiles = (n + a.tile_rows - 1) / a.tile_rows;
     const int units = (n_tiles - t0) * a.n_planes;
     const int lane = threadIdx.x;
+    const int rb = a.row_bytes;
     if (lane == 0) { mbar_init(&bar, 1); fence_barrier_init(); }
     __syncwarp();
 
@@ -200,48 +200,43 @@ compact_main_kernel(CompactArgs a)
         u = __shfl_sync(0xffffffffu, u, 0);
         if (u >= units) break;
         const int b = t0 + u / a.n_planes, p = u % a.n_planes;
-        int rb, list;
-        char* base = plane_base(a, p, rb, list);
+        int list;
+        bool owns_meta;
+        char* base = plane_base(a, p, list, owns_meta);
         const int32_t* retain_idx = a.retain_idx + (size_t)list * a.list_stride;
         const int j0 = b * a.tile_rows;
         const int j_end = min(j0 + a.tile_rows, n);
         const int js = max(j0, a.first[list]);                     // rows before the list's first stay
         if (js >= j_end) continue;                                 // (no unit ever waits for such a tile)
         const int nrows = j_end - js;
-        const bool kv = rb >= 16;
+        const size_t meta_off = (size_t)(a.n_lists == 1 ? 0 : list) * a.capacity;
 
         // ---- load the sources
-        bool ok = true;
-        if (kv) {
-            if (lane == 0) {
-                if (store_pending) bulk_wait_read0();              // the stage is free again
-                mbar_arrive_expect_tx(&bar, (uint32_t)nrows * rb);
-            }
-            __syncwarp();
-            for (int c0 = js; c0 < j_end; c0 += 32) {
-                const int r = c0 + lane;
-                const bool in = r < j_end;
-                const int src = in ? retain_idx[r] : 0;
-                int prev = __shfl_up_sync(0xffffffffu, src, 1);
-                const bool start = in && (lane == 0 || src != prev + 1);
-                const unsigned starts = __ballot_sync(0xffffffffu, start);
-                if (start) {
-                    const unsigned above = starts & ~((2u << lane) - 1u);   // later starts in this chunk
-                    const int stop = above ? c0 + __ffs(above) - 1 : min(c0 + 32, j_end);
-                    bulk_load(stage + (size_t)(r - j0) * rb, base + (size_t)src * rb, (uint32_t)(stop - r) * rb, &bar);
-                }
-            }
-            load_pending = true;
-            ok = mbar_wait_or_abort(&bar, phase, kWaitBudgetNs, abort_flag);
-            ok = __all_sync(0xffffffffu, ok) != 0;
-            if (ok) { phase ^= 1; load_pending = false; }
-        } else {                                                   // 4-byte rows via the stage
-            if (lane == 0 && store_pending) bulk_wait_read0();
-            __syncwarp();
-            int* st = reinterpret_cast<int*>(stage);
-            for (int r = js + lane; r < j_end; r += 32) st[r - j0] = reinterpret_cast<const int*>(base)[retain_idx[r]];
-            __syncwarp();
+        if (lane == 0) {
+            if (store_pending) bulk_wait_read0();                  // the stage is free again
+            mbar_arrive_expect_tx(&bar, (uint32_t)nrows * rb);
         }
+        __syncwarp();
+        for (int c0 = js; c0 < j_end; c0 += 32) {
+            const int r = c0 + lane;
+            const bool in = r < j_end;
+            const int src = in ? retain_idx[r] : 0;
+            int prev = __shfl_up_sync(0xffffffffu, src, 1);
+            const bool start = in && (lane == 0 || src != prev + 1);
+            const unsigned starts = __ballot_sync(0xffffffffu, start);
+            if (start) {
+                const unsigned above = starts & ~((2u << lane) - 1u);   // later starts in this chunk
+                const int stop = above ? c0 + __ffs(above) - 1 : min(c0 + 32, j_end);
+                bulk_load(stage + (size_t)(r - j0) * rb, base + (size_t)src * rb, (uint32_t)(stop - r) * rb, &bar);
+            }
+            if (owns_meta && in)
+                for (int m = 0; m < a.n_meta; ++m)
+                    mstage[m * a.tile_rows + (r - j0)] = reinterpret_cast<const int32_t*>(a.meta[m])[meta_off + src];
+        }
+        load_pending = true;
+        bool ok = mbar_wait_or_abort(&bar, phase, kWaitBudgetNs, abort_flag);
+        ok = __all_sync(0xffffffffu, ok) != 0;
+        if (ok) { phase ^= 1; load_pending = false; }
         if (!ok) {
             if (lane == 0) { atomicExch(&a.ctl->abort, 1); record_status(a.status, DELTAS_ERR_TIMEOUT, u); }
             break;
@@ -270,17 +265,17 @@ compact_main_kernel(CompactArgs a)
             break;
         }
 
-        // ---- store the tile (destination rows of a tile are contiguous)
-        if (kv) {
-            if (lane == 0) {
-                fence_proxy_async();
-                bulk_store(base + (size_t)js * rb, stage + (size_t)(js - j0) * rb, (uint32_t)nrows * rb);
-                bulk_commit();
-                store_pending = true;
-            }
-        } else {
-            const int* st = reinterpret_cast<const int*>(stage);
-            for (int r = js + lane; r < j_end; r += 32) reinterpret_cast<int*>(base)[r] = st[r - j0];
+        // ---- store the tile (destination rows of a tile are contiguous) and the metadata
+        if (lane == 0) {
+            fence_proxy_async();
+            bulk_store(base + (size_t)js * rb, stage + (size_t)(js - j0) * rb, (uint32_t)nrows * rb);
+            bulk_commit();
+            store_pending = true;
+        }
+        if (owns_meta) {
+            for (int r = js + lane; r < j_end; r += 32)
+                for (int m = 0; m < a.n_meta; ++m)
+                    reinterpret_cast<int32_t*>(a.meta[m])[meta_off + r] = mstage[m * a.tile_rows + (r - j0)];
             __syncwarp();                                          // the stage is rewritten next
         }
     }
@@ -407,7 +402,7 @@ CompactWsLayout compact_layout(const KvPlanes& kv, int cache_len, bool per_head)
     const size_t mt = max_tiles > 0 ? max_tiles : 1;
     const size_t n_kv = (size_t)kv.Lf * kv.Hkv;
     const size_t n_lists = per_head ? n_kv : 1;
-    const size_t n_planes = 2 * n_kv + (per_head ? 3 * n_kv : 2);
+    const size_t n_planes = 2 * n_kv;
     CompactWsLayout l;
     l.ctl = kStatusBytes;
     l.first = l.ctl + 256;
@@ -436,7 +431,7 @@ cudaError_t launch_compact(const KvPlanes& kv, bool per_head, const int32_t* ret
     a.capacity = kv.capacity;
     a.row_bytes = kv.D * elt_bytes(kv.dtype);
     a.tile_rows = tile_rows_for(a.row_bytes);
-    a.n_planes = 2 * a.n_kv_planes + a.n_meta * (per_head ? a.n_kv_planes : 1);
+    a.n_planes = 2 * a.n_kv_planes;
     a.cache_len = cache_len;
     a.max_tiles = (cache_len + a.tile_rows - 1) / a.tile_rows;
     a.retain_idx = retain_idx;
@@ -461,7 +456,7 @@ cudaError_t launch_compact(const KvPlanes& kv, bool per_head, const int32_t* ret
     e = launch_dependent(compact_need_kernel, dim3(need_blocks), dim3(256), 0, s, a);
     if (e != cudaSuccess) return e;
 
-    const int smem = a.tile_rows * a.row_bytes;
+    const int smem = a.tile_rows * (a.row_bytes + 4 * a.n_meta);
     int per_sm = 0;
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, compact_main_kernel, 32, smem);
     if (e != cudaSuccess) return e;

@@ -11,10 +11,11 @@
 //      candidate are kept in shared memory when the plane fits, else in the workspace; the slot
 //      part is the candidate's index;
 //   3. quota: for every span with more candidates than the quota q, a radix select (8-bit
-//      digits, most significant first, all spans in one pass over the candidates) narrows a key
-//      prefix until the candidates at or above it are exactly the span's best q: a span is done
-//      as soon as the digit bin it stops in is taken whole, so random scores resolve within the
-//      four score digits and the slot digits are read only for exact ties;
+//      digits, most significant first, starting at the highest bit in which two candidates'
+//      keys differ, all spans in one pass over the candidates) narrows a key prefix until the
+//      candidates at or above it are exactly the span's best q: a span is done as soon as the
+//      digit bin it stops in is taken whole, so distinct scores resolve within the score digits
+//      and the slot digits are read only for exact ties;
 //   4. fill: the same select over the candidates the quota left, as one group, for the
 //      remaining capacity R - kept;
 //   5. emit: every warp owns a contiguous stretch of slots; it counts its kept slots, a scan of
@@ -36,6 +37,7 @@ constexpr int kSlotBits = 24;                         // slots < 2^20 (DELTAS_SE
 constexpr int kKeyBits = 32 + kSlotBits;
 constexpr uint32_t kSlotMask = (1u << kSlotBits) - 1u;
 constexpr size_t kHeadSmemLimit = 220 * 1024;         // dynamic shared memory the kernel may ask for
+constexpr int kUnroll = 4;                            // candidates per lane per pass iteration
 
 enum HeadMode : int { kKeepAll = 0, kKeepNone = 1, kKeepSome = 2 };
 
@@ -65,6 +67,13 @@ __device__ __forceinline__ uint64_t cand_key(const uint32_t* keys, int c, int lo
     return ((uint64_t)keys[c] << kSlotBits) | (uint64_t)(kSlotMask - (uint32_t)(lo + c));
 }
 
+// (key(c) >> shift) >= prefix, in 32-bit arithmetic while the shift stays within the slot bits'
+// reach (the usual case: distinct scores resolve before the slot digits).
+__device__ __forceinline__ bool key_at_least(const uint32_t* keys, int c, int lo, int shift, uint64_t prefix) {
+    if (shift >= kSlotBits) return (uint64_t)(keys[c] >> (shift - kSlotBits)) >= prefix;
+    return (cand_key(keys, c, lo) >> shift) >= prefix;
+}
+
 // Per-group state of a block-wide radix select (shared memory).  A group j with mode kKeepSome
 // keeps the candidates c with (key(c) >> shift[j]) >= prefix[j]; `target` counts how many are
 // still to be found below the current prefix.
@@ -76,45 +85,77 @@ struct RadixGroups {
     int done[kHeadMaxSpans];
 };
 
-// Radix select for G groups at once.  group_of(c) returns the candidate's group, or -1 when the
-// candidate takes no part.  On return every group with mode kKeepSome has its (prefix, shift).
+// Adds one to hist[bin] for every lane with bin >= 0.  When the warp's active lanes share one
+// bin (the common case in the first digits, where most keys agree) a single atomic adds them all.
+__device__ __forceinline__ void hist_add(unsigned* hist, int bin, int lane) {
+    const unsigned act = __ballot_sync(0xffffffffu, bin >= 0);
+    if (act == 0) return;
+    const int leader = __ffs(act) - 1;
+    const int b0 = __shfl_sync(0xffffffffu, bin, leader);
+    if (__all_sync(0xffffffffu, bin < 0 || bin == b0)) {
+        if (lane == leader) atomicAdd(&hist[b0], (unsigned)__popc(act));
+    } else if (bin >= 0) {
+        atomicAdd(&hist[bin], 1u);
+    }
+}
+
+// Radix select for G groups at once over the candidates' 56-bit keys, whose bits above
+// `top_bits` are `top_prefix` for every candidate (so the digits start at the highest bit in
+// which two candidates differ).  group_of(c) returns the candidate's group, or -1 when it takes no
+// part.  Digits are 8 bits (the last one narrower), most significant first; two histogram buffers
+// alternate so that clearing the next one overlaps the scan of the current one.  On return every
+// group with mode kKeepSome has its (prefix, shift).
 template <typename GroupOf>
-__device__ void radix_select(const uint32_t* keys, int n_cand, int lo, int G, RadixGroups& rg, unsigned* hist,
-                             int* s_remaining, GroupOf group_of)
+__device__ void radix_select(const uint32_t* keys, int n_cand, int lo, int G, int top_bits, uint64_t top_prefix,
+                             RadixGroups& rg, unsigned* hist2, int* s_open, GroupOf group_of)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int j = threadIdx.x; j < G; j += kHeadThreads) {
-        rg.prefix[j] = 0;
-        rg.shift[j] = kKeyBits;
+        rg.prefix[j] = top_prefix;
+        rg.shift[j] = top_bits;
         rg.done[j] = rg.mode[j] != kKeepSome;
     }
+    for (int e = threadIdx.x; e < G * 256; e += kHeadThreads) hist2[e] = 0;
     __syncthreads();
-    for (int shift = kKeyBits - 8; shift >= 0; shift -= 8) {
-        if (threadIdx.x == 0) {
-            int left = 0;
-            for (int j = 0; j < G; ++j) left += rg.done[j] ? 0 : 1;
-            *s_remaining = left;
-        }
-        for (int e = threadIdx.x; e < G * 256; e += kHeadThreads) hist[e] = 0;
-        __syncthreads();
-        if (*s_remaining == 0) break;
-        for (int base = warp * 32; base < n_cand; base += kHeadThreads) {
-            const int c = base + lane;
-            int bin = -1;
-            if (c < n_cand) {
-                const int j = group_of(c);
-                if (j >= 0 && !rg.done[j]) {
-                    const uint64_t key = cand_key(keys, c, lo);
-                    if ((key >> (shift + 8)) == rg.prefix[j]) bin = j * 256 + (int)((key >> shift) & 255u);
+    if (threadIdx.x == 0) {
+        int open = 0;
+        for (int j = 0; j < G; ++j) open += rg.done[j] ? 0 : 1;
+        *s_open = open;
+    }
+    __syncthreads();
+    int bits = top_bits, buf = 0;
+    while (bits > 0 && *s_open > 0) {
+        const int w = min(8, bits), shift = bits - w;
+        const uint64_t dmask = (1ull << w) - 1ull;
+        unsigned* hist = hist2 + (size_t)buf * G * 256;
+        unsigned* next = hist2 + (size_t)(buf ^ 1) * G * 256;
+        // kUnroll candidates per lane and iteration: their loads are independent and overlap
+        for (int base = warp * 32 * kUnroll; base < n_cand; base += kHeadThreads * kUnroll) {
+            int bin[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int c = base + u * 32 + lane;
+                bin[u] = -1;
+                if (c < n_cand) {
+                    const int j = group_of(c);
+                    if (j >= 0 && !rg.done[j]) {
+                        if (shift >= kSlotBits) {                // score digits: 32-bit arithmetic
+                            const uint32_t k = keys[c];
+                            const int hs = bits - kSlotBits;
+                            const bool match = hs >= 32 || (uint64_t)(k >> hs) == rg.prefix[j];
+                            if (match) bin[u] = j * 256 + (int)((k >> (shift - kSlotBits)) & (uint32_t)dmask);
+                        } else {
+                            const uint64_t key = cand_key(keys, c, lo);
+                            if ((key >> bits) == rg.prefix[j]) bin[u] = j * 256 + (int)((key >> shift) & dmask);
+                        }
+                    }
                 }
             }
-            const unsigned act = __ballot_sync(0xffffffffu, bin >= 0);
-            if (bin >= 0) {
-                const unsigned peers = __match_any_sync(act, bin);
-                if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], (unsigned)__popc(peers));
-            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) hist_add(hist, bin[u], lane);
         }
         __syncthreads();
+        for (int e = threadIdx.x; e < G * 256; e += kHeadThreads) next[e] = 0;
         // one warp per open group: lane l holds digits 255-8l .. 248-8l (descending across lanes)
         for (int j = warp; j < G; j += kHeadWarps) {
             if (rg.done[j]) continue;
@@ -141,13 +182,18 @@ __device__ void radix_select(const uint32_t* keys, int n_cand, int lo, int G, Ra
                     above += h;
                 }
                 const int need = (int)(target - above);           // 1 <= need <= hist[d]
-                rg.prefix[j] = (rg.prefix[j] << 8) | (uint64_t)d;
+                rg.prefix[j] = (rg.prefix[j] << w) | (uint64_t)d;
                 rg.shift[j] = shift;
                 rg.target[j] = need;
-                rg.done[j] = (unsigned)need == hj[d];           // the bin is taken whole
+                if ((unsigned)need == hj[d]) {                    // the bin is taken whole
+                    rg.done[j] = 1;
+                    atomicSub(s_open, 1);
+                }
             }
         }
         __syncthreads();
+        bits = shift;
+        buf ^= 1;
     }
 }
 
@@ -168,16 +214,16 @@ __device__ int scan_warp_counts(int* s_cnt, int* s_total) {
     return *s_total;
 }
 
-__global__ void __launch_bounds__(kHeadThreads)
+__global__ void __launch_bounds__(kHeadThreads, 1)
 select_heads_kernel(HeadArgs a)
 {
     extern __shared__ uint4 smem_raw[];
     __shared__ RadixGroups rg;
     __shared__ int s_cnt[kHeadMaxSpans];
-    __shared__ int s_min, s_max, s_bad, s_remaining, s_total, s_fill_mode;
+    __shared__ int s_min, s_max, s_bad, s_open, s_total, s_fill;
+    __shared__ unsigned s_kmin, s_kmax;
+    __shared__ long long s_thr[kHeadMaxSpans];
     __shared__ int s_warp[kHeadWarps];
-    __shared__ uint64_t s_fill_prefix;
-    __shared__ int s_fill_shift;
 
     const int p = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -200,14 +246,24 @@ select_heads_kernel(HeadArgs a)
     const int R = a.M - a.n_s - a.n_w, N = a.N, q = R / N;
 
     // ---- 1. candidate chunk range; every chunk id must be >= 0
-    if (tid == 0) { s_min = INT_MAX; s_max = INT_MIN; s_bad = 0; }
+    if (tid == 0) { s_min = INT_MAX; s_max = INT_MIN; s_bad = 0; s_kmin = 0xffffffffu; s_kmax = 0u; }
+    if (tid < kHeadMaxSpans) s_cnt[tid] = 0;
     __syncthreads();
     {
         int mn = INT_MAX, mx = INT_MIN, bad = 0;
-        for (int i = tid; i < T; i += kHeadThreads) {
-            const int c = tok_chunk[i];
-            bad |= c < 0;
-            if (i >= lo && i < hi) { mn = min(mn, c); mx = max(mx, c); }
+        for (int i0 = tid; i0 < T; i0 += 4 * kHeadThreads) {
+            int c[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {                  // four independent loads in flight
+                const int i = i0 + u * kHeadThreads;
+                c[u] = i < T ? tok_chunk[i] : 0;
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int i = i0 + u * kHeadThreads;
+                bad |= c[u] < 0;
+                if (i >= lo && i < hi) { mn = min(mn, c[u]); mx = max(mx, c[u]); }
+            }
         }
 #pragma unroll
         for (int m = 16; m >= 1; m >>= 1) {
@@ -217,14 +273,17 @@ select_heads_kernel(HeadArgs a)
         }
         if (lane == 0) { atomicMin(&s_min, mn); atomicMax(&s_max, mx); if (bad) atomicOr(&s_bad, 1); }
     }
-    if (tid < kHeadMaxSpans) s_cnt[tid] = 0;
     __syncthreads();
     if (s_bad) {                                       // outputs unspecified; report and stop
         if (tid == 0) record_status(a.status, DELTAS_ERR_DEVICE_INDEX, p);
         return;
     }
-    const int c_lo = s_min;
-    const long long span_len = (long long)s_max - c_lo + 1;
+    // span(a) = floor((a - c_lo) * N / (c_hi - c_lo + 1)) >= j  <=>  a >= c_lo + ceil(j * len / N):
+    // the N - 1 span starts, so that a candidate's span is a search instead of a 64-bit division
+    if (tid > 0 && tid < N) {
+        const long long len = (long long)s_max - s_min + 1;
+        s_thr[tid] = (long long)s_min + ((long long)tid * len + N - 1) / N;
+    }
 
     // ---- 2. keys and spans of the candidates, span counts
     uint32_t* keys;
@@ -233,28 +292,67 @@ select_heads_kernel(HeadArgs a)
     if (a.keys_in_smem) {
         keys = reinterpret_cast<uint32_t*>(smem_raw);
         spans = reinterpret_cast<uint8_t*>(keys + n_cand);
-        hist = reinterpret_cast<unsigned*>(smem_raw) + ((size_t)n_cand * 5 + 15) / 16 * 4;
+        hist = reinterpret_cast<unsigned*>(smem_raw) + ((size_t)n_cand * 5 + 15) / 16 * 4;   // 2 x N x 256
     } else {
         keys = a.ws_keys + (size_t)p * a.cache_len;
         spans = a.ws_spans + (size_t)p * a.cache_len;
         hist = reinterpret_cast<unsigned*>(smem_raw);
     }
-    for (int base = warp * 32; base < n_cand; base += kHeadThreads) {
-        const int c = base + lane;
-        int j = -1;
-        if (c < n_cand) {
-            const int i = lo + c;
-            j = (int)(((long long)(tok_chunk[i] - c_lo) * N) / span_len);
-            keys[c] = score_order_bits(tok_score[i]);
-            spans[c] = (uint8_t)j;
+    __syncthreads();
+    {
+        unsigned kmin = 0xffffffffu, kmax = 0u;
+        for (int base = warp * 32 * kUnroll; base < n_cand; base += kHeadThreads * kUnroll) {
+            int ch[kUnroll];
+            float sc[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {                // all loads first
+                const int c = base + u * 32 + lane;
+                ch[u] = c < n_cand ? tok_chunk[lo + c] : 0;
+                sc[u] = c < n_cand ? tok_score[lo + c] : 0.f;
+            }
+            int jj[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int c = base + u * 32 + lane;
+                jj[u] = -1;
+                if (c < n_cand) {
+                    const uint32_t k = score_order_bits(sc[u]);
+                    int l = 0, h = N - 1;                  // largest j in [1, N) with ch >= start j
+                    while (l < h) {
+                        const int mid = (l + h + 1) >> 1;
+                        if ((long long)ch[u] >= s_thr[mid]) l = mid; else h = mid - 1;
+                    }
+                    jj[u] = l;
+                    keys[c] = k;
+                    spans[c] = (uint8_t)l;
+                    kmin = min(kmin, k);
+                    kmax = max(kmax, k);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) hist_add(reinterpret_cast<unsigned*>(s_cnt), jj[u], lane);
         }
-        const unsigned act = __ballot_sync(0xffffffffu, j >= 0);
-        if (j >= 0) {
-            const unsigned peers = __match_any_sync(act, j);
-            if (lane == __ffs(peers) - 1) atomicAdd(&s_cnt[j], __popc(peers));
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) {
+            kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, m));
+            kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, m));
         }
+        if (lane == 0) { atomicMin(&s_kmin, kmin); atomicMax(&s_kmax, kmax); }
     }
     __syncthreads();
+    // the digits start at the highest key bit in which two candidates differ: within the score
+    // bits, or within the slot bits when every candidate has the same score
+    int top_bits;
+    uint64_t top_prefix;
+    {
+        const uint32_t diff = s_kmin ^ s_kmax;
+        if (diff == 0) { top_bits = kSlotBits; top_prefix = s_kmin; }
+        else {
+            const int hb = 31 - __clz(diff);
+            top_bits = kSlotBits + hb + 1;
+            top_prefix = (uint64_t)(s_kmin >> hb) >> 1;
+        }
+    }
 
     // ---- 3. quota per span
     if (tid < N) {
@@ -263,53 +361,64 @@ select_heads_kernel(HeadArgs a)
         rg.target[tid] = q;
     }
     __syncthreads();
-    radix_select(keys, n_cand, lo, N, rg, hist, &s_remaining,
+    radix_select(keys, n_cand, lo, N, top_bits, top_prefix, rg, hist, &s_open,
                  [&](int c) -> int { return (int)spans[c]; });
     auto kept1 = [&](int c) -> bool {
-        const int j = spans[c];
+        const int j = spans[c] & 0x3f;
         const int m = rg.mode[j];
         if (m == kKeepAll) return true;
         if (m == kKeepNone) return false;
-        return (cand_key(keys, c, lo) >> rg.shift[j]) >= rg.prefix[j];
+        return key_at_least(keys, c, lo, rg.shift[j], rg.prefix[j]);
     };
 
     // ---- 4. fill: the remaining capacity from the best candidates the quota left.  The fill's
     // select reuses the group state, so the quota's outcome is first kept in the span byte
     // (bit 7 = kept by the quota; spans use bits 0..4).
-    for (int c = tid; c < n_cand; c += kHeadThreads)
-        if (kept1(c)) spans[c] |= 0x80u;
-    __syncthreads();
     if (tid == 0) {
         int kept = 0;
         for (int j = 0; j < N; ++j) kept += min(q, s_cnt[j]);
-        const int fill = R - kept;                     // < the candidates left, since n_cand > R
-        s_fill_mode = fill > 0 ? kKeepSome : kKeepNone;
-        rg.mode[0] = s_fill_mode;
-        rg.target[0] = fill;
+        s_fill = R - kept;                             // < the candidates left, since n_cand > R
     }
     __syncthreads();
-    if (s_fill_mode == kKeepSome)
-        radix_select(keys, n_cand, lo, 1, rg, hist, &s_remaining,
+    const int fill = s_fill;
+    if (fill > 0) {
+        for (int c0 = tid; c0 < n_cand; c0 += kHeadThreads * kUnroll) {
+            bool k[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int c = c0 + u * kHeadThreads;
+                k[u] = c < n_cand && kept1(c);
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u)
+                if (k[u]) spans[c0 + u * kHeadThreads] |= 0x80u;
+        }
+        __syncthreads();
+        if (tid == 0) { rg.mode[0] = kKeepSome; rg.target[0] = fill; }
+        __syncthreads();
+        radix_select(keys, n_cand, lo, 1, top_bits, top_prefix, rg, hist, &s_open,
                      [&](int c) -> int { return (spans[c] & 0x80u) ? -1 : 0; });
-    if (tid == 0) { s_fill_prefix = rg.prefix[0]; s_fill_shift = rg.shift[0]; }
-    __syncthreads();
-    const bool fill_on = s_fill_mode == kKeepSome;
-    const uint64_t fill_prefix = s_fill_prefix;
-    const int fill_shift = s_fill_shift;
+    }
+    const uint64_t fill_prefix = rg.prefix[0];
+    const int fill_shift = rg.shift[0];
     auto keep_slot = [&](int i) -> bool {
         if (i < lo || i >= hi) return true;
         const int c = i - lo;
+        if (fill <= 0) return kept1(c);
         if (spans[c] & 0x80u) return true;
-        return fill_on && (cand_key(keys, c, lo) >> fill_shift) >= fill_prefix;
+        return key_at_least(keys, c, lo, fill_shift, fill_prefix);
     };
 
-    // ---- 5. emit in slot order: warp w owns slots [w * seg, (w + 1) * seg)
+    // ---- 5. emit in slot order: warp w owns slots [w * seg, (w + 1) * seg).  The first pass
+    // counts and leaves each candidate's decision in bit 6 of its span byte for the second.
     const int seg = ((T + kHeadWarps - 1) / kHeadWarps + 31) & ~31;
     const int w0 = min(T, warp * seg), w1 = min(T, w0 + seg);
     int mine = 0;
     for (int i0 = w0; i0 < w1; i0 += 32) {
         const int i = i0 + lane;
-        mine += __popc(__ballot_sync(0xffffffffu, i < w1 && keep_slot(i)));
+        const bool k = i < w1 && keep_slot(i);
+        if (k && i >= lo && i < hi) spans[i - lo] |= 0x40u;
+        mine += __popc(__ballot_sync(0xffffffffu, k));
     }
     if (lane == 0) s_warp[warp] = mine;
     __syncthreads();
@@ -317,7 +426,7 @@ select_heads_kernel(HeadArgs a)
     int off = s_warp[warp];
     for (int i0 = w0; i0 < w1; i0 += 32) {
         const int i = i0 + lane;
-        const bool k = i < w1 && keep_slot(i);
+        const bool k = i < w1 && (i < lo || i >= hi || (spans[i - lo] & 0x40u));
         const unsigned b = __ballot_sync(0xffffffffu, k);
         const int at = off + __popc(b & ((1u << lane) - 1u));
         if (k && at < a.M) out[at] = i;
@@ -333,7 +442,7 @@ select_heads_kernel(HeadArgs a)
 }  // namespace
 
 size_t select_heads_smem_bytes(int n_cand, int N, bool keys_in_smem) {
-    const size_t hist = (size_t)(N < 1 ? 1 : N) * 256 * sizeof(unsigned);
+    const size_t hist = 2 * (size_t)(N < 1 ? 1 : N) * 256 * sizeof(unsigned);
     return (keys_in_smem ? ((size_t)n_cand * 5 + 15) / 16 * 16 : 0) + hist;
 }
 
