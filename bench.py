@@ -470,6 +470,13 @@ KERNEL_SOURCES = {"gdn_update": "paper_2609_27470_gb300/csrc/gdn_tc.cu",
                   "restore": "paper_2609_27470_gb300/csrc/snapshot.cu"}
 
 
+def kernel_source(workload, name):
+    """The source file of a timed kernel (the per-head selection has its own)."""
+    if name == "select" and _cfg(workload).get("signal") in ("key_norm", "value_norm"):
+        return "paper_2609_27470_gb300/csrc/select_heads.cu"
+    return KERNEL_SOURCES[name]
+
+
 class SnapshotWorkload:
     """Question-time snapshot and restore (Sec. 3.3) of a paper-shaped stream at its budget: the
     24 x 32 x 128 x 128 fp32 recurrent state (48 MiB), the 8,192-token caches of 8 layers x 4 KV
@@ -887,7 +894,7 @@ def main():
     if rl is not None:
         roofline = {"kernel": dominant, "bound": rl["bound"], "achieved": rl["achieved"], "peak": rl["peak"],
                     "unit": rl["unit"], "frac": rl["achieved"] / rl["peak"],
-                    "traffic": traffic_for(f"{args.workload}:{dominant}", KERNEL_SOURCES[dominant]),
+                    "traffic": traffic_for(f"{args.workload}:{dominant}", kernel_source(args.workload, dominant)),
                     "peak_source": f"{peaks_src} (hbm_gbs)",
                     "algorithmic_bytes_per_launch": rl["bytes_per_launch"]}
         if "tensor_frac" in rl:
