@@ -312,6 +312,18 @@ DELTAS_API deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, co
                                        const deltas_stream_buffers* src,
                                        const deltas_stream_buffers* dst, void* stream);
 
+/* The same for a stream ranked by a per-head token signal (deltas_*_heads): tok_chunk and tok_pos */
+/* of both sets are [Lf][Hkv][capacity] and every plane's entries 0 .. cache_len - 1 are copied,   */
+/* as are those of the token scores src_tok_score -> dst_tok_score ([Lf][Hkv][capacity] float).   */
+/* kv is required, and kv->capacity must be a multiple of 4 (each plane's metadata row then starts */
+/* on a 16-byte boundary); otherwise, and for the reasons above, INVALID_ARGUMENT.                 */
+DELTAS_API deltas_status deltas_copy_stream_state_heads(const deltas_gdn_desc* gdn, const deltas_kv_desc* kv,
+                                             int32_t cache_len, int32_t n_chunks,
+                                             const deltas_stream_buffers* src,
+                                             const deltas_stream_buffers* dst,
+                                             const float* src_tok_score, float* dst_tok_score,
+                                             void* stream);
+
 /* ------------------------------------------------------------------------------------------ */
 /* Per-head token signals (Sec. 4.3, the controlled comparison of retention signals, and the   */
 /* appendix table of signals).  Instead of one score per chunk, every cached token of every     */

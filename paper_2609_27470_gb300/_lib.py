@@ -39,7 +39,7 @@ EXPORTED = (
     "deltas_compact_kv_workspace_size", "deltas_compact_kv",
     "deltas_append_kv", "deltas_copy_stream_state",
     "deltas_append_kv_heads", "deltas_select_retain_heads_workspace_size", "deltas_select_retain_heads",
-    "deltas_compact_kv_heads_workspace_size", "deltas_compact_kv_heads",
+    "deltas_compact_kv_heads_workspace_size", "deltas_compact_kv_heads", "deltas_copy_stream_state_heads",
     "deltas_clear_device_status", "deltas_get_device_status",
 )
 
@@ -94,6 +94,7 @@ _sig("deltas_compact_kv_workspace_size", _SZ, _P, _I32)
 _sig("deltas_compact_kv", ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, _I32, _P, _SZ, _P)
 _sig("deltas_append_kv", ctypes.c_int, _P, _P, _P, _P, _P, _I32, _P, _P, _I32, _I32, _I32, _P)
 _sig("deltas_copy_stream_state", ctypes.c_int, _P, _P, _I32, _I32, _P, _P, _P)
+_sig("deltas_copy_stream_state_heads", ctypes.c_int, _P, _P, _I32, _I32, _P, _P, _P, _P, _P)
 _sig("deltas_append_kv_heads", ctypes.c_int, _P, _I32, _P, _P, _P, _P, _P, _I32, _P, _P, _I32, _I32, _I32, _P)
 _sig("deltas_select_retain_heads_workspace_size", _SZ, _I32, _I32)
 _sig("deltas_select_retain_heads", ctypes.c_int, _P, _I32, _I32, _I32, _P, _P, _P, _P, _P, _P, _SZ, _P)
@@ -384,13 +385,14 @@ class StreamBuffers(ctypes.Structure):
 
 
 def deltas_copy_stream_state(gdn: GdnDesc, kv: KvDesc | None, cache_len: int, n_chunks: int, src: dict, dst: dict,
-                             stream=None):
+                             stream=None, per_head: bool = False):
     """Copy a stream state between two buffer sets (dicts keyed by STREAM_BUFFERS; the cache
-    entries None when kv is None)."""
+    entries None when kv is None).  per_head: the metadata is [Lf, Hkv, capacity] and both dicts
+    also hold "tok_score" (deltas_copy_stream_state_heads)."""
     sshape = (gdn.num_layers, gdn.num_v_heads, gdn.value_dim, gdn.key_dim)
+    mshape = None if kv is None else ((kv.num_layers, kv.num_kv_heads, kv.capacity) if per_head else (kv.capacity,))
     shapes = {"state": (torch.float32, sshape), "chunk_scores": (torch.float32, None),
-              "tok_chunk": (torch.int32, (kv.capacity,) if kv else None),
-              "tok_pos": (torch.int32, (kv.capacity,) if kv else None)}
+              "tok_chunk": (torch.int32, mshape), "tok_pos": (torch.int32, mshape)}
     if kv is not None:
         cshape = (kv.num_layers, kv.num_kv_heads, kv.capacity, kv.head_dim)
         shapes["k_cache"] = shapes["v_cache"] = (_TORCH_DT[kv.dtype], cshape)
@@ -406,6 +408,16 @@ def deltas_copy_stream_state(gdn: GdnDesc, kv: KvDesc | None, cache_len: int, n_
         return StreamBuffers(*vals)
 
     s, d = pack(src, "src"), pack(dst, "dst")
+    if per_head:
+        if kv is None:
+            raise ValueError("a per-head stream state needs the kv descriptor")
+        st = _lib.deltas_copy_stream_state_heads(ctypes.byref(gdn), ctypes.byref(kv), int(cache_len), int(n_chunks),
+                                                 ctypes.byref(s), ctypes.byref(d),
+                                                 _ptr(src["tok_score"], torch.float32, mshape, "src tok_score"),
+                                                 _ptr(dst["tok_score"], torch.float32, mshape, "dst tok_score"),
+                                                 _stream(stream))
+        _check(st, "deltas_copy_stream_state_heads")
+        return
     st = _lib.deltas_copy_stream_state(ctypes.byref(gdn), ctypes.byref(kv) if kv is not None else None,
                                        int(cache_len), int(n_chunks), ctypes.byref(s), ctypes.byref(d),
                                        _stream(stream))

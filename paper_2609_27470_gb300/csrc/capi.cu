@@ -330,10 +330,13 @@ deltas_status deltas_compact_kv_heads(const deltas_kv_desc* desc, void* k_cache,
                                              static_cast<int32_t*>(workspace), as_stream(stream)));
 }
 
-deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, const deltas_kv_desc* kv,
-                                       int32_t cache_len, int32_t n_chunks,
-                                       const deltas_stream_buffers* src,
-                                       const deltas_stream_buffers* dst, void* stream)
+namespace {
+
+// One batch of copies for a stream state.  per_head: the metadata rows (and the token scores) are
+// [Lf][Hkv][capacity], one row of cache_len entries per plane, instead of one [capacity] row.
+deltas_status copy_stream_state(const deltas_gdn_desc* gdn, const deltas_kv_desc* kv, int32_t cache_len,
+                                int32_t n_chunks, const deltas_stream_buffers* src, const deltas_stream_buffers* dst,
+                                const float* src_tok_score, float* dst_tok_score, bool per_head, void* stream)
 {
     deltas_status st = check_gdn_desc(gdn);
     if (st != DELTAS_OK) return st;
@@ -351,7 +354,13 @@ deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, const deltas_
         if (cache_len < 0 || cache_len > kv->capacity) return DELTAS_ERR_INVALID_ARGUMENT;
         for (const void* p : cache_ptrs)
             if (p == nullptr || !aligned16(p)) return DELTAS_ERR_INVALID_ARGUMENT;
+        if (per_head) {             // per-plane metadata rows must start on 16-byte boundaries
+            if (!src_tok_score || !dst_tok_score || !aligned16(src_tok_score) || !aligned16(dst_tok_score))
+                return DELTAS_ERR_INVALID_ARGUMENT;
+            if (kv->capacity % 4 != 0) return DELTAS_ERR_INVALID_ARGUMENT;
+        }
     }
+    if (per_head && kv == nullptr) return DELTAS_ERR_INVALID_ARGUMENT;
     if (!aligned16(src->state) || !aligned16(dst->state)) return DELTAS_ERR_INVALID_ARGUMENT;
     if (n_chunks > 0 && (!aligned16(src->chunk_scores) || !aligned16(dst->chunk_scores)))
         return DELTAS_ERR_INVALID_ARGUMENT;
@@ -372,8 +381,11 @@ deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, const deltas_
         const int64_t planes = (int64_t)kv->num_layers * kv->num_kv_heads;
         add(src->k_cache, dst->k_cache, rb * cache_len, rb * kv->capacity, planes);
         add(src->v_cache, dst->v_cache, rb * cache_len, rb * kv->capacity, planes);
-        add(src->tok_chunk, dst->tok_chunk, (uint64_t)cache_len * 4, 0, 1);
-        add(src->tok_pos, dst->tok_pos, (uint64_t)cache_len * 4, 0, 1);
+        const int64_t meta_rows = per_head ? planes : 1;
+        const uint64_t meta_stride = per_head ? (uint64_t)kv->capacity * 4 : 0;
+        add(src->tok_chunk, dst->tok_chunk, (uint64_t)cache_len * 4, meta_stride, meta_rows);
+        add(src->tok_pos, dst->tok_pos, (uint64_t)cache_len * 4, meta_stride, meta_rows);
+        if (per_head) add(src_tok_score, dst_tok_score, (uint64_t)cache_len * 4, meta_stride, meta_rows);
     }
     // no destination range may overlap a source range or another destination range
     auto extent_end = [](const CopySeg& g) { return (uint64_t)(g.rows - 1) * g.stride + g.row_bytes; };
@@ -391,6 +403,25 @@ deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, const deltas_
         }
     }
     return from_cuda(launch_copy_batch(b, as_stream(stream)));
+}
+
+}  // namespace
+
+deltas_status deltas_copy_stream_state(const deltas_gdn_desc* gdn, const deltas_kv_desc* kv,
+                                       int32_t cache_len, int32_t n_chunks,
+                                       const deltas_stream_buffers* src,
+                                       const deltas_stream_buffers* dst, void* stream)
+{
+    return copy_stream_state(gdn, kv, cache_len, n_chunks, src, dst, nullptr, nullptr, false, stream);
+}
+
+deltas_status deltas_copy_stream_state_heads(const deltas_gdn_desc* gdn, const deltas_kv_desc* kv,
+                                             int32_t cache_len, int32_t n_chunks,
+                                             const deltas_stream_buffers* src,
+                                             const deltas_stream_buffers* dst,
+                                             const float* src_tok_score, float* dst_tok_score, void* stream)
+{
+    return copy_stream_state(gdn, kv, cache_len, n_chunks, src, dst, src_tok_score, dst_tok_score, true, stream);
 }
 
 deltas_status deltas_clear_device_status(void* workspace, void* stream) {

@@ -45,7 +45,7 @@ class StreamSnapshot:
         self.full = full
         self.buffers = {"state": torch.empty_like(s.state), "chunk_scores": torch.empty_like(s.chunk_scores)}
         if full:
-            for n in ("k_cache", "v_cache", "tok_chunk", "tok_pos"):
+            for n in ("k_cache", "v_cache", "tok_chunk", "tok_pos") + (("tok_score",) if s.per_head else ()):
                 self.buffers[n] = torch.empty_like(getattr(s, n))
         self.cache_len = self.position = self.chunk = self.evictions = 0
 
@@ -62,6 +62,8 @@ class DeltaSStream:
         self.gdn = L.gdn_desc(num_layers, num_k_heads, num_v_heads, head_dim, act_dtype, q_scale)
         self.policy = L.policy(budget_M, n_sink, n_window, n_buckets)
         self.capacity = budget_M + chunk_len
+        if signal in L.SIGNALS:          # per-plane metadata rows start on 16-byte boundaries
+            self.capacity = (self.capacity + 3) // 4 * 4
         self.kv = L.kv_desc(kv_layers, kv_heads, kv_head_dim, kv_dtype, self.capacity)
         self.chunk_len = chunk_len
         self.max_chunks = max_chunks
@@ -153,17 +155,17 @@ class DeltaSStream:
         b = {"state": self.state, "chunk_scores": self.chunk_scores}
         if full:
             b.update(k_cache=self.k_cache, v_cache=self.v_cache, tok_chunk=self.tok_chunk, tok_pos=self.tok_pos)
+            if self.per_head:
+                b["tok_score"] = self.tok_score
         return b
 
     def snapshot(self, full: bool = True, into: StreamSnapshot | None = None, stream=None) -> StreamSnapshot:
         """Save the stream state before a question (Sec. 3.3); ``into`` reuses a snapshot's buffers."""
-        if self.per_head:
-            raise ValueError("snapshot of a stream ranked by a per-head token signal is not supported")
         snap = into if into is not None else StreamSnapshot(self, full)
         if snap.full != full:
             raise ValueError("the snapshot's buffers were made for the other kind of snapshot")
         L.deltas_copy_stream_state(self.gdn, self.kv if full else None, self.cache_len, self.chunk,
-                                   self._buffers(full), snap.buffers, stream)
+                                   self._buffers(full), snap.buffers, stream, per_head=self.per_head and full)
         snap.cache_len, snap.position, snap.chunk, snap.evictions = (self.cache_len, self.position, self.chunk,
                                                                      self.evictions)
         return snap
@@ -173,6 +175,6 @@ class DeltaSStream:
         if not snap.full and self.evictions != snap.evictions:
             raise ValueError("the question evicted from the cache: only a full snapshot can restore it")
         L.deltas_copy_stream_state(self.gdn, self.kv if snap.full else None, snap.cache_len, snap.chunk,
-                                   snap.buffers, self._buffers(snap.full), stream)
+                                   snap.buffers, self._buffers(snap.full), stream, per_head=self.per_head and snap.full)
         self.cache_len, self.position, self.chunk, self.evictions = (snap.cache_len, snap.position, snap.chunk,
                                                                      snap.evictions)

@@ -25,7 +25,7 @@ def _declared():
 
 def test_every_declared_symbol_is_exported(L):
     names = _declared()
-    assert len(names) == 23, names
+    assert len(names) == 24, names
     lib = ctypes.CDLL(L.LIB_PATH)
     for n in names:
         assert hasattr(lib, n), n
@@ -152,6 +152,16 @@ def test_copy_stream_state_argument_checks(L):
     assert call(full(A), ov) == bad
     assert call(full(A), full(B), kvd=L.KvDesc(2, 2, 7, L.DELTAS_F32, 1000)) == L.DELTAS_ERR_UNSUPPORTED
     assert call(full(A), full(B), desc=L.GdnDesc(2, 2, 4, 24, 24, L.DELTAS_F32, 0.25)) == L.DELTAS_ERR_UNSUPPORTED
+
+    # the per-head variant (per-plane metadata and token scores)
+    def heads(src, dst, kvd=kv, ss=A + 6 * MB, ds=B + 6 * MB):
+        return raw.deltas_copy_stream_state_heads(ctypes.byref(gdn), ctypes.byref(kvd) if kvd else None, 500, 7,
+                                                  ctypes.byref(src), ctypes.byref(dst), ss, ds, None)
+    assert heads(full(A), full(B), kvd=None) == bad                       # the kv desc is required
+    assert heads(full(A), full(B), ss=None) == bad
+    assert heads(full(A), full(B), ds=B + 6 * MB + 4) == bad              # not 16-byte aligned
+    assert heads(full(A), full(B), kvd=L.KvDesc(2, 2, 64, L.DELTAS_BF16, 1002)) == bad   # capacity % 4
+    assert heads(full(A), full(B), ds=A + 6 * MB) == bad                  # scores copied onto themselves
 
 
 def test_write_norm_argument_checks(L):

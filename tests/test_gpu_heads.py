@@ -258,3 +258,78 @@ def test_stream_heads_matches_oracle(L, signal):
     # heads really differ in what they keep
     tp = s.tok_pos.cpu().numpy()
     assert not np.array_equal(tp[0, 0, :n], tp[0, 1, :n])
+
+
+def test_copy_stream_state_heads_is_exact(L):
+    """deltas_copy_stream_state_heads: every plane's first cache_len metadata entries and token
+    scores, the cache rows and the state are copied bit for bit; nothing past cache_len moves."""
+    dev = torch.device("cuda")
+    gdn = L.gdn_desc(2, 2, 4, 128, torch.bfloat16)
+    kv = L.kv_desc(2, 3, 256, torch.bfloat16, 1004)
+    gen = torch.Generator().manual_seed(91)
+
+    def rand_set():
+        shp = (2, 3, 1004)
+        return {"state": torch.randn(2, 4, 128, 128, generator=gen).to(dev),
+                "chunk_scores": torch.rand(40, generator=gen).to(dev),
+                "k_cache": torch.randn(*shp, 256, generator=gen).to(torch.bfloat16).to(dev),
+                "v_cache": torch.randn(*shp, 256, generator=gen).to(torch.bfloat16).to(dev),
+                "tok_chunk": torch.randint(0, 999, shp, generator=gen, dtype=torch.int32).to(dev),
+                "tok_pos": torch.randint(0, 1 << 20, shp, generator=gen, dtype=torch.int32).to(dev),
+                "tok_score": torch.randn(shp, generator=gen).to(dev)}
+    src, dst = rand_set(), rand_set()
+    before = {n: t.clone() for n, t in dst.items()}
+    n = 777
+    L.deltas_copy_stream_state(gdn, kv, n, 40, src, dst, per_head=True)
+    torch.cuda.synchronize()
+    assert torch.equal(dst["state"].view(torch.int32), src["state"].view(torch.int32))
+    for name in ("k_cache", "v_cache", "tok_chunk", "tok_pos", "tok_score"):
+        assert torch.equal(_bits(dst[name][:, :, :n]), _bits(src[name][:, :, :n])), name
+        assert torch.equal(_bits(dst[name][:, :, n:]), _bits(before[name][:, :, n:])), name
+
+
+@pytest.mark.parametrize("signal", ["key_norm", "value_norm"])
+def test_question_turn_in_a_head_stream_leaves_it_unchanged(L, signal):
+    """Sec. 3.3 question handling with a per-head signal: snapshot, a question chunk that updates
+    the state and evicts per plane, restore; the stream then equals a run without the question."""
+    from paper_2609_27470_gb300.stream import DeltaSStream
+    cfg = STREAM_CFG
+    dev = torch.device("cuda")
+    lens = cfg["lens"]
+    chunks = [inputs.gdn_chunk(cfg["L"], lens[c], cfg["Hk"], cfg["Hv"], cfg["d"], "bf16", inputs.seed_for(85, c))
+              for c in range(len(lens))]
+    kvs = [inputs.kv_chunk(cfg["Lf"], cfg["Hkv"], lens[c], cfg["D"], "bf16", inputs.seed_for(86, c))
+           for c in range(len(lens))]
+    qx = inputs.gdn_chunk(cfg["L"], 127, cfg["Hk"], cfg["Hv"], cfg["d"], "bf16", inputs.seed_for(87, 0))
+    qkv = inputs.kv_chunk(cfg["Lf"], cfg["Hkv"], 127, cfg["D"], "bf16", inputs.seed_for(88, 0))
+    s0 = inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 89)
+
+    def make():
+        return DeltaSStream(num_layers=cfg["L"], num_k_heads=cfg["Hk"], num_v_heads=cfg["Hv"], head_dim=cfg["d"],
+                            act_dtype=torch.bfloat16, kv_layers=cfg["Lf"], kv_heads=cfg["Hkv"], kv_head_dim=cfg["D"],
+                            kv_dtype=torch.bfloat16, budget_M=cfg["M"], n_sink=cfg["n_s"], n_window=cfg["n_w"],
+                            n_buckets=cfg["N"], chunk_len=max(lens), max_chunks=len(lens) + 1, state0=s0.to(dev),
+                            device=dev, signal=signal)
+
+    def feed(s, x, kv):
+        x = {k: v.to(dev) for k, v in x.items()}
+        s.step(x["q"], x["k"], x["v"], x["g"], x["beta"], kv[0].to(dev), kv[1].to(dev))
+    plain, asked = make(), make()
+    for c in range(len(lens)):
+        feed(plain, chunks[c], kvs[c])
+        if c == 7:
+            snap = asked.snapshot()
+            ev = asked.evictions
+            feed(asked, qx, qkv)
+            torch.cuda.synchronize()
+            assert asked.evictions == ev + 1
+            asked.restore(snap)
+        feed(asked, chunks[c], kvs[c])
+    torch.cuda.synchronize()
+    assert L.deltas_get_device_status(asked.workspace) == (0, 0)
+    assert (asked.cache_len, asked.position, asked.chunk, asked.evictions) == \
+        (plain.cache_len, plain.position, plain.chunk, plain.evictions)
+    n = asked.cache_len
+    assert torch.equal(asked.state.view(torch.int32), plain.state.view(torch.int32))
+    for name in ("k_cache", "v_cache", "tok_chunk", "tok_pos", "tok_score"):
+        assert torch.equal(_bits(getattr(asked, name)[:, :, :n]), _bits(getattr(plain, name)[:, :, :n])), name
