@@ -103,11 +103,15 @@ __device__ __forceinline__ void hist_add(unsigned* hist, int bin, int lane) {
 // `top_bits` are `top_prefix` for every candidate (so the digits start at the highest bit in
 // which two candidates differ).  group_of(c) returns the candidate's group, or -1 when it takes no
 // part.  Digits are 8 bits (the last one narrower), most significant first; two histogram buffers
-// alternate so that clearing the next one overlaps the scan of the current one.  On return every
-// group with mode kKeepSome has its (prefix, shift).
+// alternate so that clearing the next one overlaps the scan of the current one.  `prebuilt`: the
+// caller has already filled buffer 0 with the first digit's histogram (while it had every
+// candidate in hand anyway), and buffer 1 is zero.  On return every group with mode kKeepSome has
+// its (prefix, shift).
+__device__ __forceinline__ int first_digit_width(int top_bits) { return min(8, top_bits); }
+
 template <typename GroupOf>
 __device__ void radix_select(const uint32_t* keys, int n_cand, int lo, int G, int top_bits, uint64_t top_prefix,
-                             RadixGroups& rg, unsigned* hist2, int* s_open, GroupOf group_of)
+                             RadixGroups& rg, unsigned* hist2, int* s_open, bool prebuilt, GroupOf group_of)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int j = threadIdx.x; j < G; j += kHeadThreads) {
@@ -115,7 +119,8 @@ __device__ void radix_select(const uint32_t* keys, int n_cand, int lo, int G, in
         rg.shift[j] = top_bits;
         rg.done[j] = rg.mode[j] != kKeepSome;
     }
-    for (int e = threadIdx.x; e < G * 256; e += kHeadThreads) hist2[e] = 0;
+    if (!prebuilt)
+        for (int e = threadIdx.x; e < 2 * G * 256; e += kHeadThreads) hist2[e] = 0;
     __syncthreads();
     if (threadIdx.x == 0) {
         int open = 0;
@@ -124,13 +129,14 @@ __device__ void radix_select(const uint32_t* keys, int n_cand, int lo, int G, in
     }
     __syncthreads();
     int bits = top_bits, buf = 0;
+    bool have = prebuilt;
     while (bits > 0 && *s_open > 0) {
         const int w = min(8, bits), shift = bits - w;
         const uint64_t dmask = (1ull << w) - 1ull;
         unsigned* hist = hist2 + (size_t)buf * G * 256;
         unsigned* next = hist2 + (size_t)(buf ^ 1) * G * 256;
         // kUnroll candidates per lane and iteration: their loads are independent and overlap
-        for (int base = warp * 32 * kUnroll; base < n_cand; base += kHeadThreads * kUnroll) {
+        for (int base = warp * 32 * kUnroll; base < n_cand && !have; base += kHeadThreads * kUnroll) {
             int bin[kUnroll];
 #pragma unroll
             for (int u = 0; u < kUnroll; ++u) {
@@ -154,6 +160,7 @@ __device__ void radix_select(const uint32_t* keys, int n_cand, int lo, int G, in
 #pragma unroll
             for (int u = 0; u < kUnroll; ++u) hist_add(hist, bin[u], lane);
         }
+        have = false;
         __syncthreads();
         for (int e = threadIdx.x; e < G * 256; e += kHeadThreads) next[e] = 0;
         // one warp per open group: lane l holds digits 255-8l .. 248-8l (descending across lanes)
@@ -245,24 +252,31 @@ select_heads_kernel(HeadArgs a)
     const int lo = a.n_s, hi = T - a.n_w, n_cand = hi - lo;
     const int R = a.M - a.n_s - a.n_w, N = a.N, q = R / N;
 
-    // ---- 1. candidate chunk range; every chunk id must be >= 0
+    // ---- 1. candidate chunk range and score-key range; every chunk id must be >= 0
     if (tid == 0) { s_min = INT_MAX; s_max = INT_MIN; s_bad = 0; s_kmin = 0xffffffffu; s_kmax = 0u; }
     if (tid < kHeadMaxSpans) s_cnt[tid] = 0;
     __syncthreads();
     {
         int mn = INT_MAX, mx = INT_MIN, bad = 0;
+        unsigned kmin = 0xffffffffu, kmax = 0u;
         for (int i0 = tid; i0 < T; i0 += 4 * kHeadThreads) {
             int c[4];
+            float sc[4];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {                  // four independent loads in flight
+            for (int u = 0; u < 4; ++u) {                  // eight independent loads in flight
                 const int i = i0 + u * kHeadThreads;
                 c[u] = i < T ? tok_chunk[i] : 0;
+                sc[u] = (i >= lo && i < hi) ? tok_score[i] : 0.f;
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int i = i0 + u * kHeadThreads;
                 bad |= c[u] < 0;
-                if (i >= lo && i < hi) { mn = min(mn, c[u]); mx = max(mx, c[u]); }
+                if (i >= lo && i < hi) {
+                    mn = min(mn, c[u]); mx = max(mx, c[u]);
+                    const uint32_t k = score_order_bits(sc[u]);
+                    kmin = min(kmin, k); kmax = max(kmax, k);
+                }
             }
         }
 #pragma unroll
@@ -270,8 +284,13 @@ select_heads_kernel(HeadArgs a)
             mn = min(mn, __shfl_xor_sync(0xffffffffu, mn, m));
             mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, m));
             bad |= __shfl_xor_sync(0xffffffffu, bad, m);
+            kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, m));
+            kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, m));
         }
-        if (lane == 0) { atomicMin(&s_min, mn); atomicMax(&s_max, mx); if (bad) atomicOr(&s_bad, 1); }
+        if (lane == 0) {
+            atomicMin(&s_min, mn); atomicMax(&s_max, mx); if (bad) atomicOr(&s_bad, 1);
+            atomicMin(&s_kmin, kmin); atomicMax(&s_kmax, kmax);
+        }
     }
     __syncthreads();
     if (s_bad) {                                       // outputs unspecified; report and stop
@@ -284,62 +303,6 @@ select_heads_kernel(HeadArgs a)
         const long long len = (long long)s_max - s_min + 1;
         s_thr[tid] = (long long)s_min + ((long long)tid * len + N - 1) / N;
     }
-
-    // ---- 2. keys and spans of the candidates, span counts
-    uint32_t* keys;
-    uint8_t* spans;
-    unsigned* hist;
-    if (a.keys_in_smem) {
-        keys = reinterpret_cast<uint32_t*>(smem_raw);
-        spans = reinterpret_cast<uint8_t*>(keys + n_cand);
-        hist = reinterpret_cast<unsigned*>(smem_raw) + ((size_t)n_cand * 5 + 15) / 16 * 4;   // 2 x N x 256
-    } else {
-        keys = a.ws_keys + (size_t)p * a.cache_len;
-        spans = a.ws_spans + (size_t)p * a.cache_len;
-        hist = reinterpret_cast<unsigned*>(smem_raw);
-    }
-    __syncthreads();
-    {
-        unsigned kmin = 0xffffffffu, kmax = 0u;
-        for (int base = warp * 32 * kUnroll; base < n_cand; base += kHeadThreads * kUnroll) {
-            int ch[kUnroll];
-            float sc[kUnroll];
-#pragma unroll
-            for (int u = 0; u < kUnroll; ++u) {                // all loads first
-                const int c = base + u * 32 + lane;
-                ch[u] = c < n_cand ? tok_chunk[lo + c] : 0;
-                sc[u] = c < n_cand ? tok_score[lo + c] : 0.f;
-            }
-            int jj[kUnroll];
-#pragma unroll
-            for (int u = 0; u < kUnroll; ++u) {
-                const int c = base + u * 32 + lane;
-                jj[u] = -1;
-                if (c < n_cand) {
-                    const uint32_t k = score_order_bits(sc[u]);
-                    int l = 0, h = N - 1;                  // largest j in [1, N) with ch >= start j
-                    while (l < h) {
-                        const int mid = (l + h + 1) >> 1;
-                        if ((long long)ch[u] >= s_thr[mid]) l = mid; else h = mid - 1;
-                    }
-                    jj[u] = l;
-                    keys[c] = k;
-                    spans[c] = (uint8_t)l;
-                    kmin = min(kmin, k);
-                    kmax = max(kmax, k);
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < kUnroll; ++u) hist_add(reinterpret_cast<unsigned*>(s_cnt), jj[u], lane);
-        }
-#pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) {
-            kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, m));
-            kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, m));
-        }
-        if (lane == 0) { atomicMin(&s_kmin, kmin); atomicMax(&s_kmax, kmax); }
-    }
-    __syncthreads();
     // the digits start at the highest key bit in which two candidates differ: within the score
     // bits, or within the slot bits when every candidate has the same score
     int top_bits;
@@ -353,6 +316,60 @@ select_heads_kernel(HeadArgs a)
             top_prefix = (uint64_t)(s_kmin >> hb) >> 1;
         }
     }
+    const int dw1 = first_digit_width(top_bits), shift1 = top_bits - dw1;
+    const uint64_t dmask1 = (1ull << dw1) - 1ull;
+
+    // ---- 2. keys and spans of the candidates, span counts, and the quota's first-digit histogram
+    uint32_t* keys;
+    uint8_t* spans;
+    unsigned* hist;
+    if (a.keys_in_smem) {
+        keys = reinterpret_cast<uint32_t*>(smem_raw);
+        spans = reinterpret_cast<uint8_t*>(keys + n_cand);
+        hist = reinterpret_cast<unsigned*>(smem_raw) + ((size_t)n_cand * 5 + 15) / 16 * 4;   // 2 x N x 256
+    } else {
+        keys = a.ws_keys + (size_t)p * a.cache_len;
+        spans = a.ws_spans + (size_t)p * a.cache_len;
+        hist = reinterpret_cast<unsigned*>(smem_raw);
+    }
+    for (int e = tid; e < 2 * N * 256; e += kHeadThreads) hist[e] = 0;
+    __syncthreads();
+    for (int base = warp * 32 * kUnroll; base < n_cand; base += kHeadThreads * kUnroll) {
+        int ch[kUnroll];
+        float sc[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {                // all loads first
+            const int c = base + u * 32 + lane;
+            ch[u] = c < n_cand ? tok_chunk[lo + c] : 0;
+            sc[u] = c < n_cand ? tok_score[lo + c] : 0.f;
+        }
+        int jj[kUnroll], bin[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const int c = base + u * 32 + lane;
+            jj[u] = -1;
+            bin[u] = -1;
+            if (c < n_cand) {
+                const uint32_t k = score_order_bits(sc[u]);
+                int l = 0, h = N - 1;                      // largest j in [1, N) with ch >= start j
+                while (l < h) {
+                    const int mid = (l + h + 1) >> 1;
+                    if ((long long)ch[u] >= s_thr[mid]) l = mid; else h = mid - 1;
+                }
+                jj[u] = l;
+                keys[c] = k;
+                spans[c] = (uint8_t)l;
+                const uint64_t key = ((uint64_t)k << kSlotBits) | (uint64_t)(kSlotMask - (uint32_t)(lo + c));
+                bin[u] = l * 256 + (int)((key >> shift1) & dmask1);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            hist_add(reinterpret_cast<unsigned*>(s_cnt), jj[u], lane);
+            hist_add(hist, bin[u], lane);
+        }
+    }
+    __syncthreads();
 
     // ---- 3. quota per span
     if (tid < N) {
@@ -361,7 +378,7 @@ select_heads_kernel(HeadArgs a)
         rg.target[tid] = q;
     }
     __syncthreads();
-    radix_select(keys, n_cand, lo, N, top_bits, top_prefix, rg, hist, &s_open,
+    radix_select(keys, n_cand, lo, N, top_bits, top_prefix, rg, hist, &s_open, true,
                  [&](int c) -> int { return (int)spans[c]; });
     auto kept1 = [&](int c) -> bool {
         const int j = spans[c] & 0x3f;
@@ -373,30 +390,35 @@ select_heads_kernel(HeadArgs a)
 
     // ---- 4. fill: the remaining capacity from the best candidates the quota left.  The fill's
     // select reuses the group state, so the quota's outcome is first kept in the span byte
-    // (bit 7 = kept by the quota; spans use bits 0..4).
+    // (bit 7 = kept by the quota; spans use bits 0..4); the same pass builds the fill's first
+    // digit histogram over the candidates left.
     if (tid == 0) {
         int kept = 0;
         for (int j = 0; j < N; ++j) kept += min(q, s_cnt[j]);
         s_fill = R - kept;                             // < the candidates left, since n_cand > R
     }
+    for (int e = tid; e < 2 * 256; e += kHeadThreads) hist[e] = 0;
     __syncthreads();
     const int fill = s_fill;
     if (fill > 0) {
-        for (int c0 = tid; c0 < n_cand; c0 += kHeadThreads * kUnroll) {
-            bool k[kUnroll];
+        for (int base = warp * 32 * kUnroll; base < n_cand; base += kHeadThreads * kUnroll) {
+            int bin[kUnroll];
 #pragma unroll
             for (int u = 0; u < kUnroll; ++u) {
-                const int c = c0 + u * kHeadThreads;
-                k[u] = c < n_cand && kept1(c);
+                const int c = base + u * 32 + lane;
+                bin[u] = -1;
+                if (c < n_cand) {
+                    if (kept1(c)) spans[c] |= 0x80u;
+                    else bin[u] = (int)((cand_key(keys, c, lo) >> shift1) & dmask1);
+                }
             }
 #pragma unroll
-            for (int u = 0; u < kUnroll; ++u)
-                if (k[u]) spans[c0 + u * kHeadThreads] |= 0x80u;
+            for (int u = 0; u < kUnroll; ++u) hist_add(hist, bin[u], lane);
         }
-        __syncthreads();
+        __syncthreads();                               // every kept1() has read the quota's state
         if (tid == 0) { rg.mode[0] = kKeepSome; rg.target[0] = fill; }
         __syncthreads();
-        radix_select(keys, n_cand, lo, 1, top_bits, top_prefix, rg, hist, &s_open,
+        radix_select(keys, n_cand, lo, 1, top_bits, top_prefix, rg, hist, &s_open, true,
                      [&](int c) -> int { return (spans[c] & 0x80u) ? -1 : 0; });
     }
     const uint64_t fill_prefix = rg.prefix[0];
