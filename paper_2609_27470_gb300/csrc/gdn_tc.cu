@@ -129,13 +129,6 @@ __device__ __forceinline__ void split2(float a, float b, uint32_t& hi, uint32_t&
     lo = pack_bf16x2(a - hf.x, b - hf.y);
 }
 
-// fp32 -> the nearest tf32 value (ties away from zero), in an fp32 container
-__device__ __forceinline__ float round_tf32(float x) {
-    uint32_t y;
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(y) : "f"(x));
-    return __uint_as_float(y);
-}
-
 // D (16 x 8) += A (16 x 16, row) B (16 x 8, col) on the warp's tensor-core path, bf16 in, fp32
 // accumulate.  Fragments (g = lane / 4, t = lane % 4), each register a bf16 pair, lower k in the
 // low half: a = A[g][2t..], A[g+8][2t..], A[g][2t+8..], A[g+8][2t+8..]; b = B[2t..][g],

@@ -34,7 +34,6 @@ constexpr int kHeadThreads = 1024;
 constexpr int kHeadWarps = kHeadThreads / 32;
 constexpr int kHeadMaxSpans = 32;
 constexpr int kSlotBits = 24;                         // slots < 2^20 (DELTAS_SELECT_MAX_CACHE_LEN)
-constexpr int kKeyBits = 32 + kSlotBits;
 constexpr uint32_t kSlotMask = (1u << kSlotBits) - 1u;
 constexpr size_t kHeadSmemLimit = 220 * 1024;         // dynamic shared memory the kernel may ask for
 constexpr int kUnroll = 4;                            // candidates per lane per pass iteration
