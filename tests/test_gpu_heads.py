@@ -333,3 +333,74 @@ def test_question_turn_in_a_head_stream_leaves_it_unchanged(L, signal):
     assert torch.equal(asked.state.view(torch.int32), plain.state.view(torch.int32))
     for name in ("k_cache", "v_cache", "tok_chunk", "tok_pos", "tok_score"):
         assert torch.equal(_bits(getattr(asked, name)[:, :, :n]), _bits(getattr(plain, name)[:, :, :n])), name
+
+
+@pytest.mark.parametrize("signal", ["value_norm", "key_norm"])
+def test_paper_stream_per_head_full_size(L, signal):
+    """The paper-shaped stream ranked per KV head at full size, driven through the C ABI as the
+    benchmark drives it (8 full-attention layers x 4 KV heads x D = 256 bf16, chunks of 118-132
+    tokens cycling, budget 8192, sink 4, window 1024, 4 spans): filled past the budget, then every
+    chunk evicts.  Every eviction's 32 retain lists are checked bit for bit against the oracle's
+    selection on the chunk ids and scores read back right before it; after the last chunk every
+    plane keeps its sinks and window in stream order, sampled kept rows equal the rows they were
+    appended from, and every kept token's stored score is its signal recomputed from its row."""
+    from paper_2609_27470_gb300 import configs
+    from paper_2609_27470_gb300.stream import DeltaSStream
+    cfg = configs.PAPER
+    dev = torch.device("cuda")
+    Lf, Hkv, D, M = cfg["Lf"], cfg["Hkv"], cfg["D"], cfg["budget_M"]
+    n_s, n_w, N = cfg["n_sink"], cfg["n_window"], cfg["n_buckets"]
+    lens = [cfg["chunk_lens"][c % len(cfg["chunk_lens"])] for c in range(80)]       # about 66 fill, 14 evict
+    P = Lf * Hkv
+    s = DeltaSStream(num_layers=1, num_k_heads=1, num_v_heads=2, head_dim=128, act_dtype=torch.bfloat16,
+                     kv_layers=Lf, kv_heads=Hkv, kv_head_dim=D, kv_dtype=torch.bfloat16, budget_M=M, n_sink=n_s,
+                     n_window=n_w, n_buckets=N, chunk_len=max(lens), max_chunks=len(lens), device=dev,
+                     signal=signal)
+    kvs = [inputs.kv_chunk(Lf, Hkv, lens[c], D, "bf16", inputs.seed_for(95, c), device=dev) for c in range(len(lens))]
+    T, pos, evictions = 0, 0, 0
+    for c in range(len(lens)):
+        L.deltas_append_kv_heads(s.kv, signal, s.k_cache, s.v_cache, s.tok_chunk, s.tok_pos, s.tok_score, T,
+                                 kvs[c][0], kvs[c][1], c, pos)
+        T += lens[c]
+        pos += lens[c]
+        if T <= M:
+            continue
+        L.deltas_select_retain_heads(s.policy, T, s.tok_chunk.view(P, -1), s.tok_score.view(P, -1), s.retain_idx,
+                                     s.n_retained, None, s.workspace)
+        torch.cuda.synchronize()
+        tc_in = s.tok_chunk.view(P, -1)[:, :T].cpu().numpy()
+        ts_in = s.tok_score.view(P, -1)[:, :T].cpu().numpy()
+        ri = s.retain_idx.cpu().numpy()
+        assert s.n_retained.item() == M
+        for p in range(P):
+            idx, _ = oracle.select_retain_tokens(M, n_s, n_w, N, tc_in[p], ts_in[p])
+            assert np.array_equal(ri[p], idx), (c, p)
+        L.deltas_compact_kv_heads(s.kv, s.k_cache, s.v_cache, s.tok_chunk, s.tok_pos, s.tok_score, s.retain_idx,
+                                  s.n_retained, T, s.workspace)
+        T = M
+        evictions += 1
+    torch.cuda.synchronize()
+    assert L.deltas_get_device_status(s.workspace) == (0, 0)
+    assert evictions >= 10
+    n = T
+    tc = s.tok_chunk.view(P, -1)[:, :n].cpu().numpy()
+    tp = s.tok_pos.view(P, -1)[:, :n].cpu().numpy()
+    ts = s.tok_score.view(P, -1)[:, :n].cpu().numpy()
+    kc = s.k_cache.view(P, -1, D)[:, :n].cpu().view(torch.int16).numpy()
+    vc = s.v_cache.view(P, -1, D)[:, :n].cpu().view(torch.int16).numpy()
+    starts = np.cumsum([0] + lens)
+    for p in range(P):
+        assert np.all(np.diff(tp[p]) > 0) and tp[p][:n_s].tolist() == list(range(n_s))
+        assert tp[p][-n_w:].tolist() == list(range(starts[-1] - n_w, starts[-1]))
+        assert np.array_equal(tc[p], np.searchsorted(starts, tp[p], side="right") - 1)
+    rng = np.random.default_rng(97)
+    for p in [0, P - 1] + [int(x) for x in rng.integers(0, P, size=2)]:
+        l, h = divmod(p, Hkv)
+        for j in rng.integers(0, n, size=64):
+            c = int(tc[p, j])
+            r = int(tp[p, j] - starts[c])
+            assert np.array_equal(kc[p, j], kvs[c][0][l, h, r].cpu().view(torch.int16).numpy())
+            assert np.array_equal(vc[p, j], kvs[c][1][l, h, r].cpu().view(torch.int16).numpy())
+        src = (kc if signal == "key_norm" else vc)[p]
+        ref = oracle.row_norm_scores((src.astype(np.int32) << 16).view(np.float32), signal)
+        np.testing.assert_allclose(ts[p], ref, rtol=SCORE_RTOL, atol=0)
