@@ -66,6 +66,7 @@
 // TMEM (512 columns, M = 128 lanes = d_v): S~ [0,128), S_before [128,256), X [256,320) (X, then
 // W hi / lo packed in place), U [320,384) (likewise U~), V^T [384,448); [448,512) unused.
 #include <algorithm>
+#include <cmath>
 
 #include "internal.cuh"
 #include "tc_ptx.cuh"
@@ -253,6 +254,8 @@ struct WyArgs {
     const float* beta;
     uint8_t* rec;              // [L * Hv][n_tiles] records of kRecBytes
     int32_t* status;
+    int32_t* ho_flags;         // the update kernel's hand-over flags, reset here for this call
+    int n_ho_flags;
 };
 
 __global__ void __launch_bounds__(kWyThreads, kWyCtasPerSm)
@@ -264,6 +267,9 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
     grid_dep_launch();                                // the update kernel may take SMs as they free up
+    // the update kernel reads its hand-over flags only after this kernel has completed
+    if (blockIdx.x == 0)
+        for (int e = (int)threadIdx.x; e < a.n_ho_flags; e += kWyThreads) a.ho_flags[e] = 0;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int n = a.n_tiles;
     const int items = a.L * a.Hv * n;                 // item = (layer * Hv + head) * n + tile
@@ -612,6 +618,19 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
 // =============================================================================================
 // Update kernel: the state chain
 // =============================================================================================
+__device__ __forceinline__ int ho_load_acquire(const int32_t* p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void ho_store_release(int32_t* p, int v) {
+    asm volatile("st.release.gpu.global.b32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+// orders the tensor copies' global accesses with the generic ones around a hand-over flag
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 constexpr int kChainWarps = 16;
 constexpr int kChain = 32 * kChainWarps;         // chain threads
 constexpr int kMmaWarp = kChainWarps;            // 16
@@ -650,25 +669,83 @@ struct TcArgs {
     float* wnorm;
     const uint8_t* rec;
     int32_t* status;
+    int split;               // run equal tile runs (ChainSched), when the host found it faster
+    // hand-over between neighbouring CTAs of a head split between them (see ChainSched): one
+    // entry per CTA boundary i (CTA i -> CTA i + 1)
+    int32_t* ho_flag;        // [grid] the state after the first part is in the hand-over map
+    int32_t* ho_wflag;       // [grid] the first part's write-size sum is in ho_wsum
+    float* ho_wsum;          // [grid]
 };
 
-// Where a global tile lies: tile jt of head lh = (layer l, value head h), key head kh.  Each role
-// walks the tiles in order; a step costs integer divisions only when it crosses into the next head.
+// The CTA's work: a sequence of slots, each a run of consecutive tiles of one head.  By default
+// the CTA owns heads blockIdx.x, blockIdx.x + gridDim.x, ... whole.  When the heads do not divide
+// evenly among the CTAs and the host estimates it faster (a.split), the CTAs instead take equal
+// runs of the tile sequence in head order, so that the slowest CTA has one tile more than the
+// fastest instead of a whole head more; a head cut by a run boundary is shared by two neighbours.  CTA i runs the head
+// it shares with CTA i + 1 first (its first tiles; the state at the cut goes to hand-over entry i)
+// and the head it shares with CTA i - 1 last (its last tiles, from hand-over entry i - 1), so the
+// second part of a shared head is never waited for before its first part is long finished.
+struct ChainSched {
+    int split;
+    int pre_lh, pre_len;       // first slot: tiles [0, pre_len) of head pre_lh (none if pre_len == 0)
+    int full0, n_full;         // then n_full whole heads from full0 (every gridDim.x-th if !split)
+    int suf_lh, suf_from;      // last slot: tiles [suf_from, n) of head suf_lh (none if suf_from == 0)
+    int n_slots, NJ;
+    __device__ void init(const TcArgs& a) {
+        const int n = a.n_tiles, G = (int)gridDim.x, i = (int)blockIdx.x, H = a.L * a.Hv;
+        split = a.split && H > G && H % G != 0;
+        if (!split) {
+            pre_lh = suf_lh = -1; pre_len = suf_from = 0;
+            full0 = i; n_full = n_slots = (H - i + G - 1) / G; NJ = n_slots * n;
+            return;
+        }
+        const long long W = (long long)H * n;
+        const long long b0 = W * i / G, b1 = W * (i + 1) / G;   // at least n tiles apart (H > G)
+        const int hA = (int)(b0 / n), tA = (int)(b0 - (long long)hA * n);
+        const int hB = (int)(b1 / n), tB = (int)(b1 - (long long)hB * n);
+        suf_lh = hA; suf_from = tA;
+        full0 = tA > 0 ? hA + 1 : hA;
+        pre_lh = hB; pre_len = tB;
+        n_full = hB - full0;
+        n_slots = (pre_len > 0 ? 1 : 0) + n_full + (suf_from > 0 ? 1 : 0);
+        NJ = (int)(b1 - b0);
+    }
+    __device__ __forceinline__ bool is_prefix(int k) const { return pre_len > 0 && k == 0; }
+    __device__ __forceinline__ bool is_suffix(int k) const { return suf_from > 0 && k == n_slots - 1; }
+    __device__ void slot(int k, int n, int& lh, int& tb, int& te) const {
+        tb = 0; te = n;
+        if (!split) { lh = full0 + k * (int)gridDim.x; return; }
+        if (is_prefix(k)) { lh = pre_lh; te = pre_len; return; }
+        if (is_suffix(k)) { lh = suf_lh; tb = suf_from; return; }
+        lh = full0 + k - (pre_len > 0 ? 1 : 0);
+    }
+};
+
+// Where the CTA's current tile lies: slot k, tile jt (of [tb, te)) of head lh = (layer l, value
+// head h), key head kh.  Each role walks the tiles in order; a step costs integer divisions only
+// when it crosses into the next slot.
 struct TileCursor {
-    int jt, lh, l, h, kh;
-    __device__ __forceinline__ void set_head(int head, const TcArgs& a) {
-        lh = head; l = head / a.Hv; h = head - l * a.Hv;
+    int k, jt, te, lh, l, h, kh;
+    __device__ __forceinline__ void set_slot(int slot, const ChainSched& sc, const TcArgs& a) {
+        int tb;
+        k = slot;
+        sc.slot(slot, a.n_tiles, lh, tb, te);
+        jt = tb;
+        l = lh / a.Hv; h = lh - l * a.Hv;
         kh = (int)(((long long)h * a.Hk) / a.Hv);
     }
-    __device__ __forceinline__ void init(const TcArgs& a) { jt = 0; set_head((int)blockIdx.x, a); }
-    __device__ __forceinline__ void next(int n, const TcArgs& a) {
-        if (++jt == n) { jt = 0; set_head(lh + (int)gridDim.x, a); }
+    __device__ __forceinline__ void init(const ChainSched& sc, const TcArgs& a) {
+        if (sc.n_slots > 0) set_slot(0, sc, a);
+    }
+    __device__ __forceinline__ void next(const ChainSched& sc, const TcArgs& a) {
+        if (++jt == te && k + 1 < sc.n_slots) set_slot(k + 1, sc, a);
     }
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
 gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                     const __grid_constant__ CUtensorMap smap, TcArgs a)
+                     const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap hmap,
+                     TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
@@ -685,11 +762,12 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int n = a.n_tiles;
-    // Persistent CTA: it owns heads blockIdx.x, blockIdx.x + gridDim.x, ...  Their tiles form one
-    // sequence J = head slot * n + tile, over which every role keeps its barrier phases.
-    const int n_heads = a.L * a.Hv;
-    const int n_slots = (n_heads - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
-    const int NJ = n_slots * n;
+    // Persistent CTA: its slots (ChainSched) form one sequence of NJ tiles, over which every role
+    // keeps its barrier phases.
+    ChainSched sch;
+    sch.init(a);
+    const int n_slots = sch.n_slots;
+    const int NJ = sch.NJ;
 
     if (warp == kMmaWarp) {
         tmem_alloc(&s_tmem, kTmemCols);
@@ -709,7 +787,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         }
     }
     if (warp == kLoadWarp && lane == 0) { prefetch_tensormap(&kmap); prefetch_tensormap(&vmap); }
-    if (warp == kStateWarp && lane == 0) prefetch_tensormap(&smap);
+    if (warp == kStateWarp && lane == 0) { prefetch_tensormap(&smap); prefetch_tensormap(&hmap); }
     if (tid < kChain) {
         // the 64 x 64 identity (B operand of V^T I): row t holds 1.0 at column t
         const int t = tid >> 3, c8 = tid & 7;
@@ -839,7 +917,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         // =========================================================== K, V, records in tile order,
         // each into its buffer once the MMA that last read the buffer has completed
         TileCursor cc;
-        cc.init(a);
+        cc.init(sch, a);
         int kp[3] = {-1, -1, -1}, vp[2] = {-1, -1}, rp[2] = {-1, -1};   // last tile loaded per buffer
         // the kernel may start while the factor kernel finishes (its set-up and the first state
         // load overlap that tail); the records it wrote are read only after it has completed
@@ -872,7 +950,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             }
             __syncwarp();
             rp[b2] = J;
-            cc.next(n, a);
+            cc.next(sch, a);
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0) && lane == 0) {
             // every copy this warp issued lands before the CTA ends
@@ -886,36 +964,80 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         __syncwarp();
     } else if (warp == kStateWarp) {
         // =========================================================== state moves (lane 0).  Phases
-        // of mb_st: 0 = the first head's state staged; k + 1 = what the boundary after slot k
-        // needs: the state of slot k + 1, or (after the last slot's) a free buffer.  Phases of
-        // mb_sfree: 0 = the first state is in TMEM; k + 1 = S_after of slot k is staged.
+        // of mb_st: 0 = the first slot's state staged; k + 1 = what the boundary after slot k
+        // needs: the state of slot k + 1, or after the last slot a free buffer (when the last slot
+        // ends a head begun by CTA i - 1: that head's state before the chunk, for its drift).
+        // Phases of mb_sfree: 0 = the first state is in TMEM; k + 1 = slot k's final state is
+        // staged.  A first slot that begins a head shared with CTA i + 1 leaves its state in
+        // hand-over entry i; a last slot that ends a head shared with CTA i - 1 starts from entry
+        // i - 1, once that entry's flag is set (bounded wait).
         if (lane == 0 && n_slots > 0) {
             float* sbuf = reinterpret_cast<float*>(sm + SM_SB);
+            const int me = (int)blockIdx.x;
             int loads = 0, seen = 0;                   // copies into the staging buffer issued / landed
-            auto load_state = [&](int slot) {
-                const int lh = (int)blockIdx.x + slot * (int)gridDim.x;
+            auto load_rows = [&](const CUtensorMap* map, int row) {
                 mbar_arrive_expect_tx(&mb_st, kD * kD * 4);
 #pragma unroll
-                for (int b = 0; b < 4; ++b) tma_load_2d(sbuf + 4096 * b, &smap, &mb_st, 32 * b, lh * kD);
+                for (int b = 0; b < 4; ++b) tma_load_2d(sbuf + 4096 * b, map, &mb_st, 32 * b, row);
                 ++loads;
             };
-            load_state(0);
-            bool ok = mbar_wait_or_abort(&mb_sfree, 0, kWaitBudgetNs, abort_flag);
-            if (!ok) fail(a.status, abort_flag, 40);
+            auto load_state = [&](int slot) -> bool {
+                int lh, tb, te;
+                sch.slot(slot, n, lh, tb, te);
+                if (!sch.is_suffix(slot)) { load_rows(&smap, lh * kD); return true; }
+                grid_dep_wait();                       // the factor kernel reset the flags
+                const uint64_t t0 = global_ns();
+                while (ho_load_acquire(a.ho_flag + me - 1) == 0) {
+                    if (*abort_flag || global_ns() - t0 > kWaitBudgetNs) return false;
+                    __nanosleep(64);
+                }
+                fence_proxy_async_global();
+                load_rows(&hmap, (me - 1) * kD);
+                return true;
+            };
+            auto final_phase = [&]() {                 // what the boundary after the last slot reads
+                if (sch.is_suffix(n_slots - 1)) load_rows(&smap, sch.suf_lh * kD);
+                else mbar_arrive(&mb_st);
+            };
+            bool ok = load_state(0);
+            if (!ok) fail(a.status, abort_flag, 42);
+            if (ok) {
+                ok = mbar_wait_or_abort(&mb_sfree, 0, kWaitBudgetNs, abort_flag);
+                if (!ok) fail(a.status, abort_flag, 40);
+            }
             seen = loads;                              // the chain has consumed it
             if (ok) {
-                if (n_slots > 1) load_state(1); else mbar_arrive(&mb_st);
+                if (n_slots > 1) {
+                    ok = load_state(1);
+                    if (!ok) fail(a.status, abort_flag, 43);
+                } else {
+                    final_phase();
+                }
             }
             for (int k = 0; ok && k < n_slots; ++k) {
                 if (!mbar_wait_or_abort(&mb_sfree, (k + 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 41); break; }
                 seen = loads;
-                const int lh = (int)blockIdx.x + k * (int)gridDim.x;
+                int lh, tb, te;
+                sch.slot(k, n, lh, tb, te);
+                const bool hand_over = sch.is_prefix(k);
+                const CUtensorMap* dst = hand_over ? &hmap : &smap;
+                const int row = (hand_over ? me : lh) * kD;
 #pragma unroll
-                for (int b = 0; b < 4; ++b) tma_store_2d(&smap, sbuf + 4096 * b, 32 * b, lh * kD);
+                for (int b = 0; b < 4; ++b) tma_store_2d(dst, sbuf + 4096 * b, 32 * b, row);
                 bulk_commit();
+                if (hand_over) {
+                    bulk_wait0();                      // the state is in global memory ...
+                    fence_proxy_async_global();
+                    __threadfence();
+                    ho_store_release(a.ho_flag + me, 1);   // ... before CTA i + 1 may read it
+                }
                 if (k + 2 <= n_slots) {
-                    bulk_wait_read0();                 // S_after(k) has left the buffer
-                    if (k + 2 < n_slots) load_state(k + 2); else mbar_arrive(&mb_st);
+                    bulk_wait_read0();                 // slot k's state has left the buffer
+                    if (k + 2 < n_slots) {
+                        if (!load_state(k + 2)) { fail(a.status, abort_flag, 43); break; }
+                    } else {
+                        final_phase();
+                    }
                 }
             }
             bulk_wait0();                              // every state store is complete
@@ -930,7 +1052,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         float* sbuf = reinterpret_cast<float*>(sm + SM_SB);   // swizzled rows, see sb_idx
         int st_seen = 0;                                 // mb_st phases waited for (uniform)
         TileCursor cc;                                   // the chain's tile
-        cc.init(a);
+        cc.init(sch, a);
+        const int me = (int)blockIdx.x;
         // K(jj) (TMA tile, buffer jj % 3) in fp32 (exact, and exact in tf32) into the B operand
         // buffer of X.  Called between MMA_X(jj-1), the last reader of the buffer, and the ready
         // signal of tile jj.
@@ -975,8 +1098,29 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         // sums them over the tile's tokens into the head's total.
         const bool want_w = a.wnorm != nullptr;
         float wacc = 0.f;                                  // warp 0: the head's running sum
-        int prev_lh = -1;
+        int prev_lh = -1, prev_slot = -1;
         bool prev_last = false;
+        // a head's write-size sum: to hand-over entry i when the slot begins a head shared with
+        // CTA i + 1, else (with the first part's sum from entry i - 1 when it ends a head shared
+        // with CTA i - 1) to the output; warp 0, lane 0
+        auto put_wsum = [&](int slot, int lh, float sum) -> bool {
+            if (sch.is_prefix(slot)) {
+                a.ho_wsum[me] = sum;
+                __threadfence();
+                ho_store_release(a.ho_wflag + me, 1);
+                return true;
+            }
+            if (sch.is_suffix(slot)) {
+                const uint64_t t0 = global_ns();
+                while (ho_load_acquire(a.ho_wflag + me - 1) == 0) {
+                    if (*abort_flag || global_ns() - t0 > kWaitBudgetNs) return false;
+                    __nanosleep(64);
+                }
+                sum += *reinterpret_cast<volatile const float*>(a.ho_wsum + me - 1);
+            }
+            a.wnorm[lh] = sum;
+            return true;
+        };
         auto fold_writes = [&](int jj) {                   // warp 0: tile jj's sizes into wacc
             float* b = s_u2[jj & 1];
             float sacc = sqrtf(b[lane]) + sqrtf(b[lane + 32]);
@@ -987,8 +1131,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             wacc += sacc;
         };
         for (int j = 0; j < NJ; ++j) {                     // j: global tile index
-            const int lh = cc.lh, jt = cc.jt;              // head and tile within the head
-            const bool last = jt == n - 1;
+            const int lh = cc.lh, jt = cc.jt, slot = cc.k; // head, tile within the head, slot
+            const bool last = jt == cc.te - 1;             // the slot's last tile
             if (named_sync_or(2, kChain, *abort_flag)) break;
             if (!mbar_wait_or_abort(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
             const float gC = rec_consts(j)[64];
@@ -998,7 +1142,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 if (j > 0 && warp == 0) {
                     fold_writes(j - 1);
                     if (prev_last) {
-                        if (lane == 0) a.wnorm[prev_lh] = wacc;
+                        if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 44);
                         wacc = 0.f;
                     }
                 }
@@ -1117,6 +1261,11 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 // ---- head boundary: S_after = sig S~ out through the staging buffer, the next
                 // head's state (staged meanwhile) into TMEM, drift partials against S_before
                 const bool has_next = j + 1 < NJ;          // uniform
+                // a last slot that ends a head begun by CTA i - 1: S_before is not in TMEM (the
+                // slot started from the handed-over state) but staged, and its square sum is taken
+                // here
+                const bool shared_end = sch.is_suffix(slot);
+                float den_end = 0.f;
                 bool ok = mbar_wait_or_abort(&mb_s, j & 1, kWaitBudgetNs, abort_flag);
                 if (!ok) fail(a.status, abort_flag, 12);
                 if (!mbar_wait_or_abort(&mb_st, st_seen & 1, kWaitBudgetNs, abort_flag)) {
@@ -1133,7 +1282,17 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                         const int ch = 8 * cgp + 4 * half;     // this half's 16-byte chunks of row r
                         float sa[16], sb[16];
                         tmem_ld16(tm + lane_off + TM_S + col, sa);
-                        tmem_ld16(tm + lane_off + TM_SB + col, sb);
+                        if (shared_end) {
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
+                                sb[4 * e] = x.x; sb[4 * e + 1] = x.y; sb[4 * e + 2] = x.z; sb[4 * e + 3] = x.w;
+                            }
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) den_end = fmaf(sb[e], sb[e], den_end);
+                        } else {
+                            tmem_ld16(tm + lane_off + TM_SB + col, sb);
+                        }
                         tmem_ld_wait();
 #pragma unroll
                         for (int e = 0; e < 16; ++e) {
@@ -1167,7 +1326,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 if (has_next) warp_arrive(&mb_sready, lane);     // the next head's state is in TMEM
                 // partial sums: pairwise in fp32, over the warp's lanes and then over the 16 warps
                 // (the FP64 pipe is far too slow for this path)
-                float fn = num, fd = den;
+                float fn = num, fd = shared_end ? den_end : den;
 #pragma unroll
                 for (int m = 16; m >= 1; m >>= 1) {
                     fn += __shfl_xor_sync(0xffffffffu, fn, m);
@@ -1175,7 +1334,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
                 if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
                 if (named_sync_or(2, kChain, !ok)) break;
-                if (warp == 0 && a.partials != nullptr) {
+                if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot)) {   // a shared head's drift: at its end
                     float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
                     float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
 #pragma unroll
@@ -1192,13 +1351,14 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 sig = 1.f;
             }
             prev_lh = lh;
+            prev_slot = slot;
             prev_last = last;
-            cc.next(n, a);
+            cc.next(sch, a);
         }
         // the CTA's last tile (always a head's last) once every warp's Ũ pass has added to it
         if (want_w && NJ > 0 && !named_sync_or(2, kChain, *abort_flag) && warp == 0) {
             fold_writes(NJ - 1);
-            if (lane == 0) a.wnorm[prev_lh] = wacc;
+            if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 45);
         }
     }
 
@@ -1256,11 +1416,28 @@ bool make_state_map(CUtensorMap* map, void* base, int heads) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Scratch: the WY records, then the update kernel's hand-over area for up to one CTA per SM:
+// states [grid][128][128] fp32 (1024-aligned), flags [2][grid] int32, write-size sums [grid].
+struct TcScratch {
+    size_t rec, ho_state, ho_flags, ho_wsum, total;
+};
+
+TcScratch tc_scratch_layout(int L, int Hv, int T) {
+    const int grid = std::max(1, std::min(L * Hv, device_sm_count()));
+    TcScratch l;
+    l.rec = 0;
+    l.ho_state = ((size_t)L * Hv * ((T + kC - 1) / kC) * kRecBytes + 1023) & ~size_t(1023);
+    l.ho_flags = l.ho_state + (size_t)grid * kD * kD * 4;
+    l.ho_wsum = l.ho_flags + 2 * (size_t)grid * 4;
+    l.total = l.ho_wsum + (size_t)grid * 4;
+    return l;
+}
+
 }  // namespace
 
 size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T) {
     if (dk != kD || dv != kD || dtype != DELTAS_BF16 || L <= 0 || Hv <= 0 || T <= 0) return 0;
-    return (size_t)L * Hv * ((T + kC - 1) / kC) * kRecBytes;
+    return tc_scratch_layout(L, Hv, T).total;
 }
 
 bool gdn_tc_supported(const GdnArgs& a) {
@@ -1273,9 +1450,11 @@ bool gdn_tc_supported(const GdnArgs& a) {
 }
 
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
-    CUtensorMap kmap, vmap, smap;
+    const TcScratch sl = tc_scratch_layout(a.L, a.Hv, a.T);
+    const int grid = std::min(a.L * a.Hv, device_sm_count());
+    CUtensorMap kmap, vmap, smap, hmap;
     if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
-        !make_state_map(&smap, a.state, a.L * a.Hv))
+        !make_state_map(&smap, a.state, a.L * a.Hv) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
         return cudaErrorInvalidValue;
     static int configured_device = -1;
     int dev = 0;
@@ -1294,6 +1473,8 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     WyArgs w;
     w.L = a.L; w.Hk = a.Hk; w.Hv = a.Hv; w.T = a.T; w.n_tiles = n_tiles;
     w.g = a.g; w.beta = a.beta; w.rec = a.scratch; w.status = a.status;
+    w.ho_flags = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
+    w.n_ho_flags = 2 * grid;
     const long long items = (long long)a.L * a.Hv * n_tiles;
     const int wgrid = (int)std::min<long long>(items, (long long)sms * kWyCtasPerSm);
     gdn_wy_kernel<<<wgrid, kWyThreads, kWySmemAlloc, s>>>(kmap, w);
@@ -1304,9 +1485,23 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     TcArgs t;
     t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = n_tiles;
     t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.rec = a.scratch; t.status = a.status;
-    const int grid = std::min(a.L * a.Hv, sms);
+    t.ho_flag = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
+    t.ho_wflag = t.ho_flag + grid;
+    t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
+    // equal tile runs, with heads split between neighbouring CTAs, when they shorten the slowest
+    // CTA: a boundary between slots costs about 0.45 of a tile and a hand-over about one tile
+    // (measured: 512-token chunks gain 4 %, 124-token chunks lose 5 %)
+    t.split = 0;
+    const int H = a.L * a.Hv;
+    if (H > grid && H % grid != 0) {
+        const double whole = std::ceil((double)H / grid) * (n_tiles + 0.45);
+        const double runs = std::ceil((double)H * n_tiles / grid);
+        const double parted = runs + (runs / n_tiles + 2.0) * 0.45 + 1.0;
+        t.split = parted < whole ? 1 : 0;
+    }
+    (void)sms;
     return launch_dependent(gdn_update_tc_kernel, dim3(grid), dim3(kThreads), (size_t)kSmemAlloc, s, kmap, vmap,
-                            smap, t);
+                            smap, hmap, t);
 }
 
 }  // namespace deltas

@@ -123,11 +123,12 @@ def test_gdn_update_layer_width_chunk(L, want_out):
     _check_chunk(L, x, s0, want_out, torch.bfloat16, 128 ** -0.5)
 
 
-@pytest.mark.parametrize("T", [1, 130])
+@pytest.mark.parametrize("T", [1, 130, 500])
 def test_gdn_update_more_heads_than_sms(L, T):
     """160 (layer, head) pairs (5 layers x 32 value heads, d = 128, bf16): more heads than SMs, so
-    the tensor-core kernel's persistent CTAs each run several heads back to back; every head is
-    compared with the oracle (one tile, and three tiles with a ragged tail)."""
+    the tensor-core kernel's persistent CTAs take equal runs of tiles and most heads are split
+    between two neighbouring CTAs (the state handed over at the cut); every head's state and drift
+    partials are compared with the oracle (one tile, and three tiles with a ragged tail)."""
     x = inputs.gdn_chunk(5, T, 16, 32, 128, "bf16", inputs.seed_for(12, T))
     s0 = inputs.initial_state(5, 32, 128, inputs.seed_for(13, T))
     _check_chunk(L, x, s0, False, torch.bfloat16, 128 ** -0.5)
@@ -236,6 +237,7 @@ def test_score_kernel(L):
     (128, "bf16", 257, 2, 4, 1.0),      # tensor cores: several tiles, ragged tail, grouped keys
     (128, "bf16", 64, 1, 3, 1.0),       # one full tile, three value heads per key head
     (128, "bf16", 300, 2, 4, 4.0),      # strong decay: the deferred decay restarts every tile
+    (128, "bf16", 300, 16, 80, 1.0),    # 160 heads on fewer SMs: heads split between CTAs
     (64, "f32", 100, 2, 4, 1.0),        # CUDA-core kernel
     (16, "bf16", 33, 1, 2, 1.0),
     (128, "f32", 1, 2, 2, 1.0),
