@@ -15,8 +15,9 @@
 // in the swizzled layout the tensor core reads, -gamma and gamma_C.  The update kernel then runs
 // the part that is sequential in the tiles, the state chain, with nothing else on the SM.
 //
-// Update kernel: one persistent CTA per SM takes (layer, value head) pairs in turn; the tiles of
-// its heads form one pipeline.  A head's state lives in TMEM from its first tile to its last
+// Update kernel: one persistent CTA per SM takes (layer, value head) pairs in turn, or equal runs
+// of tiles with a head at each run boundary split between two CTAs (see ChainSched); the tiles of
+// its slots form one pipeline.  A head's state lives in TMEM from its first tile to its last
 // (S_before beside it, for the drift), so the state is read from and written to HBM exactly once;
 // the next head's state is loaded into shared memory while the current head runs, and the head
 // boundary swaps the two in one pass that also forms the drift partials.  Per tile:
@@ -1481,7 +1482,7 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     // update kernel: one persistent CTA per SM (the kernel needs the whole SM: 512 TMEM columns,
-    // ~211 KB of shared memory); each takes every grid-th head
+    // ~211 KB of shared memory); each takes every grid-th head, or an equal run of tiles
     TcArgs t;
     t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = n_tiles;
     t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.rec = a.scratch; t.status = a.status;
