@@ -4,12 +4,14 @@
 // remaining candidates -- applied to every (layer, KV head) plane with the slots' own scores.
 //
 // One 1024-thread CTA ranks one plane:
-//   1. the smallest / largest candidate chunk (block reduction; negative chunk ids are reported);
+//   1. the smallest / largest candidate chunk and score key (block reduction; negative chunk ids
+//      are reported);
 //   2. every candidate's span and its 56-bit key: the score's IEEE total-order bits (32) above
 //      the complement of the slot (24 bits, so that the earlier slot ranks higher on equal
 //      scores).  Keys are unique.  The 32-bit score part and the span (one byte) of every
 //      candidate are kept in shared memory when the plane fits, else in the workspace; the slot
-//      part is the candidate's index;
+//      part is the candidate's index.  The same pass counts the spans and builds the quota
+//      select's first-digit histogram;
 //   3. quota: for every span with more candidates than the quota q, a radix select (8-bit
 //      digits, most significant first, starting at the highest bit in which two candidates'
 //      keys differ, all spans in one pass over the candidates) narrows a key prefix until the
@@ -17,7 +19,8 @@
 //      digit bin it stops in is taken whole, so distinct scores resolve within the score digits
 //      and the slot digits are read only for exact ties;
 //   4. fill: the same select over the candidates the quota left, as one group, for the
-//      remaining capacity R - kept;
+//      remaining capacity R - kept (its first-digit histogram built by the pass that marks the
+//      quota's choices);
 //   5. emit: every warp owns a contiguous stretch of slots; it counts its kept slots, a scan of
 //      the 32 counts gives its offset, and it writes its kept slots in order (retain_idx
 //      ascending) and the mask.
