@@ -1490,14 +1490,14 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     t.ho_wflag = t.ho_flag + grid;
     t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
     // equal tile runs, with heads split between neighbouring CTAs, when they shorten the slowest
-    // CTA: a boundary between slots costs about 0.45 of a tile and a hand-over about one tile
-    // (measured: 512-token chunks gain 4 %, 124-token chunks lose 5 %)
+    // CTA: a boundary between slots costs about 0.45 of a tile and the hand-over about three
+    // tiles (measured: 512- and 1024-token chunks gain 5-6 %, chunks of 2-3 tiles lose)
     t.split = 0;
     const int H = a.L * a.Hv;
     if (H > grid && H % grid != 0) {
         const double whole = std::ceil((double)H / grid) * (n_tiles + 0.45);
         const double runs = std::ceil((double)H * n_tiles / grid);
-        const double parted = runs + (runs / n_tiles + 2.0) * 0.45 + 1.0;
+        const double parted = runs + (runs / n_tiles + 2.0) * 0.45 + 3.0;
         t.split = parted < whole ? 1 : 0;
     }
     (void)sms;
