@@ -1030,6 +1030,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     bulk_wait0();                      // the state is in global memory ...
                     fence_proxy_async_global();
                     __threadfence();
+                    grid_dep_wait();                   // (after the factor kernel's flag reset)
                     ho_store_release(a.ho_flag + me, 1);   // ... before CTA i + 1 may read it
                 }
                 if (k + 2 <= n_slots) {
@@ -1108,6 +1109,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             if (sch.is_prefix(slot)) {
                 a.ho_wsum[me] = sum;
                 __threadfence();
+                grid_dep_wait();                           // (after the factor kernel's flag reset)
                 ho_store_release(a.ho_wflag + me, 1);
                 return true;
             }
