@@ -59,6 +59,7 @@ score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk
 {
     __shared__ double term_sum[kScoreThreads / 32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    grid_dep_wait();                                   // the partials are written
     double acc = 0.0;
     for (int l = warp; l < L; l += kScoreThreads / 32) {
         float num = 0.f, den = 0.f;
@@ -94,6 +95,7 @@ __global__ void __launch_bounds__(32)
 score_write_norms_kernel(int n, const float* __restrict__ wnorm, double inv_count, int chunk_id,
                          float* __restrict__ scores)
 {
+    grid_dep_wait();                                   // the write sizes are written
     double acc = 0.0;
     for (int i = threadIdx.x; i < n; i += 32) acc += (double)wnorm[i];
 #pragma unroll
@@ -107,8 +109,8 @@ cudaError_t launch_score_write_norms(int L, int Hv, const float* wnorm, int n_to
                                      cudaStream_t s)
 {
     const double inv = n_tokens > 0 ? 1.0 / ((double)L * Hv * n_tokens) : 0.0;
-    score_write_norms_kernel<<<1, 32, 0, s>>>(L * Hv, wnorm, inv, chunk_id, scores);
-    return cudaGetLastError();
+    // scheduled while the update finishes (it waits for it before reading)
+    return launch_dependent(score_write_norms_kernel, dim3(1), dim3(32), 0, s, L * Hv, wnorm, inv, chunk_id, scores);
 }
 
 cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, const float* sa,
@@ -123,8 +125,9 @@ cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, c
 cudaError_t launch_score_chunks(int L, int Hv, const float* partials, int chunk_id, float* scores,
                                 cudaStream_t s)
 {
-    score_chunks_kernel<<<1, kScoreThreads, 0, s>>>(L, Hv, partials, chunk_id, scores);
-    return cudaGetLastError();
+    // scheduled while the update finishes (it waits for it before reading)
+    return launch_dependent(score_chunks_kernel, dim3(1), dim3(kScoreThreads), 0, s, L, Hv, partials, chunk_id,
+                            scores);
 }
 
 }  // namespace deltas

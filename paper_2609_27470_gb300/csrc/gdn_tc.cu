@@ -799,6 +799,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
     }
     if (tid == 0) s_abort = 0;
     if (tid < 2 * kC) s_u2[tid >> 6][tid & (kC - 1)] = 0.f;
+    grid_dep_launch();                                 // the next kernel (the score) may be scheduled
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
