@@ -120,7 +120,11 @@ deltas_status gdn_update(const deltas_gdn_desc* desc, int32_t n_tokens, const vo
     a.status = static_cast<int32_t*>(workspace);
     a.scratch = static_cast<uint8_t*>(workspace) + kStatusBytes;
     a.scratch_bytes = workspace_bytes - kStatusBytes;
-    if (gdn_tc_supported(a)) return from_cuda(launch_gdn_update_tc(a, as_stream(stream)));
+    // d = 128 bfloat16 without read-out runs on the tensor cores or not at all: no silent fallback
+    if (gdn_tc_shape(a)) {
+        if (!gdn_tc_supported(a)) return DELTAS_ERR_UNSUPPORTED;
+        return from_cuda(launch_gdn_update_tc(a, as_stream(stream)));
+    }
     return from_cuda(launch_gdn_update_simt(a, as_stream(stream)));
 }
 
@@ -426,7 +430,7 @@ deltas_status deltas_copy_stream_state_heads(const deltas_gdn_desc* gdn, const d
 
 deltas_status deltas_clear_device_status(void* workspace, void* stream) {
     if (workspace == nullptr) return DELTAS_ERR_WORKSPACE;
-    return from_cuda(cudaMemsetAsync(workspace, 0, 16, as_stream(stream)));
+    return from_cuda(cudaMemsetAsync(workspace, 0, kStatusBytes, as_stream(stream)));
 }
 
 deltas_status deltas_get_device_status(const void* workspace, void* stream,

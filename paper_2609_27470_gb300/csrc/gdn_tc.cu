@@ -1,71 +1,64 @@
 // Gated delta rule over one chunk on the Blackwell tensor cores (tcgen05 + TMEM + TMA), d = 128,
-// bfloat16 k/v, fp32 state, with the state-drift partials fused in.
+// bfloat16 k/v, fp32 state, with the state-drift partials fused in: one persistent kernel.
 //
 // Paper: Sec. 3.2, Eq. 1/2 (the recurrence) and Eq. 3 (drift numerator / denominator per layer
-// and head).  The chunk is processed in tiles of C = 64 tokens with the chunkwise (WY) form of
-// Eq. 1: with G the inclusive cumulative log-decay inside the tile, gamma = exp(G),
-//   A[t][i] = beta_t exp(G_t - G_i) k_t.k_i  (i < t),   T = (I + A)^-1 diag(beta),
-//   X = K S0^T,   W = V - diag(gamma) X,   U = T W,
-//   S_C = gamma_C S0 + U~^T K,   U~[t] = exp(G_C - G_t) U[t].
-// Padded tokens of a ragged last tile carry k = v = 0, g = 0, beta = 0 and change nothing.
+// and head).  The chunk is processed in sub-tiles of C = 32 tokens with the chunkwise (WY) form of
+// Eq. 1.  Inside a sub-tile let G be the inclusive cumulative log-decay, gamma_t = exp(G_t),
+// gamma_C = exp(G_{C-1}), delta_t = gamma_C / gamma_t <= 1, and X = K S0^T (row t: S0 k_t).  With
+//   A[t][i] = beta_t (gamma_t / gamma_i) k_t.k_i  (i < t),   U = (I + A)^-1 diag(beta) (V - diag(gamma) X)
+// the state after the sub-tile is S_C = gamma_C S0 + sum_t delta_t u_t k_t^T.  The decay factors
+// out of the triangular solve by a diagonal similarity, I + A = diag(gamma) (I + diag(beta) L)
+// diag(gamma)^-1 with L the strictly lower part of K K^T, so with the decay-free
+//   N_beta = (I + diag(beta) L)^-1 diag(beta)
+// the decayed writes are  U~ = diag(delta) U = N_beta (diag(delta) V - gamma_C X):  every decay
+// factor the kernel uses is at most 1, and the inverse depends on k and beta only.
 //
-// Two kernels.  T and the tile's decay constants depend on k, g and beta only, so the factor
-// kernel builds them for every (layer, value head, tile) at once, several CTAs per SM, and writes
-// one record per tile into the workspace: T~ = diag(exp(G_C - G)) T as the bfloat16 (hi, lo) pair
-// in the swizzled layout the tensor core reads, -gamma and gamma_C.  The update kernel then runs
-// the part that is sequential in the tiles, the state chain, with nothing else on the SM.
+// Work split inside one CTA (one per SM, persistent over (layer, value head) slots):
+//   producer  (4 warps, two groups of two; group g takes the sub-tiles of parity g): K K^T of a
+//             64-token tile comes from the tensor core; each group forms diag(beta) L of its
+//             sub-tile, inverts I + diag(beta) L (16 x 16 diagonal blocks by substitution, the
+//             off-diagonal block by two products) and writes the two operand images the chain
+//             reads: B1 = u diag(delta) N_beta^T as a bfloat16 (hi, lo) pair and B2 = -c N_beta^T
+//             in tf32 (u, c: the state's deferred scale, below)
+//   MMA       (1 warp, one elected lane): every tcgen05.mma, each group's completion by commit
+//   chain     (8 warps): the passes over TMEM between the state-dependent products
+//   loads     (1 warp): K (64-token tiles) and V (32-token sub-tiles) by TMA, L2 prefetch ahead
+//   state     (1 warp): each slot's state into a staging buffer by TMA, S_after out of it
+// Per sub-tile j, in tensor-pipe order:
+//   E(j)   = V^T B1                      (bf16, issued during the previous sub-tile's pass; N = 64:
+//                                         the hi and lo halves land side by side in TMEM)
+//   X      = S~ K^T                      (tf32: A = the fp32 state straight from TMEM, K exact)
+//   E(j)  += X B2                        (tf32: A = X straight from TMEM, no pass in between)
+//   pass   (chain) E = hi half + lo half, split into bfloat16 (hi, lo) A operand
+//   S~     = 2^-s S~ + E K               (bf16 (hi, lo) x K; the input state scaled by the
+//                                         instruction's power-of-two scale-input-d operand)
+// so the chain's own work per sub-tile is one pass over a 128 x 32 block.
 //
-// Update kernel: one persistent CTA per SM takes (layer, value head) pairs in turn, or equal runs
-// of tiles with a head at each run boundary split between two CTAs (see ChainSched); the tiles of
-// its slots form one pipeline.  A head's state lives in TMEM from its first tile to its last
-// (S_before beside it, for the drift), so the state is read from and written to HBM exactly once;
-// the next head's state is loaded into shared memory while the current head runs, and the head
-// boundary swaps the two in one pass that also forms the drift partials.  Per tile:
-//   V region  <- V^T                       (MMA: V tile times an identity matrix, exact)
-//   X region  <- S~ K^T                     (tf32 MMA, K exact in fp32)
-//   W pass:   W^T = V^T - sig X diag(gamma), x u_scale -> (hi, lo) in place over X   (chain)
-//   U region  <- W^T T~^T = U~^T / ...      (MMA)
-//   U~ pass:  -> (hi, lo) in place                          (chain)
-//   S~        += U~^T K                     (MMA)
-// so the chain's passes are a few loads, an FMA, a split and a store per element, and the
-// per-token decays ride on the W pass and on T~.
+// Deferred decay.  TMEM holds S~ with the true state S = sig S~.  A sub-tile with decay gamma_C
+// takes p = gamma_C sig and a shift s in [0, 15] that brings p 2^s into [1/2, 1) when it can:
+// then sig <- p 2^s, u = 1 / sig, c = 2^-s, and MMA_S scales S~ by 2^-s as it accumulates (exact).
+// When p < 2^-45 (no shift reaches 2^-30) the chain multiplies S~ by p in a pass instead, sig
+// restarts at 1, u = 1 and c = p.  So sig stays in [2^-30, 1] and u below 2^30.  The producer
+// and the chain see the same per-sub-tile constants (sig after the sub-tile, the shift, the pass
+// factor), which the producer writes beside the images.
 //
-// Precision.  Keys and values are exact in bfloat16.  The state never leaves fp32 inside the
-// tile loop: TMEM holds S~ with S = sig S~, and X reads S~ straight from TMEM as the A operand of
-// a kind::tf32 product; the hardware keeps 10 mantissa bits of S~ (a relative error below 2^-10
-// per element) while K is exact, an error that reaches the state only through the
-// delta correction and decay with it (a CPU simulation of the truncation gives a state error vs
-// fp64 of ~2e-4 at the slowest decay the inputs use, 5e-6 at a typical one).  The other products
-// take a two-term bfloat16 split (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)) of each fp32
-// operand:
-//   V^T I                           exact                                        1 MMA group
-//   X^T  = S~ K^T                   S~ (tf32, from TMEM) K (exact in tf32)       1 MMA group
-//   U~^T = W^T T~^T                  Whi T~hi + Whi T~lo + Wlo T~hi                3 MMA groups
-//   S   += U~^T K                   (U~hi + U~lo) K                              2 MMA groups
-//   K K^T (factor kernel)           exact inputs                                 1 MMA group
-// All products accumulate in fp32 in TMEM.
+// Precision.  k, v exact in bfloat16; K K^T exact in fp32.  The state-dependent products read S~
+// and X as tf32 (10 explicit mantissa bits, truncated) and B2 is rounded to tf32: errors confined
+// to the delta correction.  B1 and E take two-term bfloat16 splits (x = hi + lo, about 2^-16
+// relative).  The inverse is formed in fp32.  A CPU model of exactly these roundings gives a state
+// error against fp64 of 4.5e-4 at the slowest decay the tests use (4 chunks of 1024 tokens), 5e-6
+// at a typical one, and drift numerators within 2.2e-4.
 //
-// Deferred decay: the tile decay gamma_C is folded into the scalar sig instead of a pass that
-// multiplies S by gamma_C; the W pass applies sig and scales W by u_scale = 1 / (gamma_C sig) so that
-// MMA_S adds onto S~ directly.  When sig gamma_C would fall below 2^-30 the tile writes
-// gamma_C sig S~ back into TMEM and sig restarts at 1 (u_scale = 1), so 1 / sig stays far from the
-// fp32 range limit.  The head's last tile multiplies by sig when it reads the state out.
+// Synchronisation.  Roles hand work to each other through mbarriers only; every wait is bounded
+// (about one second, or the workspace header's override); a wait that runs out records
+// DELTAS_ERR_TIMEOUT, raises a CTA-wide abort flag so the other roles stop waiting, and the CTA
+// drains its MMAs and copies before freeing TMEM.  Heads split between neighbouring CTAs (equal
+// tile runs, see ChainSched) hand the state over through the workspace with a bit per CTA boundary
+// in the workspace header, which its reader clears after use.
 //
-// Update-kernel warp roles (19 warps):
-//   0-15  state chain: warp w serves TMEM lanes 32 (w % 4) .. + 31 (state rows) and column group
-//         w / 4; per tile the W and U~ passes (16 token columns each) and the next tile's K in
-//         fp32 (two 16-byte chunks each), at head boundaries the state swap and the drift partials
-//   16    TMEM allocation and every tcgen05.mma (one elected lane issues; the warp stays
-//         converged); it also releases the input buffers by tcgen05.commit
-//   17    tile loads: K, V (TMA) and the WY records (bulk copy), as buffers are released
-//   18    state moves: each head's state into the staging buffer, S_after out of it
-// A TMA or bulk copy occupies the issuing thread for a time that grows with its size, so no copy
-// is issued from a role on the chain's critical path.  Roles hand work to each other through
-// mbarriers only.  Every wait is bounded; a wait that runs out records DELTAS_ERR_TIMEOUT, raises
-// a CTA-wide abort flag so the other roles stop waiting, and the CTA drains its MMAs and copies
-// before freeing TMEM.
-// TMEM (512 columns, M = 128 lanes = d_v): S~ [0,128), S_before [128,256), X [256,320) (X, then
-// W hi / lo packed in place), U [320,384) (likewise U~), V^T [384,448); [448,512) unused.
+// TMEM (512 columns, 128 lanes = d_v): S~ [0,128), S_before [128,256), X [256,288),
+// E0 [288,352), E1 [352,416) (each: hi-half product [+0,+32), lo-half product [+32,+64)),
+// K K^T [416,480) (lanes 0..63), packed A of MMA_S [480,512) (hi k-step 0, 1, lo k-step 0, 1).
 #include <algorithm>
 #include <cmath>
 
@@ -77,20 +70,54 @@ namespace {
 
 using namespace tc;
 
-constexpr int kC = 64;                 // tokens per tile
+constexpr int kC = 32;                 // tokens per sub-tile
+constexpr int kTile = 64;              // tokens per tile (two sub-tiles; the schedule's unit)
 constexpr int kD = 128;                // head dim (d_k = d_v)
-constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kSigMin = 9.313225746154785e-10f;   // 2^-30: smallest deferred decay of the state
+constexpr float kHardMin = 0x1p-45f;   // p below this: the state is rescaled by a pass
 
-// ---- WY record of one (layer, value head, tile), written by the factor kernel, read by the update
-// kernel with one bulk copy:
-//   [0, 8192)       T~ hi: bfloat16 [64 t][64 i], 128-byte rows, 128-byte swizzle (K-major B operand)
-//   [8192, 16384)   T~ lo, same layout
-//   [16384, 16656)  float: -gamma[64], gamma_C, 3 unused
-constexpr uint32_t kRecT = 16384;
-constexpr uint32_t kRecConsts = 68;
-constexpr uint32_t kRecBytes = kRecT + kRecConsts * 4;
-static_assert(kRecBytes % 16 == 0, "records are bulk-copied: 16-byte multiples");
+// ---- roles
+constexpr int kChainWarps = 8;
+constexpr int kChain = 32 * kChainWarps;
+constexpr int kProdWarp0 = 8;          // 8, 9: TMEM readers of producer groups 0, 1; 10, 11: partners
+constexpr int kMmaWarp = 12;
+constexpr int kLoadWarp = 13;
+constexpr int kStateWarp = 14;
+constexpr int kThreads = 15 * 32;
+constexpr int kBarChain = 1;           // named barriers: chain (256 threads), producer groups (64)
+constexpr int kBarProd0 = 2;
+
+// ---- TMEM columns
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t TM_S = 0, TM_SB = 128, TM_X = 256, TM_E = 288, TM_KK = 416, TM_AP = 480;
+
+// ---- shared memory (bytes from a 1024-aligned base)
+constexpr uint32_t SM_K = 0;           // 3 tiles x 16 KB: 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B,
+                                       // SW128; sub-tile u in rows 32u..32u+31
+constexpr uint32_t SM_K32 = 49152;     // 16 KB: one sub-tile's K in fp32, 4 column blocks (32 dims) x 32 rows
+                                       // x 128 B, SW128 (the B operand of X); also the K K^T product's
+                                       // over-read past the last K tile (rows 64..127 of its M = 128 A)
+constexpr uint32_t SM_V = 65536;       // 3 sub-tiles x 8 KB: 2 column blocks x 32 rows x 128 B, SW128
+constexpr uint32_t SM_IMG = 90112;     // 4 slots x 12 KB: B1 hi [0, 4 KB) and lo [4, 8 KB) (32 rows x 128 B,
+                                       // the first 64 B of a row used), B2 [8, 12 KB) (32 rows x 32 fp32)
+constexpr uint32_t kImgSlot = 12288;
+constexpr uint32_t SM_SB = 139264;     // 64 KB: state staging, 4 column blocks x 128 rows x 128 B, SW128
+constexpr uint32_t SM_PW = 204800;     // producer workspaces, one per group
+constexpr int kMS = 36;                // fp32 row stride of M and N (16-byte aligned rows)
+constexpr int kPS = 20;                // fp32 row stride of the 16 x 16 product
+// beta, delta and (u, c) of the group's sub-tile are double-buffered by tile parity: the partner
+// warp writes the next tile's while the other may still read this one's
+constexpr int PW_M = 0, PW_N = 32 * kMS, PW_P = 64 * kMS, PW_BETA = PW_P + 16 * kPS, PW_DELTA = PW_BETA + 64,
+              PW_UC = PW_DELTA + 64, PW_FLOATS = PW_UC + 8;
+constexpr uint32_t kPwBytes = PW_FLOATS * 4;
+constexpr uint32_t SM_CONST = SM_PW + 2 * kPwBytes;   // 4 slots x 48 words: per-sub-tile constants
+constexpr int kConstWords = 48;        // [0,32) write-size scale per token, 32 sig after, 33 pass factor
+                                       // (< 0: none), 34 shift (int)
+constexpr uint32_t SM_BYTES = SM_CONST + 4 * kConstWords * 4;
+constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
+static_assert(SM_K32 % 1024 == 0 && SM_V % 1024 == 0 && SM_IMG % 1024 == 0 && SM_SB % 1024 == 0 &&
+              kImgSlot % 1024 == 0 && SM_PW % 16 == 0 && kPwBytes % 16 == 0, "shared-memory map");
+static_assert(SM_IMG == SM_V + 3 * 8192 && SM_SB == SM_IMG + 4 * kImgSlot && SM_PW == SM_SB + 65536, "map order");
+static_assert(kSmemAlloc + 1024 <= 232448, "shared memory budget");
 
 // Barrier over `n` threads that also returns the OR of `flag` over them (uniform result).
 __device__ __forceinline__ bool named_sync_or(int id, int n, bool flag) {
@@ -108,22 +135,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// x[0..7] -> hi = bf16(x), lo = bf16(x - hi), 8 packed values each
-__device__ __forceinline__ void split8(const float* x, uint4& hi, uint4& lo) {
-    uint32_t h[4], l[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const __nv_bfloat162 hh = __floats2bfloat162_rn(x[2 * i], x[2 * i + 1]);
-        const float2 hf = __bfloat1622float2(hh);
-        h[i] = *reinterpret_cast<const uint32_t*>(&hh);
-        l[i] = pack_bf16x2(x[2 * i] - hf.x, x[2 * i + 1] - hf.y);
-    }
-    hi = make_uint4(h[0], h[1], h[2], h[3]);
-    lo = make_uint4(l[0], l[1], l[2], l[3]);
-}
-
-// (a, b) -> packed bf16 hi = (bf16(a), bf16(b)) and lo = (bf16(a - hi_a), bf16(b - hi_b)),
-// a in the low half (the TMEM A-operand packing: even k low)
+// (a, b) -> packed bf16 hi = (bf16(a), bf16(b)) and lo = (bf16(a - hi_a), bf16(b - hi_b)), a in the
+// low half (even k low: the packing of a TMEM A operand and of a K-major row)
 __device__ __forceinline__ void split2(float a, float b, uint32_t& hi, uint32_t& lo) {
     const __nv_bfloat162 hh = __floats2bfloat162_rn(a, b);
     const float2 hf = __bfloat1622float2(hh);
@@ -131,70 +144,14 @@ __device__ __forceinline__ void split2(float a, float b, uint32_t& hi, uint32_t&
     lo = pack_bf16x2(a - hf.x, b - hf.y);
 }
 
-// D (16 x 8) += A (16 x 16, row) B (16 x 8, col) on the warp's tensor-core path, bf16 in, fp32
-// accumulate.  Fragments (g = lane / 4, t = lane % 4), each register a bf16 pair, lower k in the
-// low half: a = A[g][2t..], A[g+8][2t..], A[g][2t+8..], A[g+8][2t+8..]; b = B[2t..][g],
-// B[2t+8..][g]; d as for the tf32 form.
-__device__ __forceinline__ void mma_m16n8k16_bf16(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
-    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-                 "{%0,%1,%2,%3};"
-                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
-}
-
-// Operands stored split: row r of A is at A + r * as (32-bit words), its word p the bf16 pair of
-// hi = bf16(x) for columns (2p, 2p+1) and word a_lo + p the pair of lo = bf16(x - hi); likewise B,
-// stored n-major (row n of B's storage holds column n of B).  D (16 x 8) += A[r0 .. r0+15][0..16K)
-// B[0..16K)[n0 .. n0+7] over the three products lo*hi + hi*lo + hi*hi.
-template <int KSTEPS>
-__device__ __forceinline__ void mma_split_bf16(float (&d)[4], const uint32_t* A, int as, int a_lo, int r0,
-                                               const uint32_t* B, int bs, int b_lo, int n0, int lane) {
-    const int g = lane >> 2, t = lane & 3;
-    const uint32_t* a0 = A + (r0 + g) * as;
-    const uint32_t* a1 = A + (r0 + g + 8) * as;
-    const uint32_t* b0 = B + (n0 + g) * bs;
-#pragma unroll
-    for (int ks = 0; ks < KSTEPS; ++ks) {
-        const int p0 = 8 * ks + t, p1 = p0 + 4;
-        const uint32_t ah[4] = {a0[p0], a1[p0], a0[p1], a1[p1]};
-        const uint32_t al[4] = {a0[a_lo + p0], a1[a_lo + p0], a0[a_lo + p1], a1[a_lo + p1]};
-        const uint32_t bh[2] = {b0[p0], b0[p1]};
-        const uint32_t bl[2] = {b0[b_lo + p0], b0[b_lo + p1]};
-        mma_m16n8k16_bf16(d, al, bh);
-        mma_m16n8k16_bf16(d, ah, bl);
-        mma_m16n8k16_bf16(d, ah, bh);
-    }
-}
-
-// One element of a split row (see mma_split_bf16): hi / lo halfwords of column k; lo words start
-// lo_words after the row's first word.
-__device__ __forceinline__ void put_split(uint32_t* row, int k, float x, int lo_words = 16) {
-    const __nv_bfloat16 h = __float2bfloat16_rn(x);
-    const __nv_bfloat16 l = __float2bfloat16_rn(x - __bfloat162float(h));
-    reinterpret_cast<__nv_bfloat16*>(row)[k] = h;
-    reinterpret_cast<__nv_bfloat16*>(row + lo_words)[k] = l;
-}
-
-// 16 consecutive values -> split row of a 16-column operand (words 0..7 hi, 8..15 lo)
-__device__ __forceinline__ void put_split16(uint32_t* row, const float* x) {
-    uint32_t h[8], l[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) split2(x[2 * i], x[2 * i + 1], h[i], l[i]);
-    *reinterpret_cast<uint4*>(row) = make_uint4(h[0], h[1], h[2], h[3]);
-    *reinterpret_cast<uint4*>(row + 4) = make_uint4(h[4], h[5], h[6], h[7]);
-    *reinterpret_cast<uint4*>(row + 8) = make_uint4(l[0], l[1], l[2], l[3]);
-    *reinterpret_cast<uint4*>(row + 12) = make_uint4(l[4], l[5], l[6], l[7]);
-}
-
-// 2^x with the hardware approximation (relative error about 2^-22)
-__device__ __forceinline__ float fast_exp2(float x) {
-    float y;
-    asm("ex2.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+// fp32 -> tf32 with round-to-nearest (ties away), as the 32-bit container the tensor core reads
+__device__ __forceinline__ uint32_t to_tf32(float x) {
+    uint32_t y;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(y) : "f"(x));
     return y;
 }
 
-// All lanes of a converged warp wait; the result is the same on every lane (false if any lane's
-// wait ran out), so the warp stays converged for the elect.sync that follows.
+// All lanes of a converged warp wait; the result is the same on every lane.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
                                           const volatile int* abort) {
     const bool ok = mbar_wait_or_abort(bar, parity, budget_ns, abort);
@@ -206,486 +163,68 @@ __device__ __forceinline__ void fail(int32_t* status, volatile int* abort, int w
     *abort = 1;
 }
 
-// One arrival per warp on a chain -> MMA barrier: every lane's TMEM stores / shared-memory
-// writes were completed and fenced before the __syncwarp; lane 0 then arrives (release).
+// One arrival per warp: every lane's TMEM stores / shared-memory writes were completed and fenced
+// before the __syncwarp; lane 0 then arrives (release).
 __device__ __forceinline__ void warp_arrive(uint64_t* bar, int lane) {
     __syncwarp();
     if (lane == 0) mbar_arrive(bar);
 }
 
-// shared-memory descriptor advanced by `bytes` (the start address field counts 16-byte units)
-__device__ __forceinline__ uint64_t dadd(uint64_t desc, uint32_t bytes) { return desc + (uint64_t)(bytes >> 4); }
-
-// =============================================================================================
-// Factor kernel: T~ = diag(exp(G_C - G)) (I + A)^-1 diag(beta) and the decay constants of every tile
-// =============================================================================================
-constexpr int kWyThreads = 256;
-constexpr int kWyCtasPerSm = 4;
-constexpr uint32_t kWyTmemCols = 64;
-constexpr int FA_S = 68;               // fp32 row stride of A: 16-byte rows; a 16-byte access by 8 threads
-                                       // of 8 consecutive rows hits 8 distinct bank groups
-constexpr int FX_S = 68;               // fp32 row stride of X = (I + A)^-1 (16-byte aligned rows)
-// shared-memory map (bytes from a 1024-aligned base)
-constexpr uint32_t WY_FA = 0;                         // fp32 [64][FA_S].  Its two 32 x 32 quarters that are
-                                                      // never read as fp32 hold split operands of level 2:
-                                                      // rows 32..63 x cols 0..31 = A21 (row-major), rows
-                                                      // 0..31 x cols 32..63 = X11 stored n-major
-constexpr uint32_t WY_K = WY_FA;                      // the next item's K tile (2 column blocks (d 0-63,
-                                                      // 64-127) x 64 rows x 128 B) lands over A once level 2
-                                                      // has read it; the M = 128 product of K K^T reads the
-                                                      // 8 KB past the tile as rows 64..127 (output ignored)
-constexpr uint32_t WY_FX = WY_FA + 64 * FA_S * 4;     // fp32 [64][FX_S]; rows 0..31 x cols 32..63 (the zero
-                                                      // upper quarter) hold X22 split, row-major
-constexpr uint32_t WY_TMP = WY_FX + 64 * FX_S * 4;    // level 1 products (fp32), then level 2's P split,
-                                                      // n-major, rows of 36 words
-constexpr uint32_t WY_L1 = WY_TMP + 32 * 36 * 4;      // level-1 split operands, 6 x 16 rows of 20 words: A10,
-                                                      // A32, X11' (row-major), X22' (n-major), P1 for p = 0, 1
-constexpr int kL1S = 20;                              // row stride (words): fragment loads hit distinct banks
-constexpr uint32_t WY_TG = WY_L1 + 6 * 16 * kL1S * 4; // 2 buffers (item parity) x (G2[64], beta[64], row[64],
-                                                      // col[64], del[64], flag)
-constexpr uint32_t kTgFloats = 324;
-constexpr uint32_t WY_BYTES = WY_TG + 2 * kTgFloats * 4;
-constexpr uint32_t kWySmemAlloc = WY_BYTES + 1024;
-static_assert(WY_TG % 16 == 0 && (kTgFloats * 4) % 16 == 0, "tile factors must be 16-byte aligned");
-static_assert(kWyCtasPerSm * (kWySmemAlloc + 1024) <= 233472, "factor kernel: CTAs per SM");
-
-struct WyArgs {
-    int L, Hk, Hv, T, n_tiles;
-    const float* g;
-    const float* beta;
-    uint8_t* rec;              // [L * Hv][n_tiles] records of kRecBytes
-    int32_t* status;
-    int32_t* ho_flags;         // the update kernel's hand-over flags, reset here for this call
-    int n_ho_flags;
-};
-
-__global__ void __launch_bounds__(kWyThreads, kWyCtasPerSm)
-gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
-{
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
-    __shared__ uint64_t mb_k, mb_kk;
-    __shared__ uint32_t s_tmem;
-    __shared__ int s_fail;
-    grid_dep_launch();                                // the update kernel may take SMs as they free up
-    // the update kernel reads its hand-over flags only after this kernel has completed
-    if (blockIdx.x == 0)
-        for (int e = (int)threadIdx.x; e < a.n_ho_flags; e += kWyThreads) a.ho_flags[e] = 0;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int n = a.n_tiles;
-    const int items = a.L * a.Hv * n;                 // item = (layer * Hv + head) * n + tile
-    float* fA = reinterpret_cast<float*>(sm + WY_FA);
-    float* fX = reinterpret_cast<float*>(sm + WY_FX);
-    float* fT = reinterpret_cast<float*>(sm + WY_TMP);
-    // split level-2 operands (see the shared-memory map), row strides in 32-bit words
-    uint32_t* sA21 = reinterpret_cast<uint32_t*>(fA + 32 * FA_S);        // A[32 + r][k]
-    uint32_t* sX11 = reinterpret_cast<uint32_t*>(fA + 32);               // row n: X[k][n], k < 32
-    uint32_t* sX22 = reinterpret_cast<uint32_t*>(fX + 32);               // row r: X[32 + r][32 + k]
-    uint32_t* sP = reinterpret_cast<uint32_t*>(fT);                      // row n: P[k][n]
-    constexpr int kPS = 36;
-    // split level-1 operands: 16 x 16 blocks, rows of kL1S words (hi words 0..7, lo words 8..15)
-    uint32_t* sL1 = reinterpret_cast<uint32_t*>(sm + WY_L1);
-    uint32_t* sA10 = sL1;                                                 // A[16 + r][k]
-    uint32_t* sA32 = sL1 + 16 * kL1S;                                     // A[48 + r][32 + k]
-    uint32_t* sX11r = sL1 + 32 * kL1S;                                    // X[16 + r][16 + k]
-    uint32_t* sX22n = sL1 + 48 * kL1S;                                    // row n: X[32 + k][32 + n]
-    uint32_t* sP1 = sL1 + 64 * kL1S;                                      // p: row n of P1_p, 16 rows each
-
-    if (warp == 0) { tmem_alloc(&s_tmem, kWyTmemCols); tmem_relinquish(); }
-    if (tid == 0) {
-        mbar_init(&mb_k, 1); mbar_init(&mb_kk, 1);
-        fence_barrier_init();
-        prefetch_tensormap(&kmap);
-        s_fail = 0;
-    }
-    // The strictly upper 16 x 16 blocks of X are never written; zeros there let every level run
-    // fixed-length (unrolled) loops over the triangular factors.
-    for (int e = tid; e < 64 * FX_S; e += kWyThreads) { fX[e] = 0.f; fA[e] = 0.f; }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tm = s_tmem;
-
-    // Items are taken in reverse record order: the records written last, still in L2 when this
-    // kernel ends, are the ones of the lowest heads, which the update kernel reads first.
-    auto rec_of = [&](int it) { return items - 1 - it; };
-    auto item_pos = [&](int it, int& l, int& h, int& jt) {
-        const int r = rec_of(it), lh = r / n;
-        jt = r - lh * n; l = lh / a.Hv; h = lh - l * a.Hv;
-    };
-    int nk = 0, nkk = 0;                               // K loads (thread 0) / K K^T products (warp 0) issued
-    auto load_k = [&](int it) {                        // thread 0: the item's K tile
-        int l, h, jt;
-        item_pos(it, l, h, jt);
-        ++nk;
-        const int kh = (int)(((long long)h * a.Hk) / a.Hv);
-        mbar_arrive_expect_tx(&mb_k, 16384);
-        tma_load_4d(sm + WY_K, &kmap, &mb_k, 0, kh, jt * kC, l);
-        tma_load_4d(sm + WY_K + 8192, &kmap, &mb_k, 64, kh, jt * kC, l);
-    };
-    // g and beta of an item's 64 tokens, two per lane of warp 7, loaded one item ahead of use
-    float pg[2] = {0.f, 0.f}, pb[2] = {0.f, 0.f};
-    auto load_gb = [&](int it) {
-        int l, h, jt;
-        item_pos(it, l, h, jt);
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            const int t = jt * kC + 2 * lane + e;
-            const size_t gi = ((size_t)l * a.T + t) * a.Hv + h;
-            pg[e] = t < a.T ? a.g[gi] : 0.f;
-            pb[e] = t < a.T ? a.beta[gi] : 0.f;
-        }
-    };
-    // Decay constants of an item from the loaded g, beta (warp 7): the update kernel's -gamma and
-    // gamma_C into the record, and this kernel's G2, beta, row and column factors and
-    // exp(G_C - G) into buffer `buf`.
-    auto tile_constants = [&](int it, int buf) {
-        float incl = pg[0] + pg[1];
-#pragma unroll
-        for (int m = 1; m < 32; m <<= 1) {
-            const float y = __shfl_up_sync(0xffffffffu, incl, m);
-            if (lane >= m) incl += y;
-        }
-        const float G0 = incl - pg[1], G1 = incl;
-        const float GC = __shfl_sync(0xffffffffu, incl, 31);
-        float* rc = reinterpret_cast<float*>(a.rec + (size_t)rec_of(it) * kRecBytes + kRecT);
-        *reinterpret_cast<float2*>(rc + 2 * lane) = make_float2(-expf(G0), -expf(G1));
-        if (lane == 0) *reinterpret_cast<float4*>(rc + 64) = make_float4(expf(GC), 0.f, 0.f, 0.f);
-        const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
-        float lo2 = fminf(g20, g21), hi2 = fmaxf(g20, g21);
-#pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) {
-            lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, m));
-            hi2 = fmaxf(hi2, __shfl_xor_sync(0xffffffffu, hi2, m));
-        }
-        // exp(G_t - G_i) = row_t * col_i with the reference in the middle of the tile's range of
-        // G; both factors stay within 2^+-126 when that range spans at most 250 powers of two,
-        // otherwise the exponent is taken per entry.
-        const float ref = 0.5f * (lo2 + hi2);
-        float* tg = reinterpret_cast<float*>(sm + WY_TG) + buf * kTgFloats;
-        tg[2 * lane] = g20; tg[2 * lane + 1] = g21;
-        tg[64 + 2 * lane] = pb[0]; tg[64 + 2 * lane + 1] = pb[1];
-        tg[128 + 2 * lane] = pb[0] * fast_exp2(g20 - ref); tg[128 + 2 * lane + 1] = pb[1] * fast_exp2(g21 - ref);
-        tg[192 + 2 * lane] = fast_exp2(ref - g20); tg[192 + 2 * lane + 1] = fast_exp2(ref - g21);
-        tg[256 + 2 * lane] = expf(GC - G0); tg[256 + 2 * lane + 1] = expf(GC - G1);
-        if (lane == 0) reinterpret_cast<int*>(tg)[320] = (hi2 - lo2) <= 250.f;
-    };
-
-    // K K^T of the item-th item of this CTA into TMEM (warp 0; M = 128: rows 64..127 of A read the
-    // 8 KB past the tile, their output is ignored)
-    auto issue_kk = [&](int item) {
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(&mb_k, item & 1, kWaitBudgetNs)) != 0;
-        if (!ok) {
-            if (lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 21); s_fail = 1; }
-            return;
-        }
-        tc_fence_after();
-        const uint32_t id = idesc_bf16(128, 64, 0, 0);
-#pragma unroll
-        for (int s = 0; s < 8; ++s) {
-            const uint64_t d = sdesc_sw128(smem_u32(sm + WY_K + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
-            mma_bf16(tm, d, d, id, s > 0);
-        }
-        mma_commit(&mb_kk);
-        ++nkk;
-    };
-
-    const int first = (int)blockIdx.x;
-    if (first < items) {
-        if (tid == 0) load_k(first);
-        if (warp == 7) {
-            load_gb(first);
-            tile_constants(first, 0);
-            if (first + (int)gridDim.x < items) load_gb(first + (int)gridDim.x);
-        }
-    }
-    __syncthreads();
-    int c = 0;                                         // items done by this CTA (barrier phases)
-    for (int it = first; it < items; it += (int)gridDim.x, ++c) {
-        const float* tg = reinterpret_cast<const float*>(sm + WY_TG) + (c & 1) * kTgFloats;
-        const float* sG2 = tg;                         // G * log2(e)
-        const float* sBeta = tg + 64;
-        const float* sRow = tg + 128;                  // beta_t 2^(G2_t - ref)
-        const float* sCol = tg + 192;                  // 2^(ref - G2_i)
-        const float* sDel = tg + 256;                  // exp(G_C - G_t)
-        const int factored = reinterpret_cast<const int*>(tg)[320];
-        if (warp == 0) issue_kk(c);
-        const int q = warp & 3;
-        if (q < 2 && warp != 4) {
-            // TMEM lanes 0..63 hold K K^T: warps 0/4 rows 0..31, 1/5 rows 32..63; column half
-            // (warp >> 2).  Warp 4's quarter (rows 0..31, cols 32..63) lies above the diagonal and
-            // is never needed; warp 1's (rows 32..63, cols 0..31) is A21, stored split.
-            const bool ok = mbar_wait_or_abort(&mb_kk, c & 1, kWaitBudgetNs, &s_fail);
-            if (!ok && lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 22); s_fail = 1; }
-            tc_fence_after();
-            const int t = 32 * q + lane, c0 = 32 * (warp >> 2);
-            const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-            const float rt = factored ? sRow[t] : sBeta[t];
-            const float G2t = sG2[t];
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {     // 16 columns at a time
-                const int cb = c0 + 16 * half;
-                float kk[16], cf[16];
-                tmem_ld16(tm + lane_off + cb, kk);
-                const float* src = factored ? sCol : sG2;
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float4 v4 = *reinterpret_cast<const float4*>(src + cb + 4 * e);
-                    cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
-                }
-                tmem_ld_wait();
-#pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const float f = factored ? cf[e] : fast_exp2(G2t - cf[e]);
-                    kk[e] = (cb + e < t) ? rt * f * kk[e] : 0.f;
-                }
-                if (half == 0 && lane >= 16 && (warp == 0 || warp == 5))   // A10 / A32, split
-                    put_split16((warp == 0 ? sA10 : sA32) + (lane - 16) * kL1S, kk);
-                if (warp == 1) {                       // A21, split
-                    uint32_t* row = sA21 + (t - 32) * FA_S + 8 * half;
-                    uint32_t h[8], l[8];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) split2(kk[2 * i], kk[2 * i + 1], h[i], l[i]);
-                    *reinterpret_cast<uint4*>(row) = make_uint4(h[0], h[1], h[2], h[3]);
-                    *reinterpret_cast<uint4*>(row + 4) = make_uint4(h[4], h[5], h[6], h[7]);
-                    *reinterpret_cast<uint4*>(row + 16) = make_uint4(l[0], l[1], l[2], l[3]);
-                    *reinterpret_cast<uint4*>(row + 20) = make_uint4(l[4], l[5], l[6], l[7]);
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        *reinterpret_cast<float4*>(fA + t * FA_S + cb + 4 * e) =
-                            make_float4(kk[4 * e], kk[4 * e + 1], kk[4 * e + 2], kk[4 * e + 3]);
-                }
-            }
-        }
-        tc_fence_before();
-        __syncthreads();
-        if (s_fail) break;
-        const int nxt = it + (int)gridDim.x;
-        // level 0: four 16 x 16 diagonal blocks of (I + A)^-1, one column per thread (warps 0-1);
-        // meanwhile warp 7 prepares the next item's constants and loads the one after
-        if (tid < 64) {
-            const int B = tid >> 4, jc = tid & 15, o = 16 * B;
-            float x[16];
-#pragma unroll
-            for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
-#pragma unroll
-            for (int rr = 1; rr < 16; ++rr) {
-                float s0 = 0.f, s1 = 0.f;              // two chains: half the dependent FMAs
-#pragma unroll
-                for (int cc = 0; cc < rr; cc += 4) {
-                    const float4 av = *reinterpret_cast<const float4*>(fA + (o + rr) * FA_S + o + cc);
-                    s0 = fmaf(av.x, x[cc], s0);
-                    if (cc + 1 < rr) s1 = fmaf(av.y, x[cc + 1], s1);
-                    if (cc + 2 < rr) s0 = fmaf(av.z, x[cc + 2], s0);
-                    if (cc + 3 < rr) s1 = fmaf(av.w, x[cc + 3], s1);
-                }
-                if (rr > jc) x[rr] = -(s0 + s1);
-            }
-#pragma unroll
-            for (int rr = 0; rr < 16; ++rr) fX[(o + rr) * FX_S + o + jc] = x[rr];
-            if (B == 1) {                              // X11' row-major
-#pragma unroll
-                for (int rr = 0; rr < 16; ++rr) put_split(sX11r + rr * kL1S, jc, x[rr], 8);
-            } else if (B == 2) {                       // X22' n-major
-                put_split16(sX22n + jc * kL1S, x);
-            }
-            if (B < 2) {                               // X11, n-major: row o + jc holds column o + jc
-                uint32_t* row = sX11 + (o + jc) * FA_S;
-                if (B == 1) {                          // X[0..16][16..32] = 0 (the K tile overwrote it)
-                    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-                    *reinterpret_cast<uint4*>(row) = z; *reinterpret_cast<uint4*>(row + 4) = z;
-                    *reinterpret_cast<uint4*>(row + 16) = z; *reinterpret_cast<uint4*>(row + 20) = z;
-                }
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    uint32_t h[4], l[4];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) split2(x[8 * e + 2 * i], x[8 * e + 2 * i + 1], h[i], l[i]);
-                    *reinterpret_cast<uint4*>(row + o / 2 + 4 * e) = make_uint4(h[0], h[1], h[2], h[3]);
-                    *reinterpret_cast<uint4*>(row + 16 + o / 2 + 4 * e) = make_uint4(l[0], l[1], l[2], l[3]);
-                }
-            } else {                                   // X22, row-major
-#pragma unroll
-                for (int rr = 0; rr < 16; ++rr) put_split(sX22 + (o - 32 + rr) * FX_S, o - 32 + jc, x[rr]);
-            }
-        } else if (warp == 7 && nxt < items) {
-            tile_constants(nxt, (c + 1) & 1);
-            if (nxt + (int)gridDim.x < items) load_gb(nxt + (int)gridDim.x);
-        }
-        __syncthreads();
-        // level 1: X[2p+1][2p] = -X[2p+1][2p+1] (A[2p+1][2p] X[2p][2p]) for the 16 x 16 blocks,
-        // p = 0, 1; warps 0-3 take (p, 8-column half) = (warp / 2, warp % 2)
-        const int g = lane >> 2, tq = lane & 3;
-        if (warp < 4) {
-            const int p = warp >> 1, nc = 8 * (warp & 1);
-            float d[4] = {0.f, 0.f, 0.f, 0.f};
-            if (p == 0) mma_split_bf16<1>(d, sA10, kL1S, 8, 0, sX11, FA_S, 16, nc, lane);    // A10 X00
-            else        mma_split_bf16<1>(d, sA32, kL1S, 8, 0, sX22n, kL1S, 8, nc, lane);   // A32 X22'
-            uint32_t* P = sP1 + p * 16 * kL1S;         // n-major
-            put_split(P + (nc + 2 * tq) * kL1S, g, d[0], 8);
-            put_split(P + (nc + 2 * tq + 1) * kL1S, g, d[1], 8);
-            put_split(P + (nc + 2 * tq) * kL1S, g + 8, d[2], 8);
-            put_split(P + (nc + 2 * tq + 1) * kL1S, g + 8, d[3], 8);
-        }
-        __syncthreads();
-        if (warp < 4) {
-            const int p = warp >> 1, nc = 8 * (warp & 1);
-            const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
-            const uint32_t* P = sP1 + p * 16 * kL1S;
-            float d[4] = {0.f, 0.f, 0.f, 0.f};
-            if (p == 0) mma_split_bf16<1>(d, sX11r, kL1S, 8, 0, P, kL1S, 8, nc, lane);        // X11' P1
-            else        mma_split_bf16<1>(d, sX22 + 16 * FX_S + 8, FX_S, 16, 0, P, kL1S, 8, nc, lane);  // X33' P1'
-            fX[(ro + g) * FX_S + co + nc + 2 * tq] = -d[0]; fX[(ro + g) * FX_S + co + nc + 2 * tq + 1] = -d[1];
-            fX[(ro + g + 8) * FX_S + co + nc + 2 * tq] = -d[2]; fX[(ro + g + 8) * FX_S + co + nc + 2 * tq + 1] = -d[3];
-            if (p == 0) {                              // X[16..32][0..16] into X11, n-major
-                put_split(sX11 + (nc + 2 * tq) * FA_S, 16 + g, -d[0]);
-                put_split(sX11 + (nc + 2 * tq + 1) * FA_S, 16 + g, -d[1]);
-                put_split(sX11 + (nc + 2 * tq) * FA_S, 24 + g, -d[2]);
-                put_split(sX11 + (nc + 2 * tq + 1) * FA_S, 24 + g, -d[3]);
-            } else {                                   // X[48..64][32..48] into X22, row-major
-                put_split(sX22 + (16 + g) * FX_S, nc + 2 * tq, -d[0]);
-                put_split(sX22 + (16 + g) * FX_S, nc + 2 * tq + 1, -d[1]);
-                put_split(sX22 + (24 + g) * FX_S, nc + 2 * tq, -d[2]);
-                put_split(sX22 + (24 + g) * FX_S, nc + 2 * tq + 1, -d[3]);
-            }
-        }
-        __syncthreads();
-        // level 2: X[32:64][0:32] = -X[32:64][32:64] (A[32:64][0:32] X[0:32][0:32]) from the split
-        // operands; warp w takes the 16 x 8 output tile (w / 4, w % 4).  P = A21 X11 goes to fT
-        // split and n-major.
-        {
-            const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
-            float d[4] = {0.f, 0.f, 0.f, 0.f};
-            mma_split_bf16<2>(d, sA21, FA_S, 16, mr, sX11, FA_S, 16, nc, lane);
-            put_split(sP + (nc + 2 * tq) * kPS, mr + g, d[0]);
-            put_split(sP + (nc + 2 * tq + 1) * kPS, mr + g, d[1]);
-            put_split(sP + (nc + 2 * tq) * kPS, mr + g + 8, d[2]);
-            put_split(sP + (nc + 2 * tq + 1) * kPS, mr + g + 8, d[3]);
-        }
-        __syncthreads();
-        // A (fp32 and split) has been read for the last time: the next item's K tile lands there
-        if (tid == 0 && nxt < items) load_k(nxt);
-        {
-            const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
-            float d[4] = {0.f, 0.f, 0.f, 0.f};
-            mma_split_bf16<2>(d, sX22, FX_S, 16, mr, sP, kPS, 16, nc, lane);
-            fX[(32 + mr + g) * FX_S + nc + 2 * tq] = -d[0]; fX[(32 + mr + g) * FX_S + nc + 2 * tq + 1] = -d[1];
-            fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq] = -d[2]; fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq + 1] = -d[3];
-        }
-        __syncthreads();
-        // T~ = diag(exp(G_C - G)) X diag(beta) (upper part zero), split into the record's (hi, lo)
-        // images
-        {
-            uint8_t* rec = a.rec + (size_t)rec_of(it) * kRecBytes;
-#pragma unroll
-            for (int m = 0; m < 2; ++m) {
-                const int e = tid + kWyThreads * m;
-                const int t = e >> 3, c8 = e & 7;
-                uint4 vh = make_uint4(0u, 0u, 0u, 0u), vl = vh;
-                if (8 * c8 <= t) {                     // chunks right of the diagonal stay zero
-                    const float dt = sDel[t];
-                    const float4 x0 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8);
-                    const float4 x1 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8 + 4);
-                    const float4 b0 = *reinterpret_cast<const float4*>(sBeta + 8 * c8);
-                    const float4 b1 = *reinterpret_cast<const float4*>(sBeta + 8 * c8 + 4);
-                    const float xs[8] = {x0.x * b0.x, x0.y * b0.y, x0.z * b0.z, x0.w * b0.w,
-                                         x1.x * b1.x, x1.y * b1.y, x1.z * b1.z, x1.w * b1.w};
-                    float x[8];
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) x[k] = (8 * c8 + k <= t) ? dt * xs[k] : 0.f;
-                    split8(x, vh, vl);
-                }
-                *reinterpret_cast<uint4*>(rec + sw128_offset(t, c8)) = vh;
-                *reinterpret_cast<uint4*>(rec + 8192 + sw128_offset(t, c8)) = vl;
-            }
-        }
-        // the next item's level 0 rewrites fX's diagonal blocks: everyone has read this one's
-        __syncthreads();
-    }
-    if (tid == 0 && s_fail) {
-        // after a failure: the last K load and K K^T product issued land before TMEM is freed
-        if (nk > 0) mbar_wait(&mb_k, (nk - 1) & 1, kWaitBudgetNs);
-        if (nkk > 0) mbar_wait(&mb_kk, (nkk - 1) & 1, kWaitBudgetNs);
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) {
-        tc_fence_after();
-        tmem_dealloc(tm, kWyTmemCols);
-    }
-}
-
-// =============================================================================================
-// Update kernel: the state chain
-// =============================================================================================
-__device__ __forceinline__ int ho_load_acquire(const int32_t* p) {
+__device__ __forceinline__ int ld_acquire(const uint32_t* p) {
     int v;
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
-__device__ __forceinline__ void ho_store_release(int32_t* p, int v) {
-    asm volatile("st.release.gpu.global.b32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
-}
-// orders the tensor copies' global accesses with the generic ones around a hand-over flag
+// orders the tensor copies' global accesses with the generic ones around a hand-over bit
 __device__ __forceinline__ void fence_proxy_async_global() {
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-constexpr int kChainWarps = 16;
-constexpr int kChain = 32 * kChainWarps;         // chain threads
-constexpr int kMmaWarp = kChainWarps;            // 16
-constexpr int kLoadWarp = kChainWarps + 1;       // 17
-constexpr int kStateWarp = kChainWarps + 2;      // 18
-constexpr int kThreads = kChain + 96;
-constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t TM_S = 0, TM_SB = 128, TM_X = 256, TM_U = 320, TM_V = 384;
-
-// shared-memory map (bytes from a 1024-aligned base)
-constexpr uint32_t SM_K = 0;                     // 3 x 16 KB: K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
-constexpr uint32_t SM_K32 = 49152;               // 32 KB: K in fp32 (the B operand of X), 4 column blocks
-                                                 // (32 dims) x 64 rows x 128 B, SW128
-constexpr uint32_t SM_V = 81920;                 // 2 x 16 KB: V tile (tile parity), layout of K
-constexpr uint32_t SM_R = 114688;                // 2 x kRecSlot: WY records (tile parity)
-constexpr uint32_t kRecSlot = 17408;             // 1024-aligned slots
-constexpr uint32_t SM_I = SM_R + 2 * kRecSlot;   // 8 KB: 64 x 64 bfloat16 identity, K-major SW128
-constexpr uint32_t SM_SB = SM_I + 8192;          // 64 KB: state staging, 4 column blocks x 128 rows x 128 B, SW128
-constexpr uint32_t SM_BYTES = SM_SB + 65536;
-constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
-static_assert(SM_I % 1024 == 0 && SM_SB % 1024 == 0 && kRecSlot >= kRecBytes, "shared-memory map");
-static_assert(kSmemAlloc <= 232448, "shared memory budget");
-
-// The staging buffer holds a head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each
-// 128 rows x 128 bytes with the 128-byte swizzle (16-byte chunk ^ (row & 7)) that TMA writes and
-// reads; eight threads reading chunk c of eight consecutive rows (one row per thread) hit distinct
-// banks.  Float offset of 16-byte chunk `chunk` (0..31) of row `row`:
-__device__ __forceinline__ int sb_idx(int row, int chunk) {
-    return (chunk >> 3) * 4096 + row * 32 + (((chunk & 7) ^ (row & 7)) << 2);
+// The per-sub-tile decay bookkeeping (see the header): from p = gamma_C sig, the shift s, the
+// scale u of the V term, the coefficient c of the X term, the pass factor (< 0: no pass) and sig
+// after the sub-tile.
+struct DecayStep {
+    int shift;
+    float u, c, pass, sig;
+};
+__device__ __forceinline__ DecayStep decay_step(float p) {
+    DecayStep d;
+    if (!(p >= kHardMin)) {                            // also p = 0 or NaN-free underflow
+        d.shift = 0; d.u = 1.f; d.c = p; d.pass = p; d.sig = 1.f;
+        return d;
+    }
+    int e;
+    (void)frexpf(p, &e);                               // p = m 2^e, m in [1/2, 1)
+    d.shift = min(15, max(0, -e));
+    d.sig = ldexpf(p, d.shift);
+    d.u = 1.f / d.sig;
+    d.c = ldexpf(1.f, -d.shift);
+    d.pass = -1.f;
+    return d;
 }
 
 struct TcArgs {
-    int L, Hk, Hv, T, n_tiles;
+    int L, Hk, Hv, T, n_tiles;   // n_tiles: 64-token tiles per head
+    const float* g;              // [L][T][Hv] log-decay
+    const float* beta;           // [L][T][Hv]
     float* state;
     float* partials;
     float* wnorm;
-    const uint8_t* rec;
     int32_t* status;
-    int split;               // run equal tile runs (ChainSched), when the host found it faster
-    // hand-over between neighbouring CTAs of a head split between them (see ChainSched): one
-    // entry per CTA boundary i (CTA i -> CTA i + 1)
-    int32_t* ho_flag;        // [grid] the state after the first part is in the hand-over map
-    int32_t* ho_wflag;       // [grid] the first part's write-size sum is in ho_wsum
-    float* ho_wsum;          // [grid]
+    uint32_t* ho_bits;           // hand-over bits in the workspace header: [0, 16) state, [16, 32) sums
+    float* ho_wsum;              // [grid]
+    int split;                   // run equal tile runs (ChainSched)
 };
 
 // The CTA's work: a sequence of slots, each a run of consecutive tiles of one head.  By default
 // the CTA owns heads blockIdx.x, blockIdx.x + gridDim.x, ... whole.  When the heads do not divide
 // evenly among the CTAs and the host estimates it faster (a.split), the CTAs instead take equal
 // runs of the tile sequence in head order, so that the slowest CTA has one tile more than the
-// fastest instead of a whole head more; a head cut by a run boundary is shared by two neighbours.  CTA i runs the head
-// it shares with CTA i + 1 first (its first tiles; the state at the cut goes to hand-over entry i)
-// and the head it shares with CTA i - 1 last (its last tiles, from hand-over entry i - 1), so the
-// second part of a shared head is never waited for before its first part is long finished.
+// fastest instead of a whole head more; a head cut by a run boundary is shared by two neighbours.
+// CTA i runs the head it shares with CTA i + 1 first (its first tiles; the state at the cut goes
+// to hand-over entry i) and the head it shares with CTA i - 1 last (its last tiles, from hand-over
+// entry i - 1), so the second part of a shared head is never waited for before its first part is
+// long finished.  The split schedule is launched cooperatively, so every CTA is resident.
 struct ChainSched {
     int split;
     int pre_lh, pre_len;       // first slot: tiles [0, pre_len) of head pre_lh (none if pre_len == 0)
@@ -722,13 +261,11 @@ struct ChainSched {
     }
 };
 
-// Where the CTA's current tile lies: slot k, tile jt (of [tb, te)) of head lh = (layer l, value
-// head h), key head kh.  Each role walks the tiles in order; a step costs integer divisions only
-// when it crosses into the next slot.
+// Where a role's current tile lies: slot k, tile jt (of [tb, te)) of head lh = (layer l, value
+// head h), key head kh.
 struct TileCursor {
-    int k, jt, te, lh, l, h, kh;
+    int k, jt, tb, te, lh, l, h, kh;
     __device__ __forceinline__ void set_slot(int slot, const ChainSched& sc, const TcArgs& a) {
-        int tb;
         k = slot;
         sc.slot(slot, a.n_tiles, lh, tb, te);
         jt = tb;
@@ -736,6 +273,7 @@ struct TileCursor {
         kh = (int)(((long long)h * a.Hk) / a.Hv);
     }
     __device__ __forceinline__ void init(const ChainSched& sc, const TcArgs& a) {
+        k = -1;
         if (sc.n_slots > 0) set_slot(0, sc, a);
     }
     __device__ __forceinline__ void next(const ChainSched& sc, const TcArgs& a) {
@@ -743,224 +281,270 @@ struct TileCursor {
     }
 };
 
+// The staging buffer holds a head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each
+// 128 rows x 128 bytes with the 128-byte swizzle that TMA writes and reads.  Float offset of 16-byte
+// chunk `chunk` (0..31) of row `row`:
+__device__ __forceinline__ int sb_idx(int row, int chunk) {
+    return (chunk >> 3) * 4096 + row * 32 + (((chunk & 7) ^ (row & 7)) << 2);
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                     const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap hmap,
-                     TcArgs a)
+gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                 const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap hmap,
+                 TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
-    // copies -> roles: K (3), V (2), WY records (2) full; MMA -> loader: their empties; state
-    // staging full (mb_st) and released by the chain (mb_sfree); MMA -> chain: x, u, s; chain ->
-    // MMA: ready flags.
-    __shared__ uint64_t mb_tk[3], mb_ke[3], mb_tv[2], mb_ve[2], mb_tr[2], mb_re[2];
-    __shared__ uint64_t mb_st, mb_sfree, mb_x, mb_u, mb_s, mb_sready, mb_xready, mb_uready, mb_fin;
+    // loads -> roles: K tiles, V sub-tiles full; MMA -> loader: their empties.  producer <-> MMA:
+    // operand images full / empty (the chain's constants read too), K K^T done / read.  state
+    // staging full (mb_st) and released by the chain (mb_sfree).  MMA -> chain: u (E ready), s
+    // (state updated); chain -> MMA: sready (state and K in fp32 ready for X), uready (A packed).
+    __shared__ uint64_t mb_kfull[3], mb_kempty[3], mb_vfull[3], mb_vempty[3], mb_ifull[4], mb_iempty[4];
+    __shared__ uint64_t mb_kk, mb_kkfree, mb_st, mb_sfree, mb_sready, mb_x, mb_u, mb_uready, mb_s, mb_fin;
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ float s_red[2][kChainWarps];
-    __shared__ float s_u2[2][kC];                 // per-token squared write sizes (tile parity)
+    __shared__ float s_u2[2][kC];                     // per-token squared write sizes (sub-tile parity)
     volatile int* abort_flag = &s_abort;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int n = a.n_tiles;
-    // Persistent CTA: its slots (ChainSched) form one sequence of NJ tiles, over which every role
-    // keeps its barrier phases.
+    // bounded-wait budget: the workspace header's override (microseconds) or about one second
+    const uint32_t budget_us = reinterpret_cast<const volatile uint32_t*>(a.status)[2];
+    const uint64_t budget = budget_us ? (uint64_t)budget_us * 1000ull : kWaitBudgetNs;
     ChainSched sch;
     sch.init(a);
     const int n_slots = sch.n_slots;
-    const int NJ = sch.NJ;
+    const int NJ = sch.NJ;                            // tiles of this CTA
+    const int NS = 2 * NJ;                            // sub-tiles
+    const int me = (int)blockIdx.x;
+    uint32_t* bits_state = a.ho_bits;
+    uint32_t* bits_wsum = a.ho_bits + 16;
 
     if (warp == kMmaWarp) {
         tmem_alloc(&s_tmem, kTmemCols);
         tmem_relinquish();
         if (lane == 0) {
-            for (int b = 0; b < 3; ++b) { mbar_init(&mb_tk[b], 1); mbar_init(&mb_ke[b], 1); }
-            for (int b = 0; b < 2; ++b) {
-                mbar_init(&mb_tv[b], 1); mbar_init(&mb_ve[b], 1);
-                mbar_init(&mb_tr[b], 1); mbar_init(&mb_re[b], 1);
+            for (int b = 0; b < 3; ++b) {
+                mbar_init(&mb_kfull[b], 1); mbar_init(&mb_kempty[b], 1);
+                mbar_init(&mb_vfull[b], 1); mbar_init(&mb_vempty[b], 1);
             }
+            for (int b = 0; b < 4; ++b) { mbar_init(&mb_ifull[b], 2); mbar_init(&mb_iempty[b], 1 + kChainWarps); }
+            mbar_init(&mb_kk, 1); mbar_init(&mb_kkfree, 2);
             mbar_init(&mb_st, 1); mbar_init(&mb_sfree, kChainWarps);
-            mbar_init(&mb_x, 1); mbar_init(&mb_u, 1); mbar_init(&mb_s, 1);
-            mbar_init(&mb_sready, kChainWarps); mbar_init(&mb_xready, kChainWarps);
+            mbar_init(&mb_sready, kChainWarps); mbar_init(&mb_x, 1); mbar_init(&mb_u, 1);
             mbar_init(&mb_uready, kChainWarps);
-            mbar_init(&mb_fin, 1);
+            mbar_init(&mb_s, 1); mbar_init(&mb_fin, 1);
             fence_barrier_init();
         }
     }
     if (warp == kLoadWarp && lane == 0) { prefetch_tensormap(&kmap); prefetch_tensormap(&vmap); }
     if (warp == kStateWarp && lane == 0) { prefetch_tensormap(&smap); prefetch_tensormap(&hmap); }
-    if (tid < kChain) {
-        // the 64 x 64 identity (B operand of V^T I): row t holds 1.0 at column t
-        const int t = tid >> 3, c8 = tid & 7;
-        uint32_t w[4] = {0u, 0u, 0u, 0u};
-        if ((t >> 3) == c8) w[(t & 7) >> 1] = (t & 1) ? 0x3F800000u : 0x00003F80u;
-        *reinterpret_cast<uint4*>(sm + SM_I + sw128_offset(t, c8)) = make_uint4(w[0], w[1], w[2], w[3]);
-        fence_async_smem();
-    }
     if (tid == 0) s_abort = 0;
-    if (tid < 2 * kC) s_u2[tid >> 6][tid & (kC - 1)] = 0.f;
-    grid_dep_launch();                                 // the next kernel (the score) may be scheduled
+    if (tid < 2 * kC) s_u2[tid >> 5][tid & (kC - 1)] = 0.f;
+    grid_dep_launch();                                // the next kernel (the score) may be scheduled
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tm = s_tmem;
+    const float* cst = reinterpret_cast<const float*>(sm + SM_CONST);
 
     if (warp == kMmaWarp) {
         // =========================================================== MMA issue (converged warp;
         // one elected lane issues each group and commits it)
-        const uint64_t dK = sdesc_sw128(smem_u32(sm + SM_K), 8192, 1024);    // MN-major B of MMA_S
-        const uint64_t dK32 = sdesc_sw128(smem_u32(sm + SM_K32), 16, 1024);
-        const uint64_t dV = sdesc_sw128(smem_u32(sm + SM_V), 8192, 1024);    // MN-major A of V^T I
-        const uint64_t dR = sdesc_sw128(smem_u32(sm + SM_R), 16, 1024);
-        const uint64_t dI = sdesc_sw128(smem_u32(sm + SM_I), 16, 1024);
-        // Each group's operands are formed before the wait that releases it, so that only the
-        // MMA instructions themselves follow the wait (this warp shares its scheduler with four
-        // chain warps).
-        // V region <- V(J)^T: A = the V tile read MN-major (k-step s = tokens 16 s ..), B = I.  V(J)'s
-        // buffer is released when the product completes.
-        auto issue_vi = [&](int J) -> bool {
-            uint64_t av[4], bv[4];
+        const uint32_t idX = idesc_tf32(128, 32);
+        const uint32_t idE = idesc_bf16(128, 64, 1, 0);
+        const uint32_t idS = idesc_bf16(128, 128, 0, 1);
+        const uint32_t idK = idesc_bf16(128, 64, 0, 0);
+        // K K^T of tile J (M = 128: rows 64..127 of A read the 16 KB past the tile; their output
+        // lanes are ignored).  Waits for the tile and for both producer groups to have read the
+        // previous product out of TMEM.
+        auto issue_kk = [&](int J) -> bool {
+            const uint32_t base = smem_u32(sm + SM_K + (J % 3) * 16384);
+            uint64_t d[2][4];
 #pragma unroll
-            for (int s = 0; s < 4; ++s) {
-                av[s] = dadd(dV, (J & 1) * 16384 + s * 2048); bv[s] = dadd(dI, s * 32);
-                pin(av[s]); pin(bv[s]);
+            for (int s = 0; s < 8; ++s) {
+                d[s >> 2][s & 3] = sdesc_sw128(base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
+                pin(d[s >> 2][s & 3]);
             }
-            if (!warp_wait(&mb_tv[J & 1], (J >> 1) & 1, kWaitBudgetNs, abort_flag)) return false;
+            if (!warp_wait(&mb_kfull[J % 3], (J / 3) & 1, budget, abort_flag)) return false;
+            if (J > 0 && !warp_wait(&mb_kkfree, (J - 1) & 1, budget, abort_flag)) return false;
             tc_fence_after();
-            if (elect_one()) mma4_bf16_ss_1t(tm + TM_V, av, bv, idesc_bf16(128, 64, 1, 0), 0);
+            if (elect_one()) {
+                mma4_bf16_ss_1t(tm + TM_KK, d[0], d[0], idK, 0);
+                mma4_bf16_ss_1t(tm + TM_KK, d[1], d[1], idK, 1);
+            }
             __syncwarp();
-            mma_commit(&mb_ve[J & 1]);
+            mma_commit(&mb_kk);
             return true;
         };
-        bool ok = NJ == 0 || issue_vi(0);
-        if (!ok) fail(a.status, abort_flag, 1);
-        for (int j = 0; ok && j < NJ; ++j) {           // j: global tile index
-            {   // X region <- S~ K^T: A = the fp32 state from TMEM read as tf32 (8 columns per K = 8
-                // step), B = K in fp32.  Tile j ready for X: K(j) is converted and, at a head's first
-                // tile, the state is in TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe
-                // order).
+        // E(j) <- V(j)^T B1(j): A = the V sub-tile read MN-major, B = the 64-row (hi, lo) image
+        auto issue_einit = [&](int j) -> bool {
+            const uint32_t vb = smem_u32(sm + SM_V + (j % 3) * 8192);
+            const uint32_t ib = smem_u32(sm + SM_IMG + (j & 3) * kImgSlot);
+            const uint64_t a0 = sdesc_sw128(vb, 4096, 1024), a1 = sdesc_sw128(vb + 2048, 4096, 1024);
+            const uint64_t b0 = sdesc_sw128(ib, 16, 1024), b1 = sdesc_sw128(ib + 32, 16, 1024);
+            pin(a0); pin(a1); pin(b0); pin(b1);
+            if (!warp_wait(&mb_vfull[j % 3], (j / 3) & 1, budget, abort_flag)) return false;
+            if (!warp_wait(&mb_ifull[j & 3], (j >> 2) & 1, budget, abort_flag)) return false;
+            tc_fence_after();
+            if (elect_one()) {
+                mma_bf16_1t(tm + TM_E + (j & 1) * 64, a0, b0, idE, 0);
+                mma_bf16_1t(tm + TM_E + (j & 1) * 64, a1, b1, idE, 1);
+            }
+            __syncwarp();
+            mma_commit(&mb_vempty[j % 3]);
+            return true;
+        };
+        bool ok = true;
+        if (NS > 0) {
+            ok = issue_kk(0);
+            if (ok && NJ > 1) ok = issue_kk(1);
+            if (ok) ok = issue_einit(0);            // completes before X(0)'s commit
+            if (!ok) fail(a.status, abort_flag, 1);
+        }
+        // The tensor core does not order an MMA that reads a TMEM region as its A operand after an
+        // earlier MMA that wrote it (measured: X read by the next product lacked the last of its 16
+        // k-steps), so each such hand-off waits for the writer's commit: X before E += X B2, and
+        // the updated state before the next X.  Independent work fills the turnarounds: the next
+        // sub-tile's E product between X and E += X B2, the K K^T product during the chain's pass.
+        for (int j = 0; ok && j < NS; ++j) {
+            const uint32_t eb = tm + TM_E + (j & 1) * 64;
+            int shift = 0;
+            {   // X <- S~ K^T (A: the state from TMEM as tf32, 8 columns per K = 8 step; B: K in fp32)
                 uint32_t ax[4][4];
                 uint64_t bx[4][4];
+                const uint32_t k32 = smem_u32(sm + SM_K32);
 #pragma unroll
                 for (int s = 0; s < 16; ++s) {
                     ax[s >> 2][s & 3] = tm + TM_S + 8 * s;
-                    bx[s >> 2][s & 3] = dadd(dK32, (s >> 2) * 8192 + (s & 3) * 32);
+                    bx[s >> 2][s & 3] = sdesc_sw128(k32 + (s >> 2) * 4096 + (s & 3) * 32, 16, 1024);
                     pin(ax[s >> 2][s & 3]); pin(bx[s >> 2][s & 3]);
                 }
-                if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
+                if (!warp_wait(&mb_sready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 2); break; }
+                if (j > 0 && !warp_wait(&mb_s, (j - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 7); break; }
+                if (!warp_wait(&mb_ifull[j & 3], (j >> 2) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 3); break; }
+                // read while the image slot is held (released once its products and the chain are done)
+                shift = reinterpret_cast<const volatile int*>(cst + (j & 3) * kConstWords)[34];
                 tc_fence_after();
                 if (elect_one()) {
 #pragma unroll
-                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + TM_X, ax[g4], bx[g4], idesc_tf32(128, 64), g4 != 0);
+                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + TM_X, ax[g4], bx[g4], idX, g4 != 0);
                 }
                 __syncwarp();
                 mma_commit(&mb_x);
             }
-            {   // U region <- W^T T~^T with W (hi, lo) packed in place in X (k-step s: hi at column
-                // 16 s, lo at 16 s + 8): W hi T~ hi + W hi T~ lo + W lo T~ hi
-                uint32_t au[3][4];
-                uint64_t bu[3][4];
-                const uint32_t rb = (j & 1) * kRecSlot;
+            if (j + 1 < NS && !issue_einit(j + 1)) { fail(a.status, abort_flag, 5); break; }
+            {   // E(j) += X B2 (A: X from TMEM as tf32); E(j)'s own product completed before X's commit
+                uint32_t au[4];
+                uint64_t bu[4];
+                const uint32_t b2 = smem_u32(sm + SM_IMG + (j & 3) * kImgSlot + 8192);
 #pragma unroll
-                for (int part = 0; part < 3; ++part) {
-#pragma unroll
-                    for (int s = 0; s < 4; ++s) {
-                        au[part][s] = tm + TM_X + 16 * s + (part == 2 ? 8 : 0);
-                        bu[part][s] = dadd(dR, rb + (part == 1 ? 8192 : 0) + s * 32);
-                        pin(au[part][s]); pin(bu[part][s]);
-                    }
+                for (int s = 0; s < 4; ++s) {
+                    au[s] = tm + TM_X + 8 * s;
+                    bu[s] = sdesc_sw128(b2 + 32 * s, 16, 1024);
+                    pin(au[s]); pin(bu[s]);
                 }
-                if (!warp_wait(&mb_xready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 5); break; }
-                if (!warp_wait(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 3); break; }
+                if (!warp_wait(&mb_x, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 8); break; }
                 tc_fence_after();
-                if (elect_one()) {
-#pragma unroll
-                    for (int part = 0; part < 3; ++part)
-                        mma4_bf16_ta_1t(tm + TM_U, au[part], bu[part], idesc_bf16(128, 64, 0, 0), part != 0);
-                }
+                if (elect_one()) mma4_tf32_ta_1t(eb, au, bu, idX, 1);
                 __syncwarp();
                 mma_commit(&mb_u);
-                mma_commit(&mb_re[j & 1]);             // record slot free once MMA_U(j) has read T~
+                mma_commit(&mb_iempty[j & 3]);
             }
-            // the next tile's V^T into the V region (its last reader, the W pass of tile j, has
-            // finished: MMA_U(j) waited for xready)
-            if (j + 1 < NJ && !issue_vi(j + 1)) { fail(a.status, abort_flag, 4); break; }
-            {   // S~ += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major)
-                uint32_t as_[2][4];
-                uint64_t bs[2][4];
-                const uint32_t kb = (j % 3) * 16384;
+            // K K^T one and a half tiles ahead of the chain, while the chain runs its pass
+            if ((j & 1) && (j + 3) / 2 < NJ && !issue_kk((j + 3) / 2)) { fail(a.status, abort_flag, 4); break; }
+            {   // S~ = 2^-shift S~ + E K  (A: E hi / lo packed in TMEM; K read MN-major)
+                uint32_t as_[4];
+                uint64_t bs[4];
+                const uint32_t kb = smem_u32(sm + SM_K + ((j >> 1) % 3) * 16384) + (j & 1) * 4096;
 #pragma unroll
-                for (int part = 0; part < 2; ++part) {
-#pragma unroll
-                    for (int s = 0; s < 4; ++s) {
-                        as_[part][s] = tm + TM_U + 16 * s + (part == 1 ? 8 : 0);
-                        bs[part][s] = dadd(dK, kb + s * 2048);
-                        pin(as_[part][s]); pin(bs[part][s]);
-                    }
+                for (int s = 0; s < 4; ++s) {
+                    as_[s] = tm + TM_AP + 8 * s;
+                    bs[s] = sdesc_sw128(kb + (s & 1) * 2048, 8192, 1024);
+                    pin(as_[s]); pin(bs[s]);
                 }
-                if (!warp_wait(&mb_uready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 7); break; }
+                if (!warp_wait(&mb_uready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 6); break; }
                 tc_fence_after();
-                if (elect_one()) {
-#pragma unroll
-                    for (int part = 0; part < 2; ++part)
-                        mma4_bf16_ta_1t(tm + TM_S, as_[part], bs[part], idesc_bf16(128, 128, 0, 1), 1);
-                }
+                if (elect_one()) mma4_bf16_ta_shift_1t(shift, tm + TM_S, as_, bs, idS);
                 __syncwarp();
                 mma_commit(&mb_s);
-                mma_commit(&mb_ke[j % 3]);             // K(j)'s buffer free once MMA_S(j) has read it
+                if (j & 1) mma_commit(&mb_kempty[(j >> 1) % 3]);   // the tile's last reader
             }
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0)) {
             mma_commit(&mb_fin);                       // every MMA this warp issued has completed
-            mbar_wait(&mb_fin, 0, kWaitBudgetNs);
+            mbar_wait(&mb_fin, 0, budget);
         }
         __syncwarp();
     } else if (warp == kLoadWarp) {
-        // =========================================================== K, V, records in tile order,
-        // each into its buffer once the MMA that last read the buffer has completed
-        TileCursor cc;
+        // =========================================================== K tiles and V sub-tiles in
+        // order, each into its buffer once the MMA that last read the buffer has completed; the
+        // tiles three ahead are prefetched into L2
+        TileCursor cc, pf;
         cc.init(sch, a);
-        int kp[3] = {-1, -1, -1}, vp[2] = {-1, -1}, rp[2] = {-1, -1};   // last tile loaded per buffer
-        // the kernel may start while the factor kernel finishes (its set-up and the first state
-        // load overlap that tail); the records it wrote are read only after it has completed
+        pf.init(sch, a);
+        int kp[3] = {-1, -1, -1}, vp[3] = {-1, -1, -1};   // last tile / sub-tile loaded per buffer
         grid_dep_wait();
-        for (int J = 0; J < NJ; ++J) {
-            const int bk = J % 3, b2 = J & 1;
-            if (J >= 3 && !warp_wait(&mb_ke[bk], ((J / 3) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 30); break; }
+        // prime the prefetch cursor three tiles ahead
+        for (int i = 0; i < 3 && i < NJ; ++i) {
+            if (elect_one()) {
+                tma_prefetch_4d(&kmap, 0, pf.kh, pf.jt * kTile, pf.l);
+                tma_prefetch_4d(&kmap, 64, pf.kh, pf.jt * kTile, pf.l);
+                tma_prefetch_4d(&vmap, 0, pf.h, pf.jt * kTile, pf.l);
+                tma_prefetch_4d(&vmap, 64, pf.h, pf.jt * kTile, pf.l);
+                tma_prefetch_4d(&vmap, 0, pf.h, pf.jt * kTile + kC, pf.l);
+                tma_prefetch_4d(&vmap, 64, pf.h, pf.jt * kTile + kC, pf.l);
+            }
+            __syncwarp();
+            pf.next(sch, a);
+        }
+        bool ok = true;
+        for (int J = 0; ok && J < NJ; ++J) {
+            if (J + 3 < NJ) {
+                if (elect_one()) {
+                    tma_prefetch_4d(&kmap, 0, pf.kh, pf.jt * kTile, pf.l);
+                    tma_prefetch_4d(&kmap, 64, pf.kh, pf.jt * kTile, pf.l);
+                    tma_prefetch_4d(&vmap, 0, pf.h, pf.jt * kTile, pf.l);
+                    tma_prefetch_4d(&vmap, 64, pf.h, pf.jt * kTile, pf.l);
+                    tma_prefetch_4d(&vmap, 0, pf.h, pf.jt * kTile + kC, pf.l);
+                    tma_prefetch_4d(&vmap, 64, pf.h, pf.jt * kTile + kC, pf.l);
+                }
+                __syncwarp();
+                pf.next(sch, a);
+            }
+            const int bk = J % 3;
+            if (J >= 3 && !warp_wait(&mb_kempty[bk], ((J / 3) - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 30); break; }
             if (elect_one()) {
                 uint8_t* dst = sm + SM_K + bk * 16384;
-                mbar_arrive_expect_tx(&mb_tk[bk], 16384);
-                tma_load_4d(dst, &kmap, &mb_tk[bk], 0, cc.kh, cc.jt * kC, cc.l);
-                tma_load_4d(dst + 8192, &kmap, &mb_tk[bk], 64, cc.kh, cc.jt * kC, cc.l);
+                mbar_arrive_expect_tx(&mb_kfull[bk], 16384);
+                tma_load_4d(dst, &kmap, &mb_kfull[bk], 0, cc.kh, cc.jt * kTile, cc.l);
+                tma_load_4d(dst + 8192, &kmap, &mb_kfull[bk], 64, cc.kh, cc.jt * kTile, cc.l);
             }
             __syncwarp();
             kp[bk] = J;
-            if (J >= 2 && !warp_wait(&mb_ve[b2], ((J >> 1) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 31); break; }
-            if (elect_one()) {
-                uint8_t* dst = sm + SM_V + b2 * 16384;
-                mbar_arrive_expect_tx(&mb_tv[b2], 16384);
-                tma_load_4d(dst, &vmap, &mb_tv[b2], 0, cc.h, cc.jt * kC, cc.l);
-                tma_load_4d(dst + 8192, &vmap, &mb_tv[b2], 64, cc.h, cc.jt * kC, cc.l);
+            for (int u = 0; u < 2; ++u) {
+                const int j = 2 * J + u, bv = j % 3;
+                if (j >= 3 && !warp_wait(&mb_vempty[bv], ((j / 3) - 1) & 1, budget, abort_flag)) {
+                    fail(a.status, abort_flag, 31);
+                    ok = false;
+                    break;
+                }
+                if (elect_one()) {
+                    uint8_t* dst = sm + SM_V + bv * 8192;
+                    mbar_arrive_expect_tx(&mb_vfull[bv], 8192);
+                    tma_load_4d(dst, &vmap, &mb_vfull[bv], 0, cc.h, cc.jt * kTile + kC * u, cc.l);
+                    tma_load_4d(dst + 4096, &vmap, &mb_vfull[bv], 64, cc.h, cc.jt * kTile + kC * u, cc.l);
+                }
+                __syncwarp();
+                vp[bv] = j;
             }
-            __syncwarp();
-            vp[b2] = J;
-            if (J >= 2 && !warp_wait(&mb_re[b2], ((J >> 1) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 32); break; }
-            if (elect_one()) {
-                mbar_arrive_expect_tx(&mb_tr[b2], kRecBytes);
-                bulk_load_tx(sm + SM_R + b2 * kRecSlot, a.rec + ((size_t)cc.lh * n + cc.jt) * kRecBytes,
-                             kRecBytes, &mb_tr[b2]);
-            }
-            __syncwarp();
-            rp[b2] = J;
             cc.next(sch, a);
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0) && lane == 0) {
             // every copy this warp issued lands before the CTA ends
-            for (int b = 0; b < 3; ++b)
-                if (kp[b] >= 0) mbar_wait(&mb_tk[b], (kp[b] / 3) & 1, kWaitBudgetNs);
-            for (int b = 0; b < 2; ++b) {
-                if (vp[b] >= 0) mbar_wait(&mb_tv[b], (vp[b] >> 1) & 1, kWaitBudgetNs);
-                if (rp[b] >= 0) mbar_wait(&mb_tr[b], (rp[b] >> 1) & 1, kWaitBudgetNs);
+            for (int b = 0; b < 3; ++b) {
+                if (kp[b] >= 0) mbar_wait(&mb_kfull[b], (kp[b] / 3) & 1, budget);
+                if (vp[b] >= 0) mbar_wait(&mb_vfull[b], (vp[b] / 3) & 1, budget);
             }
         }
         __syncwarp();
@@ -972,10 +556,9 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         // Phases of mb_sfree: 0 = the first state is in TMEM; k + 1 = slot k's final state is
         // staged.  A first slot that begins a head shared with CTA i + 1 leaves its state in
         // hand-over entry i; a last slot that ends a head shared with CTA i - 1 starts from entry
-        // i - 1, once that entry's flag is set (bounded wait).
+        // i - 1 once that entry's bit is set (bounded wait), and clears the bit.
         if (lane == 0 && n_slots > 0) {
             float* sbuf = reinterpret_cast<float*>(sm + SM_SB);
-            const int me = (int)blockIdx.x;
             int loads = 0, seen = 0;                   // copies into the staging buffer issued / landed
             auto load_rows = [&](const CUtensorMap* map, int row) {
                 mbar_arrive_expect_tx(&mb_st, kD * kD * 4);
@@ -985,14 +568,16 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             };
             auto load_state = [&](int slot) -> bool {
                 int lh, tb, te;
-                sch.slot(slot, n, lh, tb, te);
+                sch.slot(slot, a.n_tiles, lh, tb, te);
                 if (!sch.is_suffix(slot)) { load_rows(&smap, lh * kD); return true; }
-                grid_dep_wait();                       // the factor kernel reset the flags
+                const uint32_t bit = 1u << ((me - 1) & 31);
+                uint32_t* w = bits_state + ((me - 1) >> 5);
                 const uint64_t t0 = global_ns();
-                while (ho_load_acquire(a.ho_flag + me - 1) == 0) {
-                    if (*abort_flag || global_ns() - t0 > kWaitBudgetNs) return false;
+                while ((ld_acquire(w) & bit) == 0) {
+                    if (*abort_flag || global_ns() - t0 > budget) return false;
                     __nanosleep(64);
                 }
+                atomicAnd(w, ~bit);                    // consumed: zero for the next call
                 fence_proxy_async_global();
                 load_rows(&hmap, (me - 1) * kD);
                 return true;
@@ -1001,10 +586,11 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 if (sch.is_suffix(n_slots - 1)) load_rows(&smap, sch.suf_lh * kD);
                 else mbar_arrive(&mb_st);
             };
+            grid_dep_wait();
             bool ok = load_state(0);
             if (!ok) fail(a.status, abort_flag, 42);
             if (ok) {
-                ok = mbar_wait_or_abort(&mb_sfree, 0, kWaitBudgetNs, abort_flag);
+                ok = mbar_wait_or_abort(&mb_sfree, 0, budget, abort_flag);
                 if (!ok) fail(a.status, abort_flag, 40);
             }
             seen = loads;                              // the chain has consumed it
@@ -1017,10 +603,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
             }
             for (int k = 0; ok && k < n_slots; ++k) {
-                if (!mbar_wait_or_abort(&mb_sfree, (k + 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 41); break; }
+                if (!mbar_wait_or_abort(&mb_sfree, (k + 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 41); break; }
                 seen = loads;
                 int lh, tb, te;
-                sch.slot(k, n, lh, tb, te);
+                sch.slot(k, a.n_tiles, lh, tb, te);
                 const bool hand_over = sch.is_prefix(k);
                 const CUtensorMap* dst = hand_over ? &hmap : &smap;
                 const int row = (hand_over ? me : lh) * kD;
@@ -1031,8 +617,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     bulk_wait0();                      // the state is in global memory ...
                     fence_proxy_async_global();
                     __threadfence();
-                    grid_dep_wait();                   // (after the factor kernel's flag reset)
-                    ho_store_release(a.ho_flag + me, 1);   // ... before CTA i + 1 may read it
+                    atomicOr(bits_state + (me >> 5), 1u << (me & 31));   // ... before CTA i + 1 reads it
                 }
                 if (k + 2 <= n_slots) {
                     bulk_wait_read0();                 // slot k's state has left the buffer
@@ -1044,31 +629,235 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
             }
             bulk_wait0();                              // every state store is complete
-            if (loads > seen) mbar_wait(&mb_st, (loads - 1) & 1, kWaitBudgetNs);   // abort: a load in flight
+            if (loads > seen) mbar_wait(&mb_st, (loads - 1) & 1, budget);   // abort: a load in flight
         }
         __syncwarp();
+    } else if (warp >= kProdWarp0) {
+        // =========================================================== producer: operand images of
+        // the sub-tiles of parity G, and the per-sub-tile decay constants
+        const int G = (warp - kProdWarp0) & 1;
+        const bool tm_warp = warp < kProdWarp0 + 2;    // reads TMEM lanes 32 G .. 32 G + 31
+        const int gt = (tm_warp ? 0 : 32) + lane;      // thread of the group, 0..63
+        float* pw = reinterpret_cast<float*>(sm + SM_PW + G * kPwBytes);
+        float* Mm = pw + PW_M;                         // diag(beta) L of the sub-tile, rows of kMS
+        float* Nm = pw + PW_N;                         // (I + diag(beta) L)^-1
+        float* Pm = pw + PW_P;                         // 16 x 16 product of the off-diagonal block
+        float* sBeta0 = pw + PW_BETA;                  // [2][32]
+        float* sDelta0 = pw + PW_DELTA;                // [2][32]
+        float* sUC0 = pw + PW_UC;                      // [2][u, c, -, -]
+        const int bar_id = kBarProd0 + G;
+        TileCursor cc;
+        cc.init(sch, a);
+        // g of tokens lane and 32 + lane of the tile, beta of this group's token lane (partner warp),
+        // loaded one tile ahead of use
+        float pg0 = 0.f, pg1 = 0.f, pb = 0.f;
+        auto load_gb = [&](const TileCursor& c) {
+            const int t0 = c.jt * kTile + lane, t1 = t0 + kC, tg = G ? t1 : t0;
+            const size_t base = (size_t)c.l * a.T;
+            pg0 = t0 < a.T ? a.g[(base + t0) * a.Hv + c.h] : 0.f;
+            pg1 = t1 < a.T ? a.g[(base + t1) * a.Hv + c.h] : 0.f;
+            pb = tg < a.T ? a.beta[(base + tg) * a.Hv + c.h] : 0.f;
+        };
+        if (!tm_warp && NJ > 0) { grid_dep_wait(); load_gb(cc); }
+        float sig = 1.f;
+        int prev_slot = -1;
+        bool failed = false;
+        for (int J = 0; J < NJ; ++J) {
+            const int j = 2 * J + G;
+            float* sBeta = sBeta0 + 32 * (J & 1);
+            float* sDelta = sDelta0 + 32 * (J & 1);
+            float* sUC = sUC0 + 4 * (J & 1);
+            float kk[32];
+            DecayStep dmine;
+            float wn = 0.f;
+            if (!tm_warp) {
+                const float g0 = pg0, g1 = pg1, bt = pb;
+                if (J + 1 < NJ) {                       // the next tile's g, beta
+                    TileCursor nx = cc;
+                    nx.next(sch, a);
+                    load_gb(nx);
+                }
+                if (cc.k != prev_slot) sig = 1.f;       // a slot starts from the true state
+                prev_slot = cc.k;
+                float G0 = g0, G1 = g1;                 // inclusive scans over the two sub-tiles
+#pragma unroll
+                for (int m = 1; m < 32; m <<= 1) {
+                    const float y0 = __shfl_up_sync(0xffffffffu, G0, m);
+                    const float y1 = __shfl_up_sync(0xffffffffu, G1, m);
+                    if (lane >= m) { G0 += y0; G1 += y1; }
+                }
+                const float GC0 = __shfl_sync(0xffffffffu, G0, 31), GC1 = __shfl_sync(0xffffffffu, G1, 31);
+                const DecayStep d0 = decay_step(expf(GC0) * sig);
+                const DecayStep d1 = decay_step(expf(GC1) * d0.sig);
+                sig = d1.sig;
+                dmine = G ? d1 : d0;
+                const float Gm = G ? G1 : G0, GCm = G ? GC1 : GC0;
+                const float delta = expf(GCm - Gm);
+                sBeta[lane] = bt;
+                sDelta[lane] = delta;
+                const float ud = dmine.u * delta;
+                wn = ud >= 0x1p-60f ? 1.f / ud : 0.f;   // column t of E is u delta_t u_t
+                if (lane == 0) { sUC[0] = dmine.u; sUC[1] = dmine.c; }
+            } else {
+                const bool ok = mbar_wait_or_abort(&mb_kk, J & 1, budget, abort_flag);
+                if (!ok) { fail(a.status, abort_flag, 20); failed = true; }
+                tc_fence_after();
+                if (ok) {
+                    tmem_ld32(tm + ((uint32_t)(32 * G) << 16) + TM_KK + 32 * G, kk);
+                    tmem_ld_wait();
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&mb_kkfree);
+            }
+            if (named_sync_or(bar_id, 64, failed || *abort_flag)) break;     // (1)
+            if (tm_warp) {                              // row t of diag(beta) L: beta_t k_t.k_c, c < t
+                const float bt = sBeta[lane];
+                float* row = Mm + lane * kMS;
+#pragma unroll
+                for (int c4 = 0; c4 < 8; ++c4) {
+                    float4 v;
+                    v.x = (4 * c4 + 0 < lane) ? bt * kk[4 * c4 + 0] : 0.f;
+                    v.y = (4 * c4 + 1 < lane) ? bt * kk[4 * c4 + 1] : 0.f;
+                    v.z = (4 * c4 + 2 < lane) ? bt * kk[4 * c4 + 2] : 0.f;
+                    v.w = (4 * c4 + 3 < lane) ? bt * kk[4 * c4 + 3] : 0.f;
+                    *reinterpret_cast<float4*>(row + 4 * c4) = v;
+                }
+            }
+            if (named_sync_or(bar_id, 64, *abort_flag)) break;               // (2)
+            if (tm_warp) {
+                // the two 16 x 16 diagonal blocks of N by forward substitution, one column per lane
+                const int b = lane >> 4, jc = lane & 15, o = 16 * b;
+                float x[16];
+#pragma unroll
+                for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
+#pragma unroll
+                for (int rr = 1; rr < 16; ++rr) {
+                    const float* mr = Mm + (o + rr) * kMS + o;
+                    float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+                    for (int c = 0; c < rr; c += 4) {
+                        const float4 v = *reinterpret_cast<const float4*>(mr + c);
+                        s0 = fmaf(v.x, x[c], s0);
+                        if (c + 1 < rr) s1 = fmaf(v.y, x[c + 1], s1);
+                        if (c + 2 < rr) s0 = fmaf(v.z, x[c + 2], s0);
+                        if (c + 3 < rr) s1 = fmaf(v.w, x[c + 3], s1);
+                    }
+                    if (rr > jc) x[rr] = -(s0 + s1);
+                }
+#pragma unroll
+                for (int rr = 0; rr < 16; ++rr) Nm[(o + rr) * kMS + o + jc] = x[rr];
+                if (b == 0) {
+#pragma unroll
+                    for (int rr = 0; rr < 16; ++rr) Nm[rr * kMS + 16 + jc] = 0.f;   // upper block
+                }
+            }
+            if (named_sync_or(bar_id, 64, *abort_flag)) break;               // (3)
+            {   // P = M10 N00, then N10 = -N11 P (16 x 16 blocks; 4 outputs per thread)
+                const int r = gt >> 2, c0 = 4 * (gt & 3);
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                const float* mrow = Mm + (16 + r) * kMS;
+#pragma unroll
+                for (int a4 = 0; a4 < 16; a4 += 4) {
+                    const float4 mv = *reinterpret_cast<const float4*>(mrow + a4);
+                    const float m4[4] = {mv.x, mv.y, mv.z, mv.w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float4 nv = *reinterpret_cast<const float4*>(Nm + (a4 + e) * kMS + c0);
+                        acc.x = fmaf(m4[e], nv.x, acc.x); acc.y = fmaf(m4[e], nv.y, acc.y);
+                        acc.z = fmaf(m4[e], nv.z, acc.z); acc.w = fmaf(m4[e], nv.w, acc.w);
+                    }
+                }
+                *reinterpret_cast<float4*>(Pm + r * kPS + c0) = acc;
+                if (named_sync_or(bar_id, 64, *abort_flag)) break;           // (4)
+                acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                const float* nrow = Nm + (16 + r) * kMS + 16;
+#pragma unroll
+                for (int a4 = 0; a4 < 16; a4 += 4) {
+                    const float4 nv = *reinterpret_cast<const float4*>(nrow + a4);
+                    const float n4[4] = {nv.x, nv.y, nv.z, nv.w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float4 pv = *reinterpret_cast<const float4*>(Pm + (a4 + e) * kPS + c0);
+                        acc.x = fmaf(n4[e], pv.x, acc.x); acc.y = fmaf(n4[e], pv.y, acc.y);
+                        acc.z = fmaf(n4[e], pv.z, acc.z); acc.w = fmaf(n4[e], pv.w, acc.w);
+                    }
+                }
+                *reinterpret_cast<float4*>(Nm + (16 + r) * kMS + c0) = make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
+            }
+            if (named_sync_or(bar_id, 64, *abort_flag)) break;               // (5)
+            // the image slot is free once sub-tile j - 4's products and the chain have read it
+            if (j >= 4) {
+                const bool ok = mbar_wait_or_abort(&mb_iempty[j & 3], ((j >> 2) - 1) & 1, budget, abort_flag);
+                if (!ok) { fail(a.status, abort_flag, 21); failed = true; }
+            }
+            if (named_sync_or(bar_id, 64, failed || *abort_flag)) break;     // (6)
+            {   // images: row t = gt / 2, columns 16 hc .. 16 hc + 15 of N_beta = N diag(beta)
+                const int t = gt >> 1, hc = gt & 1;
+                const float u = sUC[0], cX = sUC[1];
+                uint8_t* slot = sm + SM_IMG + (j & 3) * kImgSlot;
+                float nb[16], w1[16];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float4 nv = *reinterpret_cast<const float4*>(Nm + t * kMS + 16 * hc + 4 * e);
+                    const float4 bv = *reinterpret_cast<const float4*>(sBeta + 16 * hc + 4 * e);
+                    const float4 dv = *reinterpret_cast<const float4*>(sDelta + 16 * hc + 4 * e);
+                    nb[4 * e] = nv.x * bv.x; nb[4 * e + 1] = nv.y * bv.y;
+                    nb[4 * e + 2] = nv.z * bv.z; nb[4 * e + 3] = nv.w * bv.w;
+                    w1[4 * e] = u * nb[4 * e] * dv.x; w1[4 * e + 1] = u * nb[4 * e + 1] * dv.y;
+                    w1[4 * e + 2] = u * nb[4 * e + 2] * dv.z; w1[4 * e + 3] = u * nb[4 * e + 3] * dv.w;
+                }
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {          // B2 = -c N_beta, tf32, row t chunks 4 hc + e
+                    const uint4 w = make_uint4(to_tf32(-cX * nb[4 * e]), to_tf32(-cX * nb[4 * e + 1]),
+                                               to_tf32(-cX * nb[4 * e + 2]), to_tf32(-cX * nb[4 * e + 3]));
+                    *reinterpret_cast<uint4*>(slot + 8192 + sw128_offset(t, 4 * hc + e)) = w;
+                }
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {          // B1 = u N_beta diag(delta), (hi, lo)
+                    uint32_t h[4], l[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) split2(w1[8 * e + 2 * i], w1[8 * e + 2 * i + 1], h[i], l[i]);
+                    *reinterpret_cast<uint4*>(slot + sw128_offset(t, 2 * hc + e)) = make_uint4(h[0], h[1], h[2], h[3]);
+                    *reinterpret_cast<uint4*>(slot + 4096 + sw128_offset(t, 2 * hc + e)) = make_uint4(l[0], l[1], l[2], l[3]);
+                }
+            }
+            if (!tm_warp) {                             // the chain's and the MMA's constants
+                float* cs = const_cast<float*>(cst) + (j & 3) * kConstWords;
+                cs[lane] = wn;
+                if (lane == 0) {
+                    cs[32] = dmine.sig;
+                    cs[33] = dmine.pass;
+                    reinterpret_cast<int*>(cs)[34] = dmine.shift;
+                }
+            }
+            fence_async_smem();                         // generic writes -> the tensor core's reads
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&mb_ifull[j & 3]);
+            cc.next(sch, a);
+        }
     } else {
-        // =========================================================== state chain (warps 0-15)
-        const int q = warp & 3, cgp = warp >> 2;         // TMEM lane quadrant, column group
+        // =========================================================== state chain (warps 0-7)
+        const int q = warp & 3, hh = warp >> 2;          // TMEM lane quadrant, column half
         const int r = 32 * q + lane;                     // row of S (value index)
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
         float* sbuf = reinterpret_cast<float*>(sm + SM_SB);   // swizzled rows, see sb_idx
         int st_seen = 0;                                 // mb_st phases waited for (uniform)
-        TileCursor cc;                                   // the chain's tile
+        TileCursor cc;
         cc.init(sch, a);
-        const int me = (int)blockIdx.x;
-        // K(jj) (TMA tile, buffer jj % 3) in fp32 (exact, and exact in tf32) into the B operand
-        // buffer of X.  Called between MMA_X(jj-1), the last reader of the buffer, and the ready
-        // signal of tile jj.
+        // K of sub-tile jj (TMA tile, rows 32 (jj & 1) ..) in fp32 (exact, and exact in tf32) into
+        // the B operand buffer of X.  Called between MMA_X(jj-1), the last reader of the buffer, and
+        // the ready signal of sub-tile jj.
         auto make_k32 = [&](int jj) -> bool {
-            const bool ok = mbar_wait_or_abort(&mb_tk[jj % 3], (jj / 3) & 1, kWaitBudgetNs, abort_flag);
-            const uint8_t* kb = sm + SM_K + (jj % 3) * 16384;
-            uint8_t* k32 = sm + SM_K32;
+            const int bk = (jj >> 1) % 3;
+            const bool ok = mbar_wait_or_abort(&mb_kfull[bk], ((jj >> 1) / 3) & 1, budget, abort_flag);
+            const uint8_t* kb = sm + SM_K + bk * 16384;
+            const int r0 = 32 * (jj & 1);
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {                  // 64 rows x 16 chunks of 8 bf16
+            for (int u = 0; u < 2; ++u) {                  // 32 rows x 16 chunks of 8 bf16
                 const int e = tid + kChain * u;
                 const int t = e >> 4, c16 = e & 15, cb = c16 >> 3, c = c16 & 7;
-                const uint4 w = *reinterpret_cast<const uint4*>(kb + cb * 8192 + sw128_offset(t, c));
+                const uint4 w = *reinterpret_cast<const uint4*>(kb + cb * 8192 + sw128_offset(r0 + t, c));
                 const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
                 uint32_t f[8];
 #pragma unroll
@@ -1077,7 +866,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     f[2 * i + 1] = wv[i] & 0xFFFF0000u;
                 }
                 // dims 64 cb + 8 c .. + 7: fp32 block 2 cb + c / 4, chunks 2 (c % 4) and 2 (c % 4) + 1
-                uint8_t* rowp = k32 + (2 * cb + (c >> 2)) * 8192;
+                uint8_t* rowp = sm + SM_K32 + (2 * cb + (c >> 2)) * 4096;
                 const int q0 = 2 * (c & 3);
                 *reinterpret_cast<uint4*>(rowp + sw128_offset(t, q0)) = make_uint4(f[0], f[1], f[2], f[3]);
                 *reinterpret_cast<uint4*>(rowp + sw128_offset(t, q0 + 1)) = make_uint4(f[4], f[5], f[6], f[7]);
@@ -1085,22 +874,14 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             fence_async_smem();                            // generic writes -> the tensor core's reads
             return ok;
         };
-        auto rec_consts = [&](int jj) {                    // -gamma[64], gamma_C of tile jj's record
-            return reinterpret_cast<const float*>(sm + SM_R + (jj & 1) * kRecSlot + kRecT);
-        };
-        float den = 0.f;
-        // Deferred decay: TMEM holds S~ with the head's state S = sig * S~.  A tile folds its decay
-        // gamma_C into sig (the W pass applies sig and u_scale = 1 / (gamma_C sig), so MMA_S
-        // accumulates onto S~ with no pass over the state); when sig gamma_C would drop below
-        // kSigMin the tile instead writes gamma_C S back into TMEM and sig restarts at 1.
-        float sig = 1.f;
-        // Write sizes (optional): column t of the U region is u_t scaled by u_scale gamma_C /
-        // gamma_t, u_t = beta_t (v_t - alpha_t S_{t-1} k_t) the token's write.  The Ũ pass sums
-        // each column's squares over this warp's 32 rows and adds them, rescaled to u_t, into
-        // s_u2 (four warps per column); after the next barrier warp 0 takes the square roots and
-        // sums them over the tile's tokens into the head's total.
+        float den = 0.f, sig = 1.f;
+        // Write sizes (optional): column t of E is u delta_t u_t, u_t = beta_t (v_t - alpha_t S_{t-1}
+        // k_t) the token's write.  The pass sums each column's squares over the warp's 32 rows,
+        // rescales them by the constant (1 / (u delta_t))^2 and adds them into s_u2 (four warps per
+        // column); at the next sub-tile warp 0 takes the square roots and sums them into the head's
+        // total.
         const bool want_w = a.wnorm != nullptr;
-        float wacc = 0.f;                                  // warp 0: the head's running sum
+        float wacc = 0.f;                                  // warp 0: the slot's running sum
         int prev_lh = -1, prev_slot = -1;
         bool prev_last = false;
         // a head's write-size sum: to hand-over entry i when the slot begins a head shared with
@@ -1110,258 +891,243 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             if (sch.is_prefix(slot)) {
                 a.ho_wsum[me] = sum;
                 __threadfence();
-                grid_dep_wait();                           // (after the factor kernel's flag reset)
-                ho_store_release(a.ho_wflag + me, 1);
+                atomicOr(bits_wsum + (me >> 5), 1u << (me & 31));
                 return true;
             }
             if (sch.is_suffix(slot)) {
+                const uint32_t bit = 1u << ((me - 1) & 31);
+                uint32_t* w = bits_wsum + ((me - 1) >> 5);
                 const uint64_t t0 = global_ns();
-                while (ho_load_acquire(a.ho_wflag + me - 1) == 0) {
-                    if (*abort_flag || global_ns() - t0 > kWaitBudgetNs) return false;
+                while ((ld_acquire(w) & bit) == 0) {
+                    if (*abort_flag || global_ns() - t0 > budget) return false;
                     __nanosleep(64);
                 }
                 sum += *reinterpret_cast<volatile const float*>(a.ho_wsum + me - 1);
+                atomicAnd(w, ~bit);
             }
             a.wnorm[lh] = sum;
             return true;
         };
-        auto fold_writes = [&](int jj) {                   // warp 0: tile jj's sizes into wacc
+        auto fold_writes = [&](int jj) {                   // warp 0: sub-tile jj's sizes into wacc
             float* b = s_u2[jj & 1];
-            float sacc = sqrtf(b[lane]) + sqrtf(b[lane + 32]);
+            float sacc = sqrtf(b[lane]);
             b[lane] = 0.f;
-            b[lane + 32] = 0.f;
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, m);
             wacc += sacc;
         };
-        for (int j = 0; j < NJ; ++j) {                     // j: global tile index
-            const int lh = cc.lh, jt = cc.jt, slot = cc.k; // head, tile within the head, slot
-            const bool last = jt == cc.te - 1;             // the slot's last tile
-            if (named_sync_or(2, kChain, *abort_flag)) break;
-            if (!mbar_wait_or_abort(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
-            const float gC = rec_consts(j)[64];
-            float w_gamma = 0.f;                           // gamma_t of this lane's column in the Ũ pass
-            if (want_w) {
-                w_gamma = -rec_consts(j)[16 * cgp + (lane >> 1)];
-                if (j > 0 && warp == 0) {
+        bool stop = false;
+        for (int J = 0; J < NJ && !stop; ++J) {
+            for (int u = 0; u < 2; ++u) {
+                const int j = 2 * J + u;
+                const int lh = cc.lh, slot = cc.k;
+                const bool last = u == 1 && cc.jt == cc.te - 1;   // the slot's last sub-tile
+                if (named_sync_or(kBarChain, kChain, *abort_flag)) { stop = true; break; }
+                if (want_w && j > 0 && warp == 0) {
                     fold_writes(j - 1);
                     if (prev_last) {
                         if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 44);
                         wacc = 0.f;
                     }
                 }
-            }
-
-            if (j == 0) {
-                // ---- the CTA's first head: its state from the staging buffer into TMEM, as S~
-                // (sig = 1) and as S_before, and sum S_before^2
-                if (!mbar_wait_or_abort(&mb_st, 0, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 14);
-                st_seen = 1;
-                float sv[32];
+                if (j == 0) {
+                    // ---- the CTA's first slot: its state from the staging buffer into TMEM, as S~
+                    // (sig = 1) and as S_before, and sum S_before^2
+                    if (!mbar_wait_or_abort(&mb_st, 0, budget, abort_flag)) fail(a.status, abort_flag, 14);
+                    st_seen = 1;
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, 8 * cgp + e));
-                    sv[4 * e] = x.x; sv[4 * e + 1] = x.y; sv[4 * e + 2] = x.z; sv[4 * e + 3] = x.w;
+                    for (int g4 = 0; g4 < 4; ++g4) {
+                        uint32_t sv[16];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, 16 * hh + 4 * g4 + e));
+                            den = fmaf(x.x, x.x, den); den = fmaf(x.y, x.y, den);
+                            den = fmaf(x.z, x.z, den); den = fmaf(x.w, x.w, den);
+                            sv[4 * e] = __float_as_uint(x.x); sv[4 * e + 1] = __float_as_uint(x.y);
+                            sv[4 * e + 2] = __float_as_uint(x.z); sv[4 * e + 3] = __float_as_uint(x.w);
+                        }
+                        tmem_st16(tm + lane_off + TM_S + 64 * hh + 16 * g4, sv);
+                        tmem_st16(tm + lane_off + TM_SB + 64 * hh + 16 * g4, sv);
+                    }
+                    warp_arrive(&mb_sfree, lane);                    // the staging buffer has been read
+                    if (!make_k32(0)) fail(a.status, abort_flag, 16);
+                    tmem_st_wait();
+                    tc_fence_before();
+                    warp_arrive(&mb_sready, lane);
                 }
-#pragma unroll
-                for (int e = 0; e < 32; ++e) den = fmaf(sv[e], sv[e], den);
-                warp_arrive(&mb_sfree, lane);                    // the staging buffer has been read
-                tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
-                tmem_st32(tm + lane_off + TM_SB + 32 * cgp, sv);
-                if (!make_k32(0)) fail(a.status, abort_flag, 16);
-                tmem_st_wait();
-                tc_fence_before();
-                warp_arrive(&mb_sready, lane);
-            }
-            const bool rescale = sig * gC < kSigMin;       // uniform over the CTA
-            const float u_scale = rescale ? 1.f : 1.f / (gC * sig);
-
-            // ---- W pass: W^T = V^T - sig X~^T diag(gamma) from the V and X regions (X~ = S~ K^T),
-            // scaled by u_scale, (hi, lo) in place over this thread's 16 X columns (tokens 16 cgp ..)
-            if (!mbar_wait_or_abort(&mb_x, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 10);
-            tc_fence_after();
-            {
-                float xv[16], vv[16], cf[16];
-                tmem_ld16(tm + lane_off + TM_X + 16 * cgp, xv);
-                tmem_ld16(tm + lane_off + TM_V + 16 * cgp, vv);
-                const float* gm = rec_consts(j) + 16 * cgp;         // -gamma of the thread's tokens
+                // ---- E(j) is complete (and MMA_X(j) has read the state and K in fp32)
+                if (!mbar_wait_or_abort(&mb_u, j & 1, budget, abort_flag)) fail(a.status, abort_flag, 10);
+                if (!mbar_wait_or_abort(&mb_ifull[j & 3], (j >> 2) & 1, budget, abort_flag)) fail(a.status, abort_flag, 11);
+                tc_fence_after();
+                const float* cs = cst + (j & 3) * kConstWords;
+                const float pass_f = cs[33];
+                const float sig_after = cs[32];
+                float wf[16];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    const float4 g4 = *reinterpret_cast<const float4*>(gm + 4 * e);
-                    cf[4 * e] = g4.x * sig; cf[4 * e + 1] = g4.y * sig; cf[4 * e + 2] = g4.z * sig; cf[4 * e + 3] = g4.w * sig;
+                    const float4 w4 = *reinterpret_cast<const float4*>(cs + 16 * hh + 4 * e);
+                    wf[4 * e] = w4.x; wf[4 * e + 1] = w4.y; wf[4 * e + 2] = w4.z; wf[4 * e + 3] = w4.w;
                 }
-                tmem_ld_wait();
-                uint32_t hi[8], lo[8];
+                if (pass_f >= 0.f) {
+                    // the decay would take the deferred scale out of range: S~ <- p S~ (MMA_S(j) has not
+                    // been issued: it waits for this pass)
 #pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    split2(fmaf(cf[2 * i], xv[2 * i], vv[2 * i]) * u_scale,
-                           fmaf(cf[2 * i + 1], xv[2 * i + 1], vv[2 * i + 1]) * u_scale, hi[i], lo[i]);
-                tmem_st8(tm + lane_off + TM_X + 16 * cgp, hi);
-                tmem_st8(tm + lane_off + TM_X + 16 * cgp + 8, lo);
-                tmem_st_wait();
-            }
-            tc_fence_before();
-            warp_arrive(&mb_xready, lane);
-
-            // ---- while MMA_U runs: rescale S~ if the decay would underflow the deferred scale
-            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K(j+1) in fp32
-            if (rescale) {
-                const float f = gC * sig;
-                float sv[32];
-                tmem_ld32(tm + lane_off + TM_S + 32 * cgp, sv);
-                tmem_ld_wait();
-#pragma unroll
-                for (int e = 0; e < 32; ++e) sv[e] *= f;
-                tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
-                tmem_st_wait();
-            }
-            sig = rescale ? 1.f : gC * sig;                // the deferred decay after tile j
-            if (j + 1 < NJ && !make_k32(j + 1)) fail(a.status, abort_flag, 16);
-
-            // ---- U~ pass: (hi, lo) in place over this thread's 16 U columns
-            if (!mbar_wait_or_abort(&mb_u, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 11);
-            tc_fence_after();
-            {
-                float uv[16];
-                tmem_ld16(tm + lane_off + TM_U + 16 * cgp, uv);
-                tmem_ld_wait();
-                if (want_w) {
-                    // squares summed over the warp's 32 rows, column by column: halving exchanges
-                    // leave lanes 2c and 2c + 1 with column c (token 16 cgp + c) of the 16
-                    float x[16];
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) x[i] = uv[i] * uv[i];
-#pragma unroll
-                    for (int w = 8, bit = 16; w >= 1; w >>= 1, bit >>= 1) {
-                        const bool up = (lane & bit) != 0;
-#pragma unroll
-                        for (int i = 0; i < w; ++i) {
-                            const float send = up ? x[i] : x[i + w];
-                            x[i] = (up ? x[i + w] : x[i]) + __shfl_xor_sync(0xffffffffu, send, bit);
-                        }
-                    }
-                    x[0] += __shfl_xor_sync(0xffffffffu, x[0], 1);
-                    // U column -> u_t.  u_scale gamma_C is 1 / sig >= 1 unless the tile restarts
-                    // the deferred decay; then it is gamma_C, and below 2^-60 the columns of the
-                    // early tokens, scaled by gamma_C / gamma_t, are no longer representable: such
-                    // a tile contributes nothing
-                    const float sc = u_scale * gC;
-                    const float wf = sc >= 0x1p-60f ? w_gamma / sc : 0.f;
-                    if ((lane & 1) == 0) atomicAdd(&s_u2[j & 1][16 * cgp + (lane >> 1)], x[0] * wf * wf);
-                }
-                uint32_t hi[8], lo[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) split2(uv[2 * i], uv[2 * i + 1], hi[i], lo[i]);
-                tmem_st8(tm + lane_off + TM_U + 16 * cgp, hi);
-                tmem_st8(tm + lane_off + TM_U + 16 * cgp + 8, lo);
-                tmem_st_wait();
-            }
-            tc_fence_before();
-            warp_arrive(&mb_uready, lane);
-            if (!last) {
-                // the next tile of this head may start X as soon as MMA_S(j) is queued
-                warp_arrive(&mb_sready, lane);
-            } else {
-                // ---- head boundary: S_after = sig S~ out through the staging buffer, the next
-                // head's state (staged meanwhile) into TMEM, drift partials against S_before
-                const bool has_next = j + 1 < NJ;          // uniform
-                // a last slot that ends a head begun by CTA i - 1: S_before is not in TMEM (the
-                // slot started from the handed-over state) but staged, and its square sum is taken
-                // here
-                const bool shared_end = sch.is_suffix(slot);
-                float den_end = 0.f;
-                bool ok = mbar_wait_or_abort(&mb_s, j & 1, kWaitBudgetNs, abort_flag);
-                if (!ok) fail(a.status, abort_flag, 12);
-                if (!mbar_wait_or_abort(&mb_st, st_seen & 1, kWaitBudgetNs, abort_flag)) {
-                    fail(a.status, abort_flag, 14);
-                    ok = false;
-                }
-                ++st_seen;
-                tc_fence_after();
-                float num = 0.f, den_next = 0.f;
-                if (ok) {
-#pragma unroll
-                    for (int half = 0; half < 2; ++half) {
-                        const uint32_t col = 32 * cgp + 16 * half;
-                        const int ch = 8 * cgp + 4 * half;     // this half's 16-byte chunks of row r
-                        float sa[16], sb[16];
-                        tmem_ld16(tm + lane_off + TM_S + col, sa);
-                        if (shared_end) {
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
-                                sb[4 * e] = x.x; sb[4 * e + 1] = x.y; sb[4 * e + 2] = x.z; sb[4 * e + 3] = x.w;
-                            }
-#pragma unroll
-                            for (int e = 0; e < 16; ++e) den_end = fmaf(sb[e], sb[e], den_end);
-                        } else {
-                            tmem_ld16(tm + lane_off + TM_SB + col, sb);
-                        }
+                    for (int g2 = 0; g2 < 2; ++g2) {
+                        float sv[32];
+                        tmem_ld32(tm + lane_off + TM_S + 64 * hh + 32 * g2, sv);
                         tmem_ld_wait();
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            sa[e] *= sig;
-                            const float d = sa[e] - sb[e];
-                            num = fmaf(d, d, num);
-                        }
-                        if (has_next) {
-                            uint32_t sn[16];
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
-                                den_next = fmaf(x.x, x.x, den_next); den_next = fmaf(x.y, x.y, den_next);
-                                den_next = fmaf(x.z, x.z, den_next); den_next = fmaf(x.w, x.w, den_next);
-                                sn[4 * e] = __float_as_uint(x.x); sn[4 * e + 1] = __float_as_uint(x.y);
-                                sn[4 * e + 2] = __float_as_uint(x.z); sn[4 * e + 3] = __float_as_uint(x.w);
-                            }
-                            tmem_st16(tm + lane_off + TM_S + col, sn);
-                            tmem_st16(tm + lane_off + TM_SB + col, sn);
-                        }
-#pragma unroll
-                        for (int e = 0; e < 4; ++e)
-                            *reinterpret_cast<float4*>(sbuf + sb_idx(r, ch + e)) =
-                                make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
+                        for (int e = 0; e < 32; ++e) sv[e] *= pass_f;
+                        tmem_st32(tm + lane_off + TM_S + 64 * hh + 32 * g2, sv);
                     }
+                }
+                {   // ---- pass: E = hi-half product + lo-half product (+ the X term), over this
+                    // thread's 16 token columns, split into the packed (hi, lo) A operand of MMA_S
+                    const uint32_t eb = tm + lane_off + TM_E + (j & 1) * 64 + 16 * hh;
+                    float e0[16], e1[16];
+                    tmem_ld16(eb, e0);
+                    tmem_ld16(eb + 32, e1);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) e0[i] += e1[i];
+                    if (want_w) {
+                        // squares summed over the warp's 32 rows, column by column: halving exchanges
+                        // leave lanes 2c and 2c + 1 with column c of the 16
+                        float x[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) x[i] = e0[i] * e0[i];
+#pragma unroll
+                        for (int w = 8, bit = 16; w >= 1; w >>= 1, bit >>= 1) {
+                            const bool up = (lane & bit) != 0;
+#pragma unroll
+                            for (int i = 0; i < w; ++i) {
+                                const float send = up ? x[i] : x[i + w];
+                                x[i] = (up ? x[i + w] : x[i]) + __shfl_xor_sync(0xffffffffu, send, bit);
+                            }
+                        }
+                        x[0] += __shfl_xor_sync(0xffffffffu, x[0], 1);
+                        const int c = lane >> 1;
+                        float f = wf[0];
+#pragma unroll
+                        for (int i = 1; i < 16; ++i) f = (c == i) ? wf[i] : f;
+                        if ((lane & 1) == 0) atomicAdd(&s_u2[j & 1][16 * hh + c], x[0] * f * f);
+                    }
+                    uint32_t hi[8], lo[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) split2(e0[2 * i], e0[2 * i + 1], hi[i], lo[i]);
+                    tmem_st8(tm + lane_off + TM_AP + 8 * hh, hi);
+                    tmem_st8(tm + lane_off + TM_AP + 16 + 8 * hh, lo);
                     tmem_st_wait();
                 }
                 tc_fence_before();
-                fence_async_smem();                        // S_after -> the state warp's TMA store
-                warp_arrive(&mb_sfree, lane);
-                if (has_next) warp_arrive(&mb_sready, lane);     // the next head's state is in TMEM
-                // partial sums: pairwise in fp32, over the warp's lanes and then over the 16 warps
-                // (the FP64 pipe is far too slow for this path)
-                float fn = num, fd = shared_end ? den_end : den;
-#pragma unroll
-                for (int m = 16; m >= 1; m >>= 1) {
-                    fn += __shfl_xor_sync(0xffffffffu, fn, m);
-                    fd += __shfl_xor_sync(0xffffffffu, fd, m);
-                }
-                if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
-                if (named_sync_or(2, kChain, !ok)) break;
-                if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot)) {   // a shared head's drift: at its end
-                    float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
-                    float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
-#pragma unroll
-                    for (int m = kChainWarps / 2; m >= 1; m >>= 1) {
-                        pn += __shfl_xor_sync(0xffffffffu, pn, m);
-                        pd += __shfl_xor_sync(0xffffffffu, pd, m);
+                warp_arrive(&mb_uready, lane);
+                warp_arrive(&mb_iempty[j & 3], lane);            // images and constants read
+                sig = sig_after;
+                // ---- while MMA_S(j) runs: the next sub-tile's K in fp32
+                if (j + 1 < NS && !make_k32(j + 1)) fail(a.status, abort_flag, 16);
+                if (!last) {
+                    if (j + 1 < NS) warp_arrive(&mb_sready, lane);
+                } else {
+                    // ---- slot boundary: S_after = sig S~ out through the staging buffer, the next
+                    // slot's state (staged meanwhile) into TMEM, drift partials against S_before
+                    const bool has_next = j + 1 < NS;             // uniform
+                    // a last slot that ends a head begun by CTA i - 1: S_before is not in TMEM (the
+                    // slot started from the handed-over state) but staged, and its square sum is
+                    // taken here
+                    const bool shared_end = sch.is_suffix(slot);
+                    float den_end = 0.f;
+                    bool ok = mbar_wait_or_abort(&mb_s, j & 1, budget, abort_flag);
+                    if (!ok) fail(a.status, abort_flag, 12);
+                    if (!mbar_wait_or_abort(&mb_st, st_seen & 1, budget, abort_flag)) {
+                        fail(a.status, abort_flag, 14);
+                        ok = false;
                     }
-                    if (lane == 0) {
-                        a.partials[(size_t)lh * 2 + 0] = pn;
-                        a.partials[(size_t)lh * 2 + 1] = pd;
+                    ++st_seen;
+                    tc_fence_after();
+                    float num = 0.f, den_next = 0.f;
+                    if (ok) {
+#pragma unroll 1
+                        for (int g4 = 0; g4 < 4; ++g4) {
+                            const uint32_t col = 64 * hh + 16 * g4;
+                            const int ch = 16 * hh + 4 * g4;      // this group's 16-byte chunks of row r
+                            float sa[16], sb[16];
+                            tmem_ld16(tm + lane_off + TM_S + col, sa);
+                            if (shared_end) {
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) {
+                                    const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
+                                    sb[4 * e] = x.x; sb[4 * e + 1] = x.y; sb[4 * e + 2] = x.z; sb[4 * e + 3] = x.w;
+                                }
+#pragma unroll
+                                for (int e = 0; e < 16; ++e) den_end = fmaf(sb[e], sb[e], den_end);
+                            } else {
+                                tmem_ld16(tm + lane_off + TM_SB + col, sb);
+                            }
+                            tmem_ld_wait();
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                sa[e] *= sig;
+                                const float d = sa[e] - sb[e];
+                                num = fmaf(d, d, num);
+                            }
+                            if (has_next) {
+                                uint32_t sn[16];
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) {
+                                    const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
+                                    den_next = fmaf(x.x, x.x, den_next); den_next = fmaf(x.y, x.y, den_next);
+                                    den_next = fmaf(x.z, x.z, den_next); den_next = fmaf(x.w, x.w, den_next);
+                                    sn[4 * e] = __float_as_uint(x.x); sn[4 * e + 1] = __float_as_uint(x.y);
+                                    sn[4 * e + 2] = __float_as_uint(x.z); sn[4 * e + 3] = __float_as_uint(x.w);
+                                }
+                                tmem_st16(tm + lane_off + TM_S + col, sn);
+                                tmem_st16(tm + lane_off + TM_SB + col, sn);
+                            }
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                *reinterpret_cast<float4*>(sbuf + sb_idx(r, ch + e)) =
+                                    make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
+                        }
+                        tmem_st_wait();
                     }
+                    tc_fence_before();
+                    fence_async_smem();                          // S_after -> the state warp's TMA store
+                    warp_arrive(&mb_sfree, lane);
+                    if (has_next) warp_arrive(&mb_sready, lane);  // the next slot's state is in TMEM
+                    // partial sums: pairwise in fp32, over the warp's lanes and then over the warps
+                    float fn = num, fd = shared_end ? den_end : den;
+#pragma unroll
+                    for (int m = 16; m >= 1; m >>= 1) {
+                        fn += __shfl_xor_sync(0xffffffffu, fn, m);
+                        fd += __shfl_xor_sync(0xffffffffu, fd, m);
+                    }
+                    if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
+                    if (named_sync_or(kBarChain, kChain, !ok)) { stop = true; break; }
+                    if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot)) {   // a shared head: at its end
+                        float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
+                        float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
+#pragma unroll
+                        for (int m = kChainWarps / 2; m >= 1; m >>= 1) {
+                            pn += __shfl_xor_sync(0xffffffffu, pn, m);
+                            pd += __shfl_xor_sync(0xffffffffu, pd, m);
+                        }
+                        if (lane == 0) {
+                            a.partials[(size_t)lh * 2 + 0] = pn;
+                            a.partials[(size_t)lh * 2 + 1] = pd;
+                        }
+                    }
+                    den = den_next;
+                    sig = 1.f;
                 }
-                den = den_next;
-                sig = 1.f;
+                prev_lh = lh;
+                prev_slot = slot;
+                prev_last = last;
             }
-            prev_lh = lh;
-            prev_slot = slot;
-            prev_last = last;
             cc.next(sch, a);
         }
-        // the CTA's last tile (always a head's last) once every warp's Ũ pass has added to it
-        if (want_w && NJ > 0 && !named_sync_or(2, kChain, *abort_flag) && warp == 0) {
-            fold_writes(NJ - 1);
+        // the CTA's last sub-tile (always a slot's last) once every warp's pass has added to it
+        if (want_w && NS > 0 && !named_sync_or(kBarChain, kChain, *abort_flag) && warp == 0) {
+            fold_writes(NS - 1);
             if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 45);
         }
     }
@@ -1379,27 +1145,25 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = nullptr;
-    static bool tried = false;
-    if (!tried) {
-        tried = true;
+    static EncodeTiledFn fn = []() -> EncodeTiledFn {
         cudaDriverEntryPointQueryResult q;
         void* p = nullptr;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(p);
-    }
+            return reinterpret_cast<EncodeTiledFn>(p);
+        return nullptr;
+    }();
     return fn;
 }
 
-// [L][T][H][128] bfloat16 as a 4-D map (d, H, T, L): a box of 64 features x 1 head x 64 tokens,
+// [L][T][H][128] bfloat16 as a 4-D map (d, H, T, L): a box of 64 features x 1 head x `rows` tokens,
 // 128-byte swizzle; tokens past T read as zero.
-bool make_map(CUtensorMap* map, const void* base, int L, int T, int H) {
+bool make_map(CUtensorMap* map, const void* base, int L, int T, int H, int rows) {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return false;
     cuuint64_t dims[4] = {(cuuint64_t)kD, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)L};
     cuuint64_t strides[3] = {(cuuint64_t)kD * 2, (cuuint64_t)H * kD * 2, (cuuint64_t)T * H * kD * 2};
-    cuuint32_t box[4] = {64, 1, (cuuint32_t)kC, 1};
+    cuuint32_t box[4] = {64, 1, (cuuint32_t)rows, 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -1420,92 +1184,94 @@ bool make_state_map(CUtensorMap* map, void* base, int heads) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Scratch: the WY records, then the update kernel's hand-over area for up to one CTA per SM:
-// states [grid][128][128] fp32 (1024-aligned), flags [2][grid] int32, write-size sums [grid].
+// Scratch (past the workspace header): the hand-over area for up to one CTA per SM: states
+// [grid][128][128] fp32, write-size sums [grid].
 struct TcScratch {
-    size_t rec, ho_state, ho_flags, ho_wsum, total;
+    size_t ho_state, ho_wsum, total;
 };
 
-TcScratch tc_scratch_layout(int L, int Hv, int T) {
+TcScratch tc_scratch_layout(int L, int Hv) {
     const int grid = std::max(1, std::min(L * Hv, device_sm_count()));
     TcScratch l;
-    l.rec = 0;
-    l.ho_state = ((size_t)L * Hv * ((T + kC - 1) / kC) * kRecBytes + 1023) & ~size_t(1023);
-    l.ho_flags = l.ho_state + (size_t)grid * kD * kD * 4;
-    l.ho_wsum = l.ho_flags + 2 * (size_t)grid * 4;
+    l.ho_state = 0;
+    l.ho_wsum = (size_t)grid * kD * kD * 4;
     l.total = l.ho_wsum + (size_t)grid * 4;
     return l;
 }
+
+// Equal tile runs, with heads split between neighbouring CTAs, when they shorten the slowest CTA:
+// a slot boundary costs about `kBoundary` tiles and a hand-over about `kHandOver`.
+constexpr double kBoundary = 0.6, kHandOver = 2.0;
 
 }  // namespace
 
 size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T) {
     if (dk != kD || dv != kD || dtype != DELTAS_BF16 || L <= 0 || Hv <= 0 || T <= 0) return 0;
-    return tc_scratch_layout(L, Hv, T).total;
+    return tc_scratch_layout(L, Hv).total;
+}
+
+bool gdn_tc_shape(const GdnArgs& a) {
+    return a.dk == kD && a.dv == kD && a.dtype == DELTAS_BF16 && a.out == nullptr && a.T > 0;
 }
 
 bool gdn_tc_supported(const GdnArgs& a) {
-    return a.dk == kD && a.dv == kD && a.dtype == DELTAS_BF16 && a.out == nullptr && a.T > 0 &&
+    return gdn_tc_shape(a) &&
            (long long)a.L * a.Hv * kD < (1ll << 31) &&                          // TMA row coordinate
-           (long long)a.L * a.Hv * ((a.T + kC - 1) / kC) < (1ll << 31) &&       // factor-kernel items
+           a.Hk <= (1 << 24) && a.T < (1 << 30) &&
            a.scratch != nullptr &&
            a.scratch_bytes >= gdn_tc_scratch_bytes(a.L, a.Hv, a.dk, a.dv, a.dtype, a.T) &&
+           std::min(a.L * a.Hv, device_sm_count()) <= 512 &&                    // hand-over bits
            encode_fn() != nullptr;
 }
 
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
-    const TcScratch sl = tc_scratch_layout(a.L, a.Hv, a.T);
-    const int grid = std::min(a.L * a.Hv, device_sm_count());
-    CUtensorMap kmap, vmap, smap, hmap;
-    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
-        !make_state_map(&smap, a.state, a.L * a.Hv) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
-        return cudaErrorInvalidValue;
-    static int configured_device = -1;
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (configured_device != dev) {
-        cudaError_t e = cudaFuncSetAttribute(gdn_update_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)kSmemAlloc);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(gdn_wy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kWySmemAlloc);
-        if (e != cudaSuccess) return e;
-        configured_device = dev;
-    }
-    const int n_tiles = (a.T + kC - 1) / kC;
+    const TcScratch sl = tc_scratch_layout(a.L, a.Hv);
     const int sms = device_sm_count();
-    // factor kernel: one record per (layer, value head, tile), kWyCtasPerSm persistent CTAs per SM
-    WyArgs w;
-    w.L = a.L; w.Hk = a.Hk; w.Hv = a.Hv; w.T = a.T; w.n_tiles = n_tiles;
-    w.g = a.g; w.beta = a.beta; w.rec = a.scratch; w.status = a.status;
-    w.ho_flags = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
-    w.n_ho_flags = 2 * grid;
-    const long long items = (long long)a.L * a.Hv * n_tiles;
-    const int wgrid = (int)std::min<long long>(items, (long long)sms * kWyCtasPerSm);
-    gdn_wy_kernel<<<wgrid, kWyThreads, kWySmemAlloc, s>>>(kmap, w);
-    cudaError_t e = cudaGetLastError();
+    const int H = a.L * a.Hv;
+    const int grid = std::min(H, sms);
+    CUtensorMap kmap, vmap, smap, hmap;
+    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk, kTile) || !make_map(&vmap, a.v, a.L, a.T, a.Hv, kC) ||
+        !make_state_map(&smap, a.state, H) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
+        return cudaErrorInvalidValue;
+    // The attribute is per device; setting it on every launch costs little and stays correct after
+    // a device reset and from any host thread.
+    cudaError_t e = cudaFuncSetAttribute(gdn_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemAlloc);
     if (e != cudaSuccess) return e;
-    // update kernel: one persistent CTA per SM (the kernel needs the whole SM: 512 TMEM columns,
-    // ~211 KB of shared memory); each takes every grid-th head, or an equal run of tiles
+    const int n_tiles = (a.T + kTile - 1) / kTile;
     TcArgs t;
     t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = n_tiles;
-    t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.rec = a.scratch; t.status = a.status;
-    t.ho_flag = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
-    t.ho_wflag = t.ho_flag + grid;
+    t.g = a.g; t.beta = a.beta;
+    t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.status = a.status;
+    t.ho_bits = reinterpret_cast<uint32_t*>(a.status) + 4;
     t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
-    // equal tile runs, with heads split between neighbouring CTAs, when they shorten the slowest
-    // CTA: a boundary between slots costs about 0.45 of a tile and the hand-over about three
-    // tiles (measured: 512- and 1024-token chunks gain 5-6 %, chunks of 2-3 tiles lose)
     t.split = 0;
-    const int H = a.L * a.Hv;
     if (H > grid && H % grid != 0) {
-        const double whole = std::ceil((double)H / grid) * (n_tiles + 0.45);
+        const double whole = std::ceil((double)H / grid) * (n_tiles + kBoundary);
         const double runs = std::ceil((double)H * n_tiles / grid);
-        const double parted = runs + (runs / n_tiles + 2.0) * 0.45 + 3.0;
+        const double parted = runs + (runs / n_tiles + 2.0) * kBoundary + kHandOver;
         t.split = parted < whole ? 1 : 0;
     }
-    (void)sms;
-    return launch_dependent(gdn_update_tc_kernel, dim3(grid), dim3(kThreads), (size_t)kSmemAlloc, s, kmap, vmap,
-                            smap, hmap, t);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemAlloc;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    if (t.split) {
+        // every CTA must be resident: a split head's second part waits for its first
+        attr[0].id = cudaLaunchAttributeCooperative;
+        attr[0].val.cooperative = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, gdn_fused_kernel, kmap, vmap, smap, hmap, t);
+        if (e != cudaErrorCooperativeLaunchTooLarge) return e;
+        (void)cudaGetLastError();                 // fewer SMs than the grid: whole heads instead
+        t.split = 0;
+    }
+    cfg.attrs = nullptr;
+    cfg.numAttrs = 0;
+    return cudaLaunchKernelEx(&cfg, gdn_fused_kernel, kmap, vmap, smap, hmap, t);
 }
 
 }  // namespace deltas

@@ -11,7 +11,9 @@ namespace deltas {
 
 // ---------------------------------------------------------------------------------------------
 // Device status word: the first 16 bytes of every workspace.
-//   word[0] = first recorded deltas_status, word[1] = detail, words 2..3 reserved.
+//   word[0] = first recorded deltas_status, word[1] = detail, word[2] = bounded-wait budget
+//   override in microseconds (0: about one second), word[3] reserved; words 4..35 of the 256-byte
+//   header are the tensor-core update's hand-over bits (zero between calls).
 // ---------------------------------------------------------------------------------------------
 constexpr size_t kStatusBytes = 256;   // status word padded so the rest stays 256-byte aligned
 
@@ -110,7 +112,8 @@ struct CopyBatch {
 
 // Kernel launchers (return the launch error, cudaSuccess when enqueued).
 cudaError_t launch_gdn_update_simt(const GdnArgs& a, cudaStream_t s);
-bool gdn_tc_supported(const GdnArgs& a);
+bool gdn_tc_shape(const GdnArgs& a);        // d = 128, bfloat16, no read-out, tokens > 0
+bool gdn_tc_supported(const GdnArgs& a);    // ... and the tensor-core path can be launched
 size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T);
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s);
 cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, const float* sa,

@@ -128,6 +128,12 @@ __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
     asm volatile("prefetch.tensormap [%0];" :: "l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// A tile of a tensor map into L2 only (no shared memory, no completion to wait for).
+__device__ __forceinline__ void tma_prefetch_4d(const CUtensorMap* map, int c0, int c1, int c2, int c3) {
+    asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];"
+                 :: "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3) : "memory");
+}
+
 // ------------------------------------------------------------------------------ TMEM
 // whole warp
 __device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
@@ -348,6 +354,45 @@ __device__ __forceinline__ void mma4_bf16_ss_1t(uint32_t d, const uint64_t (&a)[
                  "tcgen05.mma.cta_group::1.kind::f16 [%0], %4, %8, %9, q;\n\t}"
                  :: "r"(d), "l"(a[0]), "l"(a[1]), "l"(a[2]), "l"(a[3]), "l"(b[0]), "l"(b[1]), "l"(b[2]), "l"(b[3]),
                     "r"(idesc), "r"(acc0) : "memory");
+}
+
+// Four kind::f16 MMAs into one accumulator from one thread, A from TMEM, the first of them scaling
+// the accumulator it reads by 2^-S (the instruction's scale-input-d operand: D = A B + 2^-S D), the
+// other three plain accumulations.
+template <int S>
+__device__ __forceinline__ void mma4_bf16_ta_scaled_1t(uint32_t d, const uint32_t (&a)[4], const uint64_t (&b)[4],
+                                                       uint32_t idesc) {
+    asm volatile("{\n\t.reg .pred q;\n\t"
+                 "setp.eq.b32 q, %9, %9;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %5, %9, q, %10;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%2], %6, %9, q;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%3], %7, %9, q;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%4], %8, %9, q;\n\t}"
+                 :: "r"(d), "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "l"(b[0]), "l"(b[1]), "l"(b[2]), "l"(b[3]),
+                    "r"(idesc), "n"(S) : "memory");
+}
+
+// The same with the shift chosen at run time (0..15; the operand is an immediate in the ISA).
+__device__ __forceinline__ void mma4_bf16_ta_shift_1t(int shift, uint32_t d, const uint32_t (&a)[4],
+                                                      const uint64_t (&b)[4], uint32_t idesc) {
+    switch (shift) {
+        case 0: mma4_bf16_ta_scaled_1t<0>(d, a, b, idesc); break;
+        case 1: mma4_bf16_ta_scaled_1t<1>(d, a, b, idesc); break;
+        case 2: mma4_bf16_ta_scaled_1t<2>(d, a, b, idesc); break;
+        case 3: mma4_bf16_ta_scaled_1t<3>(d, a, b, idesc); break;
+        case 4: mma4_bf16_ta_scaled_1t<4>(d, a, b, idesc); break;
+        case 5: mma4_bf16_ta_scaled_1t<5>(d, a, b, idesc); break;
+        case 6: mma4_bf16_ta_scaled_1t<6>(d, a, b, idesc); break;
+        case 7: mma4_bf16_ta_scaled_1t<7>(d, a, b, idesc); break;
+        case 8: mma4_bf16_ta_scaled_1t<8>(d, a, b, idesc); break;
+        case 9: mma4_bf16_ta_scaled_1t<9>(d, a, b, idesc); break;
+        case 10: mma4_bf16_ta_scaled_1t<10>(d, a, b, idesc); break;
+        case 11: mma4_bf16_ta_scaled_1t<11>(d, a, b, idesc); break;
+        case 12: mma4_bf16_ta_scaled_1t<12>(d, a, b, idesc); break;
+        case 13: mma4_bf16_ta_scaled_1t<13>(d, a, b, idesc); break;
+        case 14: mma4_bf16_ta_scaled_1t<14>(d, a, b, idesc); break;
+        default: mma4_bf16_ta_scaled_1t<15>(d, a, b, idesc); break;
+    }
 }
 
 // Pins register values before the next volatile statement (e.g. operands prepared ahead of a wait).
