@@ -2,52 +2,54 @@
 // bfloat16 k/v, fp32 state, with the state-drift partials fused in: one persistent kernel.
 //
 // Paper: Sec. 3.2, Eq. 1/2 (the recurrence) and Eq. 3 (drift numerator / denominator per layer
-// and head).  The chunk is processed in sub-tiles of C = 32 tokens with the chunkwise (WY) form of
-// Eq. 1.  Inside a sub-tile let G be the inclusive cumulative log-decay, gamma_t = exp(G_t),
+// and head).  The chunk is processed in tiles of C = 64 tokens with the chunkwise (WY) form of
+// Eq. 1.  Inside a tile let G be the inclusive cumulative log-decay, gamma_t = exp(G_t),
 // gamma_C = exp(G_{C-1}), delta_t = gamma_C / gamma_t <= 1, and X = K S0^T (row t: S0 k_t).  With
 //   A[t][i] = beta_t (gamma_t / gamma_i) k_t.k_i  (i < t),   U = (I + A)^-1 diag(beta) (V - diag(gamma) X)
-// the state after the sub-tile is S_C = gamma_C S0 + sum_t delta_t u_t k_t^T.  The decay factors
-// out of the triangular solve by a diagonal similarity, I + A = diag(gamma) (I + diag(beta) L)
-// diag(gamma)^-1 with L the strictly lower part of K K^T, so with the decay-free
+// the state after the tile is S_C = gamma_C S0 + sum_t delta_t u_t k_t^T.  The decay factors out of
+// the triangular solve by a diagonal similarity, I + A = diag(gamma) (I + diag(beta) L) diag(gamma)^-1
+// with L the strictly lower part of K K^T, so with the decay-free
 //   N_beta = (I + diag(beta) L)^-1 diag(beta)
 // the decayed writes are  U~ = diag(delta) U = N_beta (diag(delta) V - gamma_C X):  every decay
-// factor the kernel uses is at most 1, and the inverse depends on k and beta only.
+// factor the kernel uses is at most 1, and the inverse depends on k and beta only.  The X term
+// folds into one product with the state:  gamma_C X^T N_beta^T = S0 (K^T N_beta^T).
 //
 // Work split inside one CTA (one per SM, persistent over (layer, value head) slots):
-//   producer  (4 warps, two groups of two; group g takes the sub-tiles of parity g): K K^T of a
-//             64-token tile comes from the tensor core; each group forms diag(beta) L of its
-//             sub-tile, inverts I + diag(beta) L (16 x 16 diagonal blocks by substitution, the
-//             off-diagonal block by two products) and writes the two operand images the chain
-//             reads: B1 = u diag(delta) N_beta^T as a bfloat16 (hi, lo) pair and B2 = -c N_beta^T
-//             in tf32 (u, c: the state's deferred scale, below)
-//   MMA       (1 warp, one elected lane): every tcgen05.mma, each group's completion by commit
-//   chain     (8 warps): the passes over TMEM between the state-dependent products
-//   loads     (1 warp): K (64-token tiles) and V (32-token sub-tiles) by TMA, L2 prefetch ahead
-//   state     (1 warp): each slot's state into a staging buffer by TMA, S_after out of it
-// Per sub-tile j, in tensor-pipe order:
-//   E(j)   = V^T B1                      (bf16, issued during the previous sub-tile's pass; N = 64:
-//                                         the hi and lo halves land side by side in TMEM)
-//   X      = S~ K^T                      (tf32: A = the fp32 state straight from TMEM, K exact)
-//   E(j)  += X B2                        (tf32: A = X straight from TMEM, no pass in between)
-//   pass   (chain) E = hi half + lo half, split into bfloat16 (hi, lo) A operand
-//   S~     = 2^-s S~ + E K               (bf16 (hi, lo) x K; the input state scaled by the
-//                                         instruction's power-of-two scale-input-d operand)
-// so the chain's own work per sub-tile is one pass over a 128 x 32 block.
+//   producer (4 warps): K K^T of the tile comes from the tensor core; the producer forms
+//            diag(beta) L, inverts I + diag(beta) L (16 x 16 diagonal blocks by substitution, then
+//            two levels of block products) and writes two operand images, each a bfloat16
+//            (hi, lo) pair laid out as the two K-halves of one operand:
+//              B1 = u N_beta diag(delta)   and   B3 = N_beta
+//            (u: the state's deferred scale, below)
+//   MMA      (1 warp, one elected lane): every tcgen05.mma, each group's completion by commit
+//   chain    (8 warps): the pass over E, the K^T N_beta^T product into the B operand W, head
+//            boundaries (state in and out, drift partials)
+//   loads    (1 warp): K and V tiles by TMA, L2 prefetch of the tiles ahead and of the next state
+// Per tile j, in tensor-pipe order:
+//   E(j)  += S~ W(j)                  (tf32: A = the fp32 state straight from TMEM)
+//   Q(j+1) = K^T B3, E(j+1) = V^T B1  (bf16 (hi, lo); the chain turns Q into W(j+1) = -c Q^T in
+//                                      tf32 in shared memory)
+//   K K^T (j+2)                       (bf16, for the producer)
+//   pass   (chain) E -> bfloat16 (hi, lo), in place
+//   S~     = 2^-s S~ + E K            (the input state scaled by the instruction's power-of-two
+//                                      scale-input-d operand)
+// The tensor core does not order an MMA that reads a TMEM region as its A operand after an earlier
+// MMA that wrote it (measured), so E += S~ W waits for the previous state update's commit.
 //
-// Deferred decay.  TMEM holds S~ with the true state S = sig S~.  A sub-tile with decay gamma_C
-// takes p = gamma_C sig and a shift s in [0, 15] that brings p 2^s into [1/2, 1) when it can:
-// then sig <- p 2^s, u = 1 / sig, c = 2^-s, and MMA_S scales S~ by 2^-s as it accumulates (exact).
-// When p < 2^-45 (no shift reaches 2^-30) the chain multiplies S~ by p in a pass instead, sig
-// restarts at 1, u = 1 and c = p.  So sig stays in [2^-30, 1] and u below 2^30.  The producer
-// and the chain see the same per-sub-tile constants (sig after the sub-tile, the shift, the pass
-// factor), which the producer writes beside the images.
+// Deferred decay.  TMEM holds S~ with the true state S = sig S~.  A tile with decay gamma_C takes
+// p = gamma_C sig and a shift s in [0, 15] that brings p 2^s into [1/2, 1) when it can: then
+// sig <- p 2^s, u = 1 / sig, c = 2^-s, and the state update scales S~ by 2^-s as it accumulates
+// (exact).  When p < 2^-45 (no shift reaches 2^-30) the chain multiplies S~ by p in a pass instead,
+// sig restarts at 1, u = 1 and c = p.  So sig stays in [2^-30, 1] and u below 2^30.  The producer
+// writes each tile's constants (sig after the tile, the shift, the pass factor, c, the write-size
+// scales) beside its images.
 //
-// Precision.  k, v exact in bfloat16; K K^T exact in fp32.  The state-dependent products read S~
-// and X as tf32 (10 explicit mantissa bits, truncated) and B2 is rounded to tf32: errors confined
-// to the delta correction.  B1 and E take two-term bfloat16 splits (x = hi + lo, about 2^-16
-// relative).  The inverse is formed in fp32.  A CPU model of exactly these roundings gives a state
-// error against fp64 of 4.5e-4 at the slowest decay the tests use (4 chunks of 1024 tokens), 5e-6
-// at a typical one, and drift numerators within 2.2e-4.
+// Precision.  k, v exact in bfloat16; K K^T exact in fp32.  E += S~ W reads S~ as tf32 (10
+// explicit mantissa bits, truncated) and W is rounded to tf32: errors confined to the delta
+// correction.  B1, B3 and E take two-term bfloat16 splits (x = hi + lo, about 2^-16 relative); the
+// inverse is formed in fp32.  A CPU model of exactly these roundings gives a state error against
+// fp64 of 2.6e-4 at the slowest decay the tests use (4 chunks of 1024 tokens), 5e-6 at a typical
+// one, and drift numerators within 1.1e-4.
 //
 // Synchronisation.  Roles hand work to each other through mbarriers only; every wait is bounded
 // (about one second, or the workspace header's override); a wait that runs out records
@@ -56,9 +58,8 @@
 // tile runs, see ChainSched) hand the state over through the workspace with a bit per CTA boundary
 // in the workspace header, which its reader clears after use.
 //
-// TMEM (512 columns, 128 lanes = d_v): S~ [0,128), S_before [128,256), X [256,288),
-// E0 [288,352), E1 [352,416) (each: hi-half product [+0,+32), lo-half product [+32,+64)),
-// K K^T [416,480) (lanes 0..63), packed A of MMA_S [480,512) (hi k-step 0, 1, lo k-step 0, 1).
+// TMEM (512 columns, 128 lanes): S~ [0,128), S_before [128,256), E0 [256,320), E1 [320,384)
+// (E fp32, then its (hi, lo) A operand in place), K K^T [384,448) (lanes 0..63), Q [448,512).
 #include <algorithm>
 #include <cmath>
 
@@ -70,53 +71,48 @@ namespace {
 
 using namespace tc;
 
-constexpr int kC = 32;                 // tokens per sub-tile
-constexpr int kTile = 64;              // tokens per tile (two sub-tiles; the schedule's unit)
+constexpr int kC = 64;                 // tokens per tile
 constexpr int kD = 128;                // head dim (d_k = d_v)
 constexpr float kHardMin = 0x1p-45f;   // p below this: the state is rescaled by a pass
 
 // ---- roles
 constexpr int kChainWarps = 8;
 constexpr int kChain = 32 * kChainWarps;
-constexpr int kProdWarp0 = 8;          // 8, 9: TMEM readers of producer groups 0, 1; 10, 11: partners
+constexpr int kProdWarp0 = 8;          // 8..11: producer (warp 8 + i reads TMEM lanes 32 i ..)
+constexpr int kProd = 128;
 constexpr int kMmaWarp = 12;
 constexpr int kLoadWarp = 13;
-constexpr int kStateWarp = 14;
-constexpr int kThreads = 15 * 32;
-constexpr int kBarChain = 1;           // named barriers: chain (256 threads), producer groups (64)
-constexpr int kBarProd0 = 2;
+constexpr int kThreads = 14 * 32;
+constexpr int kBarChain = 1;           // named barriers: chain (256 threads), producer (128)
+constexpr int kBarProd = 2;
 
 // ---- TMEM columns
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t TM_S = 0, TM_SB = 128, TM_X = 256, TM_E = 288, TM_KK = 416, TM_AP = 480;
+constexpr uint32_t TM_S = 0, TM_SB = 128, TM_E = 256, TM_KK = 384, TM_Q = 448;
 
 // ---- shared memory (bytes from a 1024-aligned base)
-constexpr uint32_t SM_K = 0;           // 3 tiles x 16 KB: 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B,
-                                       // SW128; sub-tile u in rows 32u..32u+31
-constexpr uint32_t SM_K32 = 49152;     // 16 KB: one sub-tile's K in fp32, 4 column blocks (32 dims) x 32 rows
-                                       // x 128 B, SW128 (the B operand of X); also the K K^T product's
-                                       // over-read past the last K tile (rows 64..127 of its M = 128 A)
-constexpr uint32_t SM_V = 65536;       // 3 sub-tiles x 8 KB: 2 column blocks x 32 rows x 128 B, SW128
-constexpr uint32_t SM_IMG = 90112;     // 4 slots x 12 KB: B1 hi [0, 4 KB) and lo [4, 8 KB) (32 rows x 128 B,
-                                       // the first 64 B of a row used), B2 [8, 12 KB) (32 rows x 32 fp32)
-constexpr uint32_t kImgSlot = 12288;
-constexpr uint32_t SM_SB = 139264;     // 64 KB: state staging, 4 column blocks x 128 rows x 128 B, SW128
-constexpr uint32_t SM_PW = 204800;     // producer workspaces, one per group
-constexpr int kMS = 36;                // fp32 row stride of M and N (16-byte aligned rows)
-constexpr int kPS = 20;                // fp32 row stride of the 16 x 16 product
-// beta, delta and (u, c) of the group's sub-tile are double-buffered by tile parity: the partner
-// warp writes the next tile's while the other may still read this one's
-constexpr int PW_M = 0, PW_N = 32 * kMS, PW_P = 64 * kMS, PW_BETA = PW_P + 16 * kPS, PW_DELTA = PW_BETA + 64,
-              PW_UC = PW_DELTA + 64, PW_FLOATS = PW_UC + 8;
-constexpr uint32_t kPwBytes = PW_FLOATS * 4;
-constexpr uint32_t SM_CONST = SM_PW + 2 * kPwBytes;   // 4 slots x 48 words: per-sub-tile constants
-constexpr int kConstWords = 48;        // [0,32) write-size scale per token, 32 sig after, 33 pass factor
-                                       // (< 0: none), 34 shift (int)
-constexpr uint32_t SM_BYTES = SM_CONST + 4 * kConstWords * 4;
+constexpr uint32_t SM_K = 0;           // 3 tiles x 16 KB: 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B, SW128
+constexpr uint32_t SM_V = 49152;       // 2 tiles x 16 KB, same layout (also the K K^T product's over-read
+                                       // past the last K tile: rows 64..127 of its M = 128 A)
+constexpr uint32_t SM_B1 = 81920;      // 2 x 16 KB: rows t of u N_beta diag(delta): hi in column block 0,
+                                       // lo in block 1 (64 rows x 128 B each, SW128)
+constexpr uint32_t SM_B3 = 114688;     // 2 x 16 KB: N_beta, same layout
+constexpr uint32_t SM_W = 147456;      // 32 KB: W^T = -c N_beta K in tf32, rows t: 4 column blocks (32 dims)
+                                       // x 64 rows x 128 B, SW128 (the B operand of E += S~ W)
+constexpr uint32_t SM_PW = 180224;     // producer workspace
+constexpr int kMS = 68;                // fp32 row stride of M and N (16-byte aligned rows)
+constexpr int kPS = 36;                // fp32 row stride of the block products
+constexpr int PW_M = 0, PW_N = 64 * kMS, PW_P = 128 * kMS, PW_BETA = PW_P + 32 * kPS, PW_DELTA = PW_BETA + 128,
+              PW_UC = PW_DELTA + 128, PW_FLOATS = PW_UC + 8;   // beta, delta, (u, c): [2][..] by tile parity
+constexpr uint32_t SM_CONST = SM_PW + PW_FLOATS * 4;   // 2 slots x kConstWords: per-tile constants
+constexpr int kConstWords = 72;        // [0,64) write-size scale per token, 64 sig after, 65 pass factor
+                                       // (< 0: none), 66 shift (int), 67 c
+constexpr uint32_t SM_BYTES = SM_CONST + 2 * kConstWords * 4;
 constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
-static_assert(SM_K32 % 1024 == 0 && SM_V % 1024 == 0 && SM_IMG % 1024 == 0 && SM_SB % 1024 == 0 &&
-              kImgSlot % 1024 == 0 && SM_PW % 16 == 0 && kPwBytes % 16 == 0, "shared-memory map");
-static_assert(SM_IMG == SM_V + 3 * 8192 && SM_SB == SM_IMG + 4 * kImgSlot && SM_PW == SM_SB + 65536, "map order");
+static_assert(SM_V % 1024 == 0 && SM_B1 % 1024 == 0 && SM_B3 % 1024 == 0 && SM_W % 1024 == 0 &&
+              SM_PW % 16 == 0 && SM_CONST % 16 == 0, "shared-memory map");
+static_assert(SM_V == SM_K + 3 * 16384 && SM_B1 == SM_V + 2 * 16384 && SM_B3 == SM_B1 + 2 * 16384 &&
+              SM_W == SM_B3 + 2 * 16384 && SM_PW == SM_W + 32768, "map order");
 static_assert(kSmemAlloc + 1024 <= 232448, "shared memory budget");
 
 // Barrier over `n` threads that also returns the OR of `flag` over them (uniform result).
@@ -151,6 +147,48 @@ __device__ __forceinline__ uint32_t to_tf32(float x) {
     return y;
 }
 
+// D (16 x 8) += A (16 x 16, row-major) B (16 x 8) on the warp's tensor-core path, bf16 in, fp32
+// accumulate.  Fragments (g = lane / 4, t = lane % 4), each register a bf16 pair, lower k in the
+// low half: a = A[g][2t..], A[g+8][2t..], A[g][2t+8..], A[g+8][2t+8..]; b = B[2t..][g],
+// B[2t+8..][g]; d = D[g][2t, 2t+1], D[g+8][2t, 2t+1].
+__device__ __forceinline__ void mma_m16n8k16_bf16(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                 "{%0,%1,%2,%3};"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+// D (16 x 8) += A (16 x 16 KS) B (16 KS x 8) for fp32 operands in shared memory (A row-major with
+// row stride lda, B row-major B[k][n] with row stride ldb), each split into bfloat16 (hi, lo) in
+// registers and multiplied as lo hi + hi lo + hi hi (about 2^-16 relative error per product).
+template <int KS>
+__device__ __forceinline__ void mma_f32_split(float (&d)[4], const float* A, int lda, const float* B, int ldb,
+                                              int g, int t) {
+    // the three products accumulate separately (independent chains), summed at the end
+    float d1[4] = {0.f, 0.f, 0.f, 0.f}, d2[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int ks = 0; ks < KS; ++ks) {
+        const float* a0 = A + g * lda + 16 * ks + 2 * t;
+        const float2 x0 = *reinterpret_cast<const float2*>(a0);
+        const float2 x1 = *reinterpret_cast<const float2*>(a0 + 8 * lda);
+        const float2 x2 = *reinterpret_cast<const float2*>(a0 + 8);
+        const float2 x3 = *reinterpret_cast<const float2*>(a0 + 8 * lda + 8);
+        const float* b0 = B + (16 * ks + 2 * t) * ldb + g;
+        uint32_t ah[4], al[4], bh[2], bl[2];
+        split2(x0.x, x0.y, ah[0], al[0]);
+        split2(x1.x, x1.y, ah[1], al[1]);
+        split2(x2.x, x2.y, ah[2], al[2]);
+        split2(x3.x, x3.y, ah[3], al[3]);
+        split2(b0[0], b0[ldb], bh[0], bl[0]);
+        split2(b0[8 * ldb], b0[9 * ldb], bh[1], bl[1]);
+        mma_m16n8k16_bf16(d1, al, bh);
+        mma_m16n8k16_bf16(d2, ah, bl);
+        mma_m16n8k16_bf16(d, ah, bh);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) d[i] += d1[i] + d2[i];
+}
+
 // All lanes of a converged warp wait; the result is the same on every lane.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
                                           const volatile int* abort) {
@@ -170,26 +208,26 @@ __device__ __forceinline__ void warp_arrive(uint64_t* bar, int lane) {
     if (lane == 0) mbar_arrive(bar);
 }
 
-__device__ __forceinline__ int ld_acquire(const uint32_t* p) {
-    int v;
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+    uint32_t v;
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
-// orders the tensor copies' global accesses with the generic ones around a hand-over bit
-__device__ __forceinline__ void fence_proxy_async_global() {
-    asm volatile("fence.proxy.async.global;" ::: "memory");
+
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" :: "l"(p), "r"(bytes) : "memory");
 }
 
-// The per-sub-tile decay bookkeeping (see the header): from p = gamma_C sig, the shift s, the
-// scale u of the V term, the coefficient c of the X term, the pass factor (< 0: no pass) and sig
-// after the sub-tile.
+// The per-tile decay bookkeeping (see the header): from p = gamma_C sig, the shift s, the scale u
+// of the V term, the coefficient c of the state term, the pass factor (< 0: no pass) and sig after
+// the tile.
 struct DecayStep {
     int shift;
     float u, c, pass, sig;
 };
 __device__ __forceinline__ DecayStep decay_step(float p) {
     DecayStep d;
-    if (!(p >= kHardMin)) {                            // also p = 0 or NaN-free underflow
+    if (!(p >= kHardMin)) {
         d.shift = 0; d.u = 1.f; d.c = p; d.pass = p; d.sig = 1.f;
         return d;
     }
@@ -207,11 +245,12 @@ struct TcArgs {
     int L, Hk, Hv, T, n_tiles;   // n_tiles: 64-token tiles per head
     const float* g;              // [L][T][Hv] log-decay
     const float* beta;           // [L][T][Hv]
-    float* state;
+    float* state;                // [L * Hv][128][128]
     float* partials;
     float* wnorm;
     int32_t* status;
     uint32_t* ho_bits;           // hand-over bits in the workspace header: [0, 16) state, [16, 32) sums
+    float* ho_state;             // [grid][128][128]
     float* ho_wsum;              // [grid]
     int split;                   // run equal tile runs (ChainSched)
 };
@@ -281,30 +320,32 @@ struct TileCursor {
     }
 };
 
-// The staging buffer holds a head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each
-// 128 rows x 128 bytes with the 128-byte swizzle that TMA writes and reads.  Float offset of 16-byte
-// chunk `chunk` (0..31) of row `row`:
-__device__ __forceinline__ int sb_idx(int row, int chunk) {
-    return (chunk >> 3) * 4096 + row * 32 + (((chunk & 7) ^ (row & 7)) << 2);
+// 16 fp32 of a state row, global -> registers (through L2 only for data another CTA wrote)
+__device__ __forceinline__ void ld16_global(const float* p, float (&v)[16], bool cache_global) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float4 x = cache_global ? __ldcg(reinterpret_cast<const float4*>(p) + e)
+                                      : __ldg(reinterpret_cast<const float4*>(p) + e);
+        v[4 * e] = x.x; v[4 * e + 1] = x.y; v[4 * e + 2] = x.z; v[4 * e + 3] = x.w;
+    }
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                 const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap hmap,
-                 TcArgs a)
+gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
-    // loads -> roles: K tiles, V sub-tiles full; MMA -> loader: their empties.  producer <-> MMA:
-    // operand images full / empty (the chain's constants read too), K K^T done / read.  state
-    // staging full (mb_st) and released by the chain (mb_sfree).  MMA -> chain: u (E ready), s
-    // (state updated); chain -> MMA: sready (state and K in fp32 ready for X), uready (A packed).
-    __shared__ uint64_t mb_kfull[3], mb_kempty[3], mb_vfull[3], mb_vempty[3], mb_ifull[4], mb_iempty[4];
-    __shared__ uint64_t mb_kk, mb_kkfree, mb_st, mb_sfree, mb_sready, mb_x, mb_u, mb_uready, mb_s, mb_fin;
+    // loads -> roles: K, V tiles full; MMA -> loader: their empties.  producer -> MMA / chain: images
+    // and constants full (ifull); released by the products that read them and by the chain
+    // (iempty).  MMA -> producer: K K^T done (kk); producer -> MMA: read (kkfree).  MMA -> chain:
+    // Q done (q), E ready (u), state updated (s); chain -> MMA: W and the slot's state ready
+    // (ready), E packed (uready).
+    __shared__ uint64_t mb_kfull[3], mb_kempty[3], mb_vfull[2], mb_vempty[2], mb_ifull[2], mb_iempty[2];
+    __shared__ uint64_t mb_kk, mb_kkfree, mb_q, mb_ready, mb_u, mb_uready, mb_s, mb_fin;
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ float s_red[2][kChainWarps];
-    __shared__ float s_u2[2][kC];                     // per-token squared write sizes (sub-tile parity)
+    __shared__ float s_u2[2][kC];                     // per-token squared write sizes (tile parity)
     volatile int* abort_flag = &s_abort;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -313,9 +354,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     const uint64_t budget = budget_us ? (uint64_t)budget_us * 1000ull : kWaitBudgetNs;
     ChainSched sch;
     sch.init(a);
-    const int n_slots = sch.n_slots;
     const int NJ = sch.NJ;                            // tiles of this CTA
-    const int NS = 2 * NJ;                            // sub-tiles
     const int me = (int)blockIdx.x;
     uint32_t* bits_state = a.ho_bits;
     uint32_t* bits_wsum = a.ho_bits + 16;
@@ -324,40 +363,36 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         tmem_alloc(&s_tmem, kTmemCols);
         tmem_relinquish();
         if (lane == 0) {
-            for (int b = 0; b < 3; ++b) {
-                mbar_init(&mb_kfull[b], 1); mbar_init(&mb_kempty[b], 1);
+            for (int b = 0; b < 3; ++b) { mbar_init(&mb_kfull[b], 1); mbar_init(&mb_kempty[b], 1); }
+            for (int b = 0; b < 2; ++b) {
                 mbar_init(&mb_vfull[b], 1); mbar_init(&mb_vempty[b], 1);
+                mbar_init(&mb_ifull[b], 4); mbar_init(&mb_iempty[b], 1 + kChainWarps);
             }
-            for (int b = 0; b < 4; ++b) { mbar_init(&mb_ifull[b], 2); mbar_init(&mb_iempty[b], 1 + kChainWarps); }
-            mbar_init(&mb_kk, 1); mbar_init(&mb_kkfree, 2);
-            mbar_init(&mb_st, 1); mbar_init(&mb_sfree, kChainWarps);
-            mbar_init(&mb_sready, kChainWarps); mbar_init(&mb_x, 1); mbar_init(&mb_u, 1);
-            mbar_init(&mb_uready, kChainWarps);
+            mbar_init(&mb_kk, 1); mbar_init(&mb_kkfree, 2); mbar_init(&mb_q, 1);
+            mbar_init(&mb_ready, kChainWarps); mbar_init(&mb_u, 1); mbar_init(&mb_uready, kChainWarps);
             mbar_init(&mb_s, 1); mbar_init(&mb_fin, 1);
             fence_barrier_init();
         }
     }
     if (warp == kLoadWarp && lane == 0) { prefetch_tensormap(&kmap); prefetch_tensormap(&vmap); }
-    if (warp == kStateWarp && lane == 0) { prefetch_tensormap(&smap); prefetch_tensormap(&hmap); }
     if (tid == 0) s_abort = 0;
-    if (tid < 2 * kC) s_u2[tid >> 5][tid & (kC - 1)] = 0.f;
+    if (tid < 2 * kC) s_u2[tid >> 6][tid & (kC - 1)] = 0.f;
     grid_dep_launch();                                // the next kernel (the score) may be scheduled
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tm = s_tmem;
-    const float* cst = reinterpret_cast<const float*>(sm + SM_CONST);
+    float* cst = reinterpret_cast<float*>(sm + SM_CONST);
 
     if (warp == kMmaWarp) {
         // =========================================================== MMA issue (converged warp;
         // one elected lane issues each group and commits it)
-        const uint32_t idX = idesc_tf32(128, 32);
-        const uint32_t idE = idesc_bf16(128, 64, 1, 0);
+        const uint32_t idW = idesc_bf16(128, 64, 1, 0);   // Q and E products: A MN-major (K^T, V^T)
+        const uint32_t idX = idesc_tf32(128, 64);
         const uint32_t idS = idesc_bf16(128, 128, 0, 1);
         const uint32_t idK = idesc_bf16(128, 64, 0, 0);
         // K K^T of tile J (M = 128: rows 64..127 of A read the 16 KB past the tile; their output
-        // lanes are ignored).  Waits for the tile and for both producer groups to have read the
-        // previous product out of TMEM.
+        // lanes are ignored), once the tile has landed and the producer has read the previous one
         auto issue_kk = [&](int J) -> bool {
             const uint32_t base = smem_u32(sm + SM_K + (J % 3) * 16384);
             uint64_t d[2][4];
@@ -377,98 +412,94 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             mma_commit(&mb_kk);
             return true;
         };
-        // E(j) <- V(j)^T B1(j): A = the V sub-tile read MN-major, B = the 64-row (hi, lo) image
-        auto issue_einit = [&](int j) -> bool {
-            const uint32_t vb = smem_u32(sm + SM_V + (j % 3) * 8192);
-            const uint32_t ib = smem_u32(sm + SM_IMG + (j & 3) * kImgSlot);
-            const uint64_t a0 = sdesc_sw128(vb, 4096, 1024), a1 = sdesc_sw128(vb + 2048, 4096, 1024);
-            const uint64_t b0 = sdesc_sw128(ib, 16, 1024), b1 = sdesc_sw128(ib + 32, 16, 1024);
-            pin(a0); pin(a1); pin(b0); pin(b1);
-            if (!warp_wait(&mb_vfull[j % 3], (j / 3) & 1, budget, abort_flag)) return false;
-            if (!warp_wait(&mb_ifull[j & 3], (j >> 2) & 1, budget, abort_flag)) return false;
-            tc_fence_after();
+        // A (K^T or V^T: the tile read MN-major; k-steps 4..7 repeat tokens 0..63 for the lo half)
+        // times B (an image: k-steps 0..3 its hi block, 4..7 its lo block) into D
+        auto issue_img = [&](uint32_t d, uint32_t a_base, uint32_t b_base) {
+            uint64_t ad[2][4], bd[2][4];
+#pragma unroll
+            for (int s = 0; s < 8; ++s) {
+                ad[s >> 2][s & 3] = sdesc_sw128(a_base + (s & 3) * 2048, 8192, 1024);
+                bd[s >> 2][s & 3] = sdesc_sw128(b_base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
+            }
             if (elect_one()) {
-                mma_bf16_1t(tm + TM_E + (j & 1) * 64, a0, b0, idE, 0);
-                mma_bf16_1t(tm + TM_E + (j & 1) * 64, a1, b1, idE, 1);
+                mma4_bf16_ss_1t(d, ad[0], bd[0], idW, 0);
+                mma4_bf16_ss_1t(d, ad[1], bd[1], idW, 1);
             }
             __syncwarp();
-            mma_commit(&mb_vempty[j % 3]);
+        };
+        // Q(J) = K(J)^T B3(J) and E(J) = V(J)^T B1(J), once the images are written
+        auto issue_images = [&](int J) -> bool {
+            if (!warp_wait(&mb_ifull[J & 1], (J >> 1) & 1, budget, abort_flag)) return false;
+            tc_fence_after();
+            issue_img(tm + TM_Q, smem_u32(sm + SM_K + (J % 3) * 16384), smem_u32(sm + SM_B3 + (J & 1) * 16384));
+            mma_commit(&mb_q);
+            if (!warp_wait(&mb_vfull[J & 1], (J >> 1) & 1, budget, abort_flag)) return false;
+            tc_fence_after();
+            issue_img(tm + TM_E + (J & 1) * 64, smem_u32(sm + SM_V + (J & 1) * 16384),
+                      smem_u32(sm + SM_B1 + (J & 1) * 16384));
+            mma_commit(&mb_vempty[J & 1]);
+            mma_commit(&mb_iempty[J & 1]);             // the images' products are issued
             return true;
         };
         bool ok = true;
-        if (NS > 0) {
+        if (NJ > 0) {
             ok = issue_kk(0);
             if (ok && NJ > 1) ok = issue_kk(1);
-            if (ok) ok = issue_einit(0);            // completes before X(0)'s commit
+            if (ok) ok = issue_images(0);
             if (!ok) fail(a.status, abort_flag, 1);
         }
-        // The tensor core does not order an MMA that reads a TMEM region as its A operand after an
-        // earlier MMA that wrote it (measured: X read by the next product lacked the last of its 16
-        // k-steps), so each such hand-off waits for the writer's commit: X before E += X B2, and
-        // the updated state before the next X.  Independent work fills the turnarounds: the next
-        // sub-tile's E product between X and E += X B2, the K K^T product during the chain's pass.
-        for (int j = 0; ok && j < NS; ++j) {
+        for (int j = 0; ok && j < NJ; ++j) {
             const uint32_t eb = tm + TM_E + (j & 1) * 64;
             int shift = 0;
-            {   // X <- S~ K^T (A: the state from TMEM as tf32, 8 columns per K = 8 step; B: K in fp32)
+            {   // E(j) += S~ W(j) (A: the state from TMEM as tf32, 8 columns per K = 8 step; B: W in
+                // tf32).  E(j)'s own product was issued before, into the same accumulator.
                 uint32_t ax[4][4];
                 uint64_t bx[4][4];
-                const uint32_t k32 = smem_u32(sm + SM_K32);
+                const uint32_t wb = smem_u32(sm + SM_W);
 #pragma unroll
                 for (int s = 0; s < 16; ++s) {
                     ax[s >> 2][s & 3] = tm + TM_S + 8 * s;
-                    bx[s >> 2][s & 3] = sdesc_sw128(k32 + (s >> 2) * 4096 + (s & 3) * 32, 16, 1024);
+                    bx[s >> 2][s & 3] = sdesc_sw128(wb + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
                     pin(ax[s >> 2][s & 3]); pin(bx[s >> 2][s & 3]);
                 }
-                if (!warp_wait(&mb_sready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 2); break; }
-                if (j > 0 && !warp_wait(&mb_s, (j - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 7); break; }
-                if (!warp_wait(&mb_ifull[j & 3], (j >> 2) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 3); break; }
-                // read while the image slot is held (released once its products and the chain are done)
-                shift = reinterpret_cast<const volatile int*>(cst + (j & 3) * kConstWords)[34];
+                if (!warp_wait(&mb_ready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 2); break; }
+                if (j > 0 && !warp_wait(&mb_s, (j - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 3); break; }
+                // E(j)'s own product has completed: for j > 0 the state update's commit covers it
+                // (issued after it), for the first tile its own commit
+                if (j == 0 && !warp_wait(&mb_vempty[0], 0, budget, abort_flag)) { fail(a.status, abort_flag, 7); break; }
+                // the tile's images and constants are held until the chain has read them
+                shift = reinterpret_cast<const volatile int*>(cst + (j & 1) * kConstWords)[66];
                 tc_fence_after();
                 if (elect_one()) {
 #pragma unroll
-                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + TM_X, ax[g4], bx[g4], idX, g4 != 0);
+                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(eb, ax[g4], bx[g4], idX, 1);
                 }
-                __syncwarp();
-                mma_commit(&mb_x);
-            }
-            if (j + 1 < NS && !issue_einit(j + 1)) { fail(a.status, abort_flag, 5); break; }
-            {   // E(j) += X B2 (A: X from TMEM as tf32); E(j)'s own product completed before X's commit
-                uint32_t au[4];
-                uint64_t bu[4];
-                const uint32_t b2 = smem_u32(sm + SM_IMG + (j & 3) * kImgSlot + 8192);
-#pragma unroll
-                for (int s = 0; s < 4; ++s) {
-                    au[s] = tm + TM_X + 8 * s;
-                    bu[s] = sdesc_sw128(b2 + 32 * s, 16, 1024);
-                    pin(au[s]); pin(bu[s]);
-                }
-                if (!warp_wait(&mb_x, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 8); break; }
-                tc_fence_after();
-                if (elect_one()) mma4_tf32_ta_1t(eb, au, bu, idX, 1);
                 __syncwarp();
                 mma_commit(&mb_u);
-                mma_commit(&mb_iempty[j & 3]);
             }
-            // K K^T one and a half tiles ahead of the chain, while the chain runs its pass
-            if ((j & 1) && (j + 3) / 2 < NJ && !issue_kk((j + 3) / 2)) { fail(a.status, abort_flag, 4); break; }
-            {   // S~ = 2^-shift S~ + E K  (A: E hi / lo packed in TMEM; K read MN-major)
-                uint32_t as_[4];
+            // the next tile's Q and E, and K K^T two tiles ahead, while the chain runs its pass
+            if (j + 1 < NJ && !issue_images(j + 1)) { fail(a.status, abort_flag, 4); break; }
+            if (j + 2 < NJ && !issue_kk(j + 2)) { fail(a.status, abort_flag, 5); break; }
+            {   // S~ = 2^-shift S~ + E K  (A: E hi / lo packed in place; K read MN-major)
+                uint32_t ah[4], al[4];
                 uint64_t bs[4];
-                const uint32_t kb = smem_u32(sm + SM_K + ((j >> 1) % 3) * 16384) + (j & 1) * 4096;
+                const uint32_t kb = smem_u32(sm + SM_K + (j % 3) * 16384);
 #pragma unroll
                 for (int s = 0; s < 4; ++s) {
-                    as_[s] = tm + TM_AP + 8 * s;
-                    bs[s] = sdesc_sw128(kb + (s & 1) * 2048, 8192, 1024);
-                    pin(as_[s]); pin(bs[s]);
+                    ah[s] = eb + 32 * (s >> 1) + 8 * (s & 1);
+                    al[s] = ah[s] + 16;
+                    bs[s] = sdesc_sw128(kb + s * 2048, 8192, 1024);
+                    pin(ah[s]); pin(al[s]); pin(bs[s]);
                 }
                 if (!warp_wait(&mb_uready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 6); break; }
                 tc_fence_after();
-                if (elect_one()) mma4_bf16_ta_shift_1t(shift, tm + TM_S, as_, bs, idS);
+                if (elect_one()) {
+                    mma4_bf16_ta_shift_1t(shift, tm + TM_S, ah, bs, idS);
+                    mma4_bf16_ta_1t(tm + TM_S, al, bs, idS, 1);
+                }
                 __syncwarp();
                 mma_commit(&mb_s);
-                if (j & 1) mma_commit(&mb_kempty[(j >> 1) % 3]);   // the tile's last reader
+                mma_commit(&mb_kempty[j % 3]);         // the tile's last reader
             }
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0)) {
@@ -477,363 +508,303 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         }
         __syncwarp();
     } else if (warp == kLoadWarp) {
-        // =========================================================== K tiles and V sub-tiles in
-        // order, each into its buffer once the MMA that last read the buffer has completed; the
-        // tiles three ahead are prefetched into L2
+        // =========================================================== K and V tiles in order, each
+        // into its buffer once the MMA that last read the buffer has completed; the tiles three
+        // ahead and each slot's successor's state are prefetched into L2
         TileCursor cc, pf;
         cc.init(sch, a);
         pf.init(sch, a);
-        int kp[3] = {-1, -1, -1}, vp[3] = {-1, -1, -1};   // last tile / sub-tile loaded per buffer
+        int kp[3] = {-1, -1, -1}, vp[2] = {-1, -1};   // last tile loaded per buffer
         grid_dep_wait();
-        // prime the prefetch cursor three tiles ahead
+        auto prefetch_tile = [&](const TileCursor& c) {
+            tma_prefetch_4d(&kmap, 0, c.kh, c.jt * kC, c.l);
+            tma_prefetch_4d(&kmap, 64, c.kh, c.jt * kC, c.l);
+            tma_prefetch_4d(&vmap, 0, c.h, c.jt * kC, c.l);
+            tma_prefetch_4d(&vmap, 64, c.h, c.jt * kC, c.l);
+        };
         for (int i = 0; i < 3 && i < NJ; ++i) {
-            if (elect_one()) {
-                tma_prefetch_4d(&kmap, 0, pf.kh, pf.jt * kTile, pf.l);
-                tma_prefetch_4d(&kmap, 64, pf.kh, pf.jt * kTile, pf.l);
-                tma_prefetch_4d(&vmap, 0, pf.h, pf.jt * kTile, pf.l);
-                tma_prefetch_4d(&vmap, 64, pf.h, pf.jt * kTile, pf.l);
-                tma_prefetch_4d(&vmap, 0, pf.h, pf.jt * kTile + kC, pf.l);
-                tma_prefetch_4d(&vmap, 64, pf.h, pf.jt * kTile + kC, pf.l);
-            }
+            if (elect_one()) prefetch_tile(pf);
             __syncwarp();
             pf.next(sch, a);
         }
         bool ok = true;
         for (int J = 0; ok && J < NJ; ++J) {
             if (J + 3 < NJ) {
-                if (elect_one()) {
-                    tma_prefetch_4d(&kmap, 0, pf.kh, pf.jt * kTile, pf.l);
-                    tma_prefetch_4d(&kmap, 64, pf.kh, pf.jt * kTile, pf.l);
-                    tma_prefetch_4d(&vmap, 0, pf.h, pf.jt * kTile, pf.l);
-                    tma_prefetch_4d(&vmap, 64, pf.h, pf.jt * kTile, pf.l);
-                    tma_prefetch_4d(&vmap, 0, pf.h, pf.jt * kTile + kC, pf.l);
-                    tma_prefetch_4d(&vmap, 64, pf.h, pf.jt * kTile + kC, pf.l);
-                }
+                if (elect_one()) prefetch_tile(pf);
                 __syncwarp();
                 pf.next(sch, a);
             }
-            const int bk = J % 3;
+            if (cc.jt == cc.tb && cc.k + 1 < sch.n_slots && !sch.is_suffix(cc.k + 1) && elect_one()) {
+                int lh, tb, te;                          // the next slot's state, ahead of its boundary
+                sch.slot(cc.k + 1, a.n_tiles, lh, tb, te);
+                prefetch_l2_bulk(a.state + (size_t)lh * kD * kD, kD * kD * 4);
+            }
+            __syncwarp();
+            const int bk = J % 3, bv = J & 1;
             if (J >= 3 && !warp_wait(&mb_kempty[bk], ((J / 3) - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 30); break; }
             if (elect_one()) {
                 uint8_t* dst = sm + SM_K + bk * 16384;
                 mbar_arrive_expect_tx(&mb_kfull[bk], 16384);
-                tma_load_4d(dst, &kmap, &mb_kfull[bk], 0, cc.kh, cc.jt * kTile, cc.l);
-                tma_load_4d(dst + 8192, &kmap, &mb_kfull[bk], 64, cc.kh, cc.jt * kTile, cc.l);
+                tma_load_4d(dst, &kmap, &mb_kfull[bk], 0, cc.kh, cc.jt * kC, cc.l);
+                tma_load_4d(dst + 8192, &kmap, &mb_kfull[bk], 64, cc.kh, cc.jt * kC, cc.l);
             }
             __syncwarp();
             kp[bk] = J;
-            for (int u = 0; u < 2; ++u) {
-                const int j = 2 * J + u, bv = j % 3;
-                if (j >= 3 && !warp_wait(&mb_vempty[bv], ((j / 3) - 1) & 1, budget, abort_flag)) {
-                    fail(a.status, abort_flag, 31);
-                    ok = false;
-                    break;
-                }
-                if (elect_one()) {
-                    uint8_t* dst = sm + SM_V + bv * 8192;
-                    mbar_arrive_expect_tx(&mb_vfull[bv], 8192);
-                    tma_load_4d(dst, &vmap, &mb_vfull[bv], 0, cc.h, cc.jt * kTile + kC * u, cc.l);
-                    tma_load_4d(dst + 4096, &vmap, &mb_vfull[bv], 64, cc.h, cc.jt * kTile + kC * u, cc.l);
-                }
-                __syncwarp();
-                vp[bv] = j;
+            if (J >= 2 && !warp_wait(&mb_vempty[bv], ((J >> 1) - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 31); break; }
+            if (elect_one()) {
+                uint8_t* dst = sm + SM_V + bv * 16384;
+                mbar_arrive_expect_tx(&mb_vfull[bv], 16384);
+                tma_load_4d(dst, &vmap, &mb_vfull[bv], 0, cc.h, cc.jt * kC, cc.l);
+                tma_load_4d(dst + 8192, &vmap, &mb_vfull[bv], 64, cc.h, cc.jt * kC, cc.l);
             }
+            __syncwarp();
+            vp[bv] = J;
             cc.next(sch, a);
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0) && lane == 0) {
             // every copy this warp issued lands before the CTA ends
-            for (int b = 0; b < 3; ++b) {
+            for (int b = 0; b < 3; ++b)
                 if (kp[b] >= 0) mbar_wait(&mb_kfull[b], (kp[b] / 3) & 1, budget);
-                if (vp[b] >= 0) mbar_wait(&mb_vfull[b], (vp[b] / 3) & 1, budget);
-            }
-        }
-        __syncwarp();
-    } else if (warp == kStateWarp) {
-        // =========================================================== state moves (lane 0).  Phases
-        // of mb_st: 0 = the first slot's state staged; k + 1 = what the boundary after slot k
-        // needs: the state of slot k + 1, or after the last slot a free buffer (when the last slot
-        // ends a head begun by CTA i - 1: that head's state before the chunk, for its drift).
-        // Phases of mb_sfree: 0 = the first state is in TMEM; k + 1 = slot k's final state is
-        // staged.  A first slot that begins a head shared with CTA i + 1 leaves its state in
-        // hand-over entry i; a last slot that ends a head shared with CTA i - 1 starts from entry
-        // i - 1 once that entry's bit is set (bounded wait), and clears the bit.
-        if (lane == 0 && n_slots > 0) {
-            float* sbuf = reinterpret_cast<float*>(sm + SM_SB);
-            int loads = 0, seen = 0;                   // copies into the staging buffer issued / landed
-            auto load_rows = [&](const CUtensorMap* map, int row) {
-                mbar_arrive_expect_tx(&mb_st, kD * kD * 4);
-#pragma unroll
-                for (int b = 0; b < 4; ++b) tma_load_2d(sbuf + 4096 * b, map, &mb_st, 32 * b, row);
-                ++loads;
-            };
-            auto load_state = [&](int slot) -> bool {
-                int lh, tb, te;
-                sch.slot(slot, a.n_tiles, lh, tb, te);
-                if (!sch.is_suffix(slot)) { load_rows(&smap, lh * kD); return true; }
-                const uint32_t bit = 1u << ((me - 1) & 31);
-                uint32_t* w = bits_state + ((me - 1) >> 5);
-                const uint64_t t0 = global_ns();
-                while ((ld_acquire(w) & bit) == 0) {
-                    if (*abort_flag || global_ns() - t0 > budget) return false;
-                    __nanosleep(64);
-                }
-                atomicAnd(w, ~bit);                    // consumed: zero for the next call
-                fence_proxy_async_global();
-                load_rows(&hmap, (me - 1) * kD);
-                return true;
-            };
-            auto final_phase = [&]() {                 // what the boundary after the last slot reads
-                if (sch.is_suffix(n_slots - 1)) load_rows(&smap, sch.suf_lh * kD);
-                else mbar_arrive(&mb_st);
-            };
-            grid_dep_wait();
-            bool ok = load_state(0);
-            if (!ok) fail(a.status, abort_flag, 42);
-            if (ok) {
-                ok = mbar_wait_or_abort(&mb_sfree, 0, budget, abort_flag);
-                if (!ok) fail(a.status, abort_flag, 40);
-            }
-            seen = loads;                              // the chain has consumed it
-            if (ok) {
-                if (n_slots > 1) {
-                    ok = load_state(1);
-                    if (!ok) fail(a.status, abort_flag, 43);
-                } else {
-                    final_phase();
-                }
-            }
-            for (int k = 0; ok && k < n_slots; ++k) {
-                if (!mbar_wait_or_abort(&mb_sfree, (k + 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 41); break; }
-                seen = loads;
-                int lh, tb, te;
-                sch.slot(k, a.n_tiles, lh, tb, te);
-                const bool hand_over = sch.is_prefix(k);
-                const CUtensorMap* dst = hand_over ? &hmap : &smap;
-                const int row = (hand_over ? me : lh) * kD;
-#pragma unroll
-                for (int b = 0; b < 4; ++b) tma_store_2d(dst, sbuf + 4096 * b, 32 * b, row);
-                bulk_commit();
-                if (hand_over) {
-                    bulk_wait0();                      // the state is in global memory ...
-                    fence_proxy_async_global();
-                    __threadfence();
-                    atomicOr(bits_state + (me >> 5), 1u << (me & 31));   // ... before CTA i + 1 reads it
-                }
-                if (k + 2 <= n_slots) {
-                    bulk_wait_read0();                 // slot k's state has left the buffer
-                    if (k + 2 < n_slots) {
-                        if (!load_state(k + 2)) { fail(a.status, abort_flag, 43); break; }
-                    } else {
-                        final_phase();
-                    }
-                }
-            }
-            bulk_wait0();                              // every state store is complete
-            if (loads > seen) mbar_wait(&mb_st, (loads - 1) & 1, budget);   // abort: a load in flight
+            for (int b = 0; b < 2; ++b)
+                if (vp[b] >= 0) mbar_wait(&mb_vfull[b], (vp[b] >> 1) & 1, budget);
         }
         __syncwarp();
     } else if (warp >= kProdWarp0) {
-        // =========================================================== producer: operand images of
-        // the sub-tiles of parity G, and the per-sub-tile decay constants
-        const int G = (warp - kProdWarp0) & 1;
-        const bool tm_warp = warp < kProdWarp0 + 2;    // reads TMEM lanes 32 G .. 32 G + 31
-        const int gt = (tm_warp ? 0 : 32) + lane;      // thread of the group, 0..63
-        float* pw = reinterpret_cast<float*>(sm + SM_PW + G * kPwBytes);
-        float* Mm = pw + PW_M;                         // diag(beta) L of the sub-tile, rows of kMS
-        float* Nm = pw + PW_N;                         // (I + diag(beta) L)^-1
-        float* Pm = pw + PW_P;                         // 16 x 16 product of the off-diagonal block
-        float* sBeta0 = pw + PW_BETA;                  // [2][32]
-        float* sDelta0 = pw + PW_DELTA;                // [2][32]
-        float* sUC0 = pw + PW_UC;                      // [2][u, c, -, -]
-        const int bar_id = kBarProd0 + G;
+        // =========================================================== producer: the images of
+        // every tile, and its decay constants
+        const int pw = warp - kProdWarp0;              // 0..3
+        const int pt = pw * 32 + lane;                 // thread of the producer, 0..127
+        float* fws = reinterpret_cast<float*>(sm + SM_PW);
+        float* Mm = fws + PW_M;                        // diag(beta) L, rows of kMS
+        float* Nm = fws + PW_N;                        // (I + diag(beta) L)^-1 (lower part)
+        float* Pm = fws + PW_P;                        // block products
         TileCursor cc;
         cc.init(sch, a);
-        // g of tokens lane and 32 + lane of the tile, beta of this group's token lane (partner warp),
-        // loaded one tile ahead of use
-        float pg0 = 0.f, pg1 = 0.f, pb = 0.f;
+        // warp 10: g and beta of tokens lane and 32 + lane of the tile; warps 8, 9: beta of token
+        // 32 pw + lane (their rows of K K^T); loaded one tile ahead of use
+        float pg0 = 0.f, pg1 = 0.f, pb0 = 0.f, pb1 = 0.f;
         auto load_gb = [&](const TileCursor& c) {
-            const int t0 = c.jt * kTile + lane, t1 = t0 + kC, tg = G ? t1 : t0;
+            const int t0 = c.jt * kC + lane, t1 = t0 + 32;
             const size_t base = (size_t)c.l * a.T;
-            pg0 = t0 < a.T ? a.g[(base + t0) * a.Hv + c.h] : 0.f;
-            pg1 = t1 < a.T ? a.g[(base + t1) * a.Hv + c.h] : 0.f;
-            pb = tg < a.T ? a.beta[(base + tg) * a.Hv + c.h] : 0.f;
+            if (pw == 2) {
+                pg0 = t0 < a.T ? a.g[(base + t0) * a.Hv + c.h] : 0.f;
+                pg1 = t1 < a.T ? a.g[(base + t1) * a.Hv + c.h] : 0.f;
+            }
+            const int tb = (pw == 1) ? t1 : t0;
+            pb0 = tb < a.T ? a.beta[(base + tb) * a.Hv + c.h] : 0.f;
+            if (pw == 2) pb1 = t1 < a.T ? a.beta[(base + t1) * a.Hv + c.h] : 0.f;
         };
-        if (!tm_warp && NJ > 0) { grid_dep_wait(); load_gb(cc); }
+        if (pw < 3 && NJ > 0) { grid_dep_wait(); load_gb(cc); }
         float sig = 1.f;
         int prev_slot = -1;
         bool failed = false;
+        const int g = lane >> 2, tq = lane & 3;        // mma.sync fragment coordinates
         for (int J = 0; J < NJ; ++J) {
-            const int j = 2 * J + G;
-            float* sBeta = sBeta0 + 32 * (J & 1);
-            float* sDelta = sDelta0 + 32 * (J & 1);
-            float* sUC = sUC0 + 4 * (J & 1);
-            float kk[32];
-            DecayStep dmine;
-            float wn = 0.f;
-            if (!tm_warp) {
-                const float g0 = pg0, g1 = pg1, bt = pb;
-                if (J + 1 < NJ) {                       // the next tile's g, beta
-                    TileCursor nx = cc;
-                    nx.next(sch, a);
-                    load_gb(nx);
-                }
+            float* sBeta = fws + PW_BETA + 64 * (J & 1);
+            float* sDelta = fws + PW_DELTA + 64 * (J & 1);
+            float* sUC = fws + PW_UC + 4 * (J & 1);
+            DecayStep dst;
+            float wn0 = 0.f, wn1 = 0.f;
+            // this tile's g, beta (bmine: warps 8, 9 the beta of this lane's row), then the next tile's
+            const float bmine = pb0, g0 = pg0, g1 = pg1, b1 = pb1;
+            if (pw < 3 && J + 1 < NJ) {
+                TileCursor nx = cc;
+                nx.next(sch, a);
+                load_gb(nx);
+            }
+            if (pw == 2) {
+                // ---- constants of the tile's 64 tokens (lane: tokens lane and 32 + lane)
+                const float b0 = bmine;
                 if (cc.k != prev_slot) sig = 1.f;       // a slot starts from the true state
                 prev_slot = cc.k;
-                float G0 = g0, G1 = g1;                 // inclusive scans over the two sub-tiles
+                float G0 = g0, G1 = g1;                 // inclusive scans of the two halves
 #pragma unroll
                 for (int m = 1; m < 32; m <<= 1) {
                     const float y0 = __shfl_up_sync(0xffffffffu, G0, m);
                     const float y1 = __shfl_up_sync(0xffffffffu, G1, m);
                     if (lane >= m) { G0 += y0; G1 += y1; }
                 }
-                const float GC0 = __shfl_sync(0xffffffffu, G0, 31), GC1 = __shfl_sync(0xffffffffu, G1, 31);
-                const DecayStep d0 = decay_step(expf(GC0) * sig);
-                const DecayStep d1 = decay_step(expf(GC1) * d0.sig);
-                sig = d1.sig;
-                dmine = G ? d1 : d0;
-                const float Gm = G ? G1 : G0, GCm = G ? GC1 : GC0;
-                const float delta = expf(GCm - Gm);
-                sBeta[lane] = bt;
-                sDelta[lane] = delta;
-                const float ud = dmine.u * delta;
-                wn = ud >= 0x1p-60f ? 1.f / ud : 0.f;   // column t of E is u delta_t u_t
-                if (lane == 0) { sUC[0] = dmine.u; sUC[1] = dmine.c; }
-            } else {
+                G1 += __shfl_sync(0xffffffffu, G0, 31);
+                const float GC = __shfl_sync(0xffffffffu, G1, 31);
+                dst = decay_step(expf(GC) * sig);
+                sig = dst.sig;
+                const float d0 = expf(GC - G0), d1 = expf(GC - G1);
+                sBeta[lane] = b0; sBeta[32 + lane] = b1;
+                sDelta[lane] = d0; sDelta[32 + lane] = d1;
+                const float ud0 = dst.u * d0, ud1 = dst.u * d1;
+                wn0 = ud0 >= 0x1p-60f ? 1.f / ud0 : 0.f;   // column t of E is u delta_t u_t
+                wn1 = ud1 >= 0x1p-60f ? 1.f / ud1 : 0.f;
+                if (lane == 0) { sUC[0] = dst.u; sUC[1] = dst.c; }
+            } else if (pw < 2) {
+                // ---- rows 32 pw .. 32 pw + 31 of diag(beta) L from K K^T (warp 9: also the block
+                // left of the diagonal, in full)
                 const bool ok = mbar_wait_or_abort(&mb_kk, J & 1, budget, abort_flag);
                 if (!ok) { fail(a.status, abort_flag, 20); failed = true; }
                 tc_fence_after();
                 if (ok) {
-                    tmem_ld32(tm + ((uint32_t)(32 * G) << 16) + TM_KK + 32 * G, kk);
+                    const uint32_t base = tm + ((uint32_t)(32 * pw) << 16) + TM_KK;
+                    float* row = Mm + (32 * pw + lane) * kMS;
+                    float kk[32];
+                    tmem_ld32(base + 32 * pw, kk);         // the diagonal block
                     tmem_ld_wait();
+#pragma unroll
+                    for (int c4 = 0; c4 < 8; ++c4) {
+                        float4 v;
+                        v.x = (4 * c4 + 0 < lane) ? bmine * kk[4 * c4 + 0] : 0.f;
+                        v.y = (4 * c4 + 1 < lane) ? bmine * kk[4 * c4 + 1] : 0.f;
+                        v.z = (4 * c4 + 2 < lane) ? bmine * kk[4 * c4 + 2] : 0.f;
+                        v.w = (4 * c4 + 3 < lane) ? bmine * kk[4 * c4 + 3] : 0.f;
+                        *reinterpret_cast<float4*>(row + 32 * pw + 4 * c4) = v;
+                    }
+                    if (pw == 1) {                         // rows 32..63 x columns 0..31
+                        tmem_ld32(base, kk);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int c4 = 0; c4 < 8; ++c4)
+                            *reinterpret_cast<float4*>(row + 4 * c4) =
+                                make_float4(bmine * kk[4 * c4], bmine * kk[4 * c4 + 1], bmine * kk[4 * c4 + 2],
+                                            bmine * kk[4 * c4 + 3]);
+                    }
                 }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&mb_kkfree);
             }
-            if (named_sync_or(bar_id, 64, failed || *abort_flag)) break;     // (1)
-            if (tm_warp) {                              // row t of diag(beta) L: beta_t k_t.k_c, c < t
-                const float bt = sBeta[lane];
-                float* row = Mm + lane * kMS;
-#pragma unroll
-                for (int c4 = 0; c4 < 8; ++c4) {
-                    float4 v;
-                    v.x = (4 * c4 + 0 < lane) ? bt * kk[4 * c4 + 0] : 0.f;
-                    v.y = (4 * c4 + 1 < lane) ? bt * kk[4 * c4 + 1] : 0.f;
-                    v.z = (4 * c4 + 2 < lane) ? bt * kk[4 * c4 + 2] : 0.f;
-                    v.w = (4 * c4 + 3 < lane) ? bt * kk[4 * c4 + 3] : 0.f;
-                    *reinterpret_cast<float4*>(row + 4 * c4) = v;
-                }
-            }
-            if (named_sync_or(bar_id, 64, *abort_flag)) break;               // (2)
-            if (tm_warp) {
-                // the two 16 x 16 diagonal blocks of N by forward substitution, one column per lane
-                const int b = lane >> 4, jc = lane & 15, o = 16 * b;
+            if (named_sync_or(kBarProd, kProd, failed || *abort_flag)) break;        // (1)
+            if (pw < 2) {
+                // the four 16 x 16 diagonal blocks of N by forward substitution, one column per lane;
+                // the next row's coefficients are loaded while the current row is formed
+                const int o = 32 * pw + 16 * (lane >> 4), jc = lane & 15;
                 float x[16];
 #pragma unroll
                 for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
+                float4 cur[4], nxt[4];
+                cur[0] = *reinterpret_cast<const float4*>(Mm + (o + 1) * kMS + o);
 #pragma unroll
                 for (int rr = 1; rr < 16; ++rr) {
-                    const float* mr = Mm + (o + rr) * kMS + o;
-                    float s0 = 0.f, s1 = 0.f;
+                    if (rr + 1 < 16) {
 #pragma unroll
-                    for (int c = 0; c < rr; c += 4) {
-                        const float4 v = *reinterpret_cast<const float4*>(mr + c);
-                        s0 = fmaf(v.x, x[c], s0);
-                        if (c + 1 < rr) s1 = fmaf(v.y, x[c + 1], s1);
-                        if (c + 2 < rr) s0 = fmaf(v.z, x[c + 2], s0);
-                        if (c + 3 < rr) s1 = fmaf(v.w, x[c + 3], s1);
+                        for (int c4 = 0; c4 < 4; ++c4)
+                            if (4 * c4 < rr + 1) nxt[c4] = *reinterpret_cast<const float4*>(Mm + (o + rr + 1) * kMS + o + 4 * c4);
                     }
-                    if (rr > jc) x[rr] = -(s0 + s1);
+                    float s[4] = {0.f, 0.f, 0.f, 0.f};     // four short FMA chains
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        const int c = 4 * c4;
+                        if (c < rr) {
+                            s[0] = fmaf(cur[c4].x, x[c], s[0]);
+                            if (c + 1 < rr) s[1] = fmaf(cur[c4].y, x[c + 1], s[1]);
+                            if (c + 2 < rr) s[2] = fmaf(cur[c4].z, x[c + 2], s[2]);
+                            if (c + 3 < rr) s[3] = fmaf(cur[c4].w, x[c + 3], s[3]);
+                        }
+                    }
+                    if (rr > jc) x[rr] = -((s[0] + s[1]) + (s[2] + s[3]));
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) cur[c4] = nxt[c4];
                 }
 #pragma unroll
                 for (int rr = 0; rr < 16; ++rr) Nm[(o + rr) * kMS + o + jc] = x[rr];
-                if (b == 0) {
+                if ((lane >> 4) == 0) {
 #pragma unroll
-                    for (int rr = 0; rr < 16; ++rr) Nm[rr * kMS + 16 + jc] = 0.f;   // upper block
+                    for (int rr = 0; rr < 16; ++rr) Nm[(o + rr) * kMS + o + 16 + jc] = 0.f;   // block above
                 }
             }
-            if (named_sync_or(bar_id, 64, *abort_flag)) break;               // (3)
-            {   // P = M10 N00, then N10 = -N11 P (16 x 16 blocks; 4 outputs per thread)
-                const int r = gt >> 2, c0 = 4 * (gt & 3);
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                const float* mrow = Mm + (16 + r) * kMS;
-#pragma unroll
-                for (int a4 = 0; a4 < 16; a4 += 4) {
-                    const float4 mv = *reinterpret_cast<const float4*>(mrow + a4);
-                    const float m4[4] = {mv.x, mv.y, mv.z, mv.w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float4 nv = *reinterpret_cast<const float4*>(Nm + (a4 + e) * kMS + c0);
-                        acc.x = fmaf(m4[e], nv.x, acc.x); acc.y = fmaf(m4[e], nv.y, acc.y);
-                        acc.z = fmaf(m4[e], nv.z, acc.z); acc.w = fmaf(m4[e], nv.w, acc.w);
-                    }
-                }
-                *reinterpret_cast<float4*>(Pm + r * kPS + c0) = acc;
-                if (named_sync_or(bar_id, 64, *abort_flag)) break;           // (4)
-                acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                const float* nrow = Nm + (16 + r) * kMS + 16;
-#pragma unroll
-                for (int a4 = 0; a4 < 16; a4 += 4) {
-                    const float4 nv = *reinterpret_cast<const float4*>(nrow + a4);
-                    const float n4[4] = {nv.x, nv.y, nv.z, nv.w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float4 pv = *reinterpret_cast<const float4*>(Pm + (a4 + e) * kPS + c0);
-                        acc.x = fmaf(n4[e], pv.x, acc.x); acc.y = fmaf(n4[e], pv.y, acc.y);
-                        acc.z = fmaf(n4[e], pv.z, acc.z); acc.w = fmaf(n4[e], pv.w, acc.w);
-                    }
-                }
-                *reinterpret_cast<float4*>(Nm + (16 + r) * kMS + c0) = make_float4(-acc.x, -acc.y, -acc.z, -acc.w);
+            if (named_sync_or(kBarProd, kProd, *abort_flag)) break;                  // (2)
+            {   // 16 -> 32, warp (p, nh): in 32-block p, columns 8 nh .. of
+                //   P = M[16..32][0..16] N[0..16][0..16],  then  N[16..32][0..16] = -N[16..32][16..32] P
+                // (tensor-core fragments, three-term bfloat16 products)
+                const int p = pw >> 1, nh = pw & 1, o = 32 * p;
+                float d[4] = {0.f, 0.f, 0.f, 0.f};
+                mma_f32_split<1>(d, Mm + (o + 16) * kMS + o, kMS, Nm + o * kMS + o + 8 * nh, kMS, g, tq);
+                float* pp = Pm + 16 * p * kPS + 8 * nh;
+                *reinterpret_cast<float2*>(pp + g * kPS + 2 * tq) = make_float2(d[0], d[1]);
+                *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 2 * tq) = make_float2(d[2], d[3]);
+                __syncwarp();
+                float e[4] = {0.f, 0.f, 0.f, 0.f};
+                mma_f32_split<1>(e, Nm + (o + 16) * kMS + o + 16, kMS, pp, kPS, g, tq);
+                float* np = Nm + (o + 16) * kMS + o + 8 * nh;
+                *reinterpret_cast<float2*>(np + g * kMS + 2 * tq) = make_float2(-e[0], -e[1]);
+                *reinterpret_cast<float2*>(np + (g + 8) * kMS + 2 * tq) = make_float2(-e[2], -e[3]);
             }
-            if (named_sync_or(bar_id, 64, *abort_flag)) break;               // (5)
-            // the image slot is free once sub-tile j - 4's products and the chain have read it
-            if (j >= 4) {
-                const bool ok = mbar_wait_or_abort(&mb_iempty[j & 3], ((j >> 2) - 1) & 1, budget, abort_flag);
+            if (named_sync_or(kBarProd, kProd, *abort_flag)) break;                  // (3)
+            {   // 32 -> 64, warp (mt, nh): rows 16 mt .., columns 16 nh .. of
+                //   P = M[32..64][0..32] N[0..32][0..32],  then  N[32..64][0..32] = -N[32..64][32..64] P
+                const int mt = pw >> 1, nh = pw & 1;
+                float d0[4] = {0.f, 0.f, 0.f, 0.f}, d1[4] = {0.f, 0.f, 0.f, 0.f};
+                mma_f32_split<2>(d0, Mm + (32 + 16 * mt) * kMS, kMS, Nm + 16 * nh, kMS, g, tq);
+                mma_f32_split<2>(d1, Mm + (32 + 16 * mt) * kMS, kMS, Nm + 16 * nh + 8, kMS, g, tq);
+                float* pp = Pm + 16 * mt * kPS + 16 * nh;
+                *reinterpret_cast<float2*>(pp + g * kPS + 2 * tq) = make_float2(d0[0], d0[1]);
+                *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 2 * tq) = make_float2(d0[2], d0[3]);
+                *reinterpret_cast<float2*>(pp + g * kPS + 8 + 2 * tq) = make_float2(d1[0], d1[1]);
+                *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 8 + 2 * tq) = make_float2(d1[2], d1[3]);
+                if (named_sync_or(kBarProd, kProd, *abort_flag)) break;              // (4)
+                float e0[4] = {0.f, 0.f, 0.f, 0.f}, e1[4] = {0.f, 0.f, 0.f, 0.f};
+                mma_f32_split<2>(e0, Nm + (32 + 16 * mt) * kMS + 32, kMS, Pm + 16 * nh, kPS, g, tq);
+                mma_f32_split<2>(e1, Nm + (32 + 16 * mt) * kMS + 32, kMS, Pm + 16 * nh + 8, kPS, g, tq);
+                float* np = Nm + (32 + 16 * mt) * kMS + 16 * nh;
+                *reinterpret_cast<float2*>(np + g * kMS + 2 * tq) = make_float2(-e0[0], -e0[1]);
+                *reinterpret_cast<float2*>(np + (g + 8) * kMS + 2 * tq) = make_float2(-e0[2], -e0[3]);
+                *reinterpret_cast<float2*>(np + g * kMS + 8 + 2 * tq) = make_float2(-e1[0], -e1[1]);
+                *reinterpret_cast<float2*>(np + (g + 8) * kMS + 8 + 2 * tq) = make_float2(-e1[2], -e1[3]);
+            }
+            // the image slot is free once tile J - 2's products and the chain have read it
+            if (J >= 2) {
+                const bool ok = mbar_wait_or_abort(&mb_iempty[J & 1], ((J >> 1) - 1) & 1, budget, abort_flag);
                 if (!ok) { fail(a.status, abort_flag, 21); failed = true; }
             }
-            if (named_sync_or(bar_id, 64, failed || *abort_flag)) break;     // (6)
-            {   // images: row t = gt / 2, columns 16 hc .. 16 hc + 15 of N_beta = N diag(beta)
-                const int t = gt >> 1, hc = gt & 1;
-                const float u = sUC[0], cX = sUC[1];
-                uint8_t* slot = sm + SM_IMG + (j & 3) * kImgSlot;
-                float nb[16], w1[16];
+            if (named_sync_or(kBarProd, kProd, failed || *abort_flag)) break;        // (5)
+            {   // images: row t = pt / 2, columns 32 hh .. 32 hh + 31 of N_beta = N diag(beta) (zero
+                // above the diagonal)
+                const int t = pt >> 1, hh = pt & 1;
+                const float u = sUC[0];
+                uint8_t* b1 = sm + SM_B1 + (J & 1) * 16384;
+                uint8_t* b3 = sm + SM_B3 + (J & 1) * 16384;
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float4 nv = *reinterpret_cast<const float4*>(Nm + t * kMS + 16 * hc + 4 * e);
-                    const float4 bv = *reinterpret_cast<const float4*>(sBeta + 16 * hc + 4 * e);
-                    const float4 dv = *reinterpret_cast<const float4*>(sDelta + 16 * hc + 4 * e);
-                    nb[4 * e] = nv.x * bv.x; nb[4 * e + 1] = nv.y * bv.y;
-                    nb[4 * e + 2] = nv.z * bv.z; nb[4 * e + 3] = nv.w * bv.w;
-                    w1[4 * e] = u * nb[4 * e] * dv.x; w1[4 * e + 1] = u * nb[4 * e + 1] * dv.y;
-                    w1[4 * e + 2] = u * nb[4 * e + 2] * dv.z; w1[4 * e + 3] = u * nb[4 * e + 3] * dv.w;
-                }
+                for (int g8 = 0; g8 < 4; ++g8) {        // 8 columns (one 16-byte chunk of bf16) at a time
+                    const int c = 32 * hh + 8 * g8;
+                    const float4 n0 = *reinterpret_cast<const float4*>(Nm + t * kMS + c);
+                    const float4 n1 = *reinterpret_cast<const float4*>(Nm + t * kMS + c + 4);
+                    const float4 bv0 = *reinterpret_cast<const float4*>(sBeta + c);
+                    const float4 bv1 = *reinterpret_cast<const float4*>(sBeta + c + 4);
+                    const float4 dv0 = *reinterpret_cast<const float4*>(sDelta + c);
+                    const float4 dv1 = *reinterpret_cast<const float4*>(sDelta + c + 4);
+                    const float nv[8] = {n0.x, n0.y, n0.z, n0.w, n1.x, n1.y, n1.z, n1.w};
+                    const float bv[8] = {bv0.x, bv0.y, bv0.z, bv0.w, bv1.x, bv1.y, bv1.z, bv1.w};
+                    const float dv[8] = {dv0.x, dv0.y, dv0.z, dv0.w, dv1.x, dv1.y, dv1.z, dv1.w};
+                    float nb[8], w1[8];
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {          // B2 = -c N_beta, tf32, row t chunks 4 hc + e
-                    const uint4 w = make_uint4(to_tf32(-cX * nb[4 * e]), to_tf32(-cX * nb[4 * e + 1]),
-                                               to_tf32(-cX * nb[4 * e + 2]), to_tf32(-cX * nb[4 * e + 3]));
-                    *reinterpret_cast<uint4*>(slot + 8192 + sw128_offset(t, 4 * hc + e)) = w;
-                }
+                    for (int i = 0; i < 8; ++i) {
+                        nb[i] = (c + i <= t) ? nv[i] * bv[i] : 0.f;
+                        w1[i] = u * nb[i] * dv[i];
+                    }
+                    uint32_t h3[4], l3[4], h1[4], l1[4];
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {          // B1 = u N_beta diag(delta), (hi, lo)
-                    uint32_t h[4], l[4];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) split2(w1[8 * e + 2 * i], w1[8 * e + 2 * i + 1], h[i], l[i]);
-                    *reinterpret_cast<uint4*>(slot + sw128_offset(t, 2 * hc + e)) = make_uint4(h[0], h[1], h[2], h[3]);
-                    *reinterpret_cast<uint4*>(slot + 4096 + sw128_offset(t, 2 * hc + e)) = make_uint4(l[0], l[1], l[2], l[3]);
+                    for (int i = 0; i < 4; ++i) {
+                        split2(nb[2 * i], nb[2 * i + 1], h3[i], l3[i]);
+                        split2(w1[2 * i], w1[2 * i + 1], h1[i], l1[i]);
+                    }
+                    const uint32_t off = sw128_offset(t, c >> 3);
+                    *reinterpret_cast<uint4*>(b3 + off) = make_uint4(h3[0], h3[1], h3[2], h3[3]);
+                    *reinterpret_cast<uint4*>(b3 + 8192 + off) = make_uint4(l3[0], l3[1], l3[2], l3[3]);
+                    *reinterpret_cast<uint4*>(b1 + off) = make_uint4(h1[0], h1[1], h1[2], h1[3]);
+                    *reinterpret_cast<uint4*>(b1 + 8192 + off) = make_uint4(l1[0], l1[1], l1[2], l1[3]);
                 }
             }
-            if (!tm_warp) {                             // the chain's and the MMA's constants
-                float* cs = const_cast<float*>(cst) + (j & 3) * kConstWords;
-                cs[lane] = wn;
+            if (pw == 2) {                              // the chain's and the MMA's constants
+                float* cs = cst + (J & 1) * kConstWords;
+                cs[lane] = wn0;
+                cs[32 + lane] = wn1;
                 if (lane == 0) {
-                    cs[32] = dmine.sig;
-                    cs[33] = dmine.pass;
-                    reinterpret_cast<int*>(cs)[34] = dmine.shift;
+                    cs[64] = dst.sig;
+                    cs[65] = dst.pass;
+                    reinterpret_cast<int*>(cs)[66] = dst.shift;
+                    cs[67] = dst.c;
                 }
             }
             fence_async_smem();                         // generic writes -> the tensor core's reads
             __syncwarp();
-            if (lane == 0) mbar_arrive(&mb_ifull[j & 3]);
+            if (lane == 0) mbar_arrive(&mb_ifull[J & 1]);
             cc.next(sch, a);
         }
     } else {
@@ -841,45 +812,72 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         const int q = warp & 3, hh = warp >> 2;          // TMEM lane quadrant, column half
         const int r = 32 * q + lane;                     // row of S (value index)
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-        float* sbuf = reinterpret_cast<float*>(sm + SM_SB);   // swizzled rows, see sb_idx
-        int st_seen = 0;                                 // mb_st phases waited for (uniform)
         TileCursor cc;
         cc.init(sch, a);
-        // K of sub-tile jj (TMA tile, rows 32 (jj & 1) ..) in fp32 (exact, and exact in tf32) into
-        // the B operand buffer of X.  Called between MMA_X(jj-1), the last reader of the buffer, and
-        // the ready signal of sub-tile jj.
-        auto make_k32 = [&](int jj) -> bool {
-            const int bk = (jj >> 1) % 3;
-            const bool ok = mbar_wait_or_abort(&mb_kfull[bk], ((jj >> 1) / 3) & 1, budget, abort_flag);
-            const uint8_t* kb = sm + SM_K + bk * 16384;
-            const int r0 = 32 * (jj & 1);
+        // W(jj) = -c Q^T in tf32: this thread's d_k row c = r of Q, tokens 32 hh .. 32 hh + 31, into
+        // rows t of the K-major W (column block q, its 4-byte slot of row t).  Q(jj) is complete and
+        // W's last reader, E(jj-1) += S~ W(jj-1), has completed.
+        auto make_w = [&](int jj) -> bool {
+            bool ok = mbar_wait_or_abort(&mb_q, jj & 1, budget, abort_flag);
+            ok = mbar_wait_or_abort(&mb_ifull[jj & 1], (jj >> 1) & 1, budget, abort_flag) && ok;
+            tc_fence_after();
+            const float cneg = -cst[(jj & 1) * kConstWords + 67];
+            float qv[32];
+            tmem_ld32(tm + lane_off + TM_Q + 32 * hh, qv);
+            tmem_ld_wait();
+            uint8_t* wb = sm + SM_W + q * 8192 + (lane & 3) * 4;
+            const int chunk = lane >> 2;
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {                  // 32 rows x 16 chunks of 8 bf16
-                const int e = tid + kChain * u;
-                const int t = e >> 4, c16 = e & 15, cb = c16 >> 3, c = c16 & 7;
-                const uint4 w = *reinterpret_cast<const uint4*>(kb + cb * 8192 + sw128_offset(r0 + t, c));
-                const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
-                uint32_t f[8];
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    f[2 * i] = wv[i] << 16;
-                    f[2 * i + 1] = wv[i] & 0xFFFF0000u;
-                }
-                // dims 64 cb + 8 c .. + 7: fp32 block 2 cb + c / 4, chunks 2 (c % 4) and 2 (c % 4) + 1
-                uint8_t* rowp = sm + SM_K32 + (2 * cb + (c >> 2)) * 4096;
-                const int q0 = 2 * (c & 3);
-                *reinterpret_cast<uint4*>(rowp + sw128_offset(t, q0)) = make_uint4(f[0], f[1], f[2], f[3]);
-                *reinterpret_cast<uint4*>(rowp + sw128_offset(t, q0 + 1)) = make_uint4(f[4], f[5], f[6], f[7]);
+            for (int i = 0; i < 32; ++i) {
+                const int t = 32 * hh + i;
+                *reinterpret_cast<uint32_t*>(wb + sw128_offset(t, chunk)) = to_tf32(cneg * qv[i]);
             }
-            fence_async_smem();                            // generic writes -> the tensor core's reads
+            fence_async_smem();
+            tc_fence_before();
+            return ok;
+        };
+        // a slot's starting state (from the state or hand-over entry i - 1) into TMEM as S~ and
+        // S_before; `den` gets this thread's sum of squares
+        auto install = [&](int slot, float& den) -> bool {
+            int lh, tb, te;
+            sch.slot(slot, a.n_tiles, lh, tb, te);
+            const bool from_ho = sch.is_suffix(slot);
+            bool ok = true;
+            if (from_ho) {                               // one thread waits for CTA i - 1's state
+                if (tid == 0) {
+                    const uint32_t bit = 1u << ((me - 1) & 31);
+                    uint32_t* w = bits_state + ((me - 1) >> 5);
+                    const uint64_t t0 = global_ns();
+                    while ((ld_acquire(w) & bit) == 0) {
+                        if (*abort_flag || global_ns() - t0 > budget) { fail(a.status, abort_flag, 42); break; }
+                        __nanosleep(64);
+                    }
+                    atomicAnd(w, ~bit);                  // consumed: zero for the next call
+                }
+                ok = !named_sync_or(kBarChain, kChain, *abort_flag);
+            }
+            const float* src = (from_ho ? a.ho_state + (size_t)(me - 1) * kD * kD : a.state + (size_t)lh * kD * kD)
+                               + (size_t)r * kD + 64 * hh;
+            den = 0.f;
+            if (ok) {
+#pragma unroll
+                for (int g4 = 0; g4 < 4; ++g4) {
+                    float v[16];
+                    ld16_global(src + 16 * g4, v, from_ho);
+                    uint32_t u32[16];
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) { den = fmaf(v[e], v[e], den); u32[e] = __float_as_uint(v[e]); }
+                    tmem_st16(tm + lane_off + TM_S + 64 * hh + 16 * g4, u32);
+                    tmem_st16(tm + lane_off + TM_SB + 64 * hh + 16 * g4, u32);
+                }
+            }
             return ok;
         };
         float den = 0.f, sig = 1.f;
         // Write sizes (optional): column t of E is u delta_t u_t, u_t = beta_t (v_t - alpha_t S_{t-1}
         // k_t) the token's write.  The pass sums each column's squares over the warp's 32 rows,
         // rescales them by the constant (1 / (u delta_t))^2 and adds them into s_u2 (four warps per
-        // column); at the next sub-tile warp 0 takes the square roots and sums them into the head's
-        // total.
+        // column); at the next tile warp 0 takes the square roots and sums them into the head's total.
         const bool want_w = a.wnorm != nullptr;
         float wacc = 0.f;                                  // warp 0: the slot's running sum
         int prev_lh = -1, prev_slot = -1;
@@ -902,232 +900,178 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                     if (*abort_flag || global_ns() - t0 > budget) return false;
                     __nanosleep(64);
                 }
-                sum += *reinterpret_cast<volatile const float*>(a.ho_wsum + me - 1);
+                sum += __ldcg(a.ho_wsum + me - 1);
                 atomicAnd(w, ~bit);
             }
             a.wnorm[lh] = sum;
             return true;
         };
-        auto fold_writes = [&](int jj) {                   // warp 0: sub-tile jj's sizes into wacc
+        auto fold_writes = [&](int jj) {                   // warp 0: tile jj's sizes into wacc
             float* b = s_u2[jj & 1];
-            float sacc = sqrtf(b[lane]);
+            float sacc = sqrtf(b[lane]) + sqrtf(b[32 + lane]);
             b[lane] = 0.f;
+            b[32 + lane] = 0.f;
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, m);
             wacc += sacc;
         };
-        bool stop = false;
-        for (int J = 0; J < NJ && !stop; ++J) {
-            for (int u = 0; u < 2; ++u) {
-                const int j = 2 * J + u;
-                const int lh = cc.lh, slot = cc.k;
-                const bool last = u == 1 && cc.jt == cc.te - 1;   // the slot's last sub-tile
-                if (named_sync_or(kBarChain, kChain, *abort_flag)) { stop = true; break; }
-                if (want_w && j > 0 && warp == 0) {
-                    fold_writes(j - 1);
-                    if (prev_last) {
-                        if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 44);
-                        wacc = 0.f;
-                    }
+        bool stop = NJ == 0;
+        if (!stop) {
+            // ---- the CTA's first slot: its state into TMEM, and W of its first tile
+            bool ok = install(0, den);
+            ok = make_w(0) && ok;
+            tmem_st_wait();
+            tc_fence_before();
+            if (!ok) fail(a.status, abort_flag, 14);
+            warp_arrive(&mb_ready, lane);
+        }
+        for (int j = 0; j < NJ && !stop; ++j) {
+            const int lh = cc.lh, slot = cc.k;
+            const bool last = cc.jt == cc.te - 1;          // the slot's last tile
+            if (named_sync_or(kBarChain, kChain, *abort_flag)) break;
+            if (want_w && j > 0 && warp == 0) {
+                fold_writes(j - 1);
+                if (prev_last) {
+                    if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 44);
+                    wacc = 0.f;
                 }
-                if (j == 0) {
-                    // ---- the CTA's first slot: its state from the staging buffer into TMEM, as S~
-                    // (sig = 1) and as S_before, and sum S_before^2
-                    if (!mbar_wait_or_abort(&mb_st, 0, budget, abort_flag)) fail(a.status, abort_flag, 14);
-                    st_seen = 1;
+            }
+            // ---- E(j) is complete (and E += S~ W has read the state and W)
+            if (!mbar_wait_or_abort(&mb_u, j & 1, budget, abort_flag)) fail(a.status, abort_flag, 10);
+            tc_fence_after();
+            const float* cs = cst + (j & 1) * kConstWords;
+            const float pass_f = cs[65];
+            const float sig_after = cs[64];
+            const float wf = cs[32 * hh + lane];
+            if (pass_f >= 0.f) {
+                // the decay would take the deferred scale out of range: S~ <- p S~ (the state
+                // update of this tile has not been issued: it waits for this pass)
+#pragma unroll 1
+                for (int g4 = 0; g4 < 4; ++g4) {
+                    float sv[16];
+                    tmem_ld16(tm + lane_off + TM_S + 64 * hh + 16 * g4, sv);
+                    tmem_ld_wait();
+                    uint32_t su[16];
 #pragma unroll
-                    for (int g4 = 0; g4 < 4; ++g4) {
-                        uint32_t sv[16];
+                    for (int e = 0; e < 16; ++e) su[e] = __float_as_uint(sv[e] * pass_f);
+                    tmem_st16(tm + lane_off + TM_S + 64 * hh + 16 * g4, su);
+                }
+            }
+            {   // ---- pass: this thread's 32 token columns of E -> (hi, lo) A operand, in place
+                const uint32_t eb = tm + lane_off + TM_E + (j & 1) * 64 + 32 * hh;
+                float e[32];
+                tmem_ld32(eb, e);
+                tmem_ld_wait();
+                if (want_w) {
+                    // squares summed over the warp's 32 rows, column by column: halving exchanges
+                    // leave lane c with column c
+                    float x[32];
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, 16 * hh + 4 * g4 + e));
-                            den = fmaf(x.x, x.x, den); den = fmaf(x.y, x.y, den);
-                            den = fmaf(x.z, x.z, den); den = fmaf(x.w, x.w, den);
-                            sv[4 * e] = __float_as_uint(x.x); sv[4 * e + 1] = __float_as_uint(x.y);
-                            sv[4 * e + 2] = __float_as_uint(x.z); sv[4 * e + 3] = __float_as_uint(x.w);
+                    for (int i = 0; i < 32; ++i) x[i] = e[i] * e[i];
+#pragma unroll
+                    for (int w = 16; w >= 1; w >>= 1) {
+                        const bool up = (lane & w) != 0;
+#pragma unroll
+                        for (int i = 0; i < w; ++i) {
+                            const float send = up ? x[i] : x[i + w];
+                            x[i] = (up ? x[i + w] : x[i]) + __shfl_xor_sync(0xffffffffu, send, w);
                         }
-                        tmem_st16(tm + lane_off + TM_S + 64 * hh + 16 * g4, sv);
-                        tmem_st16(tm + lane_off + TM_SB + 64 * hh + 16 * g4, sv);
                     }
-                    warp_arrive(&mb_sfree, lane);                    // the staging buffer has been read
-                    if (!make_k32(0)) fail(a.status, abort_flag, 16);
-                    tmem_st_wait();
-                    tc_fence_before();
-                    warp_arrive(&mb_sready, lane);
+                    atomicAdd(&s_u2[j & 1][32 * hh + lane], x[0] * wf * wf);
                 }
-                // ---- E(j) is complete (and MMA_X(j) has read the state and K in fp32)
-                if (!mbar_wait_or_abort(&mb_u, j & 1, budget, abort_flag)) fail(a.status, abort_flag, 10);
-                if (!mbar_wait_or_abort(&mb_ifull[j & 3], (j >> 2) & 1, budget, abort_flag)) fail(a.status, abort_flag, 11);
+                uint32_t hi[16], lo[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) split2(e[2 * i], e[2 * i + 1], hi[i], lo[i]);
+                tmem_st16(eb, hi);
+                tmem_st16(eb + 16, lo);
+                tmem_st_wait();
+            }
+            tc_fence_before();
+            warp_arrive(&mb_uready, lane);
+            warp_arrive(&mb_iempty[j & 1], lane);          // the tile's constants are read
+            sig = sig_after;
+            // ---- while the state update runs: W of the next tile
+            const bool has_next = j + 1 < NJ;
+            bool ok = true;
+            if (has_next) ok = make_w(j + 1);
+            if (!ok) fail(a.status, abort_flag, 15);
+            if (last) {
+                // ---- slot boundary: S_after = sig S~ out, drift partials against S_before, the next
+                // slot's state in
+                const bool prefix = sch.is_prefix(slot);
+                const bool shared_end = sch.is_suffix(slot);   // S_before: the head's stored state
+                if (!mbar_wait_or_abort(&mb_s, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 12); ok = false; }
                 tc_fence_after();
-                const float* cs = cst + (j & 3) * kConstWords;
-                const float pass_f = cs[33];
-                const float sig_after = cs[32];
-                float wf[16];
+                float num = 0.f, den_end = 0.f;
+                float* dstp = (prefix ? a.ho_state + (size_t)me * kD * kD : a.state + (size_t)lh * kD * kD)
+                              + (size_t)r * kD + 64 * hh;
+                const float* sbp = a.state + (size_t)lh * kD * kD + (size_t)r * kD + 64 * hh;
+                if (ok) {
+#pragma unroll 1
+                    for (int g4 = 0; g4 < 4; ++g4) {
+                        float sa[16], sb[16];
+                        tmem_ld16(tm + lane_off + TM_S + 64 * hh + 16 * g4, sa);
+                        if (shared_end) {
+                            ld16_global(sbp + 16 * g4, sb, true);
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float4 w4 = *reinterpret_cast<const float4*>(cs + 16 * hh + 4 * e);
-                    wf[4 * e] = w4.x; wf[4 * e + 1] = w4.y; wf[4 * e + 2] = w4.z; wf[4 * e + 3] = w4.w;
-                }
-                if (pass_f >= 0.f) {
-                    // the decay would take the deferred scale out of range: S~ <- p S~ (MMA_S(j) has not
-                    // been issued: it waits for this pass)
-#pragma unroll
-                    for (int g2 = 0; g2 < 2; ++g2) {
-                        float sv[32];
-                        tmem_ld32(tm + lane_off + TM_S + 64 * hh + 32 * g2, sv);
+                            for (int e = 0; e < 16; ++e) den_end = fmaf(sb[e], sb[e], den_end);
+                        } else {
+                            tmem_ld16(tm + lane_off + TM_SB + 64 * hh + 16 * g4, sb);
+                        }
                         tmem_ld_wait();
 #pragma unroll
-                        for (int e = 0; e < 32; ++e) sv[e] *= pass_f;
-                        tmem_st32(tm + lane_off + TM_S + 64 * hh + 32 * g2, sv);
+                        for (int e = 0; e < 16; ++e) {
+                            sa[e] *= sig;
+                            const float d = sa[e] - sb[e];
+                            num = fmaf(d, d, num);
+                        }
+                        float4* o4 = reinterpret_cast<float4*>(dstp + 16 * g4);
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) o4[e] = make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
                     }
                 }
-                {   // ---- pass: E = hi-half product + lo-half product (+ the X term), over this
-                    // thread's 16 token columns, split into the packed (hi, lo) A operand of MMA_S
-                    const uint32_t eb = tm + lane_off + TM_E + (j & 1) * 64 + 16 * hh;
-                    float e0[16], e1[16];
-                    tmem_ld16(eb, e0);
-                    tmem_ld16(eb + 32, e1);
-                    tmem_ld_wait();
+                // partial sums: pairwise in fp32, over the warp's lanes and then over the warps
+                float fn = num, fd = shared_end ? den_end : den;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) e0[i] += e1[i];
-                    if (want_w) {
-                        // squares summed over the warp's 32 rows, column by column: halving exchanges
-                        // leave lanes 2c and 2c + 1 with column c of the 16
-                        float x[16];
+                for (int m = 16; m >= 1; m >>= 1) {
+                    fn += __shfl_xor_sync(0xffffffffu, fn, m);
+                    fd += __shfl_xor_sync(0xffffffffu, fd, m);
+                }
+                if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
+                if (prefix) __threadfence();                  // the hand-over state is in memory ...
+                if (named_sync_or(kBarChain, kChain, !ok || *abort_flag)) { stop = true; break; }
+                if (prefix && tid == 0) atomicOr(bits_state + (me >> 5), 1u << (me & 31));   // ... before CTA i + 1 reads it
+                if (warp == 0 && a.partials != nullptr && !prefix) {   // a shared head: at its end
+                    float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
+                    float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) x[i] = e0[i] * e0[i];
-#pragma unroll
-                        for (int w = 8, bit = 16; w >= 1; w >>= 1, bit >>= 1) {
-                            const bool up = (lane & bit) != 0;
-#pragma unroll
-                            for (int i = 0; i < w; ++i) {
-                                const float send = up ? x[i] : x[i + w];
-                                x[i] = (up ? x[i + w] : x[i]) + __shfl_xor_sync(0xffffffffu, send, bit);
-                            }
-                        }
-                        x[0] += __shfl_xor_sync(0xffffffffu, x[0], 1);
-                        const int c = lane >> 1;
-                        float f = wf[0];
-#pragma unroll
-                        for (int i = 1; i < 16; ++i) f = (c == i) ? wf[i] : f;
-                        if ((lane & 1) == 0) atomicAdd(&s_u2[j & 1][16 * hh + c], x[0] * f * f);
+                    for (int m = kChainWarps / 2; m >= 1; m >>= 1) {
+                        pn += __shfl_xor_sync(0xffffffffu, pn, m);
+                        pd += __shfl_xor_sync(0xffffffffu, pd, m);
                     }
-                    uint32_t hi[8], lo[8];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) split2(e0[2 * i], e0[2 * i + 1], hi[i], lo[i]);
-                    tmem_st8(tm + lane_off + TM_AP + 8 * hh, hi);
-                    tmem_st8(tm + lane_off + TM_AP + 16 + 8 * hh, lo);
+                    if (lane == 0) {
+                        a.partials[(size_t)lh * 2 + 0] = pn;
+                        a.partials[(size_t)lh * 2 + 1] = pd;
+                    }
+                }
+                if (has_next) {
+                    if (!install(slot + 1, den)) fail(a.status, abort_flag, 16);
                     tmem_st_wait();
                 }
-                tc_fence_before();
-                warp_arrive(&mb_uready, lane);
-                warp_arrive(&mb_iempty[j & 3], lane);            // images and constants read
-                sig = sig_after;
-                // ---- while MMA_S(j) runs: the next sub-tile's K in fp32
-                if (j + 1 < NS && !make_k32(j + 1)) fail(a.status, abort_flag, 16);
-                if (!last) {
-                    if (j + 1 < NS) warp_arrive(&mb_sready, lane);
-                } else {
-                    // ---- slot boundary: S_after = sig S~ out through the staging buffer, the next
-                    // slot's state (staged meanwhile) into TMEM, drift partials against S_before
-                    const bool has_next = j + 1 < NS;             // uniform
-                    // a last slot that ends a head begun by CTA i - 1: S_before is not in TMEM (the
-                    // slot started from the handed-over state) but staged, and its square sum is
-                    // taken here
-                    const bool shared_end = sch.is_suffix(slot);
-                    float den_end = 0.f;
-                    bool ok = mbar_wait_or_abort(&mb_s, j & 1, budget, abort_flag);
-                    if (!ok) fail(a.status, abort_flag, 12);
-                    if (!mbar_wait_or_abort(&mb_st, st_seen & 1, budget, abort_flag)) {
-                        fail(a.status, abort_flag, 14);
-                        ok = false;
-                    }
-                    ++st_seen;
-                    tc_fence_after();
-                    float num = 0.f, den_next = 0.f;
-                    if (ok) {
-#pragma unroll 1
-                        for (int g4 = 0; g4 < 4; ++g4) {
-                            const uint32_t col = 64 * hh + 16 * g4;
-                            const int ch = 16 * hh + 4 * g4;      // this group's 16-byte chunks of row r
-                            float sa[16], sb[16];
-                            tmem_ld16(tm + lane_off + TM_S + col, sa);
-                            if (shared_end) {
-#pragma unroll
-                                for (int e = 0; e < 4; ++e) {
-                                    const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
-                                    sb[4 * e] = x.x; sb[4 * e + 1] = x.y; sb[4 * e + 2] = x.z; sb[4 * e + 3] = x.w;
-                                }
-#pragma unroll
-                                for (int e = 0; e < 16; ++e) den_end = fmaf(sb[e], sb[e], den_end);
-                            } else {
-                                tmem_ld16(tm + lane_off + TM_SB + col, sb);
-                            }
-                            tmem_ld_wait();
-#pragma unroll
-                            for (int e = 0; e < 16; ++e) {
-                                sa[e] *= sig;
-                                const float d = sa[e] - sb[e];
-                                num = fmaf(d, d, num);
-                            }
-                            if (has_next) {
-                                uint32_t sn[16];
-#pragma unroll
-                                for (int e = 0; e < 4; ++e) {
-                                    const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
-                                    den_next = fmaf(x.x, x.x, den_next); den_next = fmaf(x.y, x.y, den_next);
-                                    den_next = fmaf(x.z, x.z, den_next); den_next = fmaf(x.w, x.w, den_next);
-                                    sn[4 * e] = __float_as_uint(x.x); sn[4 * e + 1] = __float_as_uint(x.y);
-                                    sn[4 * e + 2] = __float_as_uint(x.z); sn[4 * e + 3] = __float_as_uint(x.w);
-                                }
-                                tmem_st16(tm + lane_off + TM_S + col, sn);
-                                tmem_st16(tm + lane_off + TM_SB + col, sn);
-                            }
-#pragma unroll
-                            for (int e = 0; e < 4; ++e)
-                                *reinterpret_cast<float4*>(sbuf + sb_idx(r, ch + e)) =
-                                    make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
-                        }
-                        tmem_st_wait();
-                    }
-                    tc_fence_before();
-                    fence_async_smem();                          // S_after -> the state warp's TMA store
-                    warp_arrive(&mb_sfree, lane);
-                    if (has_next) warp_arrive(&mb_sready, lane);  // the next slot's state is in TMEM
-                    // partial sums: pairwise in fp32, over the warp's lanes and then over the warps
-                    float fn = num, fd = shared_end ? den_end : den;
-#pragma unroll
-                    for (int m = 16; m >= 1; m >>= 1) {
-                        fn += __shfl_xor_sync(0xffffffffu, fn, m);
-                        fd += __shfl_xor_sync(0xffffffffu, fd, m);
-                    }
-                    if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
-                    if (named_sync_or(kBarChain, kChain, !ok)) { stop = true; break; }
-                    if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot)) {   // a shared head: at its end
-                        float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
-                        float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
-#pragma unroll
-                        for (int m = kChainWarps / 2; m >= 1; m >>= 1) {
-                            pn += __shfl_xor_sync(0xffffffffu, pn, m);
-                            pd += __shfl_xor_sync(0xffffffffu, pd, m);
-                        }
-                        if (lane == 0) {
-                            a.partials[(size_t)lh * 2 + 0] = pn;
-                            a.partials[(size_t)lh * 2 + 1] = pd;
-                        }
-                    }
-                    den = den_next;
-                    sig = 1.f;
-                }
-                prev_lh = lh;
-                prev_slot = slot;
-                prev_last = last;
+                sig = 1.f;
             }
+            if (has_next) {
+                tc_fence_before();
+                warp_arrive(&mb_ready, lane);               // W(j + 1) (and a new slot's state) ready
+            }
+            prev_lh = lh;
+            prev_slot = slot;
+            prev_last = last;
             cc.next(sch, a);
         }
-        // the CTA's last sub-tile (always a slot's last) once every warp's pass has added to it
-        if (want_w && NS > 0 && !named_sync_or(kBarChain, kChain, *abort_flag) && warp == 0) {
-            fold_writes(NS - 1);
+        // the CTA's last tile (always a slot's last) once every warp's pass has added to it
+        if (want_w && NJ > 0 && !named_sync_or(kBarChain, kChain, *abort_flag) && warp == 0) {
+            fold_writes(NJ - 1);
             if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 45);
         }
     }
@@ -1156,30 +1100,16 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
-// [L][T][H][128] bfloat16 as a 4-D map (d, H, T, L): a box of 64 features x 1 head x `rows` tokens,
+// [L][T][H][128] bfloat16 as a 4-D map (d, H, T, L): a box of 64 features x 1 head x 64 tokens,
 // 128-byte swizzle; tokens past T read as zero.
-bool make_map(CUtensorMap* map, const void* base, int L, int T, int H, int rows) {
+bool make_map(CUtensorMap* map, const void* base, int L, int T, int H) {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return false;
     cuuint64_t dims[4] = {(cuuint64_t)kD, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)L};
     cuuint64_t strides[3] = {(cuuint64_t)kD * 2, (cuuint64_t)H * kD * 2, (cuuint64_t)T * H * kD * 2};
-    cuuint32_t box[4] = {64, 1, (cuuint32_t)rows, 1};
+    cuuint32_t box[4] = {64, 1, (cuuint32_t)kC, 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// The state [L * Hv * 128][128] fp32 as a 2-D map: a box of 32 columns x 128 rows (one column block
-// of one head), 128-byte swizzle.
-bool make_state_map(CUtensorMap* map, void* base, int heads) {
-    EncodeTiledFn enc = encode_fn();
-    if (!enc) return false;
-    cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)heads * kD};
-    cuuint64_t strides[1] = {(cuuint64_t)kD * 4};
-    cuuint32_t box[2] = {32, (cuuint32_t)kD};
-    cuuint32_t es[2] = {1, 1};
-    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -1216,7 +1146,6 @@ bool gdn_tc_shape(const GdnArgs& a) {
 
 bool gdn_tc_supported(const GdnArgs& a) {
     return gdn_tc_shape(a) &&
-           (long long)a.L * a.Hv * kD < (1ll << 31) &&                          // TMA row coordinate
            a.Hk <= (1 << 24) && a.T < (1 << 30) &&
            a.scratch != nullptr &&
            a.scratch_bytes >= gdn_tc_scratch_bytes(a.L, a.Hv, a.dk, a.dv, a.dtype, a.T) &&
@@ -1229,21 +1158,20 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     const int sms = device_sm_count();
     const int H = a.L * a.Hv;
     const int grid = std::min(H, sms);
-    CUtensorMap kmap, vmap, smap, hmap;
-    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk, kTile) || !make_map(&vmap, a.v, a.L, a.T, a.Hv, kC) ||
-        !make_state_map(&smap, a.state, H) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
-        return cudaErrorInvalidValue;
+    CUtensorMap kmap, vmap;
+    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv)) return cudaErrorInvalidValue;
     // The attribute is per device; setting it on every launch costs little and stays correct after
     // a device reset and from any host thread.
     cudaError_t e = cudaFuncSetAttribute(gdn_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSmemAlloc);
     if (e != cudaSuccess) return e;
-    const int n_tiles = (a.T + kTile - 1) / kTile;
+    const int n_tiles = (a.T + kC - 1) / kC;
     TcArgs t;
     t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = n_tiles;
     t.g = a.g; t.beta = a.beta;
     t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.status = a.status;
     t.ho_bits = reinterpret_cast<uint32_t*>(a.status) + 4;
+    t.ho_state = reinterpret_cast<float*>(a.scratch + sl.ho_state);
     t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
     t.split = 0;
     if (H > grid && H % grid != 0) {
@@ -1264,14 +1192,14 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
         attr[0].val.cooperative = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, gdn_fused_kernel, kmap, vmap, smap, hmap, t);
+        e = cudaLaunchKernelEx(&cfg, gdn_fused_kernel, kmap, vmap, t);
         if (e != cudaErrorCooperativeLaunchTooLarge) return e;
         (void)cudaGetLastError();                 // fewer SMs than the grid: whole heads instead
         t.split = 0;
     }
     cfg.attrs = nullptr;
     cfg.numAttrs = 0;
-    return cudaLaunchKernelEx(&cfg, gdn_fused_kernel, kmap, vmap, smap, hmap, t);
+    return cudaLaunchKernelEx(&cfg, gdn_fused_kernel, kmap, vmap, t);
 }
 
 }  // namespace deltas
