@@ -15,14 +15,15 @@
 // folds into one product with the state:  gamma_C X^T N_beta^T = S0 (K^T N_beta^T).
 //
 // Work split inside one CTA (one per SM, persistent over (layer, value head) slots):
-//   producer (4 warps): K K^T of the tile comes from the tensor core; the producer forms
+//   producer (two groups of 4 warps, each taking every other tile, so that a group has two tile
+//            periods for one tile): K K^T of the tile comes from the tensor core; the group forms
 //            diag(beta) L, inverts I + diag(beta) L (16 x 16 diagonal blocks by substitution, then
 //            two levels of block products) and writes two operand images, each a bfloat16
 //            (hi, lo) pair laid out as the two K-halves of one operand:
 //              B1 = u N_beta diag(delta)   and   B3 = N_beta
 //            (u: the state's deferred scale, below)
 //   MMA      (1 warp, one elected lane): every tcgen05.mma, each group's completion by commit
-//   chain    (8 warps): the pass over E, the K^T N_beta^T product into the B operand W, head
+//   chain    (4 warps): the pass over E, the K^T N_beta^T product into the B operand W, head
 //            boundaries (state in and out, drift partials)
 //   loads    (1 warp): K and V tiles by TMA, L2 prefetch of the tiles ahead and of the next state
 // Per tile j, in tensor-pipe order:
@@ -76,14 +77,15 @@ constexpr int kD = 128;                // head dim (d_k = d_v)
 constexpr float kHardMin = 0x1p-45f;   // p below this: the state is rescaled by a pass
 
 // ---- roles
-constexpr int kChainWarps = 8;
+constexpr int kChainWarps = 4;         // warps 0..3: warp q serves TMEM lanes 32 q ..
 constexpr int kChain = 32 * kChainWarps;
-constexpr int kProdWarp0 = 8;          // 8..11: producer (warp 8 + i reads TMEM lanes 32 i ..)
-constexpr int kProd = 128;
+constexpr int kProdWarp0 = 4;          // warps 4..7: producer group 1 (odd tiles), 8..11: group 0 (even);
+                                       // warp i of a group (i = warp % 4) reads TMEM lanes 32 i ..
+constexpr int kProd = 128;             // threads of a producer group
 constexpr int kMmaWarp = 12;
 constexpr int kLoadWarp = 13;
 constexpr int kThreads = 14 * 32;
-constexpr int kBarChain = 1;           // named barriers: chain (256 threads), producer (128)
+constexpr int kBarChain = 1;           // named barriers: chain, producer group 0, group 1 (128 threads each)
 constexpr int kBarProd = 2;
 
 // ---- TMEM columns
@@ -91,28 +93,34 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t TM_S = 0, TM_SB = 128, TM_E = 256, TM_KK = 384, TM_Q = 448;
 
 // ---- shared memory (bytes from a 1024-aligned base)
-constexpr uint32_t SM_K = 0;           // 3 tiles x 16 KB: 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B, SW128
-constexpr uint32_t SM_V = 49152;       // 2 tiles x 16 KB, same layout (also the K K^T product's over-read
-                                       // past the last K tile: rows 64..127 of its M = 128 A)
-constexpr uint32_t SM_B1 = 81920;      // 2 x 16 KB: rows t of u N_beta diag(delta): hi in column block 0,
-                                       // lo in block 1 (64 rows x 128 B each, SW128)
-constexpr uint32_t SM_B3 = 114688;     // 2 x 16 KB: N_beta, same layout
-constexpr uint32_t SM_W = 147456;      // 32 KB: W^T = -c N_beta K in tf32, rows t: 4 column blocks (32 dims)
+constexpr int kKSlots = 5;             // K ring: a tile's K K^T is issued three tiles before its state update
+constexpr uint32_t SM_K = 0;           // 5 tiles x 16 KB: 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B, SW128
+constexpr uint32_t SM_V = 81920;       // 16 KB, same layout (also the K K^T product's over-read past the last
+                                       // K tile: rows 64..127 of its M = 128 A)
+constexpr uint32_t SM_B1 = 98304;      // 16 KB: rows t of u N_beta diag(delta): hi in column block 0, lo in
+                                       // block 1 (64 rows x 128 B each, SW128)
+constexpr uint32_t SM_B3 = 114688;     // 16 KB: N_beta, same layout
+constexpr uint32_t SM_W = 131072;      // 32 KB: W^T = -c N_beta K in tf32, rows t: 4 column blocks (32 dims)
                                        // x 64 rows x 128 B, SW128 (the B operand of E += S~ W)
-constexpr uint32_t SM_PW = 180224;     // producer workspace
-constexpr int kMS = 68;                // fp32 row stride of M and N (16-byte aligned rows)
-constexpr int kPS = 36;                // fp32 row stride of the block products
-constexpr int PW_M = 0, PW_N = 64 * kMS, PW_P = 128 * kMS, PW_BETA = PW_P + 32 * kPS, PW_DELTA = PW_BETA + 128,
-              PW_UC = PW_DELTA + 128, PW_FLOATS = PW_UC + 8;   // beta, delta, (u, c): [2][..] by tile parity
-constexpr uint32_t SM_CONST = SM_PW + PW_FLOATS * 4;   // 2 slots x kConstWords: per-tile constants
+constexpr uint32_t SM_PW = 163840;     // producer workspaces, one per group
+// A group's workspace (fp32): rows 0..31 of M = diag(beta) L and of N = (I + diag(beta) L)^-1 hold
+// columns 0..31 only (the rest is above the diagonal), rows 32..63 all 64 columns; the block
+// products; beta, delta and (u, c) of the group's tile, double-buffered (the constants warp writes
+// the group's next tile's while the others may still read this one's).
+constexpr int kTS = 36, kBS = 68, kPS = 36;   // row strides (16-byte aligned rows)
+constexpr int PW_MT = 0, PW_MB = PW_MT + 32 * kTS, PW_NT = PW_MB + 32 * kBS, PW_NB = PW_NT + 32 * kTS,
+              PW_P = PW_NB + 32 * kBS, PW_BETA = PW_P + 32 * kPS, PW_DELTA = PW_BETA + 128, PW_UC = PW_DELTA + 128,
+              PW_FLOATS = PW_UC + 8;
+constexpr uint32_t kPwBytes = PW_FLOATS * 4;
+constexpr uint32_t SM_CONST = SM_PW + 2 * kPwBytes;   // 2 slots x kConstWords: per-tile constants
 constexpr int kConstWords = 72;        // [0,64) write-size scale per token, 64 sig after, 65 pass factor
                                        // (< 0: none), 66 shift (int), 67 c
 constexpr uint32_t SM_BYTES = SM_CONST + 2 * kConstWords * 4;
 constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
 static_assert(SM_V % 1024 == 0 && SM_B1 % 1024 == 0 && SM_B3 % 1024 == 0 && SM_W % 1024 == 0 &&
-              SM_PW % 16 == 0 && SM_CONST % 16 == 0, "shared-memory map");
-static_assert(SM_V == SM_K + 3 * 16384 && SM_B1 == SM_V + 2 * 16384 && SM_B3 == SM_B1 + 2 * 16384 &&
-              SM_W == SM_B3 + 2 * 16384 && SM_PW == SM_W + 32768, "map order");
+              kPwBytes % 16 == 0 && SM_CONST % 16 == 0, "shared-memory map");
+static_assert(SM_V == SM_K + kKSlots * 16384 && SM_B1 == SM_V + 16384 && SM_B3 == SM_B1 + 16384 &&
+              SM_W == SM_B3 + 16384 && SM_PW == SM_W + 32768, "map order");
 static_assert(kSmemAlloc + 1024 <= 232448, "shared memory budget");
 
 // Barrier over `n` threads that also returns the OR of `flag` over them (uniform result).
@@ -336,12 +344,13 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
     // loads -> roles: K, V tiles full; MMA -> loader: their empties.  producer -> MMA / chain: images
-    // and constants full (ifull); released by the products that read them and by the chain
-    // (iempty).  MMA -> producer: K K^T done (kk); producer -> MMA: read (kkfree).  MMA -> chain:
-    // Q done (q), E ready (u), state updated (s); chain -> MMA: W and the slot's state ready
-    // (ready), E packed (uready).
-    __shared__ uint64_t mb_kfull[3], mb_kempty[3], mb_vfull[2], mb_vempty[2], mb_ifull[2], mb_iempty[2];
-    __shared__ uint64_t mb_kk, mb_kkfree, mb_q, mb_ready, mb_u, mb_uready, mb_s, mb_fin;
+    // and constants full (ifull, by tile parity); the images are free once their products have
+    // completed (bfree, by the parity of the tile that used them), the constants once the chain has
+    // read them (iempty).  MMA -> producer group: K K^T done (kk, by parity); producer -> MMA: read
+    // (kkfree).  MMA -> chain: Q done (q), E ready (u), state updated (s); chain -> MMA: W and the
+    // slot's state ready (ready), E packed (uready).
+    __shared__ uint64_t mb_kfull[kKSlots], mb_kempty[kKSlots], mb_vfull, mb_vempty, mb_ifull[2], mb_iempty[2];
+    __shared__ uint64_t mb_bfree[2], mb_kk[2], mb_kkfree, mb_q, mb_ready, mb_u, mb_uready, mb_s, mb_fin;
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ float s_red[2][kChainWarps];
@@ -363,12 +372,13 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         tmem_alloc(&s_tmem, kTmemCols);
         tmem_relinquish();
         if (lane == 0) {
-            for (int b = 0; b < 3; ++b) { mbar_init(&mb_kfull[b], 1); mbar_init(&mb_kempty[b], 1); }
+            for (int b = 0; b < kKSlots; ++b) { mbar_init(&mb_kfull[b], 1); mbar_init(&mb_kempty[b], 1); }
+            mbar_init(&mb_vfull, 1); mbar_init(&mb_vempty, 1);
             for (int b = 0; b < 2; ++b) {
-                mbar_init(&mb_vfull[b], 1); mbar_init(&mb_vempty[b], 1);
-                mbar_init(&mb_ifull[b], 4); mbar_init(&mb_iempty[b], 1 + kChainWarps);
+                mbar_init(&mb_ifull[b], 4); mbar_init(&mb_iempty[b], kChainWarps);
+                mbar_init(&mb_bfree[b], 1); mbar_init(&mb_kk[b], 1);
             }
-            mbar_init(&mb_kk, 1); mbar_init(&mb_kkfree, 2); mbar_init(&mb_q, 1);
+            mbar_init(&mb_kkfree, 2); mbar_init(&mb_q, 1);
             mbar_init(&mb_ready, kChainWarps); mbar_init(&mb_u, 1); mbar_init(&mb_uready, kChainWarps);
             mbar_init(&mb_s, 1); mbar_init(&mb_fin, 1);
             fence_barrier_init();
@@ -394,14 +404,14 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         // K K^T of tile J (M = 128: rows 64..127 of A read the 16 KB past the tile; their output
         // lanes are ignored), once the tile has landed and the producer has read the previous one
         auto issue_kk = [&](int J) -> bool {
-            const uint32_t base = smem_u32(sm + SM_K + (J % 3) * 16384);
+            const uint32_t base = smem_u32(sm + SM_K + (J % kKSlots) * 16384);
             uint64_t d[2][4];
 #pragma unroll
             for (int s = 0; s < 8; ++s) {
                 d[s >> 2][s & 3] = sdesc_sw128(base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
                 pin(d[s >> 2][s & 3]);
             }
-            if (!warp_wait(&mb_kfull[J % 3], (J / 3) & 1, budget, abort_flag)) return false;
+            if (!warp_wait(&mb_kfull[J % kKSlots], (J / kKSlots) & 1, budget, abort_flag)) return false;
             if (J > 0 && !warp_wait(&mb_kkfree, (J - 1) & 1, budget, abort_flag)) return false;
             tc_fence_after();
             if (elect_one()) {
@@ -409,7 +419,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 mma4_bf16_ss_1t(tm + TM_KK, d[1], d[1], idK, 1);
             }
             __syncwarp();
-            mma_commit(&mb_kk);
+            mma_commit(&mb_kk[J & 1]);
             return true;
         };
         // A (K^T or V^T: the tile read MN-major; k-steps 4..7 repeat tokens 0..63 for the lo half)
@@ -431,20 +441,18 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         auto issue_images = [&](int J) -> bool {
             if (!warp_wait(&mb_ifull[J & 1], (J >> 1) & 1, budget, abort_flag)) return false;
             tc_fence_after();
-            issue_img(tm + TM_Q, smem_u32(sm + SM_K + (J % 3) * 16384), smem_u32(sm + SM_B3 + (J & 1) * 16384));
+            issue_img(tm + TM_Q, smem_u32(sm + SM_K + (J % kKSlots) * 16384), smem_u32(sm + SM_B3));
             mma_commit(&mb_q);
-            if (!warp_wait(&mb_vfull[J & 1], (J >> 1) & 1, budget, abort_flag)) return false;
+            if (!warp_wait(&mb_vfull, J & 1, budget, abort_flag)) return false;
             tc_fence_after();
-            issue_img(tm + TM_E + (J & 1) * 64, smem_u32(sm + SM_V + (J & 1) * 16384),
-                      smem_u32(sm + SM_B1 + (J & 1) * 16384));
-            mma_commit(&mb_vempty[J & 1]);
-            mma_commit(&mb_iempty[J & 1]);             // the images' products are issued
+            issue_img(tm + TM_E + (J & 1) * 64, smem_u32(sm + SM_V), smem_u32(sm + SM_B1));
+            mma_commit(&mb_vempty);
+            mma_commit(&mb_bfree[J & 1]);              // the images' last reader
             return true;
         };
         bool ok = true;
         if (NJ > 0) {
-            ok = issue_kk(0);
-            if (ok && NJ > 1) ok = issue_kk(1);
+            for (int J = 0; ok && J < 3 && J < NJ; ++J) ok = issue_kk(J);
             if (ok) ok = issue_images(0);
             if (!ok) fail(a.status, abort_flag, 1);
         }
@@ -466,7 +474,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 if (j > 0 && !warp_wait(&mb_s, (j - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 3); break; }
                 // E(j)'s own product has completed: for j > 0 the state update's commit covers it
                 // (issued after it), for the first tile its own commit
-                if (j == 0 && !warp_wait(&mb_vempty[0], 0, budget, abort_flag)) { fail(a.status, abort_flag, 7); break; }
+                if (j == 0 && !warp_wait(&mb_vempty, 0, budget, abort_flag)) { fail(a.status, abort_flag, 7); break; }
                 // the tile's images and constants are held until the chain has read them
                 shift = reinterpret_cast<const volatile int*>(cst + (j & 1) * kConstWords)[66];
                 tc_fence_after();
@@ -477,13 +485,14 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 __syncwarp();
                 mma_commit(&mb_u);
             }
-            // the next tile's Q and E, and K K^T two tiles ahead, while the chain runs its pass
+            // K K^T three tiles ahead (a producer group has two tile periods for its tile), the next
+            // tile's Q and E, while the chain runs its pass
+            if (j + 3 < NJ && !issue_kk(j + 3)) { fail(a.status, abort_flag, 5); break; }
             if (j + 1 < NJ && !issue_images(j + 1)) { fail(a.status, abort_flag, 4); break; }
-            if (j + 2 < NJ && !issue_kk(j + 2)) { fail(a.status, abort_flag, 5); break; }
             {   // S~ = 2^-shift S~ + E K  (A: E hi / lo packed in place; K read MN-major)
                 uint32_t ah[4], al[4];
                 uint64_t bs[4];
-                const uint32_t kb = smem_u32(sm + SM_K + (j % 3) * 16384);
+                const uint32_t kb = smem_u32(sm + SM_K + (j % kKSlots) * 16384);
 #pragma unroll
                 for (int s = 0; s < 4; ++s) {
                     ah[s] = eb + 32 * (s >> 1) + 8 * (s & 1);
@@ -499,7 +508,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 }
                 __syncwarp();
                 mma_commit(&mb_s);
-                mma_commit(&mb_kempty[j % 3]);         // the tile's last reader
+                mma_commit(&mb_kempty[j % kKSlots]);   // the tile's last reader
             }
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0)) {
@@ -508,13 +517,17 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         }
         __syncwarp();
     } else if (warp == kLoadWarp) {
-        // =========================================================== K and V tiles in order, each
-        // into its buffer once the MMA that last read the buffer has completed; the tiles three
-        // ahead and each slot's successor's state are prefetched into L2
-        TileCursor cc, pf;
-        cc.init(sch, a);
-        pf.init(sch, a);
-        int kp[3] = {-1, -1, -1}, vp[2] = {-1, -1};   // last tile loaded per buffer
+        // =========================================================== K and V tiles, each into its
+        // buffer once the MMA that last read the buffer has completed.  The V stream runs two tiles
+        // behind the K stream: the MMA takes K three tiles ahead of the state update (for K K^T) but
+        // V one tile ahead, so a V load held for its buffer must not hold up the K loads behind it.
+        // The tiles ahead of the K ring and each slot's successor's state are prefetched into L2.
+        TileCursor kc, vc, pf;
+        kc.init(sch, a);
+        vc = kc;
+        pf = kc;
+        int kp[kKSlots], vp = -1;                      // last tile loaded per buffer
+        for (int b = 0; b < kKSlots; ++b) kp[b] = -1;
         grid_dep_wait();
         auto prefetch_tile = [&](const TileCursor& c) {
             tma_prefetch_4d(&kmap, 0, c.kh, c.jt * kC, c.l);
@@ -522,138 +535,182 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             tma_prefetch_4d(&vmap, 0, c.h, c.jt * kC, c.l);
             tma_prefetch_4d(&vmap, 64, c.h, c.jt * kC, c.l);
         };
-        for (int i = 0; i < 3 && i < NJ; ++i) {
+        for (int i = 0; i < kKSlots && i < NJ; ++i) {
             if (elect_one()) prefetch_tile(pf);
             __syncwarp();
             pf.next(sch, a);
         }
+        constexpr int kVLag = 2;
         bool ok = true;
-        for (int J = 0; ok && J < NJ; ++J) {
-            if (J + 3 < NJ) {
-                if (elect_one()) prefetch_tile(pf);
+        for (int n = 0; ok && n < NJ + kVLag; ++n) {
+            if (n < NJ) {                                // K of tile n
+                if (n + kKSlots < NJ) {
+                    if (elect_one()) prefetch_tile(pf);
+                    __syncwarp();
+                    pf.next(sch, a);
+                }
+                if (kc.jt == kc.tb && kc.k + 1 < sch.n_slots && !sch.is_suffix(kc.k + 1) && elect_one()) {
+                    int lh, tb, te;                      // the next slot's state, ahead of its boundary
+                    sch.slot(kc.k + 1, a.n_tiles, lh, tb, te);
+                    prefetch_l2_bulk(a.state + (size_t)lh * kD * kD, kD * kD * 4);
+                }
                 __syncwarp();
-                pf.next(sch, a);
+                const int bk = n % kKSlots;
+                if (n >= kKSlots && !warp_wait(&mb_kempty[bk], ((n / kKSlots) - 1) & 1, budget, abort_flag)) {
+                    fail(a.status, abort_flag, 30); break;
+                }
+                if (elect_one()) {
+                    uint8_t* dst = sm + SM_K + bk * 16384;
+                    mbar_arrive_expect_tx(&mb_kfull[bk], 16384);
+                    tma_load_4d(dst, &kmap, &mb_kfull[bk], 0, kc.kh, kc.jt * kC, kc.l);
+                    tma_load_4d(dst + 8192, &kmap, &mb_kfull[bk], 64, kc.kh, kc.jt * kC, kc.l);
+                }
+                __syncwarp();
+                kp[bk] = n;
+                kc.next(sch, a);
             }
-            if (cc.jt == cc.tb && cc.k + 1 < sch.n_slots && !sch.is_suffix(cc.k + 1) && elect_one()) {
-                int lh, tb, te;                          // the next slot's state, ahead of its boundary
-                sch.slot(cc.k + 1, a.n_tiles, lh, tb, te);
-                prefetch_l2_bulk(a.state + (size_t)lh * kD * kD, kD * kD * 4);
+            const int m = n - kVLag;                     // V of tile m
+            if (m >= 0) {
+                if (m >= 1 && !warp_wait(&mb_vempty, (m - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 31); break; }
+                if (elect_one()) {
+                    uint8_t* dst = sm + SM_V;
+                    mbar_arrive_expect_tx(&mb_vfull, 16384);
+                    tma_load_4d(dst, &vmap, &mb_vfull, 0, vc.h, vc.jt * kC, vc.l);
+                    tma_load_4d(dst + 8192, &vmap, &mb_vfull, 64, vc.h, vc.jt * kC, vc.l);
+                }
+                __syncwarp();
+                vp = m;
+                vc.next(sch, a);
             }
-            __syncwarp();
-            const int bk = J % 3, bv = J & 1;
-            if (J >= 3 && !warp_wait(&mb_kempty[bk], ((J / 3) - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 30); break; }
-            if (elect_one()) {
-                uint8_t* dst = sm + SM_K + bk * 16384;
-                mbar_arrive_expect_tx(&mb_kfull[bk], 16384);
-                tma_load_4d(dst, &kmap, &mb_kfull[bk], 0, cc.kh, cc.jt * kC, cc.l);
-                tma_load_4d(dst + 8192, &kmap, &mb_kfull[bk], 64, cc.kh, cc.jt * kC, cc.l);
-            }
-            __syncwarp();
-            kp[bk] = J;
-            if (J >= 2 && !warp_wait(&mb_vempty[bv], ((J >> 1) - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 31); break; }
-            if (elect_one()) {
-                uint8_t* dst = sm + SM_V + bv * 16384;
-                mbar_arrive_expect_tx(&mb_vfull[bv], 16384);
-                tma_load_4d(dst, &vmap, &mb_vfull[bv], 0, cc.h, cc.jt * kC, cc.l);
-                tma_load_4d(dst + 8192, &vmap, &mb_vfull[bv], 64, cc.h, cc.jt * kC, cc.l);
-            }
-            __syncwarp();
-            vp[bv] = J;
-            cc.next(sch, a);
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0) && lane == 0) {
             // every copy this warp issued lands before the CTA ends
-            for (int b = 0; b < 3; ++b)
-                if (kp[b] >= 0) mbar_wait(&mb_kfull[b], (kp[b] / 3) & 1, budget);
-            for (int b = 0; b < 2; ++b)
-                if (vp[b] >= 0) mbar_wait(&mb_vfull[b], (vp[b] >> 1) & 1, budget);
+            for (int b = 0; b < kKSlots; ++b)
+                if (kp[b] >= 0) mbar_wait(&mb_kfull[b], (kp[b] / kKSlots) & 1, budget);
+            if (vp >= 0) mbar_wait(&mb_vfull, vp & 1, budget);
         }
         __syncwarp();
     } else if (warp >= kProdWarp0) {
-        // =========================================================== producer: the images of
-        // every tile, and its decay constants
-        const int pw = warp - kProdWarp0;              // 0..3
-        const int pt = pw * 32 + lane;                 // thread of the producer, 0..127
-        float* fws = reinterpret_cast<float*>(sm + SM_PW);
-        float* Mm = fws + PW_M;                        // diag(beta) L, rows of kMS
-        float* Nm = fws + PW_N;                        // (I + diag(beta) L)^-1 (lower part)
+        // =========================================================== producer: the images and decay
+        // constants of every tile; group 0 (warps 8-11) the even tiles, group 1 (warps 4-7) the odd
+        const int grp = warp >= 8 ? 0 : 1;
+        const int pw = warp & 3;                       // 0, 1: K K^T readers (TMEM lanes 32 pw ..); 2: constants
+        const int pt = pw * 32 + lane;                 // thread of the group, 0..127
+        const int bar_id = kBarProd + grp;
+        float* fws = reinterpret_cast<float*>(sm + SM_PW + grp * kPwBytes);
+        float* Mt = fws + PW_MT;                       // rows 0..31 of diag(beta) L (columns 0..31)
+        float* Mb = fws + PW_MB;                       // rows 32..63 (columns 0..63)
+        float* Nt = fws + PW_NT;                       // the same rows of (I + diag(beta) L)^-1
+        float* Nb = fws + PW_NB;
         float* Pm = fws + PW_P;                        // block products
-        TileCursor cc;
+        auto mrow = [&](int r) { return r < 32 ? Mt + r * kTS : Mb + (r - 32) * kBS; };
+        auto nrow = [&](int r) { return r < 32 ? Nt + r * kTS : Nb + (r - 32) * kBS; };
+        const int g = lane >> 2, tq = lane & 3;        // mma.sync fragment coordinates
+        // cursors at the group's tile J and at J - 1 (the deferred scale before J depends on it)
+        TileCursor cc, cq;
         cc.init(sch, a);
-        // warp 10: g and beta of tokens lane and 32 + lane of the tile; warps 8, 9: beta of token
-        // 32 pw + lane (their rows of K K^T); loaded one tile ahead of use
-        float pg0 = 0.f, pg1 = 0.f, pb0 = 0.f, pb1 = 0.f;
-        auto load_gb = [&](const TileCursor& c) {
+        cq = cc;
+        if (grp == 1 && NJ > 1) cc.next(sch, a);
+        // loads, one group-tile ahead: warp 2 the g and beta of the tile's tokens lane, 32 + lane and
+        // the g of tile J - 1 when it is in J's slot; warps 0, 1 the beta of token 32 pw + lane
+        struct Gb { float g0, g1, b0, b1, q0, q1; };
+        auto load_gb = [&](const TileCursor& c, const TileCursor& cp, bool prev_same) {
+            Gb v = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
             const int t0 = c.jt * kC + lane, t1 = t0 + 32;
             const size_t base = (size_t)c.l * a.T;
             if (pw == 2) {
-                pg0 = t0 < a.T ? a.g[(base + t0) * a.Hv + c.h] : 0.f;
-                pg1 = t1 < a.T ? a.g[(base + t1) * a.Hv + c.h] : 0.f;
+                v.g0 = t0 < a.T ? a.g[(base + t0) * a.Hv + c.h] : 0.f;
+                v.g1 = t1 < a.T ? a.g[(base + t1) * a.Hv + c.h] : 0.f;
+                v.b0 = t0 < a.T ? a.beta[(base + t0) * a.Hv + c.h] : 0.f;
+                v.b1 = t1 < a.T ? a.beta[(base + t1) * a.Hv + c.h] : 0.f;
+                if (prev_same) {
+                    const int s0 = cp.jt * kC + lane, s1 = s0 + 32;
+                    const size_t pb = (size_t)cp.l * a.T;
+                    v.q0 = s0 < a.T ? a.g[(pb + s0) * a.Hv + cp.h] : 0.f;
+                    v.q1 = s1 < a.T ? a.g[(pb + s1) * a.Hv + cp.h] : 0.f;
+                }
+            } else if (pw < 2) {
+                const int tb = t0 + 32 * pw;
+                v.b0 = tb < a.T ? a.beta[(base + tb) * a.Hv + c.h] : 0.f;
             }
-            const int tb = (pw == 1) ? t1 : t0;
-            pb0 = tb < a.T ? a.beta[(base + tb) * a.Hv + c.h] : 0.f;
-            if (pw == 2) pb1 = t1 < a.T ? a.beta[(base + t1) * a.Hv + c.h] : 0.f;
+            return v;
         };
-        if (pw < 3 && NJ > 0) { grid_dep_wait(); load_gb(cc); }
-        float sig = 1.f;
-        int prev_slot = -1;
+        // the tile's cumulative log-decay: inclusive scans of its two halves (both groups use this
+        // order, so the deferred scale they compute for a tile agrees bit for bit)
+        auto scan_tile = [&](float g0, float g1, float& G0, float& G1) {
+            G0 = g0; G1 = g1;
+#pragma unroll
+            for (int m = 1; m < 32; m <<= 1) {
+                const float y0 = __shfl_up_sync(0xffffffffu, G0, m);
+                const float y1 = __shfl_up_sync(0xffffffffu, G1, m);
+                if (lane >= m) { G0 += y0; G1 += y1; }
+            }
+            G1 += __shfl_sync(0xffffffffu, G0, 31);
+            return __shfl_sync(0xffffffffu, G1, 31);
+        };
+        Gb cur = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (pw < 3 && grp < NJ) {
+            grid_dep_wait();
+            cur = load_gb(cc, cq, grp == 1 && cq.k == cc.k);
+        }
+        float sig_last = 1.f;                          // sig after the group's previous tile
         bool failed = false;
-        const int g = lane >> 2, tq = lane & 3;        // mma.sync fragment coordinates
-        for (int J = 0; J < NJ; ++J) {
-            float* sBeta = fws + PW_BETA + 64 * (J & 1);
-            float* sDelta = fws + PW_DELTA + 64 * (J & 1);
-            float* sUC = fws + PW_UC + 4 * (J & 1);
+        for (int J = grp; J < NJ; J += 2) {
+            const int slot2 = (J >> 1) & 1;
+            float* sBeta = fws + PW_BETA + 64 * slot2;
+            float* sDelta = fws + PW_DELTA + 64 * slot2;
+            float* sUC = fws + PW_UC + 4 * slot2;
+            const bool first_of_slot = cc.jt == cc.tb;
+            const bool prev_first = cq.jt == cq.tb;    // (J - 1 in J's slot only when !first_of_slot)
+            const Gb now = cur;
+            TileCursor nq = cc, nc = cc;               // the group's next tile J + 2 and J + 1
+            if (J + 2 < NJ) {
+                nq.next(sch, a);
+                nc = nq;
+                nc.next(sch, a);
+                if (pw < 3) cur = load_gb(nc, nq, nq.k == nc.k);
+            }
             DecayStep dst;
             float wn0 = 0.f, wn1 = 0.f;
-            // this tile's g, beta (bmine: warps 8, 9 the beta of this lane's row), then the next tile's
-            const float bmine = pb0, g0 = pg0, g1 = pg1, b1 = pb1;
-            if (pw < 3 && J + 1 < NJ) {
-                TileCursor nx = cc;
-                nx.next(sch, a);
-                load_gb(nx);
-            }
             if (pw == 2) {
                 // ---- constants of the tile's 64 tokens (lane: tokens lane and 32 + lane)
-                const float b0 = bmine;
-                if (cc.k != prev_slot) sig = 1.f;       // a slot starts from the true state
-                prev_slot = cc.k;
-                float G0 = g0, G1 = g1;                 // inclusive scans of the two halves
-#pragma unroll
-                for (int m = 1; m < 32; m <<= 1) {
-                    const float y0 = __shfl_up_sync(0xffffffffu, G0, m);
-                    const float y1 = __shfl_up_sync(0xffffffffu, G1, m);
-                    if (lane >= m) { G0 += y0; G1 += y1; }
+                float sig_b = 1.f;                     // a slot starts from the true state
+                if (!first_of_slot) {                  // tile J - 1 (the other group's) in the same slot
+                    float Q0, Q1;
+                    const float GQ = scan_tile(now.q0, now.q1, Q0, Q1);
+                    sig_b = decay_step(expf(GQ) * (prev_first ? 1.f : sig_last)).sig;
                 }
-                G1 += __shfl_sync(0xffffffffu, G0, 31);
-                const float GC = __shfl_sync(0xffffffffu, G1, 31);
-                dst = decay_step(expf(GC) * sig);
-                sig = dst.sig;
+                float G0, G1;
+                const float GC = scan_tile(now.g0, now.g1, G0, G1);
+                dst = decay_step(expf(GC) * sig_b);
+                sig_last = dst.sig;
                 const float d0 = expf(GC - G0), d1 = expf(GC - G1);
-                sBeta[lane] = b0; sBeta[32 + lane] = b1;
+                sBeta[lane] = now.b0; sBeta[32 + lane] = now.b1;
                 sDelta[lane] = d0; sDelta[32 + lane] = d1;
                 const float ud0 = dst.u * d0, ud1 = dst.u * d1;
                 wn0 = ud0 >= 0x1p-60f ? 1.f / ud0 : 0.f;   // column t of E is u delta_t u_t
                 wn1 = ud1 >= 0x1p-60f ? 1.f / ud1 : 0.f;
                 if (lane == 0) { sUC[0] = dst.u; sUC[1] = dst.c; }
             } else if (pw < 2) {
-                // ---- rows 32 pw .. 32 pw + 31 of diag(beta) L from K K^T (warp 9: also the block
+                // ---- rows 32 pw .. 32 pw + 31 of diag(beta) L from K K^T (warp 1: also the block
                 // left of the diagonal, in full)
-                const bool ok = mbar_wait_or_abort(&mb_kk, J & 1, budget, abort_flag);
+                const bool ok = mbar_wait_or_abort(&mb_kk[grp], (J >> 1) & 1, budget, abort_flag);
                 if (!ok) { fail(a.status, abort_flag, 20); failed = true; }
                 tc_fence_after();
                 if (ok) {
                     const uint32_t base = tm + ((uint32_t)(32 * pw) << 16) + TM_KK;
-                    float* row = Mm + (32 * pw + lane) * kMS;
+                    float* row = mrow(32 * pw + lane);
+                    const float bt = now.b0;
                     float kk[32];
                     tmem_ld32(base + 32 * pw, kk);         // the diagonal block
                     tmem_ld_wait();
 #pragma unroll
                     for (int c4 = 0; c4 < 8; ++c4) {
                         float4 v;
-                        v.x = (4 * c4 + 0 < lane) ? bmine * kk[4 * c4 + 0] : 0.f;
-                        v.y = (4 * c4 + 1 < lane) ? bmine * kk[4 * c4 + 1] : 0.f;
-                        v.z = (4 * c4 + 2 < lane) ? bmine * kk[4 * c4 + 2] : 0.f;
-                        v.w = (4 * c4 + 3 < lane) ? bmine * kk[4 * c4 + 3] : 0.f;
+                        v.x = (4 * c4 + 0 < lane) ? bt * kk[4 * c4 + 0] : 0.f;
+                        v.y = (4 * c4 + 1 < lane) ? bt * kk[4 * c4 + 1] : 0.f;
+                        v.z = (4 * c4 + 2 < lane) ? bt * kk[4 * c4 + 2] : 0.f;
+                        v.w = (4 * c4 + 3 < lane) ? bt * kk[4 * c4 + 3] : 0.f;
                         *reinterpret_cast<float4*>(row + 32 * pw + 4 * c4) = v;
                     }
                     if (pw == 1) {                         // rows 32..63 x columns 0..31
@@ -662,15 +719,14 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
 #pragma unroll
                         for (int c4 = 0; c4 < 8; ++c4)
                             *reinterpret_cast<float4*>(row + 4 * c4) =
-                                make_float4(bmine * kk[4 * c4], bmine * kk[4 * c4 + 1], bmine * kk[4 * c4 + 2],
-                                            bmine * kk[4 * c4 + 3]);
+                                make_float4(bt * kk[4 * c4], bt * kk[4 * c4 + 1], bt * kk[4 * c4 + 2], bt * kk[4 * c4 + 3]);
                     }
                 }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&mb_kkfree);
             }
-            if (named_sync_or(kBarProd, kProd, failed || *abort_flag)) break;        // (1)
+            if (named_sync_or(bar_id, kProd, failed || *abort_flag)) break;          // (1)
             if (pw < 2) {
                 // the four 16 x 16 diagonal blocks of N by forward substitution, one column per lane;
                 // the next row's coefficients are loaded while the current row is formed
@@ -678,111 +734,120 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 float x[16];
 #pragma unroll
                 for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
-                float4 cur[4], nxt[4];
-                cur[0] = *reinterpret_cast<const float4*>(Mm + (o + 1) * kMS + o);
+                float4 cur4[4], nxt4[4];
+                cur4[0] = *reinterpret_cast<const float4*>(mrow(o + 1) + o);
 #pragma unroll
                 for (int rr = 1; rr < 16; ++rr) {
                     if (rr + 1 < 16) {
 #pragma unroll
                         for (int c4 = 0; c4 < 4; ++c4)
-                            if (4 * c4 < rr + 1) nxt[c4] = *reinterpret_cast<const float4*>(Mm + (o + rr + 1) * kMS + o + 4 * c4);
+                            if (4 * c4 < rr + 1) nxt4[c4] = *reinterpret_cast<const float4*>(mrow(o + rr + 1) + o + 4 * c4);
                     }
-                    float s[4] = {0.f, 0.f, 0.f, 0.f};     // four short FMA chains
+                    float sacc[4] = {0.f, 0.f, 0.f, 0.f};     // four short FMA chains
 #pragma unroll
                     for (int c4 = 0; c4 < 4; ++c4) {
                         const int c = 4 * c4;
                         if (c < rr) {
-                            s[0] = fmaf(cur[c4].x, x[c], s[0]);
-                            if (c + 1 < rr) s[1] = fmaf(cur[c4].y, x[c + 1], s[1]);
-                            if (c + 2 < rr) s[2] = fmaf(cur[c4].z, x[c + 2], s[2]);
-                            if (c + 3 < rr) s[3] = fmaf(cur[c4].w, x[c + 3], s[3]);
+                            sacc[0] = fmaf(cur4[c4].x, x[c], sacc[0]);
+                            if (c + 1 < rr) sacc[1] = fmaf(cur4[c4].y, x[c + 1], sacc[1]);
+                            if (c + 2 < rr) sacc[2] = fmaf(cur4[c4].z, x[c + 2], sacc[2]);
+                            if (c + 3 < rr) sacc[3] = fmaf(cur4[c4].w, x[c + 3], sacc[3]);
                         }
                     }
-                    if (rr > jc) x[rr] = -((s[0] + s[1]) + (s[2] + s[3]));
+                    if (rr > jc) x[rr] = -((sacc[0] + sacc[1]) + (sacc[2] + sacc[3]));
 #pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) cur[c4] = nxt[c4];
+                    for (int c4 = 0; c4 < 4; ++c4) cur4[c4] = nxt4[c4];
                 }
 #pragma unroll
-                for (int rr = 0; rr < 16; ++rr) Nm[(o + rr) * kMS + o + jc] = x[rr];
+                for (int rr = 0; rr < 16; ++rr) nrow(o + rr)[o + jc] = x[rr];
                 if ((lane >> 4) == 0) {
 #pragma unroll
-                    for (int rr = 0; rr < 16; ++rr) Nm[(o + rr) * kMS + o + 16 + jc] = 0.f;   // block above
+                    for (int rr = 0; rr < 16; ++rr) nrow(o + rr)[o + 16 + jc] = 0.f;   // the block above
                 }
             }
-            if (named_sync_or(kBarProd, kProd, *abort_flag)) break;                  // (2)
+            if (named_sync_or(bar_id, kProd, *abort_flag)) break;                    // (2)
             {   // 16 -> 32, warp (p, nh): in 32-block p, columns 8 nh .. of
                 //   P = M[16..32][0..16] N[0..16][0..16],  then  N[16..32][0..16] = -N[16..32][16..32] P
                 // (tensor-core fragments, three-term bfloat16 products)
                 const int p = pw >> 1, nh = pw & 1, o = 32 * p;
+                const int ld = p ? kBS : kTS;
                 float d[4] = {0.f, 0.f, 0.f, 0.f};
-                mma_f32_split<1>(d, Mm + (o + 16) * kMS + o, kMS, Nm + o * kMS + o + 8 * nh, kMS, g, tq);
+                mma_f32_split<1>(d, mrow(o + 16) + o, ld, nrow(o) + o + 8 * nh, ld, g, tq);
                 float* pp = Pm + 16 * p * kPS + 8 * nh;
                 *reinterpret_cast<float2*>(pp + g * kPS + 2 * tq) = make_float2(d[0], d[1]);
                 *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 2 * tq) = make_float2(d[2], d[3]);
                 __syncwarp();
                 float e[4] = {0.f, 0.f, 0.f, 0.f};
-                mma_f32_split<1>(e, Nm + (o + 16) * kMS + o + 16, kMS, pp, kPS, g, tq);
-                float* np = Nm + (o + 16) * kMS + o + 8 * nh;
-                *reinterpret_cast<float2*>(np + g * kMS + 2 * tq) = make_float2(-e[0], -e[1]);
-                *reinterpret_cast<float2*>(np + (g + 8) * kMS + 2 * tq) = make_float2(-e[2], -e[3]);
+                mma_f32_split<1>(e, nrow(o + 16) + o + 16, ld, pp, kPS, g, tq);
+                float* np = nrow(o + 16) + o + 8 * nh;
+                *reinterpret_cast<float2*>(np + g * ld + 2 * tq) = make_float2(-e[0], -e[1]);
+                *reinterpret_cast<float2*>(np + (g + 8) * ld + 2 * tq) = make_float2(-e[2], -e[3]);
             }
-            if (named_sync_or(kBarProd, kProd, *abort_flag)) break;                  // (3)
+            if (named_sync_or(bar_id, kProd, *abort_flag)) break;                    // (3)
             {   // 32 -> 64, warp (mt, nh): rows 16 mt .., columns 16 nh .. of
                 //   P = M[32..64][0..32] N[0..32][0..32],  then  N[32..64][0..32] = -N[32..64][32..64] P
                 const int mt = pw >> 1, nh = pw & 1;
                 float d0[4] = {0.f, 0.f, 0.f, 0.f}, d1[4] = {0.f, 0.f, 0.f, 0.f};
-                mma_f32_split<2>(d0, Mm + (32 + 16 * mt) * kMS, kMS, Nm + 16 * nh, kMS, g, tq);
-                mma_f32_split<2>(d1, Mm + (32 + 16 * mt) * kMS, kMS, Nm + 16 * nh + 8, kMS, g, tq);
+                mma_f32_split<2>(d0, Mb + 16 * mt * kBS, kBS, Nt + 16 * nh, kTS, g, tq);
+                mma_f32_split<2>(d1, Mb + 16 * mt * kBS, kBS, Nt + 16 * nh + 8, kTS, g, tq);
                 float* pp = Pm + 16 * mt * kPS + 16 * nh;
                 *reinterpret_cast<float2*>(pp + g * kPS + 2 * tq) = make_float2(d0[0], d0[1]);
                 *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 2 * tq) = make_float2(d0[2], d0[3]);
                 *reinterpret_cast<float2*>(pp + g * kPS + 8 + 2 * tq) = make_float2(d1[0], d1[1]);
                 *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 8 + 2 * tq) = make_float2(d1[2], d1[3]);
-                if (named_sync_or(kBarProd, kProd, *abort_flag)) break;              // (4)
+                if (named_sync_or(bar_id, kProd, *abort_flag)) break;                // (4)
                 float e0[4] = {0.f, 0.f, 0.f, 0.f}, e1[4] = {0.f, 0.f, 0.f, 0.f};
-                mma_f32_split<2>(e0, Nm + (32 + 16 * mt) * kMS + 32, kMS, Pm + 16 * nh, kPS, g, tq);
-                mma_f32_split<2>(e1, Nm + (32 + 16 * mt) * kMS + 32, kMS, Pm + 16 * nh + 8, kPS, g, tq);
-                float* np = Nm + (32 + 16 * mt) * kMS + 16 * nh;
-                *reinterpret_cast<float2*>(np + g * kMS + 2 * tq) = make_float2(-e0[0], -e0[1]);
-                *reinterpret_cast<float2*>(np + (g + 8) * kMS + 2 * tq) = make_float2(-e0[2], -e0[3]);
-                *reinterpret_cast<float2*>(np + g * kMS + 8 + 2 * tq) = make_float2(-e1[0], -e1[1]);
-                *reinterpret_cast<float2*>(np + (g + 8) * kMS + 8 + 2 * tq) = make_float2(-e1[2], -e1[3]);
+                mma_f32_split<2>(e0, Nb + 16 * mt * kBS + 32, kBS, Pm + 16 * nh, kPS, g, tq);
+                mma_f32_split<2>(e1, Nb + 16 * mt * kBS + 32, kBS, Pm + 16 * nh + 8, kPS, g, tq);
+                float* np = Nb + 16 * mt * kBS + 16 * nh;
+                *reinterpret_cast<float2*>(np + g * kBS + 2 * tq) = make_float2(-e0[0], -e0[1]);
+                *reinterpret_cast<float2*>(np + (g + 8) * kBS + 2 * tq) = make_float2(-e0[2], -e0[3]);
+                *reinterpret_cast<float2*>(np + g * kBS + 8 + 2 * tq) = make_float2(-e1[0], -e1[1]);
+                *reinterpret_cast<float2*>(np + (g + 8) * kBS + 8 + 2 * tq) = make_float2(-e1[2], -e1[3]);
             }
-            // the image slot is free once tile J - 2's products and the chain have read it
-            if (J >= 2) {
-                const bool ok = mbar_wait_or_abort(&mb_iempty[J & 1], ((J >> 1) - 1) & 1, budget, abort_flag);
-                if (!ok) { fail(a.status, abort_flag, 21); failed = true; }
+            // the images are free once the products of tile J - 1 (the other group's) have completed,
+            // the constants slot once the chain has read those of tile J - 2
+            if (J >= 1 && !mbar_wait_or_abort(&mb_bfree[(J - 1) & 1], ((J - 1) >> 1) & 1, budget, abort_flag)) {
+                fail(a.status, abort_flag, 21); failed = true;
             }
-            if (named_sync_or(kBarProd, kProd, failed || *abort_flag)) break;        // (5)
+            if (J >= 2 && !mbar_wait_or_abort(&mb_iempty[J & 1], ((J >> 1) - 1) & 1, budget, abort_flag)) {
+                fail(a.status, abort_flag, 22); failed = true;
+            }
+            if (named_sync_or(bar_id, kProd, failed || *abort_flag)) break;          // (5)
             {   // images: row t = pt / 2, columns 32 hh .. 32 hh + 31 of N_beta = N diag(beta) (zero
                 // above the diagonal)
                 const int t = pt >> 1, hh = pt & 1;
                 const float u = sUC[0];
-                uint8_t* b1 = sm + SM_B1 + (J & 1) * 16384;
-                uint8_t* b3 = sm + SM_B3 + (J & 1) * 16384;
+                uint8_t* b1 = sm + SM_B1;
+                uint8_t* b3 = sm + SM_B3;
+                const bool zero_half = t < 32 && hh == 1;
+                const float* nr = nrow(t) + (zero_half ? 0 : 32 * hh);
 #pragma unroll
                 for (int g8 = 0; g8 < 4; ++g8) {        // 8 columns (one 16-byte chunk of bf16) at a time
                     const int c = 32 * hh + 8 * g8;
-                    const float4 n0 = *reinterpret_cast<const float4*>(Nm + t * kMS + c);
-                    const float4 n1 = *reinterpret_cast<const float4*>(Nm + t * kMS + c + 4);
-                    const float4 bv0 = *reinterpret_cast<const float4*>(sBeta + c);
-                    const float4 bv1 = *reinterpret_cast<const float4*>(sBeta + c + 4);
-                    const float4 dv0 = *reinterpret_cast<const float4*>(sDelta + c);
-                    const float4 dv1 = *reinterpret_cast<const float4*>(sDelta + c + 4);
-                    const float nv[8] = {n0.x, n0.y, n0.z, n0.w, n1.x, n1.y, n1.z, n1.w};
-                    const float bv[8] = {bv0.x, bv0.y, bv0.z, bv0.w, bv1.x, bv1.y, bv1.z, bv1.w};
-                    const float dv[8] = {dv0.x, dv0.y, dv0.z, dv0.w, dv1.x, dv1.y, dv1.z, dv1.w};
-                    float nb[8], w1[8];
+                    uint32_t h3[4] = {0u, 0u, 0u, 0u}, l3[4] = {0u, 0u, 0u, 0u};
+                    uint32_t h1[4] = {0u, 0u, 0u, 0u}, l1[4] = {0u, 0u, 0u, 0u};
+                    if (!zero_half) {
+                        const float4 n0 = *reinterpret_cast<const float4*>(nr + 8 * g8);
+                        const float4 n1 = *reinterpret_cast<const float4*>(nr + 8 * g8 + 4);
+                        const float4 bv0 = *reinterpret_cast<const float4*>(sBeta + c);
+                        const float4 bv1 = *reinterpret_cast<const float4*>(sBeta + c + 4);
+                        const float4 dv0 = *reinterpret_cast<const float4*>(sDelta + c);
+                        const float4 dv1 = *reinterpret_cast<const float4*>(sDelta + c + 4);
+                        const float nv[8] = {n0.x, n0.y, n0.z, n0.w, n1.x, n1.y, n1.z, n1.w};
+                        const float bv[8] = {bv0.x, bv0.y, bv0.z, bv0.w, bv1.x, bv1.y, bv1.z, bv1.w};
+                        const float dv[8] = {dv0.x, dv0.y, dv0.z, dv0.w, dv1.x, dv1.y, dv1.z, dv1.w};
+                        float nb[8], w1[8];
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        nb[i] = (c + i <= t) ? nv[i] * bv[i] : 0.f;
-                        w1[i] = u * nb[i] * dv[i];
-                    }
-                    uint32_t h3[4], l3[4], h1[4], l1[4];
+                        for (int i = 0; i < 8; ++i) {
+                            nb[i] = (c + i <= t) ? nv[i] * bv[i] : 0.f;
+                            w1[i] = u * nb[i] * dv[i];
+                        }
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        split2(nb[2 * i], nb[2 * i + 1], h3[i], l3[i]);
-                        split2(w1[2 * i], w1[2 * i + 1], h1[i], l1[i]);
+                        for (int i = 0; i < 4; ++i) {
+                            split2(nb[2 * i], nb[2 * i + 1], h3[i], l3[i]);
+                            split2(w1[2 * i], w1[2 * i + 1], h1[i], l1[i]);
+                        }
                     }
                     const uint32_t off = sw128_offset(t, c >> 3);
                     *reinterpret_cast<uint4*>(b3 + off) = make_uint4(h3[0], h3[1], h3[2], h3[3]);
@@ -805,32 +870,34 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             fence_async_smem();                         // generic writes -> the tensor core's reads
             __syncwarp();
             if (lane == 0) mbar_arrive(&mb_ifull[J & 1]);
-            cc.next(sch, a);
+            cq = nq;
+            cc = nc;
         }
     } else {
-        // =========================================================== state chain (warps 0-7)
-        const int q = warp & 3, hh = warp >> 2;          // TMEM lane quadrant, column half
+        // =========================================================== state chain (warps 0-3)
+        const int q = warp;                              // TMEM lane quadrant
         const int r = 32 * q + lane;                     // row of S (value index)
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
         TileCursor cc;
         cc.init(sch, a);
-        // W(jj) = -c Q^T in tf32: this thread's d_k row c = r of Q, tokens 32 hh .. 32 hh + 31, into
-        // rows t of the K-major W (column block q, its 4-byte slot of row t).  Q(jj) is complete and
-        // W's last reader, E(jj-1) += S~ W(jj-1), has completed.
+        // W(jj) = -c Q^T in tf32: this thread's d_k row c = r of Q, tokens 0..63, into rows t of the
+        // K-major W (column block q, its 4-byte slot of row t).  Q(jj) is complete and W's last
+        // reader, E(jj-1) += S~ W(jj-1), has completed.
         auto make_w = [&](int jj) -> bool {
             bool ok = mbar_wait_or_abort(&mb_q, jj & 1, budget, abort_flag);
             ok = mbar_wait_or_abort(&mb_ifull[jj & 1], (jj >> 1) & 1, budget, abort_flag) && ok;
             tc_fence_after();
             const float cneg = -cst[(jj & 1) * kConstWords + 67];
-            float qv[32];
-            tmem_ld32(tm + lane_off + TM_Q + 32 * hh, qv);
-            tmem_ld_wait();
             uint8_t* wb = sm + SM_W + q * 8192 + (lane & 3) * 4;
             const int chunk = lane >> 2;
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                const int t = 32 * hh + i;
-                *reinterpret_cast<uint32_t*>(wb + sw128_offset(t, chunk)) = to_tf32(cneg * qv[i]);
+            for (int hh = 0; hh < 2; ++hh) {
+                float qv[32];
+                tmem_ld32(tm + lane_off + TM_Q + 32 * hh, qv);
+                tmem_ld_wait();
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    *reinterpret_cast<uint32_t*>(wb + sw128_offset(32 * hh + i, chunk)) = to_tf32(cneg * qv[i]);
             }
             fence_async_smem();
             tc_fence_before();
@@ -857,18 +924,18 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 ok = !named_sync_or(kBarChain, kChain, *abort_flag);
             }
             const float* src = (from_ho ? a.ho_state + (size_t)(me - 1) * kD * kD : a.state + (size_t)lh * kD * kD)
-                               + (size_t)r * kD + 64 * hh;
+                               + (size_t)r * kD;
             den = 0.f;
             if (ok) {
-#pragma unroll
-                for (int g4 = 0; g4 < 4; ++g4) {
+#pragma unroll 2
+                for (int g8 = 0; g8 < 8; ++g8) {
                     float v[16];
-                    ld16_global(src + 16 * g4, v, from_ho);
+                    ld16_global(src + 16 * g8, v, from_ho);
                     uint32_t u32[16];
 #pragma unroll
                     for (int e = 0; e < 16; ++e) { den = fmaf(v[e], v[e], den); u32[e] = __float_as_uint(v[e]); }
-                    tmem_st16(tm + lane_off + TM_S + 64 * hh + 16 * g4, u32);
-                    tmem_st16(tm + lane_off + TM_SB + 64 * hh + 16 * g4, u32);
+                    tmem_st16(tm + lane_off + TM_S + 16 * g8, u32);
+                    tmem_st16(tm + lane_off + TM_SB + 16 * g8, u32);
                 }
             }
             return ok;
@@ -942,22 +1009,23 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             const float* cs = cst + (j & 1) * kConstWords;
             const float pass_f = cs[65];
             const float sig_after = cs[64];
-            const float wf = cs[32 * hh + lane];
             if (pass_f >= 0.f) {
                 // the decay would take the deferred scale out of range: S~ <- p S~ (the state
                 // update of this tile has not been issued: it waits for this pass)
 #pragma unroll 1
-                for (int g4 = 0; g4 < 4; ++g4) {
+                for (int g8 = 0; g8 < 8; ++g8) {
                     float sv[16];
-                    tmem_ld16(tm + lane_off + TM_S + 64 * hh + 16 * g4, sv);
+                    tmem_ld16(tm + lane_off + TM_S + 16 * g8, sv);
                     tmem_ld_wait();
                     uint32_t su[16];
 #pragma unroll
                     for (int e = 0; e < 16; ++e) su[e] = __float_as_uint(sv[e] * pass_f);
-                    tmem_st16(tm + lane_off + TM_S + 64 * hh + 16 * g4, su);
+                    tmem_st16(tm + lane_off + TM_S + 16 * g8, su);
                 }
             }
-            {   // ---- pass: this thread's 32 token columns of E -> (hi, lo) A operand, in place
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {
+                // ---- pass: 32 token columns of E -> (hi, lo) A operand, in place
                 const uint32_t eb = tm + lane_off + TM_E + (j & 1) * 64 + 32 * hh;
                 float e[32];
                 tmem_ld32(eb, e);
@@ -965,6 +1033,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 if (want_w) {
                     // squares summed over the warp's 32 rows, column by column: halving exchanges
                     // leave lane c with column c
+                    const float wf = cs[32 * hh + lane];
                     float x[32];
 #pragma unroll
                     for (int i = 0; i < 32; ++i) x[i] = e[i] * e[i];
@@ -984,8 +1053,8 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 for (int i = 0; i < 16; ++i) split2(e[2 * i], e[2 * i + 1], hi[i], lo[i]);
                 tmem_st16(eb, hi);
                 tmem_st16(eb + 16, lo);
-                tmem_st_wait();
             }
+            tmem_st_wait();
             tc_fence_before();
             warp_arrive(&mb_uready, lane);
             warp_arrive(&mb_iempty[j & 1], lane);          // the tile's constants are read
@@ -1004,19 +1073,19 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 tc_fence_after();
                 float num = 0.f, den_end = 0.f;
                 float* dstp = (prefix ? a.ho_state + (size_t)me * kD * kD : a.state + (size_t)lh * kD * kD)
-                              + (size_t)r * kD + 64 * hh;
-                const float* sbp = a.state + (size_t)lh * kD * kD + (size_t)r * kD + 64 * hh;
+                              + (size_t)r * kD;
+                const float* sbp = a.state + (size_t)lh * kD * kD + (size_t)r * kD;
                 if (ok) {
 #pragma unroll 1
-                    for (int g4 = 0; g4 < 4; ++g4) {
+                    for (int g8 = 0; g8 < 8; ++g8) {
                         float sa[16], sb[16];
-                        tmem_ld16(tm + lane_off + TM_S + 64 * hh + 16 * g4, sa);
+                        tmem_ld16(tm + lane_off + TM_S + 16 * g8, sa);
                         if (shared_end) {
-                            ld16_global(sbp + 16 * g4, sb, true);
+                            ld16_global(sbp + 16 * g8, sb, true);
 #pragma unroll
                             for (int e = 0; e < 16; ++e) den_end = fmaf(sb[e], sb[e], den_end);
                         } else {
-                            tmem_ld16(tm + lane_off + TM_SB + 64 * hh + 16 * g4, sb);
+                            tmem_ld16(tm + lane_off + TM_SB + 16 * g8, sb);
                         }
                         tmem_ld_wait();
 #pragma unroll
@@ -1025,7 +1094,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                             const float d = sa[e] - sb[e];
                             num = fmaf(d, d, num);
                         }
-                        float4* o4 = reinterpret_cast<float4*>(dstp + 16 * g4);
+                        float4* o4 = reinterpret_cast<float4*>(dstp + 16 * g8);
 #pragma unroll
                         for (int e = 0; e < 4; ++e) o4[e] = make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
                     }
