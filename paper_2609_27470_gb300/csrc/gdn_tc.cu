@@ -197,14 +197,63 @@ __device__ __forceinline__ void mma_f32_split(float (&d)[4], const float* A, int
     for (int i = 0; i < 4; ++i) d[i] += d1[i] + d2[i];
 }
 
+// One kind::f16 MMA from TMEM A that scales the accumulator it reads by 2^-shift (the
+// instruction's scale-input-d operand, an immediate: D = A B + 2^-shift D), shift in [0, 15].
+template <int S>
+__device__ __forceinline__ void mma_bf16_ta_scaled(uint32_t d, uint32_t a, uint64_t b, uint32_t idesc) {
+    asm volatile("{\n\t.reg .pred q;\n\t"
+                 "setp.eq.b32 q, %3, %3;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, q, %4;\n\t}"
+                 :: "r"(d), "r"(a), "l"(b), "r"(idesc), "n"(S) : "memory");
+}
+__device__ __noinline__ void mma_bf16_ta_shift_1t(int shift, uint32_t d, uint32_t a, uint64_t b, uint32_t idesc) {
+    switch (shift) {
+        case 0: mma_bf16_ta_scaled<0>(d, a, b, idesc); break;
+        case 1: mma_bf16_ta_scaled<1>(d, a, b, idesc); break;
+        case 2: mma_bf16_ta_scaled<2>(d, a, b, idesc); break;
+        case 3: mma_bf16_ta_scaled<3>(d, a, b, idesc); break;
+        case 4: mma_bf16_ta_scaled<4>(d, a, b, idesc); break;
+        case 5: mma_bf16_ta_scaled<5>(d, a, b, idesc); break;
+        case 6: mma_bf16_ta_scaled<6>(d, a, b, idesc); break;
+        case 7: mma_bf16_ta_scaled<7>(d, a, b, idesc); break;
+        case 8: mma_bf16_ta_scaled<8>(d, a, b, idesc); break;
+        case 9: mma_bf16_ta_scaled<9>(d, a, b, idesc); break;
+        case 10: mma_bf16_ta_scaled<10>(d, a, b, idesc); break;
+        case 11: mma_bf16_ta_scaled<11>(d, a, b, idesc); break;
+        case 12: mma_bf16_ta_scaled<12>(d, a, b, idesc); break;
+        case 13: mma_bf16_ta_scaled<13>(d, a, b, idesc); break;
+        case 14: mma_bf16_ta_scaled<14>(d, a, b, idesc); break;
+        default: mma_bf16_ta_scaled<15>(d, a, b, idesc); break;
+    }
+}
+
+// The waits of this kernel: one try inline, the bounded loop out of line (the kernel's code must
+// stay small: every role's loop shares the SM's instruction cache, and misses are served from a
+// busy L2).
+__device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
+                                       const volatile int* abort) {
+    const long long t0 = clock64();
+    const long long budget = (long long)(budget_ns * 2);
+    for (;;) {
+        if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+        if (*abort) return false;
+        if (clock64() - t0 > budget) return false;
+    }
+}
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
+                                         const volatile int* abort) {
+    if (mbar_try_wait(bar, parity)) return true;
+    return wait_slow(bar, parity, budget_ns, abort);
+}
+
 // All lanes of a converged warp wait; the result is the same on every lane.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
                                           const volatile int* abort) {
-    const bool ok = mbar_wait_or_abort(bar, parity, budget_ns, abort);
+    const bool ok = wait_bar(bar, parity, budget_ns, abort);
     return __all_sync(0xffffffffu, ok) != 0;
 }
 
-__device__ __forceinline__ void fail(int32_t* status, volatile int* abort, int where) {
+__device__ __noinline__ void fail(int32_t* status, volatile int* abort, int where) {
     record_status(status, DELTAS_ERR_TIMEOUT, where);
     *abort = 1;
 }
@@ -220,6 +269,10 @@ __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
     uint32_t v;
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
+}
+
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+    asm volatile("prefetch.global.L2 [%0];" :: "l"(p) : "memory");
 }
 
 __device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
@@ -312,7 +365,7 @@ struct ChainSched {
 // head h), key head kh.
 struct TileCursor {
     int k, jt, tb, te, lh, l, h, kh;
-    __device__ __forceinline__ void set_slot(int slot, const ChainSched& sc, const TcArgs& a) {
+    __device__ __noinline__ void set_slot(int slot, const ChainSched& sc, const TcArgs& a) {
         k = slot;
         sc.slot(slot, a.n_tiles, lh, tb, te);
         jt = tb;
@@ -403,20 +456,19 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         const uint32_t idK = idesc_bf16(128, 64, 0, 0);
         // K K^T of tile J (M = 128: rows 64..127 of A read the 16 KB past the tile; their output
         // lanes are ignored), once the tile has landed and the producer has read the previous one
+        // (every product below is a rolled loop of single MMAs from one elected lane: the issue
+        // rate is the tensor pipe's, and the code stays small)
         auto issue_kk = [&](int J) -> bool {
-            const uint32_t base = smem_u32(sm + SM_K + (J % kKSlots) * 16384);
-            uint64_t d[2][4];
-#pragma unroll
-            for (int s = 0; s < 8; ++s) {
-                d[s >> 2][s & 3] = sdesc_sw128(base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
-                pin(d[s >> 2][s & 3]);
-            }
             if (!warp_wait(&mb_kfull[J % kKSlots], (J / kKSlots) & 1, budget, abort_flag)) return false;
             if (J > 0 && !warp_wait(&mb_kkfree, (J - 1) & 1, budget, abort_flag)) return false;
             tc_fence_after();
             if (elect_one()) {
-                mma4_bf16_ss_1t(tm + TM_KK, d[0], d[0], idK, 0);
-                mma4_bf16_ss_1t(tm + TM_KK, d[1], d[1], idK, 1);
+                const uint32_t base = smem_u32(sm + SM_K + (J % kKSlots) * 16384);
+#pragma unroll 1
+                for (int s = 0; s < 8; ++s) {
+                    const uint64_t d = sdesc_sw128(base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
+                    mma_bf16_1t(tm + TM_KK, d, d, idK, s > 0);
+                }
             }
             __syncwarp();
             mma_commit(&mb_kk[J & 1]);
@@ -425,15 +477,11 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         // A (K^T or V^T: the tile read MN-major; k-steps 4..7 repeat tokens 0..63 for the lo half)
         // times B (an image: k-steps 0..3 its hi block, 4..7 its lo block) into D
         auto issue_img = [&](uint32_t d, uint32_t a_base, uint32_t b_base) {
-            uint64_t ad[2][4], bd[2][4];
-#pragma unroll
-            for (int s = 0; s < 8; ++s) {
-                ad[s >> 2][s & 3] = sdesc_sw128(a_base + (s & 3) * 2048, 8192, 1024);
-                bd[s >> 2][s & 3] = sdesc_sw128(b_base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
-            }
             if (elect_one()) {
-                mma4_bf16_ss_1t(d, ad[0], bd[0], idW, 0);
-                mma4_bf16_ss_1t(d, ad[1], bd[1], idW, 1);
+#pragma unroll 1
+                for (int s = 0; s < 8; ++s)
+                    mma_bf16_1t(d, sdesc_sw128(a_base + (s & 3) * 2048, 8192, 1024),
+                                sdesc_sw128(b_base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024), idW, s > 0);
             }
             __syncwarp();
         };
@@ -461,15 +509,6 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             int shift = 0;
             {   // E(j) += S~ W(j) (A: the state from TMEM as tf32, 8 columns per K = 8 step; B: W in
                 // tf32).  E(j)'s own product was issued before, into the same accumulator.
-                uint32_t ax[4][4];
-                uint64_t bx[4][4];
-                const uint32_t wb = smem_u32(sm + SM_W);
-#pragma unroll
-                for (int s = 0; s < 16; ++s) {
-                    ax[s >> 2][s & 3] = tm + TM_S + 8 * s;
-                    bx[s >> 2][s & 3] = sdesc_sw128(wb + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
-                    pin(ax[s >> 2][s & 3]); pin(bx[s >> 2][s & 3]);
-                }
                 if (!warp_wait(&mb_ready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 2); break; }
                 if (j > 0 && !warp_wait(&mb_s, (j - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 3); break; }
                 // E(j)'s own product has completed: for j > 0 the state update's commit covers it
@@ -479,8 +518,11 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 shift = reinterpret_cast<const volatile int*>(cst + (j & 1) * kConstWords)[66];
                 tc_fence_after();
                 if (elect_one()) {
-#pragma unroll
-                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(eb, ax[g4], bx[g4], idX, 1);
+                    const uint32_t wb = smem_u32(sm + SM_W);
+#pragma unroll 1
+                    for (int s = 0; s < 16; ++s)
+                        mma_tf32_ta_1t(eb, tm + TM_S + 8 * s, sdesc_sw128(wb + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024),
+                                       idX, 1);
                 }
                 __syncwarp();
                 mma_commit(&mb_u);
@@ -490,21 +532,18 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             if (j + 3 < NJ && !issue_kk(j + 3)) { fail(a.status, abort_flag, 5); break; }
             if (j + 1 < NJ && !issue_images(j + 1)) { fail(a.status, abort_flag, 4); break; }
             {   // S~ = 2^-shift S~ + E K  (A: E hi / lo packed in place; K read MN-major)
-                uint32_t ah[4], al[4];
-                uint64_t bs[4];
-                const uint32_t kb = smem_u32(sm + SM_K + (j % kKSlots) * 16384);
-#pragma unroll
-                for (int s = 0; s < 4; ++s) {
-                    ah[s] = eb + 32 * (s >> 1) + 8 * (s & 1);
-                    al[s] = ah[s] + 16;
-                    bs[s] = sdesc_sw128(kb + s * 2048, 8192, 1024);
-                    pin(ah[s]); pin(al[s]); pin(bs[s]);
-                }
                 if (!warp_wait(&mb_uready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 6); break; }
                 tc_fence_after();
                 if (elect_one()) {
-                    mma4_bf16_ta_shift_1t(shift, tm + TM_S, ah, bs, idS);
-                    mma4_bf16_ta_1t(tm + TM_S, al, bs, idS, 1);
+                    // K-step s: A = E's hi (s < 4) or lo (s >= 4) columns of token block s & 3
+                    const uint32_t kb = smem_u32(sm + SM_K + (j % kKSlots) * 16384);
+                    mma_bf16_ta_shift_1t(shift, tm + TM_S, eb, sdesc_sw128(kb, 8192, 1024), idS);
+#pragma unroll 1
+                    for (int s = 1; s < 8; ++s) {
+                        const int tb = s & 3;
+                        mma_bf16_ta_1t(tm + TM_S, eb + 32 * (tb >> 1) + 8 * (tb & 1) + 16 * (s >> 2),
+                                       sdesc_sw128(kb + tb * 2048, 8192, 1024), idS, 1);
+                    }
                 }
                 __syncwarp();
                 mma_commit(&mb_s);
@@ -529,14 +568,22 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         int kp[kKSlots], vp = -1;                      // last tile loaded per buffer
         for (int b = 0; b < kKSlots; ++b) kp[b] = -1;
         grid_dep_wait();
-        auto prefetch_tile = [&](const TileCursor& c) {
-            tma_prefetch_4d(&kmap, 0, c.kh, c.jt * kC, c.l);
-            tma_prefetch_4d(&kmap, 64, c.kh, c.jt * kC, c.l);
-            tma_prefetch_4d(&vmap, 0, c.h, c.jt * kC, c.l);
-            tma_prefetch_4d(&vmap, 64, c.h, c.jt * kC, c.l);
+        auto prefetch_tile = [&](const TileCursor& c) {    // all lanes
+            if (lane == 0) {
+                tma_prefetch_4d(&kmap, 0, c.kh, c.jt * kC, c.l);
+                tma_prefetch_4d(&kmap, 64, c.kh, c.jt * kC, c.l);
+                tma_prefetch_4d(&vmap, 0, c.h, c.jt * kC, c.l);
+                tma_prefetch_4d(&vmap, 64, c.h, c.jt * kC, c.l);
+            }
+            // the tile's g and beta (one 4-byte value per token, a line apart): the producer reads
+            // them one group-tile ahead, too late to take an HBM miss off its path
+            const int t0 = c.jt * kC + lane;
+            const size_t i0 = ((size_t)c.l * a.T + t0) * a.Hv + c.h;
+            if (t0 < a.T) { prefetch_l2(a.g + i0); prefetch_l2(a.beta + i0); }
+            if (t0 + 32 < a.T) { prefetch_l2(a.g + i0 + 32 * (size_t)a.Hv); prefetch_l2(a.beta + i0 + 32 * (size_t)a.Hv); }
         };
         for (int i = 0; i < kKSlots && i < NJ; ++i) {
-            if (elect_one()) prefetch_tile(pf);
+            prefetch_tile(pf);
             __syncwarp();
             pf.next(sch, a);
         }
@@ -545,7 +592,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         for (int n = 0; ok && n < NJ + kVLag; ++n) {
             if (n < NJ) {                                // K of tile n
                 if (n + kKSlots < NJ) {
-                    if (elect_one()) prefetch_tile(pf);
+                    prefetch_tile(pf);
                     __syncwarp();
                     pf.next(sch, a);
                 }
@@ -694,7 +741,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             } else if (pw < 2) {
                 // ---- rows 32 pw .. 32 pw + 31 of diag(beta) L from K K^T (warp 1: also the block
                 // left of the diagonal, in full)
-                const bool ok = mbar_wait_or_abort(&mb_kk[grp], (J >> 1) & 1, budget, abort_flag);
+                const bool ok = wait_bar(&mb_kk[grp], (J >> 1) & 1, budget, abort_flag);
                 if (!ok) { fail(a.status, abort_flag, 20); failed = true; }
                 tc_fence_after();
                 if (ok) {
@@ -807,10 +854,10 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             }
             // the images are free once the products of tile J - 1 (the other group's) have completed,
             // the constants slot once the chain has read those of tile J - 2
-            if (J >= 1 && !mbar_wait_or_abort(&mb_bfree[(J - 1) & 1], ((J - 1) >> 1) & 1, budget, abort_flag)) {
+            if (J >= 1 && !wait_bar(&mb_bfree[(J - 1) & 1], ((J - 1) >> 1) & 1, budget, abort_flag)) {
                 fail(a.status, abort_flag, 21); failed = true;
             }
-            if (J >= 2 && !mbar_wait_or_abort(&mb_iempty[J & 1], ((J >> 1) - 1) & 1, budget, abort_flag)) {
+            if (J >= 2 && !wait_bar(&mb_iempty[J & 1], ((J >> 1) - 1) & 1, budget, abort_flag)) {
                 fail(a.status, abort_flag, 22); failed = true;
             }
             if (named_sync_or(bar_id, kProd, failed || *abort_flag)) break;          // (5)
@@ -822,7 +869,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 uint8_t* b3 = sm + SM_B3;
                 const bool zero_half = t < 32 && hh == 1;
                 const float* nr = nrow(t) + (zero_half ? 0 : 32 * hh);
-#pragma unroll
+#pragma unroll 1
                 for (int g8 = 0; g8 < 4; ++g8) {        // 8 columns (one 16-byte chunk of bf16) at a time
                     const int c = 32 * hh + 8 * g8;
                     uint32_t h3[4] = {0u, 0u, 0u, 0u}, l3[4] = {0u, 0u, 0u, 0u};
@@ -884,13 +931,13 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         // K-major W (column block q, its 4-byte slot of row t).  Q(jj) is complete and W's last
         // reader, E(jj-1) += S~ W(jj-1), has completed.
         auto make_w = [&](int jj) -> bool {
-            bool ok = mbar_wait_or_abort(&mb_q, jj & 1, budget, abort_flag);
-            ok = mbar_wait_or_abort(&mb_ifull[jj & 1], (jj >> 1) & 1, budget, abort_flag) && ok;
+            bool ok = wait_bar(&mb_q, jj & 1, budget, abort_flag);
+            ok = wait_bar(&mb_ifull[jj & 1], (jj >> 1) & 1, budget, abort_flag) && ok;
             tc_fence_after();
             const float cneg = -cst[(jj & 1) * kConstWords + 67];
             uint8_t* wb = sm + SM_W + q * 8192 + (lane & 3) * 4;
             const int chunk = lane >> 2;
-#pragma unroll
+#pragma unroll 1
             for (int hh = 0; hh < 2; ++hh) {
                 float qv[32];
                 tmem_ld32(tm + lane_off + TM_Q + 32 * hh, qv);
@@ -927,7 +974,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                                + (size_t)r * kD;
             den = 0.f;
             if (ok) {
-#pragma unroll 2
+#pragma unroll 1
                 for (int g8 = 0; g8 < 8; ++g8) {
                     float v[16];
                     ld16_global(src + 16 * g8, v, from_ho);
@@ -1004,7 +1051,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 }
             }
             // ---- E(j) is complete (and E += S~ W has read the state and W)
-            if (!mbar_wait_or_abort(&mb_u, j & 1, budget, abort_flag)) fail(a.status, abort_flag, 10);
+            if (!wait_bar(&mb_u, j & 1, budget, abort_flag)) fail(a.status, abort_flag, 10);
             tc_fence_after();
             const float* cs = cst + (j & 1) * kConstWords;
             const float pass_f = cs[65];
@@ -1023,7 +1070,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                     tmem_st16(tm + lane_off + TM_S + 16 * g8, su);
                 }
             }
-#pragma unroll
+#pragma unroll 1
             for (int hh = 0; hh < 2; ++hh) {
                 // ---- pass: 32 token columns of E -> (hi, lo) A operand, in place
                 const uint32_t eb = tm + lane_off + TM_E + (j & 1) * 64 + 32 * hh;
@@ -1069,7 +1116,7 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 // slot's state in
                 const bool prefix = sch.is_prefix(slot);
                 const bool shared_end = sch.is_suffix(slot);   // S_before: the head's stored state
-                if (!mbar_wait_or_abort(&mb_s, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 12); ok = false; }
+                if (!wait_bar(&mb_s, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 12); ok = false; }
                 tc_fence_after();
                 float num = 0.f, den_end = 0.f;
                 float* dstp = (prefix ? a.ho_state + (size_t)me * kD * kD : a.state + (size_t)lh * kD * kD)
