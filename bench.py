@@ -306,8 +306,8 @@ class StreamingWorkload:
 
     def launches_per_step(self):
         if self.s.per_head:
-            return 1 + 1 + 1 + 3                                # update, append, select, compact (3)
-        return 1 + 1 + 1 + 3 + 3                                # update, score, append, select (3), compact (3)
+            return 2 + 1 + 1 + 3                                # update (2), append, select, compact (3)
+        return 2 + 1 + 1 + 3 + 3                                # update (2), score, append, select (3), compact (3)
 
     def tokens_per_step(self):
         # the mean chunk length (exact when the timed steps are a multiple of the ring)
@@ -371,7 +371,7 @@ class GdnOnlyWorkload:
         self.step_i += 1
 
     def launches_per_step(self):
-        return 1 + 1                                            # update, score
+        return 2 + 1                                            # factor + chain kernels, score
 
     def tokens_per_step(self):
         return self.C

@@ -1,66 +1,71 @@
 // Gated delta rule over one chunk on the Blackwell tensor cores (tcgen05 + TMEM + TMA), d = 128,
-// bfloat16 k/v, fp32 state, with the state-drift partials fused in: one persistent kernel.
+// bfloat16 k/v, fp32 state, with the state-drift partials fused in.
 //
 // Paper: Sec. 3.2, Eq. 1/2 (the recurrence) and Eq. 3 (drift numerator / denominator per layer
 // and head).  The chunk is processed in tiles of C = 64 tokens with the chunkwise (WY) form of
-// Eq. 1.  Inside a tile let G be the inclusive cumulative log-decay, gamma_t = exp(G_t),
-// gamma_C = exp(G_{C-1}), delta_t = gamma_C / gamma_t <= 1, and X = K S0^T (row t: S0 k_t).  With
-//   A[t][i] = beta_t (gamma_t / gamma_i) k_t.k_i  (i < t),   U = (I + A)^-1 diag(beta) (V - diag(gamma) X)
-// the state after the tile is S_C = gamma_C S0 + sum_t delta_t u_t k_t^T.  The decay factors out of
-// the triangular solve by a diagonal similarity, I + A = diag(gamma) (I + diag(beta) L) diag(gamma)^-1
-// with L the strictly lower part of K K^T, so with the decay-free
-//   N_beta = (I + diag(beta) L)^-1 diag(beta)
-// the decayed writes are  U~ = diag(delta) U = N_beta (diag(delta) V - gamma_C X):  every decay
-// factor the kernel uses is at most 1, and the inverse depends on k and beta only.  The X term
-// folds into one product with the state:  gamma_C X^T N_beta^T = S0 (K^T N_beta^T).
+// Eq. 1: with G the inclusive cumulative log-decay inside the tile, gamma = exp(G),
+//   A[t][i] = beta_t exp(G_t - G_i) k_t.k_i  (i < t),   T = (I + A)^-1 diag(beta),
+//   X = K S0^T,   W = V - diag(gamma) X,   U = T W,
+//   S_C = gamma_C S0 + U~^T K,   U~[t] = exp(G_C - G_t) U[t].
+// Padded tokens of a ragged last tile carry k = v = 0, g = 0, beta = 0 and change nothing.
 //
-// Work split inside one CTA (one per SM, persistent over (layer, value head) slots):
-//   producer (two groups of 4 warps, each taking every other tile, so that a group has two tile
-//            periods for one tile): K K^T of the tile comes from the tensor core; the group forms
-//            diag(beta) L, inverts I + diag(beta) L (16 x 16 diagonal blocks by substitution, then
-//            two levels of block products) and writes two operand images, each a bfloat16
-//            (hi, lo) pair laid out as the two K-halves of one operand:
-//              B1 = u N_beta diag(delta)   and   B3 = N_beta
-//            (u: the state's deferred scale, below)
-//   MMA      (1 warp, one elected lane): every tcgen05.mma, each group's completion by commit
-//   chain    (4 warps): the pass over E, the K^T N_beta^T product into the B operand W, head
-//            boundaries (state in and out, drift partials)
-//   loads    (1 warp): K and V tiles by TMA, L2 prefetch of the tiles ahead and of the next state
-// Per tile j, in tensor-pipe order:
-//   E(j)  += S~ W(j)                  (tf32: A = the fp32 state straight from TMEM)
-//   Q(j+1) = K^T B3, E(j+1) = V^T B1  (bf16 (hi, lo); the chain turns Q into W(j+1) = -c Q^T in
-//                                      tf32 in shared memory)
-//   K K^T (j+2)                       (bf16, for the producer)
-//   pass   (chain) E -> bfloat16 (hi, lo), in place
-//   S~     = 2^-s S~ + E K            (the input state scaled by the instruction's power-of-two
-//                                      scale-input-d operand)
-// The tensor core does not order an MMA that reads a TMEM region as its A operand after an earlier
-// MMA that wrote it (measured), so E += S~ W waits for the previous state update's commit.
+// Two kernels.  T and the tile's decay constants depend on k, g and beta only, so the factor
+// kernel builds them for every (layer, value head, tile) at once, several CTAs per SM, and writes
+// one record per tile into the workspace: T~ = diag(exp(G_C - G)) T as the bfloat16 (hi, lo) pair
+// in the swizzled layout the tensor core reads, -gamma and gamma_C.  The update kernel then runs
+// the part that is sequential in the tiles, the state chain, with nothing else on the SM.
 //
-// Deferred decay.  TMEM holds S~ with the true state S = sig S~.  A tile with decay gamma_C takes
-// p = gamma_C sig and a shift s in [0, 15] that brings p 2^s into [1/2, 1) when it can: then
-// sig <- p 2^s, u = 1 / sig, c = 2^-s, and the state update scales S~ by 2^-s as it accumulates
-// (exact).  When p < 2^-45 (no shift reaches 2^-30) the chain multiplies S~ by p in a pass instead,
-// sig restarts at 1, u = 1 and c = p.  So sig stays in [2^-30, 1] and u below 2^30.  The producer
-// writes each tile's constants (sig after the tile, the shift, the pass factor, c, the write-size
-// scales) beside its images.
+// Update kernel: one persistent CTA per SM takes (layer, value head) pairs in turn, or equal runs
+// of tiles with a head at each run boundary split between two CTAs (see ChainSched); the tiles of
+// its slots form one pipeline.  A head's state lives in TMEM from its first tile to its last
+// (S_before beside it, for the drift), so the state is read from and written to HBM exactly once;
+// the next head's state is loaded into shared memory while the current head runs, and the head
+// boundary swaps the two in one pass that also forms the drift partials.  Per tile:
+//   V region  <- V^T                       (MMA: V tile times an identity matrix, exact)
+//   X region  <- S~ K^T                     (tf32 MMA, K exact in fp32)
+//   W pass:   W^T = V^T - sig X diag(gamma), x u_scale -> (hi, lo) in place over X   (chain)
+//   U region  <- W^T T~^T = U~^T / ...      (MMA)
+//   U~ pass:  -> (hi, lo) in place                          (chain)
+//   S~        += U~^T K                     (MMA)
+// so the chain's passes are a few loads, an FMA, a split and a store per element, and the
+// per-token decays ride on the W pass and on T~.
 //
-// Precision.  k, v exact in bfloat16; K K^T exact in fp32.  E += S~ W reads S~ as tf32 (10
-// explicit mantissa bits, truncated) and W is rounded to tf32: errors confined to the delta
-// correction.  B1, B3 and E take two-term bfloat16 splits (x = hi + lo, about 2^-16 relative); the
-// inverse is formed in fp32.  A CPU model of exactly these roundings gives a state error against
-// fp64 of 2.6e-4 at the slowest decay the tests use (4 chunks of 1024 tokens), 5e-6 at a typical
-// one, and drift numerators within 1.1e-4.
+// Precision.  Keys and values are exact in bfloat16.  The state never leaves fp32 inside the
+// tile loop: TMEM holds S~ with S = sig S~, and X reads S~ straight from TMEM as the A operand of
+// a kind::tf32 product; the hardware keeps 10 mantissa bits of S~ (a relative error below 2^-10
+// per element) while K is exact, an error that reaches the state only through the
+// delta correction and decay with it (a CPU simulation of the truncation gives a state error vs
+// fp64 of ~2e-4 at the slowest decay the inputs use, 5e-6 at a typical one).  The other products
+// take a two-term bfloat16 split (x = hi + lo, hi = bf16(x), lo = bf16(x - hi)) of each fp32
+// operand:
+//   V^T I                           exact                                        1 MMA group
+//   X^T  = S~ K^T                   S~ (tf32, from TMEM) K (exact in tf32)       1 MMA group
+//   U~^T = W^T T~^T                  Whi T~hi + Whi T~lo + Wlo T~hi                3 MMA groups
+//   S   += U~^T K                   (U~hi + U~lo) K                              2 MMA groups
+//   K K^T (factor kernel)           exact inputs                                 1 MMA group
+// All products accumulate in fp32 in TMEM.
 //
-// Synchronisation.  Roles hand work to each other through mbarriers only; every wait is bounded
-// (about one second, or the workspace header's override); a wait that runs out records
-// DELTAS_ERR_TIMEOUT, raises a CTA-wide abort flag so the other roles stop waiting, and the CTA
-// drains its MMAs and copies before freeing TMEM.  Heads split between neighbouring CTAs (equal
-// tile runs, see ChainSched) hand the state over through the workspace with a bit per CTA boundary
-// in the workspace header, which its reader clears after use.
+// Deferred decay: the tile decay gamma_C is folded into the scalar sig instead of a pass that
+// multiplies S by gamma_C; the W pass applies sig and scales W by u_scale = 1 / (gamma_C sig) so that
+// MMA_S adds onto S~ directly.  When sig gamma_C would fall below 2^-30 the tile writes
+// gamma_C sig S~ back into TMEM and sig restarts at 1 (u_scale = 1), so 1 / sig stays far from the
+// fp32 range limit.  The head's last tile multiplies by sig when it reads the state out.
 //
-// TMEM (512 columns, 128 lanes): S~ [0,128), S_before [128,256), E0 [256,320), E1 [320,384)
-// (E fp32, then its (hi, lo) A operand in place), K K^T [384,448) (lanes 0..63), Q [448,512).
+// Update-kernel warp roles (19 warps):
+//   0-15  state chain: warp w serves TMEM lanes 32 (w % 4) .. + 31 (state rows) and column group
+//         w / 4; per tile the W and U~ passes (16 token columns each) and the next tile's K in
+//         fp32 (two 16-byte chunks each), at head boundaries the state swap and the drift partials
+//   16    TMEM allocation and every tcgen05.mma (one elected lane issues; the warp stays
+//         converged); it also releases the input buffers by tcgen05.commit
+//   17    tile loads: K, V (TMA) and the WY records (bulk copy), as buffers are released
+//   18    state moves: each head's state into the staging buffer, S_after out of it
+// A TMA or bulk copy occupies the issuing thread for a time that grows with its size, so no copy
+// is issued from a role on the chain's critical path.  Roles hand work to each other through
+// mbarriers only.  Every wait is bounded; a wait that runs out records DELTAS_ERR_TIMEOUT, raises
+// a CTA-wide abort flag so the other roles stop waiting, and the CTA drains its MMAs and copies
+// before freeing TMEM.
+// TMEM (512 columns, M = 128 lanes = d_v): S~ [0,128), S_before [128,256), X [256,320) (X, then
+// W hi / lo packed in place), U [320,384) (likewise U~), V^T [384,448); [448,512) unused.
 #include <algorithm>
 #include <cmath>
 
@@ -74,54 +79,18 @@ using namespace tc;
 
 constexpr int kC = 64;                 // tokens per tile
 constexpr int kD = 128;                // head dim (d_k = d_v)
-constexpr float kHardMin = 0x1p-45f;   // p below this: the state is rescaled by a pass
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kSigMin = 9.313225746154785e-10f;   // 2^-30: smallest deferred decay of the state
 
-// ---- roles
-constexpr int kChainWarps = 4;         // warps 0..3: warp q serves TMEM lanes 32 q ..
-constexpr int kChain = 32 * kChainWarps;
-constexpr int kProdWarp0 = 4;          // warps 4..7: producer group 1 (odd tiles), 8..11: group 0 (even);
-                                       // warp i of a group (i = warp % 4) reads TMEM lanes 32 i ..
-constexpr int kProd = 128;             // threads of a producer group
-constexpr int kMmaWarp = 12;
-constexpr int kLoadWarp = 13;
-constexpr int kThreads = 14 * 32;
-constexpr int kBarChain = 1;           // named barriers: chain, producer group 0, group 1 (128 threads each)
-constexpr int kBarProd = 2;
-
-// ---- TMEM columns
-constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t TM_S = 0, TM_SB = 128, TM_E = 256, TM_KK = 384, TM_Q = 448;
-
-// ---- shared memory (bytes from a 1024-aligned base)
-constexpr int kKSlots = 5;             // K ring: a tile's K K^T is issued three tiles before its state update
-constexpr uint32_t SM_K = 0;           // 5 tiles x 16 KB: 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B, SW128
-constexpr uint32_t SM_V = 81920;       // 16 KB, same layout (also the K K^T product's over-read past the last
-                                       // K tile: rows 64..127 of its M = 128 A)
-constexpr uint32_t SM_B1 = 98304;      // 16 KB: rows t of u N_beta diag(delta): hi in column block 0, lo in
-                                       // block 1 (64 rows x 128 B each, SW128)
-constexpr uint32_t SM_B3 = 114688;     // 16 KB: N_beta, same layout
-constexpr uint32_t SM_W = 131072;      // 32 KB: W^T = -c N_beta K in tf32, rows t: 4 column blocks (32 dims)
-                                       // x 64 rows x 128 B, SW128 (the B operand of E += S~ W)
-constexpr uint32_t SM_PW = 163840;     // producer workspaces, one per group
-// A group's workspace (fp32): rows 0..31 of M = diag(beta) L and of N = (I + diag(beta) L)^-1 hold
-// columns 0..31 only (the rest is above the diagonal), rows 32..63 all 64 columns; the block
-// products; beta, delta and (u, c) of the group's tile, double-buffered (the constants warp writes
-// the group's next tile's while the others may still read this one's).
-constexpr int kTS = 36, kBS = 68, kPS = 36;   // row strides (16-byte aligned rows)
-constexpr int PW_MT = 0, PW_MB = PW_MT + 32 * kTS, PW_NT = PW_MB + 32 * kBS, PW_NB = PW_NT + 32 * kTS,
-              PW_P = PW_NB + 32 * kBS, PW_BETA = PW_P + 32 * kPS, PW_DELTA = PW_BETA + 128, PW_UC = PW_DELTA + 128,
-              PW_FLOATS = PW_UC + 8;
-constexpr uint32_t kPwBytes = PW_FLOATS * 4;
-constexpr uint32_t SM_CONST = SM_PW + 2 * kPwBytes;   // 2 slots x kConstWords: per-tile constants
-constexpr int kConstWords = 72;        // [0,64) write-size scale per token, 64 sig after, 65 pass factor
-                                       // (< 0: none), 66 shift (int), 67 c
-constexpr uint32_t SM_BYTES = SM_CONST + 2 * kConstWords * 4;
-constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
-static_assert(SM_V % 1024 == 0 && SM_B1 % 1024 == 0 && SM_B3 % 1024 == 0 && SM_W % 1024 == 0 &&
-              kPwBytes % 16 == 0 && SM_CONST % 16 == 0, "shared-memory map");
-static_assert(SM_V == SM_K + kKSlots * 16384 && SM_B1 == SM_V + 16384 && SM_B3 == SM_B1 + 16384 &&
-              SM_W == SM_B3 + 16384 && SM_PW == SM_W + 32768, "map order");
-static_assert(kSmemAlloc + 1024 <= 232448, "shared memory budget");
+// ---- WY record of one (layer, value head, tile), written by the factor kernel, read by the update
+// kernel with one bulk copy:
+//   [0, 8192)       T~ hi: bfloat16 [64 t][64 i], 128-byte rows, 128-byte swizzle (K-major B operand)
+//   [8192, 16384)   T~ lo, same layout
+//   [16384, 16656)  float: -gamma[64], gamma_C, 3 unused
+constexpr uint32_t kRecT = 16384;
+constexpr uint32_t kRecConsts = 68;
+constexpr uint32_t kRecBytes = kRecT + kRecConsts * 4;
+static_assert(kRecBytes % 16 == 0, "records are bulk-copied: 16-byte multiples");
 
 // Barrier over `n` threads that also returns the OR of `flag` over them (uniform result).
 __device__ __forceinline__ bool named_sync_or(int id, int n, bool flag) {
@@ -139,8 +108,22 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// (a, b) -> packed bf16 hi = (bf16(a), bf16(b)) and lo = (bf16(a - hi_a), bf16(b - hi_b)), a in the
-// low half (even k low: the packing of a TMEM A operand and of a K-major row)
+// x[0..7] -> hi = bf16(x), lo = bf16(x - hi), 8 packed values each
+__device__ __forceinline__ void split8(const float* x, uint4& hi, uint4& lo) {
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const __nv_bfloat162 hh = __floats2bfloat162_rn(x[2 * i], x[2 * i + 1]);
+        const float2 hf = __bfloat1622float2(hh);
+        h[i] = *reinterpret_cast<const uint32_t*>(&hh);
+        l[i] = pack_bf16x2(x[2 * i] - hf.x, x[2 * i + 1] - hf.y);
+    }
+    hi = make_uint4(h[0], h[1], h[2], h[3]);
+    lo = make_uint4(l[0], l[1], l[2], l[3]);
+}
+
+// (a, b) -> packed bf16 hi = (bf16(a), bf16(b)) and lo = (bf16(a - hi_a), bf16(b - hi_b)),
+// a in the low half (the TMEM A-operand packing: even k low)
 __device__ __forceinline__ void split2(float a, float b, uint32_t& hi, uint32_t& lo) {
     const __nv_bfloat162 hh = __floats2bfloat162_rn(a, b);
     const float2 hf = __bfloat1622float2(hh);
@@ -148,17 +131,10 @@ __device__ __forceinline__ void split2(float a, float b, uint32_t& hi, uint32_t&
     lo = pack_bf16x2(a - hf.x, b - hf.y);
 }
 
-// fp32 -> tf32 with round-to-nearest (ties away), as the 32-bit container the tensor core reads
-__device__ __forceinline__ uint32_t to_tf32(float x) {
-    uint32_t y;
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(y) : "f"(x));
-    return y;
-}
-
-// D (16 x 8) += A (16 x 16, row-major) B (16 x 8) on the warp's tensor-core path, bf16 in, fp32
+// D (16 x 8) += A (16 x 16, row) B (16 x 8, col) on the warp's tensor-core path, bf16 in, fp32
 // accumulate.  Fragments (g = lane / 4, t = lane % 4), each register a bf16 pair, lower k in the
 // low half: a = A[g][2t..], A[g+8][2t..], A[g][2t+8..], A[g+8][2t+8..]; b = B[2t..][g],
-// B[2t+8..][g]; d = D[g][2t, 2t+1], D[g+8][2t, 2t+1].
+// B[2t+8..][g]; d as for the tf32 form.
 __device__ __forceinline__ void mma_m16n8k16_bf16(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
     asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
                  "{%0,%1,%2,%3};"
@@ -166,165 +142,550 @@ __device__ __forceinline__ void mma_m16n8k16_bf16(float (&d)[4], const uint32_t 
                  : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
-// D (16 x 8) += A (16 x 16 KS) B (16 KS x 8) for fp32 operands in shared memory (A row-major with
-// row stride lda, B row-major B[k][n] with row stride ldb), each split into bfloat16 (hi, lo) in
-// registers and multiplied as lo hi + hi lo + hi hi (about 2^-16 relative error per product).
-template <int KS>
-__device__ __forceinline__ void mma_f32_split(float (&d)[4], const float* A, int lda, const float* B, int ldb,
-                                              int g, int t) {
-    // the three products accumulate separately (independent chains), summed at the end
-    float d1[4] = {0.f, 0.f, 0.f, 0.f}, d2[4] = {0.f, 0.f, 0.f, 0.f};
+// Operands stored split: row r of A is at A + r * as (32-bit words), its word p the bf16 pair of
+// hi = bf16(x) for columns (2p, 2p+1) and word a_lo + p the pair of lo = bf16(x - hi); likewise B,
+// stored n-major (row n of B's storage holds column n of B).  D (16 x 8) += A[r0 .. r0+15][0..16K)
+// B[0..16K)[n0 .. n0+7] over the three products lo*hi + hi*lo + hi*hi.
+template <int KSTEPS>
+__device__ __forceinline__ void mma_split_bf16(float (&d)[4], const uint32_t* A, int as, int a_lo, int r0,
+                                               const uint32_t* B, int bs, int b_lo, int n0, int lane) {
+    const int g = lane >> 2, t = lane & 3;
+    const uint32_t* a0 = A + (r0 + g) * as;
+    const uint32_t* a1 = A + (r0 + g + 8) * as;
+    const uint32_t* b0 = B + (n0 + g) * bs;
 #pragma unroll
-    for (int ks = 0; ks < KS; ++ks) {
-        const float* a0 = A + g * lda + 16 * ks + 2 * t;
-        const float2 x0 = *reinterpret_cast<const float2*>(a0);
-        const float2 x1 = *reinterpret_cast<const float2*>(a0 + 8 * lda);
-        const float2 x2 = *reinterpret_cast<const float2*>(a0 + 8);
-        const float2 x3 = *reinterpret_cast<const float2*>(a0 + 8 * lda + 8);
-        const float* b0 = B + (16 * ks + 2 * t) * ldb + g;
-        uint32_t ah[4], al[4], bh[2], bl[2];
-        split2(x0.x, x0.y, ah[0], al[0]);
-        split2(x1.x, x1.y, ah[1], al[1]);
-        split2(x2.x, x2.y, ah[2], al[2]);
-        split2(x3.x, x3.y, ah[3], al[3]);
-        split2(b0[0], b0[ldb], bh[0], bl[0]);
-        split2(b0[8 * ldb], b0[9 * ldb], bh[1], bl[1]);
-        mma_m16n8k16_bf16(d1, al, bh);
-        mma_m16n8k16_bf16(d2, ah, bl);
+    for (int ks = 0; ks < KSTEPS; ++ks) {
+        const int p0 = 8 * ks + t, p1 = p0 + 4;
+        const uint32_t ah[4] = {a0[p0], a1[p0], a0[p1], a1[p1]};
+        const uint32_t al[4] = {a0[a_lo + p0], a1[a_lo + p0], a0[a_lo + p1], a1[a_lo + p1]};
+        const uint32_t bh[2] = {b0[p0], b0[p1]};
+        const uint32_t bl[2] = {b0[b_lo + p0], b0[b_lo + p1]};
+        mma_m16n8k16_bf16(d, al, bh);
+        mma_m16n8k16_bf16(d, ah, bl);
         mma_m16n8k16_bf16(d, ah, bh);
     }
+}
+
+// One element of a split row (see mma_split_bf16): hi / lo halfwords of column k; lo words start
+// lo_words after the row's first word.
+__device__ __forceinline__ void put_split(uint32_t* row, int k, float x, int lo_words = 16) {
+    const __nv_bfloat16 h = __float2bfloat16_rn(x);
+    const __nv_bfloat16 l = __float2bfloat16_rn(x - __bfloat162float(h));
+    reinterpret_cast<__nv_bfloat16*>(row)[k] = h;
+    reinterpret_cast<__nv_bfloat16*>(row + lo_words)[k] = l;
+}
+
+// 16 consecutive values -> split row of a 16-column operand (words 0..7 hi, 8..15 lo)
+__device__ __forceinline__ void put_split16(uint32_t* row, const float* x) {
+    uint32_t h[8], l[8];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) d[i] += d1[i] + d2[i];
+    for (int i = 0; i < 8; ++i) split2(x[2 * i], x[2 * i + 1], h[i], l[i]);
+    *reinterpret_cast<uint4*>(row) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4*>(row + 4) = make_uint4(h[4], h[5], h[6], h[7]);
+    *reinterpret_cast<uint4*>(row + 8) = make_uint4(l[0], l[1], l[2], l[3]);
+    *reinterpret_cast<uint4*>(row + 12) = make_uint4(l[4], l[5], l[6], l[7]);
 }
 
-// One kind::f16 MMA from TMEM A that scales the accumulator it reads by 2^-shift (the
-// instruction's scale-input-d operand, an immediate: D = A B + 2^-shift D), shift in [0, 15].
-template <int S>
-__device__ __forceinline__ void mma_bf16_ta_scaled(uint32_t d, uint32_t a, uint64_t b, uint32_t idesc) {
-    asm volatile("{\n\t.reg .pred q;\n\t"
-                 "setp.eq.b32 q, %3, %3;\n\t"
-                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, q, %4;\n\t}"
-                 :: "r"(d), "r"(a), "l"(b), "r"(idesc), "n"(S) : "memory");
-}
-__device__ __noinline__ void mma_bf16_ta_shift_1t(int shift, uint32_t d, uint32_t a, uint64_t b, uint32_t idesc) {
-    switch (shift) {
-        case 0: mma_bf16_ta_scaled<0>(d, a, b, idesc); break;
-        case 1: mma_bf16_ta_scaled<1>(d, a, b, idesc); break;
-        case 2: mma_bf16_ta_scaled<2>(d, a, b, idesc); break;
-        case 3: mma_bf16_ta_scaled<3>(d, a, b, idesc); break;
-        case 4: mma_bf16_ta_scaled<4>(d, a, b, idesc); break;
-        case 5: mma_bf16_ta_scaled<5>(d, a, b, idesc); break;
-        case 6: mma_bf16_ta_scaled<6>(d, a, b, idesc); break;
-        case 7: mma_bf16_ta_scaled<7>(d, a, b, idesc); break;
-        case 8: mma_bf16_ta_scaled<8>(d, a, b, idesc); break;
-        case 9: mma_bf16_ta_scaled<9>(d, a, b, idesc); break;
-        case 10: mma_bf16_ta_scaled<10>(d, a, b, idesc); break;
-        case 11: mma_bf16_ta_scaled<11>(d, a, b, idesc); break;
-        case 12: mma_bf16_ta_scaled<12>(d, a, b, idesc); break;
-        case 13: mma_bf16_ta_scaled<13>(d, a, b, idesc); break;
-        case 14: mma_bf16_ta_scaled<14>(d, a, b, idesc); break;
-        default: mma_bf16_ta_scaled<15>(d, a, b, idesc); break;
-    }
+// 2^x with the hardware approximation (relative error about 2^-22)
+__device__ __forceinline__ float fast_exp2(float x) {
+    float y;
+    asm("ex2.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
 
-// The waits of this kernel: one try inline, the bounded loop out of line (the kernel's code must
-// stay small: every role's loop shares the SM's instruction cache, and misses are served from a
-// busy L2).
-__device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
-                                       const volatile int* abort) {
-    const long long t0 = clock64();
-    const long long budget = (long long)(budget_ns * 2);
-    for (;;) {
-        if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
-        if (*abort) return false;
-        if (clock64() - t0 > budget) return false;
-    }
-}
-__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
-                                         const volatile int* abort) {
-    if (mbar_try_wait(bar, parity)) return true;
-    return wait_slow(bar, parity, budget_ns, abort);
-}
-
-// All lanes of a converged warp wait; the result is the same on every lane.
+// All lanes of a converged warp wait; the result is the same on every lane (false if any lane's
+// wait ran out), so the warp stays converged for the elect.sync that follows.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
                                           const volatile int* abort) {
-    const bool ok = wait_bar(bar, parity, budget_ns, abort);
+    const bool ok = mbar_wait_or_abort(bar, parity, budget_ns, abort);
     return __all_sync(0xffffffffu, ok) != 0;
 }
 
-__device__ __noinline__ void fail(int32_t* status, volatile int* abort, int where) {
+__device__ __forceinline__ void fail(int32_t* status, volatile int* abort, int where) {
     record_status(status, DELTAS_ERR_TIMEOUT, where);
     *abort = 1;
 }
 
-// One arrival per warp: every lane's TMEM stores / shared-memory writes were completed and fenced
-// before the __syncwarp; lane 0 then arrives (release).
+// One arrival per warp on a chain -> MMA barrier: every lane's TMEM stores / shared-memory
+// writes were completed and fenced before the __syncwarp; lane 0 then arrives (release).
 __device__ __forceinline__ void warp_arrive(uint64_t* bar, int lane) {
     __syncwarp();
     if (lane == 0) mbar_arrive(bar);
 }
 
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
-    uint32_t v;
+// shared-memory descriptor advanced by `bytes` (the start address field counts 16-byte units)
+__device__ __forceinline__ uint64_t dadd(uint64_t desc, uint32_t bytes) { return desc + (uint64_t)(bytes >> 4); }
+
+// =============================================================================================
+// Factor kernel: T~ = diag(exp(G_C - G)) (I + A)^-1 diag(beta) and the decay constants of every tile
+// =============================================================================================
+constexpr int kWyThreads = 256;
+constexpr int kWyCtasPerSm = 4;
+constexpr uint32_t kWyTmemCols = 64;
+constexpr int FA_S = 68;               // fp32 row stride of A: 16-byte rows; a 16-byte access by 8 threads
+                                       // of 8 consecutive rows hits 8 distinct bank groups
+constexpr int FX_S = 68;               // fp32 row stride of X = (I + A)^-1 (16-byte aligned rows)
+// shared-memory map (bytes from a 1024-aligned base)
+constexpr uint32_t WY_FA = 0;                         // fp32 [64][FA_S].  Its two 32 x 32 quarters that are
+                                                      // never read as fp32 hold split operands of level 2:
+                                                      // rows 32..63 x cols 0..31 = A21 (row-major), rows
+                                                      // 0..31 x cols 32..63 = X11 stored n-major
+constexpr uint32_t WY_K = WY_FA;                      // the next item's K tile (2 column blocks (d 0-63,
+                                                      // 64-127) x 64 rows x 128 B) lands over A once level 2
+                                                      // has read it; the M = 128 product of K K^T reads the
+                                                      // 8 KB past the tile as rows 64..127 (output ignored)
+constexpr uint32_t WY_FX = WY_FA + 64 * FA_S * 4;     // fp32 [64][FX_S]; rows 0..31 x cols 32..63 (the zero
+                                                      // upper quarter) hold X22 split, row-major
+constexpr uint32_t WY_TMP = WY_FX + 64 * FX_S * 4;    // level 1 products (fp32), then level 2's P split,
+                                                      // n-major, rows of 36 words
+constexpr uint32_t WY_L1 = WY_TMP + 32 * 36 * 4;      // level-1 split operands, 6 x 16 rows of 20 words: A10,
+                                                      // A32, X11' (row-major), X22' (n-major), P1 for p = 0, 1
+constexpr int kL1S = 20;                              // row stride (words): fragment loads hit distinct banks
+constexpr uint32_t WY_TG = WY_L1 + 6 * 16 * kL1S * 4; // 2 buffers (item parity) x (G2[64], beta[64], row[64],
+                                                      // col[64], del[64], flag)
+constexpr uint32_t kTgFloats = 324;
+constexpr uint32_t WY_BYTES = WY_TG + 2 * kTgFloats * 4;
+constexpr uint32_t kWySmemAlloc = WY_BYTES + 1024;
+static_assert(WY_TG % 16 == 0 && (kTgFloats * 4) % 16 == 0, "tile factors must be 16-byte aligned");
+static_assert(kWyCtasPerSm * (kWySmemAlloc + 1024) <= 233472, "factor kernel: CTAs per SM");
+
+struct WyArgs {
+    int L, Hk, Hv, T, n_tiles;
+    const float* g;
+    const float* beta;
+    uint8_t* rec;              // [L * Hv][n_tiles] records of kRecBytes
+    int32_t* status;
+    int32_t* ho_flags;         // the update kernel's hand-over flags, reset here for this call
+    int n_ho_flags;
+};
+
+__global__ void __launch_bounds__(kWyThreads, kWyCtasPerSm)
+gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    __shared__ uint64_t mb_k, mb_kk;
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_fail;
+    grid_dep_launch();                                // the update kernel may take SMs as they free up
+    // the update kernel reads its hand-over flags only after this kernel has completed
+    if (blockIdx.x == 0)
+        for (int e = (int)threadIdx.x; e < a.n_ho_flags; e += kWyThreads) a.ho_flags[e] = 0;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int n = a.n_tiles;
+    const int items = a.L * a.Hv * n;                 // item = (layer * Hv + head) * n + tile
+    float* fA = reinterpret_cast<float*>(sm + WY_FA);
+    float* fX = reinterpret_cast<float*>(sm + WY_FX);
+    float* fT = reinterpret_cast<float*>(sm + WY_TMP);
+    // split level-2 operands (see the shared-memory map), row strides in 32-bit words
+    uint32_t* sA21 = reinterpret_cast<uint32_t*>(fA + 32 * FA_S);        // A[32 + r][k]
+    uint32_t* sX11 = reinterpret_cast<uint32_t*>(fA + 32);               // row n: X[k][n], k < 32
+    uint32_t* sX22 = reinterpret_cast<uint32_t*>(fX + 32);               // row r: X[32 + r][32 + k]
+    uint32_t* sP = reinterpret_cast<uint32_t*>(fT);                      // row n: P[k][n]
+    constexpr int kPS = 36;
+    // split level-1 operands: 16 x 16 blocks, rows of kL1S words (hi words 0..7, lo words 8..15)
+    uint32_t* sL1 = reinterpret_cast<uint32_t*>(sm + WY_L1);
+    uint32_t* sA10 = sL1;                                                 // A[16 + r][k]
+    uint32_t* sA32 = sL1 + 16 * kL1S;                                     // A[48 + r][32 + k]
+    uint32_t* sX11r = sL1 + 32 * kL1S;                                    // X[16 + r][16 + k]
+    uint32_t* sX22n = sL1 + 48 * kL1S;                                    // row n: X[32 + k][32 + n]
+    uint32_t* sP1 = sL1 + 64 * kL1S;                                      // p: row n of P1_p, 16 rows each
+
+    if (warp == 0) { tmem_alloc(&s_tmem, kWyTmemCols); tmem_relinquish(); }
+    if (tid == 0) {
+        mbar_init(&mb_k, 1); mbar_init(&mb_kk, 1);
+        fence_barrier_init();
+        prefetch_tensormap(&kmap);
+        s_fail = 0;
+    }
+    // The strictly upper 16 x 16 blocks of X are never written; zeros there let every level run
+    // fixed-length (unrolled) loops over the triangular factors.
+    for (int e = tid; e < 64 * FX_S; e += kWyThreads) { fX[e] = 0.f; fA[e] = 0.f; }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = s_tmem;
+
+    // Items are taken in reverse record order: the records written last, still in L2 when this
+    // kernel ends, are the ones of the lowest heads, which the update kernel reads first.
+    auto rec_of = [&](int it) { return items - 1 - it; };
+    auto item_pos = [&](int it, int& l, int& h, int& jt) {
+        const int r = rec_of(it), lh = r / n;
+        jt = r - lh * n; l = lh / a.Hv; h = lh - l * a.Hv;
+    };
+    int nk = 0, nkk = 0;                               // K loads (thread 0) / K K^T products (warp 0) issued
+    auto load_k = [&](int it) {                        // thread 0: the item's K tile
+        int l, h, jt;
+        item_pos(it, l, h, jt);
+        ++nk;
+        const int kh = (int)(((long long)h * a.Hk) / a.Hv);
+        mbar_arrive_expect_tx(&mb_k, 16384);
+        tma_load_4d(sm + WY_K, &kmap, &mb_k, 0, kh, jt * kC, l);
+        tma_load_4d(sm + WY_K + 8192, &kmap, &mb_k, 64, kh, jt * kC, l);
+    };
+    // g and beta of an item's 64 tokens, two per lane of warp 7, loaded one item ahead of use
+    float pg[2] = {0.f, 0.f}, pb[2] = {0.f, 0.f};
+    auto load_gb = [&](int it) {
+        int l, h, jt;
+        item_pos(it, l, h, jt);
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int t = jt * kC + 2 * lane + e;
+            const size_t gi = ((size_t)l * a.T + t) * a.Hv + h;
+            pg[e] = t < a.T ? a.g[gi] : 0.f;
+            pb[e] = t < a.T ? a.beta[gi] : 0.f;
+        }
+    };
+    // Decay constants of an item from the loaded g, beta (warp 7): the update kernel's -gamma and
+    // gamma_C into the record, and this kernel's G2, beta, row and column factors and
+    // exp(G_C - G) into buffer `buf`.
+    auto tile_constants = [&](int it, int buf) {
+        float incl = pg[0] + pg[1];
+#pragma unroll
+        for (int m = 1; m < 32; m <<= 1) {
+            const float y = __shfl_up_sync(0xffffffffu, incl, m);
+            if (lane >= m) incl += y;
+        }
+        const float G0 = incl - pg[1], G1 = incl;
+        const float GC = __shfl_sync(0xffffffffu, incl, 31);
+        float* rc = reinterpret_cast<float*>(a.rec + (size_t)rec_of(it) * kRecBytes + kRecT);
+        *reinterpret_cast<float2*>(rc + 2 * lane) = make_float2(-expf(G0), -expf(G1));
+        if (lane == 0) *reinterpret_cast<float4*>(rc + 64) = make_float4(expf(GC), 0.f, 0.f, 0.f);
+        const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
+        float lo2 = fminf(g20, g21), hi2 = fmaxf(g20, g21);
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) {
+            lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, m));
+            hi2 = fmaxf(hi2, __shfl_xor_sync(0xffffffffu, hi2, m));
+        }
+        // exp(G_t - G_i) = row_t * col_i with the reference in the middle of the tile's range of
+        // G; both factors stay within 2^+-126 when that range spans at most 250 powers of two,
+        // otherwise the exponent is taken per entry.
+        const float ref = 0.5f * (lo2 + hi2);
+        float* tg = reinterpret_cast<float*>(sm + WY_TG) + buf * kTgFloats;
+        tg[2 * lane] = g20; tg[2 * lane + 1] = g21;
+        tg[64 + 2 * lane] = pb[0]; tg[64 + 2 * lane + 1] = pb[1];
+        tg[128 + 2 * lane] = pb[0] * fast_exp2(g20 - ref); tg[128 + 2 * lane + 1] = pb[1] * fast_exp2(g21 - ref);
+        tg[192 + 2 * lane] = fast_exp2(ref - g20); tg[192 + 2 * lane + 1] = fast_exp2(ref - g21);
+        tg[256 + 2 * lane] = expf(GC - G0); tg[256 + 2 * lane + 1] = expf(GC - G1);
+        if (lane == 0) reinterpret_cast<int*>(tg)[320] = (hi2 - lo2) <= 250.f;
+    };
+
+    // K K^T of the item-th item of this CTA into TMEM (warp 0; M = 128: rows 64..127 of A read the
+    // 8 KB past the tile, their output is ignored)
+    auto issue_kk = [&](int item) {
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&mb_k, item & 1, kWaitBudgetNs)) != 0;
+        if (!ok) {
+            if (lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 21); s_fail = 1; }
+            return;
+        }
+        tc_fence_after();
+        const uint32_t id = idesc_bf16(128, 64, 0, 0);
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {
+            const uint64_t d = sdesc_sw128(smem_u32(sm + WY_K + (s >> 2) * 8192 + (s & 3) * 32), 16, 1024);
+            mma_bf16(tm, d, d, id, s > 0);
+        }
+        mma_commit(&mb_kk);
+        ++nkk;
+    };
+
+    const int first = (int)blockIdx.x;
+    if (first < items) {
+        if (tid == 0) load_k(first);
+        if (warp == 7) {
+            load_gb(first);
+            tile_constants(first, 0);
+            if (first + (int)gridDim.x < items) load_gb(first + (int)gridDim.x);
+        }
+    }
+    __syncthreads();
+    int c = 0;                                         // items done by this CTA (barrier phases)
+    for (int it = first; it < items; it += (int)gridDim.x, ++c) {
+        const float* tg = reinterpret_cast<const float*>(sm + WY_TG) + (c & 1) * kTgFloats;
+        const float* sG2 = tg;                         // G * log2(e)
+        const float* sBeta = tg + 64;
+        const float* sRow = tg + 128;                  // beta_t 2^(G2_t - ref)
+        const float* sCol = tg + 192;                  // 2^(ref - G2_i)
+        const float* sDel = tg + 256;                  // exp(G_C - G_t)
+        const int factored = reinterpret_cast<const int*>(tg)[320];
+        if (warp == 0) issue_kk(c);
+        const int q = warp & 3;
+        if (q < 2 && warp != 4) {
+            // TMEM lanes 0..63 hold K K^T: warps 0/4 rows 0..31, 1/5 rows 32..63; column half
+            // (warp >> 2).  Warp 4's quarter (rows 0..31, cols 32..63) lies above the diagonal and
+            // is never needed; warp 1's (rows 32..63, cols 0..31) is A21, stored split.
+            const bool ok = mbar_wait_or_abort(&mb_kk, c & 1, kWaitBudgetNs, &s_fail);
+            if (!ok && lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 22); s_fail = 1; }
+            tc_fence_after();
+            const int t = 32 * q + lane, c0 = 32 * (warp >> 2);
+            const uint32_t lane_off = (uint32_t)(32 * q) << 16;
+            const float rt = factored ? sRow[t] : sBeta[t];
+            const float G2t = sG2[t];
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {     // 16 columns at a time
+                const int cb = c0 + 16 * half;
+                float kk[16], cf[16];
+                tmem_ld16(tm + lane_off + cb, kk);
+                const float* src = factored ? sCol : sG2;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float4 v4 = *reinterpret_cast<const float4*>(src + cb + 4 * e);
+                    cf[4 * e] = v4.x; cf[4 * e + 1] = v4.y; cf[4 * e + 2] = v4.z; cf[4 * e + 3] = v4.w;
+                }
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const float f = factored ? cf[e] : fast_exp2(G2t - cf[e]);
+                    kk[e] = (cb + e < t) ? rt * f * kk[e] : 0.f;
+                }
+                if (half == 0 && lane >= 16 && (warp == 0 || warp == 5))   // A10 / A32, split
+                    put_split16((warp == 0 ? sA10 : sA32) + (lane - 16) * kL1S, kk);
+                if (warp == 1) {                       // A21, split
+                    uint32_t* row = sA21 + (t - 32) * FA_S + 8 * half;
+                    uint32_t h[8], l[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) split2(kk[2 * i], kk[2 * i + 1], h[i], l[i]);
+                    *reinterpret_cast<uint4*>(row) = make_uint4(h[0], h[1], h[2], h[3]);
+                    *reinterpret_cast<uint4*>(row + 4) = make_uint4(h[4], h[5], h[6], h[7]);
+                    *reinterpret_cast<uint4*>(row + 16) = make_uint4(l[0], l[1], l[2], l[3]);
+                    *reinterpret_cast<uint4*>(row + 20) = make_uint4(l[4], l[5], l[6], l[7]);
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        *reinterpret_cast<float4*>(fA + t * FA_S + cb + 4 * e) =
+                            make_float4(kk[4 * e], kk[4 * e + 1], kk[4 * e + 2], kk[4 * e + 3]);
+                }
+            }
+        }
+        tc_fence_before();
+        __syncthreads();
+        if (s_fail) break;
+        const int nxt = it + (int)gridDim.x;
+        // level 0: four 16 x 16 diagonal blocks of (I + A)^-1, one column per thread (warps 0-1);
+        // meanwhile warp 7 prepares the next item's constants and loads the one after
+        if (tid < 64) {
+            const int B = tid >> 4, jc = tid & 15, o = 16 * B;
+            float x[16];
+#pragma unroll
+            for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
+#pragma unroll
+            for (int rr = 1; rr < 16; ++rr) {
+                float s0 = 0.f, s1 = 0.f;              // two chains: half the dependent FMAs
+#pragma unroll
+                for (int cc = 0; cc < rr; cc += 4) {
+                    const float4 av = *reinterpret_cast<const float4*>(fA + (o + rr) * FA_S + o + cc);
+                    s0 = fmaf(av.x, x[cc], s0);
+                    if (cc + 1 < rr) s1 = fmaf(av.y, x[cc + 1], s1);
+                    if (cc + 2 < rr) s0 = fmaf(av.z, x[cc + 2], s0);
+                    if (cc + 3 < rr) s1 = fmaf(av.w, x[cc + 3], s1);
+                }
+                if (rr > jc) x[rr] = -(s0 + s1);
+            }
+#pragma unroll
+            for (int rr = 0; rr < 16; ++rr) fX[(o + rr) * FX_S + o + jc] = x[rr];
+            if (B == 1) {                              // X11' row-major
+#pragma unroll
+                for (int rr = 0; rr < 16; ++rr) put_split(sX11r + rr * kL1S, jc, x[rr], 8);
+            } else if (B == 2) {                       // X22' n-major
+                put_split16(sX22n + jc * kL1S, x);
+            }
+            if (B < 2) {                               // X11, n-major: row o + jc holds column o + jc
+                uint32_t* row = sX11 + (o + jc) * FA_S;
+                if (B == 1) {                          // X[0..16][16..32] = 0 (the K tile overwrote it)
+                    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+                    *reinterpret_cast<uint4*>(row) = z; *reinterpret_cast<uint4*>(row + 4) = z;
+                    *reinterpret_cast<uint4*>(row + 16) = z; *reinterpret_cast<uint4*>(row + 20) = z;
+                }
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    uint32_t h[4], l[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) split2(x[8 * e + 2 * i], x[8 * e + 2 * i + 1], h[i], l[i]);
+                    *reinterpret_cast<uint4*>(row + o / 2 + 4 * e) = make_uint4(h[0], h[1], h[2], h[3]);
+                    *reinterpret_cast<uint4*>(row + 16 + o / 2 + 4 * e) = make_uint4(l[0], l[1], l[2], l[3]);
+                }
+            } else {                                   // X22, row-major
+#pragma unroll
+                for (int rr = 0; rr < 16; ++rr) put_split(sX22 + (o - 32 + rr) * FX_S, o - 32 + jc, x[rr]);
+            }
+        } else if (warp == 7 && nxt < items) {
+            tile_constants(nxt, (c + 1) & 1);
+            if (nxt + (int)gridDim.x < items) load_gb(nxt + (int)gridDim.x);
+        }
+        __syncthreads();
+        // level 1: X[2p+1][2p] = -X[2p+1][2p+1] (A[2p+1][2p] X[2p][2p]) for the 16 x 16 blocks,
+        // p = 0, 1; warps 0-3 take (p, 8-column half) = (warp / 2, warp % 2)
+        const int g = lane >> 2, tq = lane & 3;
+        if (warp < 4) {
+            const int p = warp >> 1, nc = 8 * (warp & 1);
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            if (p == 0) mma_split_bf16<1>(d, sA10, kL1S, 8, 0, sX11, FA_S, 16, nc, lane);    // A10 X00
+            else        mma_split_bf16<1>(d, sA32, kL1S, 8, 0, sX22n, kL1S, 8, nc, lane);   // A32 X22'
+            uint32_t* P = sP1 + p * 16 * kL1S;         // n-major
+            put_split(P + (nc + 2 * tq) * kL1S, g, d[0], 8);
+            put_split(P + (nc + 2 * tq + 1) * kL1S, g, d[1], 8);
+            put_split(P + (nc + 2 * tq) * kL1S, g + 8, d[2], 8);
+            put_split(P + (nc + 2 * tq + 1) * kL1S, g + 8, d[3], 8);
+        }
+        __syncthreads();
+        if (warp < 4) {
+            const int p = warp >> 1, nc = 8 * (warp & 1);
+            const int ro = 16 * (2 * p + 1), co = 16 * (2 * p);
+            const uint32_t* P = sP1 + p * 16 * kL1S;
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            if (p == 0) mma_split_bf16<1>(d, sX11r, kL1S, 8, 0, P, kL1S, 8, nc, lane);        // X11' P1
+            else        mma_split_bf16<1>(d, sX22 + 16 * FX_S + 8, FX_S, 16, 0, P, kL1S, 8, nc, lane);  // X33' P1'
+            fX[(ro + g) * FX_S + co + nc + 2 * tq] = -d[0]; fX[(ro + g) * FX_S + co + nc + 2 * tq + 1] = -d[1];
+            fX[(ro + g + 8) * FX_S + co + nc + 2 * tq] = -d[2]; fX[(ro + g + 8) * FX_S + co + nc + 2 * tq + 1] = -d[3];
+            if (p == 0) {                              // X[16..32][0..16] into X11, n-major
+                put_split(sX11 + (nc + 2 * tq) * FA_S, 16 + g, -d[0]);
+                put_split(sX11 + (nc + 2 * tq + 1) * FA_S, 16 + g, -d[1]);
+                put_split(sX11 + (nc + 2 * tq) * FA_S, 24 + g, -d[2]);
+                put_split(sX11 + (nc + 2 * tq + 1) * FA_S, 24 + g, -d[3]);
+            } else {                                   // X[48..64][32..48] into X22, row-major
+                put_split(sX22 + (16 + g) * FX_S, nc + 2 * tq, -d[0]);
+                put_split(sX22 + (16 + g) * FX_S, nc + 2 * tq + 1, -d[1]);
+                put_split(sX22 + (24 + g) * FX_S, nc + 2 * tq, -d[2]);
+                put_split(sX22 + (24 + g) * FX_S, nc + 2 * tq + 1, -d[3]);
+            }
+        }
+        __syncthreads();
+        // level 2: X[32:64][0:32] = -X[32:64][32:64] (A[32:64][0:32] X[0:32][0:32]) from the split
+        // operands; warp w takes the 16 x 8 output tile (w / 4, w % 4).  P = A21 X11 goes to fT
+        // split and n-major.
+        {
+            const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            mma_split_bf16<2>(d, sA21, FA_S, 16, mr, sX11, FA_S, 16, nc, lane);
+            put_split(sP + (nc + 2 * tq) * kPS, mr + g, d[0]);
+            put_split(sP + (nc + 2 * tq + 1) * kPS, mr + g, d[1]);
+            put_split(sP + (nc + 2 * tq) * kPS, mr + g + 8, d[2]);
+            put_split(sP + (nc + 2 * tq + 1) * kPS, mr + g + 8, d[3]);
+        }
+        __syncthreads();
+        // A (fp32 and split) has been read for the last time: the next item's K tile lands there
+        if (tid == 0 && nxt < items) load_k(nxt);
+        {
+            const int mr = 16 * (warp >> 2), nc = 8 * (warp & 3);
+            float d[4] = {0.f, 0.f, 0.f, 0.f};
+            mma_split_bf16<2>(d, sX22, FX_S, 16, mr, sP, kPS, 16, nc, lane);
+            fX[(32 + mr + g) * FX_S + nc + 2 * tq] = -d[0]; fX[(32 + mr + g) * FX_S + nc + 2 * tq + 1] = -d[1];
+            fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq] = -d[2]; fX[(32 + mr + g + 8) * FX_S + nc + 2 * tq + 1] = -d[3];
+        }
+        __syncthreads();
+        // T~ = diag(exp(G_C - G)) X diag(beta) (upper part zero), split into the record's (hi, lo)
+        // images
+        {
+            uint8_t* rec = a.rec + (size_t)rec_of(it) * kRecBytes;
+#pragma unroll
+            for (int m = 0; m < 2; ++m) {
+                const int e = tid + kWyThreads * m;
+                const int t = e >> 3, c8 = e & 7;
+                uint4 vh = make_uint4(0u, 0u, 0u, 0u), vl = vh;
+                if (8 * c8 <= t) {                     // chunks right of the diagonal stay zero
+                    const float dt = sDel[t];
+                    const float4 x0 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8);
+                    const float4 x1 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8 + 4);
+                    const float4 b0 = *reinterpret_cast<const float4*>(sBeta + 8 * c8);
+                    const float4 b1 = *reinterpret_cast<const float4*>(sBeta + 8 * c8 + 4);
+                    const float xs[8] = {x0.x * b0.x, x0.y * b0.y, x0.z * b0.z, x0.w * b0.w,
+                                         x1.x * b1.x, x1.y * b1.y, x1.z * b1.z, x1.w * b1.w};
+                    float x[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) x[k] = (8 * c8 + k <= t) ? dt * xs[k] : 0.f;
+                    split8(x, vh, vl);
+                }
+                *reinterpret_cast<uint4*>(rec + sw128_offset(t, c8)) = vh;
+                *reinterpret_cast<uint4*>(rec + 8192 + sw128_offset(t, c8)) = vl;
+            }
+        }
+        // the next item's level 0 rewrites fX's diagonal blocks: everyone has read this one's
+        __syncthreads();
+    }
+    if (tid == 0 && s_fail) {
+        // after a failure: the last K load and K K^T product issued land before TMEM is freed
+        if (nk > 0) mbar_wait(&mb_k, (nk - 1) & 1, kWaitBudgetNs);
+        if (nkk > 0) mbar_wait(&mb_kk, (nkk - 1) & 1, kWaitBudgetNs);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tm, kWyTmemCols);
+    }
+}
+
+// =============================================================================================
+// Update kernel: the state chain
+// =============================================================================================
+__device__ __forceinline__ int ho_load_acquire(const int32_t* p) {
+    int v;
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
-
-__device__ __forceinline__ void prefetch_l2(const void* p) {
-    asm volatile("prefetch.global.L2 [%0];" :: "l"(p) : "memory");
+__device__ __forceinline__ void ho_store_release(int32_t* p, int v) {
+    asm volatile("st.release.gpu.global.b32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+// orders the tensor copies' global accesses with the generic ones around a hand-over flag
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" :: "l"(p), "r"(bytes) : "memory");
-}
+constexpr int kChainWarps = 16;
+constexpr int kChain = 32 * kChainWarps;         // chain threads
+constexpr int kMmaWarp = kChainWarps;            // 16
+constexpr int kLoadWarp = kChainWarps + 1;       // 17
+constexpr int kStateWarp = kChainWarps + 2;      // 18
+constexpr int kThreads = kChain + 96;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t TM_S = 0, TM_SB = 128, TM_X = 256, TM_U = 320, TM_V = 384;
 
-// The per-tile decay bookkeeping (see the header): from p = gamma_C sig, the shift s, the scale u
-// of the V term, the coefficient c of the state term, the pass factor (< 0: no pass) and sig after
-// the tile.
-struct DecayStep {
-    int shift;
-    float u, c, pass, sig;
-};
-__device__ __forceinline__ DecayStep decay_step(float p) {
-    DecayStep d;
-    if (!(p >= kHardMin)) {
-        d.shift = 0; d.u = 1.f; d.c = p; d.pass = p; d.sig = 1.f;
-        return d;
-    }
-    int e;
-    (void)frexpf(p, &e);                               // p = m 2^e, m in [1/2, 1)
-    d.shift = min(15, max(0, -e));
-    d.sig = ldexpf(p, d.shift);
-    d.u = 1.f / d.sig;
-    d.c = ldexpf(1.f, -d.shift);
-    d.pass = -1.f;
-    return d;
+// shared-memory map (bytes from a 1024-aligned base)
+constexpr uint32_t SM_K = 0;                     // 3 x 16 KB: K tile, 2 column blocks (d 0-63, 64-127) x 64 rows x 128 B
+constexpr uint32_t SM_K32 = 49152;               // 32 KB: K in fp32 (the B operand of X), 4 column blocks
+                                                 // (32 dims) x 64 rows x 128 B, SW128
+constexpr uint32_t SM_V = 81920;                 // 2 x 16 KB: V tile (tile parity), layout of K
+constexpr uint32_t SM_R = 114688;                // 2 x kRecSlot: WY records (tile parity)
+constexpr uint32_t kRecSlot = 17408;             // 1024-aligned slots
+constexpr uint32_t SM_I = SM_R + 2 * kRecSlot;   // 8 KB: 64 x 64 bfloat16 identity, K-major SW128
+constexpr uint32_t SM_SB = SM_I + 8192;          // 64 KB: state staging, 4 column blocks x 128 rows x 128 B, SW128
+constexpr uint32_t SM_BYTES = SM_SB + 65536;
+constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
+static_assert(SM_I % 1024 == 0 && SM_SB % 1024 == 0 && kRecSlot >= kRecBytes, "shared-memory map");
+static_assert(kSmemAlloc <= 232448, "shared memory budget");
+
+// The staging buffer holds a head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each
+// 128 rows x 128 bytes with the 128-byte swizzle (16-byte chunk ^ (row & 7)) that TMA writes and
+// reads; eight threads reading chunk c of eight consecutive rows (one row per thread) hit distinct
+// banks.  Float offset of 16-byte chunk `chunk` (0..31) of row `row`:
+__device__ __forceinline__ int sb_idx(int row, int chunk) {
+    return (chunk >> 3) * 4096 + row * 32 + (((chunk & 7) ^ (row & 7)) << 2);
 }
 
 struct TcArgs {
-    int L, Hk, Hv, T, n_tiles;   // n_tiles: 64-token tiles per head
-    const float* g;              // [L][T][Hv] log-decay
-    const float* beta;           // [L][T][Hv]
-    float* state;                // [L * Hv][128][128]
+    int L, Hk, Hv, T, n_tiles;
+    float* state;
     float* partials;
     float* wnorm;
+    const uint8_t* rec;
     int32_t* status;
-    uint32_t* ho_bits;           // hand-over bits in the workspace header: [0, 16) state, [16, 32) sums
-    float* ho_state;             // [grid][128][128]
-    float* ho_wsum;              // [grid]
-    int split;                   // run equal tile runs (ChainSched)
+    int split;               // run equal tile runs (ChainSched), when the host found it faster
+    // hand-over between neighbouring CTAs of a head split between them (see ChainSched): one
+    // entry per CTA boundary i (CTA i -> CTA i + 1)
+    int32_t* ho_flag;        // [grid] the state after the first part is in the hand-over map
+    int32_t* ho_wflag;       // [grid] the first part's write-size sum is in ho_wsum
+    float* ho_wsum;          // [grid]
 };
 
 // The CTA's work: a sequence of slots, each a run of consecutive tiles of one head.  By default
 // the CTA owns heads blockIdx.x, blockIdx.x + gridDim.x, ... whole.  When the heads do not divide
 // evenly among the CTAs and the host estimates it faster (a.split), the CTAs instead take equal
 // runs of the tile sequence in head order, so that the slowest CTA has one tile more than the
-// fastest instead of a whole head more; a head cut by a run boundary is shared by two neighbours.
-// CTA i runs the head it shares with CTA i + 1 first (its first tiles; the state at the cut goes
-// to hand-over entry i) and the head it shares with CTA i - 1 last (its last tiles, from hand-over
-// entry i - 1), so the second part of a shared head is never waited for before its first part is
-// long finished.  The split schedule is launched cooperatively, so every CTA is resident.
+// fastest instead of a whole head more; a head cut by a run boundary is shared by two neighbours.  CTA i runs the head
+// it shares with CTA i + 1 first (its first tiles; the state at the cut goes to hand-over entry i)
+// and the head it shares with CTA i - 1 last (its last tiles, from hand-over entry i - 1), so the
+// second part of a shared head is never waited for before its first part is long finished.
 struct ChainSched {
     int split;
     int pre_lh, pre_len;       // first slot: tiles [0, pre_len) of head pre_lh (none if pre_len == 0)
@@ -361,11 +722,13 @@ struct ChainSched {
     }
 };
 
-// Where a role's current tile lies: slot k, tile jt (of [tb, te)) of head lh = (layer l, value
-// head h), key head kh.
+// Where the CTA's current tile lies: slot k, tile jt (of [tb, te)) of head lh = (layer l, value
+// head h), key head kh.  Each role walks the tiles in order; a step costs integer divisions only
+// when it crosses into the next slot.
 struct TileCursor {
-    int k, jt, tb, te, lh, l, h, kh;
-    __device__ __noinline__ void set_slot(int slot, const ChainSched& sc, const TcArgs& a) {
+    int k, jt, te, lh, l, h, kh;
+    __device__ __forceinline__ void set_slot(int slot, const ChainSched& sc, const TcArgs& a) {
+        int tb;
         k = slot;
         sc.slot(slot, a.n_tiles, lh, tb, te);
         jt = tb;
@@ -373,7 +736,6 @@ struct TileCursor {
         kh = (int)(((long long)h * a.Hk) / a.Hv);
     }
     __device__ __forceinline__ void init(const ChainSched& sc, const TcArgs& a) {
-        k = -1;
         if (sc.n_slots > 0) set_slot(0, sc, a);
     }
     __device__ __forceinline__ void next(const ChainSched& sc, const TcArgs& a) {
@@ -381,619 +743,364 @@ struct TileCursor {
     }
 };
 
-// 16 fp32 of a state row, global -> registers (through L2 only for data another CTA wrote)
-__device__ __forceinline__ void ld16_global(const float* p, float (&v)[16], bool cache_global) {
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-        const float4 x = cache_global ? __ldcg(reinterpret_cast<const float4*>(p) + e)
-                                      : __ldg(reinterpret_cast<const float4*>(p) + e);
-        v[4 * e] = x.x; v[4 * e + 1] = x.y; v[4 * e + 2] = x.z; v[4 * e + 3] = x.w;
-    }
-}
-
 __global__ void __launch_bounds__(kThreads, 1)
-gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, TcArgs a)
+gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                     const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap hmap,
+                     TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
-    // loads -> roles: K, V tiles full; MMA -> loader: their empties.  producer -> MMA / chain: images
-    // and constants full (ifull, by tile parity); the images are free once their products have
-    // completed (bfree, by the parity of the tile that used them), the constants once the chain has
-    // read them (iempty).  MMA -> producer group: K K^T done (kk, by parity); producer -> MMA: read
-    // (kkfree).  MMA -> chain: Q done (q), E ready (u), state updated (s); chain -> MMA: W and the
-    // slot's state ready (ready), E packed (uready).
-    __shared__ uint64_t mb_kfull[kKSlots], mb_kempty[kKSlots], mb_vfull, mb_vempty, mb_ifull[2], mb_iempty[2];
-    __shared__ uint64_t mb_bfree[2], mb_kk[2], mb_kkfree, mb_q, mb_ready, mb_u, mb_uready, mb_s, mb_fin;
+    // copies -> roles: K (3), V (2), WY records (2) full; MMA -> loader: their empties; state
+    // staging full (mb_st) and released by the chain (mb_sfree); MMA -> chain: x, u, s; chain ->
+    // MMA: ready flags.
+    __shared__ uint64_t mb_tk[3], mb_ke[3], mb_tv[2], mb_ve[2], mb_tr[2], mb_re[2];
+    __shared__ uint64_t mb_st, mb_sfree, mb_x, mb_u, mb_s, mb_sready, mb_xready, mb_uready, mb_fin;
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ float s_red[2][kChainWarps];
-    __shared__ float s_u2[2][kC];                     // per-token squared write sizes (tile parity)
+    __shared__ float s_u2[2][kC];                 // per-token squared write sizes (tile parity)
     volatile int* abort_flag = &s_abort;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    // bounded-wait budget: the workspace header's override (microseconds) or about one second
-    const uint32_t budget_us = reinterpret_cast<const volatile uint32_t*>(a.status)[2];
-    const uint64_t budget = budget_us ? (uint64_t)budget_us * 1000ull : kWaitBudgetNs;
+    const int n = a.n_tiles;
+    // Persistent CTA: its slots (ChainSched) form one sequence of NJ tiles, over which every role
+    // keeps its barrier phases.
     ChainSched sch;
     sch.init(a);
-    const int NJ = sch.NJ;                            // tiles of this CTA
-    const int me = (int)blockIdx.x;
-    uint32_t* bits_state = a.ho_bits;
-    uint32_t* bits_wsum = a.ho_bits + 16;
+    const int n_slots = sch.n_slots;
+    const int NJ = sch.NJ;
 
     if (warp == kMmaWarp) {
         tmem_alloc(&s_tmem, kTmemCols);
         tmem_relinquish();
         if (lane == 0) {
-            for (int b = 0; b < kKSlots; ++b) { mbar_init(&mb_kfull[b], 1); mbar_init(&mb_kempty[b], 1); }
-            mbar_init(&mb_vfull, 1); mbar_init(&mb_vempty, 1);
+            for (int b = 0; b < 3; ++b) { mbar_init(&mb_tk[b], 1); mbar_init(&mb_ke[b], 1); }
             for (int b = 0; b < 2; ++b) {
-                mbar_init(&mb_ifull[b], 4); mbar_init(&mb_iempty[b], kChainWarps);
-                mbar_init(&mb_bfree[b], 1); mbar_init(&mb_kk[b], 1);
+                mbar_init(&mb_tv[b], 1); mbar_init(&mb_ve[b], 1);
+                mbar_init(&mb_tr[b], 1); mbar_init(&mb_re[b], 1);
             }
-            mbar_init(&mb_kkfree, 2); mbar_init(&mb_q, 1);
-            mbar_init(&mb_ready, kChainWarps); mbar_init(&mb_u, 1); mbar_init(&mb_uready, kChainWarps);
-            mbar_init(&mb_s, 1); mbar_init(&mb_fin, 1);
+            mbar_init(&mb_st, 1); mbar_init(&mb_sfree, kChainWarps);
+            mbar_init(&mb_x, 1); mbar_init(&mb_u, 1); mbar_init(&mb_s, 1);
+            mbar_init(&mb_sready, kChainWarps); mbar_init(&mb_xready, kChainWarps);
+            mbar_init(&mb_uready, kChainWarps);
+            mbar_init(&mb_fin, 1);
             fence_barrier_init();
         }
     }
     if (warp == kLoadWarp && lane == 0) { prefetch_tensormap(&kmap); prefetch_tensormap(&vmap); }
+    if (warp == kStateWarp && lane == 0) { prefetch_tensormap(&smap); prefetch_tensormap(&hmap); }
+    if (tid < kChain) {
+        // the 64 x 64 identity (B operand of V^T I): row t holds 1.0 at column t
+        const int t = tid >> 3, c8 = tid & 7;
+        uint32_t w[4] = {0u, 0u, 0u, 0u};
+        if ((t >> 3) == c8) w[(t & 7) >> 1] = (t & 1) ? 0x3F800000u : 0x00003F80u;
+        *reinterpret_cast<uint4*>(sm + SM_I + sw128_offset(t, c8)) = make_uint4(w[0], w[1], w[2], w[3]);
+        fence_async_smem();
+    }
     if (tid == 0) s_abort = 0;
     if (tid < 2 * kC) s_u2[tid >> 6][tid & (kC - 1)] = 0.f;
-    grid_dep_launch();                                // the next kernel (the score) may be scheduled
+    grid_dep_launch();                                 // the next kernel (the score) may be scheduled
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tm = s_tmem;
-    float* cst = reinterpret_cast<float*>(sm + SM_CONST);
 
     if (warp == kMmaWarp) {
         // =========================================================== MMA issue (converged warp;
         // one elected lane issues each group and commits it)
-        const uint32_t idW = idesc_bf16(128, 64, 1, 0);   // Q and E products: A MN-major (K^T, V^T)
-        const uint32_t idX = idesc_tf32(128, 64);
-        const uint32_t idS = idesc_bf16(128, 128, 0, 1);
-        const uint32_t idK = idesc_bf16(128, 64, 0, 0);
-        // K K^T of tile J (M = 128: rows 64..127 of A read the 16 KB past the tile; their output
-        // lanes are ignored), once the tile has landed and the producer has read the previous one
-        // (every product below is a rolled loop of single MMAs from one elected lane: the issue
-        // rate is the tensor pipe's, and the code stays small)
-        auto issue_kk = [&](int J) -> bool {
-            if (!warp_wait(&mb_kfull[J % kKSlots], (J / kKSlots) & 1, budget, abort_flag)) return false;
-            if (J > 0 && !warp_wait(&mb_kkfree, (J - 1) & 1, budget, abort_flag)) return false;
+        const uint64_t dK = sdesc_sw128(smem_u32(sm + SM_K), 8192, 1024);    // MN-major B of MMA_S
+        const uint64_t dK32 = sdesc_sw128(smem_u32(sm + SM_K32), 16, 1024);
+        const uint64_t dV = sdesc_sw128(smem_u32(sm + SM_V), 8192, 1024);    // MN-major A of V^T I
+        const uint64_t dR = sdesc_sw128(smem_u32(sm + SM_R), 16, 1024);
+        const uint64_t dI = sdesc_sw128(smem_u32(sm + SM_I), 16, 1024);
+        // Each group's operands are formed before the wait that releases it, so that only the
+        // MMA instructions themselves follow the wait (this warp shares its scheduler with four
+        // chain warps).
+        // V region <- V(J)^T: A = the V tile read MN-major (k-step s = tokens 16 s ..), B = I.  V(J)'s
+        // buffer is released when the product completes.
+        auto issue_vi = [&](int J) -> bool {
+            uint64_t av[4], bv[4];
+#pragma unroll
+            for (int s = 0; s < 4; ++s) {
+                av[s] = dadd(dV, (J & 1) * 16384 + s * 2048); bv[s] = dadd(dI, s * 32);
+                pin(av[s]); pin(bv[s]);
+            }
+            if (!warp_wait(&mb_tv[J & 1], (J >> 1) & 1, kWaitBudgetNs, abort_flag)) return false;
             tc_fence_after();
-            if (elect_one()) {
-                const uint32_t base = smem_u32(sm + SM_K + (J % kKSlots) * 16384);
-#pragma unroll 1
-                for (int s = 0; s < 8; ++s) {
-                    const uint64_t d = sdesc_sw128(base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024);
-                    mma_bf16_1t(tm + TM_KK, d, d, idK, s > 0);
+            if (elect_one()) mma4_bf16_ss_1t(tm + TM_V, av, bv, idesc_bf16(128, 64, 1, 0), 0);
+            __syncwarp();
+            mma_commit(&mb_ve[J & 1]);
+            return true;
+        };
+        bool ok = NJ == 0 || issue_vi(0);
+        if (!ok) fail(a.status, abort_flag, 1);
+        for (int j = 0; ok && j < NJ; ++j) {           // j: global tile index
+            {   // X region <- S~ K^T: A = the fp32 state from TMEM read as tf32 (8 columns per K = 8
+                // step), B = K in fp32.  Tile j ready for X: K(j) is converted and, at a head's first
+                // tile, the state is in TMEM (otherwise MMA_S(j-1), issued before, produces it in pipe
+                // order).
+                uint32_t ax[4][4];
+                uint64_t bx[4][4];
+#pragma unroll
+                for (int s = 0; s < 16; ++s) {
+                    ax[s >> 2][s & 3] = tm + TM_S + 8 * s;
+                    bx[s >> 2][s & 3] = dadd(dK32, (s >> 2) * 8192 + (s & 3) * 32);
+                    pin(ax[s >> 2][s & 3]); pin(bx[s >> 2][s & 3]);
                 }
-            }
-            __syncwarp();
-            mma_commit(&mb_kk[J & 1]);
-            return true;
-        };
-        // A (K^T or V^T: the tile read MN-major; k-steps 4..7 repeat tokens 0..63 for the lo half)
-        // times B (an image: k-steps 0..3 its hi block, 4..7 its lo block) into D
-        auto issue_img = [&](uint32_t d, uint32_t a_base, uint32_t b_base) {
-            if (elect_one()) {
-#pragma unroll 1
-                for (int s = 0; s < 8; ++s)
-                    mma_bf16_1t(d, sdesc_sw128(a_base + (s & 3) * 2048, 8192, 1024),
-                                sdesc_sw128(b_base + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024), idW, s > 0);
-            }
-            __syncwarp();
-        };
-        // Q(J) = K(J)^T B3(J) and E(J) = V(J)^T B1(J), once the images are written
-        auto issue_images = [&](int J) -> bool {
-            if (!warp_wait(&mb_ifull[J & 1], (J >> 1) & 1, budget, abort_flag)) return false;
-            tc_fence_after();
-            issue_img(tm + TM_Q, smem_u32(sm + SM_K + (J % kKSlots) * 16384), smem_u32(sm + SM_B3));
-            mma_commit(&mb_q);
-            if (!warp_wait(&mb_vfull, J & 1, budget, abort_flag)) return false;
-            tc_fence_after();
-            issue_img(tm + TM_E + (J & 1) * 64, smem_u32(sm + SM_V), smem_u32(sm + SM_B1));
-            mma_commit(&mb_vempty);
-            mma_commit(&mb_bfree[J & 1]);              // the images' last reader
-            return true;
-        };
-        bool ok = true;
-        if (NJ > 0) {
-            for (int J = 0; ok && J < 3 && J < NJ; ++J) ok = issue_kk(J);
-            if (ok) ok = issue_images(0);
-            if (!ok) fail(a.status, abort_flag, 1);
-        }
-        for (int j = 0; ok && j < NJ; ++j) {
-            const uint32_t eb = tm + TM_E + (j & 1) * 64;
-            int shift = 0;
-            {   // E(j) += S~ W(j) (A: the state from TMEM as tf32, 8 columns per K = 8 step; B: W in
-                // tf32).  E(j)'s own product was issued before, into the same accumulator.
-                if (!warp_wait(&mb_ready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 2); break; }
-                if (j > 0 && !warp_wait(&mb_s, (j - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 3); break; }
-                // E(j)'s own product has completed: for j > 0 the state update's commit covers it
-                // (issued after it), for the first tile its own commit
-                if (j == 0 && !warp_wait(&mb_vempty, 0, budget, abort_flag)) { fail(a.status, abort_flag, 7); break; }
-                // the tile's images and constants are held until the chain has read them
-                shift = reinterpret_cast<const volatile int*>(cst + (j & 1) * kConstWords)[66];
+                if (!warp_wait(&mb_sready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 2); break; }
                 tc_fence_after();
                 if (elect_one()) {
-                    const uint32_t wb = smem_u32(sm + SM_W);
-#pragma unroll 1
-                    for (int s = 0; s < 16; ++s)
-                        mma_tf32_ta_1t(eb, tm + TM_S + 8 * s, sdesc_sw128(wb + (s >> 2) * 8192 + (s & 3) * 32, 16, 1024),
-                                       idX, 1);
+#pragma unroll
+                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + TM_X, ax[g4], bx[g4], idesc_tf32(128, 64), g4 != 0);
+                }
+                __syncwarp();
+                mma_commit(&mb_x);
+            }
+            {   // U region <- W^T T~^T with W (hi, lo) packed in place in X (k-step s: hi at column
+                // 16 s, lo at 16 s + 8): W hi T~ hi + W hi T~ lo + W lo T~ hi
+                uint32_t au[3][4];
+                uint64_t bu[3][4];
+                const uint32_t rb = (j & 1) * kRecSlot;
+#pragma unroll
+                for (int part = 0; part < 3; ++part) {
+#pragma unroll
+                    for (int s = 0; s < 4; ++s) {
+                        au[part][s] = tm + TM_X + 16 * s + (part == 2 ? 8 : 0);
+                        bu[part][s] = dadd(dR, rb + (part == 1 ? 8192 : 0) + s * 32);
+                        pin(au[part][s]); pin(bu[part][s]);
+                    }
+                }
+                if (!warp_wait(&mb_xready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 5); break; }
+                if (!warp_wait(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 3); break; }
+                tc_fence_after();
+                if (elect_one()) {
+#pragma unroll
+                    for (int part = 0; part < 3; ++part)
+                        mma4_bf16_ta_1t(tm + TM_U, au[part], bu[part], idesc_bf16(128, 64, 0, 0), part != 0);
                 }
                 __syncwarp();
                 mma_commit(&mb_u);
+                mma_commit(&mb_re[j & 1]);             // record slot free once MMA_U(j) has read T~
             }
-            // K K^T three tiles ahead (a producer group has two tile periods for its tile), the next
-            // tile's Q and E, while the chain runs its pass
-            if (j + 3 < NJ && !issue_kk(j + 3)) { fail(a.status, abort_flag, 5); break; }
-            if (j + 1 < NJ && !issue_images(j + 1)) { fail(a.status, abort_flag, 4); break; }
-            {   // S~ = 2^-shift S~ + E K  (A: E hi / lo packed in place; K read MN-major)
-                if (!warp_wait(&mb_uready, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 6); break; }
+            // the next tile's V^T into the V region (its last reader, the W pass of tile j, has
+            // finished: MMA_U(j) waited for xready)
+            if (j + 1 < NJ && !issue_vi(j + 1)) { fail(a.status, abort_flag, 4); break; }
+            {   // S~ += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major)
+                uint32_t as_[2][4];
+                uint64_t bs[2][4];
+                const uint32_t kb = (j % 3) * 16384;
+#pragma unroll
+                for (int part = 0; part < 2; ++part) {
+#pragma unroll
+                    for (int s = 0; s < 4; ++s) {
+                        as_[part][s] = tm + TM_U + 16 * s + (part == 1 ? 8 : 0);
+                        bs[part][s] = dadd(dK, kb + s * 2048);
+                        pin(as_[part][s]); pin(bs[part][s]);
+                    }
+                }
+                if (!warp_wait(&mb_uready, j & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 7); break; }
                 tc_fence_after();
                 if (elect_one()) {
-                    // K-step s: A = E's hi (s < 4) or lo (s >= 4) columns of token block s & 3
-                    const uint32_t kb = smem_u32(sm + SM_K + (j % kKSlots) * 16384);
-                    mma_bf16_ta_shift_1t(shift, tm + TM_S, eb, sdesc_sw128(kb, 8192, 1024), idS);
-#pragma unroll 1
-                    for (int s = 1; s < 8; ++s) {
-                        const int tb = s & 3;
-                        mma_bf16_ta_1t(tm + TM_S, eb + 32 * (tb >> 1) + 8 * (tb & 1) + 16 * (s >> 2),
-                                       sdesc_sw128(kb + tb * 2048, 8192, 1024), idS, 1);
-                    }
+#pragma unroll
+                    for (int part = 0; part < 2; ++part)
+                        mma4_bf16_ta_1t(tm + TM_S, as_[part], bs[part], idesc_bf16(128, 128, 0, 1), 1);
                 }
                 __syncwarp();
                 mma_commit(&mb_s);
-                mma_commit(&mb_kempty[j % kKSlots]);   // the tile's last reader
+                mma_commit(&mb_ke[j % 3]);             // K(j)'s buffer free once MMA_S(j) has read it
             }
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0)) {
             mma_commit(&mb_fin);                       // every MMA this warp issued has completed
-            mbar_wait(&mb_fin, 0, budget);
+            mbar_wait(&mb_fin, 0, kWaitBudgetNs);
         }
         __syncwarp();
     } else if (warp == kLoadWarp) {
-        // =========================================================== K and V tiles, each into its
-        // buffer once the MMA that last read the buffer has completed.  The V stream runs two tiles
-        // behind the K stream: the MMA takes K three tiles ahead of the state update (for K K^T) but
-        // V one tile ahead, so a V load held for its buffer must not hold up the K loads behind it.
-        // The tiles ahead of the K ring and each slot's successor's state are prefetched into L2.
-        TileCursor kc, vc, pf;
-        kc.init(sch, a);
-        vc = kc;
-        pf = kc;
-        int kp[kKSlots], vp = -1;                      // last tile loaded per buffer
-        for (int b = 0; b < kKSlots; ++b) kp[b] = -1;
+        // =========================================================== K, V, records in tile order,
+        // each into its buffer once the MMA that last read the buffer has completed
+        TileCursor cc;
+        cc.init(sch, a);
+        int kp[3] = {-1, -1, -1}, vp[2] = {-1, -1}, rp[2] = {-1, -1};   // last tile loaded per buffer
+        // the kernel may start while the factor kernel finishes (its set-up and the first state
+        // load overlap that tail); the records it wrote are read only after it has completed
         grid_dep_wait();
-        auto prefetch_tile = [&](const TileCursor& c) {    // all lanes
-            if (lane == 0) {
-                tma_prefetch_4d(&kmap, 0, c.kh, c.jt * kC, c.l);
-                tma_prefetch_4d(&kmap, 64, c.kh, c.jt * kC, c.l);
-                tma_prefetch_4d(&vmap, 0, c.h, c.jt * kC, c.l);
-                tma_prefetch_4d(&vmap, 64, c.h, c.jt * kC, c.l);
+        for (int J = 0; J < NJ; ++J) {
+            const int bk = J % 3, b2 = J & 1;
+            if (J >= 3 && !warp_wait(&mb_ke[bk], ((J / 3) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 30); break; }
+            if (elect_one()) {
+                uint8_t* dst = sm + SM_K + bk * 16384;
+                mbar_arrive_expect_tx(&mb_tk[bk], 16384);
+                tma_load_4d(dst, &kmap, &mb_tk[bk], 0, cc.kh, cc.jt * kC, cc.l);
+                tma_load_4d(dst + 8192, &kmap, &mb_tk[bk], 64, cc.kh, cc.jt * kC, cc.l);
             }
-            // the tile's g and beta (one 4-byte value per token, a line apart): the producer reads
-            // them one group-tile ahead, too late to take an HBM miss off its path
-            const int t0 = c.jt * kC + lane;
-            const size_t i0 = ((size_t)c.l * a.T + t0) * a.Hv + c.h;
-            if (t0 < a.T) { prefetch_l2(a.g + i0); prefetch_l2(a.beta + i0); }
-            if (t0 + 32 < a.T) { prefetch_l2(a.g + i0 + 32 * (size_t)a.Hv); prefetch_l2(a.beta + i0 + 32 * (size_t)a.Hv); }
-        };
-        for (int i = 0; i < kKSlots && i < NJ; ++i) {
-            prefetch_tile(pf);
             __syncwarp();
-            pf.next(sch, a);
-        }
-        constexpr int kVLag = 2;
-        bool ok = true;
-        for (int n = 0; ok && n < NJ + kVLag; ++n) {
-            if (n < NJ) {                                // K of tile n
-                if (n + kKSlots < NJ) {
-                    prefetch_tile(pf);
-                    __syncwarp();
-                    pf.next(sch, a);
-                }
-                if (kc.jt == kc.tb && kc.k + 1 < sch.n_slots && !sch.is_suffix(kc.k + 1) && elect_one()) {
-                    int lh, tb, te;                      // the next slot's state, ahead of its boundary
-                    sch.slot(kc.k + 1, a.n_tiles, lh, tb, te);
-                    prefetch_l2_bulk(a.state + (size_t)lh * kD * kD, kD * kD * 4);
-                }
-                __syncwarp();
-                const int bk = n % kKSlots;
-                if (n >= kKSlots && !warp_wait(&mb_kempty[bk], ((n / kKSlots) - 1) & 1, budget, abort_flag)) {
-                    fail(a.status, abort_flag, 30); break;
-                }
-                if (elect_one()) {
-                    uint8_t* dst = sm + SM_K + bk * 16384;
-                    mbar_arrive_expect_tx(&mb_kfull[bk], 16384);
-                    tma_load_4d(dst, &kmap, &mb_kfull[bk], 0, kc.kh, kc.jt * kC, kc.l);
-                    tma_load_4d(dst + 8192, &kmap, &mb_kfull[bk], 64, kc.kh, kc.jt * kC, kc.l);
-                }
-                __syncwarp();
-                kp[bk] = n;
-                kc.next(sch, a);
+            kp[bk] = J;
+            if (J >= 2 && !warp_wait(&mb_ve[b2], ((J >> 1) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 31); break; }
+            if (elect_one()) {
+                uint8_t* dst = sm + SM_V + b2 * 16384;
+                mbar_arrive_expect_tx(&mb_tv[b2], 16384);
+                tma_load_4d(dst, &vmap, &mb_tv[b2], 0, cc.h, cc.jt * kC, cc.l);
+                tma_load_4d(dst + 8192, &vmap, &mb_tv[b2], 64, cc.h, cc.jt * kC, cc.l);
             }
-            const int m = n - kVLag;                     // V of tile m
-            if (m >= 0) {
-                if (m >= 1 && !warp_wait(&mb_vempty, (m - 1) & 1, budget, abort_flag)) { fail(a.status, abort_flag, 31); break; }
-                if (elect_one()) {
-                    uint8_t* dst = sm + SM_V;
-                    mbar_arrive_expect_tx(&mb_vfull, 16384);
-                    tma_load_4d(dst, &vmap, &mb_vfull, 0, vc.h, vc.jt * kC, vc.l);
-                    tma_load_4d(dst + 8192, &vmap, &mb_vfull, 64, vc.h, vc.jt * kC, vc.l);
-                }
-                __syncwarp();
-                vp = m;
-                vc.next(sch, a);
+            __syncwarp();
+            vp[b2] = J;
+            if (J >= 2 && !warp_wait(&mb_re[b2], ((J >> 1) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 32); break; }
+            if (elect_one()) {
+                mbar_arrive_expect_tx(&mb_tr[b2], kRecBytes);
+                bulk_load_tx(sm + SM_R + b2 * kRecSlot, a.rec + ((size_t)cc.lh * n + cc.jt) * kRecBytes,
+                             kRecBytes, &mb_tr[b2]);
             }
+            __syncwarp();
+            rp[b2] = J;
+            cc.next(sch, a);
         }
         if (__any_sync(0xffffffffu, *abort_flag != 0) && lane == 0) {
             // every copy this warp issued lands before the CTA ends
-            for (int b = 0; b < kKSlots; ++b)
-                if (kp[b] >= 0) mbar_wait(&mb_kfull[b], (kp[b] / kKSlots) & 1, budget);
-            if (vp >= 0) mbar_wait(&mb_vfull, vp & 1, budget);
+            for (int b = 0; b < 3; ++b)
+                if (kp[b] >= 0) mbar_wait(&mb_tk[b], (kp[b] / 3) & 1, kWaitBudgetNs);
+            for (int b = 0; b < 2; ++b) {
+                if (vp[b] >= 0) mbar_wait(&mb_tv[b], (vp[b] >> 1) & 1, kWaitBudgetNs);
+                if (rp[b] >= 0) mbar_wait(&mb_tr[b], (rp[b] >> 1) & 1, kWaitBudgetNs);
+            }
         }
         __syncwarp();
-    } else if (warp >= kProdWarp0) {
-        // =========================================================== producer: the images and decay
-        // constants of every tile; group 0 (warps 8-11) the even tiles, group 1 (warps 4-7) the odd
-        const int grp = warp >= 8 ? 0 : 1;
-        const int pw = warp & 3;                       // 0, 1: K K^T readers (TMEM lanes 32 pw ..); 2: constants
-        const int pt = pw * 32 + lane;                 // thread of the group, 0..127
-        const int bar_id = kBarProd + grp;
-        float* fws = reinterpret_cast<float*>(sm + SM_PW + grp * kPwBytes);
-        float* Mt = fws + PW_MT;                       // rows 0..31 of diag(beta) L (columns 0..31)
-        float* Mb = fws + PW_MB;                       // rows 32..63 (columns 0..63)
-        float* Nt = fws + PW_NT;                       // the same rows of (I + diag(beta) L)^-1
-        float* Nb = fws + PW_NB;
-        float* Pm = fws + PW_P;                        // block products
-        auto mrow = [&](int r) { return r < 32 ? Mt + r * kTS : Mb + (r - 32) * kBS; };
-        auto nrow = [&](int r) { return r < 32 ? Nt + r * kTS : Nb + (r - 32) * kBS; };
-        const int g = lane >> 2, tq = lane & 3;        // mma.sync fragment coordinates
-        // cursors at the group's tile J and at J - 1 (the deferred scale before J depends on it)
-        TileCursor cc, cq;
-        cc.init(sch, a);
-        cq = cc;
-        if (grp == 1 && NJ > 1) cc.next(sch, a);
-        // loads, one group-tile ahead: warp 2 the g and beta of the tile's tokens lane, 32 + lane and
-        // the g of tile J - 1 when it is in J's slot; warps 0, 1 the beta of token 32 pw + lane
-        struct Gb { float g0, g1, b0, b1, q0, q1; };
-        auto load_gb = [&](const TileCursor& c, const TileCursor& cp, bool prev_same) {
-            Gb v = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-            const int t0 = c.jt * kC + lane, t1 = t0 + 32;
-            const size_t base = (size_t)c.l * a.T;
-            if (pw == 2) {
-                v.g0 = t0 < a.T ? a.g[(base + t0) * a.Hv + c.h] : 0.f;
-                v.g1 = t1 < a.T ? a.g[(base + t1) * a.Hv + c.h] : 0.f;
-                v.b0 = t0 < a.T ? a.beta[(base + t0) * a.Hv + c.h] : 0.f;
-                v.b1 = t1 < a.T ? a.beta[(base + t1) * a.Hv + c.h] : 0.f;
-                if (prev_same) {
-                    const int s0 = cp.jt * kC + lane, s1 = s0 + 32;
-                    const size_t pb = (size_t)cp.l * a.T;
-                    v.q0 = s0 < a.T ? a.g[(pb + s0) * a.Hv + cp.h] : 0.f;
-                    v.q1 = s1 < a.T ? a.g[(pb + s1) * a.Hv + cp.h] : 0.f;
-                }
-            } else if (pw < 2) {
-                const int tb = t0 + 32 * pw;
-                v.b0 = tb < a.T ? a.beta[(base + tb) * a.Hv + c.h] : 0.f;
-            }
-            return v;
-        };
-        // the tile's cumulative log-decay: inclusive scans of its two halves (both groups use this
-        // order, so the deferred scale they compute for a tile agrees bit for bit)
-        auto scan_tile = [&](float g0, float g1, float& G0, float& G1) {
-            G0 = g0; G1 = g1;
+    } else if (warp == kStateWarp) {
+        // =========================================================== state moves (lane 0).  Phases
+        // of mb_st: 0 = the first slot's state staged; k + 1 = what the boundary after slot k
+        // needs: the state of slot k + 1, or after the last slot a free buffer (when the last slot
+        // ends a head begun by CTA i - 1: that head's state before the chunk, for its drift).
+        // Phases of mb_sfree: 0 = the first state is in TMEM; k + 1 = slot k's final state is
+        // staged.  A first slot that begins a head shared with CTA i + 1 leaves its state in
+        // hand-over entry i; a last slot that ends a head shared with CTA i - 1 starts from entry
+        // i - 1, once that entry's flag is set (bounded wait).
+        if (lane == 0 && n_slots > 0) {
+            float* sbuf = reinterpret_cast<float*>(sm + SM_SB);
+            const int me = (int)blockIdx.x;
+            int loads = 0, seen = 0;                   // copies into the staging buffer issued / landed
+            auto load_rows = [&](const CUtensorMap* map, int row) {
+                mbar_arrive_expect_tx(&mb_st, kD * kD * 4);
 #pragma unroll
-            for (int m = 1; m < 32; m <<= 1) {
-                const float y0 = __shfl_up_sync(0xffffffffu, G0, m);
-                const float y1 = __shfl_up_sync(0xffffffffu, G1, m);
-                if (lane >= m) { G0 += y0; G1 += y1; }
+                for (int b = 0; b < 4; ++b) tma_load_2d(sbuf + 4096 * b, map, &mb_st, 32 * b, row);
+                ++loads;
+            };
+            auto load_state = [&](int slot) -> bool {
+                int lh, tb, te;
+                sch.slot(slot, n, lh, tb, te);
+                if (!sch.is_suffix(slot)) { load_rows(&smap, lh * kD); return true; }
+                grid_dep_wait();                       // the factor kernel reset the flags
+                const uint64_t t0 = global_ns();
+                while (ho_load_acquire(a.ho_flag + me - 1) == 0) {
+                    if (*abort_flag || global_ns() - t0 > kWaitBudgetNs) return false;
+                    __nanosleep(64);
+                }
+                fence_proxy_async_global();
+                load_rows(&hmap, (me - 1) * kD);
+                return true;
+            };
+            auto final_phase = [&]() {                 // what the boundary after the last slot reads
+                if (sch.is_suffix(n_slots - 1)) load_rows(&smap, sch.suf_lh * kD);
+                else mbar_arrive(&mb_st);
+            };
+            bool ok = load_state(0);
+            if (!ok) fail(a.status, abort_flag, 42);
+            if (ok) {
+                ok = mbar_wait_or_abort(&mb_sfree, 0, kWaitBudgetNs, abort_flag);
+                if (!ok) fail(a.status, abort_flag, 40);
             }
-            G1 += __shfl_sync(0xffffffffu, G0, 31);
-            return __shfl_sync(0xffffffffu, G1, 31);
-        };
-        Gb cur = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        if (pw < 3 && grp < NJ) {
-            grid_dep_wait();
-            cur = load_gb(cc, cq, grp == 1 && cq.k == cc.k);
+            seen = loads;                              // the chain has consumed it
+            if (ok) {
+                if (n_slots > 1) {
+                    ok = load_state(1);
+                    if (!ok) fail(a.status, abort_flag, 43);
+                } else {
+                    final_phase();
+                }
+            }
+            for (int k = 0; ok && k < n_slots; ++k) {
+                if (!mbar_wait_or_abort(&mb_sfree, (k + 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 41); break; }
+                seen = loads;
+                int lh, tb, te;
+                sch.slot(k, n, lh, tb, te);
+                const bool hand_over = sch.is_prefix(k);
+                const CUtensorMap* dst = hand_over ? &hmap : &smap;
+                const int row = (hand_over ? me : lh) * kD;
+#pragma unroll
+                for (int b = 0; b < 4; ++b) tma_store_2d(dst, sbuf + 4096 * b, 32 * b, row);
+                bulk_commit();
+                if (hand_over) {
+                    bulk_wait0();                      // the state is in global memory ...
+                    fence_proxy_async_global();
+                    __threadfence();
+                    grid_dep_wait();                   // (after the factor kernel's flag reset)
+                    ho_store_release(a.ho_flag + me, 1);   // ... before CTA i + 1 may read it
+                }
+                if (k + 2 <= n_slots) {
+                    bulk_wait_read0();                 // slot k's state has left the buffer
+                    if (k + 2 < n_slots) {
+                        if (!load_state(k + 2)) { fail(a.status, abort_flag, 43); break; }
+                    } else {
+                        final_phase();
+                    }
+                }
+            }
+            bulk_wait0();                              // every state store is complete
+            if (loads > seen) mbar_wait(&mb_st, (loads - 1) & 1, kWaitBudgetNs);   // abort: a load in flight
         }
-        float sig_last = 1.f;                          // sig after the group's previous tile
-        bool failed = false;
-        for (int J = grp; J < NJ; J += 2) {
-            const int slot2 = (J >> 1) & 1;
-            float* sBeta = fws + PW_BETA + 64 * slot2;
-            float* sDelta = fws + PW_DELTA + 64 * slot2;
-            float* sUC = fws + PW_UC + 4 * slot2;
-            const bool first_of_slot = cc.jt == cc.tb;
-            const bool prev_first = cq.jt == cq.tb;    // (J - 1 in J's slot only when !first_of_slot)
-            const Gb now = cur;
-            TileCursor nq = cc, nc = cc;               // the group's next tile J + 2 and J + 1
-            if (J + 2 < NJ) {
-                nq.next(sch, a);
-                nc = nq;
-                nc.next(sch, a);
-                if (pw < 3) cur = load_gb(nc, nq, nq.k == nc.k);
-            }
-            DecayStep dst;
-            float wn0 = 0.f, wn1 = 0.f;
-            if (pw == 2) {
-                // ---- constants of the tile's 64 tokens (lane: tokens lane and 32 + lane)
-                float sig_b = 1.f;                     // a slot starts from the true state
-                if (!first_of_slot) {                  // tile J - 1 (the other group's) in the same slot
-                    float Q0, Q1;
-                    const float GQ = scan_tile(now.q0, now.q1, Q0, Q1);
-                    sig_b = decay_step(expf(GQ) * (prev_first ? 1.f : sig_last)).sig;
-                }
-                float G0, G1;
-                const float GC = scan_tile(now.g0, now.g1, G0, G1);
-                dst = decay_step(expf(GC) * sig_b);
-                sig_last = dst.sig;
-                const float d0 = expf(GC - G0), d1 = expf(GC - G1);
-                sBeta[lane] = now.b0; sBeta[32 + lane] = now.b1;
-                sDelta[lane] = d0; sDelta[32 + lane] = d1;
-                const float ud0 = dst.u * d0, ud1 = dst.u * d1;
-                wn0 = ud0 >= 0x1p-60f ? 1.f / ud0 : 0.f;   // column t of E is u delta_t u_t
-                wn1 = ud1 >= 0x1p-60f ? 1.f / ud1 : 0.f;
-                if (lane == 0) { sUC[0] = dst.u; sUC[1] = dst.c; }
-            } else if (pw < 2) {
-                // ---- rows 32 pw .. 32 pw + 31 of diag(beta) L from K K^T (warp 1: also the block
-                // left of the diagonal, in full)
-                const bool ok = wait_bar(&mb_kk[grp], (J >> 1) & 1, budget, abort_flag);
-                if (!ok) { fail(a.status, abort_flag, 20); failed = true; }
-                tc_fence_after();
-                if (ok) {
-                    const uint32_t base = tm + ((uint32_t)(32 * pw) << 16) + TM_KK;
-                    float* row = mrow(32 * pw + lane);
-                    const float bt = now.b0;
-                    float kk[32];
-                    tmem_ld32(base + 32 * pw, kk);         // the diagonal block
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int c4 = 0; c4 < 8; ++c4) {
-                        float4 v;
-                        v.x = (4 * c4 + 0 < lane) ? bt * kk[4 * c4 + 0] : 0.f;
-                        v.y = (4 * c4 + 1 < lane) ? bt * kk[4 * c4 + 1] : 0.f;
-                        v.z = (4 * c4 + 2 < lane) ? bt * kk[4 * c4 + 2] : 0.f;
-                        v.w = (4 * c4 + 3 < lane) ? bt * kk[4 * c4 + 3] : 0.f;
-                        *reinterpret_cast<float4*>(row + 32 * pw + 4 * c4) = v;
-                    }
-                    if (pw == 1) {                         // rows 32..63 x columns 0..31
-                        tmem_ld32(base, kk);
-                        tmem_ld_wait();
-#pragma unroll
-                        for (int c4 = 0; c4 < 8; ++c4)
-                            *reinterpret_cast<float4*>(row + 4 * c4) =
-                                make_float4(bt * kk[4 * c4], bt * kk[4 * c4 + 1], bt * kk[4 * c4 + 2], bt * kk[4 * c4 + 3]);
-                    }
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&mb_kkfree);
-            }
-            if (named_sync_or(bar_id, kProd, failed || *abort_flag)) break;          // (1)
-            if (pw < 2) {
-                // the four 16 x 16 diagonal blocks of N by forward substitution, one column per lane;
-                // the next row's coefficients are loaded while the current row is formed
-                const int o = 32 * pw + 16 * (lane >> 4), jc = lane & 15;
-                float x[16];
-#pragma unroll
-                for (int rr = 0; rr < 16; ++rr) x[rr] = (rr == jc) ? 1.f : 0.f;
-                float4 cur4[4], nxt4[4];
-                cur4[0] = *reinterpret_cast<const float4*>(mrow(o + 1) + o);
-#pragma unroll
-                for (int rr = 1; rr < 16; ++rr) {
-                    if (rr + 1 < 16) {
-#pragma unroll
-                        for (int c4 = 0; c4 < 4; ++c4)
-                            if (4 * c4 < rr + 1) nxt4[c4] = *reinterpret_cast<const float4*>(mrow(o + rr + 1) + o + 4 * c4);
-                    }
-                    float sacc[4] = {0.f, 0.f, 0.f, 0.f};     // four short FMA chains
-#pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) {
-                        const int c = 4 * c4;
-                        if (c < rr) {
-                            sacc[0] = fmaf(cur4[c4].x, x[c], sacc[0]);
-                            if (c + 1 < rr) sacc[1] = fmaf(cur4[c4].y, x[c + 1], sacc[1]);
-                            if (c + 2 < rr) sacc[2] = fmaf(cur4[c4].z, x[c + 2], sacc[2]);
-                            if (c + 3 < rr) sacc[3] = fmaf(cur4[c4].w, x[c + 3], sacc[3]);
-                        }
-                    }
-                    if (rr > jc) x[rr] = -((sacc[0] + sacc[1]) + (sacc[2] + sacc[3]));
-#pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) cur4[c4] = nxt4[c4];
-                }
-#pragma unroll
-                for (int rr = 0; rr < 16; ++rr) nrow(o + rr)[o + jc] = x[rr];
-                if ((lane >> 4) == 0) {
-#pragma unroll
-                    for (int rr = 0; rr < 16; ++rr) nrow(o + rr)[o + 16 + jc] = 0.f;   // the block above
-                }
-            }
-            if (named_sync_or(bar_id, kProd, *abort_flag)) break;                    // (2)
-            {   // 16 -> 32, warp (p, nh): in 32-block p, columns 8 nh .. of
-                //   P = M[16..32][0..16] N[0..16][0..16],  then  N[16..32][0..16] = -N[16..32][16..32] P
-                // (tensor-core fragments, three-term bfloat16 products)
-                const int p = pw >> 1, nh = pw & 1, o = 32 * p;
-                const int ld = p ? kBS : kTS;
-                float d[4] = {0.f, 0.f, 0.f, 0.f};
-                mma_f32_split<1>(d, mrow(o + 16) + o, ld, nrow(o) + o + 8 * nh, ld, g, tq);
-                float* pp = Pm + 16 * p * kPS + 8 * nh;
-                *reinterpret_cast<float2*>(pp + g * kPS + 2 * tq) = make_float2(d[0], d[1]);
-                *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 2 * tq) = make_float2(d[2], d[3]);
-                __syncwarp();
-                float e[4] = {0.f, 0.f, 0.f, 0.f};
-                mma_f32_split<1>(e, nrow(o + 16) + o + 16, ld, pp, kPS, g, tq);
-                float* np = nrow(o + 16) + o + 8 * nh;
-                *reinterpret_cast<float2*>(np + g * ld + 2 * tq) = make_float2(-e[0], -e[1]);
-                *reinterpret_cast<float2*>(np + (g + 8) * ld + 2 * tq) = make_float2(-e[2], -e[3]);
-            }
-            if (named_sync_or(bar_id, kProd, *abort_flag)) break;                    // (3)
-            {   // 32 -> 64, warp (mt, nh): rows 16 mt .., columns 16 nh .. of
-                //   P = M[32..64][0..32] N[0..32][0..32],  then  N[32..64][0..32] = -N[32..64][32..64] P
-                const int mt = pw >> 1, nh = pw & 1;
-                float d0[4] = {0.f, 0.f, 0.f, 0.f}, d1[4] = {0.f, 0.f, 0.f, 0.f};
-                mma_f32_split<2>(d0, Mb + 16 * mt * kBS, kBS, Nt + 16 * nh, kTS, g, tq);
-                mma_f32_split<2>(d1, Mb + 16 * mt * kBS, kBS, Nt + 16 * nh + 8, kTS, g, tq);
-                float* pp = Pm + 16 * mt * kPS + 16 * nh;
-                *reinterpret_cast<float2*>(pp + g * kPS + 2 * tq) = make_float2(d0[0], d0[1]);
-                *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 2 * tq) = make_float2(d0[2], d0[3]);
-                *reinterpret_cast<float2*>(pp + g * kPS + 8 + 2 * tq) = make_float2(d1[0], d1[1]);
-                *reinterpret_cast<float2*>(pp + (g + 8) * kPS + 8 + 2 * tq) = make_float2(d1[2], d1[3]);
-                if (named_sync_or(bar_id, kProd, *abort_flag)) break;                // (4)
-                float e0[4] = {0.f, 0.f, 0.f, 0.f}, e1[4] = {0.f, 0.f, 0.f, 0.f};
-                mma_f32_split<2>(e0, Nb + 16 * mt * kBS + 32, kBS, Pm + 16 * nh, kPS, g, tq);
-                mma_f32_split<2>(e1, Nb + 16 * mt * kBS + 32, kBS, Pm + 16 * nh + 8, kPS, g, tq);
-                float* np = Nb + 16 * mt * kBS + 16 * nh;
-                *reinterpret_cast<float2*>(np + g * kBS + 2 * tq) = make_float2(-e0[0], -e0[1]);
-                *reinterpret_cast<float2*>(np + (g + 8) * kBS + 2 * tq) = make_float2(-e0[2], -e0[3]);
-                *reinterpret_cast<float2*>(np + g * kBS + 8 + 2 * tq) = make_float2(-e1[0], -e1[1]);
-                *reinterpret_cast<float2*>(np + (g + 8) * kBS + 8 + 2 * tq) = make_float2(-e1[2], -e1[3]);
-            }
-            // the images are free once the products of tile J - 1 (the other group's) have completed,
-            // the constants slot once the chain has read those of tile J - 2
-            if (J >= 1 && !wait_bar(&mb_bfree[(J - 1) & 1], ((J - 1) >> 1) & 1, budget, abort_flag)) {
-                fail(a.status, abort_flag, 21); failed = true;
-            }
-            if (J >= 2 && !wait_bar(&mb_iempty[J & 1], ((J >> 1) - 1) & 1, budget, abort_flag)) {
-                fail(a.status, abort_flag, 22); failed = true;
-            }
-            if (named_sync_or(bar_id, kProd, failed || *abort_flag)) break;          // (5)
-            {   // images: row t = pt / 2, columns 32 hh .. 32 hh + 31 of N_beta = N diag(beta) (zero
-                // above the diagonal)
-                const int t = pt >> 1, hh = pt & 1;
-                const float u = sUC[0];
-                uint8_t* b1 = sm + SM_B1;
-                uint8_t* b3 = sm + SM_B3;
-                const bool zero_half = t < 32 && hh == 1;
-                const float* nr = nrow(t) + (zero_half ? 0 : 32 * hh);
-#pragma unroll 1
-                for (int g8 = 0; g8 < 4; ++g8) {        // 8 columns (one 16-byte chunk of bf16) at a time
-                    const int c = 32 * hh + 8 * g8;
-                    uint32_t h3[4] = {0u, 0u, 0u, 0u}, l3[4] = {0u, 0u, 0u, 0u};
-                    uint32_t h1[4] = {0u, 0u, 0u, 0u}, l1[4] = {0u, 0u, 0u, 0u};
-                    if (!zero_half) {
-                        const float4 n0 = *reinterpret_cast<const float4*>(nr + 8 * g8);
-                        const float4 n1 = *reinterpret_cast<const float4*>(nr + 8 * g8 + 4);
-                        const float4 bv0 = *reinterpret_cast<const float4*>(sBeta + c);
-                        const float4 bv1 = *reinterpret_cast<const float4*>(sBeta + c + 4);
-                        const float4 dv0 = *reinterpret_cast<const float4*>(sDelta + c);
-                        const float4 dv1 = *reinterpret_cast<const float4*>(sDelta + c + 4);
-                        const float nv[8] = {n0.x, n0.y, n0.z, n0.w, n1.x, n1.y, n1.z, n1.w};
-                        const float bv[8] = {bv0.x, bv0.y, bv0.z, bv0.w, bv1.x, bv1.y, bv1.z, bv1.w};
-                        const float dv[8] = {dv0.x, dv0.y, dv0.z, dv0.w, dv1.x, dv1.y, dv1.z, dv1.w};
-                        float nb[8], w1[8];
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            nb[i] = (c + i <= t) ? nv[i] * bv[i] : 0.f;
-                            w1[i] = u * nb[i] * dv[i];
-                        }
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            split2(nb[2 * i], nb[2 * i + 1], h3[i], l3[i]);
-                            split2(w1[2 * i], w1[2 * i + 1], h1[i], l1[i]);
-                        }
-                    }
-                    const uint32_t off = sw128_offset(t, c >> 3);
-                    *reinterpret_cast<uint4*>(b3 + off) = make_uint4(h3[0], h3[1], h3[2], h3[3]);
-                    *reinterpret_cast<uint4*>(b3 + 8192 + off) = make_uint4(l3[0], l3[1], l3[2], l3[3]);
-                    *reinterpret_cast<uint4*>(b1 + off) = make_uint4(h1[0], h1[1], h1[2], h1[3]);
-                    *reinterpret_cast<uint4*>(b1 + 8192 + off) = make_uint4(l1[0], l1[1], l1[2], l1[3]);
-                }
-            }
-            if (pw == 2) {                              // the chain's and the MMA's constants
-                float* cs = cst + (J & 1) * kConstWords;
-                cs[lane] = wn0;
-                cs[32 + lane] = wn1;
-                if (lane == 0) {
-                    cs[64] = dst.sig;
-                    cs[65] = dst.pass;
-                    reinterpret_cast<int*>(cs)[66] = dst.shift;
-                    cs[67] = dst.c;
-                }
-            }
-            fence_async_smem();                         // generic writes -> the tensor core's reads
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&mb_ifull[J & 1]);
-            cq = nq;
-            cc = nc;
-        }
+        __syncwarp();
     } else {
-        // =========================================================== state chain (warps 0-3)
-        const int q = warp;                              // TMEM lane quadrant
+        // =========================================================== state chain (warps 0-15)
+        const int q = warp & 3, cgp = warp >> 2;         // TMEM lane quadrant, column group
         const int r = 32 * q + lane;                     // row of S (value index)
         const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-        TileCursor cc;
+        float* sbuf = reinterpret_cast<float*>(sm + SM_SB);   // swizzled rows, see sb_idx
+        int st_seen = 0;                                 // mb_st phases waited for (uniform)
+        TileCursor cc;                                   // the chain's tile
         cc.init(sch, a);
-        // W(jj) = -c Q^T in tf32: this thread's d_k row c = r of Q, tokens 0..63, into rows t of the
-        // K-major W (column block q, its 4-byte slot of row t).  Q(jj) is complete and W's last
-        // reader, E(jj-1) += S~ W(jj-1), has completed.
-        auto make_w = [&](int jj) -> bool {
-            bool ok = wait_bar(&mb_q, jj & 1, budget, abort_flag);
-            ok = wait_bar(&mb_ifull[jj & 1], (jj >> 1) & 1, budget, abort_flag) && ok;
-            tc_fence_after();
-            const float cneg = -cst[(jj & 1) * kConstWords + 67];
-            uint8_t* wb = sm + SM_W + q * 8192 + (lane & 3) * 4;
-            const int chunk = lane >> 2;
-#pragma unroll 1
-            for (int hh = 0; hh < 2; ++hh) {
-                float qv[32];
-                tmem_ld32(tm + lane_off + TM_Q + 32 * hh, qv);
-                tmem_ld_wait();
+        const int me = (int)blockIdx.x;
+        // K(jj) (TMA tile, buffer jj % 3) in fp32 (exact, and exact in tf32) into the B operand
+        // buffer of X.  Called between MMA_X(jj-1), the last reader of the buffer, and the ready
+        // signal of tile jj.
+        auto make_k32 = [&](int jj) -> bool {
+            const bool ok = mbar_wait_or_abort(&mb_tk[jj % 3], (jj / 3) & 1, kWaitBudgetNs, abort_flag);
+            const uint8_t* kb = sm + SM_K + (jj % 3) * 16384;
+            uint8_t* k32 = sm + SM_K32;
 #pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    *reinterpret_cast<uint32_t*>(wb + sw128_offset(32 * hh + i, chunk)) = to_tf32(cneg * qv[i]);
+            for (int u = 0; u < 2; ++u) {                  // 64 rows x 16 chunks of 8 bf16
+                const int e = tid + kChain * u;
+                const int t = e >> 4, c16 = e & 15, cb = c16 >> 3, c = c16 & 7;
+                const uint4 w = *reinterpret_cast<const uint4*>(kb + cb * 8192 + sw128_offset(t, c));
+                const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
+                uint32_t f[8];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    f[2 * i] = wv[i] << 16;
+                    f[2 * i + 1] = wv[i] & 0xFFFF0000u;
+                }
+                // dims 64 cb + 8 c .. + 7: fp32 block 2 cb + c / 4, chunks 2 (c % 4) and 2 (c % 4) + 1
+                uint8_t* rowp = k32 + (2 * cb + (c >> 2)) * 8192;
+                const int q0 = 2 * (c & 3);
+                *reinterpret_cast<uint4*>(rowp + sw128_offset(t, q0)) = make_uint4(f[0], f[1], f[2], f[3]);
+                *reinterpret_cast<uint4*>(rowp + sw128_offset(t, q0 + 1)) = make_uint4(f[4], f[5], f[6], f[7]);
             }
-            fence_async_smem();
-            tc_fence_before();
+            fence_async_smem();                            // generic writes -> the tensor core's reads
             return ok;
         };
-        // a slot's starting state (from the state or hand-over entry i - 1) into TMEM as S~ and
-        // S_before; `den` gets this thread's sum of squares
-        auto install = [&](int slot, float& den) -> bool {
-            int lh, tb, te;
-            sch.slot(slot, a.n_tiles, lh, tb, te);
-            const bool from_ho = sch.is_suffix(slot);
-            bool ok = true;
-            if (from_ho) {                               // one thread waits for CTA i - 1's state
-                if (tid == 0) {
-                    const uint32_t bit = 1u << ((me - 1) & 31);
-                    uint32_t* w = bits_state + ((me - 1) >> 5);
-                    const uint64_t t0 = global_ns();
-                    while ((ld_acquire(w) & bit) == 0) {
-                        if (*abort_flag || global_ns() - t0 > budget) { fail(a.status, abort_flag, 42); break; }
-                        __nanosleep(64);
-                    }
-                    atomicAnd(w, ~bit);                  // consumed: zero for the next call
-                }
-                ok = !named_sync_or(kBarChain, kChain, *abort_flag);
-            }
-            const float* src = (from_ho ? a.ho_state + (size_t)(me - 1) * kD * kD : a.state + (size_t)lh * kD * kD)
-                               + (size_t)r * kD;
-            den = 0.f;
-            if (ok) {
-#pragma unroll 1
-                for (int g8 = 0; g8 < 8; ++g8) {
-                    float v[16];
-                    ld16_global(src + 16 * g8, v, from_ho);
-                    uint32_t u32[16];
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) { den = fmaf(v[e], v[e], den); u32[e] = __float_as_uint(v[e]); }
-                    tmem_st16(tm + lane_off + TM_S + 16 * g8, u32);
-                    tmem_st16(tm + lane_off + TM_SB + 16 * g8, u32);
-                }
-            }
-            return ok;
+        auto rec_consts = [&](int jj) {                    // -gamma[64], gamma_C of tile jj's record
+            return reinterpret_cast<const float*>(sm + SM_R + (jj & 1) * kRecSlot + kRecT);
         };
-        float den = 0.f, sig = 1.f;
-        // Write sizes (optional): column t of E is u delta_t u_t, u_t = beta_t (v_t - alpha_t S_{t-1}
-        // k_t) the token's write.  The pass sums each column's squares over the warp's 32 rows,
-        // rescales them by the constant (1 / (u delta_t))^2 and adds them into s_u2 (four warps per
-        // column); at the next tile warp 0 takes the square roots and sums them into the head's total.
+        float den = 0.f;
+        // Deferred decay: TMEM holds S~ with the head's state S = sig * S~.  A tile folds its decay
+        // gamma_C into sig (the W pass applies sig and u_scale = 1 / (gamma_C sig), so MMA_S
+        // accumulates onto S~ with no pass over the state); when sig gamma_C would drop below
+        // kSigMin the tile instead writes gamma_C S back into TMEM and sig restarts at 1.
+        float sig = 1.f;
+        // Write sizes (optional): column t of the U region is u_t scaled by u_scale gamma_C /
+        // gamma_t, u_t = beta_t (v_t - alpha_t S_{t-1} k_t) the token's write.  The Ũ pass sums
+        // each column's squares over this warp's 32 rows and adds them, rescaled to u_t, into
+        // s_u2 (four warps per column); after the next barrier warp 0 takes the square roots and
+        // sums them over the tile's tokens into the head's total.
         const bool want_w = a.wnorm != nullptr;
-        float wacc = 0.f;                                  // warp 0: the slot's running sum
+        float wacc = 0.f;                                  // warp 0: the head's running sum
         int prev_lh = -1, prev_slot = -1;
         bool prev_last = false;
         // a head's write-size sum: to hand-over entry i when the slot begins a head shared with
@@ -1003,136 +1110,192 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             if (sch.is_prefix(slot)) {
                 a.ho_wsum[me] = sum;
                 __threadfence();
-                atomicOr(bits_wsum + (me >> 5), 1u << (me & 31));
+                grid_dep_wait();                           // (after the factor kernel's flag reset)
+                ho_store_release(a.ho_wflag + me, 1);
                 return true;
             }
             if (sch.is_suffix(slot)) {
-                const uint32_t bit = 1u << ((me - 1) & 31);
-                uint32_t* w = bits_wsum + ((me - 1) >> 5);
                 const uint64_t t0 = global_ns();
-                while ((ld_acquire(w) & bit) == 0) {
-                    if (*abort_flag || global_ns() - t0 > budget) return false;
+                while (ho_load_acquire(a.ho_wflag + me - 1) == 0) {
+                    if (*abort_flag || global_ns() - t0 > kWaitBudgetNs) return false;
                     __nanosleep(64);
                 }
-                sum += __ldcg(a.ho_wsum + me - 1);
-                atomicAnd(w, ~bit);
+                sum += *reinterpret_cast<volatile const float*>(a.ho_wsum + me - 1);
             }
             a.wnorm[lh] = sum;
             return true;
         };
         auto fold_writes = [&](int jj) {                   // warp 0: tile jj's sizes into wacc
             float* b = s_u2[jj & 1];
-            float sacc = sqrtf(b[lane]) + sqrtf(b[32 + lane]);
+            float sacc = sqrtf(b[lane]) + sqrtf(b[lane + 32]);
             b[lane] = 0.f;
-            b[32 + lane] = 0.f;
+            b[lane + 32] = 0.f;
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) sacc += __shfl_xor_sync(0xffffffffu, sacc, m);
             wacc += sacc;
         };
-        bool stop = NJ == 0;
-        if (!stop) {
-            // ---- the CTA's first slot: its state into TMEM, and W of its first tile
-            bool ok = install(0, den);
-            ok = make_w(0) && ok;
-            tmem_st_wait();
-            tc_fence_before();
-            if (!ok) fail(a.status, abort_flag, 14);
-            warp_arrive(&mb_ready, lane);
-        }
-        for (int j = 0; j < NJ && !stop; ++j) {
-            const int lh = cc.lh, slot = cc.k;
-            const bool last = cc.jt == cc.te - 1;          // the slot's last tile
-            if (named_sync_or(kBarChain, kChain, *abort_flag)) break;
-            if (want_w && j > 0 && warp == 0) {
-                fold_writes(j - 1);
-                if (prev_last) {
-                    if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 44);
-                    wacc = 0.f;
+        for (int j = 0; j < NJ; ++j) {                     // j: global tile index
+            const int lh = cc.lh, jt = cc.jt, slot = cc.k; // head, tile within the head, slot
+            const bool last = jt == cc.te - 1;             // the slot's last tile
+            if (named_sync_or(2, kChain, *abort_flag)) break;
+            if (!mbar_wait_or_abort(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
+            const float gC = rec_consts(j)[64];
+            float w_gamma = 0.f;                           // gamma_t of this lane's column in the Ũ pass
+            if (want_w) {
+                w_gamma = -rec_consts(j)[16 * cgp + (lane >> 1)];
+                if (j > 0 && warp == 0) {
+                    fold_writes(j - 1);
+                    if (prev_last) {
+                        if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 44);
+                        wacc = 0.f;
+                    }
                 }
             }
-            // ---- E(j) is complete (and E += S~ W has read the state and W)
-            if (!wait_bar(&mb_u, j & 1, budget, abort_flag)) fail(a.status, abort_flag, 10);
-            tc_fence_after();
-            const float* cs = cst + (j & 1) * kConstWords;
-            const float pass_f = cs[65];
-            const float sig_after = cs[64];
-            if (pass_f >= 0.f) {
-                // the decay would take the deferred scale out of range: S~ <- p S~ (the state
-                // update of this tile has not been issued: it waits for this pass)
-#pragma unroll 1
-                for (int g8 = 0; g8 < 8; ++g8) {
-                    float sv[16];
-                    tmem_ld16(tm + lane_off + TM_S + 16 * g8, sv);
-                    tmem_ld_wait();
-                    uint32_t su[16];
+
+            if (j == 0) {
+                // ---- the CTA's first head: its state from the staging buffer into TMEM, as S~
+                // (sig = 1) and as S_before, and sum S_before^2
+                if (!mbar_wait_or_abort(&mb_st, 0, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 14);
+                st_seen = 1;
+                float sv[32];
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) su[e] = __float_as_uint(sv[e] * pass_f);
-                    tmem_st16(tm + lane_off + TM_S + 16 * g8, su);
+                for (int e = 0; e < 8; ++e) {
+                    const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, 8 * cgp + e));
+                    sv[4 * e] = x.x; sv[4 * e + 1] = x.y; sv[4 * e + 2] = x.z; sv[4 * e + 3] = x.w;
                 }
+#pragma unroll
+                for (int e = 0; e < 32; ++e) den = fmaf(sv[e], sv[e], den);
+                warp_arrive(&mb_sfree, lane);                    // the staging buffer has been read
+                tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
+                tmem_st32(tm + lane_off + TM_SB + 32 * cgp, sv);
+                if (!make_k32(0)) fail(a.status, abort_flag, 16);
+                tmem_st_wait();
+                tc_fence_before();
+                warp_arrive(&mb_sready, lane);
             }
-#pragma unroll 1
-            for (int hh = 0; hh < 2; ++hh) {
-                // ---- pass: 32 token columns of E -> (hi, lo) A operand, in place
-                const uint32_t eb = tm + lane_off + TM_E + (j & 1) * 64 + 32 * hh;
-                float e[32];
-                tmem_ld32(eb, e);
+            const bool rescale = sig * gC < kSigMin;       // uniform over the CTA
+            const float u_scale = rescale ? 1.f : 1.f / (gC * sig);
+
+            // ---- W pass: W^T = V^T - sig X~^T diag(gamma) from the V and X regions (X~ = S~ K^T),
+            // scaled by u_scale, (hi, lo) in place over this thread's 16 X columns (tokens 16 cgp ..)
+            if (!mbar_wait_or_abort(&mb_x, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 10);
+            tc_fence_after();
+            {
+                float xv[16], vv[16], cf[16];
+                tmem_ld16(tm + lane_off + TM_X + 16 * cgp, xv);
+                tmem_ld16(tm + lane_off + TM_V + 16 * cgp, vv);
+                const float* gm = rec_consts(j) + 16 * cgp;         // -gamma of the thread's tokens
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float4 g4 = *reinterpret_cast<const float4*>(gm + 4 * e);
+                    cf[4 * e] = g4.x * sig; cf[4 * e + 1] = g4.y * sig; cf[4 * e + 2] = g4.z * sig; cf[4 * e + 3] = g4.w * sig;
+                }
+                tmem_ld_wait();
+                uint32_t hi[8], lo[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    split2(fmaf(cf[2 * i], xv[2 * i], vv[2 * i]) * u_scale,
+                           fmaf(cf[2 * i + 1], xv[2 * i + 1], vv[2 * i + 1]) * u_scale, hi[i], lo[i]);
+                tmem_st8(tm + lane_off + TM_X + 16 * cgp, hi);
+                tmem_st8(tm + lane_off + TM_X + 16 * cgp + 8, lo);
+                tmem_st_wait();
+            }
+            tc_fence_before();
+            warp_arrive(&mb_xready, lane);
+
+            // ---- while MMA_U runs: rescale S~ if the decay would underflow the deferred scale
+            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K(j+1) in fp32
+            if (rescale) {
+                const float f = gC * sig;
+                float sv[32];
+                tmem_ld32(tm + lane_off + TM_S + 32 * cgp, sv);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 32; ++e) sv[e] *= f;
+                tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
+                tmem_st_wait();
+            }
+            sig = rescale ? 1.f : gC * sig;                // the deferred decay after tile j
+            if (j + 1 < NJ && !make_k32(j + 1)) fail(a.status, abort_flag, 16);
+
+            // ---- U~ pass: (hi, lo) in place over this thread's 16 U columns
+            if (!mbar_wait_or_abort(&mb_u, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 11);
+            tc_fence_after();
+            {
+                float uv[16];
+                tmem_ld16(tm + lane_off + TM_U + 16 * cgp, uv);
                 tmem_ld_wait();
                 if (want_w) {
                     // squares summed over the warp's 32 rows, column by column: halving exchanges
-                    // leave lane c with column c
-                    const float wf = cs[32 * hh + lane];
-                    float x[32];
+                    // leave lanes 2c and 2c + 1 with column c (token 16 cgp + c) of the 16
+                    float x[16];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) x[i] = e[i] * e[i];
+                    for (int i = 0; i < 16; ++i) x[i] = uv[i] * uv[i];
 #pragma unroll
-                    for (int w = 16; w >= 1; w >>= 1) {
-                        const bool up = (lane & w) != 0;
+                    for (int w = 8, bit = 16; w >= 1; w >>= 1, bit >>= 1) {
+                        const bool up = (lane & bit) != 0;
 #pragma unroll
                         for (int i = 0; i < w; ++i) {
                             const float send = up ? x[i] : x[i + w];
-                            x[i] = (up ? x[i + w] : x[i]) + __shfl_xor_sync(0xffffffffu, send, w);
+                            x[i] = (up ? x[i + w] : x[i]) + __shfl_xor_sync(0xffffffffu, send, bit);
                         }
                     }
-                    atomicAdd(&s_u2[j & 1][32 * hh + lane], x[0] * wf * wf);
+                    x[0] += __shfl_xor_sync(0xffffffffu, x[0], 1);
+                    // U column -> u_t.  u_scale gamma_C is 1 / sig >= 1 unless the tile restarts
+                    // the deferred decay; then it is gamma_C, and below 2^-60 the columns of the
+                    // early tokens, scaled by gamma_C / gamma_t, are no longer representable: such
+                    // a tile contributes nothing
+                    const float sc = u_scale * gC;
+                    const float wf = sc >= 0x1p-60f ? w_gamma / sc : 0.f;
+                    if ((lane & 1) == 0) atomicAdd(&s_u2[j & 1][16 * cgp + (lane >> 1)], x[0] * wf * wf);
                 }
-                uint32_t hi[16], lo[16];
+                uint32_t hi[8], lo[8];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) split2(e[2 * i], e[2 * i + 1], hi[i], lo[i]);
-                tmem_st16(eb, hi);
-                tmem_st16(eb + 16, lo);
+                for (int i = 0; i < 8; ++i) split2(uv[2 * i], uv[2 * i + 1], hi[i], lo[i]);
+                tmem_st8(tm + lane_off + TM_U + 16 * cgp, hi);
+                tmem_st8(tm + lane_off + TM_U + 16 * cgp + 8, lo);
+                tmem_st_wait();
             }
-            tmem_st_wait();
             tc_fence_before();
             warp_arrive(&mb_uready, lane);
-            warp_arrive(&mb_iempty[j & 1], lane);          // the tile's constants are read
-            sig = sig_after;
-            // ---- while the state update runs: W of the next tile
-            const bool has_next = j + 1 < NJ;
-            bool ok = true;
-            if (has_next) ok = make_w(j + 1);
-            if (!ok) fail(a.status, abort_flag, 15);
-            if (last) {
-                // ---- slot boundary: S_after = sig S~ out, drift partials against S_before, the next
-                // slot's state in
-                const bool prefix = sch.is_prefix(slot);
-                const bool shared_end = sch.is_suffix(slot);   // S_before: the head's stored state
-                if (!wait_bar(&mb_s, j & 1, budget, abort_flag)) { fail(a.status, abort_flag, 12); ok = false; }
+            if (!last) {
+                // the next tile of this head may start X as soon as MMA_S(j) is queued
+                warp_arrive(&mb_sready, lane);
+            } else {
+                // ---- head boundary: S_after = sig S~ out through the staging buffer, the next
+                // head's state (staged meanwhile) into TMEM, drift partials against S_before
+                const bool has_next = j + 1 < NJ;          // uniform
+                // a last slot that ends a head begun by CTA i - 1: S_before is not in TMEM (the
+                // slot started from the handed-over state) but staged, and its square sum is taken
+                // here
+                const bool shared_end = sch.is_suffix(slot);
+                float den_end = 0.f;
+                bool ok = mbar_wait_or_abort(&mb_s, j & 1, kWaitBudgetNs, abort_flag);
+                if (!ok) fail(a.status, abort_flag, 12);
+                if (!mbar_wait_or_abort(&mb_st, st_seen & 1, kWaitBudgetNs, abort_flag)) {
+                    fail(a.status, abort_flag, 14);
+                    ok = false;
+                }
+                ++st_seen;
                 tc_fence_after();
-                float num = 0.f, den_end = 0.f;
-                float* dstp = (prefix ? a.ho_state + (size_t)me * kD * kD : a.state + (size_t)lh * kD * kD)
-                              + (size_t)r * kD;
-                const float* sbp = a.state + (size_t)lh * kD * kD + (size_t)r * kD;
+                float num = 0.f, den_next = 0.f;
                 if (ok) {
-#pragma unroll 1
-                    for (int g8 = 0; g8 < 8; ++g8) {
+#pragma unroll
+                    for (int half = 0; half < 2; ++half) {
+                        const uint32_t col = 32 * cgp + 16 * half;
+                        const int ch = 8 * cgp + 4 * half;     // this half's 16-byte chunks of row r
                         float sa[16], sb[16];
-                        tmem_ld16(tm + lane_off + TM_S + 16 * g8, sa);
+                        tmem_ld16(tm + lane_off + TM_S + col, sa);
                         if (shared_end) {
-                            ld16_global(sbp + 16 * g8, sb, true);
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
+                                sb[4 * e] = x.x; sb[4 * e + 1] = x.y; sb[4 * e + 2] = x.z; sb[4 * e + 3] = x.w;
+                            }
 #pragma unroll
                             for (int e = 0; e < 16; ++e) den_end = fmaf(sb[e], sb[e], den_end);
                         } else {
-                            tmem_ld16(tm + lane_off + TM_SB + 16 * g8, sb);
+                            tmem_ld16(tm + lane_off + TM_SB + col, sb);
                         }
                         tmem_ld_wait();
 #pragma unroll
@@ -1141,12 +1304,32 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                             const float d = sa[e] - sb[e];
                             num = fmaf(d, d, num);
                         }
-                        float4* o4 = reinterpret_cast<float4*>(dstp + 16 * g8);
+                        if (has_next) {
+                            uint32_t sn[16];
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) o4[e] = make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
+                            for (int e = 0; e < 4; ++e) {
+                                const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, ch + e));
+                                den_next = fmaf(x.x, x.x, den_next); den_next = fmaf(x.y, x.y, den_next);
+                                den_next = fmaf(x.z, x.z, den_next); den_next = fmaf(x.w, x.w, den_next);
+                                sn[4 * e] = __float_as_uint(x.x); sn[4 * e + 1] = __float_as_uint(x.y);
+                                sn[4 * e + 2] = __float_as_uint(x.z); sn[4 * e + 3] = __float_as_uint(x.w);
+                            }
+                            tmem_st16(tm + lane_off + TM_S + col, sn);
+                            tmem_st16(tm + lane_off + TM_SB + col, sn);
+                        }
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            *reinterpret_cast<float4*>(sbuf + sb_idx(r, ch + e)) =
+                                make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
                     }
+                    tmem_st_wait();
                 }
-                // partial sums: pairwise in fp32, over the warp's lanes and then over the warps
+                tc_fence_before();
+                fence_async_smem();                        // S_after -> the state warp's TMA store
+                warp_arrive(&mb_sfree, lane);
+                if (has_next) warp_arrive(&mb_sready, lane);     // the next head's state is in TMEM
+                // partial sums: pairwise in fp32, over the warp's lanes and then over the 16 warps
+                // (the FP64 pipe is far too slow for this path)
                 float fn = num, fd = shared_end ? den_end : den;
 #pragma unroll
                 for (int m = 16; m >= 1; m >>= 1) {
@@ -1154,10 +1337,8 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                     fd += __shfl_xor_sync(0xffffffffu, fd, m);
                 }
                 if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
-                if (prefix) __threadfence();                  // the hand-over state is in memory ...
-                if (named_sync_or(kBarChain, kChain, !ok || *abort_flag)) { stop = true; break; }
-                if (prefix && tid == 0) atomicOr(bits_state + (me >> 5), 1u << (me & 31));   // ... before CTA i + 1 reads it
-                if (warp == 0 && a.partials != nullptr && !prefix) {   // a shared head: at its end
+                if (named_sync_or(2, kChain, !ok)) break;
+                if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot)) {   // a shared head's drift: at its end
                     float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
                     float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
 #pragma unroll
@@ -1170,23 +1351,16 @@ gdn_fused_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                         a.partials[(size_t)lh * 2 + 1] = pd;
                     }
                 }
-                if (has_next) {
-                    if (!install(slot + 1, den)) fail(a.status, abort_flag, 16);
-                    tmem_st_wait();
-                }
+                den = den_next;
                 sig = 1.f;
-            }
-            if (has_next) {
-                tc_fence_before();
-                warp_arrive(&mb_ready, lane);               // W(j + 1) (and a new slot's state) ready
             }
             prev_lh = lh;
             prev_slot = slot;
             prev_last = last;
             cc.next(sch, a);
         }
-        // the CTA's last tile (always a slot's last) once every warp's pass has added to it
-        if (want_w && NJ > 0 && !named_sync_or(kBarChain, kChain, *abort_flag) && warp == 0) {
+        // the CTA's last tile (always a head's last) once every warp's Ũ pass has added to it
+        if (want_w && NJ > 0 && !named_sync_or(2, kChain, *abort_flag) && warp == 0) {
             fold_writes(NJ - 1);
             if (lane == 0 && !put_wsum(prev_slot, prev_lh, wacc)) fail(a.status, abort_flag, 45);
         }
@@ -1205,14 +1379,16 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = []() -> EncodeTiledFn {
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
         cudaDriverEntryPointQueryResult q;
         void* p = nullptr;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            return reinterpret_cast<EncodeTiledFn>(p);
-        return nullptr;
-    }();
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
     return fn;
 }
 
@@ -1230,30 +1406,42 @@ bool make_map(CUtensorMap* map, const void* base, int L, int T, int H) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Scratch (past the workspace header): the hand-over area for up to one CTA per SM: states
-// [grid][128][128] fp32, write-size sums [grid].
+// The state [L * Hv * 128][128] fp32 as a 2-D map: a box of 32 columns x 128 rows (one column block
+// of one head), 128-byte swizzle.
+bool make_state_map(CUtensorMap* map, void* base, int heads) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)heads * kD};
+    cuuint64_t strides[1] = {(cuuint64_t)kD * 4};
+    cuuint32_t box[2] = {32, (cuuint32_t)kD};
+    cuuint32_t es[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Scratch: the WY records, then the update kernel's hand-over area for up to one CTA per SM:
+// states [grid][128][128] fp32 (1024-aligned), flags [2][grid] int32, write-size sums [grid].
 struct TcScratch {
-    size_t ho_state, ho_wsum, total;
+    size_t rec, ho_state, ho_flags, ho_wsum, total;
 };
 
-TcScratch tc_scratch_layout(int L, int Hv) {
+TcScratch tc_scratch_layout(int L, int Hv, int T) {
     const int grid = std::max(1, std::min(L * Hv, device_sm_count()));
     TcScratch l;
-    l.ho_state = 0;
-    l.ho_wsum = (size_t)grid * kD * kD * 4;
+    l.rec = 0;
+    l.ho_state = ((size_t)L * Hv * ((T + kC - 1) / kC) * kRecBytes + 1023) & ~size_t(1023);
+    l.ho_flags = l.ho_state + (size_t)grid * kD * kD * 4;
+    l.ho_wsum = l.ho_flags + 2 * (size_t)grid * 4;
     l.total = l.ho_wsum + (size_t)grid * 4;
     return l;
 }
-
-// Equal tile runs, with heads split between neighbouring CTAs, when they shorten the slowest CTA:
-// a slot boundary costs about `kBoundary` tiles and a hand-over about `kHandOver`.
-constexpr double kBoundary = 0.6, kHandOver = 2.0;
 
 }  // namespace
 
 size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T) {
     if (dk != kD || dv != kD || dtype != DELTAS_BF16 || L <= 0 || Hv <= 0 || T <= 0) return 0;
-    return tc_scratch_layout(L, Hv).total;
+    return tc_scratch_layout(L, Hv, T).total;
 }
 
 bool gdn_tc_shape(const GdnArgs& a) {
@@ -1262,60 +1450,66 @@ bool gdn_tc_shape(const GdnArgs& a) {
 
 bool gdn_tc_supported(const GdnArgs& a) {
     return gdn_tc_shape(a) &&
-           a.Hk <= (1 << 24) && a.T < (1 << 30) &&
+           (long long)a.L * a.Hv * kD < (1ll << 31) &&                          // TMA row coordinate
+           (long long)a.L * a.Hv * ((a.T + kC - 1) / kC) < (1ll << 31) &&       // factor-kernel items
            a.scratch != nullptr &&
            a.scratch_bytes >= gdn_tc_scratch_bytes(a.L, a.Hv, a.dk, a.dv, a.dtype, a.T) &&
-           std::min(a.L * a.Hv, device_sm_count()) <= 512 &&                    // hand-over bits
            encode_fn() != nullptr;
 }
 
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
-    const TcScratch sl = tc_scratch_layout(a.L, a.Hv);
-    const int sms = device_sm_count();
-    const int H = a.L * a.Hv;
-    const int grid = std::min(H, sms);
-    CUtensorMap kmap, vmap;
-    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv)) return cudaErrorInvalidValue;
-    // The attribute is per device; setting it on every launch costs little and stays correct after
-    // a device reset and from any host thread.
-    cudaError_t e = cudaFuncSetAttribute(gdn_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemAlloc);
-    if (e != cudaSuccess) return e;
+    const TcScratch sl = tc_scratch_layout(a.L, a.Hv, a.T);
+    const int grid = std::min(a.L * a.Hv, device_sm_count());
+    CUtensorMap kmap, vmap, smap, hmap;
+    if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
+        !make_state_map(&smap, a.state, a.L * a.Hv) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
+        return cudaErrorInvalidValue;
+    static int configured_device = -1;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (configured_device != dev) {
+        cudaError_t e = cudaFuncSetAttribute(gdn_update_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kSmemAlloc);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(gdn_wy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kWySmemAlloc);
+        if (e != cudaSuccess) return e;
+        configured_device = dev;
+    }
     const int n_tiles = (a.T + kC - 1) / kC;
+    const int sms = device_sm_count();
+    // factor kernel: one record per (layer, value head, tile), kWyCtasPerSm persistent CTAs per SM
+    WyArgs w;
+    w.L = a.L; w.Hk = a.Hk; w.Hv = a.Hv; w.T = a.T; w.n_tiles = n_tiles;
+    w.g = a.g; w.beta = a.beta; w.rec = a.scratch; w.status = a.status;
+    w.ho_flags = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
+    w.n_ho_flags = 2 * grid;
+    const long long items = (long long)a.L * a.Hv * n_tiles;
+    const int wgrid = (int)std::min<long long>(items, (long long)sms * kWyCtasPerSm);
+    gdn_wy_kernel<<<wgrid, kWyThreads, kWySmemAlloc, s>>>(kmap, w);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // update kernel: one persistent CTA per SM (the kernel needs the whole SM: 512 TMEM columns,
+    // ~211 KB of shared memory); each takes every grid-th head, or an equal run of tiles
     TcArgs t;
     t.L = a.L; t.Hk = a.Hk; t.Hv = a.Hv; t.T = a.T; t.n_tiles = n_tiles;
-    t.g = a.g; t.beta = a.beta;
-    t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.status = a.status;
-    t.ho_bits = reinterpret_cast<uint32_t*>(a.status) + 4;
-    t.ho_state = reinterpret_cast<float*>(a.scratch + sl.ho_state);
+    t.state = a.state; t.partials = a.partials; t.wnorm = a.wnorm; t.rec = a.scratch; t.status = a.status;
+    t.ho_flag = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
+    t.ho_wflag = t.ho_flag + grid;
     t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
+    // equal tile runs, with heads split between neighbouring CTAs, when they shorten the slowest
+    // CTA: a boundary between slots costs about 0.45 of a tile and the hand-over about three
+    // tiles (measured: 512- and 1024-token chunks gain 5-6 %, chunks of 2-3 tiles lose)
     t.split = 0;
+    const int H = a.L * a.Hv;
     if (H > grid && H % grid != 0) {
-        const double whole = std::ceil((double)H / grid) * (n_tiles + kBoundary);
+        const double whole = std::ceil((double)H / grid) * (n_tiles + 0.45);
         const double runs = std::ceil((double)H * n_tiles / grid);
-        const double parted = runs + (runs / n_tiles + 2.0) * kBoundary + kHandOver;
+        const double parted = runs + (runs / n_tiles + 2.0) * 0.45 + 3.0;
         t.split = parted < whole ? 1 : 0;
     }
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemAlloc;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    if (t.split) {
-        // every CTA must be resident: a split head's second part waits for its first
-        attr[0].id = cudaLaunchAttributeCooperative;
-        attr[0].val.cooperative = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, gdn_fused_kernel, kmap, vmap, t);
-        if (e != cudaErrorCooperativeLaunchTooLarge) return e;
-        (void)cudaGetLastError();                 // fewer SMs than the grid: whole heads instead
-        t.split = 0;
-    }
-    cfg.attrs = nullptr;
-    cfg.numAttrs = 0;
-    return cudaLaunchKernelEx(&cfg, gdn_fused_kernel, kmap, vmap, t);
+    (void)sms;
+    return launch_dependent(gdn_update_tc_kernel, dim3(grid), dim3(kThreads), (size_t)kSmemAlloc, s, kmap, vmap,
+                            smap, hmap, t);
 }
 
 }  // namespace deltas

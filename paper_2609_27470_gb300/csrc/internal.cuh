@@ -12,8 +12,7 @@ namespace deltas {
 // ---------------------------------------------------------------------------------------------
 // Device status word: the first 16 bytes of every workspace.
 //   word[0] = first recorded deltas_status, word[1] = detail, word[2] = bounded-wait budget
-//   override in microseconds (0: about one second), word[3] reserved; words 4..35 of the 256-byte
-//   header are the tensor-core update's hand-over bits (zero between calls).
+//   override in microseconds (0: about one second), word[3] reserved.
 // ---------------------------------------------------------------------------------------------
 constexpr size_t kStatusBytes = 256;   // status word padded so the rest stays 256-byte aligned
 
