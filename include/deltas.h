@@ -27,7 +27,9 @@
  *   status word: kernels that detect an error on the device (a bounded wait that ran out, an
  *   out-of-range index) record the first such error there and skip the unsafe part of their
  *   work.  Zero it once with deltas_clear_device_status before first use; read it with
- *   deltas_get_device_status.  Calls sharing a workspace must be ordered on one stream.
+ *   deltas_get_device_status.  Calls sharing a workspace must be ordered on one stream.  After a
+ *   call that recorded an error, its outputs (and, for in-place calls, its in/out buffers) are
+ *   unspecified: parts of the work may have completed before the error stopped the rest.
  * - Return value: DELTAS_OK when the work was enqueued; DELTAS_ERR_INVALID_ARGUMENT /
  *   DELTAS_ERR_UNSUPPORTED / DELTAS_ERR_WORKSPACE when the host-side checks reject the call
  *   (nothing is enqueued then); DELTAS_ERR_CUDA when a launch failed.  No exception crosses the
@@ -231,8 +233,9 @@ DELTAS_API deltas_status deltas_select_retain(const deltas_policy* policy, int32
 /* scratch is a fixed device array inside the library sized for                                 */
 /* DELTAS_SELECT_STATIC_MAX_CACHE_LEN slots (about 2.25 MiB); a larger cache_len returns        */
 /* DELTAS_ERR_UNSUPPORTED with nothing enqueued.                                                */
-/*   - The first call on a device looks up the array's address (with that device current, the  */
-/*     stream must belong to it) and caches it; make that first call before any stream capture. */
+/*   - Every call looks up the array's address in the current context (the stream must belong  */
+/*     to the current device); the first call on a device loads the library's module there, so */
+/*     make it before any stream capture.                                                       */
 /*   - All calls on a device share the array.  Calls whose kernels may run at the same time on   */
 /*     the GPU (streams with no ordering between them) race and give undefined results.         */
 /*   - Each call clears the status word at the head of the array on its stream before the       */
@@ -392,6 +395,16 @@ DELTAS_API deltas_status deltas_compact_kv_heads(const deltas_kv_desc* desc, voi
 
 /* Enqueue a zeroing of the status word. */
 DELTAS_API deltas_status deltas_clear_device_status(void* workspace, void* stream);
+
+/* Enqueue on `stream` a write of the workspace's bounded-wait budget (word 2 of the status
+ * header): every wait of a kernel that runs with this workspace gives up after `budget_ns`
+ * nanoseconds (0, the value deltas_clear_device_status leaves: about one second) and records
+ * DELTAS_ERR_TIMEOUT; the waits that drain a kernel's own copies and MMAs before it exits keep the
+ * one-second budget.  Not a paper operation: a wait that runs out is the library's answer to a
+ * peer that never arrives (a CTA that cannot become resident, say), and a small budget lets a
+ * test or a latency-bound caller make that path run.  The host value is copied before the call
+ * returns. */
+DELTAS_API deltas_status deltas_set_wait_budget(void* workspace, uint32_t budget_ns, void* stream);
 
 /* Synchronise `stream`, then read the status word: *status_out = first recorded deltas_status
  * (DELTAS_OK if none), *detail_out = kernel-specific detail (e.g. the offending index); either

@@ -40,7 +40,7 @@ EXPORTED = (
     "deltas_append_kv", "deltas_copy_stream_state",
     "deltas_append_kv_heads", "deltas_select_retain_heads_workspace_size", "deltas_select_retain_heads",
     "deltas_compact_kv_heads_workspace_size", "deltas_compact_kv_heads", "deltas_copy_stream_state_heads",
-    "deltas_clear_device_status", "deltas_get_device_status",
+    "deltas_clear_device_status", "deltas_set_wait_budget", "deltas_get_device_status",
 )
 
 
@@ -101,6 +101,7 @@ _sig("deltas_select_retain_heads", ctypes.c_int, _P, _I32, _I32, _I32, _P, _P, _
 _sig("deltas_compact_kv_heads_workspace_size", _SZ, _P, _I32)
 _sig("deltas_compact_kv_heads", ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, _I32, _P, _I32, _P, _SZ, _P)
 _sig("deltas_clear_device_status", ctypes.c_int, _P, _P)
+_sig("deltas_set_wait_budget", ctypes.c_int, _P, ctypes.c_uint32, _P)
 _sig("deltas_get_device_status", ctypes.c_int, _P, _P, _P, _P)
 
 _TORCH_DT = {DELTAS_F32: torch.float32, DELTAS_BF16: torch.bfloat16}
@@ -427,6 +428,12 @@ def deltas_copy_stream_state(gdn: GdnDesc, kv: KvDesc | None, cache_len: int, n_
 def deltas_clear_device_status(workspace, stream=None):
     _check(_lib.deltas_clear_device_status(_ptr(workspace, torch.uint8, None, "workspace"), _stream(stream)),
            "deltas_clear_device_status")
+
+
+def deltas_set_wait_budget(workspace, budget_ns: int, stream=None):
+    """Bounded-wait budget of the kernels that run with this workspace (0: about one second)."""
+    _check(_lib.deltas_set_wait_budget(_ptr(workspace, torch.uint8, None, "workspace"), int(budget_ns),
+                                       _stream(stream)), "deltas_set_wait_budget")
 
 
 def deltas_get_device_status(workspace, stream=None):

@@ -433,6 +433,13 @@ deltas_status deltas_clear_device_status(void* workspace, void* stream) {
     return from_cuda(cudaMemsetAsync(workspace, 0, kStatusBytes, as_stream(stream)));
 }
 
+deltas_status deltas_set_wait_budget(void* workspace, uint32_t budget_ns, void* stream) {
+    if (workspace == nullptr) return DELTAS_ERR_WORKSPACE;
+    const uint32_t v = budget_ns;      // pageable source: copied before cudaMemcpyAsync returns
+    return from_cuda(cudaMemcpyAsync(static_cast<uint8_t*>(workspace) + 8, &v, sizeof(v), cudaMemcpyHostToDevice,
+                                     as_stream(stream)));
+}
+
 deltas_status deltas_get_device_status(const void* workspace, void* stream,
                                        int32_t* status_out, int32_t* detail_out)
 {

@@ -19,8 +19,8 @@
 // form across tiles.  Units are claimed through an atomic ticket in tile-major order, so a unit
 // only waits for units that were claimed earlier by running CTAs whose loads complete without
 // waiting on anything: no deadlock.
-// Every wait is bounded (about one second); a wait that runs out records DELTAS_ERR_TIMEOUT,
-// raises the abort flag and skips its writes.  Traffic is the algorithmic minimum: each moved row
+// Every wait is bounded (about one second, or the workspace's budget); a wait that runs out
+// records DELTAS_ERR_TIMEOUT, raises the abort flag and skips its writes.  Traffic is the algorithmic minimum: each moved row
 // is read once and written once; rows that do not move are not touched.
 #include <algorithm>
 #include <climits>
@@ -179,6 +179,7 @@ compact_main_kernel(CompactArgs a)
 
     grid_dep_wait();                                   // the prepass is done
     volatile int* abort_flag = &a.ctl->abort;
+    const uint64_t budget = wait_budget_ns(a.status);  // the drain below keeps kWaitBudgetNs
     if (*abort_flag) return;
     const int n = *a.n_retained;
     const int first_min = a.ctl->first_min;
@@ -234,7 +235,7 @@ compact_main_kernel(CompactArgs a)
                     mstage[m * a.tile_rows + (r - j0)] = reinterpret_cast<const int32_t*>(a.meta[m])[meta_off + src];
         }
         load_pending = true;
-        bool ok = mbar_wait_or_abort(&bar, phase, kWaitBudgetNs, abort_flag);
+        bool ok = mbar_wait_or_abort(&bar, phase, budget, abort_flag);
         ok = __all_sync(0xffffffffu, ok) != 0;
         if (ok) { phase ^= 1; load_pending = false; }
         if (!ok) {
@@ -256,7 +257,7 @@ compact_main_kernel(CompactArgs a)
             for (;;) {
                 const bool ready = (mine >= b) || load_acquire(f) != 0;
                 if (__all_sync(0xffffffffu, ready)) break;
-                if (*abort_flag || global_ns() - t_start > kWaitBudgetNs) { ok = false; break; }
+                if (*abort_flag || global_ns() - t_start > budget) { ok = false; break; }
                 __nanosleep(32);
             }
         }

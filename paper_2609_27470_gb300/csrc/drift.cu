@@ -6,10 +6,10 @@
 // The difference is formed element by element before squaring, never as
 // |A|^2 - 2<A,B> + |B|^2, which cancels badly when the drift is small.
 //
-// score_chunks: one CTA reduces the [L][Hv][2] partials in a fixed order (lane-strided double
-// sums, a fixed xor tree per layer, layer terms added in a fixed order), applies
-// sqrt(num_l)/sqrt(den_l) per layer with the zero-norm reading (0/0 -> 0, x/0 -> +inf) and stores
-// the layer mean as the chunk's score.
+// score_chunks: one CTA reduces the [L][Hv][2] partials in a fixed order (one warp per layer:
+// lane-strided float sums over the heads, a fixed xor tree), applies sqrt(num_l)/sqrt(den_l) per
+// layer in float with the zero-norm reading (0/0 -> 0, x/0 -> +inf), adds the layer terms in
+// double in a fixed order and stores the layer mean as the chunk's score.
 #include "internal.cuh"
 
 namespace deltas {

@@ -1115,6 +1115,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 return true;
             }
             if (sch.is_suffix(slot)) {
+                grid_dep_wait();                           // (the factor kernel's reset of the flag is complete)
                 const uint64_t t0 = global_ns();
                 while (ho_load_acquire(a.ho_wflag + me - 1) == 0) {
                     if (*abort_flag || global_ns() - t0 > kWaitBudgetNs) return false;
@@ -1464,16 +1465,12 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
         !make_state_map(&smap, a.state, a.L * a.Hv) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
         return cudaErrorInvalidValue;
-    static int configured_device = -1;
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (configured_device != dev) {
+    {   // set on every launch (cheap, and right for whichever device and context is current)
         cudaError_t e = cudaFuncSetAttribute(gdn_update_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)kSmemAlloc);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(gdn_wy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kWySmemAlloc);
         if (e != cudaSuccess) return e;
-        configured_device = dev;
     }
     const int n_tiles = (a.T + kC - 1) / kC;
     const int sms = device_sm_count();

@@ -11,8 +11,8 @@ namespace deltas {
 
 // ---------------------------------------------------------------------------------------------
 // Device status word: the first 16 bytes of every workspace.
-//   word[0] = first recorded deltas_status, word[1] = detail, word[2] = bounded-wait budget
-//   override in microseconds (0: about one second), word[3] reserved.
+//   word[0] = first recorded deltas_status, word[1] = detail, word[2] = bounded-wait budget in
+//   nanoseconds (0: kWaitBudgetNs), word[3] reserved.
 // ---------------------------------------------------------------------------------------------
 constexpr size_t kStatusBytes = 256;   // status word padded so the rest stays 256-byte aligned
 
@@ -31,6 +31,13 @@ __device__ __forceinline__ uint64_t global_ns() {
 
 // Bounded-wait budget for every device-side spin (inter-CTA flags, mbarriers): about one second.
 constexpr uint64_t kWaitBudgetNs = 1000000000ull;
+
+// The budget of one call's waits: word 2 of its workspace header (nanoseconds, set by
+// deltas_set_wait_budget), or kWaitBudgetNs when that word is zero.
+__device__ __forceinline__ uint64_t wait_budget_ns(const int32_t* status) {
+    const uint32_t v = status != nullptr ? reinterpret_cast<const volatile uint32_t*>(status)[2] : 0u;
+    return v != 0u ? (uint64_t)v : kWaitBudgetNs;
+}
 
 __device__ __forceinline__ float to_f32(float x) { return x; }
 __device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }

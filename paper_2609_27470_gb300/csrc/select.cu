@@ -519,15 +519,13 @@ cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_
 // HBM through its own pool or arena, or code running where cudaMalloc and friends are not allowed).
 //
 // The scratch is one file-scope array sized for DELTAS_SELECT_STATIC_MAX_CACHE_LEN slots.  Its
-// address is looked up with cudaGetSymbolAddress the first time the entry point runs on a device
-// (with that device current) and cached per device.  Every call on a device shares the array and
+// address is looked up with cudaGetSymbolAddress on every call, with the caller's device current
+// (the first call on a device loads the module there, so make it before any stream capture).  Every call on a device shares the array and
 // finds it as the previous call left it: the status word at its head is the only part that has to
 // start at zero, and it is cleared on the caller's stream before each launch; every other word the
 // kernel reads was written earlier in the same launch.  Calls whose kernels can overlap on the GPU
 // (different streams without ordering between them) race on the array.
 // -------------------------------------------------------------------------------------------------
-#include <mutex>
-
 namespace {
 
 constexpr size_t kStaticMaxSlots = DELTAS_SELECT_STATIC_MAX_CACHE_LEN;
@@ -538,21 +536,12 @@ static_assert(kStaticScratchBytes % 256 == 0, "every scratch array must stay 256
 
 static __device__ __align__(256) unsigned char g_select_scratch[kStaticScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_scratch_mutex;
-void* g_scratch_ptr[kMaxDevices] = {};
-
+// The array's device address, looked up on every call: it belongs to the current context (a device
+// reset or another context on the same device gives it another), and the lookup allocates nothing.
 deltas_status static_scratch_for_current_device(void** out) {
-    int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess) return DELTAS_ERR_CUDA;
-    if (dev < 0 || dev >= kMaxDevices) return DELTAS_ERR_UNSUPPORTED;
-    std::lock_guard<std::mutex> lock(g_scratch_mutex);
-    if (g_scratch_ptr[dev] == nullptr) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_select_scratch) != cudaSuccess || p == nullptr) return DELTAS_ERR_CUDA;
-        g_scratch_ptr[dev] = p;
-    }
-    *out = g_scratch_ptr[dev];
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_select_scratch) != cudaSuccess || p == nullptr) return DELTAS_ERR_CUDA;
+    *out = p;
     return DELTAS_OK;
 }
 

@@ -493,15 +493,10 @@ cudaError_t launch_select_heads(const deltas_policy& pol, int n_planes, int cach
     const int n_cand = std::max(0, cache_len - a.n_s - a.n_w);
     a.keys_in_smem = select_heads_smem_bytes(n_cand, a.N, true) <= kHeadSmemLimit;
     const size_t smem = select_heads_smem_bytes(n_cand, a.N, a.keys_in_smem != 0);
-    static int configured_device = -1;                 // the attribute is set once per device
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    // set on every launch (cheap, and right for whichever device and context is current)
+    const cudaError_t e = cudaFuncSetAttribute(select_heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)kHeadSmemLimit);
     if (e != cudaSuccess) return e;
-    if (configured_device != dev) {
-        e = cudaFuncSetAttribute(select_heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kHeadSmemLimit);
-        if (e != cudaSuccess) return e;
-        configured_device = dev;
-    }
     return launch_dependent(select_heads_kernel, dim3(n_planes), dim3(kHeadThreads), smem, s, a);
 }
 

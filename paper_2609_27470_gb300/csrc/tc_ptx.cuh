@@ -41,6 +41,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
+// Non-blocking test of a phase (try_wait may suspend the thread for a system-dependent time).
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{\n\t.reg .pred p;\n\t"
+                 "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                 "selp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+    return ok != 0;
+}
+
 // try_wait that lets the hardware suspend the thread until the phase completes or about
 // `hint_ns` nanoseconds pass, so a waiting warp takes no issue slots from the warps doing work.
 __device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
@@ -57,9 +67,15 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t pari
 // "budget_ns" is approximate: cycles = ns * 2 (about one second at the 2.07 GHz boost clock,
 // proportionally longer at lower clocks).
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t budget_ns) {
-    if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     const long long budget = (long long)(budget_ns * 2);
+    if (budget_ns < 20000u) {
+        for (;;) {
+            if (mbar_test_wait(bar, parity)) return true;
+            if (clock64() - t0 > budget) return false;
+        }
+    }
+    if (mbar_try_wait(bar, parity)) return true;
     for (;;) {
         if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
         if (clock64() - t0 > budget) return false;
@@ -69,9 +85,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
 // As mbar_wait, but also gives up as soon as *abort becomes nonzero (another role failed).
 __device__ __forceinline__ bool mbar_wait_or_abort(uint64_t* bar, uint32_t parity, uint64_t budget_ns,
                                                    const volatile int* abort) {
-    if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     const long long budget = (long long)(budget_ns * 2);
+    if (budget_ns < 20000u) {          // a short budget: non-blocking tests, so it holds to the cycle
+        for (;;) {
+            if (mbar_test_wait(bar, parity)) return true;
+            if (*abort) return false;
+            if (clock64() - t0 > budget) return false;
+        }
+    }
+    if (mbar_try_wait(bar, parity)) return true;
     for (;;) {
         if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
         if (*abort) return false;

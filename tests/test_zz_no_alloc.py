@@ -80,13 +80,24 @@ def test_static_select_matches_workspace_select_twice(L):
     """Two calls in a row on different inputs (the second finds the first one's leftovers in the
     shared scratch), each equal to the workspace entry point's result: bit-exact, as every
     selection test is."""
+    rng = np.random.default_rng(4)
+    stream_tc = np.repeat(np.arange(40, dtype=np.int32), 512)        # 40 runs of one chunk each
+    stream_sc = rng.exponential(size=40).astype(np.float32)
+    stream_sc[[7, 21]] = stream_sc[3]
+    keep_tc = np.repeat(np.arange(10, dtype=np.int32), 500)          # 5000 slots under the budget
     cases = [
         (L.policy(20000, 4, 1024, 4), *_case(1, 60000, 3000, 6)),     # largest size, thousands of runs
         (L.policy(9000, 4, 512, 3), *_case(2, 23000, 700, 4)),        # smaller, other policy
+        # right after a many-run call: a streaming-shaped cache with a few dozen runs (the decision
+        # kernel's direct path, which stages run starts, kept counts and offsets in the scratch)
+        (L.policy(16000, 4, 1024, 4), stream_tc, stream_sc),
+        # right after an eviction: a cache within the budget (everything kept; a stale emit flag
+        # from the previous call must not be used)
+        (L.policy(8000, 4, 1024, 4), keep_tc, rng.exponential(size=10).astype(np.float32)),
     ]
     for pol, tc, sc in cases:
         (n_ref, idx_ref, mask_ref), (n, idx, mask) = _select_both(L, pol, tc, sc)
-        assert n_ref == pol.budget_M and n == n_ref
+        assert n_ref == min(pol.budget_M, tc.size) and n == n_ref
         assert np.array_equal(idx, idx_ref)
         assert np.array_equal(mask, mask_ref)
 
