@@ -397,6 +397,58 @@ class GdnOnlyWorkload:
         return self.scores[i: i + 1]
 
 
+class DriftWorkload:
+    """drift: the standalone drift partials (deltas_state_drift) of a whole stack's states plus the
+    chunk score, one chunk per step, from a ring of (S_before, S_after) pairs larger than L2."""
+    name = "drift"
+
+    def __init__(self, dev, L, cfg=None):
+        cfg = dict(cfg or configs.DRIFT)
+        self.cfg = cfg
+        self.L = L
+        self.gdn = L.gdn_desc(cfg["L"], cfg["Hk"], cfg["Hv"], cfg["d"], torch.bfloat16)
+        self.pairs = [(inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 60 + 2 * i, device=dev),
+                       inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 61 + 2 * i, device=dev))
+                      for i in range(cfg["ring"])]
+        self.part = torch.zeros(cfg["L"], cfg["Hv"], 2, device=dev)
+        self.scores = torch.zeros(cfg["n_chunks"], device=dev)
+        self.ws = L.alloc_workspace(L.deltas_state_drift_workspace_size(self.gdn), dev)
+        self.step_i = 0
+
+    def step(self, timer):
+        sb, sa = self.pairs[self.step_i % len(self.pairs)]
+        with timer.mark("drift"):
+            self.L.deltas_state_drift(self.gdn, sb, sa, self.part, self.ws)
+        with timer.mark("score"):
+            self.L.deltas_score_chunks(self.cfg["L"], self.cfg["Hv"], self.part,
+                                       self.step_i % self.cfg["n_chunks"], self.scores)
+        self.step_i += 1
+
+    def launches_per_step(self):
+        return 1 + 1                                            # drift, score
+
+    def tokens_per_step(self):
+        return self.cfg["chunk_len"]
+
+    def kernel_roofline(self, name, avg_ms, peaks, steps):
+        if name != "drift":
+            return None
+        c = self.cfg
+        by = 2.0 * c["L"] * c["Hv"] * c["d"] * c["d"] * 4 + c["L"] * c["Hv"] * 8   # both states read, partials written
+        return {"bound": "hbm", "achieved": by / (avg_ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "bytes_per_launch": by}
+
+    def post_step(self):
+        pass
+
+    def h2d_tensors(self, i=0):
+        return list(self.pairs[i % len(self.pairs)])
+
+    def result_scalar(self):
+        i = (self.step_i - 1) % self.cfg["n_chunks"]
+        return self.scores[i: i + 1]
+
+
 class KvWorkload:
     """One eviction on a full 64k-token cache per step (select + compact); the cache is restored
     from a pristine copy between steps (outside the timed events)."""
@@ -467,6 +519,7 @@ KERNEL_SOURCES = {"gdn_update": "paper_2609_27470_gb300/csrc/gdn_tc.cu",
                   "score": "paper_2609_27470_gb300/csrc/drift.cu",
                   "append": "paper_2609_27470_gb300/csrc/compact.cu",
                   "snapshot": "paper_2609_27470_gb300/csrc/snapshot.cu",
+                  "drift": "paper_2609_27470_gb300/csrc/drift.cu",
                   "restore": "paper_2609_27470_gb300/csrc/snapshot.cu"}
 
 
@@ -555,6 +608,8 @@ def make_workload(name, dev, L):
         return GdnOnlyWorkload(dev, L, configs.LAYER)
     if name == "kv":
         return KvWorkload(dev, L)
+    if name == "drift":
+        return DriftWorkload(dev, L)
     if name == "snapshot":
         return SnapshotWorkload(dev, L)
     raise ValueError(name)
@@ -635,14 +690,43 @@ def e2e_pipelined(wl, host, steps, stream, dev, timer_off):
 
 # ----------------------------------------------------------------------------------- CPU oracle
 
-def oracle_sample(workload: str, budget_s: float = 12.0):
-    """Times the CPU oracle (single thread) on a bounded sample of one step of the workload and
-    extrapolates to a whole step.  Returns (tokens_per_s, sample description, seconds spent)."""
+def _pool_time(fn, n_items, threads):
+    """Seconds for fn(i), i < n_items, on `threads` threads (the oracle's C calls release the GIL)."""
+    t0 = time.perf_counter()
+    if threads <= 1:
+        for i in range(n_items):
+            fn(i)
+    else:
+        from concurrent.futures import ThreadPoolExecutor
+        with ThreadPoolExecutor(max_workers=threads) as ex:
+            list(ex.map(fn, range(n_items)))
+    return time.perf_counter() - t0
+
+
+def oracle_sample(workload: str, budget_s: float = 12.0, threads: int = 1):
+    """Times the CPU oracle on a bounded sample of one step of the workload and extrapolates to a
+    whole step: on one thread, or with the independent (layer, head) recurrences and compaction
+    planes spread over `threads` threads.  Returns (tokens_per_s, sample description, seconds
+    spent, extrapolation factor of the sampled part)."""
     import oracle
     t_start = time.perf_counter()
     cfg = _cfg(workload)
     parts = []
     total = 0.0
+    factor = 1.0
+    if workload == "drift":
+        heads_total = cfg["L"] * cfg["Hv"]
+        n = max(64, 8 * threads)
+        sb = inputs.initial_state(1, n, cfg["d"], 60).double().numpy()
+        sa = inputs.initial_state(1, n, cfg["d"], 61).double().numpy()
+        t = _pool_time(lambda i: oracle.drift_partials(sb[:, i:i + 1], sa[:, i:i + 1]), n, threads)
+        factor = heads_total / n
+        total += t * factor
+        p = np.ones((cfg["L"], cfg["Hv"], 2))
+        t0 = time.perf_counter()
+        oracle.chunk_score(p)
+        total += time.perf_counter() - t0
+        parts.append(f"drift of {n} (layer,head) state pairs x{factor:.0f} extrapolated; score of {cfg['L']} layers")
     head_signal = cfg.get("signal") in ("key_norm", "value_norm")
     if workload in ("streaming", "paper", "paper_write_norm", "paper_key_norm", "paper_value_norm", "stack",
                     "layer"):
@@ -652,24 +736,26 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         x = inputs.gdn_chunk(1, C, 1, 1, cfg["d"], "bf16", 77)
         f = {k: v.float().numpy() for k, v in x.items()}
         s0 = inputs.initial_state(1, 1, cfg["d"], 78).double().numpy()
-        t0 = time.perf_counter()
-        reps = 0
-        while True:
+
+        def one_head(_):
             if workload == "paper_write_norm":
-                S, _, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0, want_write_norms=True)
+                oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0, want_write_norms=True)
             elif head_signal:                              # the state moves; no drift is formed
-                S, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
+                oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
             else:
                 S, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
                 oracle.drift_partials(s0, S)
-            reps += 1
-            if reps >= n_heads and time.perf_counter() - t0 > budget_s * 0.5:
+        batch = max(n_heads, threads)
+        reps, t_sum = 0, 0.0
+        while True:
+            t_sum += _pool_time(one_head, batch, threads)
+            reps += batch
+            if t_sum > budget_s * 0.5 or reps >= 64 * max(1, threads):
                 break
-            if reps >= 64:
-                break
-        t_head = (time.perf_counter() - t0) / reps
+        t_head = t_sum / reps
+        factor = heads_total / reps
         total += t_head * heads_total
-        parts.append(f"gdn: {reps} (layer,head) x {C} tokens, x{heads_total / reps:.0f} extrapolated")
+        parts.append(f"gdn: {reps} (layer,head) x {C} tokens on {threads} thread(s), x{factor:.0f} extrapolated")
     if workload == "snapshot":
         # the oracle's question handling copies the whole stream state (numpy .copy()); timed on
         # a 64 MiB slice and scaled to the bytes of one save and one restore
@@ -705,11 +791,10 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         t_sel = time.perf_counter() - t0
         planes_total = 2 * cfg["Lf"] * cfg["Hkv"]
         plane = np.random.default_rng(6).integers(-2**15, 2**15, size=(2, T, cfg["D"]), dtype=np.int16)
-        t0 = time.perf_counter()
-        oracle.compact_rows(plane, idx, T)
-        t_cmp = (time.perf_counter() - t0) * planes_total / 2
+        n_pairs = max(1, min(threads, planes_total // 2))
+        t_cmp = _pool_time(lambda i: oracle.compact_rows(plane, idx, T), n_pairs, threads) * planes_total / (2 * n_pairs)
         total += t_sel + t_cmp
-        parts.append(f"select on {T} slots; compact 2 of {planes_total} planes x{planes_total // 2}")
+        parts.append(f"select on {T} slots; compact {2 * n_pairs} of {planes_total} planes x{planes_total // (2 * n_pairs)}")
     if head_signal:
         # score the chunk's rows, then per (layer, KV head) plane: select among M + C slots with
         # per-token scores and gather the plane's K and V rows; one plane timed, x planes
@@ -735,28 +820,37 @@ def oracle_sample(workload: str, budget_s: float = 12.0):
         t_cmp = time.perf_counter() - t0
         total += t_score + P * (t_sel + t_cmp)
         parts.append(f"score {P}x{C} rows; select on {T} slots and compact K, V, metadata of 1 of {P} planes x{P}")
-    return _tokens(workload) / total, "; ".join(parts), time.perf_counter() - t_start
+    return _tokens(workload) / total, "; ".join(parts), time.perf_counter() - t_start, factor
 
 
 # ----------------------------------------------------------------------------------- main
 
 def run_reference(args):
+    """The oracle as it stands, on this host's cores, one sampled step per timed step: each timed
+    step runs the oracle on a bounded sample of the workload's step (a few (layer, head)
+    recurrences and compaction planes), and `value` extrapolates the sample to the whole step.
+    ms_per_step is the wall time of the sampled steps actually run, so steps x ms_per_step is the
+    time this arm took."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    vals = []
-    desc = ""
+    vals, walls = [], []
+    desc, factor = "", 1.0
     for _ in range(args.warmup):
         oracle_sample(args.workload, budget_s=1.0)
     for _ in range(args.steps):
-        v, desc, _ = oracle_sample(args.workload, budget_s=2.0)
+        v, desc, wall, factor = oracle_sample(args.workload, budget_s=2.0)
         vals.append(v)
+        walls.append(wall)
     value = float(np.median(vals))
     out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
-           "warmup": args.warmup, "ms_per_step": 1e3 * _tokens(args.workload) / value,
+           "warmup": args.warmup, "ms_per_step": 1e3 * float(np.mean(walls)),
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic", "impl": "reference",
            "config": config_line(args.workload),
+           "timing": {"per_step": "one bounded sample of the workload's step, extrapolated to the whole step",
+                      "extrapolation_factor": factor,
+                      "ms_per_full_step_extrapolated": 1e3 * _tokens(args.workload) / value},
            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": desc},
            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
@@ -782,7 +876,7 @@ def config_line(workload):
 
 def _cfg(workload):
     return {"streaming": configs.STREAMING, "paper": configs.PAPER, "stack": configs.STACK,
-            "layer": configs.LAYER, "kv": configs.KV, "snapshot": configs.PAPER,
+            "layer": configs.LAYER, "kv": configs.KV, "snapshot": configs.PAPER, "drift": configs.DRIFT,
             "paper_write_norm": configs.PAPER_WRITE_NORM, "paper_key_norm": configs.PAPER_KEY_NORM,
             "paper_value_norm": configs.PAPER_VALUE_NORM}[workload]
 
@@ -806,7 +900,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="streaming",
                     choices=["streaming", "paper", "paper_write_norm", "paper_key_norm", "paper_value_norm",
-                             "stack", "layer", "kv", "snapshot"])
+                             "stack", "layer", "kv", "snapshot", "drift"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
@@ -913,8 +1007,11 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, desc, _ = oracle_sample(args.workload)
-        cpu = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": desc}
+        v, desc, _, _ = oracle_sample(args.workload)
+        n_cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+        va, desc_a, _, _ = oracle_sample(args.workload, budget_s=6.0, threads=n_cores)
+        cpu = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": desc,
+               "all_cores": {"value": va, "unit": "tokens/s", "cores": n_cores, "sample": desc_a}}
 
     if rank == 0:
         cfg_line = config_line(args.workload)

@@ -28,6 +28,10 @@ LAYER = dict(name="layer", L=1, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=102
 STACK = dict(name="stack", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=1024, n_chunks=256,
              ring=8)
 
+# the standalone drift (Eq. 3) of the full stack's states: S_before and S_after of 24 layers x 32
+# value heads x 128 x 128 fp32 (48 MiB each), a ring of 4 pairs (384 MiB, beyond L2)
+DRIFT = dict(name="drift", L=24, Hk=16, Hv=32, d=128, chunk_len=512, n_chunks=4096, ring=4)
+
 KV = dict(name="kv", Lf=8, Hkv=2, D=256, kv_dtype="bf16", chunk_len=1024, n_chunks=64,
           budget_M=16384)
 

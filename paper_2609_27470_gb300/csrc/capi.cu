@@ -2,12 +2,51 @@
 //
 // This layer validates arguments on the host (nothing is enqueued when a check fails), carves the
 // caller's workspace, and enqueues the kernels on the caller's stream.  It allocates nothing.
+#include <algorithm>
 #include <cstdint>
 #include <cstring>
+#include <mutex>
+
+#include <cuda.h>
 
 #include "internal.cuh"
 
 namespace deltas {
+
+// The SMs the current context may use: its SM resource (a green context's partition, the whole
+// device for an ordinary context), else the device attribute.  Asked on every call: the answer
+// belongs to the context, not to the device ordinal.  The driver calls come through the runtime's
+// entry-point lookup (no link against libcuda).
+int context_sm_count() {
+    using GetCurrentFn = CUresult (*)(CUcontext*);
+    using GetResourceFn = CUresult (*)(CUcontext, CUdevResource*, CUdevResourceType);
+    static GetCurrentFn get_current = nullptr;
+    static GetResourceFn get_resource = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        cudaDriverEntryPointQueryResult q;
+        void* p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<GetCurrentFn>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetDevResource", &p, 12040, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_resource = reinterpret_cast<GetResourceFn>(p);
+    });
+    const int device = device_sm_count();
+    if (get_current != nullptr && get_resource != nullptr) {
+        CUcontext ctx = nullptr;
+        if (get_current(&ctx) == CUDA_SUCCESS && ctx != nullptr) {
+            CUdevResource r;
+            std::memset(&r, 0, sizeof(r));
+            if (get_resource(ctx, &r, CU_DEV_RESOURCE_TYPE_SM) == CUDA_SUCCESS && r.type == CU_DEV_RESOURCE_TYPE_SM &&
+                r.sm.smCount > 0)
+                return std::min((int)r.sm.smCount, device);
+        }
+    }
+    return device;
+}
 
 int device_sm_count() {
     // cached per device: the attribute query is cheap but not free

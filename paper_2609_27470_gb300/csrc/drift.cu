@@ -1,7 +1,7 @@
 // State drift (Sec. 3.2, Eq. 3) from two stored states, and the chunk score from drift partials.
 //
 // state_drift: one CTA per (layer, value head) streams both d_v x d_k states once with 16-byte
-// loads (HBM-bound: 2 * 4 * d_v * d_k bytes per head) and writes
+// loads, four pairs in flight per thread (HBM-bound: 2 * 4 * d_v * d_k bytes per head), and writes
 //   partials[l][h] = { sum (S_after - S_before)^2, sum S_before^2 }.
 // The difference is formed element by element before squaring, never as
 // |A|^2 - 2<A,B> + |B|^2, which cancels badly when the drift is small.
@@ -16,6 +16,7 @@ namespace deltas {
 namespace {
 
 constexpr int kDriftThreads = 256;
+constexpr int kDriftUnroll = 4;        // float4 pairs in flight per thread
 
 __global__ void __launch_bounds__(kDriftThreads)
 state_drift_kernel(int n_elem4, const float4* __restrict__ sb, const float4* __restrict__ sa,
@@ -23,19 +24,29 @@ state_drift_kernel(int n_elem4, const float4* __restrict__ sb, const float4* __r
 {
     const size_t base = (size_t)blockIdx.x * n_elem4;
     float num = 0.f, den = 0.f;
-    for (int e = threadIdx.x; e < n_elem4; e += kDriftThreads) {
-        const float4 b = __ldcs(sb + base + e);   // streamed once: evict-first
-        const float4 a = __ldcs(sa + base + e);
-        const float dx = a.x - b.x, dy = a.y - b.y, dz = a.z - b.z, dw = a.w - b.w;
-        num += dx * dx + dy * dy + dz * dz + dw * dw;
-        den += b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
+    for (int e = threadIdx.x; e < n_elem4; e += kDriftThreads * kDriftUnroll) {
+        float4 b[kDriftUnroll], a[kDriftUnroll];
+#pragma unroll
+        for (int u = 0; u < kDriftUnroll; ++u) {          // every load issued before any use
+            const int i = e + u * kDriftThreads;
+            if (i < n_elem4) { b[u] = __ldcs(sb + base + i); a[u] = __ldcs(sa + base + i); }   // streamed once
+            else { b[u] = make_float4(0.f, 0.f, 0.f, 0.f); a[u] = b[u]; }
+        }
+#pragma unroll
+        for (int u = 0; u < kDriftUnroll; ++u) {
+            const float dx = a[u].x - b[u].x, dy = a[u].y - b[u].y, dz = a[u].z - b[u].z, dw = a[u].w - b[u].w;
+            num += dx * dx + dy * dy + dz * dz + dw * dw;
+            den += b[u].x * b[u].x + b[u].y * b[u].y + b[u].z * b[u].z + b[u].w * b[u].w;
+        }
     }
-    double dn = num, dd = den;
+    // a pairwise tree over the warp in float (the FP64 pipe is slow on this part), then the
+    // warps' sums added in double in warp order
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1) {
-        dn += __shfl_xor_sync(0xffffffffu, dn, m);
-        dd += __shfl_xor_sync(0xffffffffu, dd, m);
+        num += __shfl_xor_sync(0xffffffffu, num, m);
+        den += __shfl_xor_sync(0xffffffffu, den, m);
     }
+    const double dn = num, dd = den;
     __shared__ double red[2][kDriftThreads / 32];
     if ((threadIdx.x & 31) == 0) { red[0][threadIdx.x >> 5] = dn; red[1][threadIdx.x >> 5] = dd; }
     __syncthreads();

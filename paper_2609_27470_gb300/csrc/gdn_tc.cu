@@ -1459,8 +1459,11 @@ bool gdn_tc_supported(const GdnArgs& a) {
 }
 
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
-    const TcScratch sl = tc_scratch_layout(a.L, a.Hv, a.T);
-    const int grid = std::min(a.L * a.Hv, device_sm_count());
+    const TcScratch sl = tc_scratch_layout(a.L, a.Hv, a.T);   // hand-over space for device_sm_count() CTAs
+    // one chain CTA per SM that this context may use (a CTA waits at its end for its neighbour's
+    // hand-over, so the grid must not exceed what can be resident)
+    const int sms = context_sm_count();
+    const int grid = std::min(a.L * a.Hv, sms);
     CUtensorMap kmap, vmap, smap, hmap;
     if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
         !make_state_map(&smap, a.state, a.L * a.Hv) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
@@ -1473,7 +1476,6 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
         if (e != cudaSuccess) return e;
     }
     const int n_tiles = (a.T + kC - 1) / kC;
-    const int sms = device_sm_count();
     // factor kernel: one record per (layer, value head, tile), kWyCtasPerSm persistent CTAs per SM
     WyArgs w;
     w.L = a.L; w.Hk = a.Hk; w.Hv = a.Hv; w.T = a.T; w.n_tiles = n_tiles;

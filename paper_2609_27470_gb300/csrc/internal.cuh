@@ -151,6 +151,7 @@ cudaError_t launch_compact_kv_heads(const KvPlanes& kv, const int32_t* retain_id
 cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_new, const void* v_new,
                              int n_new, int chunk_id, int first_pos, cudaStream_t s);
 
-int device_sm_count();
+int device_sm_count();     // the device's SMs (cached per device)
+int context_sm_count();    // the SMs the current context may use (<= device_sm_count())
 
 }  // namespace deltas
