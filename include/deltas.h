@@ -132,6 +132,11 @@ DELTAS_API const char* deltas_status_string(int32_t status);
 /* Workspace: the status word plus, for d = 128 bf16 without read-out, the per-tile factors of  */
 /* the chunkwise form (16,656 bytes per layer, value head and 64-token tile), written and read   */
 /* within the call.                                                                             */
+/* Kernels: d = 128 bfloat16 without read-out runs on the tensor cores (a factor kernel and a   */
+/* state-chain kernel), or returns UNSUPPORTED when that path cannot be launched (no silent     */
+/* fallback).  Every other call, the read-out (out != NULL) included, runs token by token on    */
+/* the CUDA cores: the read-out's query tiles do not fit beside the state chain's buffers in    */
+/* one SM's shared memory.                                                                      */
 /* ------------------------------------------------------------------------------------------ */
 DELTAS_API size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens);
 
