@@ -358,13 +358,16 @@ class GdnOnlyWorkload:
         self.part = torch.zeros(cfg["L"], cfg["Hv"], 2, device=dev)
         self.scores = torch.zeros(cfg["n_chunks"], device=dev)
         self.ws = L.alloc_workspace(L.deltas_gdn_chunk_update_workspace_size(self.gdn, self.C), dev)
+        self.with_out = bool(cfg.get("with_out"))
+        self.out = (torch.empty(cfg["L"], self.C, cfg["Hv"], cfg["d"], dtype=torch.bfloat16, device=dev)
+                    if self.with_out else None)
         self.step_i = 0
 
     def step(self, timer):
         x = self.ring[self.step_i]
         with timer.mark("gdn_update"):
-            self.L.deltas_gdn_chunk_update(self.gdn, self.C, None, x["k"], x["v"], x["g"], x["beta"], self.state,
-                                           None, self.part, self.ws)
+            self.L.deltas_gdn_chunk_update(self.gdn, self.C, x["q"] if self.with_out else None, x["k"], x["v"],
+                                           x["g"], x["beta"], self.state, self.out, self.part, self.ws)
         with timer.mark("score"):
             self.L.deltas_score_chunks(self.cfg["L"], self.cfg["Hv"], self.part,
                                        self.step_i % self.cfg["n_chunks"], self.scores)
@@ -380,8 +383,8 @@ class GdnOnlyWorkload:
         if name != "gdn_update":
             return None
         cfg = self.cfg
-        by = algorithmic_gdn_bytes(cfg["L"], self.C, cfg["Hk"], cfg["Hv"], cfg["d"], 2, False)
-        fl = algorithmic_gdn_flops(cfg["L"], self.C, cfg["Hv"], cfg["d"], False)
+        by = algorithmic_gdn_bytes(cfg["L"], self.C, cfg["Hk"], cfg["Hv"], cfg["d"], 2, self.with_out)
+        fl = algorithmic_gdn_flops(cfg["L"], self.C, cfg["Hv"], cfg["d"], self.with_out)
         return {"bound": "hbm", "achieved": by / (avg_ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "bytes_per_launch": by, "tensor_frac": fl / (avg_ms * 1e-3) / 1e12 / peaks["bf16_tflops_sustained"]}
 
@@ -390,7 +393,7 @@ class GdnOnlyWorkload:
 
     def h2d_tensors(self, i=0):
         x = self.ring[i]
-        return [x["k"], x["v"], x["g"], x["beta"]]
+        return ([x["q"]] if self.with_out else []) + [x["k"], x["v"], x["g"], x["beta"]]
 
     def result_scalar(self):
         i = (self.step_i - 1) % self.cfg["n_chunks"]
@@ -606,6 +609,8 @@ def make_workload(name, dev, L):
         return GdnOnlyWorkload(dev, L, configs.STACK)
     if name == "layer":
         return GdnOnlyWorkload(dev, L, configs.LAYER)
+    if name == "layer_out":
+        return GdnOnlyWorkload(dev, L, configs.LAYER_OUT)
     if name == "kv":
         return KvWorkload(dev, L)
     if name == "drift":
@@ -729,7 +734,7 @@ def oracle_sample(workload: str, budget_s: float = 12.0, threads: int = 1):
         parts.append(f"drift of {n} (layer,head) state pairs x{factor:.0f} extrapolated; score of {cfg['L']} layers")
     head_signal = cfg.get("signal") in ("key_norm", "value_norm")
     if workload in ("streaming", "paper", "paper_write_norm", "paper_key_norm", "paper_value_norm", "stack",
-                    "layer"):
+                    "layer", "layer_out"):
         C = int(round(_tokens(workload)))
         heads_total = cfg["L"] * cfg["Hv"]
         n_heads = 2
@@ -742,6 +747,9 @@ def oracle_sample(workload: str, budget_s: float = 12.0, threads: int = 1):
                 oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0, want_write_norms=True)
             elif head_signal:                              # the state moves; no drift is formed
                 oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
+            elif cfg.get("with_out"):                      # with the layer output
+                S, _ = oracle.gdn_recurrence(f["q"], f["k"], f["v"], f["g"], f["beta"], s0, want_out=True)
+                oracle.drift_partials(s0, S)
             else:
                 S, _ = oracle.gdn_recurrence(None, f["k"], f["v"], f["g"], f["beta"], s0)
                 oracle.drift_partials(s0, S)
@@ -861,7 +869,7 @@ def config_line(workload):
     c = _cfg(workload)
     line = {"workload": workload, "l2": "flushed between timed steps (256 MiB write)",
             "inputs": "ring of 8 distinct per-chunk input sets, generated on device"}
-    for key in ("L", "Hk", "Hv", "d", "chunk_len", "chunk_lens", "Lf", "Hkv", "D", "budget_M", "n_sink",
+    for key in ("L", "Hk", "Hv", "d", "chunk_len", "chunk_lens", "with_out", "Lf", "Hkv", "D", "budget_M", "n_sink",
                 "n_window", "n_buckets", "signal"):
         if key in c:
             line[key] = c[key]
@@ -876,7 +884,7 @@ def config_line(workload):
 
 def _cfg(workload):
     return {"streaming": configs.STREAMING, "paper": configs.PAPER, "stack": configs.STACK,
-            "layer": configs.LAYER, "kv": configs.KV, "snapshot": configs.PAPER, "drift": configs.DRIFT,
+            "layer": configs.LAYER, "layer_out": configs.LAYER_OUT, "kv": configs.KV, "snapshot": configs.PAPER, "drift": configs.DRIFT,
             "paper_write_norm": configs.PAPER_WRITE_NORM, "paper_key_norm": configs.PAPER_KEY_NORM,
             "paper_value_norm": configs.PAPER_VALUE_NORM}[workload]
 
@@ -900,7 +908,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="streaming",
                     choices=["streaming", "paper", "paper_write_norm", "paper_key_norm", "paper_value_norm",
-                             "stack", "layer", "kv", "snapshot", "drift"])
+                             "stack", "layer", "layer_out", "kv", "snapshot", "drift"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)

@@ -24,6 +24,8 @@ TINY = dict(name="tiny", L=1, Hk=2, Hv=2, d=16, dtype="f32", chunk_len=64, n_chu
             Lf=1, Hkv=2, D=16, kv_dtype="f32", budget_M=256, zero_state=True)
 
 LAYER = dict(name="layer", L=1, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=1024, n_chunks=16)
+# the same with the layer output o_t = q_scale S_t q_t (Alg. 1 Prefill) asked for
+LAYER_OUT = dict(LAYER, name="layer_out", with_out=True)
 
 STACK = dict(name="stack", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=1024, n_chunks=256,
              ring=8)
