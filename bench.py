@@ -357,8 +357,10 @@ class GdnOnlyWorkload:
         self.state = inputs.initial_state(cfg["L"], cfg["Hv"], cfg["d"], 51, device=dev)
         self.part = torch.zeros(cfg["L"], cfg["Hv"], 2, device=dev)
         self.scores = torch.zeros(cfg["n_chunks"], device=dev)
-        self.ws = L.alloc_workspace(L.deltas_gdn_chunk_update_workspace_size(self.gdn, self.C), dev)
         self.with_out = bool(cfg.get("with_out"))
+        size = (L.deltas_gdn_chunk_update_readout_workspace_size if self.with_out else
+                L.deltas_gdn_chunk_update_workspace_size)(self.gdn, self.C)
+        self.ws = L.alloc_workspace(size, dev)
         self.out = (torch.empty(cfg["L"], self.C, cfg["Hv"], cfg["d"], dtype=torch.bfloat16, device=dev)
                     if self.with_out else None)
         self.step_i = 0
@@ -374,7 +376,7 @@ class GdnOnlyWorkload:
         self.step_i += 1
 
     def launches_per_step(self):
-        return 2 + 1                                            # factor + chain kernels, score
+        return 2 + (1 if self.with_out else 0) + 1              # factor + chain (+ read-out) kernels, score
 
     def tokens_per_step(self):
         return self.C

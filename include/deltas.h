@@ -129,16 +129,22 @@ DELTAS_API const char* deltas_status_string(int32_t status);
 /* n_tokens = 0 leaves the state unchanged (partials then hold 0 and ||S_before||^2).          */
 /* Errors: INVALID_ARGUMENT for NULL/misaligned pointers, negative sizes or Hv % Hk != 0;      */
 /* UNSUPPORTED for d_k != d_v or d_k outside {16,32,64,128}; WORKSPACE for a short workspace. */
-/* Workspace: the status word plus, for d = 128 bf16 without read-out, the per-tile factors of  */
-/* the chunkwise form (16,656 bytes per layer, value head and 64-token tile), written and read   */
-/* within the call.                                                                             */
-/* Kernels: d = 128 bfloat16 without read-out runs on the tensor cores (a factor kernel and a   */
-/* state-chain kernel), or returns UNSUPPORTED when that path cannot be launched (no silent     */
-/* fallback).  Every other call, the read-out (out != NULL) included, runs token by token on    */
-/* the CUDA cores: the read-out's query tiles do not fit beside the state chain's buffers in    */
-/* one SM's shared memory.                                                                      */
+/* Workspace: the status word plus, for d = 128 bf16, the per-tile factors of the chunkwise     */
+/* form (16,656 bytes per layer, value head and 64-token tile; 16,912 with the read-out),       */
+/* written and read within the call.  A call with out != NULL needs                            */
+/* deltas_gdn_chunk_update_readout_workspace_size bytes: for d = 128 bf16 that adds each       */
+/* token's write u_t (512 bytes per token and value head) and the state at the start of every  */
+/* 128-token block (64 KiB per block and value head); a shorter workspace returns WORKSPACE.   */
+/* Kernels: d = 128 bfloat16 runs on the tensor cores (a factor kernel, a state-chain kernel   */
+/* and, with out != NULL, a read-out kernel that forms each 128-token block's outputs from the */
+/* block's starting state and writes), or returns UNSUPPORTED when that path cannot be         */
+/* launched (no silent fallback).  Every other shape runs token by token on the CUDA cores.    */
 /* ------------------------------------------------------------------------------------------ */
 DELTAS_API size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens);
+
+/* Workspace bytes for a deltas_gdn_chunk_update(_write_norms) call that passes out != NULL    */
+/* (>= deltas_gdn_chunk_update_workspace_size; equal to it except for d = 128 bfloat16).      */
+DELTAS_API size_t deltas_gdn_chunk_update_readout_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens);
 
 DELTAS_API deltas_status deltas_gdn_chunk_update(const deltas_gdn_desc* desc, int32_t n_tokens,
                                       const void* q, const void* k, const void* v,

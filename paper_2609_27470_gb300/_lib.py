@@ -32,7 +32,8 @@ DELTAS_BF16 = 1
 
 EXPORTED = (
     "deltas_version", "deltas_status_string",
-    "deltas_gdn_chunk_update_workspace_size", "deltas_gdn_chunk_update",
+    "deltas_gdn_chunk_update_workspace_size", "deltas_gdn_chunk_update_readout_workspace_size",
+    "deltas_gdn_chunk_update",
     "deltas_state_drift_workspace_size", "deltas_state_drift",
     "deltas_score_chunks", "deltas_gdn_chunk_update_write_norms", "deltas_score_write_norms",
     "deltas_select_retain_workspace_size", "deltas_select_retain", "deltas_select_retain_static",
@@ -81,6 +82,7 @@ def _sig(name, res, *args):
 _sig("deltas_version", ctypes.c_char_p)
 _sig("deltas_status_string", ctypes.c_char_p, _I32)
 _sig("deltas_gdn_chunk_update_workspace_size", _SZ, _P, _I32)
+_sig("deltas_gdn_chunk_update_readout_workspace_size", _SZ, _P, _I32)
 _sig("deltas_gdn_chunk_update", ctypes.c_int, _P, _I32, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P)
 _sig("deltas_state_drift_workspace_size", _SZ, _P)
 _sig("deltas_state_drift", ctypes.c_int, _P, _P, _P, _P, _P, _SZ, _P)
@@ -171,6 +173,10 @@ def alloc_workspace(nbytes: int, device=None) -> torch.Tensor:
 
 def deltas_gdn_chunk_update_workspace_size(desc: GdnDesc, n_tokens: int) -> int:
     return int(_lib.deltas_gdn_chunk_update_workspace_size(ctypes.byref(desc), int(n_tokens)))
+
+
+def deltas_gdn_chunk_update_readout_workspace_size(desc: GdnDesc, n_tokens: int) -> int:
+    return int(_lib.deltas_gdn_chunk_update_readout_workspace_size(ctypes.byref(desc), int(n_tokens)))
 
 
 def deltas_gdn_chunk_update(desc: GdnDesc, n_tokens: int, q, k, v, g, beta, state, out, drift_partials,

@@ -129,7 +129,13 @@ const char* deltas_status_string(int32_t s) {
 size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens) {
     if (desc == nullptr || n_tokens <= 0) return kStatusBytes;
     return kStatusBytes + gdn_tc_scratch_bytes(desc->num_layers, desc->num_v_heads, desc->key_dim,
-                                               desc->value_dim, desc->dtype, n_tokens);
+                                               desc->value_dim, desc->dtype, n_tokens, false);
+}
+
+size_t deltas_gdn_chunk_update_readout_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens) {
+    if (desc == nullptr || n_tokens <= 0) return kStatusBytes;
+    return kStatusBytes + gdn_tc_scratch_bytes(desc->num_layers, desc->num_v_heads, desc->key_dim,
+                                               desc->value_dim, desc->dtype, n_tokens, true);
 }
 
 namespace {
@@ -149,7 +155,9 @@ deltas_status gdn_update(const deltas_gdn_desc* desc, int32_t n_tokens, const vo
     }
     if (drift_partials && !aligned16(drift_partials)) return DELTAS_ERR_INVALID_ARGUMENT;
     if (write_norms && !aligned16(write_norms)) return DELTAS_ERR_INVALID_ARGUMENT;
-    st = check_workspace(workspace, workspace_bytes, deltas_gdn_chunk_update_workspace_size(desc, n_tokens));
+    st = check_workspace(workspace, workspace_bytes,
+                         out ? deltas_gdn_chunk_update_readout_workspace_size(desc, n_tokens)
+                             : deltas_gdn_chunk_update_workspace_size(desc, n_tokens));
     if (st != DELTAS_OK) return st;
     GdnArgs a;
     a.L = desc->num_layers; a.Hk = desc->num_k_heads; a.Hv = desc->num_v_heads;
@@ -159,7 +167,7 @@ deltas_status gdn_update(const deltas_gdn_desc* desc, int32_t n_tokens, const vo
     a.status = static_cast<int32_t*>(workspace);
     a.scratch = static_cast<uint8_t*>(workspace) + kStatusBytes;
     a.scratch_bytes = workspace_bytes - kStatusBytes;
-    // d = 128 bfloat16 without read-out runs on the tensor cores or not at all: no silent fallback
+    // d = 128 bfloat16 runs on the tensor cores or not at all: no silent fallback
     if (gdn_tc_shape(a)) {
         if (!gdn_tc_supported(a)) return DELTAS_ERR_UNSUPPORTED;
         return from_cuda(launch_gdn_update_tc(a, as_stream(stream)));

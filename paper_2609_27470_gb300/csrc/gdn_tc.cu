@@ -87,10 +87,15 @@ constexpr float kSigMin = 9.313225746154785e-10f;   // 2^-30: smallest deferred 
 //   [0, 8192)       T~ hi: bfloat16 [64 t][64 i], 128-byte rows, 128-byte swizzle (K-major B operand)
 //   [8192, 16384)   T~ lo, same layout
 //   [16384, 16656)  float: -gamma[64], gamma_C, 3 unused
+// With the read-out the record holds T itself (no row decay) and, after the constants above,
+//   [16656, 16912)  float: exp(G_C - G_t)[64], the row decays, applied by the update kernel
+// so that the update kernel sees each token's write u_t undecayed.
 constexpr uint32_t kRecT = 16384;
 constexpr uint32_t kRecConsts = 68;
 constexpr uint32_t kRecBytes = kRecT + kRecConsts * 4;
-static_assert(kRecBytes % 16 == 0, "records are bulk-copied: 16-byte multiples");
+constexpr uint32_t kRecBytesOut = kRecBytes + kC * 4;
+static_assert(kRecBytes % 16 == 0 && kRecBytesOut % 16 == 0, "records are bulk-copied: 16-byte multiples");
+__host__ __device__ constexpr uint32_t rec_bytes(bool out) { return out ? kRecBytesOut : kRecBytes; }
 
 // Barrier over `n` threads that also returns the OR of `flag` over them (uniform result).
 __device__ __forceinline__ bool named_sync_or(int id, int n, bool flag) {
@@ -251,9 +256,10 @@ static_assert(kWyCtasPerSm * (kWySmemAlloc + 1024) <= 233472, "factor kernel: CT
 
 struct WyArgs {
     int L, Hk, Hv, T, n_tiles;
+    int out;                   // records for the read-out: T and the row decays (see the record)
     const float* g;
     const float* beta;
-    uint8_t* rec;              // [L * Hv][n_tiles] records of kRecBytes
+    uint8_t* rec;              // [L * Hv][n_tiles] records of rec_bytes(out)
     int32_t* status;
     int32_t* ho_flags;         // the update kernel's hand-over flags, reset here for this call
     int n_ho_flags;
@@ -348,9 +354,10 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         }
         const float G0 = incl - pg[1], G1 = incl;
         const float GC = __shfl_sync(0xffffffffu, incl, 31);
-        float* rc = reinterpret_cast<float*>(a.rec + (size_t)rec_of(it) * kRecBytes + kRecT);
+        float* rc = reinterpret_cast<float*>(a.rec + (size_t)rec_of(it) * rec_bytes(a.out) + kRecT);
         *reinterpret_cast<float2*>(rc + 2 * lane) = make_float2(-expf(G0), -expf(G1));
         if (lane == 0) *reinterpret_cast<float4*>(rc + 64) = make_float4(expf(GC), 0.f, 0.f, 0.f);
+        if (a.out) *reinterpret_cast<float2*>(rc + kRecConsts + 2 * lane) = make_float2(expf(GC - G0), expf(GC - G1));
         const float g20 = G0 * kLog2e, g21 = G1 * kLog2e;
         float lo2 = fminf(g20, g21), hi2 = fmaxf(g20, g21);
 #pragma unroll
@@ -575,16 +582,16 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
         }
         __syncthreads();
         // T~ = diag(exp(G_C - G)) X diag(beta) (upper part zero), split into the record's (hi, lo)
-        // images
+        // images; for the read-out T = X diag(beta)
         {
-            uint8_t* rec = a.rec + (size_t)rec_of(it) * kRecBytes;
+            uint8_t* rec = a.rec + (size_t)rec_of(it) * rec_bytes(a.out);
 #pragma unroll
             for (int m = 0; m < 2; ++m) {
                 const int e = tid + kWyThreads * m;
                 const int t = e >> 3, c8 = e & 7;
                 uint4 vh = make_uint4(0u, 0u, 0u, 0u), vl = vh;
                 if (8 * c8 <= t) {                     // chunks right of the diagonal stay zero
-                    const float dt = sDel[t];
+                    const float dt = a.out ? 1.f : sDel[t];
                     const float4 x0 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8);
                     const float4 x1 = *reinterpret_cast<const float4*>(fX + t * FX_S + 8 * c8 + 4);
                     const float4 b0 = *reinterpret_cast<const float4*>(sBeta + 8 * c8);
@@ -652,7 +659,7 @@ constexpr uint32_t SM_I = SM_R + 2 * kRecSlot;   // 8 KB: 64 x 64 bfloat16 ident
 constexpr uint32_t SM_SB = SM_I + 8192;          // 64 KB: state staging, 4 column blocks x 128 rows x 128 B, SW128
 constexpr uint32_t SM_BYTES = SM_SB + 65536;
 constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
-static_assert(SM_I % 1024 == 0 && SM_SB % 1024 == 0 && kRecSlot >= kRecBytes, "shared-memory map");
+static_assert(SM_I % 1024 == 0 && SM_SB % 1024 == 0 && kRecSlot >= kRecBytesOut, "shared-memory map");
 static_assert(kSmemAlloc <= 232448, "shared memory budget");
 
 // The staging buffer holds a head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each
@@ -676,6 +683,10 @@ struct TcArgs {
     int32_t* ho_flag;        // [grid] the state after the first part is in the hand-over map
     int32_t* ho_wflag;       // [grid] the first part's write-size sum is in ho_wsum
     float* ho_wsum;          // [grid]
+    // read-out: each token's write u_t, and the state at the start of every 128-token block
+    float* ubuf;             // [L * Hv][d_v][Tp] fp32: u_t (token-contiguous rows)
+    float* snap;             // [L * Hv][n_blk][d_v][d_k] fp32
+    int Tp, n_blk;           // Tp = 64 n_tiles, n_blk = ceil(n_tiles / 2)
 };
 
 // The CTA's work: a sequence of slots, each a run of consecutive tiles of one head.  By default
@@ -743,6 +754,7 @@ struct TileCursor {
     }
 };
 
+template <bool kOut>
 __global__ void __launch_bounds__(kThreads, 1)
 gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap hmap,
@@ -946,9 +958,9 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             vp[b2] = J;
             if (J >= 2 && !warp_wait(&mb_re[b2], ((J >> 1) - 1) & 1, kWaitBudgetNs, abort_flag)) { fail(a.status, abort_flag, 32); break; }
             if (elect_one()) {
-                mbar_arrive_expect_tx(&mb_tr[b2], kRecBytes);
-                bulk_load_tx(sm + SM_R + b2 * kRecSlot, a.rec + ((size_t)cc.lh * n + cc.jt) * kRecBytes,
-                             kRecBytes, &mb_tr[b2]);
+                constexpr uint32_t RB = rec_bytes(kOut);
+                mbar_arrive_expect_tx(&mb_tr[b2], RB);
+                bulk_load_tx(sm + SM_R + b2 * kRecSlot, a.rec + ((size_t)cc.lh * n + cc.jt) * RB, RB, &mb_tr[b2]);
             }
             __syncwarp();
             rp[b2] = J;
@@ -1181,6 +1193,17 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             // scaled by u_scale, (hi, lo) in place over this thread's 16 X columns (tokens 16 cgp ..)
             if (!mbar_wait_or_abort(&mb_x, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 10);
             tc_fence_after();
+            // read-out: the row decays of the thread's 16 tokens, taken now (the record's slot is
+            // released to the next load once MMA_U(j) completes, before the U~ pass)
+            float dl[kOut ? 16 : 1];
+            if constexpr (kOut) {
+                const float* src = rec_consts(j) + kRecConsts + 16 * cgp;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float4 d4 = *reinterpret_cast<const float4*>(src + 4 * e);
+                    dl[4 * e] = d4.x; dl[4 * e + 1] = d4.y; dl[4 * e + 2] = d4.z; dl[4 * e + 3] = d4.w;
+                }
+            }
             {
                 float xv[16], vv[16], cf[16];
                 tmem_ld16(tm + lane_off + TM_X + 16 * cgp, xv);
@@ -1205,16 +1228,28 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             warp_arrive(&mb_xready, lane);
 
             // ---- while MMA_U runs: rescale S~ if the decay would underflow the deferred scale
-            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K(j+1) in fp32
-            if (rescale) {
-                const float f = gC * sig;
+            // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K(j+1) in fp32.  For the
+            // read-out, a tile that starts a 128-token block also writes the state before it,
+            // sig S~ (row r, columns 32 cgp ..).
+            const bool snap = kOut && (jt & 1) == 0;       // uniform over the CTA
+            if (rescale || snap) {
                 float sv[32];
                 tmem_ld32(tm + lane_off + TM_S + 32 * cgp, sv);
                 tmem_ld_wait();
+                if (snap) {
+                    float* dst = a.snap + (((size_t)lh * a.n_blk + (jt >> 1)) * kD + r) * kD + 32 * cgp;
 #pragma unroll
-                for (int e = 0; e < 32; ++e) sv[e] *= f;
-                tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
-                tmem_st_wait();
+                    for (int e = 0; e < 8; ++e)
+                        *reinterpret_cast<float4*>(dst + 4 * e) =
+                            make_float4(sv[4 * e] * sig, sv[4 * e + 1] * sig, sv[4 * e + 2] * sig, sv[4 * e + 3] * sig);
+                }
+                if (rescale) {
+                    const float f = gC * sig;
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) sv[e] *= f;
+                    tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
+                    tmem_st_wait();
+                }
             }
             sig = rescale ? 1.f : gC * sig;                // the deferred decay after tile j
             if (j + 1 < NJ && !make_k32(j + 1)) fail(a.status, abort_flag, 16);
@@ -1226,6 +1261,15 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 float uv[16];
                 tmem_ld16(tm + lane_off + TM_U + 16 * cgp, uv);
                 tmem_ld_wait();
+                if constexpr (kOut) {
+                    // with the record's undecayed T the column is u_t u_scale = u_t / sig: u_t out
+                    // for the read-out (tokens jt 64 + 16 cgp .. of row r)
+                    float* dst = a.ubuf + ((size_t)lh * kD + r) * a.Tp + jt * kC + 16 * cgp;
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        *reinterpret_cast<float4*>(dst + 4 * e) =
+                            make_float4(uv[4 * e] * sig, uv[4 * e + 1] * sig, uv[4 * e + 2] * sig, uv[4 * e + 3] * sig);
+                }
                 if (want_w) {
                     // squares summed over the warp's 32 rows, column by column: halving exchanges
                     // leave lanes 2c and 2c + 1 with column c (token 16 cgp + c) of the 16
@@ -1246,9 +1290,19 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     // the deferred decay; then it is gamma_C, and below 2^-60 the columns of the
                     // early tokens, scaled by gamma_C / gamma_t, are no longer representable: such
                     // a tile contributes nothing
-                    const float sc = u_scale * gC;
-                    const float wf = sc >= 0x1p-60f ? w_gamma / sc : 0.f;
+                    float wf;
+                    if constexpr (kOut) {
+                        wf = sig;                          // the column is u_t / sig
+                    } else {
+                        const float sc = u_scale * gC;
+                        wf = sc >= 0x1p-60f ? w_gamma / sc : 0.f;
+                    }
                     if ((lane & 1) == 0) atomicAdd(&s_u2[j & 1][16 * cgp + (lane >> 1)], x[0] * wf * wf);
+                }
+                if constexpr (kOut) {
+                    // the row decay exp(G_C - G_t) that T~ carries on the path without read-out
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) uv[e] *= dl[e];
                 }
                 uint32_t hi[8], lo[8];
 #pragma unroll
@@ -1375,6 +1429,276 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
     }
 }
 
+// =============================================================================================
+// Read-out kernel: o_t = q_scale S_t q_t for every token of the chunk
+// =============================================================================================
+// Unrolling Eq. 1 from the state S_b before a block of 128 tokens, with G the inclusive cumulative
+// log-decay inside the block and u_i = beta_i (v_i - alpha_i S_{i-1} k_i) the write of token i,
+//   S_t = exp(G_t) S_b + sum_{i <= t} exp(G_t - G_i) u_i k_i^T,
+// so the block's outputs are, at once,
+//   O = (P o D) U + diag(exp(G)) Q S_b^T,    P = Q K^T,   D[t][i] = exp(G_t - G_i) for i <= t, else 0,
+// with U the rows u_i.  The update kernel leaves u_i and S_b in the workspace; this kernel takes one
+// (layer, value head, block) item at a time: P by a bfloat16 MMA (exact inputs) into TMEM, P o D
+// (in place) and diag(exp(G)) Q formed in fp32 in TMEM as the A operands of two kind::tf32 MMAs
+// that accumulate O, then O q_scale to the output.  Items run one after another on a persistent CTA
+// per SM; the next item's Q and K load while O is formed, its U and S_b during the store.
+// Warp w serves TMEM lanes 32 (w % 4) .. + 31 (the block's tokens) and column half w / 4.
+constexpr int kRoThreads = 256;
+constexpr int kRoBlk = 128;                            // tokens per item (two update tiles)
+constexpr uint32_t kRoTmemCols = 512;
+constexpr uint32_t RT_P = 0, RT_Q = 128, RT_O = 256;  // TMEM: P (then P o D), diag(exp(G)) Q, O
+// shared-memory map (bytes from a 1024-aligned base)
+constexpr uint32_t RO_Q = 0;        // 32 KB: Q, 2 column blocks (d 0-63, 64-127) x 128 rows x 128 B, SW128
+constexpr uint32_t RO_K = 32768;    // 32 KB: K, same layout
+constexpr uint32_t RO_U = 65536;    // 64 KB: U^T [d_v][128 tokens] fp32, 4 column blocks x 128 rows x 128 B
+constexpr uint32_t RO_S = 131072;   // 64 KB: S_b [d_v][d_k] fp32, same layout
+constexpr uint32_t kRoSmemAlloc = 196608 + 1024;
+
+struct RoArgs {
+    int L, Hk, Hv, T, n_blk;
+    float q_scale;
+    const float* g;
+    __nv_bfloat16* out;
+    int32_t* status;
+};
+
+__global__ void __launch_bounds__(kRoThreads, 1)
+gdn_readout_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                   const __grid_constant__ CUtensorMap umap, const __grid_constant__ CUtensorMap bmap,
+                   RoArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    __shared__ uint64_t mb_qk, mb_us, mb_p, mb_o;
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_abort;
+    __shared__ __align__(16) float s_g2[kRoBlk];      // G log2(e) of the item's tokens
+    volatile int* abort_flag = &s_abort;
+    grid_dep_launch();
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int items = a.L * a.Hv * a.n_blk;            // item = (layer * Hv + head) * n_blk + block
+    if (warp == 0) { tmem_alloc(&s_tmem, kRoTmemCols); tmem_relinquish(); }
+    if (tid == 32) {
+        mbar_init(&mb_qk, 1); mbar_init(&mb_us, 1); mbar_init(&mb_p, 1); mbar_init(&mb_o, 1);
+        fence_barrier_init();
+        prefetch_tensormap(&qmap); prefetch_tensormap(&kmap);
+        prefetch_tensormap(&umap); prefetch_tensormap(&bmap);
+        s_abort = 0;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = s_tmem;
+
+    auto load_qk = [&](int it) {                       // thread 0: the item's Q and K blocks
+        const int lh = it / a.n_blk, b = it - lh * a.n_blk, l = lh / a.Hv, h = lh - l * a.Hv;
+        const int kh = (int)(((long long)h * a.Hk) / a.Hv);
+        mbar_arrive_expect_tx(&mb_qk, 4 * 16384);
+#pragma unroll
+        for (int th = 0; th < 2; ++th) {
+#pragma unroll
+            for (int cb = 0; cb < 2; ++cb) {
+                const uint32_t off = cb * 16384 + th * 8192;
+                tma_load_4d(sm + RO_Q + off, &qmap, &mb_qk, 64 * cb, kh, b * kRoBlk + 64 * th, l);
+                tma_load_4d(sm + RO_K + off, &kmap, &mb_qk, 64 * cb, kh, b * kRoBlk + 64 * th, l);
+            }
+        }
+    };
+    auto load_us = [&](int it) {                       // thread 0: the item's U^T and S_b
+        const int lh = it / a.n_blk, b = it - lh * a.n_blk;
+        mbar_arrive_expect_tx(&mb_us, 8 * 16384);
+#pragma unroll
+        for (int cb = 0; cb < 4; ++cb) {
+            tma_load_2d(sm + RO_U + cb * 16384, &umap, &mb_us, b * kRoBlk + 32 * cb, lh * kD);
+            tma_load_2d(sm + RO_S + cb * 16384, &bmap, &mb_us, 32 * cb, (lh * a.n_blk + b) * kD);
+        }
+    };
+    int n_qk = 0, n_us = 0, n_p = 0, n_o = 0;          // copies / MMA groups issued (thread 0 / warp 0)
+    const int first = (int)blockIdx.x, G = (int)gridDim.x;
+    // q, k and g are inputs of the call; U and S_b are written by the update kernel, which the
+    // wait covers
+    if (tid == 0 && first < items) { load_qk(first); ++n_qk; }
+    grid_dep_wait();
+    if (tid == 0 && first < items) { load_us(first); ++n_us; }
+
+    const int q4 = warp & 3, hc = warp >> 2;
+    const int t = 32 * q4 + lane;                      // the thread's token row of the block
+    const uint32_t lane_off = (uint32_t)(32 * q4) << 16;
+    int c = 0;
+    for (int it = first; it < items; it += G, ++c) {
+        const int lh = it / a.n_blk, b = it - lh * a.n_blk, l = lh / a.Hv, h = lh - l * a.Hv;
+        const int nxt = it + G;
+        if (warp == 4) {
+            // inclusive cumulative log-decay of the block's tokens, four per lane (past T: g = 0)
+            float gv[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int tok = b * kRoBlk + 4 * lane + e;
+                gv[e] = tok < a.T ? a.g[((size_t)l * a.T + tok) * a.Hv + h] : 0.f;
+            }
+            gv[1] += gv[0]; gv[2] += gv[1]; gv[3] += gv[2];
+            float incl = gv[3];
+#pragma unroll
+            for (int m = 1; m < 32; m <<= 1) {
+                const float y = __shfl_up_sync(0xffffffffu, incl, m);
+                if (lane >= m) incl += y;
+            }
+            const float base = incl - gv[3];
+            *reinterpret_cast<float4*>(s_g2 + 4 * lane) =
+                make_float4((base + gv[0]) * kLog2e, (base + gv[1]) * kLog2e, (base + gv[2]) * kLog2e,
+                            (base + gv[3]) * kLog2e);
+        }
+        if (warp == 0) {                               // P = Q K^T
+            uint64_t aq[2][4], bk[2][4];
+#pragma unroll
+            for (int s = 0; s < 8; ++s) {
+                const uint32_t off = (s >> 2) * 16384 + (s & 3) * 32;
+                aq[s >> 2][s & 3] = sdesc_sw128(smem_u32(sm + RO_Q + off), 16, 1024);
+                bk[s >> 2][s & 3] = sdesc_sw128(smem_u32(sm + RO_K + off), 16, 1024);
+            }
+            if (warp_wait(&mb_qk, c & 1, kWaitBudgetNs, abort_flag)) {
+                tc_fence_after();
+                if (elect_one()) {
+                    mma4_bf16_ss_1t(tm + RT_P, aq[0], bk[0], idesc_bf16(128, 128, 0, 0), 0);
+                    mma4_bf16_ss_1t(tm + RT_P, aq[1], bk[1], idesc_bf16(128, 128, 0, 0), 1);
+                }
+                __syncwarp();
+                mma_commit(&mb_p);
+                ++n_p;
+            } else if (lane == 0) {
+                fail(a.status, abort_flag, 60);
+            }
+        }
+        bool ok = mbar_wait_or_abort(&mb_p, c & 1, kWaitBudgetNs, abort_flag);
+        if (!ok && !*abort_flag) fail(a.status, abort_flag, 61);
+        if (__syncthreads_or(!ok)) break;              // (also publishes s_g2)
+        tc_fence_after();
+        {
+            // P o D in place: columns 64 hc .. + 63 of row t; a 16-column group right of every
+            // row of the warp is all zero
+            const float g2t = s_g2[t];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int c0 = 64 * hc + 16 * k;
+                uint32_t o[16];
+                if (c0 <= 32 * q4 + 31) {              // uniform over the warp
+                    float p[16];
+                    tmem_ld16(tm + lane_off + RT_P + c0, p);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e4 = 0; e4 < 4; ++e4) {
+                        const float4 gi = *reinterpret_cast<const float4*>(s_g2 + c0 + 4 * e4);
+                        const float gg[4] = {gi.x, gi.y, gi.z, gi.w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int i = c0 + 4 * e4 + e;
+                            o[4 * e4 + e] = __float_as_uint(i <= t ? p[4 * e4 + e] * fast_exp2(g2t - gg[e]) : 0.f);
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) o[e] = 0u;
+                }
+                tmem_st16(tm + lane_off + RT_P + c0, o);
+            }
+            // diag(exp(G)) Q: dims 64 hc .. + 63 of row t, from the swizzled bfloat16 block
+            const float gam = fast_exp2(g2t);
+            const uint8_t* qb = sm + RO_Q + hc * 16384;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                uint32_t o[16];
+#pragma unroll
+                for (int h2 = 0; h2 < 2; ++h2) {
+                    const uint4 w = *reinterpret_cast<const uint4*>(qb + sw128_offset(t, 2 * k + h2));
+                    const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        o[8 * h2 + 2 * i] = __float_as_uint(__uint_as_float(wv[i] << 16) * gam);
+                        o[8 * h2 + 2 * i + 1] = __float_as_uint(__uint_as_float(wv[i] & 0xFFFF0000u) * gam);
+                    }
+                }
+                tmem_st16(tm + lane_off + RT_Q + 64 * hc + 16 * k, o);
+            }
+            tmem_st_wait();
+        }
+        fence_async_smem();                            // Q's generic reads before the next TMA write
+        tc_fence_before();
+        __syncthreads();
+        // Q and K have been read (P is complete, diag(exp(G)) Q formed): the next item's blocks
+        if (tid == 0 && nxt < items) { load_qk(nxt); ++n_qk; }
+        if (warp == 0) {                               // O = (P o D) U + (diag(exp(G)) Q) S_b^T
+            uint32_t ap[4][4], aq[4][4];
+            uint64_t bu[4][4], bs[4][4];
+#pragma unroll
+            for (int s = 0; s < 16; ++s) {
+                const uint32_t off = (s >> 2) * 16384 + (s & 3) * 32;
+                ap[s >> 2][s & 3] = tm + RT_P + 8 * s;
+                aq[s >> 2][s & 3] = tm + RT_Q + 8 * s;
+                bu[s >> 2][s & 3] = sdesc_sw128(smem_u32(sm + RO_U + off), 16, 1024);
+                bs[s >> 2][s & 3] = sdesc_sw128(smem_u32(sm + RO_S + off), 16, 1024);
+            }
+            if (warp_wait(&mb_us, c & 1, kWaitBudgetNs, abort_flag)) {
+                tc_fence_after();
+                if (elect_one()) {
+#pragma unroll
+                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + RT_O, ap[g4], bu[g4], idesc_tf32(128, 128), g4 != 0);
+#pragma unroll
+                    for (int g4 = 0; g4 < 4; ++g4) mma4_tf32_ta_1t(tm + RT_O, aq[g4], bs[g4], idesc_tf32(128, 128), 1);
+                }
+                __syncwarp();
+                mma_commit(&mb_o);
+                ++n_o;
+            } else if (lane == 0) {
+                fail(a.status, abort_flag, 62);
+            }
+        }
+        ok = mbar_wait_or_abort(&mb_o, c & 1, kWaitBudgetNs, abort_flag);
+        if (!ok && !*abort_flag) fail(a.status, abort_flag, 63);
+        if (__syncthreads_or(!ok)) break;
+        tc_fence_after();
+        // U and S_b have been read: the next item's
+        if (tid == 0 && nxt < items) { load_us(nxt); ++n_us; }
+        {   // O q_scale -> bfloat16, dims 64 hc .. + 63 of the token's output row
+            const int tok = b * kRoBlk + t;
+            __nv_bfloat16* dst = a.out + (((size_t)l * a.T + tok) * a.Hv + h) * kD + 64 * hc;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                float o[16];
+                tmem_ld16(tm + lane_off + RT_O + 64 * hc + 16 * k, o);
+                tmem_ld_wait();
+                if (tok < a.T) {
+                    uint32_t w[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) w[i] = pack_bf16x2(o[2 * i] * a.q_scale, o[2 * i + 1] * a.q_scale);
+                    uint4* d4 = reinterpret_cast<uint4*>(dst + 16 * k);
+                    d4[0] = make_uint4(w[0], w[1], w[2], w[3]);
+                    d4[1] = make_uint4(w[4], w[5], w[6], w[7]);
+                }
+            }
+        }
+        tc_fence_before();
+        __syncthreads();                               // O has been read
+    }
+    if (*abort_flag) {
+        // after a failure: what this CTA issued lands before TMEM is freed and the CTA ends (at
+        // most one phase of each barrier is outstanding)
+        if (tid == 0) {
+            if (n_qk > 0) mbar_wait(&mb_qk, (n_qk - 1) & 1, kWaitBudgetNs);
+            if (n_us > 0) mbar_wait(&mb_us, (n_us - 1) & 1, kWaitBudgetNs);
+        }
+        if (warp == 0 && lane == 0) {
+            if (n_p > 0) mbar_wait(&mb_p, (n_p - 1) & 1, kWaitBudgetNs);
+            if (n_o > 0) mbar_wait(&mb_o, (n_o - 1) & 1, kWaitBudgetNs);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tm, kRoTmemCols);
+    }
+}
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -1407,13 +1731,13 @@ bool make_map(CUtensorMap* map, const void* base, int L, int T, int H) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// The state [L * Hv * 128][128] fp32 as a 2-D map: a box of 32 columns x 128 rows (one column block
-// of one head), 128-byte swizzle.
-bool make_state_map(CUtensorMap* map, void* base, int heads) {
+// fp32 rows [rows][cols] as a 2-D map: a box of 32 columns x 128 rows, 128-byte swizzle; columns
+// past `cols` read as zero.
+bool make_rows_map(CUtensorMap* map, void* base, long long rows, int cols) {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return false;
-    cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)heads * kD};
-    cuuint64_t strides[1] = {(cuuint64_t)kD * 4};
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)cols * 4};
     cuuint32_t box[2] = {32, (cuuint32_t)kD};
     cuuint32_t es[2] = {1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, es,
@@ -1421,68 +1745,95 @@ bool make_state_map(CUtensorMap* map, void* base, int heads) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The state [heads * 128][128] fp32: a box is one column block of one head.
+bool make_state_map(CUtensorMap* map, void* base, long long heads) {
+    return make_rows_map(map, base, heads * kD, kD);
+}
+
 // Scratch: the WY records, then the update kernel's hand-over area for up to one CTA per SM:
-// states [grid][128][128] fp32 (1024-aligned), flags [2][grid] int32, write-size sums [grid].
+// states [grid][128][128] fp32 (1024-aligned), flags [2][grid] int32, write-size sums [grid];
+// with the read-out, then each token's write u_t [L * Hv][128][64 n_tiles] fp32 and the state at
+// the start of every 128-token block [L * Hv][n_blk][128][128] fp32 (both 1024-aligned).
 struct TcScratch {
-    size_t rec, ho_state, ho_flags, ho_wsum, total;
+    size_t rec, ho_state, ho_flags, ho_wsum, ubuf, snap, total;
 };
 
-TcScratch tc_scratch_layout(int L, int Hv, int T) {
+size_t align1k(size_t x) { return (x + 1023) & ~size_t(1023); }
+
+TcScratch tc_scratch_layout(int L, int Hv, int T, bool out) {
     const int grid = std::max(1, std::min(L * Hv, device_sm_count()));
+    const size_t n_tiles = (size_t)(T + kC - 1) / kC, n_blk = (n_tiles + 1) / 2, heads = (size_t)L * Hv;
     TcScratch l;
     l.rec = 0;
-    l.ho_state = ((size_t)L * Hv * ((T + kC - 1) / kC) * kRecBytes + 1023) & ~size_t(1023);
+    l.ho_state = align1k(heads * n_tiles * rec_bytes(out));
     l.ho_flags = l.ho_state + (size_t)grid * kD * kD * 4;
     l.ho_wsum = l.ho_flags + 2 * (size_t)grid * 4;
     l.total = l.ho_wsum + (size_t)grid * 4;
+    l.ubuf = l.snap = 0;
+    if (out) {
+        l.ubuf = align1k(l.total);
+        l.snap = align1k(l.ubuf + heads * kD * n_tiles * kC * 4);
+        l.total = l.snap + heads * n_blk * kD * kD * 4;
+    }
     return l;
 }
 
 }  // namespace
 
-size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T) {
+size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T, bool out) {
     if (dk != kD || dv != kD || dtype != DELTAS_BF16 || L <= 0 || Hv <= 0 || T <= 0) return 0;
-    return tc_scratch_layout(L, Hv, T).total;
+    return tc_scratch_layout(L, Hv, T, out).total;
 }
 
 bool gdn_tc_shape(const GdnArgs& a) {
-    return a.dk == kD && a.dv == kD && a.dtype == DELTAS_BF16 && a.out == nullptr && a.T > 0;
+    return a.dk == kD && a.dv == kD && a.dtype == DELTAS_BF16 && a.T > 0;
 }
 
 bool gdn_tc_supported(const GdnArgs& a) {
+    const long long n_tiles = (a.T + kC - 1) / kC;
     return gdn_tc_shape(a) &&
            (long long)a.L * a.Hv * kD < (1ll << 31) &&                          // TMA row coordinate
-           (long long)a.L * a.Hv * ((a.T + kC - 1) / kC) < (1ll << 31) &&       // factor-kernel items
+           (long long)a.L * a.Hv * n_tiles < (1ll << 31) &&                     // factor-kernel items
+           (long long)a.L * a.Hv * ((n_tiles + 1) / 2) * kD < (1ll << 31) &&    // read-out block rows
            a.scratch != nullptr &&
-           a.scratch_bytes >= gdn_tc_scratch_bytes(a.L, a.Hv, a.dk, a.dv, a.dtype, a.T) &&
+           a.scratch_bytes >= gdn_tc_scratch_bytes(a.L, a.Hv, a.dk, a.dv, a.dtype, a.T, a.out != nullptr) &&
            encode_fn() != nullptr;
 }
 
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
-    const TcScratch sl = tc_scratch_layout(a.L, a.Hv, a.T);   // hand-over space for device_sm_count() CTAs
+    const bool out = a.out != nullptr;
+    const TcScratch sl = tc_scratch_layout(a.L, a.Hv, a.T, out);   // hand-over space for device_sm_count() CTAs
     // one chain CTA per SM that this context may use (a CTA waits at its end for its neighbour's
     // hand-over, so the grid must not exceed what can be resident)
     const int sms = context_sm_count();
     const int grid = std::min(a.L * a.Hv, sms);
-    CUtensorMap kmap, vmap, smap, hmap;
+    const int n_tiles = (a.T + kC - 1) / kC, n_blk = (n_tiles + 1) / 2;
+    const long long heads = (long long)a.L * a.Hv;
+    CUtensorMap kmap, vmap, smap, hmap, qmap, umap, bmap;
     if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
-        !make_state_map(&smap, a.state, a.L * a.Hv) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
+        !make_state_map(&smap, a.state, heads) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
         return cudaErrorInvalidValue;
+    if (out && (!make_map(&qmap, a.q, a.L, a.T, a.Hk) ||
+                !make_rows_map(&umap, a.scratch + sl.ubuf, heads * kD, n_tiles * kC) ||
+                !make_state_map(&bmap, a.scratch + sl.snap, heads * n_blk)))
+        return cudaErrorInvalidValue;
+    auto chain = out ? gdn_update_tc_kernel<true> : gdn_update_tc_kernel<false>;
     {   // set on every launch (cheap, and right for whichever device and context is current)
-        cudaError_t e = cudaFuncSetAttribute(gdn_update_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)kSmemAlloc);
+        cudaError_t e = cudaFuncSetAttribute(chain, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemAlloc);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(gdn_wy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kWySmemAlloc);
+        if (e == cudaSuccess && out)
+            e = cudaFuncSetAttribute(gdn_readout_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kRoSmemAlloc);
         if (e != cudaSuccess) return e;
     }
-    const int n_tiles = (a.T + kC - 1) / kC;
     // factor kernel: one record per (layer, value head, tile), kWyCtasPerSm persistent CTAs per SM
     WyArgs w;
-    w.L = a.L; w.Hk = a.Hk; w.Hv = a.Hv; w.T = a.T; w.n_tiles = n_tiles;
+    w.L = a.L; w.Hk = a.Hk; w.Hv = a.Hv; w.T = a.T; w.n_tiles = n_tiles; w.out = out ? 1 : 0;
     w.g = a.g; w.beta = a.beta; w.rec = a.scratch; w.status = a.status;
     w.ho_flags = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
     w.n_ho_flags = 2 * grid;
-    const long long items = (long long)a.L * a.Hv * n_tiles;
+    const long long items = heads * n_tiles;
     const int wgrid = (int)std::min<long long>(items, (long long)sms * kWyCtasPerSm);
     gdn_wy_kernel<<<wgrid, kWyThreads, kWySmemAlloc, s>>>(kmap, w);
     cudaError_t e = cudaGetLastError();
@@ -1495,6 +1846,10 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     t.ho_flag = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
     t.ho_wflag = t.ho_flag + grid;
     t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
+    t.ubuf = out ? reinterpret_cast<float*>(a.scratch + sl.ubuf) : nullptr;
+    t.snap = out ? reinterpret_cast<float*>(a.scratch + sl.snap) : nullptr;
+    t.Tp = n_tiles * kC;
+    t.n_blk = n_blk;
     // equal tile runs, with heads split between neighbouring CTAs, when they shorten the slowest
     // CTA: a boundary between slots costs about 0.45 of a tile and the hand-over about three
     // tiles (measured: 512- and 1024-token chunks gain 5-6 %, chunks of 2-3 tiles lose)
@@ -1506,9 +1861,16 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
         const double parted = runs + (runs / n_tiles + 2.0) * 0.45 + 3.0;
         t.split = parted < whole ? 1 : 0;
     }
-    (void)sms;
-    return launch_dependent(gdn_update_tc_kernel, dim3(grid), dim3(kThreads), (size_t)kSmemAlloc, s, kmap, vmap,
-                            smap, hmap, t);
+    e = launch_dependent(chain, dim3(grid), dim3(kThreads), (size_t)kSmemAlloc, s, kmap, vmap, smap, hmap, t);
+    if (e != cudaSuccess || !out) return e;
+    // read-out kernel: one persistent CTA per SM over the (layer, value head, 128-token block) items;
+    // its CTAs take the SMs the update kernel leaves free and wait there for its results
+    RoArgs r;
+    r.L = a.L; r.Hk = a.Hk; r.Hv = a.Hv; r.T = a.T; r.n_blk = n_blk; r.q_scale = a.q_scale;
+    r.g = a.g; r.out = static_cast<__nv_bfloat16*>(a.out); r.status = a.status;
+    const int rgrid = (int)std::min<long long>(heads * n_blk, sms);
+    return launch_dependent(gdn_readout_kernel, dim3(rgrid), dim3(kRoThreads), (size_t)kRoSmemAlloc, s, qmap, kmap,
+                            umap, bmap, r);
 }
 
 }  // namespace deltas

@@ -118,9 +118,10 @@ struct CopyBatch {
 
 // Kernel launchers (return the launch error, cudaSuccess when enqueued).
 cudaError_t launch_gdn_update_simt(const GdnArgs& a, cudaStream_t s);
-bool gdn_tc_shape(const GdnArgs& a);        // d = 128, bfloat16, no read-out, tokens > 0
+bool gdn_tc_shape(const GdnArgs& a);        // d = 128, bfloat16, tokens > 0
 bool gdn_tc_supported(const GdnArgs& a);    // ... and the tensor-core path can be launched
-size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T);
+// workspace past the status word for the tensor-core path (with or without the read-out)
+size_t gdn_tc_scratch_bytes(int L, int Hv, int dk, int dv, int dtype, int T, bool out);
 cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s);
 cudaError_t launch_state_drift(int L, int Hv, int dv, int dk, const float* sb, const float* sa,
                                float* partials, cudaStream_t s);

@@ -25,7 +25,7 @@ def _declared():
 
 def test_every_declared_symbol_is_exported(L):
     names = _declared()
-    assert len(names) == 25, names
+    assert len(names) == 26, names
     lib = ctypes.CDLL(L.LIB_PATH)
     for n in names:
         assert hasattr(lib, n), n
@@ -42,6 +42,14 @@ def test_version_and_status_strings(L):
 def test_workspace_sizes(L):
     d = L.GdnDesc(24, 16, 32, 128, 128, L.DELTAS_BF16, 0.088)
     assert L.deltas_gdn_chunk_update_workspace_size(d, 1024) >= 16
+    # the read-out keeps each token's write (512 B per token-head) and every 128-token block's
+    # starting state (64 KiB per block-head) beyond the factor records; only d = 128 bf16 has them
+    plain, ro = (L.deltas_gdn_chunk_update_workspace_size(d, 1024),
+                 L.deltas_gdn_chunk_update_readout_workspace_size(d, 1024))
+    assert ro - plain >= 24 * 32 * (1024 * 512 + 8 * 65536)
+    d64 = L.GdnDesc(2, 2, 4, 64, 64, L.DELTAS_BF16, 0.125)
+    assert (L.deltas_gdn_chunk_update_readout_workspace_size(d64, 100) ==
+            L.deltas_gdn_chunk_update_workspace_size(d64, 100))
     assert L.deltas_state_drift_workspace_size(d) >= 16
     a = L.deltas_select_retain_workspace_size(1000)
     b = L.deltas_select_retain_workspace_size(100000)

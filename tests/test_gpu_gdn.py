@@ -48,7 +48,9 @@ def _run_gpu(L, x, state, want_out, dtype, q_scale):
     st = state.to(dev).clone()
     out = torch.empty(Lg, T, Hv, d, dtype=dtype, device=dev) if want_out else None
     part = torch.full((Lg, Hv, 2), -1.0, device=dev)
-    ws = L.alloc_workspace(L.deltas_gdn_chunk_update_workspace_size(desc, T), dev)
+    size = (L.deltas_gdn_chunk_update_readout_workspace_size if want_out else
+            L.deltas_gdn_chunk_update_workspace_size)(desc, T)
+    ws = L.alloc_workspace(size, dev)
     L.deltas_gdn_chunk_update(desc, T, xs["q"] if want_out else None, xs["k"], xs["v"], xs["g"], xs["beta"],
                               st, out, part, ws)
     torch.cuda.synchronize()
@@ -81,7 +83,8 @@ def _check_chunk(L, x, state0, want_out, dtype, q_scale):
 def test_gdn_update_shapes(L, d, dtype, T, want_out):
     """Every head size, both activation dtypes, ragged token counts (one token, a tile minus one,
     exactly one tile, several tiles with a ragged tail), grouped keys (Hk=2, Hv=4), two layers,
-    with and without the read-out (d = 128 bf16 without read-out runs on the tensor cores)."""
+    with and without the read-out (d = 128 bf16 runs on the tensor cores, the read-out there in a
+    third kernel over 128-token blocks: T = 100 and 257 end inside a block's second tile)."""
     tdt = torch.float32 if dtype == "f32" else torch.bfloat16
     x = inputs.gdn_chunk(2, T, 2, 4, d, dtype, inputs.seed_for(1, d, T))
     s0 = inputs.initial_state(2, 4, d, inputs.seed_for(2, d, T))
@@ -123,35 +126,44 @@ def test_gdn_update_layer_width_chunk(L, want_out):
     _check_chunk(L, x, s0, want_out, torch.bfloat16, 128 ** -0.5)
 
 
-@pytest.mark.parametrize("T", [1, 130, 500])
-def test_gdn_update_more_heads_than_sms(L, T):
+@pytest.mark.parametrize("T,want_out", [(1, False), (130, False), (500, False), (130, True), (500, True)])
+def test_gdn_update_more_heads_than_sms(L, T, want_out):
     """160 (layer, head) pairs (5 layers x 32 value heads, d = 128, bf16): more heads than SMs, so
     the tensor-core kernel's persistent CTAs take equal runs of tiles and most heads are split
     between two neighbouring CTAs (the state handed over at the cut); every head's state and drift
-    partials are compared with the oracle (one tile, and three tiles with a ragged tail)."""
+    partials are compared with the oracle (one tile, and three tiles with a ragged tail), and with
+    the read-out every output (a cut may fall inside a 128-token read-out block, whose starting
+    state and writes then come from two CTAs)."""
     x = inputs.gdn_chunk(5, T, 16, 32, 128, "bf16", inputs.seed_for(12, T))
     s0 = inputs.initial_state(5, 32, 128, inputs.seed_for(13, T))
-    _check_chunk(L, x, s0, False, torch.bfloat16, 128 ** -0.5)
+    _check_chunk(L, x, s0, want_out, torch.bfloat16, 128 ** -0.5)
 
 
-def test_gdn_update_stack_width_sampled(L):
+@pytest.mark.parametrize("want_out", [False, True])
+def test_gdn_update_stack_width_sampled(L, want_out):
     """The full stack's width (24 layers x 32 value heads, d = 128, bf16, one 1024-token chunk)
-    in the launch configuration the benchmark times; the oracle checks a sample of 12 (layer,
-    head) pairs, each replayed from the same S_before."""
+    in the launch configuration the benchmark times, with and without the read-out; the oracle
+    checks a sample of 12 (layer, head) pairs, each replayed from the same S_before."""
     Lg, Hk, Hv, d, T = 24, 16, 32, 128, 1024
+    qs = 128 ** -0.5
     x = inputs.gdn_chunk(Lg, T, Hk, Hv, d, "bf16", inputs.seed_for(8, 2, 0))
     s0 = inputs.initial_state(Lg, Hv, d, 10)
-    st, _, part = _run_gpu(L, x, s0, False, torch.bfloat16, None)
+    st, out, part = _run_gpu(L, x, s0, want_out, torch.bfloat16, qs)
     rng = np.random.default_rng(3)
     pairs = [(0, 0), (Lg - 1, Hv - 1)] + [(int(rng.integers(Lg)), int(rng.integers(Hv))) for _ in range(10)]
     for (l, h) in pairs:
         kh = h * Hk // Hv
-        sub = {k: x[k][l:l + 1] for k in ("k", "v", "g", "beta")}
-        S_ref, _ = oracle.gdn_recurrence(None, _f64(sub["k"][:, :, kh:kh + 1]), _f64(sub["v"][:, :, h:h + 1]),
-                                         _f64(sub["g"][:, :, h:h + 1]), _f64(sub["beta"][:, :, h:h + 1]),
-                                         _f64(s0[l:l + 1, h:h + 1]))
+        sub = {k: x[k][l:l + 1] for k in ("q", "k", "v", "g", "beta")}
+        S_ref, o_ref = oracle.gdn_recurrence(_f64(sub["q"][:, :, kh:kh + 1]), _f64(sub["k"][:, :, kh:kh + 1]),
+                                             _f64(sub["v"][:, :, h:h + 1]), _f64(sub["g"][:, :, h:h + 1]),
+                                             _f64(sub["beta"][:, :, h:h + 1]), _f64(s0[l:l + 1, h:h + 1]),
+                                             q_scale=qs, want_out=want_out)
         rel = _per_head_rel(_f64(st[l:l + 1, h:h + 1]), S_ref).max()
         assert rel <= STATE_TOL, (l, h, rel)
+        if want_out:
+            o = _f64(out[l:l + 1, :, h:h + 1]).transpose(0, 2, 1, 3)
+            orl = _per_head_rel(o, o_ref.transpose(0, 2, 1, 3)).max()
+            assert orl <= STATE_TOL + 2.0 ** -8, (l, h, orl)
         p_ref = oracle.drift_partials(_f64(s0[l:l + 1, h:h + 1]), S_ref)[0, 0]
         np.testing.assert_allclose(_f64(part[l, h]), p_ref, rtol=1e-3)
     # every head moved and no head was left untouched or non-finite
@@ -181,6 +193,7 @@ def test_gdn_update_other_head_groupings(L, Hk, Hv):
     x = inputs.gdn_chunk(2, 257, Hk, Hv, 128, "bf16", inputs.seed_for(15, Hk, Hv))
     state0 = inputs.initial_state(2, Hv, 128, 16)
     _check_chunk(L, x, state0, False, torch.bfloat16, None)
+    _check_chunk(L, x, state0, True, torch.bfloat16, 0.3)
 
 
 @pytest.mark.parametrize("decay_scale", [0.0, 4.0])
@@ -199,6 +212,9 @@ def test_gdn_update_decay_extremes(L, decay_scale):
         assert (g == 0).all()
     state0 = inputs.initial_state(Lg, Hv, d, 14)
     _check_chunk(L, x, state0, False, torch.bfloat16, None)
+    # the read-out: a block's outputs weigh each earlier write of the block by exp(G_t - G_i) and
+    # its starting state by exp(G_t), both far below the fp32 range here for most pairs
+    _check_chunk(L, x, state0, True, torch.bfloat16, 0.2)
 
 
 def test_state_drift_kernel(L):
@@ -297,3 +313,61 @@ def test_write_norm_score(L):
     sc = scores.cpu().numpy()
     assert sc[7] == pytest.approx(oracle.write_norm_score(wn.astype(np.float64), 125), rel=1e-6)
     assert sc[8] == 0.0 and sc[6] == -1.0
+
+
+# ---------------------------------------------------------------- read-out on the tensor cores
+
+def test_readout_needs_its_workspace(L):
+    """A d = 128 bfloat16 call with out != NULL runs the read-out kernel, which keeps each token's
+    write and the block states in the workspace: the plain workspace size is refused (WORKSPACE),
+    the read-out size is accepted, and the outputs match the oracle."""
+    Lg, Hk, Hv, d, T = 1, 2, 4, 128, 200
+    dev = torch.device("cuda")
+    desc = L.gdn_desc(Lg, Hk, Hv, d, torch.bfloat16, 0.25)
+    small = L.deltas_gdn_chunk_update_workspace_size(desc, T)
+    big = L.deltas_gdn_chunk_update_readout_workspace_size(desc, T)
+    assert big > small
+    x = inputs.gdn_chunk(Lg, T, Hk, Hv, d, "bf16", inputs.seed_for(80, T))
+    xs = {k: v.to(dev) for k, v in x.items()}
+    st = torch.zeros(Lg, Hv, d, d, device=dev)
+    out = torch.empty(Lg, T, Hv, d, dtype=torch.bfloat16, device=dev)
+    with pytest.raises(L.DeltasError) as e:
+        L.deltas_gdn_chunk_update(desc, T, xs["q"], xs["k"], xs["v"], xs["g"], xs["beta"], st, out, None,
+                                  L.alloc_workspace(small, dev))
+    assert e.value.status == L.DELTAS_ERR_WORKSPACE
+    s0 = inputs.initial_state(Lg, Hv, d, 81)
+    _check_chunk(L, x, s0, True, torch.bfloat16, 0.25)
+
+
+@pytest.mark.parametrize("decay", [1.0, 4.0])
+def test_readout_with_write_norms(L, decay):
+    """The read-out and the write sizes in one call: outputs, state, drift partials and write
+    sizes against the oracle (the read-out path applies each tile's row decays in the state
+    chain instead of the factor records, so its state is checked on its own, not against the
+    path without read-out)."""
+    Lg, Hk, Hv, d, T = 2, 2, 4, 128, 300
+    x = inputs.gdn_chunk(Lg, T, Hk, Hv, d, "bf16", inputs.seed_for(82, int(decay)))
+    x["g"] = x["g"] * decay
+    s0 = inputs.initial_state(Lg, Hv, d, 83)
+    dev = torch.device("cuda")
+    desc = L.gdn_desc(Lg, Hk, Hv, d, torch.bfloat16, 0.125)
+    xs = {k: v.to(dev) for k, v in x.items()}
+    st = s0.to(dev).clone()
+    out = torch.empty(Lg, T, Hv, d, dtype=torch.bfloat16, device=dev)
+    part = torch.full((Lg, Hv, 2), -1.0, device=dev)
+    wn = torch.full((Lg, Hv), -1.0, device=dev)
+    ws = L.alloc_workspace(L.deltas_gdn_chunk_update_readout_workspace_size(desc, T), dev)
+    L.deltas_gdn_chunk_update(desc, T, xs["q"], xs["k"], xs["v"], xs["g"], xs["beta"], st, out, part, ws,
+                              write_norms=wn)
+    torch.cuda.synchronize()
+    assert L.deltas_get_device_status(ws) == (0, 0)
+    S_ref, o_ref, wn_ref = oracle.gdn_recurrence(_f64(x["q"]), _f64(x["k"]), _f64(x["v"]), _f64(x["g"]),
+                                                 _f64(x["beta"]), _f64(s0), q_scale=0.125, want_out=True,
+                                                 want_write_norms=True)
+    assert _per_head_rel(_f64(st), S_ref).max() <= STATE_TOL
+    o = _f64(out).transpose(0, 2, 1, 3)
+    assert _per_head_rel(o, o_ref.transpose(0, 2, 1, 3)).max() <= STATE_TOL + 2.0 ** -8
+    p_ref = oracle.drift_partials(_f64(s0), S_ref)
+    np.testing.assert_allclose(_f64(part)[..., 0], p_ref[..., 0], rtol=1e-3)
+    np.testing.assert_allclose(_f64(part)[..., 1], p_ref[..., 1], rtol=1e-5)
+    np.testing.assert_allclose(_f64(wn), wn_ref, rtol=1e-3, atol=0)
