@@ -683,10 +683,13 @@ struct TcArgs {
     int32_t* ho_flag;        // [grid] the state after the first part is in the hand-over map
     int32_t* ho_wflag;       // [grid] the first part's write-size sum is in ho_wsum
     float* ho_wsum;          // [grid]
-    // read-out: each token's write u_t, and the state at the start of every 128-token block
-    float* ubuf;             // [L * Hv][d_v][Tp] fp32: u_t (token-contiguous rows)
-    float* snap;             // [L * Hv][n_blk][d_v][d_k] fp32
-    int Tp, n_blk;           // Tp = 64 n_tiles, n_blk = ceil(n_tiles / 2)
+    // read-out: each token's write u_t, and the state at the start of every 128-token block,
+    // both as B operands of the read-out's MMAs (N = d_v rows, K-major, no swizzle): chunks of 4
+    // consecutive K values, each chunk's 128 rows of 16 bytes contiguous (a warp's 32 rows of one
+    // chunk are one 512-byte store)
+    float* ubuf;             // [L * Hv][16 n_tiles token chunks][d_v][4] fp32
+    float* snap;             // [L * Hv][n_blk][32 d_k chunks][d_v][4] fp32
+    int n_blk;               // ceil(n_tiles / 2)
 };
 
 // The CTA's work: a sequence of slots, each a run of consecutive tiles of one head.  By default
@@ -1237,10 +1240,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tmem_ld32(tm + lane_off + TM_S + 32 * cgp, sv);
                 tmem_ld_wait();
                 if (snap) {
-                    float* dst = a.snap + (((size_t)lh * a.n_blk + (jt >> 1)) * kD + r) * kD + 32 * cgp;
+                    float* dst = a.snap + ((((size_t)lh * a.n_blk + (jt >> 1)) * 32 + 8 * cgp) * kD + r) * 4;
 #pragma unroll
                     for (int e = 0; e < 8; ++e)
-                        *reinterpret_cast<float4*>(dst + 4 * e) =
+                        *reinterpret_cast<float4*>(dst + e * kD * 4) =
                             make_float4(sv[4 * e] * sig, sv[4 * e + 1] * sig, sv[4 * e + 2] * sig, sv[4 * e + 3] * sig);
                 }
                 if (rescale) {
@@ -1264,10 +1267,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 if constexpr (kOut) {
                     // with the record's undecayed T the column is u_t u_scale = u_t / sig: u_t out
                     // for the read-out (tokens jt 64 + 16 cgp .. of row r)
-                    float* dst = a.ubuf + ((size_t)lh * kD + r) * a.Tp + jt * kC + 16 * cgp;
+                    float* dst = a.ubuf + ((((size_t)lh * n + jt) * 16 + 4 * cgp) * kD + r) * 4;
 #pragma unroll
                     for (int e = 0; e < 4; ++e)
-                        *reinterpret_cast<float4*>(dst + 4 * e) =
+                        *reinterpret_cast<float4*>(dst + e * kD * 4) =
                             make_float4(uv[4 * e] * sig, uv[4 * e + 1] * sig, uv[4 * e + 2] * sig, uv[4 * e + 3] * sig);
                 }
                 if (want_w) {
@@ -1450,22 +1453,22 @@ constexpr uint32_t RT_P = 0, RT_Q = 128, RT_O = 256;  // TMEM: P (then P o D), d
 // shared-memory map (bytes from a 1024-aligned base)
 constexpr uint32_t RO_Q = 0;        // 32 KB: Q, 2 column blocks (d 0-63, 64-127) x 128 rows x 128 B, SW128
 constexpr uint32_t RO_K = 32768;    // 32 KB: K, same layout
-constexpr uint32_t RO_U = 65536;    // 64 KB: U^T [d_v][128 tokens] fp32, 4 column blocks x 128 rows x 128 B
-constexpr uint32_t RO_S = 131072;   // 64 KB: S_b [d_v][d_k] fp32, same layout
+constexpr uint32_t RO_U = 65536;    // 64 KB: U, [32 token chunks][d_v][4] fp32 (N = d_v, K = tokens, no swizzle)
+constexpr uint32_t RO_S = 131072;   // 64 KB: S_b, [32 d_k chunks][d_v][4] fp32 (N = d_v, K = d_k, no swizzle)
 constexpr uint32_t kRoSmemAlloc = 196608 + 1024;
 
 struct RoArgs {
-    int L, Hk, Hv, T, n_blk;
+    int L, Hk, Hv, T, n_tiles, n_blk;
     float q_scale;
     const float* g;
+    const float* ubuf;       // the update kernel's u_t and block states (TcArgs::ubuf, TcArgs::snap)
+    const float* snap;
     __nv_bfloat16* out;
     int32_t* status;
 };
 
 __global__ void __launch_bounds__(kRoThreads, 1)
-gdn_readout_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
-                   const __grid_constant__ CUtensorMap umap, const __grid_constant__ CUtensorMap bmap,
-                   RoArgs a)
+gdn_readout_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap, RoArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
@@ -1482,7 +1485,6 @@ gdn_readout_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_consta
         mbar_init(&mb_qk, 1); mbar_init(&mb_us, 1); mbar_init(&mb_p, 1); mbar_init(&mb_o, 1);
         fence_barrier_init();
         prefetch_tensormap(&qmap); prefetch_tensormap(&kmap);
-        prefetch_tensormap(&umap); prefetch_tensormap(&bmap);
         s_abort = 0;
     }
     tc_fence_before();
@@ -1504,14 +1506,15 @@ gdn_readout_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_consta
             }
         }
     };
-    auto load_us = [&](int it) {                       // thread 0: the item's U^T and S_b
+    // the item's block has two update tiles, or one (the last block of an odd tile count: its
+    // second half of U is zero-filled in shared memory)
+    auto block_tiles = [&](int it) { return min(2, a.n_tiles - 2 * (it % a.n_blk)); };
+    auto load_us = [&](int it) {                       // thread 0: the item's U and S_b (bulk copies)
         const int lh = it / a.n_blk, b = it - lh * a.n_blk;
-        mbar_arrive_expect_tx(&mb_us, 8 * 16384);
-#pragma unroll
-        for (int cb = 0; cb < 4; ++cb) {
-            tma_load_2d(sm + RO_U + cb * 16384, &umap, &mb_us, b * kRoBlk + 32 * cb, lh * kD);
-            tma_load_2d(sm + RO_S + cb * 16384, &bmap, &mb_us, 32 * cb, (lh * a.n_blk + b) * kD);
-        }
+        const uint32_t ub = (uint32_t)block_tiles(it) * 32768u;
+        mbar_arrive_expect_tx(&mb_us, ub + 65536u);
+        bulk_load_tx(sm + RO_U, a.ubuf + ((size_t)lh * a.n_tiles + 2 * b) * 16 * kD * 4, ub, &mb_us);
+        bulk_load_tx(sm + RO_S, a.snap + ((size_t)lh * a.n_blk + b) * 32 * kD * 4, 65536u, &mb_us);
     };
     int n_qk = 0, n_us = 0, n_p = 0, n_o = 0;          // copies / MMA groups issued (thread 0 / warp 0)
     const int first = (int)blockIdx.x, G = (int)gridDim.x;
@@ -1573,6 +1576,11 @@ gdn_readout_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_consta
         if (!ok && !*abort_flag) fail(a.status, abort_flag, 61);
         if (__syncthreads_or(!ok)) break;              // (also publishes s_g2)
         tc_fence_after();
+        if (block_tiles(it) == 1) {                    // (the previous item's MMAs have read U)
+            float4* z = reinterpret_cast<float4*>(sm + RO_U + 32768);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) z[tid + kRoThreads * e] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
         {
             // P o D in place: columns 64 hc .. + 63 of row t; a 16-column group right of every
             // row of the warp is all zero
@@ -1631,11 +1639,11 @@ gdn_readout_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_consta
             uint64_t bu[4][4], bs[4][4];
 #pragma unroll
             for (int s = 0; s < 16; ++s) {
-                const uint32_t off = (s >> 2) * 16384 + (s & 3) * 32;
                 ap[s >> 2][s & 3] = tm + RT_P + 8 * s;
                 aq[s >> 2][s & 3] = tm + RT_Q + 8 * s;
-                bu[s >> 2][s & 3] = sdesc_sw128(smem_u32(sm + RO_U + off), 16, 1024);
-                bs[s >> 2][s & 3] = sdesc_sw128(smem_u32(sm + RO_S + off), 16, 1024);
+                // K = 8 per MMA: two 4-element chunks of 2048 bytes
+                bu[s >> 2][s & 3] = sdesc_interleave(smem_u32(sm + RO_U) + 4096 * s, 2048, 128);
+                bs[s >> 2][s & 3] = sdesc_interleave(smem_u32(sm + RO_S) + 4096 * s, 2048, 128);
             }
             if (warp_wait(&mb_us, c & 1, kWaitBudgetNs, abort_flag)) {
                 tc_fence_after();
@@ -1752,8 +1760,9 @@ bool make_state_map(CUtensorMap* map, void* base, long long heads) {
 
 // Scratch: the WY records, then the update kernel's hand-over area for up to one CTA per SM:
 // states [grid][128][128] fp32 (1024-aligned), flags [2][grid] int32, write-size sums [grid];
-// with the read-out, then each token's write u_t [L * Hv][128][64 n_tiles] fp32 and the state at
-// the start of every 128-token block [L * Hv][n_blk][128][128] fp32 (both 1024-aligned).
+// with the read-out, then each token's write u_t (128 floats per token and value head) and the
+// state at the start of every 128-token block (128 x 128 floats per block and value head), both
+// 1024-aligned, in the layouts of TcArgs::ubuf and TcArgs::snap.
 struct TcScratch {
     size_t rec, ho_state, ho_flags, ho_wsum, ubuf, snap, total;
 };
@@ -1809,14 +1818,11 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     const int grid = std::min(a.L * a.Hv, sms);
     const int n_tiles = (a.T + kC - 1) / kC, n_blk = (n_tiles + 1) / 2;
     const long long heads = (long long)a.L * a.Hv;
-    CUtensorMap kmap, vmap, smap, hmap, qmap, umap, bmap;
+    CUtensorMap kmap, vmap, smap, hmap, qmap;
     if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
         !make_state_map(&smap, a.state, heads) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
         return cudaErrorInvalidValue;
-    if (out && (!make_map(&qmap, a.q, a.L, a.T, a.Hk) ||
-                !make_rows_map(&umap, a.scratch + sl.ubuf, heads * kD, n_tiles * kC) ||
-                !make_state_map(&bmap, a.scratch + sl.snap, heads * n_blk)))
-        return cudaErrorInvalidValue;
+    if (out && !make_map(&qmap, a.q, a.L, a.T, a.Hk)) return cudaErrorInvalidValue;
     auto chain = out ? gdn_update_tc_kernel<true> : gdn_update_tc_kernel<false>;
     {   // set on every launch (cheap, and right for whichever device and context is current)
         cudaError_t e = cudaFuncSetAttribute(chain, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemAlloc);
@@ -1848,7 +1854,6 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
     t.ubuf = out ? reinterpret_cast<float*>(a.scratch + sl.ubuf) : nullptr;
     t.snap = out ? reinterpret_cast<float*>(a.scratch + sl.snap) : nullptr;
-    t.Tp = n_tiles * kC;
     t.n_blk = n_blk;
     // equal tile runs, with heads split between neighbouring CTAs, when they shorten the slowest
     // CTA: a boundary between slots costs about 0.45 of a tile and the hand-over about three
@@ -1866,11 +1871,10 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     // read-out kernel: one persistent CTA per SM over the (layer, value head, 128-token block) items;
     // its CTAs take the SMs the update kernel leaves free and wait there for its results
     RoArgs r;
-    r.L = a.L; r.Hk = a.Hk; r.Hv = a.Hv; r.T = a.T; r.n_blk = n_blk; r.q_scale = a.q_scale;
-    r.g = a.g; r.out = static_cast<__nv_bfloat16*>(a.out); r.status = a.status;
+    r.L = a.L; r.Hk = a.Hk; r.Hv = a.Hv; r.T = a.T; r.n_tiles = n_tiles; r.n_blk = n_blk; r.q_scale = a.q_scale;
+    r.g = a.g; r.ubuf = t.ubuf; r.snap = t.snap; r.out = static_cast<__nv_bfloat16*>(a.out); r.status = a.status;
     const int rgrid = (int)std::min<long long>(heads * n_blk, sms);
-    return launch_dependent(gdn_readout_kernel, dim3(rgrid), dim3(kRoThreads), (size_t)kRoSmemAlloc, s, qmap, kmap,
-                            umap, bmap, r);
+    return launch_dependent(gdn_readout_kernel, dim3(rgrid), dim3(kRoThreads), (size_t)kRoSmemAlloc, s, qmap, kmap, r);
 }
 
 }  // namespace deltas

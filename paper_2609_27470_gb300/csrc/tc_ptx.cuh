@@ -269,6 +269,15 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo_byt
            ((uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
 }
 
+// Shared-memory matrix descriptor without swizzle, K-major: the operand is a grid of core matrices
+// of 8 rows x 16 bytes, each stored as 128 contiguous bytes; LBO = byte stride between core
+// matrices along K, SBO = byte stride between 8-row groups along M/N.  Step K by advancing the
+// start by the LBO per 16 bytes of K.
+__device__ __forceinline__ uint64_t sdesc_interleave(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo_bytes) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo_bytes >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32) | (1ull << 46);
+}
+
 // Instruction descriptor, kind::f16 with bf16 A and B, fp32 accumulator; bit 13 negates A.
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn_major, int b_mn_major, int negate_a = 0) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)negate_a << 13) | ((uint32_t)a_mn_major << 15) |
