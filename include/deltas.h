@@ -408,13 +408,17 @@ DELTAS_API deltas_status deltas_compact_kv_heads(const deltas_kv_desc* desc, voi
 DELTAS_API deltas_status deltas_clear_device_status(void* workspace, void* stream);
 
 /* Enqueue on `stream` a write of the workspace's bounded-wait budget (word 2 of the status
- * header): every wait of a kernel that runs with this workspace gives up after `budget_ns`
- * nanoseconds (0, the value deltas_clear_device_status leaves: about one second) and records
- * DELTAS_ERR_TIMEOUT; the waits that drain a kernel's own copies and MMAs before it exits keep the
- * one-second budget.  Not a paper operation: a wait that runs out is the library's answer to a
- * peer that never arrives (a CTA that cannot become resident, say), and a small budget lets a
- * test or a latency-bound caller make that path run.  The host value is copied before the call
- * returns. */
+ * header): a wait bounded by it gives up after `budget_ns` nanoseconds (0, the value
+ * deltas_clear_device_status leaves: about one second) and records DELTAS_ERR_TIMEOUT; the other
+ * roles of that kernel then stop at their next wait, drain the copies and MMAs they issued (those
+ * drains keep the one-second bound) and return.  It bounds every wait of the selection and
+ * compaction kernels, and the first wait of each kernel of deltas_gdn_chunk_update (the factor
+ * kernel's first key tile, the state chain's first value tile, the read-out's first query and key
+ * blocks); the per-tile waits of the update keep the one-second bound, since a bound read at run
+ * time there made the latency-bound state chain about 5 % slower.  Not a paper operation: a wait
+ * that runs out is the library's answer to a peer that never arrives (a CTA that cannot become
+ * resident, say), and a small budget lets a test make that path run.  The host value is copied
+ * before the call returns. */
 DELTAS_API deltas_status deltas_set_wait_budget(void* workspace, uint32_t budget_ns, void* stream);
 
 /* Synchronise `stream`, then read the status word: *status_out = first recorded deltas_status

@@ -211,12 +211,6 @@ __device__ __forceinline__ void fail(int32_t* status, volatile int* abort, int w
     *abort = 1;
 }
 
-// One arrival per warp on a chain -> MMA barrier: every lane's TMEM stores / shared-memory
-// writes were completed and fenced before the __syncwarp; lane 0 then arrives (release).
-__device__ __forceinline__ void warp_arrive(uint64_t* bar, int lane) {
-    __syncwarp();
-    if (lane == 0) mbar_arrive(bar);
-}
 
 // shared-memory descriptor advanced by `bytes` (the start address field counts 16-byte units)
 __device__ __forceinline__ uint64_t dadd(uint64_t desc, uint32_t bytes) { return desc + (uint64_t)(bytes >> 4); }
@@ -280,6 +274,9 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int n = a.n_tiles;
     const int items = a.L * a.Hv * n;                 // item = (layer * Hv + head) * n + tile
+    // The workspace's wait budget bounds the CTA's first wait; the later ones keep the fixed bound
+    // (a bound read at run time in every wait of these latency-bound kernels measured slower).
+    const uint64_t budget0 = wait_budget_ns(a.status);
     float* fA = reinterpret_cast<float*>(sm + WY_FA);
     float* fX = reinterpret_cast<float*>(sm + WY_FX);
     float* fT = reinterpret_cast<float*>(sm + WY_TMP);
@@ -381,7 +378,8 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap kmap, WyArgs a)
     // K K^T of the item-th item of this CTA into TMEM (warp 0; M = 128: rows 64..127 of A read the
     // 8 KB past the tile, their output is ignored)
     auto issue_kk = [&](int item) {
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(&mb_k, item & 1, kWaitBudgetNs)) != 0;
+        const bool ok = __all_sync(0xffffffffu, item == 0 ? mbar_wait(&mb_k, 0, budget0)
+                                                           : mbar_wait(&mb_k, item & 1, kWaitBudgetNs)) != 0;
         if (!ok) {
             if (lane == 0) { record_status(a.status, DELTAS_ERR_TIMEOUT, 21); s_fail = 1; }
             return;
@@ -833,21 +831,24 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         // chain warps).
         // V region <- V(J)^T: A = the V tile read MN-major (k-step s = tokens 16 s ..), B = I.  V(J)'s
         // buffer is released when the product completes.
-        auto issue_vi = [&](int J) -> bool {
+        auto issue_vi = [&](int J, uint64_t budget) -> bool {
             uint64_t av[4], bv[4];
 #pragma unroll
             for (int s = 0; s < 4; ++s) {
                 av[s] = dadd(dV, (J & 1) * 16384 + s * 2048); bv[s] = dadd(dI, s * 32);
                 pin(av[s]); pin(bv[s]);
             }
-            if (!warp_wait(&mb_tv[J & 1], (J >> 1) & 1, kWaitBudgetNs, abort_flag)) return false;
+            if (!warp_wait(&mb_tv[J & 1], (J >> 1) & 1, budget, abort_flag)) return false;
             tc_fence_after();
             if (elect_one()) mma4_bf16_ss_1t(tm + TM_V, av, bv, idesc_bf16(128, 64, 1, 0), 0);
             __syncwarp();
             mma_commit(&mb_ve[J & 1]);
             return true;
         };
-        bool ok = NJ == 0 || issue_vi(0);
+        // the workspace's wait budget bounds this first wait (V of the CTA's first tile); the
+        // per-tile waits keep the fixed bound (a bound read at run time in every wait of this
+        // latency-bound chain measured 5 % slower)
+        bool ok = NJ == 0 || issue_vi(0, wait_budget_ns(a.status));
         if (!ok) fail(a.status, abort_flag, 1);
         for (int j = 0; ok && j < NJ; ++j) {           // j: global tile index
             {   // X region <- S~ K^T: A = the fp32 state from TMEM read as tf32 (8 columns per K = 8
@@ -899,7 +900,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             }
             // the next tile's V^T into the V region (its last reader, the W pass of tile j, has
             // finished: MMA_U(j) waited for xready)
-            if (j + 1 < NJ && !issue_vi(j + 1)) { fail(a.status, abort_flag, 4); break; }
+            if (j + 1 < NJ && !issue_vi(j + 1, kWaitBudgetNs)) { fail(a.status, abort_flag, 4); break; }
             {   // S~ += U~^T K  (A: U~ hi / lo packed in place in U; K read MN-major)
                 uint32_t as_[2][4];
                 uint64_t bs[2][4];
@@ -1021,8 +1022,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             if (ok) {
                 ok = mbar_wait_or_abort(&mb_sfree, 0, kWaitBudgetNs, abort_flag);
                 if (!ok) fail(a.status, abort_flag, 40);
+                else seen = loads;                     // the chain has consumed it (so it landed)
             }
-            seen = loads;                              // the chain has consumed it
             if (ok) {
                 if (n_slots > 1) {
                     ok = load_state(1);
@@ -1075,8 +1076,24 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
         // K(jj) (TMA tile, buffer jj % 3) in fp32 (exact, and exact in tf32) into the B operand
         // buffer of X.  Called between MMA_X(jj-1), the last reader of the buffer, and the ready
         // signal of tile jj.
+        // A chain warp arrives (lane 0, for the warp) on sready / xready / uready / sfree only while
+        // every wait of lane 0 has seen its phase complete: the MMA and state warps take a completed
+        // phase as proof that the copies the passes waited for have landed (after another role
+        // failed, they would otherwise release buffers whose copies may still be in flight).
+        bool failed = false;
+        auto cwait = [&](uint64_t* bar, uint32_t parity, int where) {
+            const bool ok = mbar_wait_or_abort(bar, parity, kWaitBudgetNs, abort_flag);
+            if (!ok) { fail(a.status, abort_flag, where); failed = true; }
+            return ok;
+        };
+        // (one arrival per warp: every lane's TMEM stores / shared-memory writes were completed and
+        // fenced before the __syncwarp; lane 0 then arrives, a release)
+        auto carrive = [&](uint64_t* bar) {
+            __syncwarp();
+            if (lane == 0 && !failed) mbar_arrive(bar);
+        };
         auto make_k32 = [&](int jj) -> bool {
-            const bool ok = mbar_wait_or_abort(&mb_tk[jj % 3], (jj / 3) & 1, kWaitBudgetNs, abort_flag);
+            const bool ok = cwait(&mb_tk[jj % 3], (jj / 3) & 1, 16);
             const uint8_t* kb = sm + SM_K + (jj % 3) * 16384;
             uint8_t* k32 = sm + SM_K32;
 #pragma unroll
@@ -1154,7 +1171,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             const int lh = cc.lh, jt = cc.jt, slot = cc.k; // head, tile within the head, slot
             const bool last = jt == cc.te - 1;             // the slot's last tile
             if (named_sync_or(2, kChain, *abort_flag)) break;
-            if (!mbar_wait_or_abort(&mb_tr[j & 1], (j >> 1) & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 13);
+            cwait(&mb_tr[j & 1], (j >> 1) & 1, 13);
             const float gC = rec_consts(j)[64];
             float w_gamma = 0.f;                           // gamma_t of this lane's column in the Ũ pass
             if (want_w) {
@@ -1171,7 +1188,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             if (j == 0) {
                 // ---- the CTA's first head: its state from the staging buffer into TMEM, as S~
                 // (sig = 1) and as S_before, and sum S_before^2
-                if (!mbar_wait_or_abort(&mb_st, 0, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 14);
+                cwait(&mb_st, 0, 14);
                 st_seen = 1;
                 float sv[32];
 #pragma unroll
@@ -1181,20 +1198,20 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
 #pragma unroll
                 for (int e = 0; e < 32; ++e) den = fmaf(sv[e], sv[e], den);
-                warp_arrive(&mb_sfree, lane);                    // the staging buffer has been read
+                carrive(&mb_sfree);                              // the staging buffer has been read
                 tmem_st32(tm + lane_off + TM_S + 32 * cgp, sv);
                 tmem_st32(tm + lane_off + TM_SB + 32 * cgp, sv);
-                if (!make_k32(0)) fail(a.status, abort_flag, 16);
+                make_k32(0);
                 tmem_st_wait();
                 tc_fence_before();
-                warp_arrive(&mb_sready, lane);
+                carrive(&mb_sready);
             }
             const bool rescale = sig * gC < kSigMin;       // uniform over the CTA
             const float u_scale = rescale ? 1.f : 1.f / (gC * sig);
 
             // ---- W pass: W^T = V^T - sig X~^T diag(gamma) from the V and X regions (X~ = S~ K^T),
             // scaled by u_scale, (hi, lo) in place over this thread's 16 X columns (tokens 16 cgp ..)
-            if (!mbar_wait_or_abort(&mb_x, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 10);
+            cwait(&mb_x, j & 1, 10);
             tc_fence_after();
             // read-out: the row decays of the thread's 16 tokens, taken now (the record's slot is
             // released to the next load once MMA_U(j) completes, before the U~ pass)
@@ -1228,7 +1245,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tmem_st_wait();
             }
             tc_fence_before();
-            warp_arrive(&mb_xready, lane);
+            carrive(&mb_xready);
 
             // ---- while MMA_U runs: rescale S~ if the decay would underflow the deferred scale
             // (MMA_X(j) has read S~; MMA_S(j) waits for uready), and K(j+1) in fp32.  For the
@@ -1255,10 +1272,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
             }
             sig = rescale ? 1.f : gC * sig;                // the deferred decay after tile j
-            if (j + 1 < NJ && !make_k32(j + 1)) fail(a.status, abort_flag, 16);
+            if (j + 1 < NJ) make_k32(j + 1);
 
             // ---- U~ pass: (hi, lo) in place over this thread's 16 U columns
-            if (!mbar_wait_or_abort(&mb_u, j & 1, kWaitBudgetNs, abort_flag)) fail(a.status, abort_flag, 11);
+            cwait(&mb_u, j & 1, 11);
             tc_fence_after();
             {
                 float uv[16];
@@ -1315,10 +1332,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 tmem_st_wait();
             }
             tc_fence_before();
-            warp_arrive(&mb_uready, lane);
+            carrive(&mb_uready);
             if (!last) {
                 // the next tile of this head may start X as soon as MMA_S(j) is queued
-                warp_arrive(&mb_sready, lane);
+                carrive(&mb_sready);
             } else {
                 // ---- head boundary: S_after = sig S~ out through the staging buffer, the next
                 // head's state (staged meanwhile) into TMEM, drift partials against S_before
@@ -1328,12 +1345,9 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 // here
                 const bool shared_end = sch.is_suffix(slot);
                 float den_end = 0.f;
-                bool ok = mbar_wait_or_abort(&mb_s, j & 1, kWaitBudgetNs, abort_flag);
-                if (!ok) fail(a.status, abort_flag, 12);
-                if (!mbar_wait_or_abort(&mb_st, st_seen & 1, kWaitBudgetNs, abort_flag)) {
-                    fail(a.status, abort_flag, 14);
-                    ok = false;
-                }
+                bool ok = cwait(&mb_s, j & 1, 12);
+                if (!cwait(&mb_st, st_seen & 1, 14)) ok = false;
+                ok = __all_sync(0xffffffffu, ok) != 0;     // (the pass below is warp-collective)
                 ++st_seen;
                 tc_fence_after();
                 float num = 0.f, den_next = 0.f;
@@ -1384,8 +1398,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
                 tc_fence_before();
                 fence_async_smem();                        // S_after -> the state warp's TMA store
-                warp_arrive(&mb_sfree, lane);
-                if (has_next) warp_arrive(&mb_sready, lane);     // the next head's state is in TMEM
+                carrive(&mb_sfree);
+                if (has_next) carrive(&mb_sready);               // the next head's state is in TMEM
                 // partial sums: pairwise in fp32, over the warp's lanes and then over the 16 warps
                 // (the FP64 pipe is far too slow for this path)
                 float fn = num, fd = shared_end ? den_end : den;
@@ -1559,7 +1573,8 @@ gdn_readout_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_consta
                 aq[s >> 2][s & 3] = sdesc_sw128(smem_u32(sm + RO_Q + off), 16, 1024);
                 bk[s >> 2][s & 3] = sdesc_sw128(smem_u32(sm + RO_K + off), 16, 1024);
             }
-            if (warp_wait(&mb_qk, c & 1, kWaitBudgetNs, abort_flag)) {
+            if (c == 0 ? warp_wait(&mb_qk, 0, wait_budget_ns(a.status), abort_flag)   // (the workspace's
+                       : warp_wait(&mb_qk, c & 1, kWaitBudgetNs, abort_flag)) {      //  budget: first wait)
                 tc_fence_after();
                 if (elect_one()) {
                     mma4_bf16_ss_1t(tm + RT_P, aq[0], bk[0], idesc_bf16(128, 128, 0, 0), 0);

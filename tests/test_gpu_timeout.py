@@ -1,5 +1,7 @@
 """The bounded-wait path on the GPU: a wait that runs out records DELTAS_ERR_TIMEOUT in the
-workspace's status word, the call returns, and the next call with the default budget is correct.
+workspace's status word, the call returns, and the next call with the default budget is correct
+(the compaction's waits, and the first wait of each of the update's kernels, after which every
+other role of the kernel stops on the abort flag and drains).
 
 No wait here is left without a limit and nothing faults: the test only shortens the budget of
 the waits (deltas_set_wait_budget) so that they give up at their first check.  A compaction unit
@@ -58,3 +60,49 @@ def test_compact_wait_runs_out_then_recovers(L):
     rk, rv, rtc, rtp = oracle.compact_kv(_np(kc), _np(vc), tc, tp, keep, cap)
     assert np.array_equal(_np(k.cpu()), rk) and np.array_equal(_np(v.cpu()), rv)
     assert np.array_equal(t1.cpu().numpy(), rtc) and np.array_equal(t2.cpu().numpy(), rtp)
+
+
+def _rel(a, b):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return float(np.max(np.sqrt(np.sum((a - b) ** 2, axis=(-2, -1)) / np.sum(b ** 2, axis=(-2, -1)))))
+
+
+@pytest.mark.parametrize("want_out", [False, True])
+def test_update_wait_runs_out_then_recovers(L, want_out):
+    """The tensor-core update (d = 128 bf16: factor kernel, state chain and, with the read-out,
+    the read-out kernel) with a 1 ns wait budget, which bounds each kernel's first wait: those
+    waits give up, the other roles stop at their next wait (they see the abort flag), drain the
+    copies and products they issued and free TMEM; the call ends with DELTAS_ERR_TIMEOUT
+    recorded.  The same call with the default budget, from the restored state, then matches the
+    oracle."""
+    Lg, Hk, Hv, d, T = 1, 2, 4, 128, 200
+    x = inputs.gdn_chunk(Lg, T, Hk, Hv, d, "bf16", inputs.seed_for(90, int(want_out)))
+    s0 = inputs.initial_state(Lg, Hv, d, 91)
+    dev = torch.device("cuda")
+    desc = L.gdn_desc(Lg, Hk, Hv, d, torch.bfloat16, 0.25)
+    size = (L.deltas_gdn_chunk_update_readout_workspace_size if want_out else
+            L.deltas_gdn_chunk_update_workspace_size)(desc, T)
+    ws = L.alloc_workspace(size, dev)
+    xs = {k: v.to(dev) for k, v in x.items()}
+    st = s0.to(dev).clone()
+    out = torch.empty(Lg, T, Hv, d, dtype=torch.bfloat16, device=dev) if want_out else None
+    part = torch.zeros(Lg, Hv, 2, device=dev)
+    q = xs["q"] if want_out else None
+
+    L.deltas_set_wait_budget(ws, 1)
+    L.deltas_gdn_chunk_update(desc, T, q, xs["k"], xs["v"], xs["g"], xs["beta"], st, out, part, ws)
+    status, where = L.deltas_get_device_status(ws)
+    assert status == L.DELTAS_ERR_TIMEOUT and where > 0
+
+    L.deltas_clear_device_status(ws)
+    st.copy_(s0.to(dev))
+    L.deltas_gdn_chunk_update(desc, T, q, xs["k"], xs["v"], xs["g"], xs["beta"], st, out, part, ws)
+    assert L.deltas_get_device_status(ws) == (0, 0)
+    f64 = lambda t: t.float().cpu().double().numpy()       # noqa: E731
+    S_ref, o_ref = oracle.gdn_recurrence(f64(x["q"]), f64(x["k"]), f64(x["v"]), f64(x["g"]), f64(x["beta"]),
+                                         f64(s0), q_scale=0.25, want_out=want_out)
+    assert _rel(f64(st), S_ref) <= 2e-3
+    if want_out:
+        o = f64(out).transpose(0, 2, 1, 3)
+        assert _rel(o, o_ref.transpose(0, 2, 1, 3)) <= 2e-3 + 2.0 ** -8
