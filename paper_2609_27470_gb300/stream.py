@@ -54,7 +54,7 @@ class DeltaSStream:
     def __init__(self, *, num_layers, num_k_heads, num_v_heads, head_dim, act_dtype: torch.dtype,
                  kv_layers, kv_heads, kv_head_dim, kv_dtype: torch.dtype, budget_M, n_sink=0,
                  n_window=0, n_buckets=1, chunk_len, max_chunks, q_scale=None, state0=None,
-                 device="cuda", signal: str = "drift"):
+                 device="cuda", signal: str = "drift", read_out: bool = False):
         if signal not in ("drift", "write_norm") + tuple(L.SIGNALS):
             raise ValueError(f"unknown signal {signal!r}")
         self.signal = signal
@@ -82,12 +82,17 @@ class DeltaSStream:
         lists = (kv_layers * kv_heads, budget_M) if self.per_head else (budget_M,)
         self.retain_idx = torch.zeros(lists, dtype=torch.int32, device=dev)
         self.n_retained = torch.zeros(1, dtype=torch.int32, device=dev)
+        # read_out: step() may be given ``out`` (the layer output o_t); the update's workspace then
+        # also holds each token's write and the block states (d = 128 bf16)
+        gdn_ws = (L.deltas_gdn_chunk_update_readout_workspace_size if read_out else
+                  L.deltas_gdn_chunk_update_workspace_size)(self.gdn, chunk_len)
+        self.read_out = read_out
         if self.per_head:
-            ws = max(L.deltas_gdn_chunk_update_workspace_size(self.gdn, chunk_len),
+            ws = max(gdn_ws,
                      L.deltas_select_retain_heads_workspace_size(kv_layers * kv_heads, self.capacity),
                      L.deltas_compact_kv_heads_workspace_size(self.kv, self.capacity))
         else:
-            ws = max(L.deltas_gdn_chunk_update_workspace_size(self.gdn, chunk_len),
+            ws = max(gdn_ws,
                      L.deltas_select_retain_workspace_size(self.capacity),
                      L.deltas_compact_kv_workspace_size(self.kv, self.capacity))
         self.workspace = L.alloc_workspace(ws, dev)
@@ -102,6 +107,8 @@ class DeltaSStream:
         if c >= self.max_chunks:
             raise ValueError("stream longer than max_chunks")
         T = int(k.shape[1])
+        if out is not None and not self.read_out:
+            raise ValueError("step(out=...) needs a stream built with read_out=True")
         L.deltas_gdn_chunk_update(self.gdn, T, q, k, v, g, beta, self.state, out, self.partials,
                                   self.workspace, stream, write_norms=self.write_norms)
         if self.per_head:

@@ -75,3 +75,44 @@ def test_stream_matches_oracle(cfg):
     assert np.array_equal(_np(s.v_cache[:, :, :n].cpu()), ref.v_cache[:, :, :n])
     assert np.array_equal(s.tok_chunk[:n].cpu().numpy(), ref.tok_chunk[:n])
     assert np.array_equal(s.tok_pos[:n].cpu().numpy(), ref.tok_pos[:n])
+
+
+def test_stream_read_out_paper_shape():
+    """Alg. 1 Prefill with the layer output: the paper's chunk lengths (118-132 tokens, every
+    chunk a ragged tail, blocks of 128 read-out tokens cut at different places) through a stream
+    built with read_out=True (d = 128 bf16: the tensor-core update and read-out kernels), with
+    evictions running in between; every chunk's outputs against the oracle replayed from the
+    stream's own state before the chunk, and a stream without read_out refuses an output buffer."""
+    import oracle
+    from paper_2609_27470_gb300.stream import DeltaSStream
+    dev = torch.device("cuda")
+    Lg, Hk, Hv, d = 2, 2, 4, 128
+    lens = [118, 132, 124, 121, 129, 119, 127, 125]
+    qs = 128 ** -0.5
+    mk = lambda ro: DeltaSStream(num_layers=Lg, num_k_heads=Hk, num_v_heads=Hv, head_dim=d, act_dtype=torch.bfloat16,
+                                 kv_layers=1, kv_heads=2, kv_head_dim=128, kv_dtype=torch.bfloat16, budget_M=300,
+                                 n_sink=4, n_window=64, n_buckets=2, chunk_len=max(lens), max_chunks=len(lens),
+                                 state0=inputs.initial_state(Lg, Hv, d, 7).to(dev), device=dev, q_scale=qs,
+                                 read_out=ro)
+    s = mk(True)
+    f64 = lambda t: t.float().cpu().double().numpy()       # noqa: E731
+    for c, T in enumerate(lens):
+        x = {k: v.to(dev) for k, v in inputs.gdn_chunk(Lg, T, Hk, Hv, d, "bf16", inputs.seed_for(8, c)).items()}
+        kn, vn = inputs.kv_chunk(1, 2, T, 128, "bf16", inputs.seed_for(9, c))
+        s_before = s.state.clone()
+        out = torch.empty(Lg, T, Hv, d, dtype=torch.bfloat16, device=dev)
+        s.step(x["q"], x["k"], x["v"], x["g"], x["beta"], kn.to(dev), vn.to(dev), out=out)
+        torch.cuda.synchronize()
+        _, o_ref = oracle.gdn_recurrence(f64(x["q"]), f64(x["k"]), f64(x["v"]), f64(x["g"]), f64(x["beta"]),
+                                         f64(s_before), q_scale=qs, want_out=True)
+        o = f64(out)
+        rel = np.sqrt(((o - o_ref) ** 2).sum(axis=(1, 3)) / (o_ref ** 2).sum(axis=(1, 3)))
+        assert rel.max() <= 2e-3 + 2.0 ** -8, (c, rel.max())
+    from paper_2609_27470_gb300 import _lib as L
+    assert L.deltas_get_device_status(s.workspace) == (0, 0) and s.evictions > 0
+    plain = mk(False)
+    x = {k: v.to(dev) for k, v in inputs.gdn_chunk(Lg, lens[0], Hk, Hv, d, "bf16", 1).items()}
+    kn, vn = inputs.kv_chunk(1, 2, lens[0], 128, "bf16", 2)
+    with pytest.raises(ValueError):
+        plain.step(x["q"], x["k"], x["v"], x["g"], x["beta"], kn.to(dev), vn.to(dev),
+                   out=torch.empty(Lg, lens[0], Hv, d, dtype=torch.bfloat16, device=dev))

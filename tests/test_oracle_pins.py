@@ -235,6 +235,38 @@ def test_output_reads_the_updated_state():
         np.testing.assert_allclose(o[0, t, 0], 0.3 * St[0, 0] @ q[0, t, 0].astype(np.float64), rtol=1e-13, atol=1e-14)
 
 
+@pytest.mark.parametrize("blk", [1, 5, 8, 13])
+def test_block_readout_identity(blk):
+    """The algebra the GPU read-out uses, checked against the oracle's token loop: unrolling Eq. 1
+    from the state S_b before a block, S_t = exp(G_t) S_b + sum_{i <= t} exp(G_t - G_i) u_i k_i^T
+    (G the inclusive cumulative log-decay inside the block, u_i = beta_i (v_i - alpha_i S_{i-1} k_i)
+    the write of token i), so a block's outputs are q_scale ((Q K^T o D) U + diag(exp(G)) Q S_b^T).
+    Blocks of several lengths (one token, and lengths that do not divide T) over 30 tokens."""
+    rng = np.random.default_rng(20 + blk)
+    T, d, qs = 30, 6, 0.4
+    q, k, v, g, beta = _rand_inputs(rng, 1, T, 1, 1, d, decay=0.5)
+    S0 = rng.standard_normal((1, 1, d, d))
+    _, o_ref = oracle.gdn_recurrence(q, k, v, g, beta, S0, q_scale=qs, want_out=True)
+    q, k, v = (x[0, :, 0].astype(np.float64) for x in (q, k, v))
+    g, beta = (x[0, :, 0].astype(np.float64) for x in (g, beta))
+    S = S0[0, 0].copy()
+    u = np.zeros((T, d))
+    for t in range(T):                     # the writes u_t of the token loop (plain numpy)
+        a = np.exp(g[t])
+        u[t] = beta[t] * (v[t] - a * S @ k[t])
+        S = a * S + np.outer(u[t], k[t])
+    S = S0[0, 0].copy()
+    o = np.zeros((T, d))
+    for b0 in range(0, T, blk):
+        b1 = min(T, b0 + blk)
+        G = np.cumsum(g[b0:b1])
+        D = np.tril(np.exp(G[:, None] - G[None, :]))
+        Q, K, U = q[b0:b1], k[b0:b1], u[b0:b1]
+        o[b0:b1] = qs * (((Q @ K.T) * D) @ U + np.exp(G)[:, None] * (Q @ S.T))
+        S = np.exp(G[-1]) * S + (np.exp(G[-1] - G)[:, None] * U).T @ K     # the state after the block
+    np.testing.assert_allclose(o, o_ref[0, :, 0], rtol=1e-11, atol=1e-12)
+
+
 # ---------------------------------------------------------------- drift (Eq. 3)
 
 def test_drift_hand_worked_two_layers():
