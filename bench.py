@@ -609,6 +609,8 @@ def make_workload(name, dev, L):
         return StreamingWorkload(dev, L, _cfg(name))
     if name == "stack":
         return GdnOnlyWorkload(dev, L, configs.STACK)
+    if name == "stack_out":
+        return GdnOnlyWorkload(dev, L, configs.STACK_OUT)
     if name == "layer":
         return GdnOnlyWorkload(dev, L, configs.LAYER)
     if name == "layer_out":
@@ -736,7 +738,7 @@ def oracle_sample(workload: str, budget_s: float = 12.0, threads: int = 1):
         parts.append(f"drift of {n} (layer,head) state pairs x{factor:.0f} extrapolated; score of {cfg['L']} layers")
     head_signal = cfg.get("signal") in ("key_norm", "value_norm")
     if workload in ("streaming", "paper", "paper_write_norm", "paper_key_norm", "paper_value_norm", "stack",
-                    "layer", "layer_out"):
+                    "stack_out", "layer", "layer_out"):
         C = int(round(_tokens(workload)))
         heads_total = cfg["L"] * cfg["Hv"]
         n_heads = 2
@@ -886,6 +888,7 @@ def config_line(workload):
 
 def _cfg(workload):
     return {"streaming": configs.STREAMING, "paper": configs.PAPER, "stack": configs.STACK,
+            "stack_out": configs.STACK_OUT,
             "layer": configs.LAYER, "layer_out": configs.LAYER_OUT, "kv": configs.KV, "snapshot": configs.PAPER, "drift": configs.DRIFT,
             "paper_write_norm": configs.PAPER_WRITE_NORM, "paper_key_norm": configs.PAPER_KEY_NORM,
             "paper_value_norm": configs.PAPER_VALUE_NORM}[workload]
@@ -910,7 +913,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="streaming",
                     choices=["streaming", "paper", "paper_write_norm", "paper_key_norm", "paper_value_norm",
-                             "stack", "layer", "layer_out", "kv", "snapshot", "drift"])
+                             "stack", "stack_out", "layer", "layer_out", "kv", "snapshot", "drift"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)

@@ -29,6 +29,8 @@ LAYER_OUT = dict(LAYER, name="layer_out", with_out=True)
 
 STACK = dict(name="stack", L=24, Hk=16, Hv=32, d=128, dtype="bf16", chunk_len=1024, n_chunks=256,
              ring=8)
+# the same with the layer output of every layer
+STACK_OUT = dict(STACK, name="stack_out", with_out=True)
 
 # the standalone drift (Eq. 3) of the full stack's states: S_before and S_after of 24 layers x 32
 # value heads x 128 x 128 fp32 (48 MiB each), a ring of 4 pairs (384 MiB, beyond L2)
