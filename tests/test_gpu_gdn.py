@@ -371,3 +371,28 @@ def test_readout_with_write_norms(L, decay):
     np.testing.assert_allclose(_f64(part)[..., 0], p_ref[..., 0], rtol=1e-3)
     np.testing.assert_allclose(_f64(part)[..., 1], p_ref[..., 1], rtol=1e-5)
     np.testing.assert_allclose(_f64(wn), wn_ref, rtol=1e-3, atol=0)
+
+
+@pytest.mark.parametrize("T", [128, 129, 191, 192, 256])
+def test_readout_block_boundaries(L, T):
+    """Token counts at and around the read-out's 128-token blocks: a block that ends the chunk
+    exactly, one token into the next block, a last block of one tile (its second half absent and
+    zero-filled) and of two."""
+    x = inputs.gdn_chunk(1, T, 2, 4, 128, "bf16", inputs.seed_for(84, T))
+    s0 = inputs.initial_state(1, 4, 128, inputs.seed_for(85, T))
+    _check_chunk(L, x, s0, True, torch.bfloat16, 128 ** -0.5)
+
+
+def test_readout_zero_tokens(L):
+    """n_tokens = 0 with an output buffer: nothing is written, the state is unchanged."""
+    dev = torch.device("cuda")
+    desc = L.gdn_desc(1, 2, 4, 128, torch.bfloat16, 0.25)
+    s0 = inputs.initial_state(1, 4, 128, 86)
+    st = s0.to(dev).clone()
+    big = torch.full((1, 1, 4, 128), 7.0, dtype=torch.bfloat16, device=dev)   # zero-token views of it
+    q = torch.zeros(1, 1, 2, 128, dtype=torch.bfloat16, device=dev)
+    ws = L.alloc_workspace(L.deltas_gdn_chunk_update_readout_workspace_size(desc, 0), dev)
+    L.deltas_gdn_chunk_update(desc, 0, q[:, :0], None, None, None, None, st, big[:, :0], None, ws)
+    torch.cuda.synchronize()
+    assert L.deltas_get_device_status(ws) == (0, 0)
+    assert torch.equal(st.cpu(), s0) and bool((big == 7.0).all())
