@@ -681,6 +681,9 @@ struct TcArgs {
     int32_t* ho_flag;        // [grid] the state after the first part is in the hand-over map
     int32_t* ho_wflag;       // [grid] the first part's write-size sum is in ho_wsum
     float* ho_wsum;          // [grid]
+    // segments (see ChainSched): seg > 1 runs each head's tiles as seg segments on 2 seg - 1
+    // CTAs, whose end states go to the hand-over map's rows (CTA i: rows 128 i ..)
+    int seg;
     // read-out: each token's write u_t, and the state at the start of every 128-token block,
     // both as B operands of the read-out's MMAs (N = d_v rows, K-major, no swizzle): chunks of 4
     // consecutive K values, each chunk's 128 rows of 16 bytes contiguous (a warp's 32 rows of one
@@ -698,14 +701,37 @@ struct TcArgs {
 // it shares with CTA i + 1 first (its first tiles; the state at the cut goes to hand-over entry i)
 // and the head it shares with CTA i - 1 last (its last tiles, from hand-over entry i - 1), so the
 // second part of a shared head is never waited for before its first part is long finished.
+//
+// Segments.  When the heads are few (a single layer: 32 heads on 152 SMs) the tiles of one head
+// run in series on one CTA while most SMs idle.  A run of tiles is an affine map of the state,
+// S_end = S_start A + B, so the host may cut each head's tiles into seg segments: CTA 0 of the
+// head's 2 seg - 1 runs segment 0 from the state; for each later segment s, one CTA runs it from
+// S = I with v = 0 (its end state is A_s) and one from S = 0 (B_s).  The CTAs write their end
+// states to the hand-over map; gdn_segment_combine_kernel then forms
+// S_after = (S_0 A_1 + B_1) A_2 + B_2 ... and the drift partials.
 struct ChainSched {
+    int seg_mode;              // 0: not segmented; 1: segment 0 (from the state); 2: from I, v = 0;
+                               // 3: from 0
+    int seg_lh, seg_tb, seg_te;
     int split;
     int pre_lh, pre_len;       // first slot: tiles [0, pre_len) of head pre_lh (none if pre_len == 0)
     int full0, n_full;         // then n_full whole heads from full0 (every gridDim.x-th if !split)
     int suf_lh, suf_from;      // last slot: tiles [suf_from, n) of head suf_lh (none if suf_from == 0)
     int n_slots, NJ;
-    __device__ void init(const TcArgs& a) {
+    __device__ __forceinline__ void init(const TcArgs& a, bool segmented) {
         const int n = a.n_tiles, G = (int)gridDim.x, i = (int)blockIdx.x, H = a.L * a.Hv;
+        seg_mode = 0;
+        if (segmented) {
+            const int per = 2 * a.seg - 1, hd = i / per, r = i - hd * per, sg = (r + 1) >> 1;
+            seg_mode = r == 0 ? 1 : (r & 1) ? 2 : 3;
+            seg_lh = hd;
+            seg_tb = (int)((long long)sg * n / a.seg);          // balanced cuts: >= 4 tiles each
+            seg_te = (int)((long long)(sg + 1) * n / a.seg);
+            split = 0;
+            pre_lh = suf_lh = -1; pre_len = suf_from = 0;
+            full0 = hd; n_full = n_slots = 1; NJ = seg_te - seg_tb;
+            return;
+        }
         split = a.split && H > G && H % G != 0;
         if (!split) {
             pre_lh = suf_lh = -1; pre_len = suf_from = 0;
@@ -726,6 +752,7 @@ struct ChainSched {
     __device__ __forceinline__ bool is_prefix(int k) const { return pre_len > 0 && k == 0; }
     __device__ __forceinline__ bool is_suffix(int k) const { return suf_from > 0 && k == n_slots - 1; }
     __device__ void slot(int k, int n, int& lh, int& tb, int& te) const {
+        if (seg_mode) { lh = seg_lh; tb = seg_tb; te = seg_te; return; }
         tb = 0; te = n;
         if (!split) { lh = full0 + k * (int)gridDim.x; return; }
         if (is_prefix(k)) { lh = pre_lh; te = pre_len; return; }
@@ -755,7 +782,7 @@ struct TileCursor {
     }
 };
 
-template <bool kOut>
+template <bool kOut, bool kSeg>
 __global__ void __launch_bounds__(kThreads, 1)
 gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap smap, const __grid_constant__ CUtensorMap hmap,
@@ -779,7 +806,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
     // Persistent CTA: its slots (ChainSched) form one sequence of NJ tiles, over which every role
     // keeps its barrier phases.
     ChainSched sch;
-    sch.init(a);
+    sch.init(a, kSeg);
     const int n_slots = sch.n_slots;
     const int NJ = sch.NJ;
 
@@ -1002,6 +1029,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             auto load_state = [&](int slot) -> bool {
                 int lh, tb, te;
                 sch.slot(slot, n, lh, tb, te);
+                if (kSeg && sch.seg_mode >= 2) { mbar_arrive(&mb_st); return true; }   // the chain forms it
                 if (!sch.is_suffix(slot)) { load_rows(&smap, lh * kD); return true; }
                 grid_dep_wait();                       // the factor kernel reset the flags
                 const uint64_t t0 = global_ns();
@@ -1038,8 +1066,9 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 int lh, tb, te;
                 sch.slot(k, n, lh, tb, te);
                 const bool hand_over = sch.is_prefix(k);
-                const CUtensorMap* dst = hand_over ? &hmap : &smap;
-                const int row = (hand_over ? me : lh) * kD;
+                const bool to_h = hand_over || kSeg;      // (a segment's end state: row me)
+                const CUtensorMap* dst = to_h ? &hmap : &smap;
+                const int row = (to_h ? me : lh) * kD;
 #pragma unroll
                 for (int b = 0; b < 4; ++b) tma_store_2d(dst, sbuf + 4096 * b, 32 * b, row);
                 bulk_commit();
@@ -1191,10 +1220,15 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 cwait(&mb_st, 0, 14);
                 st_seen = 1;
                 float sv[32];
+                if (kSeg && sch.seg_mode >= 2) {           // a later segment: from I or from 0
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, 8 * cgp + e));
-                    sv[4 * e] = x.x; sv[4 * e + 1] = x.y; sv[4 * e + 2] = x.z; sv[4 * e + 3] = x.w;
+                    for (int e = 0; e < 32; ++e) sv[e] = (sch.seg_mode == 2 && r == 32 * cgp + e) ? 1.f : 0.f;
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float4 x = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, 8 * cgp + e));
+                        sv[4 * e] = x.x; sv[4 * e + 1] = x.y; sv[4 * e + 2] = x.z; sv[4 * e + 3] = x.w;
+                    }
                 }
 #pragma unroll
                 for (int e = 0; e < 32; ++e) den = fmaf(sv[e], sv[e], den);
@@ -1235,6 +1269,10 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     cf[4 * e] = g4.x * sig; cf[4 * e + 1] = g4.y * sig; cf[4 * e + 2] = g4.z * sig; cf[4 * e + 3] = g4.w * sig;
                 }
                 tmem_ld_wait();
+                if (kSeg && sch.seg_mode == 2) {           // the run that forms a segment's A: v = 0
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) vv[e] = 0.f;
+                }
                 uint32_t hi[8], lo[8];
 #pragma unroll
                 for (int i = 0; i < 8; ++i)
@@ -1410,7 +1448,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
                 if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
                 if (named_sync_or(2, kChain, !ok)) break;
-                if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot)) {   // a shared head's drift: at its end
+                if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot) && !kSeg) {
+                    // (a shared head's drift: at its end; a segmented head's: the combine kernel's)
                     float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
                     float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
 #pragma unroll
@@ -1443,6 +1482,176 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
     if (warp == kMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tm, kTmemCols);
+    }
+}
+
+// =============================================================================================
+// Segment combine: S_after = S_0 A_1 + B_1 for heads the chain ran in two segments
+// =============================================================================================
+// One CTA of 512 threads per head.  Bulk copies bring S_0 and A_1 (fp32, 64 KB each, in turn through
+// the result tile) to be split into bfloat16 (hi, lo) images (S_0 K-major, rows r and K = d; A_1
+// MN-major, K rows d and N = d'); three tcgen05 products S0_hi A_hi + S0_hi A_lo + S0_lo A_hi
+// accumulate S_0 A_1 in TMEM (fp32; the dropped lo * lo term is below 2^-16 relative); then B_1 and
+// S_before are copied into the freed image space, the TMEM rows go to the padded result tile (warp
+// w: lane quarter w % 4, column quarter w / 4), and coalesced passes over shared memory form
+// S_after = S_0 A_1 + B_1, store it and take the drift sums (per thread in float, a fixed tree over
+// each warp, the warps in order).
+constexpr int kCbThreads = 4 * kD;
+constexpr int kCbPad = kD + 4;                          // fp32 row stride of the result tile
+constexpr uint32_t CB_XH = 0, CB_XL = 32768;            // S_0 images: 2 column blocks x 128 rows x 128 B; then S_before
+constexpr uint32_t CB_AH = 65536, CB_AL = 98304;        // A images: 2 N blocks (d' 0-63, 64-127) x 128 K rows; then B
+constexpr uint32_t CB_D = 131072;                       // staging of S_0 and A (dense), then the result tile [128][kCbPad]
+constexpr uint32_t kCbSmem = CB_D + kD * kCbPad * 4 + 1024;
+constexpr uint32_t kMat = kD * kD * 4;                  // one 128 x 128 fp32 matrix
+
+struct CbArgs {
+    const float* ends;       // the chain CTAs' end states, [chain CTA][128][128] fp32 (3 per head)
+    float* state;            // [heads][128][128]: in S_before, out S_after
+    float* partials;         // [heads][2] or null
+    int32_t* status;
+};
+
+// The dense 128 x 128 fp32 matrix at m (shared memory) as (hi, lo) bfloat16 images, 128-byte
+// swizzled, two 16 KB column blocks (elements 0-63, 64-127); thread t takes 8-element chunks t,
+// t + kCbThreads, ...
+__device__ __forceinline__ void split_images(const float* m, uint8_t* hi, uint8_t* lo) {
+#pragma unroll
+    for (int u = 0; u < kD * kD / 8 / kCbThreads; ++u) {
+        const int idx = (int)threadIdx.x + kCbThreads * u, row = idx >> 4, ch = idx & 15;
+        const float4* src = reinterpret_cast<const float4*>(m + row * kD + 8 * ch);
+        const float4 a = src[0], b = src[1];
+        const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        uint4 vh, vl;
+        split8(x, vh, vl);
+        const uint32_t off = (ch >> 3) * 16384 + sw128_offset(row, ch & 7);
+        *reinterpret_cast<uint4*>(hi + off) = vh;
+        *reinterpret_cast<uint4*>(lo + off) = vl;
+    }
+}
+
+__global__ void __launch_bounds__(kCbThreads, 1)
+gdn_segment_combine_kernel(CbArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    float* dt = reinterpret_cast<float*>(sm + CB_D);
+    __shared__ uint64_t mb_ld, mb_d;
+    __shared__ uint32_t s_tmem;
+    __shared__ float s_red[2][kCbThreads / 32];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int q = warp & 3, cq = warp >> 2;
+    const uint32_t lane_off = (uint32_t)(32 * q) << 16;
+    const int head = blockIdx.x;
+    const uint8_t* base = reinterpret_cast<const uint8_t*>(a.ends) + (size_t)head * 3 * kMat;
+    float* st = a.state + (size_t)head * kD * kD;
+    if (warp == 0) { tmem_alloc(&s_tmem, kD); tmem_relinquish(); }
+    if (tid == 32) { mbar_init(&mb_ld, 1); mbar_init(&mb_d, 1); fence_barrier_init(); }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = s_tmem;
+    grid_dep_wait();                                   // the chain's end states are written
+    int n_ld = 0;                                      // bulk-copy groups issued (thread 0)
+    bool ok = true;
+    auto load = [&](void* dst0, const void* src0, void* dst1, const void* src1) {   // thread 0
+        mbar_arrive_expect_tx(&mb_ld, src1 ? 2 * kMat : kMat);
+        bulk_load_tx(dst0, src0, kMat, &mb_ld);
+        if (src1) bulk_load_tx(dst1, src1, kMat, &mb_ld);
+    };
+    auto wait_ld = [&](int where) {                    // everyone; uniform result
+        const bool w = mbar_wait(&mb_ld, (n_ld - 1) & 1, kWaitBudgetNs);
+        if (!w) record_status(a.status, DELTAS_ERR_TIMEOUT, where);
+        ok = __syncthreads_or(!w) == 0;
+    };
+    if (tid == 0) load(dt, base, nullptr, nullptr);    // S_0
+    ++n_ld;
+    wait_ld(70);
+    if (ok) split_images(dt, sm + CB_XH, sm + CB_XL);
+    __syncthreads();                                   // the staging buffer is free again
+    if (ok) {
+        if (tid == 0) load(dt, base + kMat, nullptr, nullptr);    // A_1
+        ++n_ld;
+        wait_ld(71);
+    }
+    if (ok) {
+        split_images(dt, sm + CB_AH, sm + CB_AL);
+        fence_async_smem();                            // the images -> the tensor core
+        tc_fence_before();
+        __syncthreads();
+        if (warp == 0) {
+            tc_fence_after();
+            if (elect_one()) {
+                const uint32_t id = idesc_bf16(128, 128, 0, 1);
+#pragma unroll
+                for (int term = 0; term < 3; ++term) {   // S0_hi A_hi, S0_hi A_lo, S0_lo A_hi
+                    const uint32_t xb = term == 2 ? CB_XL : CB_XH, ab = term == 1 ? CB_AL : CB_AH;
+#pragma unroll
+                    for (int s = 0; s < 8; ++s) {        // K = 16 per MMA
+                        const uint64_t da = sdesc_sw128(smem_u32(sm + xb + (s >> 2) * 16384 + (s & 3) * 32), 16, 1024);
+                        const uint64_t db = sdesc_sw128(smem_u32(sm + ab + s * 2048), 16384, 1024);
+                        mma_bf16_1t(tm, da, db, id, (term | s) != 0);
+                    }
+                }
+            }
+            __syncwarp();
+            mma_commit(&mb_d);
+        }
+        const bool w = mbar_wait(&mb_d, 0, kWaitBudgetNs);
+        if (!w) record_status(a.status, DELTAS_ERR_TIMEOUT, 72);
+        ok = __syncthreads_or(!w) == 0;
+    }
+    if (ok) {
+        // the images have been read: B_1 and S_before into their space, meanwhile S_0 A_1 into the tile
+        if (tid == 0) load(sm + CB_AH, base + 2 * kMat, sm + CB_XH, st);
+        ++n_ld;
+        tc_fence_after();
+        {
+            const int row = 32 * q + lane;
+            float d[32];
+            tmem_ld32(tm + lane_off + 32 * cq, d);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 32; e += 4)
+                *reinterpret_cast<float4*>(dt + row * kCbPad + 32 * cq + e) = make_float4(d[e], d[e + 1], d[e + 2], d[e + 3]);
+        }
+        wait_ld(73);                                   // (also orders the tile's writes before the pass)
+    }
+    if (ok) {
+        const float* sB = reinterpret_cast<const float*>(sm + CB_AH);
+        const float* sS = reinterpret_cast<const float*>(sm + CB_XH);
+        float num = 0.f, den = 0.f;
+#pragma unroll
+        for (int u = 0; u < kD * kD / 4 / kCbThreads; ++u) {
+            const int idx = tid + kCbThreads * u, row = idx >> 5, c4 = idx & 31;
+            const float4 dv = reinterpret_cast<const float4*>(dt + row * kCbPad)[c4];
+            const float4 b = reinterpret_cast<const float4*>(sB + row * kD)[c4];
+            const float4 sb = reinterpret_cast<const float4*>(sS + row * kD)[c4];
+            const float4 sa = make_float4(dv.x + b.x, dv.y + b.y, dv.z + b.z, dv.w + b.w);
+            const float d0 = sa.x - sb.x, d1 = sa.y - sb.y, d2 = sa.z - sb.z, d3 = sa.w - sb.w;
+            num += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+            den += sb.x * sb.x + sb.y * sb.y + sb.z * sb.z + sb.w * sb.w;
+            reinterpret_cast<float4*>(st + (size_t)row * kD)[c4] = sa;
+        }
+#pragma unroll
+        for (int m = 16; m >= 1; m >>= 1) {
+            num += __shfl_xor_sync(0xffffffffu, num, m);
+            den += __shfl_xor_sync(0xffffffffu, den, m);
+        }
+        if (lane == 0) { s_red[0][warp] = num; s_red[1][warp] = den; }
+    } else if (tid == 0 && n_ld > 0) {
+        mbar_wait(&mb_ld, (n_ld - 1) & 1, kWaitBudgetNs);   // (after a failure: the last copies land)
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (ok && tid == 0 && a.partials != nullptr) {
+        float n = 0.f, d = 0.f;
+        for (int w = 0; w < kCbThreads / 32; ++w) { n += s_red[0][w]; d += s_red[1][w]; }
+        a.partials[(size_t)head * 2] = n;
+        a.partials[(size_t)head * 2 + 1] = d;
+    }
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tm, kD);
     }
 }
 
@@ -1784,12 +1993,22 @@ struct TcScratch {
 
 size_t align1k(size_t x) { return (x + 1023) & ~size_t(1023); }
 
+// Segments per head (see ChainSched) for a call without read-out or write sizes: two when three
+// CTAs per head fit on the SMs and each half keeps at least 4 tiles (the combine costs a few
+// microseconds), else 1 (not segmented: the heads share the SMs).
+int segments_for(int heads, int n_tiles, int sms) {
+    return ((long long)heads * 3 <= sms && n_tiles >= 8) ? 2 : 1;
+}
+
 TcScratch tc_scratch_layout(int L, int Hv, int T, bool out) {
-    const int grid = std::max(1, std::min(L * Hv, device_sm_count()));
+    const int sms = device_sm_count();
     const size_t n_tiles = (size_t)(T + kC - 1) / kC, n_blk = (n_tiles + 1) / 2, heads = (size_t)L * Hv;
+    // the chain's grid: one CTA per SM at most, or 2 seg - 1 per head when segmented
+    const int sg = out ? 1 : segments_for(L * Hv, (int)n_tiles, sms);
+    const int grid = std::max(1, sg > 1 ? L * Hv * (2 * sg - 1) : std::min(L * Hv, sms));
     TcScratch l;
     l.rec = 0;
-    l.ho_state = align1k(heads * n_tiles * rec_bytes(out));
+    l.ho_state = align1k(heads * n_tiles * rec_bytes(out));          // hand-over / segment end states
     l.ho_flags = l.ho_state + (size_t)grid * kD * kD * 4;
     l.ho_wsum = l.ho_flags + 2 * (size_t)grid * 4;
     l.total = l.ho_wsum + (size_t)grid * 4;
@@ -1830,15 +2049,19 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     // one chain CTA per SM that this context may use (a CTA waits at its end for its neighbour's
     // hand-over, so the grid must not exceed what can be resident)
     const int sms = context_sm_count();
-    const int grid = std::min(a.L * a.Hv, sms);
     const int n_tiles = (a.T + kC - 1) / kC, n_blk = (n_tiles + 1) / 2;
     const long long heads = (long long)a.L * a.Hv;
+    // few heads: each head's tiles in segments on 2 seg - 1 CTAs (not with the read-out or the write
+    // sizes: a later segment's run does not see the true state)
+    const int sg = (out || a.wnorm != nullptr) ? 1 : segments_for(a.L * a.Hv, n_tiles, sms);
+    const int grid = sg > 1 ? a.L * a.Hv * (2 * sg - 1) : std::min(a.L * a.Hv, sms);
     CUtensorMap kmap, vmap, smap, hmap, qmap;
     if (!make_map(&kmap, a.k, a.L, a.T, a.Hk) || !make_map(&vmap, a.v, a.L, a.T, a.Hv) ||
         !make_state_map(&smap, a.state, heads) || !make_state_map(&hmap, a.scratch + sl.ho_state, grid))
         return cudaErrorInvalidValue;
     if (out && !make_map(&qmap, a.q, a.L, a.T, a.Hk)) return cudaErrorInvalidValue;
-    auto chain = out ? gdn_update_tc_kernel<true> : gdn_update_tc_kernel<false>;
+    auto chain = out ? gdn_update_tc_kernel<true, false>
+                     : sg > 1 ? gdn_update_tc_kernel<false, true> : gdn_update_tc_kernel<false, false>;
     {   // set on every launch (cheap, and right for whichever device and context is current)
         cudaError_t e = cudaFuncSetAttribute(chain, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemAlloc);
         if (e == cudaSuccess)
@@ -1846,6 +2069,9 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
         if (e == cudaSuccess && out)
             e = cudaFuncSetAttribute(gdn_readout_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)kRoSmemAlloc);
+        if (e == cudaSuccess && sg > 1)
+            e = cudaFuncSetAttribute(gdn_segment_combine_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kCbSmem);
         if (e != cudaSuccess) return e;
     }
     // factor kernel: one record per (layer, value head, tile), kWyCtasPerSm persistent CTAs per SM
@@ -1867,6 +2093,7 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     t.ho_flag = reinterpret_cast<int32_t*>(a.scratch + sl.ho_flags);
     t.ho_wflag = t.ho_flag + grid;
     t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
+    t.seg = sg;
     t.ubuf = out ? reinterpret_cast<float*>(a.scratch + sl.ubuf) : nullptr;
     t.snap = out ? reinterpret_cast<float*>(a.scratch + sl.snap) : nullptr;
     t.n_blk = n_blk;
@@ -1875,14 +2102,23 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     // tiles (measured: 512- and 1024-token chunks gain 5-6 %, chunks of 2-3 tiles lose)
     t.split = 0;
     const int H = a.L * a.Hv;
-    if (H > grid && H % grid != 0) {
+    if (sg == 1 && H > grid && H % grid != 0) {
         const double whole = std::ceil((double)H / grid) * (n_tiles + 0.45);
         const double runs = std::ceil((double)H * n_tiles / grid);
         const double parted = runs + (runs / n_tiles + 2.0) * 0.45 + 3.0;
         t.split = parted < whole ? 1 : 0;
     }
     e = launch_dependent(chain, dim3(grid), dim3(kThreads), (size_t)kSmemAlloc, s, kmap, vmap, smap, hmap, t);
-    if (e != cudaSuccess || !out) return e;
+    if (e != cudaSuccess) return e;
+    if (sg > 1) {
+        // segment combine: S_after and the drift partials of every head from its CTAs' end states
+        CbArgs c;
+        c.ends = reinterpret_cast<const float*>(a.scratch + sl.ho_state);
+        c.state = a.state; c.partials = a.partials; c.status = a.status;
+        return launch_dependent(gdn_segment_combine_kernel, dim3((unsigned)heads), dim3(kCbThreads),
+                                (size_t)kCbSmem, s, c);
+    }
+    if (!out) return e;
     // read-out kernel: one persistent CTA per SM over the (layer, value head, 128-token block) items;
     // its CTAs take the SMs the update kernel leaves free and wait there for its results
     RoArgs r;

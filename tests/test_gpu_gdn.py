@@ -396,3 +396,21 @@ def test_readout_zero_tokens(L):
     torch.cuda.synchronize()
     assert L.deltas_get_device_status(ws) == (0, 0)
     assert torch.equal(st.cpu(), s0) and bool((big == 7.0).all())
+
+
+@pytest.mark.parametrize("Lg,Hk,Hv,T,decay", [
+    (1, 2, 4, 1024, 0.1),     # 4 heads: two segments of 8 tiles (3 CTAs per head)
+    (1, 4, 8, 1000, 0.1),     # 8 heads, a ragged last tile in the second segment
+    (1, 1, 2, 512, 4.0),      # strong decay: the runs from I and from 0 restart their deferred decay
+    (1, 1, 2, 1024, 0.0),     # no decay: the affine maps keep their full range
+    (1, 16, 32, 512, 0.1),    # the single layer's heads, 8 tiles: two segments of 4
+    (1, 16, 32, 449, 0.1),    # 8 tiles, the second segment ending in a one-token tile
+])
+def test_gdn_update_segments(L, Lg, Hk, Hv, T, decay):
+    """Few heads (at most a third of the SMs) and at least 8 tiles: the state chain runs each head's
+    tiles as two segments, the second once from S = I with v = 0 and once from S = 0, and the
+    combine forms S_after = S_0 A_1 + B_1 and the drift partials; state and partials against the
+    oracle."""
+    x = inputs.gdn_chunk(Lg, T, Hk, Hv, 128, "bf16", inputs.seed_for(89, T, Hv), decay_scale=decay)
+    s0 = inputs.initial_state(Lg, Hv, 128, inputs.seed_for(90, T, Hv))
+    _check_chunk(L, x, s0, False, torch.bfloat16, None)
