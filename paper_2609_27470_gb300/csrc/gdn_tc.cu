@@ -658,6 +658,7 @@ constexpr uint32_t SM_SB = SM_I + 8192;          // 64 KB: state staging, 4 colu
 constexpr uint32_t SM_BYTES = SM_SB + 65536;
 constexpr uint32_t kSmemAlloc = SM_BYTES + 1024;
 static_assert(SM_I % 1024 == 0 && SM_SB % 1024 == 0 && kRecSlot >= kRecBytesOut, "shared-memory map");
+static_assert(SM_SB >= 131072, "the segment combine's images ([0, 128 KB)) lie below the staging buffer");
 static_assert(kSmemAlloc <= 232448, "shared memory budget");
 
 // The staging buffer holds a head's [d_v][d_k] fp32 state as four column blocks of 32 floats, each
@@ -681,9 +682,9 @@ struct TcArgs {
     int32_t* ho_flag;        // [grid] the state after the first part is in the hand-over map
     int32_t* ho_wflag;       // [grid] the first part's write-size sum is in ho_wsum
     float* ho_wsum;          // [grid]
-    // segments (see ChainSched): seg > 1 runs each head's tiles as seg segments on 2 seg - 1
-    // CTAs, whose end states go to the hand-over map's rows (CTA i: rows 128 i ..)
+    // segments (see ChainSched): seg = 2 runs each head's tiles as two segments on three CTAs
     int seg;
+    uint8_t* ho_base;        // the hand-over states (the hmap rows): CTA i's 64 KB at ho_base + 64 KB i
     // read-out: each token's write u_t, and the state at the start of every 128-token block,
     // both as B operands of the read-out's MMAs (N = d_v rows, K-major, no swizzle): chunks of 4
     // consecutive K values, each chunk's 128 rows of 16 bytes contiguous (a warp's 32 rows of one
@@ -704,11 +705,12 @@ struct TcArgs {
 //
 // Segments.  When the heads are few (a single layer: 32 heads on 152 SMs) the tiles of one head
 // run in series on one CTA while most SMs idle.  A run of tiles is an affine map of the state,
-// S_end = S_start A + B, so the host may cut each head's tiles into seg segments: CTA 0 of the
-// head's 2 seg - 1 runs segment 0 from the state; for each later segment s, one CTA runs it from
-// S = I with v = 0 (its end state is A_s) and one from S = 0 (B_s).  The CTAs write their end
-// states to the hand-over map; gdn_segment_combine_kernel then forms
-// S_after = (S_0 A_1 + B_1) A_2 + B_2 ... and the drift partials.
+// S_end = S_start A + B, so the host may cut each head's tiles in two halves on three CTAs: CTA 0
+// runs the first half from the state, CTA 1 the second half from S = I with v = 0 (its end state
+// is A, written as the bfloat16 (hi, lo) images of an MN-major MMA operand) and CTA 2 from S = 0
+// (B, fp32); both raise their hand-over flag.  CTA 0 then waits for them (bounded), forms
+// S_0 A by three tcgen05 products from its own state and A's images, sets S~ = S_0 A + B (B through
+// its staging buffer) and leaves through the ordinary head boundary (S_after, drift partials).
 struct ChainSched {
     int seg_mode;              // 0: not segmented; 1: segment 0 (from the state); 2: from I, v = 0;
                                // 3: from 0
@@ -795,6 +797,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
     // MMA: ready flags.
     __shared__ uint64_t mb_tk[3], mb_ke[3], mb_tv[2], mb_ve[2], mb_tr[2], mb_re[2];
     __shared__ uint64_t mb_st, mb_sfree, mb_x, mb_u, mb_s, mb_sready, mb_xready, mb_uready, mb_fin;
+    __shared__ uint64_t mb_end, mb_cimg, mb_cd, mb_ca;   // segment combine (CTA 0 of a head): MMAs done,
+                                                         // S_0 images, the product, A's images
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     __shared__ float s_red[2][kChainWarps];
@@ -824,6 +828,7 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
             mbar_init(&mb_sready, kChainWarps); mbar_init(&mb_xready, kChainWarps);
             mbar_init(&mb_uready, kChainWarps);
             mbar_init(&mb_fin, 1);
+            mbar_init(&mb_end, 1); mbar_init(&mb_cimg, kChainWarps); mbar_init(&mb_cd, 1); mbar_init(&mb_ca, 1);
             fence_barrier_init();
         }
     }
@@ -953,6 +958,31 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 mma_commit(&mb_ke[j % 3]);             // K(j)'s buffer free once MMA_S(j) has read it
             }
         }
+        if (kSeg && sch.seg_mode == 1 && ok) {
+            // segment combine: S_0 A into the X / U columns, from CTA 0's state images (K-major) and
+            // A's images (MN-major), once every MMA of the chain has completed
+            mma_commit(&mb_end);
+            if (warp_wait(&mb_cimg, 0, kWaitBudgetNs, abort_flag) && warp_wait(&mb_ca, 0, kWaitBudgetNs, abort_flag)) {
+                tc_fence_after();
+                if (elect_one()) {
+                    const uint32_t id = idesc_bf16(128, 128, 0, 1);
+#pragma unroll
+                    for (int term = 0; term < 3; ++term) {   // S0_hi A_hi, S0_hi A_lo, S0_lo A_hi
+                        const uint32_t xb = term == 2 ? 32768u : 0u, ab = term == 1 ? 98304u : 65536u;
+#pragma unroll
+                        for (int s = 0; s < 8; ++s) {        // K = 16 per MMA
+                            const uint64_t da = sdesc_sw128(smem_u32(sm + xb + (s >> 2) * 16384 + (s & 3) * 32), 16, 1024);
+                            const uint64_t db = sdesc_sw128(smem_u32(sm + ab + s * 2048), 16384, 1024);
+                            mma_bf16_1t(tm + TM_X, da, db, id, (term | s) != 0);
+                        }
+                    }
+                }
+                __syncwarp();
+                mma_commit(&mb_cd);
+            } else {
+                fail(a.status, abort_flag, 8);
+            }
+        }
         if (__any_sync(0xffffffffu, *abort_flag != 0)) {
             mma_commit(&mb_fin);                       // every MMA this warp issued has completed
             mbar_wait(&mb_fin, 0, kWaitBudgetNs);
@@ -1041,9 +1071,32 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 load_rows(&hmap, (me - 1) * kD);
                 return true;
             };
-            auto final_phase = [&]() {                 // what the boundary after the last slot reads
-                if (sch.is_suffix(n_slots - 1)) load_rows(&smap, sch.suf_lh * kD);
-                else mbar_arrive(&mb_st);
+            int ca = 0;                                // (segment combine) A's images copy issued
+            auto wait_flag = [&](int idx) -> bool {    // hand-over entry idx published (bounded)
+                grid_dep_wait();                       // (the factor kernel reset the flags)
+                const uint64_t t0 = global_ns();
+                while (ho_load_acquire(a.ho_flag + idx) == 0) {
+                    if (*abort_flag || global_ns() - t0 > kWaitBudgetNs) return false;
+                    __nanosleep(64);
+                }
+                fence_proxy_async_global();
+                return true;
+            };
+            auto final_phase = [&]() -> bool {         // what the boundary after the last slot reads
+                if (sch.is_suffix(n_slots - 1)) { load_rows(&smap, sch.suf_lh * kD); return true; }
+                if (kSeg && sch.seg_mode == 1) {
+                    // segment combine: B (CTA me + 2) into the staging buffer; A's images (CTA me + 1)
+                    // into the tile buffers once every MMA of the chain has completed
+                    if (!wait_flag(me + 2)) return false;
+                    load_rows(&hmap, (me + 2) * kD);
+                    if (!mbar_wait_or_abort(&mb_end, 0, kWaitBudgetNs, abort_flag) || !wait_flag(me + 1)) return false;
+                    mbar_arrive_expect_tx(&mb_ca, 65536);
+                    bulk_load_tx(sm + 65536, a.ho_base + (size_t)(me + 1) * 65536, 65536, &mb_ca);
+                    ca = 1;
+                    return true;
+                }
+                mbar_arrive(&mb_st);
+                return true;
             };
             bool ok = load_state(0);
             if (!ok) fail(a.status, abort_flag, 42);
@@ -1057,7 +1110,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     ok = load_state(1);
                     if (!ok) fail(a.status, abort_flag, 43);
                 } else {
-                    final_phase();
+                    ok = final_phase();
+                    if (!ok) fail(a.status, abort_flag, 46);
                 }
             }
             for (int k = 0; ok && k < n_slots; ++k) {
@@ -1066,13 +1120,18 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 int lh, tb, te;
                 sch.slot(k, n, lh, tb, te);
                 const bool hand_over = sch.is_prefix(k);
-                const bool to_h = hand_over || kSeg;      // (a segment's end state: row me)
-                const CUtensorMap* dst = to_h ? &hmap : &smap;
-                const int row = (to_h ? me : lh) * kD;
+                const bool seg_end = kSeg && sch.seg_mode >= 2;   // a segment run's end: hand-over entry me
+                if (kSeg && sch.seg_mode == 2) {
+                    bulk_store(a.ho_base + (size_t)me * 65536, sm, 65536);   // A: the images the chain wrote
+                } else {
+                    const bool to_h = hand_over || seg_end;
+                    const CUtensorMap* dst = to_h ? &hmap : &smap;
+                    const int row = (to_h ? me : lh) * kD;
 #pragma unroll
-                for (int b = 0; b < 4; ++b) tma_store_2d(dst, sbuf + 4096 * b, 32 * b, row);
+                    for (int b = 0; b < 4; ++b) tma_store_2d(dst, sbuf + 4096 * b, 32 * b, row);
+                }
                 bulk_commit();
-                if (hand_over) {
+                if (hand_over || seg_end) {
                     bulk_wait0();                      // the state is in global memory ...
                     fence_proxy_async_global();
                     __threadfence();
@@ -1083,13 +1142,15 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                     bulk_wait_read0();                 // slot k's state has left the buffer
                     if (k + 2 < n_slots) {
                         if (!load_state(k + 2)) { fail(a.status, abort_flag, 43); break; }
-                    } else {
-                        final_phase();
+                    } else if (!final_phase()) {
+                        fail(a.status, abort_flag, 46);
+                        break;
                     }
                 }
             }
             bulk_wait0();                              // every state store is complete
             if (loads > seen) mbar_wait(&mb_st, (loads - 1) & 1, kWaitBudgetNs);   // abort: a load in flight
+            if (ca) mbar_wait(&mb_ca, 0, kWaitBudgetNs);   // (A's images have landed)
         }
         __syncwarp();
     } else {
@@ -1388,6 +1449,44 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 ok = __all_sync(0xffffffffu, ok) != 0;     // (the pass below is warp-collective)
                 ++st_seen;
                 tc_fence_after();
+                if (kSeg && sch.seg_mode == 1 && ok) {
+                    // segment combine: S_0 = sig S~ as bfloat16 (hi, lo) K-major images (row r, this
+                    // warp's 32 columns) in the free tile buffers, then S~ = S_0 A + B from the
+                    // product and the staged B, sig = 1: the pass below writes S_after and the drift
+                    {
+                        float sv[32];
+                        tmem_ld32(tm + lane_off + TM_S + 32 * cgp, sv);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) sv[e] *= sig;
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            uint4 vh, vl;
+                            split8(sv + 8 * c, vh, vl);
+                            const uint32_t off = (cgp >> 1) * 16384 + sw128_offset(r, 4 * (cgp & 1) + c);
+                            *reinterpret_cast<uint4*>(sm + off) = vh;
+                            *reinterpret_cast<uint4*>(sm + 32768 + off) = vl;
+                        }
+                    }
+                    fence_async_smem();
+                    tc_fence_before();
+                    carrive(&mb_cimg);
+                    ok = __all_sync(0xffffffffu, cwait(&mb_cd, 0, 17)) != 0;
+                    if (ok) {
+                        tc_fence_after();
+                        float dv[32];
+                        tmem_ld32(tm + lane_off + TM_X + 32 * cgp, dv);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const float4 b = *reinterpret_cast<const float4*>(sbuf + sb_idx(r, 8 * cgp + e));
+                            dv[4 * e] += b.x; dv[4 * e + 1] += b.y; dv[4 * e + 2] += b.z; dv[4 * e + 3] += b.w;
+                        }
+                        tmem_st32(tm + lane_off + TM_S + 32 * cgp, dv);
+                        tmem_st_wait();
+                        sig = 1.f;
+                    }
+                }
                 float num = 0.f, den_next = 0.f;
                 if (ok) {
 #pragma unroll
@@ -1431,6 +1530,16 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                         for (int e = 0; e < 4; ++e)
                             *reinterpret_cast<float4*>(sbuf + sb_idx(r, ch + e)) =
                                 make_float4(sa[4 * e], sa[4 * e + 1], sa[4 * e + 2], sa[4 * e + 3]);
+                        if (kSeg && sch.seg_mode == 2) {       // A: row r's (hi, lo) images, MN-major
+#pragma unroll
+                            for (int c2 = 0; c2 < 2; ++c2) {
+                                uint4 vh, vl;
+                                split8(sa + 8 * c2, vh, vl);
+                                const uint32_t off = (cgp >> 1) * 16384 + sw128_offset(r, 4 * (cgp & 1) + 2 * half + c2);
+                                *reinterpret_cast<uint4*>(sm + off) = vh;
+                                *reinterpret_cast<uint4*>(sm + 32768 + off) = vl;
+                            }
+                        }
                     }
                     tmem_st_wait();
                 }
@@ -1448,8 +1557,8 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
                 }
                 if (lane == 0) { s_red[0][warp] = fn; s_red[1][warp] = fd; }
                 if (named_sync_or(2, kChain, !ok)) break;
-                if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot) && !kSeg) {
-                    // (a shared head's drift: at its end; a segmented head's: the combine kernel's)
+                if (warp == 0 && a.partials != nullptr && !sch.is_prefix(slot) && (!kSeg || sch.seg_mode == 1)) {
+                    // (a shared head's drift: at its end; a segmented head's: CTA 0's, after the combine)
                     float pn = lane < kChainWarps ? s_red[0][lane] : 0.f;
                     float pd = lane < kChainWarps ? s_red[1][lane] : 0.f;
 #pragma unroll
@@ -1482,176 +1591,6 @@ gdn_update_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_cons
     if (warp == kMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tm, kTmemCols);
-    }
-}
-
-// =============================================================================================
-// Segment combine: S_after = S_0 A_1 + B_1 for heads the chain ran in two segments
-// =============================================================================================
-// One CTA of 512 threads per head.  Bulk copies bring S_0 and A_1 (fp32, 64 KB each, in turn through
-// the result tile) to be split into bfloat16 (hi, lo) images (S_0 K-major, rows r and K = d; A_1
-// MN-major, K rows d and N = d'); three tcgen05 products S0_hi A_hi + S0_hi A_lo + S0_lo A_hi
-// accumulate S_0 A_1 in TMEM (fp32; the dropped lo * lo term is below 2^-16 relative); then B_1 and
-// S_before are copied into the freed image space, the TMEM rows go to the padded result tile (warp
-// w: lane quarter w % 4, column quarter w / 4), and coalesced passes over shared memory form
-// S_after = S_0 A_1 + B_1, store it and take the drift sums (per thread in float, a fixed tree over
-// each warp, the warps in order).
-constexpr int kCbThreads = 4 * kD;
-constexpr int kCbPad = kD + 4;                          // fp32 row stride of the result tile
-constexpr uint32_t CB_XH = 0, CB_XL = 32768;            // S_0 images: 2 column blocks x 128 rows x 128 B; then S_before
-constexpr uint32_t CB_AH = 65536, CB_AL = 98304;        // A images: 2 N blocks (d' 0-63, 64-127) x 128 K rows; then B
-constexpr uint32_t CB_D = 131072;                       // staging of S_0 and A (dense), then the result tile [128][kCbPad]
-constexpr uint32_t kCbSmem = CB_D + kD * kCbPad * 4 + 1024;
-constexpr uint32_t kMat = kD * kD * 4;                  // one 128 x 128 fp32 matrix
-
-struct CbArgs {
-    const float* ends;       // the chain CTAs' end states, [chain CTA][128][128] fp32 (3 per head)
-    float* state;            // [heads][128][128]: in S_before, out S_after
-    float* partials;         // [heads][2] or null
-    int32_t* status;
-};
-
-// The dense 128 x 128 fp32 matrix at m (shared memory) as (hi, lo) bfloat16 images, 128-byte
-// swizzled, two 16 KB column blocks (elements 0-63, 64-127); thread t takes 8-element chunks t,
-// t + kCbThreads, ...
-__device__ __forceinline__ void split_images(const float* m, uint8_t* hi, uint8_t* lo) {
-#pragma unroll
-    for (int u = 0; u < kD * kD / 8 / kCbThreads; ++u) {
-        const int idx = (int)threadIdx.x + kCbThreads * u, row = idx >> 4, ch = idx & 15;
-        const float4* src = reinterpret_cast<const float4*>(m + row * kD + 8 * ch);
-        const float4 a = src[0], b = src[1];
-        const float x[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-        uint4 vh, vl;
-        split8(x, vh, vl);
-        const uint32_t off = (ch >> 3) * 16384 + sw128_offset(row, ch & 7);
-        *reinterpret_cast<uint4*>(hi + off) = vh;
-        *reinterpret_cast<uint4*>(lo + off) = vl;
-    }
-}
-
-__global__ void __launch_bounds__(kCbThreads, 1)
-gdn_segment_combine_kernel(CbArgs a)
-{
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t* sm = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
-    float* dt = reinterpret_cast<float*>(sm + CB_D);
-    __shared__ uint64_t mb_ld, mb_d;
-    __shared__ uint32_t s_tmem;
-    __shared__ float s_red[2][kCbThreads / 32];
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int q = warp & 3, cq = warp >> 2;
-    const uint32_t lane_off = (uint32_t)(32 * q) << 16;
-    const int head = blockIdx.x;
-    const uint8_t* base = reinterpret_cast<const uint8_t*>(a.ends) + (size_t)head * 3 * kMat;
-    float* st = a.state + (size_t)head * kD * kD;
-    if (warp == 0) { tmem_alloc(&s_tmem, kD); tmem_relinquish(); }
-    if (tid == 32) { mbar_init(&mb_ld, 1); mbar_init(&mb_d, 1); fence_barrier_init(); }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tm = s_tmem;
-    grid_dep_wait();                                   // the chain's end states are written
-    int n_ld = 0;                                      // bulk-copy groups issued (thread 0)
-    bool ok = true;
-    auto load = [&](void* dst0, const void* src0, void* dst1, const void* src1) {   // thread 0
-        mbar_arrive_expect_tx(&mb_ld, src1 ? 2 * kMat : kMat);
-        bulk_load_tx(dst0, src0, kMat, &mb_ld);
-        if (src1) bulk_load_tx(dst1, src1, kMat, &mb_ld);
-    };
-    auto wait_ld = [&](int where) {                    // everyone; uniform result
-        const bool w = mbar_wait(&mb_ld, (n_ld - 1) & 1, kWaitBudgetNs);
-        if (!w) record_status(a.status, DELTAS_ERR_TIMEOUT, where);
-        ok = __syncthreads_or(!w) == 0;
-    };
-    if (tid == 0) load(dt, base, nullptr, nullptr);    // S_0
-    ++n_ld;
-    wait_ld(70);
-    if (ok) split_images(dt, sm + CB_XH, sm + CB_XL);
-    __syncthreads();                                   // the staging buffer is free again
-    if (ok) {
-        if (tid == 0) load(dt, base + kMat, nullptr, nullptr);    // A_1
-        ++n_ld;
-        wait_ld(71);
-    }
-    if (ok) {
-        split_images(dt, sm + CB_AH, sm + CB_AL);
-        fence_async_smem();                            // the images -> the tensor core
-        tc_fence_before();
-        __syncthreads();
-        if (warp == 0) {
-            tc_fence_after();
-            if (elect_one()) {
-                const uint32_t id = idesc_bf16(128, 128, 0, 1);
-#pragma unroll
-                for (int term = 0; term < 3; ++term) {   // S0_hi A_hi, S0_hi A_lo, S0_lo A_hi
-                    const uint32_t xb = term == 2 ? CB_XL : CB_XH, ab = term == 1 ? CB_AL : CB_AH;
-#pragma unroll
-                    for (int s = 0; s < 8; ++s) {        // K = 16 per MMA
-                        const uint64_t da = sdesc_sw128(smem_u32(sm + xb + (s >> 2) * 16384 + (s & 3) * 32), 16, 1024);
-                        const uint64_t db = sdesc_sw128(smem_u32(sm + ab + s * 2048), 16384, 1024);
-                        mma_bf16_1t(tm, da, db, id, (term | s) != 0);
-                    }
-                }
-            }
-            __syncwarp();
-            mma_commit(&mb_d);
-        }
-        const bool w = mbar_wait(&mb_d, 0, kWaitBudgetNs);
-        if (!w) record_status(a.status, DELTAS_ERR_TIMEOUT, 72);
-        ok = __syncthreads_or(!w) == 0;
-    }
-    if (ok) {
-        // the images have been read: B_1 and S_before into their space, meanwhile S_0 A_1 into the tile
-        if (tid == 0) load(sm + CB_AH, base + 2 * kMat, sm + CB_XH, st);
-        ++n_ld;
-        tc_fence_after();
-        {
-            const int row = 32 * q + lane;
-            float d[32];
-            tmem_ld32(tm + lane_off + 32 * cq, d);
-            tmem_ld_wait();
-#pragma unroll
-            for (int e = 0; e < 32; e += 4)
-                *reinterpret_cast<float4*>(dt + row * kCbPad + 32 * cq + e) = make_float4(d[e], d[e + 1], d[e + 2], d[e + 3]);
-        }
-        wait_ld(73);                                   // (also orders the tile's writes before the pass)
-    }
-    if (ok) {
-        const float* sB = reinterpret_cast<const float*>(sm + CB_AH);
-        const float* sS = reinterpret_cast<const float*>(sm + CB_XH);
-        float num = 0.f, den = 0.f;
-#pragma unroll
-        for (int u = 0; u < kD * kD / 4 / kCbThreads; ++u) {
-            const int idx = tid + kCbThreads * u, row = idx >> 5, c4 = idx & 31;
-            const float4 dv = reinterpret_cast<const float4*>(dt + row * kCbPad)[c4];
-            const float4 b = reinterpret_cast<const float4*>(sB + row * kD)[c4];
-            const float4 sb = reinterpret_cast<const float4*>(sS + row * kD)[c4];
-            const float4 sa = make_float4(dv.x + b.x, dv.y + b.y, dv.z + b.z, dv.w + b.w);
-            const float d0 = sa.x - sb.x, d1 = sa.y - sb.y, d2 = sa.z - sb.z, d3 = sa.w - sb.w;
-            num += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
-            den += sb.x * sb.x + sb.y * sb.y + sb.z * sb.z + sb.w * sb.w;
-            reinterpret_cast<float4*>(st + (size_t)row * kD)[c4] = sa;
-        }
-#pragma unroll
-        for (int m = 16; m >= 1; m >>= 1) {
-            num += __shfl_xor_sync(0xffffffffu, num, m);
-            den += __shfl_xor_sync(0xffffffffu, den, m);
-        }
-        if (lane == 0) { s_red[0][warp] = num; s_red[1][warp] = den; }
-    } else if (tid == 0 && n_ld > 0) {
-        mbar_wait(&mb_ld, (n_ld - 1) & 1, kWaitBudgetNs);   // (after a failure: the last copies land)
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (ok && tid == 0 && a.partials != nullptr) {
-        float n = 0.f, d = 0.f;
-        for (int w = 0; w < kCbThreads / 32; ++w) { n += s_red[0][w]; d += s_red[1][w]; }
-        a.partials[(size_t)head * 2] = n;
-        a.partials[(size_t)head * 2 + 1] = d;
-    }
-    if (warp == 0) {
-        tc_fence_after();
-        tmem_dealloc(tm, kD);
     }
 }
 
@@ -2069,9 +2008,7 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
         if (e == cudaSuccess && out)
             e = cudaFuncSetAttribute(gdn_readout_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)kRoSmemAlloc);
-        if (e == cudaSuccess && sg > 1)
-            e = cudaFuncSetAttribute(gdn_segment_combine_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)kCbSmem);
+
         if (e != cudaSuccess) return e;
     }
     // factor kernel: one record per (layer, value head, tile), kWyCtasPerSm persistent CTAs per SM
@@ -2094,6 +2031,7 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     t.ho_wflag = t.ho_flag + grid;
     t.ho_wsum = reinterpret_cast<float*>(a.scratch + sl.ho_wsum);
     t.seg = sg;
+    t.ho_base = a.scratch + sl.ho_state;
     t.ubuf = out ? reinterpret_cast<float*>(a.scratch + sl.ubuf) : nullptr;
     t.snap = out ? reinterpret_cast<float*>(a.scratch + sl.snap) : nullptr;
     t.n_blk = n_blk;
@@ -2110,14 +2048,6 @@ cudaError_t launch_gdn_update_tc(const GdnArgs& a, cudaStream_t s) {
     }
     e = launch_dependent(chain, dim3(grid), dim3(kThreads), (size_t)kSmemAlloc, s, kmap, vmap, smap, hmap, t);
     if (e != cudaSuccess) return e;
-    if (sg > 1) {
-        // segment combine: S_after and the drift partials of every head from its CTAs' end states
-        CbArgs c;
-        c.ends = reinterpret_cast<const float*>(a.scratch + sl.ho_state);
-        c.state = a.state; c.partials = a.partials; c.status = a.status;
-        return launch_dependent(gdn_segment_combine_kernel, dim3((unsigned)heads), dim3(kCbThreads),
-                                (size_t)kCbSmem, s, c);
-    }
     if (!out) return e;
     // read-out kernel: one persistent CTA per SM over the (layer, value head, 128-token block) items;
     // its CTAs take the SMs the update kernel leaves free and wait there for its results
