@@ -138,8 +138,8 @@ DELTAS_API const char* deltas_status_string(int32_t status);
 /* Kernels: d = 128 bfloat16 runs on the tensor cores (a factor kernel, a state-chain kernel   */
 /* and, with out != NULL, a read-out kernel that forms each 128-token block's outputs from the */
 /* block's starting state and writes; when few heads leave most SMs idle and neither out nor  */
-/* write sizes are asked for, the chain runs each head's tiles as two segments on three CTAs  */
-/* and a combine kernel joins them), or returns UNSUPPORTED when that path cannot be launched  */
+/* write sizes are asked for, the chain runs each head's tiles as two segments on three CTAs, */
+/* the first joining them at its end), or returns UNSUPPORTED when that path cannot be launched */
 /* (no silent fallback).  Every other shape runs token by token on the CUDA cores.            */
 /* ------------------------------------------------------------------------------------------ */
 DELTAS_API size_t deltas_gdn_chunk_update_workspace_size(const deltas_gdn_desc* desc, int32_t n_tokens);
