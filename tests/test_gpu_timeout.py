@@ -68,15 +68,17 @@ def _rel(a, b):
     return float(np.max(np.sqrt(np.sum((a - b) ** 2, axis=(-2, -1)) / np.sum(b ** 2, axis=(-2, -1)))))
 
 
-@pytest.mark.parametrize("want_out", [False, True])
-def test_update_wait_runs_out_then_recovers(L, want_out):
+@pytest.mark.parametrize("want_out,T", [(False, 200), (True, 200), (False, 1024)])
+def test_update_wait_runs_out_then_recovers(L, want_out, T):
     """The tensor-core update (d = 128 bf16: factor kernel, state chain and, with the read-out,
     the read-out kernel) with a 1 ns wait budget, which bounds each kernel's first wait: those
     waits give up, the other roles stop at their next wait (they see the abort flag), drain the
     copies and products they issued and free TMEM; the call ends with DELTAS_ERR_TIMEOUT
     recorded.  The same call with the default budget, from the restored state, then matches the
-    oracle."""
-    Lg, Hk, Hv, d, T = 1, 2, 4, 128, 200
+    oracle.  With 1024 tokens (16 tiles, 4 heads) the heads run as two segments on three CTAs, and
+    the first-segment CTA's bounded waits for its siblings and for the combine product also stop
+    on the abort."""
+    Lg, Hk, Hv, d = 1, 2, 4, 128
     x = inputs.gdn_chunk(Lg, T, Hk, Hv, d, "bf16", inputs.seed_for(90, int(want_out)))
     s0 = inputs.initial_state(Lg, Hv, d, 91)
     dev = torch.device("cuda")
