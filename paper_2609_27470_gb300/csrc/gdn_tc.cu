@@ -16,8 +16,9 @@
 // the part that is sequential in the tiles, the state chain, with nothing else on the SM.
 //
 // Update kernel: one persistent CTA per SM takes (layer, value head) pairs in turn, or equal runs
-// of tiles with a head at each run boundary split between two CTAs (see ChainSched); the tiles of
-// its slots form one pipeline.  A head's state lives in TMEM from its first tile to its last
+// of tiles with a head at each run boundary split between two CTAs, or, with few heads, two
+// segments of each head on three CTAs (see ChainSched); the tiles of its slots form one pipeline.
+// With the read-out a third kernel (gdn_readout_kernel) forms the outputs.  A head's state lives in TMEM from its first tile to its last
 // (S_before beside it, for the drift), so the state is read from and written to HBM exactly once;
 // the next head's state is loaded into shared memory while the current head runs, and the head
 // boundary swaps the two in one pass that also forms the drift partials.  Per tile:
