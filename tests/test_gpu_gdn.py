@@ -405,6 +405,9 @@ def test_readout_zero_tokens(L):
     (1, 1, 2, 1024, 0.0),     # no decay: the affine maps keep their full range
     (1, 16, 32, 512, 0.1),    # the single layer's heads, 8 tiles: two segments of 4
     (1, 16, 32, 449, 0.1),    # 8 tiles, the second segment ending in a one-token tile
+    (2, 8, 16, 640, 0.1),     # two layers (the CTA groups span layers), 10 tiles
+    (1, 25, 50, 512, 0.1),    # 50 heads: 150 CTAs, the most that fit on 152 SMs
+    (1, 4, 4, 512, 0.1),      # one value head per key head
 ])
 def test_gdn_update_segments(L, Lg, Hk, Hv, T, decay):
     """Few heads (at most a third of the SMs) and at least 8 tiles: the state chain runs each head's
