@@ -126,6 +126,22 @@ def test_select_large_caches(L, T, n_ch, run_max):
     _assert_same_selection(L, T - 1, 0, 0, 1, tc, sc)
 
 
+@pytest.mark.parametrize("T,run_max,n_s,n_w", [(65536, 6, 4, 1024), (65537, 6, 4, 1024), (65536, 1, 0, 0),
+                                             (4097, 3, 1023, 1025), (2048, 1024, 1024, 0)])
+def test_select_scan_block_edges(L, T, run_max, n_s, n_w):
+    """Runs of 1 to run_max slots cross the run scan's 1024-slot block edges; a cache of 64k
+    slots and one of a slot more (a one-slot last block); sink and window ends on and next to a
+    block edge; one token per chunk makes 64k runs (the radix path)."""
+    rng = np.random.default_rng(T + run_max)
+    lens = rng.integers(1, run_max + 1, size=T)
+    tc = np.repeat(np.arange(lens.size, dtype=np.int32), lens)[:T].astype(np.int32)
+    n_ch = int(tc[-1]) + 1
+    sc = rng.exponential(size=n_ch).astype(np.float32)
+    sc[rng.integers(0, n_ch, size=6)] = sc[1]
+    _assert_same_selection(L, T // 3 + n_s + n_w, n_s, n_w, 4, tc, sc)
+    _assert_same_selection(L, T - 1, 0, 0, 1, tc, sc)
+
+
 def test_select_edge_cases(L):
     rng = np.random.default_rng(105)
     tc = np.repeat(np.arange(10, dtype=np.int32), 10)
@@ -145,6 +161,13 @@ def test_select_reports_bad_chunk_ids(L):
     tc = np.array([0, 1, 2, 7, 3], np.int32)
     idx, mask, st = gpu_select(L, 2, 0, 0, 1, tc, np.ones(4, np.float32))
     assert st == (L.DELTAS_ERR_DEVICE_INDEX, 3)
+    # bad ids in later scan blocks (one on a block edge): the last bad slot is reported
+    for T in (3000, 70000):
+        tc = np.repeat(np.arange(T // 10, dtype=np.int32), 10)
+        tc[1024] = -1
+        tc[T - 500] = T // 10
+        idx, mask, st = gpu_select(L, T // 2, 0, 0, 1, tc, np.ones(T // 10, np.float32))
+        assert st == (L.DELTAS_ERR_DEVICE_INDEX, T - 500)
 
 
 # ----------------------------------------------------------------------------- compaction
