@@ -305,10 +305,20 @@ select_retain_kernel(SelArgs a)
     }
     if (lane == 0) { s_cmin[warp] = cmin; s_cmax[warp] = cmax; }
     if (tid < kMaxSpans) s_span_total[tid] = 0;
+    // the small path's pair sums, in the radix path's histogram space after the block counts and
+    // offsets of the gather below
+    int* s_above = reinterpret_cast<int*>(s_hist) + 2 * kSelThreads;
+    int* s_above2 = s_above + kSmallRuns;
+    static_assert(2 * kSelThreads + 2 * kSmallRuns <= kMaxSpans * 256, "histogram space");
+    for (int r = tid; r < kSmallRuns; r += kSelThreads) { s_above[r] = 0; s_above2[r] = 0; }
     __syncthreads();
     const bool small = n_runs <= kSmallRuns;
-    int c_lo = INT_MAX, c_hi = INT_MIN;
-    for (int w = 0; w < kSelWarps; ++w) { c_lo = min(c_lo, s_cmin[w]); c_hi = max(c_hi, s_cmax[w]); }
+    int c_lo = s_cmin[lane], c_hi = s_cmax[lane];            // (kSelWarps == 32)
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+        c_lo = min(c_lo, __shfl_xor_sync(0xffffffffu, c_lo, m));
+        c_hi = max(c_hi, __shfl_xor_sync(0xffffffffu, c_hi, m));
+    }
     const long long span_width = (long long)c_hi - c_lo + 1;
     int* r_start = small ? s_rstart : a.ws.run_start;
     int* r_len = small ? s_rlen : a.ws.run_len;
@@ -351,35 +361,44 @@ select_retain_kernel(SelArgs a)
     const int fill = R - granted;
 
     if (small) {
-        // ---- C/D (at most 512 runs, one per thread): a run keeps the part of its span quota
-        // (then of the fill) that the runs ranked above it leave over.
-        int k1 = 0, rem = 0, len = 0, st = 0;
-        uint64_t key = 0;
-        if (tid < n_runs) {
-            len = s_rlen[tid]; st = s_rstart[tid]; key = s_rkey[tid];
-            const int j = s_rspan[tid];
+        // ---- C/D (at most 512 runs): a run keeps the part of its span quota (then of the fill)
+        // that the runs ranked above it leave over.  The weight above run i is summed over all
+        // pairs (i, r) by the whole CTA: thread t takes run i = t mod P (P = 32 or the next power
+        // of two >= n_runs) and the t / P-th of 1024 / P slices of the runs r.
+        const int P = n_runs <= 32 ? 32 : 1 << (32 - __clz(n_runs - 1));
+        const int n_sl = kSelThreads / P;
+        const int i = tid & (P - 1), sl = tid / P;
+        const int per = (n_runs + n_sl - 1) / n_sl;
+        const int r_lo = min(sl * per, n_runs), r_hi = min(r_lo + per, n_runs);
+        if (i < n_runs) {
+            const int j = s_rspan[i];
+            const uint64_t key = s_rkey[i];
             int above = 0;
-            for (int r = 0; r < n_runs; ++r)
+            for (int r = r_lo; r < r_hi; ++r)
                 if (s_rspan[r] == j && s_rkey[r] > key) above += s_rlen[r];
-            k1 = min(len, max(0, s_target[j] - above));
-            rem = len - k1;
+            if (above) atomicAdd(&s_above[i], above);
         }
         __syncthreads();
+        int k1 = 0, rem = 0;
         if (tid < n_runs) {
+            const int len = s_rlen[tid];
+            k1 = min(len, max(0, s_target[s_rspan[tid]] - s_above[tid]));
+            rem = len - k1;
             s_rlen[tid] = rem;
-            s_rkey[tid] = (key & 0xFFFFFFFF00000000ull) | (uint64_t)(~(uint32_t)(st + k1));
+            s_rkey[tid] = (s_rkey[tid] & 0xFFFFFFFF00000000ull) | (uint64_t)(~(uint32_t)(s_rstart[tid] + k1));
+        }
+        __syncthreads();
+        if (fill > 0 && i < n_runs && s_rlen[i] > 0) {
+            const uint64_t key2 = s_rkey[i];
+            int above = 0;
+            for (int r = r_lo; r < r_hi; ++r)
+                if (s_rkey[r] > key2) above += s_rlen[r];
+            if (above) atomicAdd(&s_above2[i], above);
         }
         __syncthreads();
         int kept = 0;
         if (tid < n_runs) {
-            int k2 = 0;
-            if (fill > 0 && rem > 0) {
-                const uint64_t key2 = s_rkey[tid];
-                int above = 0;
-                for (int r = 0; r < n_runs; ++r)
-                    if (s_rkey[r] > key2) above += s_rlen[r];
-                k2 = min(rem, max(0, fill - above));
-            }
+            const int k2 = (fill > 0 && rem > 0) ? min(rem, max(0, fill - s_above2[tid])) : 0;
             kept = k1 + k2;
             s_rkept[tid] = kept;
         }
@@ -450,13 +469,26 @@ select_retain_kernel(SelArgs a)
 // ---- E. every slot writes itself: a candidate slot goes to retain_idx if it lies in its run's
 // kept prefix (its run found by binary search over the run starts); sink and window slots are
 // copied through.  Grid-wide, one slot per thread.
+constexpr int kEmitRuns = 2048;   // runs staged in shared memory by each emit block
+
 __global__ void __launch_bounds__(256)
 select_emit_kernel(SelArgs a)
 {
+    __shared__ int s_start[kEmitRuns], s_kept[kEmitRuns], s_off[kEmitRuns];
     grid_dep_wait();                                   // the decision is complete
     if (!a.ctl->emit) return;
     const int n_runs = a.ctl->n_runs;
     const int T = a.T, lo = a.n_s, hi = T - a.n_w;
+    const bool staged = n_runs <= kEmitRuns;          // else the search runs on the workspace
+    if (staged) {
+        for (int r = threadIdx.x; r < n_runs; r += blockDim.x) {
+            s_start[r] = a.ws.run_start[r]; s_kept[r] = a.ws.kept[r]; s_off[r] = a.ws.out_off[r];
+        }
+        __syncthreads();
+    }
+    const int* run_start = staged ? s_start : a.ws.run_start;
+    const int* run_kept = staged ? s_kept : a.ws.kept;
+    const int* run_off = staged ? s_off : a.ws.out_off;
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
         if (i < lo) {
             a.retain_idx[i] = i;
@@ -468,11 +500,11 @@ select_emit_kernel(SelArgs a)
             int l = 0, h = n_runs - 1;                     // last run with start <= i
             while (l < h) {
                 const int m = (l + h + 1) >> 1;
-                if (a.ws.run_start[m] <= i) l = m; else h = m - 1;
+                if (run_start[m] <= i) l = m; else h = m - 1;
             }
-            const int pos = i - a.ws.run_start[l];
-            const bool keep = pos < a.ws.kept[l];
-            if (keep) a.retain_idx[a.n_s + a.ws.out_off[l] + pos] = i;
+            const int pos = i - run_start[l];
+            const bool keep = pos < run_kept[l];
+            if (keep) a.retain_idx[a.n_s + run_off[l] + pos] = i;
             if (a.mask) a.mask[i] = keep ? 1 : 0;
         }
     }
