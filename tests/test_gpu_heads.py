@@ -99,7 +99,9 @@ SELECT_CASES = [
     (3, 500, 600, 4, 128, 4),          # no eviction: the identity
     (5, 2049, 1024, 4, 1000, 0),       # N = 0 read as one span
     (16, 33280, 32768, 4, 1024, 4),    # streaming shape: keys in shared memory
-    (16, 65536, 16384, 4, 1024, 4),    # 64k slots: keys in the workspace
+    (16, 65536, 16384, 4, 1024, 4),    # 64k slots: a quarter per CTA, keys in shared memory
+    (2, 180000, 60000, 4, 1024, 4),    # 180k slots: keys in the workspace
+    (3, 9, 5, 1, 1, 2),                # fewer candidates than the cluster has CTAs per plane
 ]
 
 
@@ -130,17 +132,24 @@ def test_select_heads_matches_oracle(L, planes, T, M, n_s, n_w, N, with_mask):
             assert np.array_equal(m[:T], mask) and np.all(m[T:] == 7)
 
 
-def test_select_heads_reports_negative_chunk_ids(L):
+@pytest.mark.parametrize("slot,n_s,n_w", [(50, 0, 0), (1, 4, 10), (97, 4, 10)])
+def test_select_heads_reports_negative_chunk_ids(L, slot, n_s, n_w):
+    """A negative chunk id among the candidates, in the sink or in the window of plane 1 (each
+    checked by a different CTA of the plane's cluster) is reported; the call then recovers."""
     dev = torch.device("cuda")
     tc = torch.zeros(2, 100, dtype=torch.int32)
-    tc[1, 50] = -3
+    tc[1, slot] = -3
     ts = torch.randn(2, 100)
     ws = L.alloc_workspace(L.deltas_select_retain_heads_workspace_size(2, 100), dev)
     L.deltas_clear_device_status(ws)
     ri = torch.zeros(2, 60, dtype=torch.int32, device=dev)
     nr = torch.zeros(1, dtype=torch.int32, device=dev)
-    L.deltas_select_retain_heads(L.policy(60, 0, 0, 1), 100, tc.to(dev), ts.to(dev), ri, nr, None, ws)
+    L.deltas_select_retain_heads(L.policy(60, n_s, n_w, 1), 100, tc.to(dev), ts.to(dev), ri, nr, None, ws)
     assert L.deltas_get_device_status(ws)[0] == L.DELTAS_ERR_DEVICE_INDEX
+    L.deltas_clear_device_status(ws)
+    tc[1, slot] = 0
+    L.deltas_select_retain_heads(L.policy(60, n_s, n_w, 1), 100, tc.to(dev), ts.to(dev), ri, nr, None, ws)
+    assert L.deltas_get_device_status(ws) == (0, 0) and nr.item() == 60
 
 
 @pytest.mark.parametrize("D,dt,T,M", [
