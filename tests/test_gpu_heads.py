@@ -102,6 +102,7 @@ SELECT_CASES = [
     (16, 65536, 16384, 4, 1024, 4),    # 64k slots: a quarter per CTA, keys in shared memory
     (2, 180000, 60000, 4, 1024, 4),    # 180k slots: keys in the workspace
     (3, 9, 5, 1, 1, 2),                # fewer candidates than the cluster has CTAs per plane
+    (48, 2000, 1500, 4, 128, 4),       # more planes than clusters resident at once
 ]
 
 
