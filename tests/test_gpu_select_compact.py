@@ -110,11 +110,12 @@ def test_select_streaming_shape(L):
     _assert_same_selection(L, 32768, 4, 1024, 4, tc, sc)
 
 
-@pytest.mark.parametrize("T,n_ch,run_max", [(100000, 700, 400), (150000, 20000, 6)])
+@pytest.mark.parametrize("T,n_ch,run_max", [(100000, 700, 400), (150000, 20000, 6), (262144, 900, 700),
+                                            (262145, 900, 700), (300000, 30000, 6)])
 def test_select_large_caches(L, T, n_ch, run_max):
-    """Caches past the one-CTA size (64k slots) take the grid-wide run scan, the decision kernel
-    and the grid-wide emission: a few hundred long runs (ranked in shared memory) and tens of
-    thousands of short ones (the radix path); the paper's policy and exact score ties."""
+    """Large caches through the grid-wide run scan, the decision kernel and the grid-wide
+    emission: a few hundred long runs (ranked in shared memory) and tens of thousands of short
+    ones (the radix path), 256k slots and one slot more, the paper's policy and exact score ties."""
     rng = np.random.default_rng(T + n_ch)
     lens = rng.integers(1, run_max + 1, size=4 * T // (run_max + 1) + 8)
     ids = np.sort(rng.integers(0, n_ch, size=lens.size)).astype(np.int32)
