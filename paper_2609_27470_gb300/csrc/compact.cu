@@ -85,6 +85,8 @@ __device__ __forceinline__ char* plane_base(const CompactArgs& a, int p, int& li
 
 __global__ void compact_init_kernel(CompactArgs a) {
     grid_dep_launch();                                 // the prepass may be scheduled now
+    grid_dep_wait();                                   // the previous call (which may share the
+                                                       // workspace) is done before the reset
     const int total = a.n_planes * a.max_tiles;
     for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total + a.n_lists; e += gridDim.x * blockDim.x) {
         if (e < total) a.flags[e] = 0;
@@ -299,6 +301,8 @@ append_kv_kernel(char* k_cache, char* v_cache, int n_kv_planes, int capacity, in
                  const char* k_new, const char* v_new, int n_new, int32_t* tok_chunk, int32_t* tok_pos,
                  int chunk_id, int first_pos, int blocks_per_plane)
 {
+    grid_dep_wait();                                   // earlier work on the caches is done
+    grid_dep_launch();
     const int b = blockIdx.x;
     const int n_copy_blocks = 2 * n_kv_planes * blocks_per_plane;
     if (b >= n_copy_blocks) {                                  // metadata of the new rows
@@ -358,6 +362,8 @@ append_kv_heads_kernel(char* k_cache, char* v_cache, int n_kv_planes, int capaci
                        int cache_len, const char* k_new, const char* v_new, int n_new, int32_t* tok_chunk,
                        int32_t* tok_pos, float* tok_score, int key_signal, int chunk_id, int first_pos)
 {
+    grid_dep_wait();                                   // earlier work on the caches is done
+    grid_dep_launch();
     const long long row = (long long)blockIdx.x * kAppendHeadsWarps + (threadIdx.x >> 5);
     if (row >= (long long)n_kv_planes * n_new) return;
     const int lane = threadIdx.x & 31;
@@ -446,12 +452,10 @@ cudaError_t launch_compact(const KvPlanes& kv, bool per_head, const int32_t* ret
     const int sms = device_sm_count();
     const long long init_items = (long long)a.n_planes * a.max_tiles + a.n_lists;
     const int init_blocks = (int)std::min<long long>(4ll * sms, (init_items + 255) / 256 + 1);
-    compact_init_kernel<<<init_blocks, 256, 0, s>>>(a);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_dependent(compact_init_kernel, dim3(init_blocks), dim3(256), 0, s, a);
     if (e != cudaSuccess) return e;
-    // the prepass and the moves start while their predecessor finishes (each waits for it before
-    // reading or writing anything); the flag reset above is not overlapped: it writes the
-    // workspace that the preceding call may still be using
+    // the reset, the prepass and the moves start while their predecessor finishes (each waits for
+    // it before reading or writing anything: the preceding call may share the workspace)
     const long long need_items = (long long)cache_len * a.n_lists;
     const int need_blocks = (int)std::min<long long>(4ll * sms, (need_items + 255) / 256);
     e = launch_dependent(compact_need_kernel, dim3(need_blocks), dim3(256), 0, s, a);
@@ -501,11 +505,12 @@ cudaError_t launch_append_kv(const KvPlanes& kv, int cache_len, const void* k_ne
     const long long copy_blocks = 2ll * kv.Lf * kv.Hkv * blocks_per_plane;
     const int meta_blocks = (n_new + kAppendThreads - 1) / kAppendThreads;
     if (copy_blocks + meta_blocks > INT_MAX) return cudaErrorInvalidValue;
-    append_kv_kernel<<<(int)(copy_blocks + meta_blocks), kAppendThreads, 0, s>>>(
-        static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache), kv.Lf * kv.Hkv, kv.capacity, rb, cache_len,
-        static_cast<const char*>(k_new), static_cast<const char*>(v_new), n_new, kv.tok_chunk, kv.tok_pos, chunk_id,
-        first_pos, blocks_per_plane);
-    return cudaGetLastError();
+    // scheduled while the previous kernel finishes (it waits for it before touching memory)
+    return launch_dependent(append_kv_kernel, dim3((int)(copy_blocks + meta_blocks)), dim3(kAppendThreads), 0, s,
+                            static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache), kv.Lf * kv.Hkv,
+                            kv.capacity, rb, cache_len, static_cast<const char*>(k_new),
+                            static_cast<const char*>(v_new), n_new, kv.tok_chunk, kv.tok_pos, chunk_id, first_pos,
+                            blocks_per_plane);
 }
 
 cudaError_t launch_append_kv_heads(const KvPlanes& kv, int signal, int cache_len, const void* k_new,
@@ -516,11 +521,11 @@ cudaError_t launch_append_kv_heads(const KvPlanes& kv, int signal, int cache_len
     const long long rows = (long long)kv.Lf * kv.Hkv * n_new;
     const long long blocks = (rows + kAppendHeadsWarps - 1) / kAppendHeadsWarps;
     if (blocks > INT_MAX) return cudaErrorInvalidValue;
-    append_kv_heads_kernel<<<(int)blocks, kAppendHeadsWarps * 32, 0, s>>>(
-        static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache), kv.Lf * kv.Hkv, kv.capacity, rb,
-        kv.dtype == DELTAS_BF16 ? 1 : 0, cache_len, static_cast<const char*>(k_new), static_cast<const char*>(v_new),
-        n_new, kv.tok_chunk, kv.tok_pos, kv.tok_score, signal == DELTAS_SIGNAL_KEY_NORM ? 1 : 0, chunk_id, first_pos);
-    return cudaGetLastError();
+    return launch_dependent(append_kv_heads_kernel, dim3((int)blocks), dim3(kAppendHeadsWarps * 32), 0, s,
+                            static_cast<char*>(kv.k_cache), static_cast<char*>(kv.v_cache), kv.Lf * kv.Hkv,
+                            kv.capacity, rb, kv.dtype == DELTAS_BF16 ? 1 : 0, cache_len,
+                            static_cast<const char*>(k_new), static_cast<const char*>(v_new), n_new, kv.tok_chunk,
+                            kv.tok_pos, kv.tok_score, signal == DELTAS_SIGNAL_KEY_NORM ? 1 : 0, chunk_id, first_pos);
 }
 
 }  // namespace deltas

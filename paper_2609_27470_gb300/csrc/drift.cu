@@ -70,6 +70,7 @@ score_chunks_kernel(int L, int Hv, const float* __restrict__ partials, int chunk
 {
     __shared__ double term_sum[kScoreThreads / 32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    grid_dep_launch();                                 // the next call's kernel may be scheduled now
     grid_dep_wait();                                   // the partials are written
     double acc = 0.0;
     for (int l = warp; l < L; l += kScoreThreads / 32) {
@@ -106,6 +107,7 @@ __global__ void __launch_bounds__(32)
 score_write_norms_kernel(int n, const float* __restrict__ wnorm, double inv_count, int chunk_id,
                          float* __restrict__ scores)
 {
+    grid_dep_launch();                                 // the next call's kernel may be scheduled now
     grid_dep_wait();                                   // the write sizes are written
     double acc = 0.0;
     for (int i = threadIdx.x; i < n; i += 32) acc += (double)wnorm[i];

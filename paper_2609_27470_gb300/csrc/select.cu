@@ -187,6 +187,7 @@ select_runs_kernel(SelArgs a)
     __shared__ int s_wsum[kScanThreads / 32];
     __shared__ int s_min[kScanThreads / 32], s_max[kScanThreads / 32], s_bad[kScanThreads / 32];
     grid_dep_launch();                                 // the decision kernel may be scheduled now
+    grid_dep_wait();                                   // the cache's chunk ids (and all earlier work)
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int T = a.T, lo = a.n_s, hi = T - a.n_w;
     const int b0 = blockIdx.x * kScanSlots;
@@ -530,8 +531,8 @@ cudaError_t launch_select_retain(const deltas_policy& p, int cache_len, int num_
     a.ctl = reinterpret_cast<SelCtl*>(static_cast<char*>(ws) + kSelCtlOffset);
     a.ws = carve(ws, cache_len);
     if (cache_len > 0) {
-        select_runs_kernel<<<(cache_len + kScanSlots - 1) / kScanSlots, kScanThreads, 0, s>>>(a);
-        cudaError_t e0 = cudaGetLastError();
+        const cudaError_t e0 = launch_dependent(select_runs_kernel, dim3((cache_len + kScanSlots - 1) / kScanSlots),
+                                                dim3(kScanThreads), 0, s, a);
         if (e0 != cudaSuccess) return e0;
     }
     // the decision and the emission start while their predecessor finishes (each waits for it
