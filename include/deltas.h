@@ -377,8 +377,11 @@ DELTAS_API deltas_status deltas_append_kv_heads(const deltas_kv_desc* desc, int3
 /*   retain_idx  [num_planes][M] int32  out: row p = the kept slots of plane p, ascending        */
 /*   n_retained  [1] int32 (device)     out: min(cache_len, M), the same for every plane        */
 /*   mask        [num_planes][plane_stride] uint8  out: 1 = kept; NULL to skip                   */
-/* One CTA ranks one plane (a radix select on the score's total-order bits, then on the slot    */
-/* for ties); the plane's keys sit in shared memory when they fit, else in the workspace.       */
+/* A cluster of four CTAs ranks one plane, each CTA a quarter of its candidates (a radix select */
+/* on the score's total-order bits, then on the slot for ties, with the four CTAs' counts added */
+/* through distributed shared memory); the keys sit in shared memory when they fit, else in the  */
+/* workspace.  The launch needs four SMs of one GPC free at once for each cluster: a context    */
+/* limited to fewer SMs than that gets the launch error back (DELTAS_ERR_CUDA).                 */
 /* A negative tok_chunk value is reported as DEVICE_INDEX.  cache_len above                     */
 /* DELTAS_SELECT_MAX_CACHE_LEN or plane_stride < cache_len: UNSUPPORTED / INVALID_ARGUMENT.     */
 DELTAS_API size_t deltas_select_retain_heads_workspace_size(int32_t num_planes, int32_t cache_len);
